@@ -1,0 +1,439 @@
+/*
+ * KV-PRM verify-token scoring -- CPU ORACLE.  TEST INFRASTRUCTURE ONLY.
+ *
+ * Only tests/, __graft_entry__.smoke() and bench.py's CPU-baseline leg may
+ * load this file's library.  The CUDA scoring library never links, calls or
+ * falls back to it, and the two share no code.
+ *
+ * What it computes (one candidate trajectory b with a cached length L_b; all
+ * arithmetic in IEEE double, sums taken in plain index order):
+ *
+ *   Scoring, Sec. 4.1 Eq. (score): one verify token v is forwarded through the
+ *   scorer's N_L layers against the existing per-layer cache (K, V), and the
+ *   reward is s = P(+) = softmax([z_-, z_+]) taken at the "+" entry, where z_-
+ *   and z_+ are the logits of the judgment tokens (App. B.2).  Only those two
+ *   rows of the output head are needed: P(+) = 1 / (1 + exp(z_- - z_+)).
+ *
+ *   The verify token is appended at the end of the sequence (Sec. 1), so it
+ *   sits at position p = L_b and, like any causal decoder token, also attends
+ *   to its own key/value (softmax over L_b + 1 entries).  Its own k/v are not
+ *   written into the cache.
+ *
+ *   Attention read-out, App. A.3: head_i = softmax(q_i^T K / sqrt(d_k)) V.
+ *   Grouped-query heads: query head h reads kv head floor(h / G), G = n_q/n_kv.
+ *
+ *   Per layer (pre-norm decoder block; the cost of Eq. (cost_kv) is this
+ *   block's attention term c_attn*d*L plus its feed-forward term c_ffn*d^2):
+ *     x   = RMSNorm(h) * g_attn                     eps = rms_eps
+ *     q,k,v = W_qkv x                               rows: [q heads | k heads | v heads]
+ *     q,k = RoPE(q, k; p = L_b)                     rotate-half pairs (i, i + hd/2),
+ *                                                   angle p * base^(-2i/hd)
+ *     o_h = softmax over {cache of b} U {self} of q_h.k_j / sqrt(hd), times v_j
+ *     h  += W_o o
+ *     x   = RMSNorm(h) * g_mlp
+ *     h  += W_down (SiLU(W_gate x) * (W_up x))      W_gate_up rows: [gate | up]
+ *   then x = RMSNorm(h) * g_final, z_+ = w_plus . x, z_- = w_minus . x.
+ *
+ * Precision contract ("mirror" mode): the paper trains and serves in bf16
+ * (App. B.1), so weights and cached K/V are bf16 values, and the oracle rounds
+ * to bf16 (round to nearest, ties to even) exactly where the scoring library
+ * stores bf16: every projection input (x after each norm, the attention output
+ * o, the SiLU(gate)*up product, the final x), the rotated q, and the self k/v.
+ * "exact" mode skips those intermediate roundings.
+ *
+ * Inputs arrive through provider callbacks (weights one matrix at a time, the
+ * logical per-candidate K/V one layer at a time), so full-size workloads need
+ * no host copy of the whole model or cache.
+ */
+#include <math.h>
+#include <pthread.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+/* weight kinds, as asked of the weight provider */
+enum { K_EMBED = 0, K_FINAL_NORM, K_W_PLUS, K_W_MINUS, K_ATTN_NORM, K_W_QKV, K_W_O, K_MLP_NORM, K_W_GATE_UP, K_W_DOWN };
+
+typedef int (*oracle_weight_fn)(void* user, int kind, int layer, uint16_t* out, int64_t n);
+typedef int (*oracle_kv_fn)(void* user, int layer, int cand, uint16_t* K, uint16_t* V, int64_t L);
+
+typedef struct {
+    int n_layers, d_model, n_q_heads, n_kv_heads, head_dim, d_ff;
+    double rope_base, rms_eps;
+    int mirror;   /* 1: bf16 rounding at the precision contract's points; 0: exact */
+    int nthreads;
+} oracle_cfg;
+
+/* ------------------------------------------------------------------ numbers */
+static inline double bf16_to_f64(uint16_t b) {
+    uint32_t u = (uint32_t)b << 16;
+    float f;
+    memcpy(&f, &u, 4);
+    return (double)f;
+}
+
+/* Round a double to the nearest bf16 value (ties to even): 8 significant bits,
+ * exponent range of IEEE binary32, subnormal quantum 2^-133. */
+double oracle_bf16_round(double x) {
+    if (x == 0.0 || !isfinite(x)) return x;
+    int e;
+    frexp(x, &e);                       /* x = m * 2^e, 0.5 <= |m| < 1 */
+    int qe = e - 8;
+    if (qe < -133) qe = -133;
+    double r = ldexp(nearbyint(ldexp(x, -qe)), qe);
+    if (fabs(r) >= 0x1p128) return copysign(INFINITY, x);
+    return r;
+}
+
+static inline double rnd(const oracle_cfg* c, double x) { return c->mirror ? oracle_bf16_round(x) : x; }
+
+/* ------------------------------------------------------------ parallel for */
+typedef void (*idx_fn)(void* ctx, int64_t i);
+typedef struct { idx_fn fn; void* ctx; int64_t n; int t, nt; } pf_job;
+static void* pf_run(void* p) {
+    pf_job* j = (pf_job*)p;
+    for (int64_t i = j->t; i < j->n; i += j->nt) j->fn(j->ctx, i);
+    return NULL;
+}
+static void par_for(int64_t n, int nthreads, idx_fn fn, void* ctx) {
+    if (nthreads > 128) nthreads = 128;
+    if (nthreads <= 1 || n <= 1) {
+        for (int64_t i = 0; i < n; ++i) fn(ctx, i);
+        return;
+    }
+    if (nthreads > n) nthreads = (int)n;
+    pthread_t th[128];
+    pf_job jobs[128];
+    int ok[128];
+    for (int t = 0; t < nthreads; ++t) {
+        jobs[t] = (pf_job){ fn, ctx, n, t, nthreads };
+        ok[t] = pthread_create(&th[t], NULL, pf_run, &jobs[t]) == 0;
+        if (!ok[t]) pf_run(&jobs[t]);
+    }
+    for (int t = 0; t < nthreads; ++t)
+        if (ok[t]) pthread_join(th[t], NULL);
+}
+
+/* --------------------------------------------------------------- primitives */
+
+/* RMSNorm: out = h / sqrt(mean(h^2) + eps) * g. */
+void oracle_rmsnorm(const double* h, const uint16_t* g, int d, double eps, double* out) {
+    double ss = 0.0;
+    for (int i = 0; i < d; ++i) ss += h[i] * h[i];
+    double r = 1.0 / sqrt(ss / d + eps);
+    for (int i = 0; i < d; ++i) out[i] = h[i] * r * bf16_to_f64(g[i]);
+}
+
+/* Rotary embedding, rotate-half convention: for i < hd/2 the pair
+ * (x_i, x_{i+hd/2}) is rotated by the angle pos * base^(-2i/hd). */
+void oracle_rope(double* x, int hd, double pos, double base) {
+    int half = hd / 2;
+    for (int i = 0; i < half; ++i) {
+        double ang = pos * pow(base, -2.0 * i / hd);
+        double c = cos(ang), s = sin(ang);
+        double a = x[i], b = x[i + half];
+        x[i] = a * c - b * s;
+        x[i + half] = b * c + a * s;
+    }
+}
+
+/* Attention read-out of one query head (App. A.3), with the verify token's own
+ * key/value as the last entry:
+ *   s_j = q . K_j / sqrt(hd) for j < L,   s_L = q . k_self / sqrt(hd)
+ *   w = softmax(s),  o = sum_j w_j V_j + w_L v_self.
+ * K and V are bf16 rows with `stride` elements between consecutive tokens.
+ * If `weights` is non-NULL it receives the L + 1 softmax weights. */
+void oracle_attend(const double* q, const uint16_t* K, const uint16_t* V, int64_t L, int64_t stride,
+                   const double* k_self, const double* v_self, int hd, double* o, double* weights) {
+    double scale = 1.0 / sqrt((double)hd);
+    double* s = (double*)malloc(sizeof(double) * (size_t)(L + 1));
+    for (int64_t j = 0; j < L; ++j) {
+        double acc = 0.0;
+        for (int d = 0; d < hd; ++d) acc += q[d] * bf16_to_f64(K[j * stride + d]);
+        s[j] = acc * scale;
+    }
+    {
+        double acc = 0.0;
+        for (int d = 0; d < hd; ++d) acc += q[d] * k_self[d];
+        s[L] = acc * scale;
+    }
+#if ORACLE_MUTANT == 1 /* planted mistake: the verify token ignores itself */
+    if (L > 0) s[L] = -INFINITY;
+#endif
+    double m = s[0];
+    for (int64_t j = 1; j <= L; ++j)
+        if (s[j] > m) m = s[j];
+    double l = 0.0;
+    for (int64_t j = 0; j <= L; ++j) {
+        s[j] = exp(s[j] - m);
+        l += s[j];
+    }
+    for (int d = 0; d < hd; ++d) o[d] = 0.0;
+    for (int64_t j = 0; j < L; ++j) {
+        double w = s[j] / l;
+        for (int d = 0; d < hd; ++d) o[d] += w * bf16_to_f64(V[j * stride + d]);
+    }
+    {
+        double w = s[L] / l;
+        for (int d = 0; d < hd; ++d) o[d] += w * v_self[d];
+    }
+    if (weights)
+        for (int64_t j = 0; j <= L; ++j) weights[j] = s[j] / l;
+    free(s);
+}
+
+/* Reward head (Eq. score): P(+) = softmax([z_-, z_+]) at "+" = 1/(1+exp(z_- - z_+)). */
+double oracle_reward(const double* x, const uint16_t* w_plus, const uint16_t* w_minus, int d) {
+    double zp = 0.0, zm = 0.0;
+    for (int i = 0; i < d; ++i) {
+        zp += bf16_to_f64(w_plus[i]) * x[i];
+        zm += bf16_to_f64(w_minus[i]) * x[i];
+    }
+#if ORACLE_MUTANT == 7 /* planted mistake: the "-" entry is read as P(+) */
+    return 1.0 / (1.0 + exp(zp - zm));
+#else
+    return 1.0 / (1.0 + exp(zm - zp));
+#endif
+}
+
+/* ------------------------------------------------------------- projections */
+/* y[i][r] (+)= sum_c W[r][c] * x[i][c] for n candidates; W is bf16 [rows][cols]. */
+typedef struct {
+    const uint16_t* W; int rows, cols; const double* x; double* y; int n; int accumulate; int transposed;
+} proj_ctx;
+static void proj_row(void* p, int64_t r) {
+    const proj_ctx* c = (const proj_ctx*)p;
+    for (int i = 0; i < c->n; ++i) {
+        const double* xi = c->x + (int64_t)i * c->cols;
+        double acc = 0.0;
+        for (int k = 0; k < c->cols; ++k) {
+            int64_t idx = c->transposed ? (int64_t)k * c->rows + r : r * (int64_t)c->cols + k;
+            acc += bf16_to_f64(c->W[idx]) * xi[k];
+        }
+        double* yi = c->y + (int64_t)i * c->rows + r;
+        *yi = c->accumulate ? *yi + acc : acc;
+    }
+}
+static void project(const oracle_cfg* cfg, const uint16_t* W, int rows, int cols, const double* x, double* y, int n,
+                    int accumulate, int transposed) {
+    proj_ctx c = { W, rows, cols, x, y, n, accumulate, transposed };
+    par_for(rows, cfg->nthreads, proj_row, &c);
+}
+
+/* ------------------------------------------------------------- attention */
+typedef struct {
+    const oracle_cfg* cfg;
+    const double* q;        /* [n][nq][hd]   rotated (and rounded in mirror mode) */
+    const double* kself;    /* [n][nkv][hd] */
+    const double* vself;    /* [n][nkv][hd] */
+    uint16_t* const* K;     /* per candidate [L][nkv][hd] */
+    uint16_t* const* V;
+    const int64_t* lens;
+    double* o;              /* [n][nq][hd] */
+} attn_ctx;
+static void attn_item(void* p, int64_t it) {
+    const attn_ctx* c = (const attn_ctx*)p;
+    const oracle_cfg* cfg = c->cfg;
+    int nq = cfg->n_q_heads, nkv = cfg->n_kv_heads, hd = cfg->head_dim, G = nq / nkv;
+    int i = (int)(it / nq), h = (int)(it % nq);
+#if ORACLE_MUTANT == 3 /* planted mistake: interleaved instead of contiguous head groups */
+    int g = h % nkv;
+#elif ORACLE_MUTANT == 12 /* planted mistake: every query head reads kv head 0 */
+    int g = 0;
+    (void)G;
+#else
+    int g = h / G;
+#endif
+    const double* q = c->q + ((int64_t)i * nq + h) * hd;
+    double qs[1024];
+#if ORACLE_MUTANT == 4 /* planted mistake: scores not divided by sqrt(hd) */
+    for (int d = 0; d < hd; ++d) qs[d] = q[d] * sqrt((double)hd);
+#else
+    for (int d = 0; d < hd; ++d) qs[d] = q[d];
+#endif
+    oracle_attend(qs, c->K[i] + (int64_t)g * hd, c->V[i] + (int64_t)g * hd, c->lens[i], (int64_t)nkv * hd,
+                  c->kself + ((int64_t)i * nkv + g) * hd, c->vself + ((int64_t)i * nkv + g) * hd, hd,
+                  c->o + ((int64_t)i * nq + h) * hd, NULL);
+}
+
+/* ------------------------------------------------------------------ scorer */
+/*
+ * Score n candidates.  cand_ids[i] is passed to the kv provider; lens[i] is its
+ * cached length L.  Outputs: p_plus[n]; if non-NULL, attn_out[N_L][n][nq*hd]
+ * (each layer's attention output o before rounding) and h_out[n][d] (final
+ * residual stream).  Returns 0, or a negative code when a provider fails or
+ * memory runs out.
+ */
+int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracle_kv_fn kvfn, void* kvuser, int n,
+                 const int32_t* cand_ids, const int64_t* lens, double* p_plus, double* attn_out, double* h_out) {
+    const int NL = cfg->n_layers, d = cfg->d_model, nq = cfg->n_q_heads, nkv = cfg->n_kv_heads, hd = cfg->head_dim;
+    const int ff = cfg->d_ff, qkv_rows = (nq + 2 * nkv) * hd;
+    if (hd > 1024 || hd % 2 || nq % nkv) return -1;
+    int rc = 0;
+    uint16_t *embed = malloc(2 * (size_t)d), *gfin = malloc(2 * (size_t)d), *wp = malloc(2 * (size_t)d),
+             *wm = malloc(2 * (size_t)d), *gattn = malloc(2 * (size_t)d), *gmlp = malloc(2 * (size_t)d);
+    uint16_t *Wqkv = malloc(2 * (size_t)qkv_rows * d), *Wo = malloc(2 * (size_t)d * nq * hd),
+             *Wgu = malloc(2 * (size_t)2 * ff * d), *Wd = malloc(2 * (size_t)d * ff);
+    double *h = calloc((size_t)n * d, 8), *x = calloc((size_t)n * d, 8), *qkv = calloc((size_t)n * qkv_rows, 8);
+    double *q = calloc((size_t)n * nq * hd, 8), *ks = calloc((size_t)n * nkv * hd, 8),
+           *vs = calloc((size_t)n * nkv * hd, 8), *o = calloc((size_t)n * nq * hd, 8);
+    double *gu = calloc((size_t)n * 2 * ff, 8), *a = calloc((size_t)n * ff, 8);
+    uint16_t** K = calloc((size_t)n, sizeof(uint16_t*));
+    uint16_t** V = calloc((size_t)n, sizeof(uint16_t*));
+    if (!embed || !gfin || !wp || !wm || !gattn || !gmlp || !Wqkv || !Wo || !Wgu || !Wd || !h || !x || !qkv || !q ||
+        !ks || !vs || !o || !gu || !a || !K || !V) {
+        rc = -2;
+        goto done;
+    }
+    for (int i = 0; i < n; ++i) {
+        size_t sz = 2 * (size_t)(lens[i] > 0 ? lens[i] : 1) * nkv * hd;
+        K[i] = malloc(sz);
+        V[i] = malloc(sz);
+        if (!K[i] || !V[i]) { rc = -2; goto done; }
+    }
+    if (wfn(wuser, K_EMBED, 0, embed, d) || wfn(wuser, K_FINAL_NORM, 0, gfin, d) || wfn(wuser, K_W_PLUS, 0, wp, d) ||
+        wfn(wuser, K_W_MINUS, 0, wm, d)) { rc = -3; goto done; }
+
+    /* the verify token's embedding starts every candidate's residual stream */
+    for (int i = 0; i < n; ++i)
+        for (int c = 0; c < d; ++c) h[(int64_t)i * d + c] = bf16_to_f64(embed[c]);
+
+    for (int l = 0; l < NL; ++l) {
+        if (wfn(wuser, K_ATTN_NORM, l, gattn, d) || wfn(wuser, K_W_QKV, l, Wqkv, (int64_t)qkv_rows * d) ||
+            wfn(wuser, K_W_O, l, Wo, (int64_t)d * nq * hd) || wfn(wuser, K_MLP_NORM, l, gmlp, d) ||
+            wfn(wuser, K_W_GATE_UP, l, Wgu, (int64_t)2 * ff * d) || wfn(wuser, K_W_DOWN, l, Wd, (int64_t)d * ff)) {
+            rc = -3;
+            goto done;
+        }
+        for (int i = 0; i < n; ++i)
+            if (lens[i] > 0 && kvfn(kvuser, l, cand_ids[i], K[i], V[i], lens[i])) { rc = -4; goto done; }
+
+        /* attention block */
+        for (int i = 0; i < n; ++i) {
+            double* xi = x + (int64_t)i * d;
+#if ORACLE_MUTANT == 9 /* planted mistake: eps left out of the norm */
+            oracle_rmsnorm(h + (int64_t)i * d, gattn, d, 0.0, xi);
+#else
+            oracle_rmsnorm(h + (int64_t)i * d, gattn, d, cfg->rms_eps, xi);
+#endif
+            for (int c = 0; c < d; ++c) xi[c] = rnd(cfg, xi[c]);
+        }
+        project(cfg, Wqkv, qkv_rows, d, x, qkv, n, 0, 0);
+        for (int i = 0; i < n; ++i) {
+            const double* r = qkv + (int64_t)i * qkv_rows;
+#if ORACLE_MUTANT == 8 /* planted mistake: verify token placed on the last cached position */
+            double pos = (double)lens[i] - 1.0;
+#else
+            double pos = (double)lens[i];
+#endif
+            for (int hh = 0; hh < nq; ++hh) {
+                double* qh = q + ((int64_t)i * nq + hh) * hd;
+                memcpy(qh, r + (int64_t)hh * hd, 8 * (size_t)hd);
+#if ORACLE_MUTANT == 2 /* planted mistake: rotation in the wrong direction */
+                oracle_rope(qh, hd, -pos, cfg->rope_base);
+#else
+                oracle_rope(qh, hd, pos, cfg->rope_base);
+#endif
+                for (int c = 0; c < hd; ++c) qh[c] = rnd(cfg, qh[c]);
+            }
+            for (int g = 0; g < nkv; ++g) {
+                double* kh = ks + ((int64_t)i * nkv + g) * hd;
+                double* vh = vs + ((int64_t)i * nkv + g) * hd;
+                memcpy(kh, r + (int64_t)(nq + g) * hd, 8 * (size_t)hd);
+                memcpy(vh, r + (int64_t)(nq + nkv + g) * hd, 8 * (size_t)hd);
+                oracle_rope(kh, hd, pos, cfg->rope_base);
+                for (int c = 0; c < hd; ++c) {
+                    kh[c] = rnd(cfg, kh[c]);
+                    vh[c] = rnd(cfg, vh[c]);
+                }
+            }
+        }
+        attn_ctx ac = { cfg, q, ks, vs, K, V, lens, o };
+        par_for((int64_t)n * nq, cfg->nthreads, attn_item, &ac);
+        if (attn_out) memcpy(attn_out + (int64_t)l * n * nq * hd, o, 8 * (size_t)n * nq * hd);
+        for (int64_t e = 0; e < (int64_t)n * nq * hd; ++e) o[e] = rnd(cfg, o[e]);
+#if ORACLE_MUTANT == 5 /* planted mistake: output projection applied transposed */
+        project(cfg, Wo, d, nq * hd, o, h, n, 1, 1);
+#else
+        project(cfg, Wo, d, nq * hd, o, h, n, 1, 0);
+#endif
+
+        /* feed-forward block */
+        for (int i = 0; i < n; ++i) {
+            double* xi = x + (int64_t)i * d;
+            oracle_rmsnorm(h + (int64_t)i * d, gmlp, d, cfg->rms_eps, xi);
+            for (int c = 0; c < d; ++c) xi[c] = rnd(cfg, xi[c]);
+        }
+        project(cfg, Wgu, 2 * ff, d, x, gu, n, 0, 0);
+        for (int i = 0; i < n; ++i)
+            for (int j = 0; j < ff; ++j) {
+                double gt = gu[(int64_t)i * 2 * ff + j], up = gu[(int64_t)i * 2 * ff + ff + j];
+#if ORACLE_MUTANT == 10 /* planted mistake: gate not passed through SiLU */
+                double act = gt * up;
+#elif ORACLE_MUTANT == 14 /* planted mistake: gate and up exchanged */
+                double act = up / (1.0 + exp(-up)) * gt;
+#else
+                double act = gt / (1.0 + exp(-gt)) * up;
+#endif
+                a[(int64_t)i * ff + j] = rnd(cfg, act);
+            }
+#if ORACLE_MUTANT == 6 /* planted mistake: feed-forward output replaces the residual stream */
+        project(cfg, Wd, d, ff, a, h, n, 0, 0);
+#else
+        project(cfg, Wd, d, ff, a, h, n, 1, 0);
+#endif
+    }
+
+    /* reward head on the final-normed stream */
+    for (int i = 0; i < n; ++i) {
+        double* xi = x + (int64_t)i * d;
+        oracle_rmsnorm(h + (int64_t)i * d, gfin, d, cfg->rms_eps, xi);
+        for (int c = 0; c < d; ++c) xi[c] = rnd(cfg, xi[c]);
+        p_plus[i] = oracle_reward(xi, wp, wm, d);
+    }
+    if (h_out) memcpy(h_out, h, 8 * (size_t)n * d);
+
+done:
+    if (K)
+        for (int i = 0; i < n; ++i) free(K[i]);
+    if (V)
+        for (int i = 0; i < n; ++i) free(V[i]);
+    free(K); free(V);
+    free(embed); free(gfin); free(wp); free(wm); free(gattn); free(gmlp);
+    free(Wqkv); free(Wo); free(Wgu); free(Wd);
+    free(h); free(x); free(qkv); free(q); free(ks); free(vs); free(o); free(gu); free(a);
+    return rc;
+}
+
+/* ----------------------------------------------- dense in-memory providers */
+/* Weights held in caller arrays: top[kind] for kinds 0..3, layer[kind-4][l] otherwise. */
+typedef struct {
+    const uint16_t* top[4];
+    const uint16_t* const* layer[6];
+} oracle_dense_weights;
+
+int oracle_dense_weight_provider(void* user, int kind, int layer, uint16_t* out, int64_t n) {
+    const oracle_dense_weights* w = (const oracle_dense_weights*)user;
+    const uint16_t* src = kind < 4 ? w->top[kind] : w->layer[kind - 4][layer];
+    if (!src) return -1;
+    memcpy(out, src, 2 * (size_t)n);
+    return 0;
+}
+
+/* Logical K/V held in caller arrays: K[l * n_cand + cand] -> [L][nkv][hd]. */
+typedef struct {
+    int n_cand;
+    int64_t per_token;              /* nkv * hd */
+    const uint16_t* const* K;
+    const uint16_t* const* V;
+    const int64_t* lens;
+} oracle_dense_kv;
+
+int oracle_dense_kv_provider(void* user, int layer, int cand, uint16_t* K, uint16_t* V, int64_t L) {
+    const oracle_dense_kv* c = (const oracle_dense_kv*)user;
+    if (cand < 0 || cand >= c->n_cand || c->lens[cand] != L) return -1;
+    int64_t slot = (int64_t)layer * c->n_cand + cand;
+    memcpy(K, c->K[slot], 2 * (size_t)(L * c->per_token));
+    memcpy(V, c->V[slot], 2 * (size_t)(L * c->per_token));
+    return 0;
+}

@@ -1,0 +1,129 @@
+"""Pins for the CPU oracle: checks against facts the paper and the mathematics
+fix, written as plain functions so the mutation tests can run them against
+oracle builds with planted mistakes.  Each raises AssertionError on failure."""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+import torch
+import torch.nn.functional as F
+
+import kvsynth as ks
+import oracle
+from oracle.reencode import reencode
+
+RNG = np.random.default_rng(20260101)
+
+
+def _bits(x):
+    return ks.f64_to_bf16_bits(np.asarray(x, dtype=np.float64))
+
+
+def pin_bf16_round(m=0):
+    # ties to even around 1.0 (bf16 spacing 2^-7 there) and torch's own fp32->bf16 rounding
+    assert oracle.bf16_round(1.0 + 2.0 ** -8, m) == 1.0
+    assert oracle.bf16_round(1.0 + 3 * 2.0 ** -8, m) == 1.0 + 2.0 ** -6
+    assert oracle.bf16_round(-(1.0 + 3 * 2.0 ** -8), m) == -(1.0 + 2.0 ** -6)
+    x = RNG.normal(0, 3, 2000).astype(np.float32)
+    ref = torch.from_numpy(x).to(torch.bfloat16).double().numpy()
+    got = np.array([oracle.bf16_round(float(v), m) for v in x])
+    assert np.array_equal(got, ref)
+
+
+def pin_rmsnorm(m=0):
+    d, eps = 64, 1e-6
+    g = _bits(RNG.normal(1, 0.2, d))
+    gf = ks.bf16_bits_to_f64(g)
+    for c in (0.5, -3.0, 1e-3):
+        out = oracle.rmsnorm(np.full(d, c), g, eps, m)
+        np.testing.assert_allclose(out, c / math.sqrt(c * c + eps) * gf, rtol=1e-14, atol=0)
+    h = RNG.normal(0, 1, d)
+    ref = F.rms_norm(torch.from_numpy(h), (d,), weight=torch.from_numpy(gf), eps=eps).numpy()
+    np.testing.assert_allclose(oracle.rmsnorm(h, g, eps, m), ref, rtol=1e-13)
+
+
+def pin_rope(m=0):
+    hd, base = 64, 1e4
+    x = RNG.normal(0, 1, hd)
+    np.testing.assert_array_equal(oracle.rope(x, 0.0, base, m), x)
+    for p in (1.0, 17.0, 4096.0, 32768.0):
+        np.testing.assert_allclose(np.linalg.norm(oracle.rope(x, p, base, m)), np.linalg.norm(x), rtol=1e-13)
+    # one pair (hd = 2): a plain rotation by `pos` radians
+    r = oracle.rope(np.array([1.0, 0.0]), 0.7, base, m)
+    np.testing.assert_allclose(r, [math.cos(0.7), math.sin(0.7)], rtol=1e-15, atol=1e-16)
+    # relative position: <R(m)q, R(n)k> depends on m - n only
+    q, k = RNG.normal(0, 1, hd), RNG.normal(0, 1, hd)
+    a = oracle.rope(q, 100.0, base, m) @ oracle.rope(k, 90.0, base, m)
+    b = oracle.rope(q, 1010.0, base, m) @ oracle.rope(k, 1000.0, base, m)
+    assert abs(a - b) < 1e-10 * (1 + abs(a))
+
+
+def pin_attend(m=0):
+    hd = 64
+    q = RNG.normal(0, 1, hd)
+    ks_, vs_ = RNG.normal(0, 1, hd), RNG.normal(0, 1, hd)
+    # (i) empty cache: the verify token reads its own value
+    o, w = oracle.attend(q, np.zeros((0, hd), np.uint16), np.zeros((0, hd), np.uint16), ks_, vs_, m)
+    np.testing.assert_array_equal(o, vs_)
+    np.testing.assert_array_equal(w, [1.0])
+    # (ii) identical keys (all equal to the self key): the mean of the values
+    L = 9
+    kb = np.tile(_bits(ks_), (L, 1))
+    ksr = ks.bf16_bits_to_f64(_bits(ks_))
+    V = _bits(RNG.normal(0, 1, (L, hd)))
+    o, w = oracle.attend(q, kb, V, ksr, vs_, m)
+    mean = (ks.bf16_bits_to_f64(V).sum(0) + vs_) / (L + 1)
+    np.testing.assert_allclose(o, mean, rtol=1e-12, atol=1e-14)
+    # (iii) q = 0: uniform weights
+    K = _bits(RNG.normal(0, 1, (L, hd)))
+    o, w = oracle.attend(np.zeros(hd), K, V, ks_, vs_, m)
+    np.testing.assert_allclose(o, mean, rtol=1e-12, atol=1e-14)
+    # (iv) two entries: weight of the cached one is sigmoid(s_1 - s_self)
+    o, w = oracle.attend(q, K[:1], V[:1], ks_, vs_, m)
+    s1 = q @ ks.bf16_bits_to_f64(K[0]) / math.sqrt(hd)
+    s2 = q @ ks_ / math.sqrt(hd)
+    np.testing.assert_allclose(w[0], 1.0 / (1.0 + math.exp(s2 - s1)), rtol=1e-13)
+    # (v) weights sum to one; (vi) invariance to the order of cached positions
+    L = 257
+    K = _bits(RNG.normal(0, 1, (L, hd)))
+    V = _bits(RNG.normal(0, 1, (L, hd)))
+    o, w = oracle.attend(q, K, V, ks_, vs_, m)
+    assert abs(w.sum() - 1.0) < 1e-12
+    perm = RNG.permutation(L)
+    o2, _ = oracle.attend(q, K[perm], V[perm], ks_, vs_, m)
+    np.testing.assert_allclose(o2, o, rtol=1e-12, atol=1e-14)
+    # library cross-check: causal SDPA row L over [K; k_self]
+    Kf = torch.from_numpy(np.vstack([ks.bf16_bits_to_f64(K), ks_[None]]))
+    Vf = torch.from_numpy(np.vstack([ks.bf16_bits_to_f64(V), vs_[None]]))
+    ref = F.scaled_dot_product_attention(torch.from_numpy(q)[None, None], Kf[None], Vf[None])[0, 0].numpy()
+    np.testing.assert_allclose(o, ref, rtol=1e-11, atol=1e-13)
+
+
+def pin_reward(m=0):
+    d = 128
+    x = RNG.normal(0, 1, d)
+    w1 = _bits(RNG.normal(0, 0.02, d))
+    w2 = _bits(RNG.normal(0, 0.02, d))
+    assert oracle.reward(x, w1, w1, m) == 0.5
+    p = oracle.reward(x, w1, w2, m)
+    zp, zm = ks.bf16_bits_to_f64(w1) @ x, ks.bf16_bits_to_f64(w2) @ x
+    ref = torch.softmax(torch.tensor([zm, zp], dtype=torch.float64), 0)[1].item()
+    assert abs(p - ref) < 1e-15
+    assert abs(oracle.reward(x, w2, w1, m) - (1 - p)) < 1e-15
+
+
+def pin_reencode(m=0, lens=(0, 1, 5, 16, 17, 40), mirror=True, arch=None):
+    """Verify-against-cache == last position of a full causal forward over [x; v]."""
+    arch = arch or ks.ARCH_TINY
+    t = ks.Tables.make(0.2)
+    W = ks.host_weights(arch, 77, t)
+    for L in lens:
+        xs = np.random.default_rng(1000 + L).normal(0, 1, (L, arch.d_model))
+        p, attn, cache = reencode(arch, W, xs, mirror)
+        r = oracle.score_dense(arch, W, [[cache[l]] for l in range(arch.n_layers)], mirror=mirror, mutant=m)
+        assert abs(p - r.p_plus[0]) < 1e-12, (L, p, r.p_plus[0])
+        np.testing.assert_allclose(r.attn[:, 0], attn, rtol=1e-9, atol=1e-12)
+
+
+ALL_PINS = [pin_bf16_round, pin_rmsnorm, pin_rope, pin_attend, pin_reward, pin_reencode]

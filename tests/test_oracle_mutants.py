@@ -1,0 +1,31 @@
+"""Each planted mistake in the oracle (compiled with -DORACLE_MUTANT=n) must be
+caught by at least one pin, so the pins constrain every step of the scorer."""
+import pytest
+
+from tests import oracle_pins as P
+
+MUTANTS = {
+    1: "verify token ignores its own key/value",
+    2: "RoPE rotates the wrong way",
+    3: "interleaved instead of contiguous query-head groups",
+    4: "scores not scaled by 1/sqrt(hd)",
+    5: "output projection transposed",
+    6: "feed-forward output replaces the residual",
+    7: "P(+) read from the '-' entry",
+    8: "verify token placed at position L-1",
+    9: "RMSNorm without eps",
+    10: "gate not passed through SiLU",
+    12: "all query heads read kv head 0",
+    14: "gate and up exchanged",
+}
+
+
+@pytest.mark.parametrize("mutant", sorted(MUTANTS))
+def test_mutant_is_caught(mutant):
+    caught = []
+    for pin in P.ALL_PINS:
+        try:
+            pin(mutant)
+        except AssertionError:
+            caught.append(pin.__name__)
+    assert caught, f"planted mistake {mutant} ({MUTANTS[mutant]}) passed every pin"
