@@ -1,0 +1,205 @@
+/*
+ * kvprm.h -- C ABI of the GB300 (sm_103a) KV-PRM verify-token scoring library.
+ *
+ * KV-PRM (Sec. 4.1, Eq. score) scores a candidate trajectory by forwarding one
+ * "verify" token through the scorer's layers; at every layer its query attends
+ * over the generator's existing per-layer key/value cache of that candidate
+ * (the attention read-out of App. A.3, k = 1 query in the depth-k read-out of
+ * Def. 1), and a two-logit head over the judgment tokens "+"/"-" (App. B.2)
+ * gives the reward s = P(+) = softmax([z_-, z_+]) at "+".  The cost per call is
+ * N_L * (c_attn d L + c_ffn d^2) (Eq. cost_kv): the cache is read once and the
+ * scorer's weights are streamed once per call, for all candidates together.
+ *
+ * Conventions (all entry points):
+ *  - Return 0 (KVPRM_OK) or a positive KVPRM_E* code; no entry point aborts.
+ *    kvprm_last_error() describes the last failure on a context.  All
+ *    argument checks run on the host before anything is enqueued.
+ *  - "device" pointers are CUDA device (or managed) memory on the device that
+ *    was current when the context was created; "host" pointers are ordinary
+ *    host memory.  Tensors are dense, row-major, 16-byte aligned.
+ *  - bf16 = IEEE bfloat16 bit patterns (uint16 storage).
+ *  - A context is used by one host thread at a time.  Work is enqueued on the
+ *    caller's CUDA stream (NULL = legacy default stream).
+ *  - The library never writes the caller's weights or key/value pages.
+ */
+#ifndef KVPRM_H
+#define KVPRM_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define KVPRM_API __attribute__((visibility("default")))
+#else
+#define KVPRM_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum {
+  KVPRM_OK = 0,
+  KVPRM_EINVAL = 1,       /* malformed argument (null pointer, bad shape, misalignment) */
+  KVPRM_ECAPACITY = 2,    /* more candidates, or a longer cache, than the context was created for */
+  KVPRM_EINDEX = 3,       /* a block-table entry outside [0, n_pages) */
+  KVPRM_ECUDA = 4,        /* a CUDA runtime/driver call failed */
+  KVPRM_ENOMEM = 5,       /* device or pinned-host allocation failed */
+  KVPRM_ETIMEOUT = 6,     /* a bounded in-kernel wait gave up (blocking calls, kvprm_check_device) */
+  KVPRM_EUNSUPPORTED = 7  /* a shape this build does not implement */
+};
+
+/* Scorer shape and context capacity.
+ *  n_layers N_L, d_model d, n_q_heads, n_kv_heads (GQA: query head h reads kv
+ *  head floor(h / G), G = n_q_heads / n_kv_heads, 1 <= G <= 16), head_dim in
+ *  {64, 128}, d_ff (SiLU-gated MLP width), page_size must be 16.
+ *  rope_base: rotary base (rotate-half pairs (i, i + hd/2), angle
+ *  p * base^(-2i/hd), the verify token at position p = L_b).  rms_eps: RMSNorm
+ *  epsilon.  max_candidates in [1, 256]; max_blocks_per_seq = the row length of
+ *  every block table passed to this context.
+ *  d_model, n_q_heads*head_dim and d_ff must be multiples of 64. */
+typedef struct {
+  int32_t n_layers, d_model, n_q_heads, n_kv_heads, head_dim, d_ff, page_size;
+  float rope_base, rms_eps;
+  int32_t max_candidates, max_blocks_per_seq;
+} kvprm_config;
+
+/* Scorer weights: device bf16, row-major [out][in], borrowed (must outlive the
+ * context; not copied).  Per-layer members are HOST arrays of N_L device
+ * pointers (the arrays themselves are read during kvprm_create only).
+ *  embed_verify [d]     the verify token's embedding row
+ *  final_norm   [d]     final RMSNorm gain
+ *  w_plus, w_minus [d]  output-head rows of the "+" and "-" judgment tokens
+ *  attn_norm[l] [d]     pre-attention RMSNorm gain
+ *  w_qkv[l]     [(n_q + 2 n_kv) hd][d]   rows: q heads, then k heads, then v heads
+ *  w_o[l]       [d][n_q hd]
+ *  mlp_norm[l]  [d]     pre-MLP RMSNorm gain
+ *  w_gate_up[l] [2 d_ff][d]              rows: gate, then up
+ *  w_down[l]    [d][d_ff]                                                   */
+typedef struct {
+  const void* embed_verify;
+  const void* final_norm;
+  const void* w_plus;
+  const void* w_minus;
+  const void* const* attn_norm;
+  const void* const* w_qkv;
+  const void* const* w_o;
+  const void* const* mlp_norm;
+  const void* const* w_gate_up;
+  const void* const* w_down;
+} kvprm_weights;
+
+typedef struct kvprm_ctx kvprm_ctx;
+
+/* Create a scoring context: validates the shape, borrows the weights, builds
+ * the weight tensor maps and allocates the device workspace (sized for
+ * max_candidates x max_blocks_per_seq) on the current device.  On failure
+ * *out is NULL and the return code says why (details are not retrievable
+ * without a context).  Sec. 4.1 "Architecture". */
+KVPRM_API int kvprm_create(const kvprm_config* cfg, const kvprm_weights* weights, kvprm_ctx** out);
+
+/* Free the workspace.  Waits for work the context enqueued.  NULL is a no-op. */
+KVPRM_API void kvprm_destroy(kvprm_ctx* ctx);
+
+/* Human-readable description of the last failure on ctx ("" if none).  The
+ * string is owned by the context and valid until the next call on it. */
+KVPRM_API const char* kvprm_last_error(const kvprm_ctx* ctx);
+
+/* Score n_candidates trajectories against their paged caches (Sec. 4.1 Eq.
+ * score; the verify token is appended after each candidate's cache, Sec. 1).
+ *  kv_pages     device bf16 [N_L][n_pages][2][n_kv_heads][16][head_dim]:
+ *               per layer and physical page, the 16 cached keys (index 0) and
+ *               values (index 1) of every kv head.  Keys are post-RoPE.
+ *  n_pages      physical pages per layer in kv_pages.
+ *  block_table  host int32 [n_candidates][max_blocks_per_seq]: logical page j
+ *               of candidate b (positions 16j .. 16j+15) is physical page
+ *               block_table[b][j].  Candidates may share pages (beam / MCTS
+ *               siblings).  Entries j >= ceil(seq_lens[b] / 16) are ignored.
+ *  seq_lens     host int32 [n_candidates]: cached length L_b in
+ *               [0, 16 * max_blocks_per_seq].  L_b = 0 is legal (the verify
+ *               token then attends to itself only).
+ *  n_candidates 0 .. max_candidates (0 is a no-op).
+ *  rewards      host float [n_candidates]: P(+) per candidate.
+ *  stream       cudaStream_t or NULL.
+ * Blocking: returns after rewards are written.  The verify token's own k/v are
+ * kept in the workspace, never written into kv_pages. */
+KVPRM_API int kvprm_score(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const int32_t* block_table,
+                const int32_t* seq_lens, int32_t n_candidates, float* rewards, void* stream);
+
+/* As kvprm_score, but stream-ordered: d_rewards is device float [n_candidates]
+ * and the call returns once the work is enqueued.  block_table and seq_lens are
+ * host arrays; they are copied before the call returns. */
+KVPRM_API int kvprm_score_async(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const int32_t* block_table,
+                      const int32_t* seq_lens, int32_t n_candidates, float* d_rewards, void* stream);
+
+/* As kvprm_score, but with the cache in HOST memory: h_kv_pages has the
+ * kv_pages layout above (pinned memory gives full copy bandwidth).  The pages
+ * are copied into a library-owned device pool (grown on demand) on `stream`
+ * before scoring; rewards is a host array.  Blocking. */
+KVPRM_API int kvprm_score_host(kvprm_ctx* ctx, const void* h_kv_pages, int64_t n_pages, const int32_t* block_table,
+                     const int32_t* seq_lens, int32_t n_candidates, float* rewards, void* stream);
+
+/* Paged GQA attention read-out alone (App. A.3 with the self entry; the inner
+ * step of kvprm_score), for callers that already hold the verify token's
+ * rotated query and its own key/value:
+ *  kv_layer  device bf16 [n_pages][2][n_kv_heads][16][head_dim] (one layer)
+ *  q         device float [n_candidates][n_q_heads][head_dim]
+ *  k_self, v_self  device float [n_candidates][n_kv_heads][head_dim]
+ *  out       device float [n_candidates][n_q_heads][head_dim]
+ * block_table / seq_lens as in kvprm_score.  Stream-ordered. */
+KVPRM_API int kvprm_attention(kvprm_ctx* ctx, const void* kv_layer, int64_t n_pages, const int32_t* block_table,
+                    const int32_t* seq_lens, int32_t n_candidates, const void* q, const void* k_self,
+                    const void* v_self, float* out, void* stream);
+
+/* One projection of the verify-token forward alone (the c_ffn d^2 term of
+ * Eq. cost_kv), batched over candidates: Y[n][M] = X[n][K] * W[M][K]^T with
+ * bf16 inputs and fp32 accumulation, using the context's split-K GEMM and
+ * workspace.  W device bf16 [M][K] (16-byte aligned, K a multiple of 8),
+ * X device bf16 [n][K], Y device float [n][M]; 1 <= n <= max_candidates and
+ * M * n must fit the context's partial buffer (any M, K of the context's
+ * scorer shape does).  Stream-ordered. */
+KVPRM_API int kvprm_projection(kvprm_ctx* ctx, const void* W, int32_t M, int32_t K, const void* X, int32_t n,
+                               float* Y, void* stream);
+
+/* Final residual stream h (float [n_candidates][d_model], before the final
+ * RMSNorm) of the last kvprm_score* call, copied to device memory d_out
+ * (stream-ordered on the last call's stream). */
+KVPRM_API int kvprm_debug_hidden(kvprm_ctx* ctx, float* d_out);
+
+/* Debug capture.  flags bit 0: keep every layer's attention output (the
+ * combine result o, float, before its bf16 rounding) of each later
+ * kvprm_score* call.  kvprm_debug_attn_out copies the last call's capture to
+ * device float [N_L][n_candidates][n_q_heads * head_dim] (stream-ordered on
+ * the last call's stream).  Bit 1: keep every layer's rotated q, self k and
+ * self v (float); bit 2: keep the residual stream after every layer (float).
+ * kvprm_debug_layers copies them: which = 1 q [N_L][n][n_q*hd], 2 k_self
+ * [N_L][n][n_kv*hd], 3 v_self (same), 4 h [N_L][n][d_model]. */
+KVPRM_API int kvprm_set_debug(kvprm_ctx* ctx, int flags);
+KVPRM_API int kvprm_debug_attn_out(kvprm_ctx* ctx, float* d_out);
+KVPRM_API int kvprm_debug_layers(kvprm_ctx* ctx, int which, void* d_out);
+
+/* Page resolution of the last kvprm_score* call (the block-table walk the
+ * attention kernel performs): phys_row[j] = block_table[b][j / 16] * 16 + j % 16
+ * for j < seq_lens[b], computed on the device; phys_row is host int64 [L_b].
+ * Blocking. */
+KVPRM_API int kvprm_resolve(kvprm_ctx* ctx, int32_t b, int64_t* phys_row);
+
+/* Device-side status: returns KVPRM_OK, or KVPRM_ETIMEOUT if an in-kernel
+ * bounded wait gave up since the last check (the flag is then cleared).
+ * Synchronises the context's last stream. */
+KVPRM_API int kvprm_check_device(kvprm_ctx* ctx);
+
+/* Per-kernel-class timing of kvprm_score* calls, measured with CUDA events on
+ * the scoring stream while enabled (adds one event pair per timed launch).
+ * Classes: 0 projection GEMMs, 1 paged attention (split-K), 2 attention
+ * combine, 3 fused norm / RoPE / SiLU / head kernels.  kvprm_get_profile
+ * synchronises, accumulates the recorded pairs and returns per class the
+ * launch count and total milliseconds since profiling was enabled. */
+enum { KVPRM_PROF_GEMM = 0, KVPRM_PROF_ATTN = 1, KVPRM_PROF_COMBINE = 2, KVPRM_PROF_FUSED = 3, KVPRM_PROF_N = 4 };
+KVPRM_API int kvprm_set_profile(kvprm_ctx* ctx, int enable);
+KVPRM_API int kvprm_get_profile(kvprm_ctx* ctx, int64_t* launches, double* total_ms);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KVPRM_H */

@@ -82,7 +82,7 @@ def lib(mutant: int = 0) -> ctypes.CDLL:
         L.oracle_reward.argtypes = [_f64p, _u16p, _u16p, ctypes.c_int]
         L.oracle_score.argtypes = [ctypes.POINTER(OracleCfg), ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
                                    ctypes.c_void_p, ctypes.c_int, ctypes.POINTER(ctypes.c_int32),
-                                   ctypes.POINTER(ctypes.c_int64), _f64p, _f64p, _f64p]
+                                   ctypes.POINTER(ctypes.c_int64), _f64p, _f64p, _f64p, _f64p, _f64p]
         _libs[mutant] = L
     return _libs[mutant]
 
@@ -141,37 +141,42 @@ def reward(x, wp_bits, wm_bits, mutant: int = 0) -> float:
 
 # ------------------------------------------------------------------ scorer
 class Result:
-    def __init__(self, p_plus, attn, hidden):
-        self.p_plus, self.attn, self.hidden = p_plus, attn, hidden
+    def __init__(self, p_plus, attn, hidden, qkv=None, h_layers=None):
+        self.p_plus, self.attn, self.hidden, self.qkv, self.h_layers = p_plus, attn, hidden, qkv, h_layers
 
 
-def _score(arch, wfn, wuser, kvfn, kvuser, cand_ids, lens, mirror, want_attn, want_hidden, nthreads, mutant):
+def _score(arch, wfn, wuser, kvfn, kvuser, cand_ids, lens, mirror, want_attn, want_hidden, nthreads, mutant,
+           want_layers=False):
     n = len(cand_ids)
     ids = np.ascontiguousarray(cand_ids, np.int32)
     lens = np.ascontiguousarray(lens, np.int64)
     p = np.empty(n)
     attn = np.empty((arch.n_layers, n, arch.n_q_heads * arch.head_dim)) if want_attn else None
     hid = np.empty((n, arch.d_model)) if want_hidden else None
+    qkv = np.empty((arch.n_layers, n, arch.qkv_rows)) if want_layers else None
+    hl = np.empty((arch.n_layers, n, arch.d_model)) if want_layers else None
     cfg = OracleCfg.from_arch(arch, mirror, nthreads)
     rc = lib(mutant).oracle_score(ctypes.byref(cfg), wfn, wuser, kvfn, kvuser, n,
                                   ids.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)),
                                   lens.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)), p.ctypes.data_as(_f64p),
                                   attn.ctypes.data_as(_f64p) if attn is not None else None,
-                                  hid.ctypes.data_as(_f64p) if hid is not None else None)
+                                  hid.ctypes.data_as(_f64p) if hid is not None else None,
+                                  qkv.ctypes.data_as(_f64p) if qkv is not None else None,
+                                  hl.ctypes.data_as(_f64p) if hl is not None else None)
     if rc != 0:
         raise RuntimeError(f"oracle_score failed with code {rc}")
-    return Result(p, attn, hid)
+    return Result(p, attn, hid, qkv, hl)
 
 
 def score_synth(w, tables, cand_ids=None, mirror: bool = True, want_attn: bool = True, want_hidden: bool = False,
-                nthreads: int | None = None, mutant: int = 0) -> Result:
+                nthreads: int | None = None, mutant: int = 0, want_layers: bool = False) -> Result:
     """Score candidates of a kvsynth workload; K/V come from their logical token identities."""
     import kvsynth
     prov = kvsynth.Providers(w, tables, nthreads)
     ids = list(range(w.n_candidates)) if cand_ids is None else list(cand_ids)
     lens = [len(w.cand_seg[i]) for i in ids]
     return _score(w.arch, prov.weight_fn, prov.user, prov.kv_fn, prov.user, ids, lens, mirror, want_attn, want_hidden,
-                  nthreads, mutant)
+                  nthreads, mutant, want_layers)
 
 
 def score_dense(arch, weights: dict, kv: list, mirror: bool = True, want_attn: bool = True, want_hidden: bool = False,

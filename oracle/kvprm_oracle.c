@@ -34,12 +34,17 @@
  *     h  += W_down (SiLU(W_gate x) * (W_up x))      W_gate_up rows: [gate | up]
  *   then x = RMSNorm(h) * g_final, z_+ = w_plus . x, z_- = w_minus . x.
  *
- * Precision contract ("mirror" mode): the paper trains and serves in bf16
- * (App. B.1), so weights and cached K/V are bf16 values, and the oracle rounds
- * to bf16 (round to nearest, ties to even) exactly where the scoring library
- * stores bf16: every projection input (x after each norm, the attention output
- * o, the SiLU(gate)*up product, the final x), the rotated q, and the self k/v.
- * "exact" mode skips those intermediate roundings.
+ * Precision.  The paper trains and serves in bf16 (App. B.1), so weights and
+ * cached K/V are bf16 values.  "exact" mode (mirror = 0) computes everything
+ * else exactly (double) on those bf16 inputs; it is the reference the CUDA
+ * library is compared with.  "mirror" mode (mirror = 1) additionally rounds to
+ * bf16 (nearest, ties to even) every activation a bf16 inference stack would
+ * round: each projection input (x after each norm, the attention output o,
+ * the SiLU(gate)*up product, the final x), the rotated q and the self k/v.  It
+ * measures how far such a stack drifts from the exact value; it is not used
+ * as a reference because two correct bf16 stacks that round from different
+ * intermediate precisions disagree by whole bf16 ulps, and those differences
+ * compound from layer to layer.
  *
  * Inputs arrive through provider callbacks (weights one matrix at a time, the
  * logical per-candidate K/V one layer at a time), so full-size workloads need
@@ -260,12 +265,15 @@ static void attn_item(void* p, int64_t it) {
 /*
  * Score n candidates.  cand_ids[i] is passed to the kv provider; lens[i] is its
  * cached length L.  Outputs: p_plus[n]; if non-NULL, attn_out[N_L][n][nq*hd]
- * (each layer's attention output o before rounding) and h_out[n][d] (final
- * residual stream).  Returns 0, or a negative code when a provider fails or
+ * (each layer's attention output o before rounding), h_out[n][d] (final
+ * residual stream), qkv_out[N_L][n][(nq+2nkv)*hd] (each layer's rotated q,
+ * self k and self v as the attention consumes them) and
+ * h_layers_out[N_L][n][d] (residual stream after each layer).  Returns 0, or a negative code when a provider fails or
  * memory runs out.
  */
 int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracle_kv_fn kvfn, void* kvuser, int n,
-                 const int32_t* cand_ids, const int64_t* lens, double* p_plus, double* attn_out, double* h_out) {
+                 const int32_t* cand_ids, const int64_t* lens, double* p_plus, double* attn_out, double* h_out,
+                 double* qkv_out, double* h_layers_out) {
     const int NL = cfg->n_layers, d = cfg->d_model, nq = cfg->n_q_heads, nkv = cfg->n_kv_heads, hd = cfg->head_dim;
     const int ff = cfg->d_ff, qkv_rows = (nq + 2 * nkv) * hd;
     if (hd > 1024 || hd % 2 || nq % nkv) return -1;
@@ -348,6 +356,13 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
                 }
             }
         }
+        if (qkv_out)
+            for (int i = 0; i < n; ++i) {
+                double* dst = qkv_out + ((int64_t)l * n + i) * qkv_rows;
+                memcpy(dst, q + (int64_t)i * nq * hd, 8 * (size_t)nq * hd);
+                memcpy(dst + (int64_t)nq * hd, ks + (int64_t)i * nkv * hd, 8 * (size_t)nkv * hd);
+                memcpy(dst + (int64_t)(nq + nkv) * hd, vs + (int64_t)i * nkv * hd, 8 * (size_t)nkv * hd);
+            }
         attn_ctx ac = { cfg, q, ks, vs, K, V, lens, o };
         par_for((int64_t)n * nq, cfg->nthreads, attn_item, &ac);
         if (attn_out) memcpy(attn_out + (int64_t)l * n * nq * hd, o, 8 * (size_t)n * nq * hd);
@@ -382,6 +397,7 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
 #else
         project(cfg, Wd, d, ff, a, h, n, 1, 0);
 #endif
+        if (h_layers_out) memcpy(h_layers_out + (int64_t)l * n * d, h, 8 * (size_t)n * d);
     }
 
     /* reward head on the final-normed stream */

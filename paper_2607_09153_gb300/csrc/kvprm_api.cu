@@ -1,0 +1,935 @@
+// C ABI of the KV-PRM scoring library (declared in include/kvprm.h): context
+// creation, host-side validation, block-table upload, tensor maps, the
+// per-call launch sequence of the verify-token forward (Sec. 4.1 Eq. score),
+// and its replay as a CUDA graph.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cstdarg>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/kvprm.h"
+#include "kernels.h"
+
+using kvprm::AttnPlan;
+using kvprm::AttnShape;
+using kvprm::GemmPlan;
+using kvprm::ModelDims;
+typedef __nv_bfloat16 bf16;
+
+namespace {
+
+constexpr int kSplitCap = 32;   // max split-K partials of the attention per (candidate, head)
+
+struct CallPlan {
+  int n = 0, n_pad = 0, max_pages = 0;
+  GemmPlan g_qkv, g_o, g_gu, g_down;
+  AttnPlan attn;
+};
+
+struct GraphKey {
+  int n = -1, n_pad = -1, n_split = -1, pps = -1, debug = -1, profile = -1, pdl = -1;
+  const void* pool = nullptr;
+  int64_t n_pages = -1;
+  bool operator==(const GraphKey& o) const {
+    return n == o.n && n_pad == o.n_pad && n_split == o.n_split && pps == o.pps && debug == o.debug &&
+           profile == o.profile && pdl == o.pdl && pool == o.pool && n_pages == o.n_pages;
+  }
+};
+
+struct ProfMark {
+  int cls;
+  cudaEvent_t a, b;
+};
+
+}  // namespace
+
+struct kvprm_ctx {
+  kvprm_config cfg{};
+  int device = 0, num_sms = 148;
+  ModelDims md{};
+  AttnShape as{};
+  PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+  // borrowed weights
+  const bf16 *embed = nullptr, *final_norm = nullptr, *w_plus = nullptr, *w_minus = nullptr;
+  std::vector<const bf16*> attn_norm, mlp_norm;
+  std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_down;
+  // workspace
+  int npad_max = 16;
+  float* h = nullptr;
+  bf16 *xhi = nullptr, *xlo = nullptr, *ohi = nullptr, *olo = nullptr, *ahi = nullptr, *alo = nullptr;
+  float* part = nullptr;
+  size_t part_elems = 0;
+  float *q = nullptr, *kself = nullptr, *vself = nullptr;
+  bf16 *qhi = nullptr, *qlo = nullptr;
+  float *apart_o = nullptr, *apart_ml = nullptr;
+  float2* rope = nullptr;
+  int32_t* tables_d = nullptr;   // [Bmax] seq_lens, then [Bmax][max_blocks] block table
+  float* rewards_d = nullptr;
+  int* err_d = nullptr;
+  float* dbg = nullptr;
+  float *dbg_q = nullptr, *dbg_k = nullptr, *dbg_v = nullptr;
+  float* dbg_h = nullptr;
+  bf16* dummy_pool = nullptr;
+  int debug_flags = 0;
+  int last_n = 0;
+  // pinned staging
+  int32_t* staging = nullptr;
+  float* h_rewards = nullptr;
+  int* h_err = nullptr;
+  cudaEvent_t staging_ev = nullptr;
+  bool staging_pending = false;
+  // activation tensor maps (depend on the padded batch)
+  int tm_x_npad = -1;
+  CUtensorMap tm_xhi{}, tm_xlo{}, tm_ohi{}, tm_olo{}, tm_ahi{}, tm_alo{};
+  // pool tensor map (depends on the caller's pool)
+  const void* pool_ptr = nullptr;
+  int64_t pool_pages = -1;
+  int64_t pool_rows = -1;
+  CUtensorMap tm_pool{};
+  // library-owned device pool for kvprm_score_host
+  void* dev_pool = nullptr;
+  size_t dev_pool_bytes = 0;
+  // graph replay
+  cudaStream_t cap_stream = nullptr;
+  bool use_graph = true, use_pdl = true;
+  GraphKey gkey;
+  cudaGraphExec_t gexec = nullptr;
+  std::vector<ProfMark> graph_marks;
+  // profiling
+  bool profile = false;
+  std::vector<ProfMark> live_marks;   // marks recorded in the current (non-graph) capture
+  int64_t prof_launches[KVPRM_PROF_N] = {0, 0, 0, 0};
+  double prof_ms[KVPRM_PROF_N] = {0, 0, 0, 0};
+  std::string last_error;
+  cudaStream_t last_stream = nullptr;
+};
+
+namespace {
+
+int fail(kvprm_ctx* c, int code, const char* fmt, ...) __attribute__((format(printf, 3, 4)));
+int fail(kvprm_ctx* c, int code, const char* fmt, ...) {
+  if (c) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    c->last_error = buf;
+  }
+  return code;
+}
+
+int cuda_fail(kvprm_ctx* c, cudaError_t e, const char* what) {
+  return fail(c, KVPRM_ECUDA, "%s: %s (%s)", what, cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+#define CK(call, what)                                     \
+  do {                                                     \
+    cudaError_t e_ = (call);                               \
+    if (e_ != cudaSuccess) return cuda_fail(ctx, e_, what); \
+  } while (0)
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int make_map(kvprm_ctx* ctx, CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint32_t box_inner,
+             uint32_t box_outer, const char* what) {
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {inner * 2};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = ctx->encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(ctx, KVPRM_ECUDA, "cuTensorMapEncodeTiled(%s) failed with %d", what, (int)r);
+  return KVPRM_OK;
+}
+
+template <typename T>
+int dalloc(kvprm_ctx* ctx, T** p, size_t count, const char* what) {
+  cudaError_t e = cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T) > 0 ? count * sizeof(T) : 16);
+  if (e != cudaSuccess) {
+    *p = nullptr;
+    cudaGetLastError();
+    return fail(ctx, KVPRM_ENOMEM, "cudaMalloc(%s, %zu bytes): %s", what, count * sizeof(T), cudaGetErrorString(e));
+  }
+  e = cudaMemset(*p, 0, count * sizeof(T) > 0 ? count * sizeof(T) : 16);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaMemset");
+  return KVPRM_OK;
+}
+
+void free_ctx(kvprm_ctx* c) {
+  if (!c) return;
+  cudaFree(c->h);
+  cudaFree(c->xhi);
+  cudaFree(c->xlo);
+  cudaFree(c->ohi);
+  cudaFree(c->olo);
+  cudaFree(c->ahi);
+  cudaFree(c->alo);
+  cudaFree(c->qhi);
+  cudaFree(c->qlo);
+  cudaFree(c->part);
+  cudaFree(c->q);
+  cudaFree(c->kself);
+  cudaFree(c->vself);
+  cudaFree(c->apart_o);
+  cudaFree(c->apart_ml);
+  cudaFree(c->rope);
+  cudaFree(c->tables_d);
+  cudaFree(c->rewards_d);
+  cudaFree(c->err_d);
+  cudaFree(c->dbg);
+  cudaFree(c->dbg_q);
+  cudaFree(c->dbg_k);
+  cudaFree(c->dbg_v);
+  cudaFree(c->dbg_h);
+  cudaFree(c->dummy_pool);
+  cudaFree(c->dev_pool);
+  if (c->staging) cudaFreeHost(c->staging);
+  if (c->h_rewards) cudaFreeHost(c->h_rewards);
+  if (c->h_err) cudaFreeHost(c->h_err);
+  if (c->staging_ev) cudaEventDestroy(c->staging_ev);
+  if (c->gexec) cudaGraphExecDestroy(c->gexec);
+  for (auto& m : c->graph_marks) {
+    cudaEventDestroy(m.a);
+    cudaEventDestroy(m.b);
+  }
+  for (auto& m : c->live_marks) {
+    cudaEventDestroy(m.a);
+    cudaEventDestroy(m.b);
+  }
+  if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
+  delete c;
+}
+
+// ---------------------------------------------------------------- per-call checks and plan
+int validate_tables(kvprm_ctx* ctx, int64_t n_pages, const int32_t* bt, const int32_t* sl, int32_t n, int* max_pages) {
+  if (n < 0) return fail(ctx, KVPRM_EINVAL, "n_candidates = %d is negative", n);
+  if (n > ctx->cfg.max_candidates)
+    return fail(ctx, KVPRM_ECAPACITY, "n_candidates = %d exceeds max_candidates = %d", n, ctx->cfg.max_candidates);
+  if (n > 0 && (!bt || !sl)) return fail(ctx, KVPRM_EINVAL, "block_table and seq_lens must not be NULL");
+  const int mb = ctx->cfg.max_blocks_per_seq;
+  int mp = 0;
+  for (int b = 0; b < n; ++b) {
+    const int L = sl[b];
+    if (L < 0) return fail(ctx, KVPRM_EINVAL, "seq_lens[%d] = %d is negative", b, L);
+    if (static_cast<int64_t>(L) > static_cast<int64_t>(mb) * 16)
+      return fail(ctx, KVPRM_ECAPACITY, "seq_lens[%d] = %d exceeds 16 * max_blocks_per_seq = %lld", b, L,
+                  static_cast<long long>(mb) * 16);
+    const int np = (L + 15) / 16;
+    if (np > mp) mp = np;
+    for (int j = 0; j < np; ++j) {
+      const int32_t p = bt[static_cast<int64_t>(b) * mb + j];
+      if (p < 0 || p >= n_pages)
+        return fail(ctx, KVPRM_EINDEX, "block_table[%d][%d] = %d is outside [0, %lld)", b, j, p,
+                    static_cast<long long>(n_pages));
+    }
+  }
+  *max_pages = mp;
+  return KVPRM_OK;
+}
+
+int upload_tables(kvprm_ctx* ctx, const int32_t* bt, const int32_t* sl, int32_t n, cudaStream_t st) {
+  const int Bmax = ctx->cfg.max_candidates, mb = ctx->cfg.max_blocks_per_seq;
+  if (ctx->staging_pending) {
+    CK(cudaEventSynchronize(ctx->staging_ev), "cudaEventSynchronize(staging)");
+    ctx->staging_pending = false;
+  }
+  std::memcpy(ctx->staging, sl, sizeof(int32_t) * n);
+  std::memcpy(ctx->staging + Bmax, bt, sizeof(int32_t) * static_cast<size_t>(n) * mb);
+  const size_t count = static_cast<size_t>(Bmax) + static_cast<size_t>(n) * mb;
+  CK(cudaMemcpyAsync(ctx->tables_d, ctx->staging, count * sizeof(int32_t), cudaMemcpyHostToDevice, st),
+     "cudaMemcpyAsync(tables)");
+  CK(cudaEventRecord(ctx->staging_ev, st), "cudaEventRecord(staging)");
+  ctx->staging_pending = true;
+  return KVPRM_OK;
+}
+
+int ensure_pool_map(kvprm_ctx* ctx, const void* pool, int64_t n_pages, int layers) {
+  if (ctx->pool_ptr == pool && ctx->pool_pages == n_pages && ctx->pool_rows >= 0 &&
+      ctx->pool_rows == static_cast<int64_t>(layers) * n_pages * 2 * ctx->cfg.n_kv_heads * 16)
+    return KVPRM_OK;
+  const int64_t rows = static_cast<int64_t>(layers) * n_pages * 2 * ctx->cfg.n_kv_heads * 16;
+  if (rows >= (static_cast<int64_t>(1) << 31))
+    return fail(ctx, KVPRM_EUNSUPPORTED, "pool of %lld rows exceeds the 2^31-row tensor-map limit",
+                static_cast<long long>(rows));
+  int rc = make_map(ctx, &ctx->tm_pool, pool, ctx->cfg.head_dim, rows, 64, 16, "kv pool");
+  if (rc) return rc;
+  ctx->pool_ptr = pool;
+  ctx->pool_pages = n_pages;
+  ctx->pool_rows = rows;
+  return KVPRM_OK;
+}
+
+int ensure_x_maps(kvprm_ctx* ctx, int n_pad) {
+  if (ctx->tm_x_npad == n_pad) return KVPRM_OK;
+  int rc;
+  const uint64_t d = ctx->md.d, dq = static_cast<uint64_t>(ctx->md.n_q) * ctx->md.hd, ff = ctx->md.ff;
+  if ((rc = make_map(ctx, &ctx->tm_xhi, ctx->xhi, d, n_pad, 64, n_pad, "x_hi"))) return rc;
+  if ((rc = make_map(ctx, &ctx->tm_xlo, ctx->xlo, d, n_pad, 64, n_pad, "x_lo"))) return rc;
+  if ((rc = make_map(ctx, &ctx->tm_ohi, ctx->ohi, dq, n_pad, 64, n_pad, "o_hi"))) return rc;
+  if ((rc = make_map(ctx, &ctx->tm_olo, ctx->olo, dq, n_pad, 64, n_pad, "o_lo"))) return rc;
+  if ((rc = make_map(ctx, &ctx->tm_ahi, ctx->ahi, ff, n_pad, 64, n_pad, "a_hi"))) return rc;
+  if ((rc = make_map(ctx, &ctx->tm_alo, ctx->alo, ff, n_pad, 64, n_pad, "a_lo"))) return rc;
+  ctx->tm_x_npad = n_pad;
+  return KVPRM_OK;
+}
+
+CallPlan make_plan(kvprm_ctx* ctx, int n, int max_pages) {
+  CallPlan p;
+  p.n = n;
+  p.n_pad = (n + 15) / 16 * 16;
+  p.max_pages = max_pages;
+  const ModelDims& m = ctx->md;
+  p.g_qkv = kvprm::plan_gemm(m.qkv_rows, m.d, p.n_pad, ctx->num_sms, true);
+  p.g_o = kvprm::plan_gemm(m.d, m.n_q * m.hd, p.n_pad, ctx->num_sms, true);
+  p.g_gu = kvprm::plan_gemm(2 * m.ff, m.d, p.n_pad, ctx->num_sms, true);
+  p.g_down = kvprm::plan_gemm(m.d, m.ff, p.n_pad, ctx->num_sms, true);
+  p.attn = kvprm::plan_attention(ctx->as, n, max_pages, ctx->num_sms, kSplitCap);
+  return p;
+}
+
+// ---------------------------------------------------------------- launch sequence
+struct Enq {
+  kvprm_ctx* ctx;
+  cudaStream_t st;
+  bool pdl;
+  bool prof;
+  std::vector<ProfMark>* marks;
+  bool capturing = false;
+  cudaError_t rec(cudaEvent_t ev) {
+    return capturing ? cudaEventRecordWithFlags(ev, st, cudaEventRecordExternal) : cudaEventRecord(ev, st);
+  }
+  int begin(int cls, cudaEvent_t* ev_b) {
+    if (!prof) return KVPRM_OK;
+    ProfMark m{cls, nullptr, nullptr};
+    CK(cudaEventCreate(&m.a), "cudaEventCreate");
+    CK(cudaEventCreate(&m.b), "cudaEventCreate");
+    CK(rec(m.a), "cudaEventRecord");
+    marks->push_back(m);
+    *ev_b = m.b;
+    return KVPRM_OK;
+  }
+  int end(cudaEvent_t ev_b) {
+    if (!prof) return KVPRM_OK;
+    CK(rec(ev_b), "cudaEventRecord");
+    return KVPRM_OK;
+  }
+};
+
+#define LAUNCH(cls, expr, what)                    \
+  do {                                             \
+    cudaEvent_t evb_ = nullptr;                    \
+    int rc_ = E.begin(cls, &evb_);                 \
+    if (rc_) return rc_;                           \
+    cudaError_t e_ = (expr);                       \
+    if (e_ != cudaSuccess) return cuda_fail(ctx, e_, what); \
+    rc_ = E.end(evb_);                             \
+    if (rc_) return rc_;                           \
+  } while (0)
+
+int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
+  const ModelDims& m = ctx->md;
+  const int n = P.n, np = P.n_pad;
+  const int32_t* sl = ctx->tables_d;
+  const int32_t* bt = ctx->tables_d + ctx->cfg.max_candidates;
+  cudaStream_t st = E.st;
+  const bool pdl = E.pdl;
+  const int NL = ctx->cfg.n_layers;
+  const kvprm::HiLo X{ctx->xhi, ctx->xlo}, Q{ctx->qhi, ctx->qlo}, O{ctx->ohi, ctx->olo}, A{ctx->ahi, ctx->alo};
+  LAUNCH(KVPRM_PROF_FUSED, kvprm::launch_rope_table(sl, n, m.hd, ctx->cfg.rope_base, ctx->rope, st, false), "rope");
+  LAUNCH(KVPRM_PROF_FUSED, kvprm::launch_embed_norm(m, ctx->embed, ctx->attn_norm[0], n, ctx->h, X, st, pdl),
+         "embed_norm");
+  for (int l = 0; l < NL; ++l) {
+    LAUNCH(KVPRM_PROF_GEMM,
+           kvprm::launch_gemm(P.g_qkv, &ctx->tm_qkv[l], &ctx->tm_xhi, &ctx->tm_xlo, ctx->part, m.qkv_rows, n, np,
+                              ctx->err_d, st, pdl),
+           "gemm_qkv");
+    LAUNCH(KVPRM_PROF_FUSED,
+           kvprm::launch_qkv_post(m, ctx->part, P.g_qkv.splits, n, ctx->rope, ctx->q, Q, ctx->kself, ctx->vself, st,
+                                  pdl),
+           "qkv_post");
+    if (ctx->debug_flags & 2) {
+      const size_t nq = static_cast<size_t>(n) * m.n_q * m.hd, nk = static_cast<size_t>(n) * m.n_kv * m.hd;
+      CK(cudaMemcpyAsync(ctx->dbg_q + l * nq, ctx->q, nq * 4, cudaMemcpyDeviceToDevice, st), "debug q");
+      CK(cudaMemcpyAsync(ctx->dbg_k + l * nk, ctx->kself, nk * 4, cudaMemcpyDeviceToDevice, st), "debug k");
+      CK(cudaMemcpyAsync(ctx->dbg_v + l * nk, ctx->vself, nk * 4, cudaMemcpyDeviceToDevice, st), "debug v");
+    }
+    LAUNCH(KVPRM_PROF_ATTN,
+           kvprm::launch_attn_split(ctx->as, P.attn, &ctx->tm_pool, l, bt, sl, ctx->qhi, ctx->qlo, n, ctx->apart_o,
+                                    ctx->apart_ml, ctx->err_d, st, pdl),
+           "attn_split");
+    float* dbg = (ctx->debug_flags & 1) ? ctx->dbg + static_cast<size_t>(l) * n * m.n_q * m.hd : nullptr;
+    LAUNCH(KVPRM_PROF_COMBINE,
+           kvprm::launch_attn_combine(ctx->as, P.attn, sl, ctx->q, ctx->kself, ctx->vself, ctx->apart_o,
+                                      ctx->apart_ml, n, O.hi, O.lo, nullptr, dbg, st, pdl),
+           "attn_combine");
+    LAUNCH(KVPRM_PROF_GEMM,
+           kvprm::launch_gemm(P.g_o, &ctx->tm_o[l], &ctx->tm_ohi, &ctx->tm_olo, ctx->part, m.d, n, np, ctx->err_d, st,
+                              pdl),
+           "gemm_o");
+    LAUNCH(KVPRM_PROF_FUSED,
+           kvprm::launch_resid_norm(m, ctx->part, P.g_o.splits, n, ctx->h, ctx->mlp_norm[l], X, nullptr, nullptr,
+                                    nullptr, st, pdl),
+           "resid_norm");
+    LAUNCH(KVPRM_PROF_GEMM,
+           kvprm::launch_gemm(P.g_gu, &ctx->tm_gu[l], &ctx->tm_xhi, &ctx->tm_xlo, ctx->part, 2 * m.ff, n, np,
+                              ctx->err_d, st, pdl),
+           "gemm_gate_up");
+    LAUNCH(KVPRM_PROF_FUSED, kvprm::launch_silu_mul(m, ctx->part, P.g_gu.splits, n, A, st, pdl), "silu_mul");
+    LAUNCH(KVPRM_PROF_GEMM,
+           kvprm::launch_gemm(P.g_down, &ctx->tm_down[l], &ctx->tm_ahi, &ctx->tm_alo, ctx->part, m.d, n, np,
+                              ctx->err_d, st, pdl),
+           "gemm_down");
+    if (l + 1 < NL) {
+      LAUNCH(KVPRM_PROF_FUSED,
+             kvprm::launch_resid_norm(m, ctx->part, P.g_down.splits, n, ctx->h, ctx->attn_norm[l + 1], X, nullptr,
+                                      nullptr, nullptr, st, pdl),
+             "resid_norm");
+    } else {
+      LAUNCH(KVPRM_PROF_FUSED,
+             kvprm::launch_resid_norm(m, ctx->part, P.g_down.splits, n, ctx->h, ctx->final_norm, X, ctx->w_plus,
+                                      ctx->w_minus, ctx->rewards_d, st, pdl),
+             "reward_head");
+    }
+    if (ctx->debug_flags & 4) {
+      const size_t nh = static_cast<size_t>(n) * m.d;
+      CK(cudaMemcpyAsync(ctx->dbg_h + l * nh, ctx->h, nh * 4, cudaMemcpyDeviceToDevice, st), "debug h");
+    }
+  }
+  return KVPRM_OK;
+}
+
+int accumulate_marks(kvprm_ctx* ctx, std::vector<ProfMark>& marks, bool destroy) {
+  for (auto& mk : marks) {
+    float ms = 0.f;
+    CK(cudaEventElapsedTime(&ms, mk.a, mk.b), "cudaEventElapsedTime");
+    ctx->prof_launches[mk.cls] += 1;
+    ctx->prof_ms[mk.cls] += ms;
+    if (destroy) {
+      cudaEventDestroy(mk.a);
+      cudaEventDestroy(mk.b);
+    }
+  }
+  if (destroy) marks.clear();
+  return KVPRM_OK;
+}
+
+void drop_graph(kvprm_ctx* ctx) {
+  if (ctx->gexec) cudaGraphExecDestroy(ctx->gexec);
+  ctx->gexec = nullptr;
+  for (auto& m : ctx->graph_marks) {
+    cudaEventDestroy(m.a);
+    cudaEventDestroy(m.b);
+  }
+  ctx->graph_marks.clear();
+  ctx->gkey = GraphKey();
+}
+
+// Score into ctx->rewards_d on stream `st` (stream-ordered).
+int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const int32_t* bt, const int32_t* sl, int32_t n,
+                 cudaStream_t st) {
+  int max_pages = 0;
+  int rc = validate_tables(ctx, n_pages, bt, sl, n, &max_pages);
+  if (rc) return rc;
+  if (n == 0) return KVPRM_OK;
+  const void* pool = kv_pages;
+  int64_t pages = n_pages;
+  if (max_pages == 0) {   // no cached token anywhere: the pool is never read
+    pool = ctx->dummy_pool;
+    pages = 1;
+  } else {
+    if (!kv_pages) return fail(ctx, KVPRM_EINVAL, "kv_pages is NULL");
+    if (!aligned16(kv_pages)) return fail(ctx, KVPRM_EINVAL, "kv_pages is not 16-byte aligned");
+  }
+  if ((rc = ensure_pool_map(ctx, pool, pages, ctx->cfg.n_layers))) return rc;
+  ctx->as.layer_rows = pages * 2 * ctx->cfg.n_kv_heads * 16;
+  const CallPlan P = make_plan(ctx, n, max_pages);
+  if ((rc = ensure_x_maps(ctx, P.n_pad))) return rc;
+  if ((rc = upload_tables(ctx, bt, sl, n, st))) return rc;
+  ctx->last_n = n;
+  ctx->last_stream = st;
+
+  if (!ctx->use_graph) {
+    Enq E{ctx, st, ctx->use_pdl && !ctx->profile, ctx->profile, &ctx->live_marks};
+    if ((rc = enqueue_forward(ctx, P, E))) return rc;
+    if (ctx->profile) {
+      CK(cudaStreamSynchronize(st), "cudaStreamSynchronize(profile)");
+      if ((rc = accumulate_marks(ctx, ctx->live_marks, true))) return rc;
+    }
+    return KVPRM_OK;
+  }
+  GraphKey key;
+  key.n = n;
+  key.n_pad = P.n_pad;
+  key.n_split = P.attn.n_split;
+  key.pps = P.attn.pages_per_split;
+  key.debug = ctx->debug_flags;
+  key.profile = ctx->profile ? 1 : 0;
+  key.pdl = ctx->use_pdl ? 1 : 0;
+  key.pool = pool;
+  key.n_pages = pages;
+  if (!(ctx->gexec && key == ctx->gkey)) {
+    drop_graph(ctx);
+    CK(cudaStreamBeginCapture(ctx->cap_stream, cudaStreamCaptureModeThreadLocal), "cudaStreamBeginCapture");
+    Enq E{ctx, ctx->cap_stream, ctx->use_pdl && !ctx->profile, ctx->profile, &ctx->graph_marks};
+    E.capturing = true;
+    rc = enqueue_forward(ctx, P, E);
+    cudaGraph_t graph = nullptr;
+    cudaError_t e = cudaStreamEndCapture(ctx->cap_stream, &graph);
+    if (rc) {
+      if (graph) cudaGraphDestroy(graph);
+      return rc;
+    }
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaStreamEndCapture");
+    e = cudaGraphInstantiate(&ctx->gexec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (e != cudaSuccess) {
+      ctx->gexec = nullptr;
+      return cuda_fail(ctx, e, "cudaGraphInstantiate");
+    }
+    ctx->gkey = key;
+  }
+  CK(cudaGraphLaunch(ctx->gexec, st), "cudaGraphLaunch");
+  if (ctx->profile) {
+    CK(cudaStreamSynchronize(st), "cudaStreamSynchronize(profile)");
+    if ((rc = accumulate_marks(ctx, ctx->graph_marks, false))) return rc;
+  }
+  return KVPRM_OK;
+}
+
+int finish_blocking(kvprm_ctx* ctx, int32_t n, float* rewards, cudaStream_t st) {
+  if (n == 0) return KVPRM_OK;
+  CK(cudaMemcpyAsync(ctx->h_rewards, ctx->rewards_d, sizeof(float) * n, cudaMemcpyDeviceToHost, st),
+     "cudaMemcpyAsync(rewards)");
+  CK(cudaMemcpyAsync(ctx->h_err, ctx->err_d, sizeof(int), cudaMemcpyDeviceToHost, st), "cudaMemcpyAsync(err)");
+  CK(cudaStreamSynchronize(st), "cudaStreamSynchronize");
+  if (*ctx->h_err) {
+    cudaMemsetAsync(ctx->err_d, 0, sizeof(int), st);
+    return fail(ctx, KVPRM_ETIMEOUT, "a bounded device wait timed out; results are invalid");
+  }
+  std::memcpy(rewards, ctx->h_rewards, sizeof(float) * n);
+  return KVPRM_OK;
+}
+
+bool env_off(const char* name) {
+  const char* v = std::getenv(name);
+  return v && v[0] == '1';
+}
+
+}  // namespace
+
+// ======================================================================== C ABI
+extern "C" {
+
+int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** out) {
+  if (!out) return KVPRM_EINVAL;
+  *out = nullptr;
+  if (!cfg || !w) return KVPRM_EINVAL;
+  const kvprm_config& c = *cfg;
+  if (c.n_layers < 1 || c.d_model < 64 || c.n_q_heads < 1 || c.n_kv_heads < 1 || c.d_ff < 64) return KVPRM_EINVAL;
+  if (c.page_size != 16) return KVPRM_EUNSUPPORTED;
+  if (c.head_dim != 64 && c.head_dim != 128) return KVPRM_EUNSUPPORTED;
+  if (c.n_q_heads % c.n_kv_heads != 0) return KVPRM_EINVAL;
+  if (c.n_q_heads / c.n_kv_heads > 16) return KVPRM_EUNSUPPORTED;
+  if (c.d_model % 64 || c.d_ff % 64 || (c.n_q_heads * c.head_dim) % 64) return KVPRM_EUNSUPPORTED;
+  if (c.max_candidates < 1 || c.max_candidates > 256) return KVPRM_ECAPACITY;
+  if (c.max_blocks_per_seq < 1) return KVPRM_EINVAL;
+  if (!(c.rms_eps >= 0.f) || !(c.rope_base > 0.f)) return KVPRM_EINVAL;
+  if (!w->embed_verify || !w->final_norm || !w->w_plus || !w->w_minus || !w->attn_norm || !w->w_qkv || !w->w_o ||
+      !w->mlp_norm || !w->w_gate_up || !w->w_down)
+    return KVPRM_EINVAL;
+  for (int l = 0; l < c.n_layers; ++l)
+    if (!w->attn_norm[l] || !w->w_qkv[l] || !w->w_o[l] || !w->mlp_norm[l] || !w->w_gate_up[l] || !w->w_down[l])
+      return KVPRM_EINVAL;
+  for (int l = 0; l < c.n_layers; ++l)
+    if (!aligned16(w->w_qkv[l]) || !aligned16(w->w_o[l]) || !aligned16(w->w_gate_up[l]) || !aligned16(w->w_down[l]))
+      return KVPRM_EINVAL;
+
+  kvprm_ctx* ctx = new (std::nothrow) kvprm_ctx();
+  if (!ctx) return KVPRM_ENOMEM;
+  ctx->cfg = c;
+  int rc = KVPRM_OK;
+#define CREATE_CK(call)             \
+  do {                              \
+    if ((rc = (call)) != KVPRM_OK) { \
+      free_ctx(ctx);                \
+      return rc;                    \
+    }                               \
+  } while (0)
+  auto cu = [&](cudaError_t e, const char* what) { return e == cudaSuccess ? KVPRM_OK : cuda_fail(ctx, e, what); };
+  CREATE_CK(cu(cudaGetDevice(&ctx->device), "cudaGetDevice"));
+  CREATE_CK(cu(cudaDeviceGetAttribute(&ctx->num_sms, cudaDevAttrMultiProcessorCount, ctx->device), "sm count"));
+  {
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    CREATE_CK(cu(cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q),
+                 "cudaGetDriverEntryPointByVersion"));
+    if (!fn || q != cudaDriverEntryPointSuccess) {
+      free_ctx(ctx);
+      return KVPRM_ECUDA;
+    }
+    ctx->encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }
+  CREATE_CK(cu(kvprm::gemm_configure(), "gemm_configure"));
+  CREATE_CK(cu(kvprm::attention_configure(), "attention_configure"));
+
+  ModelDims& m = ctx->md;
+  m.d = c.d_model;
+  m.n_q = c.n_q_heads;
+  m.n_kv = c.n_kv_heads;
+  m.hd = c.head_dim;
+  m.ff = c.d_ff;
+  m.qkv_rows = (c.n_q_heads + 2 * c.n_kv_heads) * c.head_dim;
+  m.eps = c.rms_eps;
+  AttnShape& as = ctx->as;
+  as.n_q = m.n_q;
+  as.n_kv = m.n_kv;
+  as.hd = m.hd;
+  as.group = m.n_q / m.n_kv;
+  as.max_blocks = c.max_blocks_per_seq;
+  as.layer_rows = 0;   // set per call from the pool
+
+  ctx->embed = static_cast<const bf16*>(w->embed_verify);
+  ctx->final_norm = static_cast<const bf16*>(w->final_norm);
+  ctx->w_plus = static_cast<const bf16*>(w->w_plus);
+  ctx->w_minus = static_cast<const bf16*>(w->w_minus);
+  const int NL = c.n_layers;
+  ctx->attn_norm.resize(NL);
+  ctx->mlp_norm.resize(NL);
+  ctx->tm_qkv.resize(NL);
+  ctx->tm_o.resize(NL);
+  ctx->tm_gu.resize(NL);
+  ctx->tm_down.resize(NL);
+  for (int l = 0; l < NL; ++l) {
+    ctx->attn_norm[l] = static_cast<const bf16*>(w->attn_norm[l]);
+    ctx->mlp_norm[l] = static_cast<const bf16*>(w->mlp_norm[l]);
+    CREATE_CK(make_map(ctx, &ctx->tm_qkv[l], w->w_qkv[l], m.d, m.qkv_rows, 64, 128, "w_qkv"));
+    CREATE_CK(make_map(ctx, &ctx->tm_o[l], w->w_o[l], static_cast<uint64_t>(m.n_q) * m.hd, m.d, 64, 128, "w_o"));
+    CREATE_CK(make_map(ctx, &ctx->tm_gu[l], w->w_gate_up[l], m.d, 2 * static_cast<uint64_t>(m.ff), 64, 128,
+                       "w_gate_up"));
+    CREATE_CK(make_map(ctx, &ctx->tm_down[l], w->w_down[l], m.ff, m.d, 64, 128, "w_down"));
+  }
+
+  const int Bmax = c.max_candidates;
+  ctx->npad_max = (Bmax + 15) / 16 * 16;
+  const size_t Bp = ctx->npad_max;
+  CREATE_CK(dalloc(ctx, &ctx->h, static_cast<size_t>(Bmax) * m.d, "h"));
+  CREATE_CK(dalloc(ctx, &ctx->xhi, Bp * m.d, "x_hi"));
+  CREATE_CK(dalloc(ctx, &ctx->xlo, Bp * m.d, "x_lo"));
+  CREATE_CK(dalloc(ctx, &ctx->ohi, Bp * m.n_q * m.hd, "o_hi"));
+  CREATE_CK(dalloc(ctx, &ctx->olo, Bp * m.n_q * m.hd, "o_lo"));
+  CREATE_CK(dalloc(ctx, &ctx->ahi, Bp * m.ff, "a_hi"));
+  CREATE_CK(dalloc(ctx, &ctx->alo, Bp * m.ff, "a_lo"));
+  {
+    // split-K partials: splits * n * M, with splits <= max(1, 2*SMs / m_tiles) per GEMM
+    size_t need = 0;
+    const int shapes[4][2] = {{m.qkv_rows, m.d}, {m.d, m.n_q * m.hd}, {2 * m.ff, m.d}, {m.d, m.ff}};
+    for (int npad = 16; npad <= ctx->npad_max; npad += 16)
+      for (auto& s : shapes) {
+        GemmPlan g = kvprm::plan_gemm(s[0], s[1], npad, ctx->num_sms, true);
+        size_t e = static_cast<size_t>(g.splits) * Bmax * s[0];
+        if (e > need) need = e;
+      }
+    ctx->part_elems = need;
+    CREATE_CK(dalloc(ctx, &ctx->part, need, "gemm partials"));
+  }
+  CREATE_CK(dalloc(ctx, &ctx->q, static_cast<size_t>(Bmax) * m.n_q * m.hd, "q"));
+  CREATE_CK(dalloc(ctx, &ctx->qhi, static_cast<size_t>(Bmax) * m.n_q * m.hd, "q_hi"));
+  CREATE_CK(dalloc(ctx, &ctx->qlo, static_cast<size_t>(Bmax) * m.n_q * m.hd, "q_lo"));
+  CREATE_CK(dalloc(ctx, &ctx->kself, static_cast<size_t>(Bmax) * m.n_kv * m.hd, "k_self"));
+  CREATE_CK(dalloc(ctx, &ctx->vself, static_cast<size_t>(Bmax) * m.n_kv * m.hd, "v_self"));
+  CREATE_CK(dalloc(ctx, &ctx->apart_o, static_cast<size_t>(Bmax) * m.n_q * kSplitCap * m.hd, "attn partials"));
+  CREATE_CK(dalloc(ctx, &ctx->apart_ml, static_cast<size_t>(Bmax) * m.n_q * kSplitCap * 2, "attn stats"));
+  CREATE_CK(dalloc(ctx, &ctx->rope, static_cast<size_t>(Bmax) * (m.hd / 2), "rope table"));
+  CREATE_CK(dalloc(ctx, &ctx->tables_d, static_cast<size_t>(Bmax) * (1 + c.max_blocks_per_seq), "tables"));
+  CREATE_CK(dalloc(ctx, &ctx->rewards_d, static_cast<size_t>(Bmax), "rewards"));
+  CREATE_CK(dalloc(ctx, &ctx->err_d, 1, "err"));
+  CREATE_CK(dalloc(ctx, &ctx->dummy_pool, static_cast<size_t>(NL) * 2 * m.n_kv * 16 * m.hd, "dummy pool"));
+  {
+    cudaError_t e =
+        cudaMallocHost(reinterpret_cast<void**>(&ctx->staging), sizeof(int32_t) * Bmax * (1 + c.max_blocks_per_seq));
+    if (e == cudaSuccess) e = cudaMallocHost(reinterpret_cast<void**>(&ctx->h_rewards), sizeof(float) * Bmax);
+    if (e == cudaSuccess) e = cudaMallocHost(reinterpret_cast<void**>(&ctx->h_err), sizeof(int));
+    if (e != cudaSuccess) {
+      cudaGetLastError();
+      free_ctx(ctx);
+      return KVPRM_ENOMEM;
+    }
+  }
+  CREATE_CK(cu(cudaEventCreateWithFlags(&ctx->staging_ev, cudaEventDisableTiming), "cudaEventCreate"));
+  CREATE_CK(cu(cudaStreamCreateWithFlags(&ctx->cap_stream, cudaStreamNonBlocking), "cudaStreamCreate"));
+  ctx->use_graph = !env_off("KVPRM_NO_GRAPH");
+  ctx->use_pdl = !env_off("KVPRM_NO_PDL");
+  CREATE_CK(cu(cudaDeviceSynchronize(), "cudaDeviceSynchronize(create)"));
+#undef CREATE_CK
+  *out = ctx;
+  return KVPRM_OK;
+}
+
+void kvprm_destroy(kvprm_ctx* ctx) {
+  if (!ctx) return;
+  cudaDeviceSynchronize();
+  free_ctx(ctx);
+}
+
+const char* kvprm_last_error(const kvprm_ctx* ctx) { return ctx ? ctx->last_error.c_str() : ""; }
+
+int kvprm_score_async(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const int32_t* block_table,
+                      const int32_t* seq_lens, int32_t n, float* d_rewards, void* stream) {
+  if (!ctx) return KVPRM_EINVAL;
+  if (n > 0 && !d_rewards) return fail(ctx, KVPRM_EINVAL, "d_rewards is NULL");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int rc = score_device(ctx, kv_pages, n_pages, block_table, seq_lens, n, st);
+  if (rc || n == 0) return rc;
+  CK(cudaMemcpyAsync(d_rewards, ctx->rewards_d, sizeof(float) * n, cudaMemcpyDeviceToDevice, st),
+     "cudaMemcpyAsync(d_rewards)");
+  return KVPRM_OK;
+}
+
+int kvprm_score(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const int32_t* block_table,
+                const int32_t* seq_lens, int32_t n, float* rewards, void* stream) {
+  if (!ctx) return KVPRM_EINVAL;
+  if (n > 0 && !rewards) return fail(ctx, KVPRM_EINVAL, "rewards is NULL");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int rc = score_device(ctx, kv_pages, n_pages, block_table, seq_lens, n, st);
+  if (rc) return rc;
+  return finish_blocking(ctx, n, rewards, st);
+}
+
+int kvprm_score_host(kvprm_ctx* ctx, const void* h_kv_pages, int64_t n_pages, const int32_t* block_table,
+                     const int32_t* seq_lens, int32_t n, float* rewards, void* stream) {
+  if (!ctx) return KVPRM_EINVAL;
+  if (n > 0 && !rewards) return fail(ctx, KVPRM_EINVAL, "rewards is NULL");
+  if (n_pages < 0) return fail(ctx, KVPRM_EINVAL, "n_pages is negative");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t bytes = static_cast<size_t>(ctx->cfg.n_layers) * n_pages * 2 * ctx->cfg.n_kv_heads * 16 *
+                       ctx->cfg.head_dim * sizeof(bf16);
+  const void* pool = nullptr;
+  if (bytes > 0) {
+    if (!h_kv_pages) return fail(ctx, KVPRM_EINVAL, "h_kv_pages is NULL");
+    if (bytes > ctx->dev_pool_bytes) {
+      CK(cudaStreamSynchronize(st), "cudaStreamSynchronize(pool grow)");
+      cudaFree(ctx->dev_pool);
+      ctx->dev_pool = nullptr;
+      ctx->dev_pool_bytes = 0;
+      drop_graph(ctx);
+      ctx->pool_ptr = nullptr;
+      cudaError_t e = cudaMalloc(&ctx->dev_pool, bytes);
+      if (e != cudaSuccess) {
+        cudaGetLastError();
+        return fail(ctx, KVPRM_ENOMEM, "cudaMalloc(device pool, %zu bytes) failed", bytes);
+      }
+      ctx->dev_pool_bytes = bytes;
+    }
+    CK(cudaMemcpyAsync(ctx->dev_pool, h_kv_pages, bytes, cudaMemcpyHostToDevice, st), "cudaMemcpyAsync(pool)");
+    pool = ctx->dev_pool;
+  }
+  int rc = score_device(ctx, pool, n_pages, block_table, seq_lens, n, st);
+  if (rc) return rc;
+  return finish_blocking(ctx, n, rewards, st);
+}
+
+int kvprm_attention(kvprm_ctx* ctx, const void* kv_layer, int64_t n_pages, const int32_t* block_table,
+                    const int32_t* seq_lens, int32_t n, const void* q, const void* k_self, const void* v_self,
+                    float* out, void* stream) {
+  if (!ctx) return KVPRM_EINVAL;
+  int max_pages = 0;
+  int rc = validate_tables(ctx, n_pages, block_table, seq_lens, n, &max_pages);
+  if (rc) return rc;
+  if (n == 0) return KVPRM_OK;
+  if (!q || !k_self || !v_self || !out) return fail(ctx, KVPRM_EINVAL, "q, k_self, v_self and out must be non-NULL");
+  if (!aligned16(q) || !aligned16(k_self) || !aligned16(v_self))
+    return fail(ctx, KVPRM_EINVAL, "q, k_self and v_self must be 16-byte aligned");
+  const kvprm::HiLo Q{ctx->qhi, ctx->qlo};
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const void* pool = kv_layer;
+  int64_t pages = n_pages;
+  if (max_pages == 0) {
+    pool = ctx->dummy_pool;
+    pages = 1;
+  } else {
+    if (!kv_layer) return fail(ctx, KVPRM_EINVAL, "kv_layer is NULL");
+    if (!aligned16(kv_layer)) return fail(ctx, KVPRM_EINVAL, "kv_layer is not 16-byte aligned");
+  }
+  if ((rc = ensure_pool_map(ctx, pool, pages, 1))) return rc;
+  if ((rc = upload_tables(ctx, block_table, seq_lens, n, st))) return rc;
+  AttnShape as = ctx->as;
+  as.layer_rows = pages * 2 * ctx->cfg.n_kv_heads * 16;
+  const AttnPlan P = kvprm::plan_attention(as, n, max_pages, ctx->num_sms, kSplitCap);
+  const int32_t* sl = ctx->tables_d;
+  const int32_t* bt = ctx->tables_d + ctx->cfg.max_candidates;
+  Enq E{ctx, st, false, ctx->profile, &ctx->live_marks};
+  LAUNCH(KVPRM_PROF_FUSED,
+         kvprm::launch_split_hilo(static_cast<const float*>(q), static_cast<int64_t>(n) * ctx->md.n_q * ctx->md.hd, Q,
+                                  st),
+         "split_hilo");
+  LAUNCH(KVPRM_PROF_ATTN,
+         kvprm::launch_attn_split(as, P, &ctx->tm_pool, 0, bt, sl, Q.hi, Q.lo, n, ctx->apart_o, ctx->apart_ml,
+                                  ctx->err_d, st, false),
+         "attn_split");
+  LAUNCH(KVPRM_PROF_COMBINE,
+         kvprm::launch_attn_combine(as, P, sl, static_cast<const float*>(q), static_cast<const float*>(k_self),
+                                    static_cast<const float*>(v_self), ctx->apart_o, ctx->apart_ml, n, ctx->ohi,
+                                    ctx->olo, out, nullptr, st, false),
+         "attn_combine");
+  ctx->last_n = n;
+  ctx->last_stream = st;
+  if (ctx->profile) {
+    CK(cudaStreamSynchronize(st), "cudaStreamSynchronize(profile)");
+    if ((rc = accumulate_marks(ctx, ctx->live_marks, true))) return rc;
+  }
+  // the next full score call must rebuild its pool map (this call pointed it at one layer)
+  ctx->pool_ptr = nullptr;
+  drop_graph(ctx);
+  return KVPRM_OK;
+}
+
+int kvprm_projection(kvprm_ctx* ctx, const void* W, int32_t M, int32_t K, const void* X, int32_t n, float* Y,
+                     void* stream) {
+  if (!ctx) return KVPRM_EINVAL;
+  if (!W || !X || !Y) return fail(ctx, KVPRM_EINVAL, "W, X and Y must be non-NULL");
+  if (M < 1 || K < 8 || K % 8) return fail(ctx, KVPRM_EINVAL, "bad projection shape M=%d K=%d", M, K);
+  if (n < 1 || n > ctx->cfg.max_candidates)
+    return fail(ctx, KVPRM_ECAPACITY, "n = %d outside [1, max_candidates = %d]", n, ctx->cfg.max_candidates);
+  if (!aligned16(W) || !aligned16(X)) return fail(ctx, KVPRM_EINVAL, "W and X must be 16-byte aligned");
+  const int n_pad = (n + 15) / 16 * 16;
+  const GemmPlan g = kvprm::plan_gemm(M, K, n_pad, ctx->num_sms, false);
+  if (static_cast<size_t>(g.splits) * n * M > ctx->part_elems)
+    return fail(ctx, KVPRM_ECAPACITY, "projection %dx%d for %d candidates exceeds the partial buffer", M, K, n);
+  CUtensorMap tw, tx;
+  int rc;
+  if ((rc = make_map(ctx, &tw, W, K, M, 64, 128, "W"))) return rc;
+  if ((rc = make_map(ctx, &tx, X, K, n, 64, n_pad, "X"))) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  Enq E{ctx, st, false, ctx->profile, &ctx->live_marks};
+  LAUNCH(KVPRM_PROF_GEMM, kvprm::launch_gemm(g, &tw, &tx, nullptr, ctx->part, M, n, n_pad, ctx->err_d, st, false),
+         "gemm");
+  LAUNCH(KVPRM_PROF_FUSED, kvprm::launch_split_sum(ctx->part, g.splits, static_cast<int64_t>(n) * M, Y, st),
+         "split_sum");
+  ctx->last_stream = st;
+  if (ctx->profile) {
+    CK(cudaStreamSynchronize(st), "cudaStreamSynchronize(profile)");
+    if ((rc = accumulate_marks(ctx, ctx->live_marks, true))) return rc;
+  }
+  return KVPRM_OK;
+}
+
+int kvprm_debug_hidden(kvprm_ctx* ctx, float* d_out) {
+  if (!ctx || !d_out) return KVPRM_EINVAL;
+  CK(cudaMemcpyAsync(d_out, ctx->h, sizeof(float) * ctx->last_n * ctx->md.d, cudaMemcpyDeviceToDevice,
+                     ctx->last_stream),
+     "cudaMemcpyAsync(hidden)");
+  return KVPRM_OK;
+}
+
+int kvprm_set_debug(kvprm_ctx* ctx, int flags) {
+  if (!ctx) return KVPRM_EINVAL;
+  if ((flags & 1) && !ctx->dbg) {
+    const size_t count = static_cast<size_t>(ctx->cfg.n_layers) * ctx->cfg.max_candidates * ctx->md.n_q * ctx->md.hd;
+    int rc = dalloc(ctx, &ctx->dbg, count, "debug capture");
+    if (rc) return rc;
+  }
+  const size_t NB = static_cast<size_t>(ctx->cfg.n_layers) * ctx->cfg.max_candidates;
+  if ((flags & 2) && !ctx->dbg_q) {
+    int rc = dalloc(ctx, &ctx->dbg_q, NB * ctx->md.n_q * ctx->md.hd, "debug q");
+    if (!rc) rc = dalloc(ctx, &ctx->dbg_k, NB * ctx->md.n_kv * ctx->md.hd, "debug k");
+    if (!rc) rc = dalloc(ctx, &ctx->dbg_v, NB * ctx->md.n_kv * ctx->md.hd, "debug v");
+    if (rc) return rc;
+  }
+  if ((flags & 4) && !ctx->dbg_h) {
+    int rc = dalloc(ctx, &ctx->dbg_h, NB * ctx->md.d, "debug h");
+    if (rc) return rc;
+  }
+  ctx->debug_flags = flags;
+  return KVPRM_OK;
+}
+
+int kvprm_debug_layers(kvprm_ctx* ctx, int which, void* d_out) {
+  if (!ctx || !d_out) return KVPRM_EINVAL;
+  const size_t L = static_cast<size_t>(ctx->cfg.n_layers) * ctx->last_n;
+  const void* src = nullptr;
+  size_t bytes = 0;
+  if (which >= 1 && which <= 3) {
+    if (!(ctx->debug_flags & 2)) return fail(ctx, KVPRM_EINVAL, "q/k/v capture (flag 2) is not enabled");
+    src = which == 1 ? ctx->dbg_q : (which == 2 ? ctx->dbg_k : ctx->dbg_v);
+    bytes = L * (which == 1 ? ctx->md.n_q : ctx->md.n_kv) * ctx->md.hd * 4;
+  } else if (which == 4) {
+    if (!(ctx->debug_flags & 4)) return fail(ctx, KVPRM_EINVAL, "hidden-state capture (flag 4) is not enabled");
+    src = ctx->dbg_h;
+    bytes = L * ctx->md.d * 4;
+  } else {
+    return fail(ctx, KVPRM_EINVAL, "unknown capture %d", which);
+  }
+  CK(cudaMemcpyAsync(d_out, src, bytes, cudaMemcpyDeviceToDevice, ctx->last_stream), "cudaMemcpyAsync(debug)");
+  return KVPRM_OK;
+}
+
+int kvprm_debug_attn_out(kvprm_ctx* ctx, float* d_out) {
+  if (!ctx || !d_out) return KVPRM_EINVAL;
+  if (!(ctx->debug_flags & 1) || !ctx->dbg) return fail(ctx, KVPRM_EINVAL, "debug capture is not enabled");
+  const size_t count = static_cast<size_t>(ctx->cfg.n_layers) * ctx->last_n * ctx->md.n_q * ctx->md.hd;
+  CK(cudaMemcpyAsync(d_out, ctx->dbg, count * sizeof(float), cudaMemcpyDeviceToDevice, ctx->last_stream),
+     "cudaMemcpyAsync(debug)");
+  return KVPRM_OK;
+}
+
+int kvprm_resolve(kvprm_ctx* ctx, int32_t b, int64_t* phys_row) {
+  if (!ctx || !phys_row) return KVPRM_EINVAL;
+  if (b < 0 || b >= ctx->last_n) return fail(ctx, KVPRM_EINVAL, "candidate %d not in the last call", b);
+  cudaStream_t st = ctx->last_stream;
+  int32_t L = 0;
+  CK(cudaMemcpyAsync(&L, ctx->tables_d + b, sizeof(int32_t), cudaMemcpyDeviceToHost, st), "cudaMemcpy(len)");
+  CK(cudaStreamSynchronize(st), "cudaStreamSynchronize");
+  if (L == 0) return KVPRM_OK;
+  int64_t* d = nullptr;
+  CK(cudaMalloc(&d, sizeof(int64_t) * L), "cudaMalloc(resolve)");
+  cudaError_t e = kvprm::launch_resolve(ctx->tables_d + ctx->cfg.max_candidates, ctx->tables_d,
+                                        ctx->cfg.max_blocks_per_seq, b, d, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(phys_row, d, sizeof(int64_t) * L, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  cudaFree(d);
+  if (e != cudaSuccess) return cuda_fail(ctx, e, "resolve");
+  return KVPRM_OK;
+}
+
+int kvprm_check_device(kvprm_ctx* ctx) {
+  if (!ctx) return KVPRM_EINVAL;
+  CK(cudaStreamSynchronize(ctx->last_stream), "cudaStreamSynchronize");
+  CK(cudaMemcpy(ctx->h_err, ctx->err_d, sizeof(int), cudaMemcpyDeviceToHost), "cudaMemcpy(err)");
+  if (*ctx->h_err) {
+    CK(cudaMemset(ctx->err_d, 0, sizeof(int)), "cudaMemset(err)");
+    return fail(ctx, KVPRM_ETIMEOUT, "a bounded device wait timed out");
+  }
+  return KVPRM_OK;
+}
+
+int kvprm_set_profile(kvprm_ctx* ctx, int enable) {
+  if (!ctx) return KVPRM_EINVAL;
+  if (enable && !ctx->profile) {
+    for (int i = 0; i < KVPRM_PROF_N; ++i) {
+      ctx->prof_launches[i] = 0;
+      ctx->prof_ms[i] = 0.0;
+    }
+  }
+  ctx->profile = enable != 0;
+  return KVPRM_OK;
+}
+
+int kvprm_get_profile(kvprm_ctx* ctx, int64_t* launches, double* total_ms) {
+  if (!ctx || !launches || !total_ms) return KVPRM_EINVAL;
+  for (int i = 0; i < KVPRM_PROF_N; ++i) {
+    launches[i] = ctx->prof_launches[i];
+    total_ms[i] = ctx->prof_ms[i];
+  }
+  return KVPRM_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,228 @@
+"""ctypes binding of the scoring library's C ABI (include/kvprm.h).
+
+Names mirror the C entry points; this module only marshals arguments (device
+pointers from torch tensors, host arrays from numpy) and turns non-zero status
+codes into exceptions.  Every step of the scoring path runs in the CUDA
+library; there is no Python or CPU fallback: if the library cannot be built or
+loaded, importing it raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+from . import build as _build
+
+KVPRM_OK, KVPRM_EINVAL, KVPRM_ECAPACITY, KVPRM_EINDEX, KVPRM_ECUDA, KVPRM_ENOMEM, KVPRM_ETIMEOUT, \
+    KVPRM_EUNSUPPORTED = range(8)
+PROF_GEMM, PROF_ATTN, PROF_COMBINE, PROF_FUSED = range(4)
+PROF_NAMES = ("gemm", "attention", "combine", "fused")
+
+
+class KvprmError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"kvprm error {code}: {msg}")
+        self.code = code
+
+
+class KvprmConfig(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int32), ("d_model", ctypes.c_int32), ("n_q_heads", ctypes.c_int32),
+                ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32), ("d_ff", ctypes.c_int32),
+                ("page_size", ctypes.c_int32), ("rope_base", ctypes.c_float), ("rms_eps", ctypes.c_float),
+                ("max_candidates", ctypes.c_int32), ("max_blocks_per_seq", ctypes.c_int32)]
+
+
+_VPP = ctypes.POINTER(ctypes.c_void_p)
+
+
+class KvprmWeights(ctypes.Structure):
+    _fields_ = [("embed_verify", ctypes.c_void_p), ("final_norm", ctypes.c_void_p), ("w_plus", ctypes.c_void_p),
+                ("w_minus", ctypes.c_void_p), ("attn_norm", _VPP), ("w_qkv", _VPP), ("w_o", _VPP),
+                ("mlp_norm", _VPP), ("w_gate_up", _VPP), ("w_down", _VPP)]
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """Load (building first if the sources changed) the in-tree libkvprm.so."""
+    global _lib
+    if _lib is None:
+        path = _build.build()
+        L = ctypes.CDLL(path)
+        vp, i32, i64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64
+        i32p, i64p, f32p = ctypes.POINTER(ctypes.c_int32), ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_float)
+        L.kvprm_create.argtypes = [ctypes.POINTER(KvprmConfig), ctypes.POINTER(KvprmWeights), ctypes.POINTER(vp)]
+        L.kvprm_destroy.argtypes = [vp]
+        L.kvprm_destroy.restype = None
+        L.kvprm_last_error.argtypes = [vp]
+        L.kvprm_last_error.restype = ctypes.c_char_p
+        L.kvprm_score.argtypes = [vp, vp, i64, i32p, i32p, i32, f32p, vp]
+        L.kvprm_score_async.argtypes = [vp, vp, i64, i32p, i32p, i32, vp, vp]
+        L.kvprm_score_host.argtypes = [vp, vp, i64, i32p, i32p, i32, f32p, vp]
+        L.kvprm_attention.argtypes = [vp, vp, i64, i32p, i32p, i32, vp, vp, vp, vp, vp]
+        L.kvprm_projection.argtypes = [vp, vp, i32, i32, vp, i32, vp, vp]
+        L.kvprm_debug_hidden.argtypes = [vp, vp]
+        L.kvprm_set_debug.argtypes = [vp, ctypes.c_int]
+        L.kvprm_debug_attn_out.argtypes = [vp, vp]
+        L.kvprm_debug_layers.argtypes = [vp, ctypes.c_int, vp]
+        L.kvprm_resolve.argtypes = [vp, i32, i64p]
+        L.kvprm_check_device.argtypes = [vp]
+        L.kvprm_set_profile.argtypes = [vp, ctypes.c_int]
+        L.kvprm_get_profile.argtypes = [vp, i64p, ctypes.POINTER(ctypes.c_double)]
+        _lib = L
+    return _lib
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def _check(ctx, rc: int) -> None:
+    if rc != KVPRM_OK:
+        msg = lib().kvprm_last_error(ctx).decode() if ctx else ""
+        raise KvprmError(rc, msg)
+
+
+def _i32(a) -> np.ndarray:
+    return np.ascontiguousarray(a, dtype=np.int32)
+
+
+def _p(a: np.ndarray, t):
+    return a.ctypes.data_as(ctypes.POINTER(t))
+
+
+# ------------------------------------------------------------------ same-name wrappers
+def kvprm_create(config: KvprmConfig, weights: KvprmWeights) -> ctypes.c_void_p:
+    ctx = ctypes.c_void_p()
+    rc = lib().kvprm_create(ctypes.byref(config), ctypes.byref(weights), ctypes.byref(ctx))
+    if rc != KVPRM_OK:
+        raise KvprmError(rc, "kvprm_create failed")
+    return ctx
+
+
+def kvprm_destroy(ctx) -> None:
+    lib().kvprm_destroy(ctx)
+
+
+def kvprm_score(ctx, kv_pages_ptr: int, n_pages: int, block_table, seq_lens, n: int, stream_ptr: int = 0) -> np.ndarray:
+    bt, sl = _i32(block_table), _i32(seq_lens)
+    out = np.zeros(n, np.float32)
+    _check(ctx, lib().kvprm_score(ctx, kv_pages_ptr, n_pages, _p(bt, ctypes.c_int32), _p(sl, ctypes.c_int32), n,
+                                  _p(out, ctypes.c_float), stream_ptr))
+    return out
+
+
+def kvprm_score_async(ctx, kv_pages_ptr: int, n_pages: int, block_table, seq_lens, n: int, d_rewards_ptr: int,
+                      stream_ptr: int = 0) -> None:
+    bt, sl = _i32(block_table), _i32(seq_lens)
+    _check(ctx, lib().kvprm_score_async(ctx, kv_pages_ptr, n_pages, _p(bt, ctypes.c_int32), _p(sl, ctypes.c_int32),
+                                        n, d_rewards_ptr, stream_ptr))
+
+
+def kvprm_score_host(ctx, h_kv_pages_ptr: int, n_pages: int, block_table, seq_lens, n: int, stream_ptr: int = 0,
+                     out: np.ndarray | None = None) -> np.ndarray:
+    bt, sl = _i32(block_table), _i32(seq_lens)
+    if out is None:
+        out = np.zeros(n, np.float32)
+    _check(ctx, lib().kvprm_score_host(ctx, h_kv_pages_ptr, n_pages, _p(bt, ctypes.c_int32), _p(sl, ctypes.c_int32),
+                                       n, _p(out, ctypes.c_float), stream_ptr))
+    return out
+
+
+def kvprm_attention(ctx, kv_layer_ptr: int, n_pages: int, block_table, seq_lens, n: int, q_ptr: int, k_self_ptr: int,
+                    v_self_ptr: int, out_ptr: int, stream_ptr: int = 0) -> None:
+    bt, sl = _i32(block_table), _i32(seq_lens)
+    _check(ctx, lib().kvprm_attention(ctx, kv_layer_ptr, n_pages, _p(bt, ctypes.c_int32), _p(sl, ctypes.c_int32), n,
+                                      q_ptr, k_self_ptr, v_self_ptr, out_ptr, stream_ptr))
+
+
+def kvprm_projection(ctx, W_ptr: int, M: int, K: int, X_ptr: int, n: int, Y_ptr: int, stream_ptr: int = 0) -> None:
+    _check(ctx, lib().kvprm_projection(ctx, W_ptr, M, K, X_ptr, n, Y_ptr, stream_ptr))
+
+
+def kvprm_debug_hidden(ctx, d_out_ptr: int) -> None:
+    _check(ctx, lib().kvprm_debug_hidden(ctx, d_out_ptr))
+
+
+def kvprm_set_debug(ctx, flags: int) -> None:
+    _check(ctx, lib().kvprm_set_debug(ctx, flags))
+
+
+def kvprm_debug_attn_out(ctx, d_out_ptr: int) -> None:
+    _check(ctx, lib().kvprm_debug_attn_out(ctx, d_out_ptr))
+
+
+def kvprm_debug_layers(ctx, which: int, d_out_ptr: int) -> None:
+    _check(ctx, lib().kvprm_debug_layers(ctx, which, d_out_ptr))
+
+
+def kvprm_resolve(ctx, b: int, length: int) -> np.ndarray:
+    out = np.zeros(max(length, 1), np.int64)
+    _check(ctx, lib().kvprm_resolve(ctx, b, _p(out, ctypes.c_int64)))
+    return out[:length]
+
+
+def kvprm_check_device(ctx) -> None:
+    _check(ctx, lib().kvprm_check_device(ctx))
+
+
+def kvprm_set_profile(ctx, enable: bool) -> None:
+    _check(ctx, lib().kvprm_set_profile(ctx, int(enable)))
+
+
+def kvprm_get_profile(ctx) -> dict:
+    n = np.zeros(4, np.int64)
+    ms = np.zeros(4, np.float64)
+    _check(ctx, lib().kvprm_get_profile(ctx, _p(n, ctypes.c_int64), ms.ctypes.data_as(ctypes.POINTER(ctypes.c_double))))
+    return {PROF_NAMES[i]: (int(n[i]), float(ms[i])) for i in range(4)}
+
+
+# ------------------------------------------------------------------ torch convenience
+class Scorer:
+    """Owns a context for a scorer whose weights are torch bf16 CUDA tensors.
+
+    weights = {'embed_verify', 'final_norm', 'w_plus', 'w_minus'} -> tensor, and
+    'layers' -> list of {'attn_norm', 'w_qkv', 'w_o', 'mlp_norm', 'w_gate_up', 'w_down'}."""
+
+    def __init__(self, n_layers, d_model, n_q_heads, n_kv_heads, head_dim, d_ff, weights: dict, max_candidates: int,
+                 max_blocks_per_seq: int, rope_base: float = 1e4, rms_eps: float = 1e-6):
+        self.cfg = KvprmConfig(n_layers, d_model, n_q_heads, n_kv_heads, head_dim, d_ff, 16, rope_base, rms_eps,
+                               max_candidates, max_blocks_per_seq)
+        arr = ctypes.c_void_p * n_layers
+        lay = weights["layers"]
+        self._arrays = {k: arr(*[lay[l][k].data_ptr() for l in range(n_layers)])
+                        for k in ("attn_norm", "w_qkv", "w_o", "mlp_norm", "w_gate_up", "w_down")}
+        self._weights = weights   # keep the tensors alive
+        cast = lambda a: ctypes.cast(a, _VPP)  # noqa: E731
+        self.w = KvprmWeights(weights["embed_verify"].data_ptr(), weights["final_norm"].data_ptr(),
+                              weights["w_plus"].data_ptr(), weights["w_minus"].data_ptr(),
+                              cast(self._arrays["attn_norm"]), cast(self._arrays["w_qkv"]), cast(self._arrays["w_o"]),
+                              cast(self._arrays["mlp_norm"]), cast(self._arrays["w_gate_up"]),
+                              cast(self._arrays["w_down"]))
+        self.ctx = kvprm_create(self.cfg, self.w)
+
+    def close(self):
+        if self.ctx:
+            kvprm_destroy(self.ctx)
+            self.ctx = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def score(self, kv_pages, block_table, seq_lens, stream=None) -> np.ndarray:
+        import torch
+        st = (stream or torch.cuda.current_stream()).cuda_stream
+        n_pages = kv_pages.shape[1]
+        return kvprm_score(self.ctx, kv_pages.data_ptr(), n_pages, block_table, seq_lens, len(seq_lens), st)
+
+    def score_async(self, kv_pages, block_table, seq_lens, d_rewards, stream=None) -> None:
+        import torch
+        st = (stream or torch.cuda.current_stream()).cuda_stream
+        kvprm_score_async(self.ctx, kv_pages.data_ptr(), kv_pages.shape[1], block_table, seq_lens, len(seq_lens),
+                          d_rewards.data_ptr(), st)

@@ -1,0 +1,158 @@
+"""GPU parity: the C-ABI CUDA scoring path against the CPU oracle (exact mode:
+bf16 weights and cache, exact activations) on seeded inputs -- P(+) within 1e-3
+absolute; every layer's attention output within 2e-3 relative inf-norm, full
+chain, not teacher-forced -- plus edge cases, indexing and error handling."""
+import numpy as np
+import pytest
+
+import kvsynth as ks
+import oracle
+from tests.gpu_util import ATTN_RTOL, compare, make_scorer, require_gpu, run_gpu
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("gain_std", [0.0, 0.2])
+def test_tiny_workload(gain_std):
+    t = ks.Tables.make(gain_std)
+    w = ks.make_workload("tiny", gain_std=gain_std)
+    r, attn, _, _ = run_gpu(w, t)
+    compare(w, t, gpu_rewards=r, gpu_attn=attn, label=f"tiny g{gain_std}")
+
+
+def test_ragged_and_page_edges():
+    t = ks.Tables.make(0.2)
+    w = ks.distinct("ragged", ks.ARCH_TINY, 21, [0, 1, 15, 16, 17, 31, 33, 100, 257, 1000], gain_std=0.2)
+    r, attn, _, _ = run_gpu(w, t)
+    compare(w, t, gpu_rewards=r, gpu_attn=attn, label="ragged")
+
+
+def test_all_empty_caches():
+    t = ks.Tables.make(0.2)
+    w = ks.distinct("empty", ks.ARCH_TINY, 22, [0, 0, 0], gain_std=0.2)
+    r, attn, _, _ = run_gpu(w, t)
+    compare(w, t, gpu_rewards=r, gpu_attn=attn, label="empty")
+
+
+def test_shared_pages_tree():
+    t = ks.Tables.make(0.2)
+    w = ks.mcts_tree("tree", ks.ARCH_TINY, 23, branching=3, depth=3, lo=5, hi=70, gain_std=0.2)
+    r, attn, _, _ = run_gpu(w, t)
+    compare(w, t, gpu_rewards=r, gpu_attn=attn, label="tree")
+
+
+@pytest.mark.parametrize("B", [1, 17, 40])
+def test_batch_padding(B):
+    t = ks.Tables.make(0.2)
+    lens = [(37 * b) % 300 for b in range(B)]
+    w = ks.distinct("batch", ks.ARCH_TINY, 24 + B, lens, gain_std=0.2)
+    r, attn, _, _ = run_gpu(w, t)
+    compare(w, t, gpu_rewards=r, gpu_attn=attn, label=f"B={B}")
+
+
+@pytest.mark.parametrize("arch,lens", [
+    (ks.Arch(2, 1536, 12, 2, 128, 8960), [2048] * 16),                   # 1.5B layer shapes, G = 6
+    (ks.Arch(2, 3584, 28, 4, 128, 18944), [1, 300, 4096, 777, 64, 2000]),  # 7B layer shapes, G = 7
+    (ks.Arch(2, 4096, 32, 8, 128, 14336), [5000, 4096, 1]),               # 8B layer shapes, G = 4
+    (ks.Arch(2, 512, 16, 1, 64, 512), [0, 50, 129]),                      # G = 16 (two MMA row groups)
+])
+def test_layer_shapes(arch, lens):
+    t = ks.Tables.make(0.2)
+    w = ks.distinct("shapes", arch, 31, lens, gain_std=0.2)
+    r, attn, _, _ = run_gpu(w, t)
+    compare(w, t, gpu_rewards=r, gpu_attn=attn, label=f"arch {arch.d_model}/{arch.n_q_heads}/{arch.n_kv_heads}")
+
+
+def test_attention_teacher_forced():
+    """kvprm_attention on given fp32 q / self k / self v against the oracle's read-out."""
+    torch = require_gpu()
+    import paper_2607_09153_gb300 as kp
+    arch = ks.Arch(1, 512, 12, 2, 128, 512)
+    t = ks.Tables.make()
+    w = ks.distinct("attn", arch, 41, [0, 1, 16, 17, 250, 2049, 4096])
+    dev = ks.DeviceInputs(w, t)
+    sc = make_scorer(dev, w.n_candidates, w.max_blocks)
+    rng = np.random.default_rng(5)
+    B, nq, nkv, hd = w.n_candidates, arch.n_q_heads, arch.n_kv_heads, arch.head_dim
+    qf = rng.normal(0, 0.8, (B, nq, hd)).astype(np.float32)
+    kf = rng.normal(0, 1, (B, nkv, hd)).astype(np.float32)
+    vf = rng.normal(0, 1, (B, nkv, hd)).astype(np.float32)
+    q, k, v = (torch.from_numpy(a).cuda() for a in (qf, kf, vf))
+    out = torch.empty((B, nq, hd), dtype=torch.float32, device="cuda")
+    kp.kvprm_attention(sc.ctx, dev.pool[0].data_ptr(), dev.n_pages, w.block_table, w.seq_lens, B, q.data_ptr(),
+                       k.data_ptr(), v.data_ptr(), out.data_ptr(), torch.cuda.current_stream().cuda_stream)
+    torch.cuda.synchronize()
+    got = out.cpu().numpy().astype(np.float64)
+    worst = 0.0
+    for b in range(B):
+        K, V = ks.host_kv_logical(w, 0, b, t)
+        for h in range(nq):
+            g = h // (nq // nkv)
+            o, _ = oracle.attend(qf[b, h].astype(np.float64), K[:, g, :], V[:, g, :], kf[b, g].astype(np.float64),
+                                 vf[b, g].astype(np.float64))
+            e = np.abs(got[b, h] - o).max() / np.abs(o).max()
+            worst = max(worst, e)
+    print(f"teacher-forced attention: max rel err {worst:.3e}")
+    assert worst <= ATTN_RTOL
+
+
+def test_resolve_bit_exact():
+    import paper_2607_09153_gb300 as kp
+    t = ks.Tables.make()
+    w = ks.mcts_tree("resolve", ks.ARCH_TINY, 42, branching=2, depth=3, lo=3, hi=50)
+    _, _, dev, sc = run_gpu(w, t, debug=False)
+    for b in range(w.n_candidates):
+        L = int(w.seq_lens[b])
+        got = kp.kvprm_resolve(sc.ctx, b, L)
+        pos = np.arange(L)
+        ref = w.block_table[b, pos // 16].astype(np.int64) * 16 + pos % 16
+        np.testing.assert_array_equal(got, ref)
+        # and the rows it names hold the candidate's logical tokens
+        seg = w.page_seg.reshape(-1)[got]
+        off = w.page_off.reshape(-1)[got]
+        np.testing.assert_array_equal(seg, w.cand_seg[b])
+        np.testing.assert_array_equal(off, w.cand_off[b])
+
+
+def test_deterministic_and_host_path():
+    import paper_2607_09153_gb300 as kp
+    torch = require_gpu()
+    t = ks.Tables.make(0.2)
+    w = ks.distinct("det", ks.ARCH_TINY, 43, [5, 600, 1234, 64], gain_std=0.2)
+    r1, _, dev, sc = run_gpu(w, t, debug=False)
+    r2 = sc.score(dev.pool, w.block_table, w.seq_lens)
+    assert np.array_equal(r1.astype(np.float32), r2)
+    host_pool = dev.pool.cpu().pin_memory()
+    r3 = kp.kvprm_score_host(sc.ctx, host_pool.data_ptr(), dev.n_pages, w.block_table, w.seq_lens, w.n_candidates,
+                             torch.cuda.current_stream().cuda_stream)
+    assert np.array_equal(r3, r2)
+    d = torch.empty(w.n_candidates, dtype=torch.float32, device="cuda")
+    sc.score_async(dev.pool, w.block_table, w.seq_lens, d)
+    torch.cuda.synchronize()
+    assert np.array_equal(d.cpu().numpy(), r2)
+
+
+def test_host_side_errors():
+    import paper_2607_09153_gb300 as kp
+    t = ks.Tables.make()
+    w = ks.distinct("err", ks.ARCH_TINY, 44, [20, 40])
+    _, _, dev, sc = run_gpu(w, t, debug=False)
+    bt = w.block_table.copy()
+    bt[1, 1] = dev.n_pages            # out of range page id
+    with pytest.raises(kp.KvprmError) as e:
+        sc.score(dev.pool, bt, w.seq_lens)
+    assert e.value.code == 3
+    bt = w.block_table.copy()
+    bt[0, 2] = -7                     # beyond ceil(20/16) = 2 blocks: ignored
+    sc.score(dev.pool, bt, w.seq_lens)
+    with pytest.raises(kp.KvprmError) as e:    # longer than max_blocks * 16
+        sc.score(dev.pool, w.block_table, np.array([20, 16 * w.max_blocks + 1], np.int32))
+    assert e.value.code == 2
+    with pytest.raises(kp.KvprmError) as e:    # more candidates than the context holds
+        kp.kvprm_score(sc.ctx, dev.pool.data_ptr(), dev.n_pages, np.zeros((3, w.max_blocks), np.int32),
+                       np.zeros(3, np.int32), 3)
+    assert e.value.code == 2
+    with pytest.raises(kp.KvprmError) as e:
+        sc.score(dev.pool, w.block_table, np.array([20, -1], np.int32))
+    assert e.value.code == 1
+    assert kp.kvprm_score(sc.ctx, 0, 0, np.zeros((0, 1), np.int32), np.zeros(0, np.int32), 0).size == 0
