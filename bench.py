@@ -1,0 +1,408 @@
+"""Benchmark of KV-PRM verify-token scoring on GB300.
+
+One step = one kvprm_score call: the verify token of every candidate in the
+batch forwarded through all layers against its paged cache (embedding, per
+layer RMSNorm / QKV / RoPE / paged split-K attention / combine / O / RMSNorm /
+SiLU-gated MLP, final norm and the two-logit head).  Default workload: the
+1.5B-shaped scorer (28 layers, d=1536, 12/2 heads, hd=128, MLP 8960) scoring
+B=16 candidates with distinct caches of L=2048 (page size 16), seeded
+synthetic bf16 weights N(0, 0.02) and K/V N(0, 1).
+
+Printed (rank 0, one JSON line): scores/s over the timed steps with inputs
+resident in HBM (`value`), the same through the host-buffer C-ABI call with
+the cache copied host->device every step (`e2e`), the per-kernel-class CUDA
+event times of a second timed pass, the roofline of the dominant kernel and
+of the attention kernel, the SM clocks seen during the timed region, and the
+CPU oracle timed on a bounded sample of the same workload (`cpu_baseline`).
+
+`--impl reference` times the CPU oracle alone (the reference arm).
+Multi-GPU (torchrun): each rank scores its own replica batch (candidates
+shard with no exchange), weak scaling, max time over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import ctypes
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+HBM_NOMINAL_GBS = 8000.0   # the 8 TB/s denominator the metric is quoted against
+METRIC = "verify-token scores/sec"
+
+
+def load_peaks() -> dict:
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "src": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "src": "fallback"}
+
+
+# ---------------------------------------------------------------- distributed
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend=backend)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{gpu_index}.csv")
+
+    def start(self):
+        os.makedirs(os.path.dirname(self.path), exist_ok=True)
+        try:
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.fh,
+                                         stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.fh.close()
+        sm, smax, reasons, power = [], [], set(), []
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+                power.append(float(parts[3]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm), "power_w_max": max(power) if power else None}
+
+
+# ---------------------------------------------------------------- workload
+def algorithmic_bytes(w) -> dict:
+    import kvsynth as ks
+    a = w.arch
+    per = {
+        "gemm_qkv": a.n_layers * 2 * a.qkv_rows * a.d_model,
+        "gemm_o": a.n_layers * 2 * a.d_model * a.n_q_heads * a.head_dim,
+        "gemm_gate_up": a.n_layers * 2 * 2 * a.d_ff * a.d_model,
+        "gemm_down": a.n_layers * 2 * a.d_model * a.d_ff,
+        "attention": w.unique_kv_bytes(),
+    }
+    per["weights_total"] = a.weight_bytes()
+    per["call_total"] = per["weights_total"] + per["attention"]
+    del ks
+    return per
+
+
+def source_hash(files: list[str]) -> str:
+    h = hashlib.sha256()
+    for f in files:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+KERNEL_SOURCES = {
+    "gemm": ["paper_2607_09153_gb300/csrc/gemm_tc.cu", "paper_2607_09153_gb300/csrc/ptx.cuh"],
+    "attention": ["paper_2607_09153_gb300/csrc/attention.cu", "paper_2607_09153_gb300/csrc/ptx.cuh"],
+}
+
+
+def ncu_traffic(kernel: str, workload: str):
+    """Per-launch DRAM bytes from the committed ncu summary, if it was taken on
+    the current kernel source (else None)."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+        e = rec[workload][kernel]
+        fam = "gemm" if kernel.startswith("gemm") else "attention"
+        if e.get("source_hash") != source_hash(KERNEL_SOURCES[fam]):
+            return None
+        return float(e["dram_bytes_per_launch"])
+    except Exception:
+        return None
+
+
+# ---------------------------------------------------------------- CPU oracle
+def cpu_oracle_time(w, tables, budget_s: float = 12.0, max_cands: int | None = None):
+    """Time the oracle (exact mode) on a bounded sample of the workload's candidates."""
+    import kvsynth as ks
+    import oracle
+    nthreads = os.cpu_count() or 1
+    a = w.arch
+    t0 = time.perf_counter()
+    W = ks.host_weights(a, w.seed, tables)
+    t_gen = time.perf_counter() - t0
+    cap = w.n_candidates if max_cands is None else min(max_cands, w.n_candidates)
+
+    def run(ids):
+        kv = [[ks.host_kv_logical(w, l, b, tables) for b in ids] for l in range(a.n_layers)]
+        t = time.perf_counter()
+        oracle.score_dense(a, W, kv, mirror=False, want_attn=False, nthreads=nthreads)
+        return time.perf_counter() - t
+
+    t1 = run([0])
+    n = int(max(1, min(cap, budget_s / max(t1, 1e-3))))
+    if n > 1:
+        ids = list(range(n))
+        tn = run(ids)
+    else:
+        ids, tn = [0], t1
+    return {"value": n / tn, "unit": "scores/s", "cores": nthreads, "kind": "oracle",
+            "sample": f"{n} of {w.n_candidates} candidates of {w.name}, fp64 exact mode, {tn:.2f} s "
+                      f"(weights generated beforehand in {t_gen:.1f} s, not timed)"}
+
+
+def run_reference(args, world, rank):
+    """The reference arm: the CPU oracle as it stands, on this host's cores."""
+    if rank != 0:
+        return
+    import kvsynth as ks
+    w = ks.make_workload(args.workload)
+    t = ks.Tables.make()
+    samples = []
+    budget = max(5.0, 60.0 / max(1, args.steps + args.warmup))
+    for i in range(args.warmup + args.steps):
+        r = cpu_oracle_time(w, t, budget_s=budget, max_cands=4)
+        if i >= args.warmup:
+            samples.append(r)
+    val = float(np.mean([s["value"] for s in samples]))
+    line = {"impl": "reference", "metric": METRIC, "value": val, "unit": "scores/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * w.n_candidates / val,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": workload_config(w, args),
+            "cpu_baseline": {"value": val, "unit": "scores/s", "cores": samples[0]["cores"], "kind": "oracle",
+                             "sample": samples[0]["sample"]},
+            "e2e": {"value": val, "unit": "scores/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def workload_config(w, args) -> dict:
+    a = w.arch
+    return {"workload": w.name, "layers": a.n_layers, "d_model": a.d_model, "n_q_heads": a.n_q_heads,
+            "n_kv_heads": a.n_kv_heads, "head_dim": a.head_dim, "d_ff": a.d_ff, "candidates": w.n_candidates,
+            "seq_len_min": int(w.seq_lens.min()), "seq_len_max": int(w.seq_lens.max()), "page_size": a.page_size,
+            "unique_pages": int(len(set(np.concatenate([w.block_table[b, :(int(w.seq_lens[b]) + 15) // 16]
+                                                        for b in range(w.n_candidates)]).tolist()))),
+            "l2": "inputs exceed L2 (weights + cache >> 129 MB); no flush", "parallelism": f"replicas{args.gpus}"}
+
+
+# ---------------------------------------------------------------- GPU arm
+def make_scorer(dev, max_candidates: int, max_blocks: int):
+    import kvsynth as ks
+    from paper_2607_09153_gb300 import Scorer
+    a = dev.arch
+    wt = {"embed_verify": dev.top[ks.EMBED], "final_norm": dev.top[ks.FINAL_NORM], "w_plus": dev.top[ks.W_PLUS],
+          "w_minus": dev.top[ks.W_MINUS],
+          "layers": [{"attn_norm": L[ks.ATTN_NORM], "w_qkv": L[ks.W_QKV], "w_o": L[ks.W_O], "mlp_norm": L[ks.MLP_NORM],
+                      "w_gate_up": L[ks.W_GATE_UP], "w_down": L[ks.W_DOWN]} for L in dev.layers]}
+    return Scorer(a.n_layers, a.d_model, a.n_q_heads, a.n_kv_heads, a.head_dim, a.d_ff, wt, max_candidates, max_blocks,
+                  a.rope_base, a.rms_eps)
+
+
+def run_gpu(args, world, rank, local):
+    import torch
+
+    import kvsynth as ks
+    import paper_2607_09153_gb300 as kp
+
+    torch.cuda.set_device(local)
+    w = ks.make_workload(args.workload)
+    tables = ks.Tables.make()
+    dev = ks.DeviceInputs(w, tables)
+    a = w.arch
+    B = w.n_candidates
+    sc = make_scorer(dev, B, w.max_blocks)
+    stream = torch.cuda.Stream()
+    sp = stream.cuda_stream
+    d_rewards = torch.empty(B, dtype=torch.float32, device="cuda")
+    pool_ptr, n_pages = dev.pool.data_ptr(), dev.n_pages
+    bt, sl = np.ascontiguousarray(w.block_table), np.ascontiguousarray(w.seq_lens)
+
+    def step():
+        kp.kvprm_score_async(sc.ctx, pool_ptr, n_pages, bt, sl, B, d_rewards.data_ptr(), sp)
+
+    # ---- warm-up, then the device-resident timed region
+    for _ in range(args.warmup):
+        step()
+    stream.synchronize()
+    clocks = ClockSampler(local)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.start()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        step()
+    ev1.record(stream)
+    ev1.synchronize()
+    torch.cuda.synchronize()
+    barrier(world)
+    clk = clocks.stop()
+    ms = ev0.elapsed_time(ev1)
+    ms = max_over_ranks(ms, world)
+    value = world * B * args.steps / (ms / 1000.0)
+    kp.kvprm_check_device(sc.ctx)
+
+    # ---- end to end through the host-buffer call (cache copied H2D every step)
+    host_pool = dev.pool.cpu().pin_memory()
+    rewards = np.zeros(B, np.float32)
+    e2e_steps = max(3, args.steps // 10)
+    for _ in range(2):
+        kp.kvprm_score_host(sc.ctx, host_pool.data_ptr(), n_pages, bt, sl, B, sp, rewards)
+    barrier(world)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        kp.kvprm_score_host(sc.ctx, host_pool.data_ptr(), n_pages, bt, sl, B, sp, rewards)
+    t_e2e = max_over_ranks(time.perf_counter() - t0, world)
+    e2e = {"value": world * B * e2e_steps / t_e2e, "unit": "scores/s",
+           "h2d_bytes_per_step": int(host_pool.numel() * 2 + bt.nbytes + sl.nbytes),
+           "d2h_bytes_per_step": int(B * 4 + 4), "steps": e2e_steps,
+           "path": "kvprm_score_host: pinned host cache + host tables -> rewards on host"}
+    del host_pool
+
+    # ---- second timed pass: per-kernel-class CUDA event times
+    prof_steps = max(3, min(args.steps, args.profile_steps))
+    kp.kvprm_set_profile(sc.ctx, True)
+    for _ in range(prof_steps):
+        step()
+    prof = kp.kvprm_get_profile(sc.ctx)
+    kp.kvprm_set_profile(sc.ctx, False)
+    stream.synchronize()
+
+    launches_per_step = sum(n for n, _ in prof.values()) / prof_steps
+    alg = algorithmic_bytes(w)
+    peaks = load_peaks()
+    kernels = {}
+    for name, (n, tot) in prof.items():
+        if n == 0:
+            continue
+        kernels[name] = {"launches": n, "total_ms": round(tot, 4), "avg_us": round(1000 * tot / n, 3),
+                         "share": None}
+    total_ms = sum(k["total_ms"] for k in kernels.values())
+    for k in kernels.values():
+        k["share"] = round(k["total_ms"] / total_ms, 4)
+
+    def roof(name):
+        n, tot = prof[name]
+        per_launch = alg[name] / a.n_layers
+        avg_s = tot / n / 1000.0
+        ach = per_launch / avg_s / 1e9
+        return {"bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": round(ach / peaks["hbm_gbs"], 4), "peak_src": peaks["src"],
+                "traffic": ncu_traffic(name, w.name), "kernel": name,
+                "algorithmic_bytes_per_launch": int(per_launch), "avg_launch_us": round(avg_s * 1e6, 3)}
+
+    dominant = max((k for k in kernels if k in alg), key=lambda k: kernels[k]["total_ms"])
+    attn = roof("attention")
+    attention_obj = {"achieved_gbs": attn["achieved"], "frac_of_8tbs": round(attn["achieved"] / HBM_NOMINAL_GBS, 4),
+                     "frac_of_measured": attn["frac"], "unique_kv_bytes_per_step": alg["attention"],
+                     "avg_launch_us": attn["avg_launch_us"]}
+    step_bytes = alg["call_total"]
+    line = {
+        "metric": METRIC, "value": round(value, 2), "unit": "scores/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 5), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "accumulate": "f32",
+        "data": "synthetic (seeded bf16 weights N(0,0.02), K/V N(0,1), random-init)",
+        "config": workload_config(w, args),
+        "e2e": e2e,
+        "gpu_launches": int(round(launches_per_step)) * args.steps,
+        "roofline": roof(dominant),
+        "attention": attention_obj,
+        "whole_call": {"bytes_per_step": step_bytes,
+                       "achieved_gbs": round(step_bytes / (ms / args.steps / 1000.0) / 1e9, 1),
+                       "frac_of_8tbs": round(step_bytes / (ms / args.steps / 1000.0) / 1e9 / HBM_NOMINAL_GBS, 4)},
+        "kernels": kernels,
+        "profile_steps": prof_steps,
+        "clocks": clk,
+    }
+    sc.close()
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_oracle_time(w, tables, budget_s=args.cpu_budget)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def main():
+    import kvsynth as ks
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="qwen1p5b_b16_l2048", choices=list(ks.WORKLOAD_NAMES))
+    ap.add_argument("--profile-steps", type=int, default=50)
+    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    world, rank, local = dist_setup()
+    if args.impl == "reference":
+        run_reference(args, world, rank)
+    else:
+        run_gpu(args, world, rank, local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

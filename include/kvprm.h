@@ -189,12 +189,22 @@ KVPRM_API int kvprm_resolve(kvprm_ctx* ctx, int32_t b, int64_t* phys_row);
 KVPRM_API int kvprm_check_device(kvprm_ctx* ctx);
 
 /* Per-kernel-class timing of kvprm_score* calls, measured with CUDA events on
- * the scoring stream while enabled (adds one event pair per timed launch).
- * Classes: 0 projection GEMMs, 1 paged attention (split-K), 2 attention
- * combine, 3 fused norm / RoPE / SiLU / head kernels.  kvprm_get_profile
- * synchronises, accumulates the recorded pairs and returns per class the
- * launch count and total milliseconds since profiling was enabled. */
-enum { KVPRM_PROF_GEMM = 0, KVPRM_PROF_ATTN = 1, KVPRM_PROF_COMBINE = 2, KVPRM_PROF_FUSED = 3, KVPRM_PROF_N = 4 };
+ * the scoring stream while enabled (one event pair per launch; programmatic
+ * launch overlap is switched off meanwhile, so each launch is timed alone).
+ * Classes: 0..3 the QKV, O, gate/up and down projections, 4 paged attention
+ * (split-K), 5 attention combine, 6 fused norm / RoPE / SiLU / head kernels.
+ * Profiled calls synchronise the stream.  kvprm_get_profile returns per class
+ * the launch count and total milliseconds since profiling was enabled. */
+enum {
+  KVPRM_PROF_GEMM_QKV = 0,
+  KVPRM_PROF_GEMM_O = 1,
+  KVPRM_PROF_GEMM_GATE_UP = 2,
+  KVPRM_PROF_GEMM_DOWN = 3,
+  KVPRM_PROF_ATTN = 4,
+  KVPRM_PROF_COMBINE = 5,
+  KVPRM_PROF_FUSED = 6,
+  KVPRM_PROF_N = 7
+};
 KVPRM_API int kvprm_set_profile(kvprm_ctx* ctx, int enable);
 KVPRM_API int kvprm_get_profile(kvprm_ctx* ctx, int64_t* launches, double* total_ms);
 

@@ -105,8 +105,8 @@ struct kvprm_ctx {
   // profiling
   bool profile = false;
   std::vector<ProfMark> live_marks;   // marks recorded in the current (non-graph) capture
-  int64_t prof_launches[KVPRM_PROF_N] = {0, 0, 0, 0};
-  double prof_ms[KVPRM_PROF_N] = {0, 0, 0, 0};
+  int64_t prof_launches[KVPRM_PROF_N] = {};
+  double prof_ms[KVPRM_PROF_N] = {};
   std::string last_error;
   cudaStream_t last_stream = nullptr;
 };
@@ -348,7 +348,7 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
   LAUNCH(KVPRM_PROF_FUSED, kvprm::launch_embed_norm(m, ctx->embed, ctx->attn_norm[0], n, ctx->h, X, st, pdl),
          "embed_norm");
   for (int l = 0; l < NL; ++l) {
-    LAUNCH(KVPRM_PROF_GEMM,
+    LAUNCH(KVPRM_PROF_GEMM_QKV,
            kvprm::launch_gemm(P.g_qkv, &ctx->tm_qkv[l], &ctx->tm_xhi, &ctx->tm_xlo, ctx->part, m.qkv_rows, n, np,
                               ctx->err_d, st, pdl),
            "gemm_qkv");
@@ -371,7 +371,7 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
            kvprm::launch_attn_combine(ctx->as, P.attn, sl, ctx->q, ctx->kself, ctx->vself, ctx->apart_o,
                                       ctx->apart_ml, n, O.hi, O.lo, nullptr, dbg, st, pdl),
            "attn_combine");
-    LAUNCH(KVPRM_PROF_GEMM,
+    LAUNCH(KVPRM_PROF_GEMM_O,
            kvprm::launch_gemm(P.g_o, &ctx->tm_o[l], &ctx->tm_ohi, &ctx->tm_olo, ctx->part, m.d, n, np, ctx->err_d, st,
                               pdl),
            "gemm_o");
@@ -379,12 +379,12 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
            kvprm::launch_resid_norm(m, ctx->part, P.g_o.splits, n, ctx->h, ctx->mlp_norm[l], X, nullptr, nullptr,
                                     nullptr, st, pdl),
            "resid_norm");
-    LAUNCH(KVPRM_PROF_GEMM,
+    LAUNCH(KVPRM_PROF_GEMM_GATE_UP,
            kvprm::launch_gemm(P.g_gu, &ctx->tm_gu[l], &ctx->tm_xhi, &ctx->tm_xlo, ctx->part, 2 * m.ff, n, np,
                               ctx->err_d, st, pdl),
            "gemm_gate_up");
     LAUNCH(KVPRM_PROF_FUSED, kvprm::launch_silu_mul(m, ctx->part, P.g_gu.splits, n, A, st, pdl), "silu_mul");
-    LAUNCH(KVPRM_PROF_GEMM,
+    LAUNCH(KVPRM_PROF_GEMM_DOWN,
            kvprm::launch_gemm(P.g_down, &ctx->tm_down[l], &ctx->tm_ahi, &ctx->tm_alo, ctx->part, m.d, n, np,
                               ctx->err_d, st, pdl),
            "gemm_down");
@@ -810,7 +810,7 @@ int kvprm_projection(kvprm_ctx* ctx, const void* W, int32_t M, int32_t K, const 
   if ((rc = make_map(ctx, &tx, X, K, n, 64, n_pad, "X"))) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   Enq E{ctx, st, false, ctx->profile, &ctx->live_marks};
-  LAUNCH(KVPRM_PROF_GEMM, kvprm::launch_gemm(g, &tw, &tx, nullptr, ctx->part, M, n, n_pad, ctx->err_d, st, false),
+  LAUNCH(KVPRM_PROF_GEMM_QKV, kvprm::launch_gemm(g, &tw, &tx, nullptr, ctx->part, M, n, n_pad, ctx->err_d, st, false),
          "gemm");
   LAUNCH(KVPRM_PROF_FUSED, kvprm::launch_split_sum(ctx->part, g.splits, static_cast<int64_t>(n) * M, Y, st),
          "split_sum");

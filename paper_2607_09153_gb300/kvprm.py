@@ -17,8 +17,7 @@ from . import build as _build
 
 KVPRM_OK, KVPRM_EINVAL, KVPRM_ECAPACITY, KVPRM_EINDEX, KVPRM_ECUDA, KVPRM_ENOMEM, KVPRM_ETIMEOUT, \
     KVPRM_EUNSUPPORTED = range(8)
-PROF_GEMM, PROF_ATTN, PROF_COMBINE, PROF_FUSED = range(4)
-PROF_NAMES = ("gemm", "attention", "combine", "fused")
+PROF_NAMES = ("gemm_qkv", "gemm_o", "gemm_gate_up", "gemm_down", "attention", "combine", "fused")
 
 
 class KvprmError(RuntimeError):
@@ -174,10 +173,12 @@ def kvprm_set_profile(ctx, enable: bool) -> None:
 
 
 def kvprm_get_profile(ctx) -> dict:
-    n = np.zeros(4, np.int64)
-    ms = np.zeros(4, np.float64)
+    """{class name: (launches, total ms)} since profiling was enabled."""
+    k = len(PROF_NAMES)
+    n = np.zeros(k, np.int64)
+    ms = np.zeros(k, np.float64)
     _check(ctx, lib().kvprm_get_profile(ctx, _p(n, ctypes.c_int64), ms.ctypes.data_as(ctypes.POINTER(ctypes.c_double))))
-    return {PROF_NAMES[i]: (int(n[i]), float(ms[i])) for i in range(4)}
+    return {PROF_NAMES[i]: (int(n[i]), float(ms[i])) for i in range(k)}
 
 
 # ------------------------------------------------------------------ torch convenience
