@@ -165,6 +165,36 @@ KVPRM_API int kvprm_projection(kvprm_ctx* ctx, const void* W, int32_t M, int32_t
  * (stream-ordered on the last call's stream). */
 KVPRM_API int kvprm_debug_hidden(kvprm_ctx* ctx, float* d_out);
 
+/* The paged attention read-out (as kvprm_attention) for callers that cannot
+ * allocate device memory -- e.g. a serving runtime that reserves all GPU memory
+ * up front and forbids allocations afterwards, or code running inside another
+ * framework's memory-managed region.  The paper has no counterpart; this is a
+ * deployment variant.  It needs no context and calls no cudaMalloc / cudaFree
+ * or allocating routine: its scratch is one static device array of
+ * KVPRM_NOALLOC_SCRATCH_BYTES that every GPU loading this library holds until
+ * the process exits.
+ *  kv_layer     device bf16 [n_pages][2][n_kv_heads][16][head_dim] (one layer)
+ *  block_table  host int32 [n_candidates][max_blocks_per_seq]; seq_lens host int32
+ *               [n_candidates] (validated and copied into the scratch array)
+ *  q            device float [n_candidates][n_q_heads][head_dim]
+ *  k_self, v_self  device float [n_candidates][n_kv_heads][head_dim]
+ *  out          device float [n_candidates][n_q_heads][head_dim]
+ * Stream-ordered.  Returns KVPRM_ECAPACITY when the block table, query and
+ * split partials would not fit in the array even with one split per sequence
+ * (roughly n_candidates * n_q_heads * head_dim * 18 B plus the tables), and
+ * the other codes as kvprm_attention (no detailed message: there is no
+ * context).  The first call on a device, made with that device current, looks
+ * up the array's address (cudaGetSymbolAddress) and configures the kernels:
+ * make it before any stream capture.  All calls share the array, which keeps
+ * the last call's contents; calls that overlap on the GPU race with each other
+ * and must be serialised by the caller.  An in-kernel bounded-wait timeout is
+ * recorded in the array but not reported by this entry point. */
+#define KVPRM_NOALLOC_SCRATCH_BYTES (32u << 20)
+KVPRM_API int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, const int32_t* block_table,
+                                      int32_t max_blocks_per_seq, const int32_t* seq_lens, int32_t n_candidates,
+                                      int32_t n_q_heads, int32_t n_kv_heads, int32_t head_dim, const float* q,
+                                      const float* k_self, const float* v_self, float* out, void* stream);
+
 /* Debug capture.  flags bit 0: keep every layer's attention output (the
  * combine result o, float, before its bf16 rounding) of each later
  * kvprm_score* call.  kvprm_debug_attn_out copies the last call's capture to

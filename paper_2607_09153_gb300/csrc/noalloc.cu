@@ -1,0 +1,201 @@
+// kvprm_attention_noalloc: the paged attention read-out for callers that must
+// not allocate device memory -- for example a serving runtime that reserves
+// all of its GPU memory up front and forbids allocations afterwards, or code
+// that runs inside another framework's memory-managed region where a
+// cudaMalloc would break the owner's accounting or stall on a device-wide
+// synchronisation.  It needs no context: its scratch (the copied block table
+// and lengths, the query split into bf16 hi/lo parts, the split-K partials and
+// an error word) lives in one file-scope device array, so every GPU that loads
+// this library holds that array until the process exits.
+//
+// Set-up: the first call on a device (with that device current) looks up the
+// array's device address with cudaGetSymbolAddress and configures the kernels;
+// make that first call before any stream capture.  All calls share the array
+// and it keeps the last call's contents, so calls that overlap on the GPU (on
+// different streams, or from several host threads) race and corrupt each
+// other's results; serialise them.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cstring>
+#include <mutex>
+
+#include "../../include/kvprm.h"
+#include "kernels.h"
+
+namespace {
+
+static __device__ __align__(256) unsigned char g_scratch[KVPRM_NOALLOC_SCRATCH_BYTES];
+
+constexpr int kMaxDevices = 64;
+constexpr int kSplitCapMax = 32;
+
+struct DeviceState {
+  bool ready = false;
+  unsigned char* scratch = nullptr;
+};
+std::mutex g_mu;
+DeviceState g_dev[kMaxDevices];
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+// Once per device, with that device current: the array's device address and
+// the kernels' shared-memory limits.  Returns a KVPRM_* status.
+int setup_current_device(unsigned char** scratch) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return KVPRM_ECUDA;
+  std::lock_guard<std::mutex> lock(g_mu);
+  DeviceState& s = g_dev[dev];
+  if (!s.ready) {
+    void* ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_scratch) != cudaSuccess || ptr == nullptr) return KVPRM_ECUDA;
+    if (kvprm::attention_configure() != cudaSuccess) return KVPRM_ECUDA;
+    if (!g_encode) {
+      void* fn = nullptr;
+      cudaDriverEntryPointQueryResult q;
+      if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
+              cudaSuccess ||
+          !fn || q != cudaDriverEntryPointSuccess)
+        return KVPRM_ECUDA;
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    s.scratch = static_cast<unsigned char*>(ptr);
+    s.ready = true;
+  }
+  *scratch = s.scratch;
+  return KVPRM_OK;
+}
+
+size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+struct Carve {
+  size_t err, sl, bt, qhi, qlo, ohi, olo, pml, po, total;
+};
+
+Carve carve(int n, int max_blocks, int n_q, int hd, int n_split) {
+  Carve c;
+  size_t off = 0;
+  c.err = off;
+  off = align256(off + sizeof(int));
+  c.sl = off;
+  off = align256(off + sizeof(int32_t) * n);
+  c.bt = off;
+  off = align256(off + sizeof(int32_t) * static_cast<size_t>(n) * max_blocks);
+  const size_t qe = static_cast<size_t>(n) * n_q * hd;
+  c.qhi = off;
+  off = align256(off + 2 * qe);
+  c.qlo = off;
+  off = align256(off + 2 * qe);
+  c.ohi = off;
+  off = align256(off + 2 * qe);
+  c.olo = off;
+  off = align256(off + 2 * qe);
+  c.pml = off;
+  off = align256(off + sizeof(float) * static_cast<size_t>(n) * n_q * n_split * 2);
+  c.po = off;
+  off = align256(off + sizeof(float) * qe * n_split);
+  c.total = off;
+  return c;
+}
+
+}  // namespace
+
+extern "C" int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, const int32_t* block_table,
+                                       int32_t max_blocks_per_seq, const int32_t* seq_lens, int32_t n_candidates,
+                                       int32_t n_q_heads, int32_t n_kv_heads, int32_t head_dim, const float* q,
+                                       const float* k_self, const float* v_self, float* out, void* stream) {
+  const int n = n_candidates;
+  if (n < 0 || n_q_heads < 1 || n_kv_heads < 1 || max_blocks_per_seq < 1 || n_pages < 0) return KVPRM_EINVAL;
+  if (head_dim != 64 && head_dim != 128) return KVPRM_EUNSUPPORTED;
+  if (n_q_heads % n_kv_heads || n_q_heads / n_kv_heads > 16) return KVPRM_EUNSUPPORTED;
+  if (n == 0) return KVPRM_OK;
+  if (!block_table || !seq_lens || !q || !k_self || !v_self || !out) return KVPRM_EINVAL;
+  auto al16 = [](const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; };
+  if (!al16(q) || !al16(k_self) || !al16(v_self)) return KVPRM_EINVAL;
+  // host-side validation of the tables, as in kvprm_attention
+  int max_pages = 0;
+  for (int b = 0; b < n; ++b) {
+    const int L = seq_lens[b];
+    if (L < 0) return KVPRM_EINVAL;
+    if (static_cast<int64_t>(L) > static_cast<int64_t>(max_blocks_per_seq) * 16) return KVPRM_ECAPACITY;
+    const int np = (L + 15) / 16;
+    if (np > max_pages) max_pages = np;
+    for (int j = 0; j < np; ++j) {
+      const int32_t p = block_table[static_cast<int64_t>(b) * max_blocks_per_seq + j];
+      if (p < 0 || p >= n_pages) return KVPRM_EINDEX;
+    }
+  }
+  if (max_pages > 0 && (!kv_layer || !al16(kv_layer))) return KVPRM_EINVAL;
+
+  unsigned char* scratch = nullptr;
+  int rc = setup_current_device(&scratch);
+  if (rc) return rc;
+
+  kvprm::AttnShape as;
+  as.n_q = n_q_heads;
+  as.n_kv = n_kv_heads;
+  as.hd = head_dim;
+  as.group = n_q_heads / n_kv_heads;
+  as.max_blocks = max_blocks_per_seq;
+  int dev = 0, sms = 148;
+  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return KVPRM_ECUDA;
+  // the largest split count (<= kSplitCapMax) whose partials fit in the array
+  kvprm::AttnPlan plan;
+  Carve cv;
+  for (int cap = kSplitCapMax;; cap /= 2) {
+    plan = kvprm::plan_attention(as, n, max_pages, sms, cap);
+    cv = carve(n, max_blocks_per_seq, n_q_heads, head_dim, plan.n_split);
+    if (cv.total <= static_cast<size_t>(KVPRM_NOALLOC_SCRATCH_BYTES)) break;
+    if (cap == 1) return KVPRM_ECAPACITY;   // even one split per sequence does not fit
+  }
+
+  // tensor map over this layer's pages (built on the host stack; no allocation)
+  const void* pool = kv_layer;
+  int64_t pages = n_pages;
+  if (max_pages == 0) {   // nothing is read from the pool; any valid address serves the map
+    pool = scratch;
+    pages = 1;
+  }
+  const int64_t rows = pages * 2 * n_kv_heads * 16;
+  if (rows >= (static_cast<int64_t>(1) << 31)) return KVPRM_EUNSUPPORTED;
+  as.layer_rows = rows;
+  CUtensorMap tm;
+  {
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(head_dim), static_cast<cuuint64_t>(rows)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(head_dim) * 2};
+    cuuint32_t box[2] = {64, 16};
+    cuuint32_t estr[2] = {1, 1};
+    if (g_encode(&tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(pool), dims, strides, box, estr,
+                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return KVPRM_ECUDA;
+  }
+
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int* err = reinterpret_cast<int*>(scratch + cv.err);
+  int32_t* d_sl = reinterpret_cast<int32_t*>(scratch + cv.sl);
+  int32_t* d_bt = reinterpret_cast<int32_t*>(scratch + cv.bt);
+  kvprm::HiLo Q{reinterpret_cast<__nv_bfloat16*>(scratch + cv.qhi), reinterpret_cast<__nv_bfloat16*>(scratch + cv.qlo)};
+  __nv_bfloat16* ohi = reinterpret_cast<__nv_bfloat16*>(scratch + cv.ohi);
+  __nv_bfloat16* olo = reinterpret_cast<__nv_bfloat16*>(scratch + cv.olo);
+  float* pml = reinterpret_cast<float*>(scratch + cv.pml);
+  float* po = reinterpret_cast<float*>(scratch + cv.po);
+
+  // the error word must start at zero; everything else is written before it is read
+  if (cudaMemsetAsync(err, 0, sizeof(int), st) != cudaSuccess) return KVPRM_ECUDA;
+  if (cudaMemcpyAsync(d_sl, seq_lens, sizeof(int32_t) * n, cudaMemcpyHostToDevice, st) != cudaSuccess)
+    return KVPRM_ECUDA;
+  if (cudaMemcpyAsync(d_bt, block_table, sizeof(int32_t) * static_cast<size_t>(n) * max_blocks_per_seq,
+                      cudaMemcpyHostToDevice, st) != cudaSuccess)
+    return KVPRM_ECUDA;
+  if (kvprm::launch_split_hilo(q, static_cast<int64_t>(n) * n_q_heads * head_dim, Q, st) != cudaSuccess)
+    return KVPRM_ECUDA;
+  if (kvprm::launch_attn_split(as, plan, &tm, 0, d_bt, d_sl, Q.hi, Q.lo, n, po, pml, err, st, false) != cudaSuccess)
+    return KVPRM_ECUDA;
+  if (kvprm::launch_attn_combine(as, plan, d_sl, q, k_self, v_self, po, pml, n, ohi, olo, out, nullptr, st, false) !=
+      cudaSuccess)
+    return KVPRM_ECUDA;
+  return KVPRM_OK;
+}

@@ -64,6 +64,7 @@ def lib() -> ctypes.CDLL:
         L.kvprm_attention.argtypes = [vp, vp, i64, i32p, i32p, i32, vp, vp, vp, vp, vp]
         L.kvprm_projection.argtypes = [vp, vp, i32, i32, vp, i32, vp, vp]
         L.kvprm_debug_hidden.argtypes = [vp, vp]
+        L.kvprm_attention_noalloc.argtypes = [vp, i64, i32p, i32, i32p, i32, i32, i32, i32, vp, vp, vp, vp, vp]
         L.kvprm_set_debug.argtypes = [vp, ctypes.c_int]
         L.kvprm_debug_attn_out.argtypes = [vp, vp]
         L.kvprm_debug_layers.argtypes = [vp, ctypes.c_int, vp]
@@ -144,6 +145,19 @@ def kvprm_projection(ctx, W_ptr: int, M: int, K: int, X_ptr: int, n: int, Y_ptr:
 
 def kvprm_debug_hidden(ctx, d_out_ptr: int) -> None:
     _check(ctx, lib().kvprm_debug_hidden(ctx, d_out_ptr))
+
+
+def kvprm_attention_noalloc(kv_layer_ptr: int, n_pages: int, block_table, seq_lens, n_q_heads: int, n_kv_heads: int,
+                            head_dim: int, q_ptr: int, k_self_ptr: int, v_self_ptr: int, out_ptr: int,
+                            stream_ptr: int = 0) -> None:
+    """The attention read-out through the entry point that allocates nothing (no context)."""
+    bt, sl = _i32(block_table), _i32(seq_lens)
+    n = len(sl)
+    rc = lib().kvprm_attention_noalloc(kv_layer_ptr, n_pages, _p(bt, ctypes.c_int32), bt.shape[1] if bt.ndim == 2 else 1,
+                                       _p(sl, ctypes.c_int32), n, n_q_heads, n_kv_heads, head_dim, q_ptr, k_self_ptr,
+                                       v_self_ptr, out_ptr, stream_ptr)
+    if rc != KVPRM_OK:
+        raise KvprmError(rc, "kvprm_attention_noalloc failed")
 
 
 def kvprm_set_debug(ctx, flags: int) -> None:
