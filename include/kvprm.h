@@ -236,6 +236,15 @@ enum {
   KVPRM_PROF_N = 7
 };
 KVPRM_API int kvprm_set_profile(kvprm_ctx* ctx, int enable);
+
+/* Device timeline of the last kvprm_score* call, recorded by the kernels
+ * themselves with the GPU global timer while enabled (two atomics per CTA;
+ * launch overlap is kept).  kvprm_get_trace synchronises and fills, per launch
+ * in issue order, its class (as for profiling), the start of its first CTA and
+ * the end of its last CTA in microseconds from the first start; returns the
+ * number of records written, or a negative KVPRM_E* code. */
+KVPRM_API int kvprm_set_trace(kvprm_ctx* ctx, int enable);
+KVPRM_API int kvprm_get_trace(kvprm_ctx* ctx, int32_t max_records, int32_t* cls, double* start_us, double* end_us);
 KVPRM_API int kvprm_get_profile(kvprm_ctx* ctx, int64_t* launches, double* total_ms);
 
 #ifdef __cplusplus

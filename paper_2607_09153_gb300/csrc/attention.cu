@@ -15,7 +15,11 @@
 //    8..15 of the same instruction (their results are summed), so the split
 //    costs no extra MMAs; with 8 < G <= 16 hi and lo take one MMA each;
 //  - the four warps' (m, l, O) are merged in shared memory and written as one
-//    unnormalised split partial.
+//    unnormalised split partial;
+//  - the last CTA of a (candidate, kv head) to finish (an atomic arrival
+//    counter, no waiting) merges that group's splits together with the verify
+//    token's own entry and writes the attention output as a bf16 (hi, lo)
+//    pair for the O projection.
 // All scores are kept in log2 units (scaled by log2(e) / sqrt(hd)).
 #include <cuda_bf16.h>
 
@@ -42,12 +46,72 @@ __device__ __forceinline__ int32_t phys_page(const int32_t* __restrict__ bt, int
   return bt[static_cast<int64_t>(b) * max_blocks + j];
 }
 
+// Merge the ns split partials of every query head of group g of candidate b
+// with the verify token's own entry s_self = q . k_self / sqrt(hd):
+//   M = max(m_i, s_self), o = (sum_i 2^(m_i - M) o_i + 2^(s_self - M) v_self)
+//                             / (sum_i 2^(m_i - M) l_i + 2^(s_self - M)),
+// summed in split order.  One warp per head (5 warps, heads strided).
+template <int HD>
+__device__ __forceinline__ void merge_group(int b, int g, int n_q, int n_kv, int group, int ns, int n_split,
+                                            const float* __restrict__ part_o, const float* __restrict__ part_ml,
+                                            const AttnMerge& mg) {
+  constexpr int kPer = HD / 32;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t hk = static_cast<int64_t>(b) * n_kv + g;
+  for (int r = warp; r < group; r += kThreads / 32) {
+    const int64_t hq = static_cast<int64_t>(b) * n_q + static_cast<int64_t>(g) * group + r;
+    float qv[kPer], vv[kPer];
+    float dot = 0.f;
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) {
+      const int d = lane + 32 * j;
+      qv[j] = mg.q[hq * HD + d];
+      dot += qv[j] * mg.kself[hk * HD + d];
+      vv[j] = mg.vself[hk * HD + d];
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
+    const float s_self = dot * (kLog2e * rsqrtf(static_cast<float>(HD)));
+    const float mi = lane < ns ? __ldcg(part_ml + (hq * n_split + lane) * 2) : -INFINITY;
+    const float li = lane < ns ? __ldcg(part_ml + (hq * n_split + lane) * 2 + 1) : 0.f;
+    float M = fmaxf(mi, s_self);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
+    const float wi = lane < ns ? exp2f(mi - M) : 0.f;
+    const float wself = exp2f(s_self - M);
+    float lsum = wself;
+    for (int i = 0; i < ns; ++i) lsum += __shfl_sync(0xffffffffu, wi * li, i);
+    const float inv = 1.0f / lsum;
+    float acc[kPer];
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) acc[j] = wself * vv[j];
+    const float* po = part_o + hq * n_split * HD + lane;
+    for (int i = 0; i < ns; ++i) {
+      const float w = __shfl_sync(0xffffffffu, wi, i);
+#pragma unroll
+      for (int j = 0; j < kPer; ++j) acc[j] += w * __ldcg(po + i * HD + 32 * j);
+    }
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) {
+      const int d = lane + 32 * j;
+      const float out = acc[j] * inv;
+      const __nv_bfloat16 hi = __float2bfloat16_rn(out);
+      mg.o_hi[hq * HD + d] = hi;
+      mg.o_lo[hq * HD + d] = __float2bfloat16_rn(out - __bfloat162float(hi));
+      if (mg.out_f32) mg.out_f32[hq * HD + d] = out;
+      if (mg.dbg) mg.dbg[hq * HD + d] = out;
+    }
+  }
+}
+
 template <int HD, bool TWO_ROWS>
 __global__ void __launch_bounds__(kThreads) attn_split_kernel(
     const __grid_constant__ CUtensorMap tm_pool, int64_t layer_row0, const int32_t* __restrict__ bt,
     const int32_t* __restrict__ seq_lens, const __nv_bfloat16* __restrict__ q_hi,
     const __nv_bfloat16* __restrict__ q_lo, int n_q, int n_kv, int group, int max_blocks, int pages_per_split,
-    int n_split, float* __restrict__ part_o, float* __restrict__ part_ml, int* err) {
+    int n_split, float* __restrict__ part_o, float* __restrict__ part_ml, AttnMerge mg, int* err,
+    unsigned long long* ts) {
+  trace_begin(ts);
   constexpr int kSub = HD / 64;                       // 64-column sub-tiles per row
   constexpr uint32_t kBlockBytes = kSub * 16 * 128;   // one K (or V) page of one kv head
   constexpr uint32_t kPageBytes = 2 * kBlockBytes;
@@ -66,6 +130,8 @@ __global__ void __launch_bounds__(kThreads) attn_split_kernel(
   const int p1 = min(n_pages_b, p0 + pages_per_split);
   if (p0 >= p1) {
     grid_dep_wait();
+    if (n_pages_b == 0 && split == 0) merge_group<HD>(b, g, n_q, n_kv, group, 0, n_split, part_o, part_ml, mg);
+    trace_end(ts);
     return;
   }
   const int np = p1 - p0;
@@ -83,6 +149,7 @@ __global__ void __launch_bounds__(kThreads) attn_split_kernel(
     for (int i = lane; i < np; i += 32) bt_s[i] = phys_page(bt, b, max_blocks, p0 + i);
   }
   __syncthreads();
+  grid_dep_launch();   // the next kernel may start; it waits for this grid before reading its output
 
   const int gid = lane >> 2, tig = lane & 3;
   float m_run[2] = {-INFINITY, -INFINITY};
@@ -330,56 +397,19 @@ __global__ void __launch_bounds__(kThreads) attn_split_kernel(
       }
     }
   }
-  grid_dep_launch();
-}
-
-template <int HD>
-__global__ void __launch_bounds__(HD) attn_combine_kernel(const int32_t* __restrict__ seq_lens,
-                                                          const float* __restrict__ q, const float* __restrict__ kself,
-                                                          const float* __restrict__ vself,
-                                                          const float* __restrict__ part_o,
-                                                          const float* __restrict__ part_ml, int n_q, int n_kv,
-                                                          int pages_per_split, int n_split,
-                                                          __nv_bfloat16* __restrict__ o_hi,
-                                                          __nv_bfloat16* __restrict__ o_lo, float* __restrict__ out_f32,
-                                                          float* __restrict__ dbg) {
-  __shared__ float red[HD / 32];
-  const int h = blockIdx.x, b = blockIdx.y, d = threadIdx.x;
-  const int g = h / (n_q / n_kv);
-  grid_dep_wait();
-  const int L = seq_lens[b];
-  const int n_pages_b = (L + 15) >> 4;
-  const int ns = (n_pages_b + pages_per_split - 1) / pages_per_split;
-  const int64_t hq = static_cast<int64_t>(b) * n_q + h;
-  const int64_t hk = static_cast<int64_t>(b) * n_kv + g;
-  // the verify token's own entry: s_self = q . k_self / sqrt(hd)  (log2 units)
-  float prod = q[hq * HD + d] * kself[hk * HD + d];
-#pragma unroll
-  for (int off = 16; off > 0; off >>= 1) prod += __shfl_xor_sync(0xffffffffu, prod, off);
-  if ((d & 31) == 0) red[d >> 5] = prod;
+  // the last split of this (candidate, kv head) to arrive merges all of them
+  __shared__ int s_last;
+  __threadfence();
   __syncthreads();
-  float dot = 0.f;
-#pragma unroll
-  for (int w = 0; w < HD / 32; ++w) dot += red[w];
-  const float s_self = dot * (kLog2e * rsqrtf(static_cast<float>(HD)));
-  float M = s_self;
-  for (int i = 0; i < ns; ++i) M = fmaxf(M, part_ml[(hq * n_split + i) * 2]);
-  float f = exp2f(s_self - M);
-  float lsum = f;
-  float acc = f * vself[hk * HD + d];
-  for (int i = 0; i < ns; ++i) {
-    const float mi = part_ml[(hq * n_split + i) * 2], li = part_ml[(hq * n_split + i) * 2 + 1];
-    const float fi = exp2f(mi - M);
-    lsum += fi * li;
-    acc += fi * part_o[(hq * n_split + i) * HD + d];
+  const int ns_b = (n_pages_b + pages_per_split - 1) / pages_per_split;
+  if (threadIdx.x == 0) s_last = atomicAdd(&mg.counter[b * n_kv + g], 1) == ns_b - 1;
+  __syncthreads();
+  if (s_last) {
+    __threadfence();
+    merge_group<HD>(b, g, n_q, n_kv, group, ns_b, n_split, part_o, part_ml, mg);
+    if (threadIdx.x == 0) mg.counter[b * n_kv + g] = 0;   // ready for the next layer
   }
-  const float out = acc / lsum;
-  const __nv_bfloat16 hi = __float2bfloat16_rn(out);
-  o_hi[hq * HD + d] = hi;
-  o_lo[hq * HD + d] = __float2bfloat16_rn(out - __bfloat162float(hi));
-  if (out_f32) out_f32[hq * HD + d] = out;
-  if (dbg) dbg[hq * HD + d] = out;
-  grid_dep_launch();
+  trace_end(ts);
 }
 
 __global__ void resolve_kernel(const int32_t* __restrict__ bt, const int32_t* __restrict__ seq_lens, int max_blocks,
@@ -399,8 +429,8 @@ cudaError_t set_smem(K kernel) {
 AttnPlan plan_attention(const AttnShape& s, int n_cand, int max_pages, int num_sms, int split_cap) {
   AttnPlan p;
   const int pairs = n_cand * s.n_kv;
-  const int target = 4 * num_sms;
-  int ns = (target + pairs - 1) / (pairs > 0 ? pairs : 1);
+  const int target = 2 * num_sms;   // one wave at two CTAs per SM: every CTA can prefetch before q is ready
+  int ns = target / (pairs > 0 ? pairs : 1);
   if (ns < 1) ns = 1;
   if (ns > split_cap) ns = split_cap;
   if (max_pages < 1) max_pages = 1;
@@ -436,8 +466,8 @@ static cudaLaunchConfig_t make_cfg(dim3 grid, dim3 block, size_t smem, cudaStrea
 
 cudaError_t launch_attn_split(const AttnShape& s, const AttnPlan& p, const CUtensorMap* tm_pool, int layer,
                               const int32_t* bt, const int32_t* seq_lens, const __nv_bfloat16* q_hi,
-                              const __nv_bfloat16* q_lo, int n_cand, float* part_o, float* part_ml, int* err,
-                              cudaStream_t stream, bool pdl) {
+                              const __nv_bfloat16* q_lo, int n_cand, float* part_o, float* part_ml,
+                              const AttnMerge& mg, int* err, cudaStream_t stream, bool pdl, unsigned long long* ts) {
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg =
       make_cfg(dim3(p.n_split, s.n_kv, n_cand), dim3(kThreads), p.smem_bytes, stream, attr, pdl);
@@ -446,28 +476,15 @@ cudaError_t launch_attn_split(const AttnShape& s, const AttnPlan& p, const CUten
   if (s.hd == 128) {
     if (two)
       return cudaLaunchKernelEx(&cfg, attn_split_kernel<128, true>, *tm_pool, row0, bt, seq_lens, q_hi, q_lo, s.n_q, s.n_kv,
-                                s.group, s.max_blocks, p.pages_per_split, p.n_split, part_o, part_ml, err);
+                                s.group, s.max_blocks, p.pages_per_split, p.n_split, part_o, part_ml, mg, err, ts);
     return cudaLaunchKernelEx(&cfg, attn_split_kernel<128, false>, *tm_pool, row0, bt, seq_lens, q_hi, q_lo, s.n_q, s.n_kv,
-                              s.group, s.max_blocks, p.pages_per_split, p.n_split, part_o, part_ml, err);
+                              s.group, s.max_blocks, p.pages_per_split, p.n_split, part_o, part_ml, mg, err, ts);
   }
   if (two)
     return cudaLaunchKernelEx(&cfg, attn_split_kernel<64, true>, *tm_pool, row0, bt, seq_lens, q_hi, q_lo, s.n_q, s.n_kv,
-                              s.group, s.max_blocks, p.pages_per_split, p.n_split, part_o, part_ml, err);
+                              s.group, s.max_blocks, p.pages_per_split, p.n_split, part_o, part_ml, mg, err, ts);
   return cudaLaunchKernelEx(&cfg, attn_split_kernel<64, false>, *tm_pool, row0, bt, seq_lens, q_hi, q_lo, s.n_q, s.n_kv,
-                            s.group, s.max_blocks, p.pages_per_split, p.n_split, part_o, part_ml, err);
-}
-
-cudaError_t launch_attn_combine(const AttnShape& s, const AttnPlan& p, const int32_t* seq_lens, const float* q,
-                                const float* kself, const float* vself, const float* part_o, const float* part_ml,
-                                int n_cand, __nv_bfloat16* o_hi, __nv_bfloat16* o_lo, float* out_f32, float* dbg,
-                                cudaStream_t stream, bool pdl) {
-  cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = make_cfg(dim3(s.n_q, n_cand), dim3(s.hd), 0, stream, attr, pdl);
-  if (s.hd == 128)
-    return cudaLaunchKernelEx(&cfg, attn_combine_kernel<128>, seq_lens, q, kself, vself, part_o, part_ml, s.n_q,
-                              s.n_kv, p.pages_per_split, p.n_split, o_hi, o_lo, out_f32, dbg);
-  return cudaLaunchKernelEx(&cfg, attn_combine_kernel<64>, seq_lens, q, kself, vself, part_o, part_ml, s.n_q, s.n_kv,
-                            p.pages_per_split, p.n_split, o_hi, o_lo, out_f32, dbg);
+                            s.group, s.max_blocks, p.pages_per_split, p.n_split, part_o, part_ml, mg, err, ts);
 }
 
 cudaError_t launch_resolve(const int32_t* bt, const int32_t* seq_lens, int max_blocks, int b, int64_t* out,

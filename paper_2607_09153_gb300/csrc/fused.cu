@@ -1,17 +1,16 @@
-// Small fused kernels around the projections, each reducing the GEMM's split-K
-// partials in a fixed order (deterministic) and applying the next step of the
-// decoder block for the verify token (Sec. 4.1; cost term c_ffn d^2 of Eq.
-// cost_kv is in the GEMMs, these are the O(d) glue).  All arithmetic is fp32;
-// an activation that feeds a tensor-core contraction is stored as a bf16
-// (hi, lo) pair, hi = bf16(x), lo = bf16(x - hi), so no bf16 rounding of the
-// activation itself enters the result.
+// Small kernels around the projections of the verify-token forward (Sec. 4.1;
+// the c_ffn d^2 and c_attn d L terms of Eq. cost_kv live in the GEMMs and the
+// attention, these are the O(d) glue).  All arithmetic is fp32; an activation
+// that feeds a tensor-core contraction is stored as a bf16 (hi, lo) pair,
+// hi = bf16(x), lo = bf16(x - hi), so no bf16 rounding of the activation
+// itself enters the result.
 //   rope_table   cos/sin of p * base^(-2i/hd) at p = L_b (fp64 angles)
-//   embed_norm   h = e_v ; x = RMSNorm(h) * g
-//   qkv_post     q, k, v = sum of splits ; RoPE(q, k)
-//   resid_norm   h += sum of splits ; x = RMSNorm(h) * g, or, after the last
-//                layer, x = RMSNorm(h) * g_final and
-//                P(+) = 1 / (1 + exp(w_minus.x - w_plus.x))   (Eq. score)
-//   silu_mul     a = SiLU(gate) * up
+//   embed_norm   h = e_v ; per-tile sums of squares of h ; x = RMSNorm(h) * g
+//   norm         x = h * r * g with r = 1/sqrt(mean(h^2) + eps), mean(h^2)
+//                from the per-128-row-tile sums of squares the residual
+//                GEMM epilogue wrote (summed in tile order: deterministic)
+//   head         x = RMSNorm(h) * g_final ; P(+) = 1/(1 + exp(w_minus.x - w_plus.x))
+//                (Eq. score, App. B.2)
 #include <cuda_bf16.h>
 
 #include "kernels.h"
@@ -40,19 +39,39 @@ __device__ __forceinline__ float block_sum(float v, float* red) {
   return t;
 }
 
-__global__ void rope_table_kernel(const int32_t* __restrict__ seq_lens, int hd, double base, float2* __restrict__ tab) {
+// 1/sqrt(mean(h^2) + eps) of candidate b from the per-tile sums of squares,
+// summed in tile order by one thread and broadcast through shared memory.
+__device__ __forceinline__ float row_rscale(const float* __restrict__ sumsq, int m_tiles, int n_cand, int b, int d,
+                                            float eps, float* slot) {
+  if (threadIdx.x == 0) {
+    float s = 0.f;
+    for (int t = 0; t < m_tiles; ++t) s += sumsq[static_cast<int64_t>(t) * n_cand + b];
+    *slot = 1.0f / sqrtf(s / d + eps);
+  }
+  __syncthreads();
+  return *slot;
+}
+
+__global__ void rope_table_kernel(const int32_t* __restrict__ seq_lens, int hd, double base, float2* __restrict__ tab,
+                                  unsigned long long* ts) {
+  trace_begin(ts);
+  grid_dep_launch();
   grid_dep_wait();
   const int b = blockIdx.x, i = threadIdx.x;
   if (i < hd / 2) {
     const double ang = static_cast<double>(seq_lens[b]) * pow(base, -2.0 * i / hd);
     tab[b * (hd / 2) + i] = make_float2(static_cast<float>(cos(ang)), static_cast<float>(sin(ang)));
   }
-  grid_dep_launch();
+  trace_end(ts);
 }
 
+// One CTA per candidate: h = e_v, its per-tile sums of squares, and x.
 __global__ void embed_norm_kernel(const __nv_bfloat16* __restrict__ e_v, const __nv_bfloat16* __restrict__ gain,
-                                  int d, float eps, float* __restrict__ h, HiLo x) {
+                                  int d, float eps, int n_cand, float* __restrict__ h, float* __restrict__ sumsq,
+                                  HiLo x, unsigned long long* ts) {
+  trace_begin(ts);
   __shared__ float red[32];
+  grid_dep_launch();
   grid_dep_wait();
   const int b = blockIdx.x;
   float ss = 0.f;
@@ -61,106 +80,62 @@ __global__ void embed_norm_kernel(const __nv_bfloat16* __restrict__ e_v, const _
     h[static_cast<int64_t>(b) * d + c] = v;
     ss += v * v;
   }
-  const float r = 1.0f / sqrtf(block_sum(ss, red) / d + eps);
+  const float total = block_sum(ss, red);
+  // per-tile partial sums, as the residual GEMM epilogue writes them (only their sum is used)
+  const int m_tiles = (d + 127) / 128;
+  if (threadIdx.x < m_tiles) {
+    float t = 0.f;
+    for (int c = threadIdx.x * 128; c < min(d, threadIdx.x * 128 + 128); ++c) {
+      const float v = __bfloat162float(e_v[c]);
+      t += v * v;
+    }
+    sumsq[static_cast<int64_t>(threadIdx.x) * n_cand + b] = t;
+  }
+  const float r = 1.0f / sqrtf(total / d + eps);
   for (int c = threadIdx.x; c < d; c += blockDim.x)
     store_hilo(x, static_cast<int64_t>(b) * d + c, __bfloat162float(e_v[c]) * r * __bfloat162float(gain[c]));
-  grid_dep_launch();
+  trace_end(ts);
 }
 
-__global__ void qkv_post_kernel(const float* __restrict__ part, int splits, int n_cand, int M, int n_q, int n_kv,
-                                int hd, const float2* __restrict__ rope, float* __restrict__ q, HiLo qp,
-                                float* __restrict__ kself, float* __restrict__ vself) {
-  grid_dep_wait();
-  const int hs = blockIdx.x, b = blockIdx.y, i = threadIdx.x, half = hd / 2;
-  if (i < half) {
-    const int64_t base = static_cast<int64_t>(b) * M + static_cast<int64_t>(hs) * hd;
-    const int64_t sstride = static_cast<int64_t>(n_cand) * M;
-    float a = 0.f, c = 0.f;
-    for (int s = 0; s < splits; ++s) {
-      a += part[s * sstride + base + i];
-      c += part[s * sstride + base + i + half];
-    }
-    if (hs < n_q + n_kv) {   // rotate-half RoPE for q and k at p = L_b
-      const float2 cs = rope[b * half + i];
-      const float a2 = a * cs.x - c * cs.y;
-      const float c2 = c * cs.x + a * cs.y;
-      a = a2;
-      c = c2;
-    }
-    if (hs < n_q) {
-      const int64_t o = (static_cast<int64_t>(b) * n_q + hs) * hd;
-      q[o + i] = a;
-      q[o + i + half] = c;
-      store_hilo(qp, o + i, a);
-      store_hilo(qp, o + i + half, c);
-    } else {
-      float* dst = hs < n_q + n_kv ? kself + (static_cast<int64_t>(b) * n_kv + (hs - n_q)) * hd
-                                   : vself + (static_cast<int64_t>(b) * n_kv + (hs - n_q - n_kv)) * hd;
-      dst[i] = a;
-      dst[i + half] = c;
-    }
-  }
+// grid (n_cand, ceil(d / blockDim)): elementwise RMSNorm from the tile sums.
+__global__ void norm_kernel(const float* __restrict__ h, const float* __restrict__ sumsq, int m_tiles, int n_cand,
+                            int d, float eps, const __nv_bfloat16* __restrict__ gain, HiLo x,
+                            unsigned long long* ts) {
+  trace_begin(ts);
+  __shared__ float slot;
   grid_dep_launch();
-}
-
-__global__ void resid_norm_kernel(const float* __restrict__ part, int splits, int n_cand, int d, float eps,
-                                  float* __restrict__ h, const __nv_bfloat16* __restrict__ gain, HiLo x,
-                                  const __nv_bfloat16* __restrict__ w_plus,
-                                  const __nv_bfloat16* __restrict__ w_minus, float* __restrict__ rewards) {
-  __shared__ float red[32];
   grid_dep_wait();
   const int b = blockIdx.x;
-  float* hb = h + static_cast<int64_t>(b) * d;
-  const int64_t sstride = static_cast<int64_t>(n_cand) * d;
-  float ss = 0.f;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) {
-    float v = hb[c];
-    for (int s = 0; s < splits; ++s) v += part[s * sstride + static_cast<int64_t>(b) * d + c];
-    hb[c] = v;
-    ss += v * v;
+  const float r = row_rscale(sumsq, m_tiles, n_cand, b, d, eps, &slot);
+  const int c = blockIdx.y * blockDim.x + threadIdx.x;
+  if (c < d) {
+    const int64_t i = static_cast<int64_t>(b) * d + c;
+    store_hilo(x, i, h[i] * r * __bfloat162float(gain[c]));
   }
-  const float r = 1.0f / sqrtf(block_sum(ss, red) / d + eps);
-  if (w_plus == nullptr) {
-    for (int c = threadIdx.x; c < d; c += blockDim.x)
-      store_hilo(x, static_cast<int64_t>(b) * d + c, hb[c] * r * __bfloat162float(gain[c]));
-  } else {
-    float zp = 0.f, zm = 0.f;
-    for (int c = threadIdx.x; c < d; c += blockDim.x) {
-      const float xf = hb[c] * r * __bfloat162float(gain[c]);
-      zp += xf * __bfloat162float(w_plus[c]);
-      zm += xf * __bfloat162float(w_minus[c]);
-    }
-    zp = block_sum(zp, red);
-    zm = block_sum(zm, red);
-    if (threadIdx.x == 0) rewards[b] = 1.0f / (1.0f + expf(zm - zp));
-  }
-  grid_dep_launch();
+  trace_end(ts);
 }
 
-__global__ void silu_mul_kernel(const float* __restrict__ part, int splits, int n_cand, int ff, HiLo a) {
+__global__ void head_kernel(const float* __restrict__ h, const float* __restrict__ sumsq, int m_tiles, int n_cand,
+                            int d, float eps, const __nv_bfloat16* __restrict__ gain,
+                            const __nv_bfloat16* __restrict__ w_plus, const __nv_bfloat16* __restrict__ w_minus,
+                            float* __restrict__ rewards, unsigned long long* ts) {
+  trace_begin(ts);
+  __shared__ float red[32];
+  __shared__ float slot;
+  grid_dep_launch();
   grid_dep_wait();
-  const int64_t total = static_cast<int64_t>(n_cand) * ff;
-  const int64_t sstride = total * 2;
-  for (int64_t idx = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; idx < total;
-       idx += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int64_t b = idx / ff, j = idx - b * ff;
-    float g = 0.f, u = 0.f;
-    for (int s = 0; s < splits; ++s) {
-      g += part[s * sstride + b * 2 * ff + j];
-      u += part[s * sstride + b * 2 * ff + ff + j];
-    }
-    store_hilo(a, idx, g / (1.0f + expf(-g)) * u);
+  const int b = blockIdx.x;
+  const float r = row_rscale(sumsq, m_tiles, n_cand, b, d, eps, &slot);
+  float zp = 0.f, zm = 0.f;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    const float xf = h[static_cast<int64_t>(b) * d + c] * r * __bfloat162float(gain[c]);
+    zp += xf * __bfloat162float(w_plus[c]);
+    zm += xf * __bfloat162float(w_minus[c]);
   }
-  grid_dep_launch();
-}
-
-__global__ void split_sum_kernel(const float* __restrict__ part, int splits, int64_t count, float* __restrict__ out) {
-  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < count;
-       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    float v = 0.f;
-    for (int s = 0; s < splits; ++s) v += part[s * count + i];
-    out[i] = v;
-  }
+  zp = block_sum(zp, red);
+  zm = block_sum(zm, red);
+  if (threadIdx.x == 0) rewards[b] = 1.0f / (1.0f + expf(zm - zp));
+  trace_end(ts);
 }
 
 __global__ void split_hilo_kernel(const float* __restrict__ in, int64_t count, HiLo out) {
@@ -185,34 +160,35 @@ cudaLaunchConfig_t make_cfg(dim3 grid, dim3 block, cudaStream_t st, cudaLaunchAt
 }  // namespace
 
 cudaError_t launch_rope_table(const int32_t* seq_lens, int n_cand, int hd, double base, float2* table,
-                              cudaStream_t stream, bool pdl) {
+                              cudaStream_t stream, bool pdl, unsigned long long* ts) {
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = make_cfg(dim3(n_cand), dim3(64), stream, attr, pdl);
-  return cudaLaunchKernelEx(&cfg, rope_table_kernel, seq_lens, hd, base, table);
+  return cudaLaunchKernelEx(&cfg, rope_table_kernel, seq_lens, hd, base, table, ts);
 }
 
 cudaError_t launch_embed_norm(const ModelDims& m, const __nv_bfloat16* e_v, const __nv_bfloat16* gain, int n_cand,
-                              float* h, HiLo x, cudaStream_t stream, bool pdl) {
+                              float* h, float* sumsq, HiLo x, cudaStream_t stream, bool pdl,
+                              unsigned long long* ts) {
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = make_cfg(dim3(n_cand), dim3(256), stream, attr, pdl);
-  return cudaLaunchKernelEx(&cfg, embed_norm_kernel, e_v, gain, m.d, m.eps, h, x);
+  return cudaLaunchKernelEx(&cfg, embed_norm_kernel, e_v, gain, m.d, m.eps, n_cand, h, sumsq, x, ts);
 }
 
-cudaError_t launch_qkv_post(const ModelDims& m, const float* part, int splits, int n_cand, const float2* rope,
-                            float* q, HiLo qp, float* kself, float* vself, cudaStream_t stream, bool pdl) {
+cudaError_t launch_norm(const ModelDims& m, const float* h, const float* sumsq, int m_tiles, int n_cand,
+                        const __nv_bfloat16* gain, HiLo x, cudaStream_t stream, bool pdl, unsigned long long* ts) {
   cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = make_cfg(dim3(m.n_q + 2 * m.n_kv, n_cand), dim3(64), stream, attr, pdl);
-  return cudaLaunchKernelEx(&cfg, qkv_post_kernel, part, splits, n_cand, m.qkv_rows, m.n_q, m.n_kv, m.hd, rope, q,
-                            qp, kself, vself);
+  const int threads = 256;
+  cudaLaunchConfig_t cfg = make_cfg(dim3(n_cand, (m.d + threads - 1) / threads), dim3(threads), stream, attr, pdl);
+  return cudaLaunchKernelEx(&cfg, norm_kernel, h, sumsq, m_tiles, n_cand, m.d, m.eps, gain, x, ts);
 }
 
-cudaError_t launch_resid_norm(const ModelDims& m, const float* part, int splits, int n_cand, float* h,
-                              const __nv_bfloat16* gain, HiLo x, const __nv_bfloat16* w_plus,
-                              const __nv_bfloat16* w_minus, float* rewards, cudaStream_t stream, bool pdl) {
+cudaError_t launch_head(const ModelDims& m, const float* h, const float* sumsq, int m_tiles, int n_cand,
+                        const __nv_bfloat16* gain, const __nv_bfloat16* w_plus, const __nv_bfloat16* w_minus,
+                        float* rewards, cudaStream_t stream, bool pdl, unsigned long long* ts) {
   cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = make_cfg(dim3(n_cand), dim3(512), stream, attr, pdl);
-  return cudaLaunchKernelEx(&cfg, resid_norm_kernel, part, splits, n_cand, m.d, m.eps, h, gain, x, w_plus, w_minus,
-                            rewards);
+  cudaLaunchConfig_t cfg = make_cfg(dim3(n_cand), dim3(256), stream, attr, pdl);
+  return cudaLaunchKernelEx(&cfg, head_kernel, h, sumsq, m_tiles, n_cand, m.d, m.eps, gain, w_plus, w_minus,
+                            rewards, ts);
 }
 
 cudaError_t launch_split_hilo(const float* in, int64_t count, HiLo out, cudaStream_t stream) {
@@ -221,24 +197,6 @@ cudaError_t launch_split_hilo(const float* in, int64_t count, HiLo out, cudaStre
   if (blocks < 1) blocks = 1;
   split_hilo_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(in, count, out);
   return cudaGetLastError();
-}
-
-cudaError_t launch_split_sum(const float* part, int splits, int64_t count, float* out, cudaStream_t stream) {
-  int64_t blocks = (count + 255) / 256;
-  if (blocks > 152 * 8) blocks = 152 * 8;
-  if (blocks < 1) blocks = 1;
-  split_sum_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(part, splits, count, out);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_silu_mul(const ModelDims& m, const float* part, int splits, int n_cand, HiLo a,
-                            cudaStream_t stream, bool pdl) {
-  cudaLaunchAttribute attr[1];
-  const int64_t total = static_cast<int64_t>(n_cand) * m.ff;
-  int64_t blocks = (total + 255) / 256;
-  if (blocks > 152 * 8) blocks = 152 * 8;
-  cudaLaunchConfig_t cfg = make_cfg(dim3(static_cast<unsigned>(blocks)), dim3(256), stream, attr, pdl);
-  return cudaLaunchKernelEx(&cfg, silu_mul_kernel, part, splits, n_cand, m.ff, a);
 }
 
 }  // namespace kvprm

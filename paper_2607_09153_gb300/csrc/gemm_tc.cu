@@ -1,20 +1,29 @@
-// Projection GEMM for the verify token, batched over candidates (the
-// c_ffn * d^2 term of Eq. cost_kv): part[s][n][m] = sum_{k in split s} W[m][k] * X[n][k].
-//
-// The activation X arrives as a pair of bf16 tensors (hi, lo) with
-// X = hi + lo to ~2^-17 relative: each K step issues two MMAs (W*hi, W*lo)
-// into the same fp32 accumulator, so the contraction sees the fp32
-// activation, not a bf16 rounding of it (the weights are bf16 by definition).
+// Projection GEMMs of the verify-token forward, batched over candidates (the
+// c_ffn * d^2 term of Eq. cost_kv): Y[n][m] = sum_k W[m][k] * X[n][k].
 //
 // The weight matrix is the streamed operand (read once from HBM per call), so
 // it is the MMA's A operand: M = 128 weight rows per CTA, N = the candidate
 // batch padded to a multiple of 16 (16..256), K in 64-element tiles.  A
 // producer thread streams W and X tiles with TMA (128-byte swizzle) through a
 // multi-stage mbarrier ring; one thread issues tcgen05.mma (kind::f16, bf16 x
-// bf16 -> fp32) into a TMEM accumulator; four warps read TMEM back with
-// tcgen05.ld and store fp32 split-K partials.  K is split across CTAs so that
-// every SM streams weights; the consumer kernel reduces the splits in a fixed
-// order (deterministic, no float atomics) fused with its own epilogue.
+// bf16 -> fp32) into a TMEM accumulator.  The activation X arrives as a bf16
+// (hi, lo) pair, X = hi + lo to ~2^-17 relative, and each K step issues two
+// MMAs (W*hi, W*lo) into the same accumulator, so the contraction sees the
+// fp32 activation (the weights are bf16 by definition).
+//
+// K is split across the CTAs of a thread-block cluster (one cluster per
+// 128-row tile) so that every SM streams weights.  The splits are reduced
+// inside the cluster through distributed shared memory in rank order
+// (deterministic, no float atomics): each CTA parks its accumulator in its own
+// shared memory, and CTA r sums the candidate columns [r*N/cs, (r+1)*N/cs)
+// over all ranks and applies the epilogue of the step:
+//   PLAIN  out[n][m] = y
+//   QKV    RoPE on the q and k rows (rotate-half pairs inside a head) -> q
+//          (fp32 and bf16 hi/lo), self k, self v (fp32)
+//   RESID  h[n][m] += y, and the tile's sum of squares of the new h per
+//          candidate (the next RMSNorm reads these partial sums)
+//   SILU   rows are 64 gate rows and the matching 64 up rows (two TMA boxes
+//          per stage); a = SiLU(gate) * up as a bf16 hi/lo pair
 #include "kernels.h"
 #include "ptx.cuh"
 
@@ -30,26 +39,54 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~static_cast<uintptr_t>(1023));
 }
 
-__global__ void __launch_bounds__(128) gemm_wstream_kernel(const __grid_constant__ CUtensorMap tmW,
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Load a float at the same shared-memory offset in cluster CTA `rank`.
+__device__ __forceinline__ float ld_peer(const float* local, uint32_t rank) {
+  uint32_t a;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(smem_u32(local)), "r"(rank));
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(a) : "memory");
+  return v;
+}
+__device__ __forceinline__ void store_hilo(__nv_bfloat16* hi, __nv_bfloat16* lo, int64_t i, float x) {
+  const __nv_bfloat16 h = __float2bfloat16_rn(x);
+  hi[i] = h;
+  lo[i] = __float2bfloat16_rn(x - __bfloat162float(h));
+}
+
+__global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant__ CUtensorMap tmW,
                                                            const __grid_constant__ CUtensorMap tmX,
                                                            const __grid_constant__ CUtensorMap tmXlo, int has_lo,
-                                                           float* __restrict__ part, int M, int n_valid, int n_pad,
-                                                           int k_tiles, int kt_per_split, int stages,
-                                                           uint32_t tmem_cols, int* err) {
+                                                           int k_tiles, int cs, int stages, uint32_t tmem_cols,
+                                                           int n_pad, GemmEpilogue ep, int* err, unsigned long long* ts) {
+  trace_begin(ts);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
   const uint32_t x_bytes = static_cast<uint32_t>(n_pad) * kBK * 2;
   const uint32_t stage_bytes = kWTileBytes + x_bytes * (has_lo ? 2u : 1u);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + stages * stage_bytes);
+  const uint32_t acc_bytes = static_cast<uint32_t>(n_pad) * kBM * 4;
+  const uint32_t ring_bytes = stages * stage_bytes > acc_bytes ? stages * stage_bytes : acc_bytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + ring_bytes);
   uint64_t* empty = full + stages;
   uint64_t* done = empty + stages;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
+  float* red = reinterpret_cast<float*>(tmem_slot + 4);   // 64 floats for per-column block sums
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m_tile = blockIdx.x, split = blockIdx.y;
-  const int kt0 = split * kt_per_split;
-  const int kt1 = min(k_tiles, kt0 + kt_per_split);
-  const int nk = kt1 - kt0;
+  const int m_tile = blockIdx.x / cs;
+  const uint32_t rank = cluster_rank();
+  const int kps = (k_tiles + cs - 1) / cs;
+  const int kt0 = static_cast<int>(rank) * kps;
+  const int kt1 = min(k_tiles, kt0 + kps);
+  const int nk = kt1 > kt0 ? kt1 - kt0 : 0;
+  const bool silu = ep.mode == GemmEpilogue::SILU;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < stages; ++s) {
@@ -70,18 +107,29 @@ __global__ void __launch_bounds__(128) gemm_wstream_kernel(const __grid_constant
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // Let the next kernel in the stream start its own independent prologue and
+  // streaming now; it waits for this grid's completion before touching what
+  // this grid writes.
+  grid_dep_launch();
 
-  if (warp == 0 && lane == 0) {
+  if (warp == 0 && lane == 0 && nk > 0) {
     // ---------------- TMA producer
     const uint64_t pol_w = policy_evict_first();
     const uint64_t pol_x = policy_evict_last();
+    auto load_w = [&](uint8_t* st, int kt, uint64_t* bar) {
+      if (!silu) {
+        tma_load_2d(st, &tmW, bar, kt * kBK, m_tile * kBM, pol_w);
+      } else {   // 64 gate rows, then the matching 64 up rows
+        tma_load_2d(st, &tmW, bar, kt * kBK, m_tile * 64, pol_w);
+        tma_load_2d(st + kWTileBytes / 2, &tmW, bar, kt * kBK, ep.ff + m_tile * 64, pol_w);
+      }
+    };
     // Weights do not depend on the preceding kernel: start streaming the first
     // ring's worth of W before waiting for the activations it produces.
     const int pre = min(stages, nk);
     for (int i = 0; i < pre; ++i) {
-      uint8_t* st = smem + i * stage_bytes;
       mbar_arrive_expect_tx(&full[i], stage_bytes);
-      tma_load_2d(st, &tmW, &full[i], (kt0 + i) * kBK, m_tile * kBM, pol_w);
+      load_w(smem + i * stage_bytes, kt0 + i, &full[i]);
     }
     grid_dep_wait();
     for (int i = 0; i < pre; ++i) {
@@ -95,21 +143,17 @@ __global__ void __launch_bounds__(128) gemm_wstream_kernel(const __grid_constant
       if (!mbar_wait(&empty[s], (use & 1u) ^ 1u, err)) break;
       uint8_t* st = smem + s * stage_bytes;
       mbar_arrive_expect_tx(&full[s], stage_bytes);
-      tma_load_2d(st, &tmW, &full[s], (kt0 + i) * kBK, m_tile * kBM, pol_w);
+      load_w(st, kt0 + i, &full[s]);
       tma_load_2d(st + kWTileBytes, &tmX, &full[s], (kt0 + i) * kBK, 0, pol_x);
       if (has_lo) tma_load_2d(st + kWTileBytes + x_bytes, &tmXlo, &full[s], (kt0 + i) * kBK, 0, pol_x);
     }
-  } else if (warp == 1 && lane == 0) {
+  } else if (warp == 1 && lane == 0 && nk > 0) {
     // ---------------- MMA issuer
     const uint32_t idesc = idesc_bf16_f32(kBM, n_pad);
-    bool ok = true;
-    for (int i = 0; i < nk && ok; ++i) {
+    for (int i = 0; i < nk; ++i) {
       const int s = i % stages;
       const uint32_t use = static_cast<uint32_t>(i / stages);
-      if (!mbar_wait(&full[s], use & 1u, err)) {
-        ok = false;
-        break;
-      }
+      if (!mbar_wait(&full[s], use & 1u, err)) break;
       tc_fence_after();
       const uint32_t a_base = smem_u32(smem + s * stage_bytes);
       const uint32_t b_base = a_base + kWTileBytes;
@@ -125,46 +169,168 @@ __global__ void __launch_bounds__(128) gemm_wstream_kernel(const __grid_constant
   }
   __syncwarp();
 
-  // ---------------- epilogue: TMEM -> registers -> fp32 partials
-  const bool have = __all_sync(0xffffffffu, mbar_wait(done, 0, err));   // also reconverges the warp
+  // ---------------- accumulator -> own shared memory, acc[c][m] (fp32, c < n_pad, m < 128)
+  const bool have = nk > 0 ? __all_sync(0xffffffffu, mbar_wait(done, 0, err)) : true;
   tc_fence_after();
-  grid_dep_launch();
-  grid_dep_wait();
-  const int m = m_tile * kBM + warp * 32 + lane;
-  if (have && nk > 0) {
-    float* out = part + static_cast<size_t>(split) * n_valid * M;
-    for (int c0 = 0; c0 < n_pad; c0 += 16) {
-      float v[16];
+  float* acc = reinterpret_cast<float*>(smem);   // the ring is idle once `done` has fired
+  const int m = warp * 32 + lane;
+  for (int c0 = 0; c0 < n_pad; c0 += 16) {
+    float v[16];
+    if (nk > 0 && have) {
       tmem_ld16(tmem + (static_cast<uint32_t>(warp * 32) << 16) + static_cast<uint32_t>(c0), v);
-      if (m < M) {
+    } else {
 #pragma unroll
-        for (int j = 0; j < 16; ++j)
-          if (c0 + j < n_valid) out[static_cast<size_t>(c0 + j) * M + m] = v[j];
+      for (int j = 0; j < 16; ++j) v[j] = 0.f;
+    }
+#pragma unroll
+    for (int j = 0; j < 16; ++j) acc[(c0 + j) * kBM + m] = v[j];
+  }
+  tc_fence_before();
+  cluster_sync();   // every rank's partial is parked
+
+  // ---------------- reduce this rank's candidate columns over the cluster, then the epilogue
+  grid_dep_wait();   // outputs may still be read by kernels that precede this one
+  const int cols = n_pad / cs;
+  const int cbeg = static_cast<int>(rank) * cols;
+  const int cend = min(cbeg + cols, ep.n_valid);
+  const int nc = cend > cbeg ? cend - cbeg : 0;
+  // Step 1: acc[c][m] <- sum over ranks of acc_r[c][m] for this rank's columns
+  // (only this rank reads them, so it may overwrite its own copy).  Two columns
+  // per round trip when the cluster has <= 8 ranks, all peer loads in flight.
+  {
+    const int step = cs <= 8 ? 2 : 1;
+    for (int c = cbeg; c < cend; c += step) {
+      const bool two = step == 2 && c + 1 < cend;
+      float v[16];
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        const int r = step == 2 ? (k & 7) : k;
+        const int cc = (step == 2 && k >= 8) ? c + 1 : c;
+        const bool use = r < cs && (cc == c || two);
+        v[k] = use ? ld_peer(acc + cc * kBM + m, static_cast<uint32_t>(r)) : 0.f;
+      }
+      if (step == 2) {
+        float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          s0 += v[k];
+          s1 += v[8 + k];
+        }
+        __syncwarp();
+        acc[c * kBM + m] = s0;
+        if (two) acc[(c + 1) * kBM + m] = s1;
+      } else {
+        float s0 = 0.f;
+#pragma unroll
+        for (int k = 0; k < 16; ++k) s0 += v[k];
+        acc[c * kBM + m] = s0;
       }
     }
   }
-  tc_fence_before();
   __syncthreads();
+  // Step 2: the epilogue over (row, column) pairs, all threads in parallel
+  if (ep.mode == GemmEpilogue::PLAIN) {
+    const int gm = m_tile * kBM + m;
+    if (gm < ep.M)
+      for (int c = cbeg; c < cend; ++c) ep.out[static_cast<int64_t>(c) * ep.M + gm] = acc[c * kBM + m];
+  } else if (ep.mode == GemmEpilogue::RESID) {
+    const int gm = m_tile * kBM + m;
+    float* sq_s = red;   // [16 columns][4 warps]
+    for (int c0 = cbeg; c0 < cend; c0 += 16) {
+      const int c1 = min(cend, c0 + 16);
+      for (int c = c0; c < c1; ++c) {
+        float hv = 0.f;
+        if (gm < ep.M) {
+          float* hp = ep.h + static_cast<int64_t>(c) * ep.M + gm;
+          hv = *hp + acc[c * kBM + m];
+          *hp = hv;
+        }
+        float sq = hv * hv;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
+        if (lane == 0) sq_s[(c - c0) * 4 + warp] = sq;
+      }
+      __syncthreads();
+      if (threadIdx.x < c1 - c0) {
+        const float* q4 = sq_s + threadIdx.x * 4;
+        ep.sumsq[static_cast<int64_t>(m_tile) * ep.n_valid + c0 + threadIdx.x] = (q4[0] + q4[1]) + (q4[2] + q4[3]);
+      }
+      __syncthreads();
+    }
+  } else if (ep.mode == GemmEpilogue::SILU) {
+    const int r = m & 63, half_sel = m >> 6;   // two column groups of 64 threads
+    const int j = m_tile * 64 + r;
+    if (j < ep.ff)
+      for (int c = cbeg + half_sel; c < cend; c += 2) {
+        const float g = acc[c * kBM + r], u = acc[c * kBM + 64 + r];
+        store_hilo(ep.a_hi, ep.a_lo, static_cast<int64_t>(c) * ep.ff + j, g / (1.0f + expf(-g)) * u);
+      }
+  } else {   // QKV: pair p = m & 63 of this tile, two column groups of 64 threads
+    const int p = m & 63, half_sel = m >> 6;
+    const int hd = ep.hd, half = hd / 2;
+    const int row_a = (p / half) * hd + (p % half);   // first element of the pair, within the tile
+    const int row_b = row_a + half;
+    const int grow = m_tile * kBM + row_a;              // row of W_qkv
+    const int head = grow / hd, i = grow % hd;          // i < half
+    for (int c = cbeg + half_sel; c < cend; c += 2) {
+      float a = acc[c * kBM + row_a], b = acc[c * kBM + row_b];
+      if (head < ep.n_q + ep.n_kv) {
+        const float2 cs2 = ep.rope[c * half + i];
+        const float a2 = a * cs2.x - b * cs2.y;
+        const float b2 = b * cs2.x + a * cs2.y;
+        a = a2;
+        b = b2;
+      }
+      if (head < ep.n_q) {
+        const int64_t o = (static_cast<int64_t>(c) * ep.n_q + head) * hd + i;
+        ep.q[o] = a;
+        ep.q[o + half] = b;
+        store_hilo(ep.q_hi, ep.q_lo, o, a);
+        store_hilo(ep.q_hi, ep.q_lo, o + half, b);
+      } else if (head < ep.n_q + 2 * ep.n_kv) {
+        const bool is_k = head < ep.n_q + ep.n_kv;
+        const int kvh = is_k ? head - ep.n_q : head - ep.n_q - ep.n_kv;
+        float* dst = (is_k ? ep.kself : ep.vself) + (static_cast<int64_t>(c) * ep.n_kv + kvh) * hd + i;
+        dst[0] = a;
+        dst[half] = b;
+      }
+    }
+  }
+  (void)nc;
+  cluster_sync();   // peers have finished reading this CTA's partial
   if (warp == 1) tmem_dealloc(tmem, tmem_cols);
+  trace_end(ts);
 }
 
 }  // namespace
 
-GemmPlan plan_gemm(int M, int K, int n_pad, int num_sms, bool has_lo) {
+GemmPlan plan_gemm(int M, int K, int n_pad, int num_sms, bool has_lo, bool gate_up) {
   GemmPlan p;
   p.has_lo = has_lo;
-  p.m_tiles = (M + kBM - 1) / kBM;
+  p.gate_up = gate_up;
+  p.m_tiles = gate_up ? (M + 63) / 64 : (M + kBM - 1) / kBM;   // gate/up: M = d_ff, 64 pairs per tile
   p.k_tiles = (K + kBK - 1) / kBK;
   const uint32_t stage_bytes = kWTileBytes + static_cast<uint32_t>(n_pad) * kBK * 2 * (has_lo ? 2u : 1u);
   int stages = static_cast<int>((112u * 1024u) / stage_bytes);
   p.stages = stages < 2 ? 2 : (stages > 8 ? 8 : stages);
-  p.smem_bytes = static_cast<size_t>(p.stages) * stage_bytes + 1024 /*align*/ + 256 /*barriers*/;
-  const int target = 2 * num_sms;
-  int s = target / p.m_tiles;
-  if (s < 1) s = 1;
-  if (s > p.k_tiles) s = p.k_tiles;
-  p.kt_per_split = (p.k_tiles + s - 1) / s;
-  p.splits = (p.k_tiles + p.kt_per_split - 1) / p.kt_per_split;
+  // the parked accumulator (n_pad x 128 fp32) reuses the ring
+  size_t ring = static_cast<size_t>(p.stages) * stage_bytes;
+  const size_t acc = static_cast<size_t>(n_pad) * kBM * 4;
+  if (ring < acc) ring = acc;
+  p.smem_bytes = ring + 1024 /*align*/ + 512 /*barriers, TMEM slot, block sums*/;
+  // cluster size: the largest power of two <= 16 that keeps the CTA count within
+  // two per SM and gives every rank at least two K tiles
+  int cs = 1;
+  while (cs < 16 && p.m_tiles * cs * 2 <= 2 * num_sms && cs * 4 <= p.k_tiles && cs * 2 <= n_pad) cs *= 2;
+  p.cluster = cs;
+  p.splits = cs;
+  p.kt_per_split = (p.k_tiles + cs - 1) / cs;
+  // a ring deeper than the K tiles one CTA streams only holds shared memory
+  // that overlapping kernels could use
+  if (p.stages > p.kt_per_split) p.stages = p.kt_per_split < 2 ? 2 : p.kt_per_split;
+  ring = static_cast<size_t>(p.stages) * stage_bytes;
+  if (ring < acc) ring = acc;
+  p.smem_bytes = ring + 1024 /*align*/ + 512 /*barriers, TMEM slot, block sums*/;
   uint32_t cols = 32;
   while (cols < static_cast<uint32_t>(n_pad)) cols <<= 1;
   p.tmem_cols = cols;
@@ -172,23 +338,30 @@ GemmPlan plan_gemm(int M, int K, int n_pad, int num_sms, bool has_lo) {
 }
 
 cudaError_t gemm_configure() {
-  return cudaFuncSetAttribute(gemm_wstream_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+  cudaError_t e = cudaFuncSetAttribute(gemm_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(gemm_cluster_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
 }
 
 cudaError_t launch_gemm(const GemmPlan& p, const CUtensorMap* tmW, const CUtensorMap* tmX, const CUtensorMap* tmXlo,
-                        float* part, int M, int n_valid, int n_pad, int* err, cudaStream_t stream, bool pdl) {
+                        const GemmEpilogue& ep, int n_pad, int* err, cudaStream_t stream, bool pdl,
+                        unsigned long long* ts) {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(p.m_tiles, p.splits, 1);
+  cfg.gridDim = dim3(p.m_tiles * p.cluster, 1, 1);
   cfg.blockDim = dim3(128, 1, 1);
   cfg.dynamicSmemBytes = p.smem_bytes;
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = p.cluster;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, gemm_wstream_kernel, *tmW, *tmX, p.has_lo ? *tmXlo : *tmX, p.has_lo ? 1 : 0, part,
-                            M, n_valid, n_pad, p.k_tiles, p.kt_per_split, p.stages, p.tmem_cols, err);
+  cfg.numAttrs = pdl ? 2 : 1;
+  return cudaLaunchKernelEx(&cfg, gemm_cluster_kernel, *tmW, *tmX, p.has_lo ? *tmXlo : *tmX, p.has_lo ? 1 : 0,
+                            p.k_tiles, p.cluster, p.stages, p.tmem_cols, n_pad, ep, err, ts);
 }
 
 }  // namespace kvprm

@@ -34,12 +34,12 @@ struct CallPlan {
 };
 
 struct GraphKey {
-  int n = -1, n_pad = -1, n_split = -1, pps = -1, debug = -1, profile = -1, pdl = -1;
+  int n = -1, n_pad = -1, n_split = -1, pps = -1, debug = -1, profile = -1, pdl = -1, trace = -1;
   const void* pool = nullptr;
   int64_t n_pages = -1;
   bool operator==(const GraphKey& o) const {
     return n == o.n && n_pad == o.n_pad && n_split == o.n_split && pps == o.pps && debug == o.debug &&
-           profile == o.profile && pdl == o.pdl && pool == o.pool && n_pages == o.n_pages;
+           profile == o.profile && pdl == o.pdl && trace == o.trace && pool == o.pool && n_pages == o.n_pages;
   }
 };
 
@@ -64,11 +64,12 @@ struct kvprm_ctx {
   int npad_max = 16;
   float* h = nullptr;
   bf16 *xhi = nullptr, *xlo = nullptr, *ohi = nullptr, *olo = nullptr, *ahi = nullptr, *alo = nullptr;
-  float* part = nullptr;
-  size_t part_elems = 0;
+  float* sumsq = nullptr;   // [ceil(d / 128)][Bmax] per-tile sums of squares of h
+  int d_tiles = 0;
   float *q = nullptr, *kself = nullptr, *vself = nullptr;
   bf16 *qhi = nullptr, *qlo = nullptr;
   float *apart_o = nullptr, *apart_ml = nullptr;
+  int* attn_counter = nullptr;   // [Bmax][n_kv] split-arrival counters
   float2* rope = nullptr;
   int32_t* tables_d = nullptr;   // [Bmax] seq_lens, then [Bmax][max_blocks] block table
   float* rewards_d = nullptr;
@@ -98,10 +99,16 @@ struct kvprm_ctx {
   size_t dev_pool_bytes = 0;
   // graph replay
   cudaStream_t cap_stream = nullptr;
+
   bool use_graph = true, use_pdl = true;
   GraphKey gkey;
   cudaGraphExec_t gexec = nullptr;
   std::vector<ProfMark> graph_marks;
+  // device timeline trace of the last call: [slot][2] (see trace_begin / trace_end)
+  bool trace = false;
+  unsigned long long* trace_d = nullptr;
+  int trace_cap = 0, trace_n = 0;
+  std::vector<int> trace_cls;
   // profiling
   bool profile = false;
   std::vector<ProfMark> live_marks;   // marks recorded in the current (non-graph) capture
@@ -175,12 +182,14 @@ void free_ctx(kvprm_ctx* c) {
   cudaFree(c->alo);
   cudaFree(c->qhi);
   cudaFree(c->qlo);
-  cudaFree(c->part);
+  cudaFree(c->sumsq);
+  cudaFree(c->trace_d);
   cudaFree(c->q);
   cudaFree(c->kself);
   cudaFree(c->vself);
   cudaFree(c->apart_o);
   cudaFree(c->apart_ml);
+  cudaFree(c->attn_counter);
   cudaFree(c->rope);
   cudaFree(c->tables_d);
   cudaFree(c->rewards_d);
@@ -206,6 +215,7 @@ void free_ctx(kvprm_ctx* c) {
     cudaEventDestroy(m.b);
   }
   if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
+
   delete c;
 }
 
@@ -288,10 +298,10 @@ CallPlan make_plan(kvprm_ctx* ctx, int n, int max_pages) {
   p.n_pad = (n + 15) / 16 * 16;
   p.max_pages = max_pages;
   const ModelDims& m = ctx->md;
-  p.g_qkv = kvprm::plan_gemm(m.qkv_rows, m.d, p.n_pad, ctx->num_sms, true);
-  p.g_o = kvprm::plan_gemm(m.d, m.n_q * m.hd, p.n_pad, ctx->num_sms, true);
-  p.g_gu = kvprm::plan_gemm(2 * m.ff, m.d, p.n_pad, ctx->num_sms, true);
-  p.g_down = kvprm::plan_gemm(m.d, m.ff, p.n_pad, ctx->num_sms, true);
+  p.g_qkv = kvprm::plan_gemm(m.qkv_rows, m.d, p.n_pad, ctx->num_sms, true, false);
+  p.g_o = kvprm::plan_gemm(m.d, m.n_q * m.hd, p.n_pad, ctx->num_sms, true, false);
+  p.g_gu = kvprm::plan_gemm(m.ff, m.d, p.n_pad, ctx->num_sms, true, true);
+  p.g_down = kvprm::plan_gemm(m.d, m.ff, p.n_pad, ctx->num_sms, true, false);
   p.attn = kvprm::plan_attention(ctx->as, n, max_pages, ctx->num_sms, kSplitCap);
   return p;
 }
@@ -317,6 +327,11 @@ struct Enq {
     *ev_b = m.b;
     return KVPRM_OK;
   }
+  unsigned long long* trace_slot(int cls) {
+    if (!ctx->trace || ctx->trace_n >= ctx->trace_cap) return nullptr;
+    ctx->trace_cls.push_back(cls);
+    return ctx->trace_d + 2 * static_cast<size_t>(ctx->trace_n++);
+  }
   int end(cudaEvent_t ev_b) {
     if (!prof) return KVPRM_OK;
     CK(rec(ev_b), "cudaEventRecord");
@@ -326,6 +341,8 @@ struct Enq {
 
 #define LAUNCH(cls, expr, what)                    \
   do {                                             \
+    unsigned long long* TS = E.trace_slot(cls);    \
+    (void)TS;                                      \
     cudaEvent_t evb_ = nullptr;                    \
     int rc_ = E.begin(cls, &evb_);                 \
     if (rc_) return rc_;                           \
@@ -343,60 +360,78 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
   cudaStream_t st = E.st;
   const bool pdl = E.pdl;
   const int NL = ctx->cfg.n_layers;
-  const kvprm::HiLo X{ctx->xhi, ctx->xlo}, Q{ctx->qhi, ctx->qlo}, O{ctx->ohi, ctx->olo}, A{ctx->ahi, ctx->alo};
-  LAUNCH(KVPRM_PROF_FUSED, kvprm::launch_rope_table(sl, n, m.hd, ctx->cfg.rope_base, ctx->rope, st, false), "rope");
-  LAUNCH(KVPRM_PROF_FUSED, kvprm::launch_embed_norm(m, ctx->embed, ctx->attn_norm[0], n, ctx->h, X, st, pdl),
+  const kvprm::HiLo X{ctx->xhi, ctx->xlo}, O{ctx->ohi, ctx->olo};
+  kvprm::GemmEpilogue eq;   // QKV projection -> rotated q, self k / v
+  eq.mode = kvprm::GemmEpilogue::QKV;
+  eq.M = m.qkv_rows;
+  eq.n_valid = n;
+  eq.rope = ctx->rope;
+  eq.n_q = m.n_q;
+  eq.n_kv = m.n_kv;
+  eq.hd = m.hd;
+  eq.q = ctx->q;
+  eq.q_hi = ctx->qhi;
+  eq.q_lo = ctx->qlo;
+  eq.kself = ctx->kself;
+  eq.vself = ctx->vself;
+  kvprm::GemmEpilogue er;   // O and down projections -> residual stream + tile sums of squares
+  er.mode = kvprm::GemmEpilogue::RESID;
+  er.M = m.d;
+  er.n_valid = n;
+  er.h = ctx->h;
+  er.sumsq = ctx->sumsq;
+  kvprm::GemmEpilogue es;   // gate/up projection -> SiLU(gate) * up
+  es.mode = kvprm::GemmEpilogue::SILU;
+  es.M = m.ff;
+  es.n_valid = n;
+  es.ff = m.ff;
+  es.a_hi = ctx->ahi;
+  es.a_lo = ctx->alo;
+  ctx->trace_n = 0;
+  ctx->trace_cls.clear();
+  if (ctx->trace)
+    CK(cudaMemsetAsync(ctx->trace_d, 0xFF, sizeof(unsigned long long) * 2 * ctx->trace_cap, st), "trace reset");
+  CK(cudaMemsetAsync(ctx->attn_counter, 0, sizeof(int) * static_cast<size_t>(n) * m.n_kv, st), "counter reset");
+  LAUNCH(KVPRM_PROF_FUSED, kvprm::launch_rope_table(sl, n, m.hd, ctx->cfg.rope_base, ctx->rope, st, false, TS), "rope");
+  LAUNCH(KVPRM_PROF_FUSED,
+         kvprm::launch_embed_norm(m, ctx->embed, ctx->attn_norm[0], n, ctx->h, ctx->sumsq, X, st, pdl, TS),
          "embed_norm");
   for (int l = 0; l < NL; ++l) {
     LAUNCH(KVPRM_PROF_GEMM_QKV,
-           kvprm::launch_gemm(P.g_qkv, &ctx->tm_qkv[l], &ctx->tm_xhi, &ctx->tm_xlo, ctx->part, m.qkv_rows, n, np,
-                              ctx->err_d, st, pdl),
+           kvprm::launch_gemm(P.g_qkv, &ctx->tm_qkv[l], &ctx->tm_xhi, &ctx->tm_xlo, eq, np, ctx->err_d, st, pdl, TS),
            "gemm_qkv");
-    LAUNCH(KVPRM_PROF_FUSED,
-           kvprm::launch_qkv_post(m, ctx->part, P.g_qkv.splits, n, ctx->rope, ctx->q, Q, ctx->kself, ctx->vself, st,
-                                  pdl),
-           "qkv_post");
     if (ctx->debug_flags & 2) {
       const size_t nq = static_cast<size_t>(n) * m.n_q * m.hd, nk = static_cast<size_t>(n) * m.n_kv * m.hd;
       CK(cudaMemcpyAsync(ctx->dbg_q + l * nq, ctx->q, nq * 4, cudaMemcpyDeviceToDevice, st), "debug q");
       CK(cudaMemcpyAsync(ctx->dbg_k + l * nk, ctx->kself, nk * 4, cudaMemcpyDeviceToDevice, st), "debug k");
       CK(cudaMemcpyAsync(ctx->dbg_v + l * nk, ctx->vself, nk * 4, cudaMemcpyDeviceToDevice, st), "debug v");
     }
+    float* dbg = (ctx->debug_flags & 1) ? ctx->dbg + static_cast<size_t>(l) * n * m.n_q * m.hd : nullptr;
+    const kvprm::AttnMerge mg{ctx->q, ctx->kself, ctx->vself, ctx->attn_counter, O.hi, O.lo, nullptr, dbg};
     LAUNCH(KVPRM_PROF_ATTN,
            kvprm::launch_attn_split(ctx->as, P.attn, &ctx->tm_pool, l, bt, sl, ctx->qhi, ctx->qlo, n, ctx->apart_o,
-                                    ctx->apart_ml, ctx->err_d, st, pdl),
+                                    ctx->apart_ml, mg, ctx->err_d, st, pdl, TS),
            "attn_split");
-    float* dbg = (ctx->debug_flags & 1) ? ctx->dbg + static_cast<size_t>(l) * n * m.n_q * m.hd : nullptr;
-    LAUNCH(KVPRM_PROF_COMBINE,
-           kvprm::launch_attn_combine(ctx->as, P.attn, sl, ctx->q, ctx->kself, ctx->vself, ctx->apart_o,
-                                      ctx->apart_ml, n, O.hi, O.lo, nullptr, dbg, st, pdl),
-           "attn_combine");
     LAUNCH(KVPRM_PROF_GEMM_O,
-           kvprm::launch_gemm(P.g_o, &ctx->tm_o[l], &ctx->tm_ohi, &ctx->tm_olo, ctx->part, m.d, n, np, ctx->err_d, st,
-                              pdl),
+           kvprm::launch_gemm(P.g_o, &ctx->tm_o[l], &ctx->tm_ohi, &ctx->tm_olo, er, np, ctx->err_d, st, pdl, TS),
            "gemm_o");
     LAUNCH(KVPRM_PROF_FUSED,
-           kvprm::launch_resid_norm(m, ctx->part, P.g_o.splits, n, ctx->h, ctx->mlp_norm[l], X, nullptr, nullptr,
-                                    nullptr, st, pdl),
-           "resid_norm");
+           kvprm::launch_norm(m, ctx->h, ctx->sumsq, ctx->d_tiles, n, ctx->mlp_norm[l], X, st, pdl, TS),
+           "norm_mlp");
     LAUNCH(KVPRM_PROF_GEMM_GATE_UP,
-           kvprm::launch_gemm(P.g_gu, &ctx->tm_gu[l], &ctx->tm_xhi, &ctx->tm_xlo, ctx->part, 2 * m.ff, n, np,
-                              ctx->err_d, st, pdl),
+           kvprm::launch_gemm(P.g_gu, &ctx->tm_gu[l], &ctx->tm_xhi, &ctx->tm_xlo, es, np, ctx->err_d, st, pdl, TS),
            "gemm_gate_up");
-    LAUNCH(KVPRM_PROF_FUSED, kvprm::launch_silu_mul(m, ctx->part, P.g_gu.splits, n, A, st, pdl), "silu_mul");
     LAUNCH(KVPRM_PROF_GEMM_DOWN,
-           kvprm::launch_gemm(P.g_down, &ctx->tm_down[l], &ctx->tm_ahi, &ctx->tm_alo, ctx->part, m.d, n, np,
-                              ctx->err_d, st, pdl),
+           kvprm::launch_gemm(P.g_down, &ctx->tm_down[l], &ctx->tm_ahi, &ctx->tm_alo, er, np, ctx->err_d, st, pdl, TS),
            "gemm_down");
     if (l + 1 < NL) {
       LAUNCH(KVPRM_PROF_FUSED,
-             kvprm::launch_resid_norm(m, ctx->part, P.g_down.splits, n, ctx->h, ctx->attn_norm[l + 1], X, nullptr,
-                                      nullptr, nullptr, st, pdl),
-             "resid_norm");
+             kvprm::launch_norm(m, ctx->h, ctx->sumsq, ctx->d_tiles, n, ctx->attn_norm[l + 1], X, st, pdl, TS),
+             "norm_attn");
     } else {
       LAUNCH(KVPRM_PROF_FUSED,
-             kvprm::launch_resid_norm(m, ctx->part, P.g_down.splits, n, ctx->h, ctx->final_norm, X, ctx->w_plus,
-                                      ctx->w_minus, ctx->rewards_d, st, pdl),
+             kvprm::launch_head(m, ctx->h, ctx->sumsq, ctx->d_tiles, n, ctx->final_norm, ctx->w_plus, ctx->w_minus,
+                                ctx->rewards_d, st, pdl, TS),
              "reward_head");
     }
     if (ctx->debug_flags & 4) {
@@ -474,6 +509,7 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   key.debug = ctx->debug_flags;
   key.profile = ctx->profile ? 1 : 0;
   key.pdl = ctx->use_pdl ? 1 : 0;
+  key.trace = ctx->trace ? 1 : 0;
   key.pool = pool;
   key.n_pages = pages;
   if (!(ctx->gexec && key == ctx->gkey)) {
@@ -613,7 +649,7 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
     ctx->mlp_norm[l] = static_cast<const bf16*>(w->mlp_norm[l]);
     CREATE_CK(make_map(ctx, &ctx->tm_qkv[l], w->w_qkv[l], m.d, m.qkv_rows, 64, 128, "w_qkv"));
     CREATE_CK(make_map(ctx, &ctx->tm_o[l], w->w_o[l], static_cast<uint64_t>(m.n_q) * m.hd, m.d, 64, 128, "w_o"));
-    CREATE_CK(make_map(ctx, &ctx->tm_gu[l], w->w_gate_up[l], m.d, 2 * static_cast<uint64_t>(m.ff), 64, 128,
+    CREATE_CK(make_map(ctx, &ctx->tm_gu[l], w->w_gate_up[l], m.d, 2 * static_cast<uint64_t>(m.ff), 64, 64,
                        "w_gate_up"));
     CREATE_CK(make_map(ctx, &ctx->tm_down[l], w->w_down[l], m.ff, m.d, 64, 128, "w_down"));
   }
@@ -628,19 +664,8 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   CREATE_CK(dalloc(ctx, &ctx->olo, Bp * m.n_q * m.hd, "o_lo"));
   CREATE_CK(dalloc(ctx, &ctx->ahi, Bp * m.ff, "a_hi"));
   CREATE_CK(dalloc(ctx, &ctx->alo, Bp * m.ff, "a_lo"));
-  {
-    // split-K partials: splits * n * M, with splits <= max(1, 2*SMs / m_tiles) per GEMM
-    size_t need = 0;
-    const int shapes[4][2] = {{m.qkv_rows, m.d}, {m.d, m.n_q * m.hd}, {2 * m.ff, m.d}, {m.d, m.ff}};
-    for (int npad = 16; npad <= ctx->npad_max; npad += 16)
-      for (auto& s : shapes) {
-        GemmPlan g = kvprm::plan_gemm(s[0], s[1], npad, ctx->num_sms, true);
-        size_t e = static_cast<size_t>(g.splits) * Bmax * s[0];
-        if (e > need) need = e;
-      }
-    ctx->part_elems = need;
-    CREATE_CK(dalloc(ctx, &ctx->part, need, "gemm partials"));
-  }
+  ctx->d_tiles = (m.d + 127) / 128;
+  CREATE_CK(dalloc(ctx, &ctx->sumsq, static_cast<size_t>(ctx->d_tiles) * Bmax, "tile sums of squares"));
   CREATE_CK(dalloc(ctx, &ctx->q, static_cast<size_t>(Bmax) * m.n_q * m.hd, "q"));
   CREATE_CK(dalloc(ctx, &ctx->qhi, static_cast<size_t>(Bmax) * m.n_q * m.hd, "q_hi"));
   CREATE_CK(dalloc(ctx, &ctx->qlo, static_cast<size_t>(Bmax) * m.n_q * m.hd, "q_lo"));
@@ -648,6 +673,7 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   CREATE_CK(dalloc(ctx, &ctx->vself, static_cast<size_t>(Bmax) * m.n_kv * m.hd, "v_self"));
   CREATE_CK(dalloc(ctx, &ctx->apart_o, static_cast<size_t>(Bmax) * m.n_q * kSplitCap * m.hd, "attn partials"));
   CREATE_CK(dalloc(ctx, &ctx->apart_ml, static_cast<size_t>(Bmax) * m.n_q * kSplitCap * 2, "attn stats"));
+  CREATE_CK(dalloc(ctx, &ctx->attn_counter, static_cast<size_t>(Bmax) * m.n_kv, "attn counters"));
   CREATE_CK(dalloc(ctx, &ctx->rope, static_cast<size_t>(Bmax) * (m.hd / 2), "rope table"));
   CREATE_CK(dalloc(ctx, &ctx->tables_d, static_cast<size_t>(Bmax) * (1 + c.max_blocks_per_seq), "tables"));
   CREATE_CK(dalloc(ctx, &ctx->rewards_d, static_cast<size_t>(Bmax), "rewards"));
@@ -771,15 +797,13 @@ int kvprm_attention(kvprm_ctx* ctx, const void* kv_layer, int64_t n_pages, const
          kvprm::launch_split_hilo(static_cast<const float*>(q), static_cast<int64_t>(n) * ctx->md.n_q * ctx->md.hd, Q,
                                   st),
          "split_hilo");
+  CK(cudaMemsetAsync(ctx->attn_counter, 0, sizeof(int) * static_cast<size_t>(n) * ctx->md.n_kv, st), "counter reset");
+  const kvprm::AttnMerge mg{static_cast<const float*>(q), static_cast<const float*>(k_self),
+                            static_cast<const float*>(v_self), ctx->attn_counter, ctx->ohi, ctx->olo, out, nullptr};
   LAUNCH(KVPRM_PROF_ATTN,
-         kvprm::launch_attn_split(as, P, &ctx->tm_pool, 0, bt, sl, Q.hi, Q.lo, n, ctx->apart_o, ctx->apart_ml,
+         kvprm::launch_attn_split(as, P, &ctx->tm_pool, 0, bt, sl, Q.hi, Q.lo, n, ctx->apart_o, ctx->apart_ml, mg,
                                   ctx->err_d, st, false),
          "attn_split");
-  LAUNCH(KVPRM_PROF_COMBINE,
-         kvprm::launch_attn_combine(as, P, sl, static_cast<const float*>(q), static_cast<const float*>(k_self),
-                                    static_cast<const float*>(v_self), ctx->apart_o, ctx->apart_ml, n, ctx->ohi,
-                                    ctx->olo, out, nullptr, st, false),
-         "attn_combine");
   ctx->last_n = n;
   ctx->last_stream = st;
   if (ctx->profile) {
@@ -801,19 +825,19 @@ int kvprm_projection(kvprm_ctx* ctx, const void* W, int32_t M, int32_t K, const 
     return fail(ctx, KVPRM_ECAPACITY, "n = %d outside [1, max_candidates = %d]", n, ctx->cfg.max_candidates);
   if (!aligned16(W) || !aligned16(X)) return fail(ctx, KVPRM_EINVAL, "W and X must be 16-byte aligned");
   const int n_pad = (n + 15) / 16 * 16;
-  const GemmPlan g = kvprm::plan_gemm(M, K, n_pad, ctx->num_sms, false);
-  if (static_cast<size_t>(g.splits) * n * M > ctx->part_elems)
-    return fail(ctx, KVPRM_ECAPACITY, "projection %dx%d for %d candidates exceeds the partial buffer", M, K, n);
+  const GemmPlan g = kvprm::plan_gemm(M, K, n_pad, ctx->num_sms, false, false);
   CUtensorMap tw, tx;
   int rc;
   if ((rc = make_map(ctx, &tw, W, K, M, 64, 128, "W"))) return rc;
   if ((rc = make_map(ctx, &tx, X, K, n, 64, n_pad, "X"))) return rc;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  kvprm::GemmEpilogue ep;
+  ep.mode = kvprm::GemmEpilogue::PLAIN;
+  ep.M = M;
+  ep.n_valid = n;
+  ep.out = Y;
   Enq E{ctx, st, false, ctx->profile, &ctx->live_marks};
-  LAUNCH(KVPRM_PROF_GEMM_QKV, kvprm::launch_gemm(g, &tw, &tx, nullptr, ctx->part, M, n, n_pad, ctx->err_d, st, false),
-         "gemm");
-  LAUNCH(KVPRM_PROF_FUSED, kvprm::launch_split_sum(ctx->part, g.splits, static_cast<int64_t>(n) * M, Y, st),
-         "split_sum");
+  LAUNCH(KVPRM_PROF_GEMM_QKV, kvprm::launch_gemm(g, &tw, &tx, nullptr, ep, n_pad, ctx->err_d, st, false), "gemm");
   ctx->last_stream = st;
   if (ctx->profile) {
     CK(cudaStreamSynchronize(st), "cudaStreamSynchronize(profile)");
@@ -909,6 +933,38 @@ int kvprm_check_device(kvprm_ctx* ctx) {
     return fail(ctx, KVPRM_ETIMEOUT, "a bounded device wait timed out");
   }
   return KVPRM_OK;
+}
+
+int kvprm_set_trace(kvprm_ctx* ctx, int enable) {
+  if (!ctx) return KVPRM_EINVAL;
+  if (enable && !ctx->trace_d) {
+    ctx->trace_cap = 2 + 8 * ctx->cfg.n_layers + 8;
+    int rc = dalloc(ctx, &ctx->trace_d, static_cast<size_t>(2) * ctx->trace_cap, "trace");
+    if (rc) return rc;
+  }
+  ctx->trace = enable != 0;
+  return KVPRM_OK;
+}
+
+int kvprm_get_trace(kvprm_ctx* ctx, int32_t max_records, int32_t* cls, double* start_us, double* end_us) {
+  if (!ctx || max_records < 0 || (max_records > 0 && (!cls || !start_us || !end_us))) return -KVPRM_EINVAL;
+  if (!ctx->trace_d || ctx->trace_n == 0) return 0;
+  if (cudaStreamSynchronize(ctx->last_stream) != cudaSuccess) return -KVPRM_ECUDA;
+  std::vector<unsigned long long> raw(2 * static_cast<size_t>(ctx->trace_n));
+  if (cudaMemcpy(raw.data(), ctx->trace_d, raw.size() * sizeof(unsigned long long), cudaMemcpyDeviceToHost) !=
+      cudaSuccess)
+    return -KVPRM_ECUDA;
+  unsigned long long t0 = ~0ull;
+  for (int i = 0; i < ctx->trace_n; ++i)
+    if (raw[2 * i] < t0) t0 = raw[2 * i];
+  const int n = ctx->trace_n < max_records ? ctx->trace_n : max_records;
+  for (int i = 0; i < n; ++i) {
+    cls[i] = ctx->trace_cls[i];
+    start_us[i] = (raw[2 * i] == ~0ull) ? -1.0 : 1e-3 * static_cast<double>(raw[2 * i] - t0);
+    const unsigned long long e = ~raw[2 * i + 1];
+    end_us[i] = (raw[2 * i + 1] == ~0ull) ? -1.0 : 1e-3 * static_cast<double>(e - t0);
+  }
+  return n;
 }
 
 int kvprm_set_profile(kvprm_ctx* ctx, int enable) {

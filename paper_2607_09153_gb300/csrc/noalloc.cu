@@ -70,14 +70,16 @@ int setup_current_device(unsigned char** scratch) {
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
 struct Carve {
-  size_t err, sl, bt, qhi, qlo, ohi, olo, pml, po, total;
+  size_t err, cnt, sl, bt, qhi, qlo, ohi, olo, pml, po, total;
 };
 
-Carve carve(int n, int max_blocks, int n_q, int hd, int n_split) {
+Carve carve(int n, int max_blocks, int n_q, int n_kv, int hd, int n_split) {
   Carve c;
   size_t off = 0;
   c.err = off;
   off = align256(off + sizeof(int));
+  c.cnt = off;
+  off = align256(off + sizeof(int) * static_cast<size_t>(n) * n_kv);
   c.sl = off;
   off = align256(off + sizeof(int32_t) * n);
   c.bt = off;
@@ -146,7 +148,7 @@ extern "C" int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, co
   Carve cv;
   for (int cap = kSplitCapMax;; cap /= 2) {
     plan = kvprm::plan_attention(as, n, max_pages, sms, cap);
-    cv = carve(n, max_blocks_per_seq, n_q_heads, head_dim, plan.n_split);
+    cv = carve(n, max_blocks_per_seq, n_q_heads, n_kv_heads, head_dim, plan.n_split);
     if (cv.total <= static_cast<size_t>(KVPRM_NOALLOC_SCRATCH_BYTES)) break;
     if (cap == 1) return KVPRM_ECAPACITY;   // even one split per sequence does not fit
   }
@@ -183,8 +185,12 @@ extern "C" int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, co
   float* pml = reinterpret_cast<float*>(scratch + cv.pml);
   float* po = reinterpret_cast<float*>(scratch + cv.po);
 
-  // the error word must start at zero; everything else is written before it is read
+  int* cnt = reinterpret_cast<int*>(scratch + cv.cnt);
+  // the error word and the split-arrival counters must start at zero; everything
+  // else is written before it is read
   if (cudaMemsetAsync(err, 0, sizeof(int), st) != cudaSuccess) return KVPRM_ECUDA;
+  if (cudaMemsetAsync(cnt, 0, sizeof(int) * static_cast<size_t>(n) * n_kv_heads, st) != cudaSuccess)
+    return KVPRM_ECUDA;
   if (cudaMemcpyAsync(d_sl, seq_lens, sizeof(int32_t) * n, cudaMemcpyHostToDevice, st) != cudaSuccess)
     return KVPRM_ECUDA;
   if (cudaMemcpyAsync(d_bt, block_table, sizeof(int32_t) * static_cast<size_t>(n) * max_blocks_per_seq,
@@ -192,9 +198,8 @@ extern "C" int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, co
     return KVPRM_ECUDA;
   if (kvprm::launch_split_hilo(q, static_cast<int64_t>(n) * n_q_heads * head_dim, Q, st) != cudaSuccess)
     return KVPRM_ECUDA;
-  if (kvprm::launch_attn_split(as, plan, &tm, 0, d_bt, d_sl, Q.hi, Q.lo, n, po, pml, err, st, false) != cudaSuccess)
-    return KVPRM_ECUDA;
-  if (kvprm::launch_attn_combine(as, plan, d_sl, q, k_self, v_self, po, pml, n, ohi, olo, out, nullptr, st, false) !=
+  const kvprm::AttnMerge mg{q, k_self, v_self, cnt, ohi, olo, out, nullptr};
+  if (kvprm::launch_attn_split(as, plan, &tm, 0, d_bt, d_sl, Q.hi, Q.lo, n, po, pml, mg, err, st, false) !=
       cudaSuccess)
     return KVPRM_ECUDA;
   return KVPRM_OK;

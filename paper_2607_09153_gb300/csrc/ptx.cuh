@@ -25,6 +25,17 @@ __device__ __forceinline__ uint64_t global_timer_ns() {
   return t;
 }
 
+// ---------------------------------------------------------------- tracing
+// Optional per-launch timeline (global timer, ns): ts[0] = earliest CTA start,
+// ts[1] = bitwise complement of the latest CTA end, so that both fields reduce
+// with atomicMin from an all-ones reset.  ts == nullptr disables it.
+__device__ __forceinline__ void trace_begin(unsigned long long* ts) {
+  if (ts && threadIdx.x == 0) atomicMin(&ts[0], static_cast<unsigned long long>(global_timer_ns()));
+}
+__device__ __forceinline__ void trace_end(unsigned long long* ts) {
+  if (ts && threadIdx.x == 0) atomicMin(&ts[1], ~static_cast<unsigned long long>(global_timer_ns()));
+}
+
 // ---------------------------------------------------------------- mbarrier
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");

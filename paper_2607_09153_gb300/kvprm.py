@@ -71,6 +71,8 @@ def lib() -> ctypes.CDLL:
         L.kvprm_resolve.argtypes = [vp, i32, i64p]
         L.kvprm_check_device.argtypes = [vp]
         L.kvprm_set_profile.argtypes = [vp, ctypes.c_int]
+        L.kvprm_set_trace.argtypes = [vp, ctypes.c_int]
+        L.kvprm_get_trace.argtypes = [vp, i32, i32p, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)]
         L.kvprm_get_profile.argtypes = [vp, i64p, ctypes.POINTER(ctypes.c_double)]
         _lib = L
     return _lib
@@ -184,6 +186,23 @@ def kvprm_check_device(ctx) -> None:
 
 def kvprm_set_profile(ctx, enable: bool) -> None:
     _check(ctx, lib().kvprm_set_profile(ctx, int(enable)))
+
+
+def kvprm_set_trace(ctx, enable: bool) -> None:
+    _check(ctx, lib().kvprm_set_trace(ctx, int(enable)))
+
+
+def kvprm_get_trace(ctx, max_records: int = 4096) -> list:
+    """[(class name, start us, end us)] of the last call's launches, in issue order."""
+    cls = np.zeros(max_records, np.int32)
+    t0 = np.zeros(max_records, np.float64)
+    t1 = np.zeros(max_records, np.float64)
+    n = lib().kvprm_get_trace(ctx, max_records, _p(cls, ctypes.c_int32),
+                              t0.ctypes.data_as(ctypes.POINTER(ctypes.c_double)),
+                              t1.ctypes.data_as(ctypes.POINTER(ctypes.c_double)))
+    if n < 0:
+        _check(ctx, -n)
+    return [(PROF_NAMES[cls[i]], float(t0[i]), float(t1[i])) for i in range(n)]
 
 
 def kvprm_get_profile(ctx) -> dict:
