@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <vector>
+
 namespace kvprm {
 
 // ---------------------------------------------------------------- projection GEMM
@@ -48,14 +50,35 @@ struct AttnShape {
   int max_blocks;               // block-table row length
   int64_t layer_rows;           // rows (of hd elements) per layer in the pool map: n_pages * 2 * n_kv * 16
 };
-struct AttnPlan {
-  int n_split = 1;              // splits of the page range per (candidate, kv head)
-  int pages_per_split = 1;
-  size_t smem_bytes = 0;
+// One unit of attention work (see attention.cu): a run of physical pages of one
+// candidate (kind 0) or pages shared by up to 8 candidates (kind 1).
+struct AttnItem {
+  int32_t kind;
+  int32_t cand;        // kind 0: the candidate; kind 1: offset into AttnWork::cands
+  int32_t n_cands;     // kind 1: candidates (<= 8)
+  int32_t page_off;    // offset into AttnWork::pages
+  int32_t n_pages;     // 0: an empty cache (self entry only)
+  int32_t last_valid;  // valid tokens in the item's last page (1..16)
+  int32_t slot;        // kind 0: the candidate's partial slot; kind 1: offset into AttnWork::slots
+  int32_t pad;
 };
-AttnPlan plan_attention(const AttnShape& s, int n_cand, int max_pages, int num_sms, int split_cap);
+struct AttnWork {            // device arrays
+  const AttnItem* items;
+  const int32_t* pages;      // physical page ids
+  const int32_t* cands;      // candidates of shared items
+  const int32_t* slots;      // their partial slots
+  const int32_t* nslots;     // [B] partial slots of each candidate
+  int n_items;
+};
+struct AttnWorkHost {
+  std::vector<AttnItem> items;
+  std::vector<int32_t> pages, cands, slots, nslots;
+  int max_item_pages = 0;
+};
+bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks, int n_kv, int hd, int num_sms,
+                     int slot_cap, bool share, AttnWorkHost& w);
+size_t attention_smem_bytes(int hd, int max_item_pages);
 cudaError_t attention_configure();
-// part_o [B][n_q][n_split][hd] (unnormalised), part_ml [B][n_q][n_split][2] (max in log2 units, sum)
 // Inputs and outputs of the split merge done by the last CTA of each (candidate, kv head).
 struct AttnMerge {
   const float* q;       // [B][n_q][hd] rotated query (fp32)
@@ -67,12 +90,12 @@ struct AttnMerge {
   float* out_f32;       // optional fp32 copy
   float* dbg;           // optional fp32 copy
 };
-// q_hi / q_lo: bf16 pair of the rotated query [B][n_q][hd]
-cudaError_t launch_attn_split(const AttnShape& s, const AttnPlan& p, const CUtensorMap* tm_pool, int layer,
-                              const int32_t* bt, const int32_t* seq_lens, const __nv_bfloat16* q_hi,
-                              const __nv_bfloat16* q_lo, int n_cand, float* part_o, float* part_ml,
-                              const AttnMerge& mg, int* err, cudaStream_t stream, bool pdl,
-                              unsigned long long* ts = nullptr);
+// q_hi / q_lo: bf16 pair of the rotated query [B][n_q][hd]; partial slots
+// [B][n_q][stride][hd] (values) and [B][n_q][stride][2] (max in log2 units, sum)
+cudaError_t launch_attention(const AttnShape& s, const AttnWork& wk, int max_item_pages, const CUtensorMap* tm_pool,
+                             int layer, const __nv_bfloat16* q_hi, const __nv_bfloat16* q_lo, int stride,
+                             float* part_o, float* part_ml, const AttnMerge& mg, int* err, cudaStream_t stream,
+                             bool pdl, unsigned long long* ts = nullptr);
 cudaError_t launch_resolve(const int32_t* bt, const int32_t* seq_lens, int max_blocks, int b, int64_t* out,
                            cudaStream_t stream);
 

@@ -17,7 +17,6 @@
 #include "../../include/kvprm.h"
 #include "kernels.h"
 
-using kvprm::AttnPlan;
 using kvprm::AttnShape;
 using kvprm::GemmPlan;
 using kvprm::ModelDims;
@@ -30,15 +29,16 @@ constexpr int kSplitCap = 32;   // max split-K partials of the attention per (ca
 struct CallPlan {
   int n = 0, n_pad = 0, max_pages = 0;
   GemmPlan g_qkv, g_o, g_gu, g_down;
-  AttnPlan attn;
+  int n_items = 0, max_item_pages = 0;   // attention work list (see build_attn_work)
 };
 
 struct GraphKey {
-  int n = -1, n_pad = -1, n_split = -1, pps = -1, debug = -1, profile = -1, pdl = -1, trace = -1;
+  int n = -1, n_pad = -1, n_items = -1, max_item_pages = -1, debug = -1, profile = -1, pdl = -1, trace = -1;
   const void* pool = nullptr;
   int64_t n_pages = -1;
   bool operator==(const GraphKey& o) const {
-    return n == o.n && n_pad == o.n_pad && n_split == o.n_split && pps == o.pps && debug == o.debug &&
+    return n == o.n && n_pad == o.n_pad && n_items == o.n_items && max_item_pages == o.max_item_pages &&
+           debug == o.debug &&
            profile == o.profile && pdl == o.pdl && trace == o.trace && pool == o.pool && n_pages == o.n_pages;
   }
 };
@@ -71,7 +71,12 @@ struct kvprm_ctx {
   float *apart_o = nullptr, *apart_ml = nullptr;
   int* attn_counter = nullptr;   // [Bmax][n_kv] split-arrival counters
   float2* rope = nullptr;
-  int32_t* tables_d = nullptr;   // [Bmax] seq_lens, then [Bmax][max_blocks] block table
+  int32_t* tables_d = nullptr;   // [Bmax] seq_lens, [Bmax][max_blocks] block table, then the attention work
+  // attention work list: host plan of the current call and fixed offsets (ints) in tables_d / staging
+  kvprm::AttnWorkHost work_host;
+  size_t off_items = 0, off_pages = 0, off_cands = 0, off_slots = 0, off_nslots = 0, tables_ints = 0;
+  size_t cap_items = 0, cap_pages = 0, cap_cands = 0;
+  bool share_pages = true;
   float* rewards_d = nullptr;
   int* err_d = nullptr;
   float* dbg = nullptr;
@@ -246,20 +251,57 @@ int validate_tables(kvprm_ctx* ctx, int64_t n_pages, const int32_t* bt, const in
   return KVPRM_OK;
 }
 
+// Plan the attention work of this call on the host (build_attn_work).
+int plan_work(kvprm_ctx* ctx, const int32_t* bt, const int32_t* sl, int32_t n) {
+  kvprm::AttnWorkHost& w = ctx->work_host;
+  if (!kvprm::build_attn_work(bt, sl, n, ctx->cfg.max_blocks_per_seq, ctx->cfg.n_kv_heads, ctx->cfg.head_dim,
+                              ctx->num_sms, kSplitCap, ctx->share_pages, w))
+    return fail(ctx, KVPRM_EUNSUPPORTED, "attention work does not fit %d partial slots per candidate", kSplitCap);
+  if (w.items.size() > ctx->cap_items || w.pages.size() > ctx->cap_pages || w.cands.size() > ctx->cap_cands)
+    return fail(ctx, KVPRM_ECAPACITY, "attention work list exceeds the context's capacity");
+  return KVPRM_OK;
+}
+
+// Copy the tables and the planned work into pinned staging and then to the device.
 int upload_tables(kvprm_ctx* ctx, const int32_t* bt, const int32_t* sl, int32_t n, cudaStream_t st) {
   const int Bmax = ctx->cfg.max_candidates, mb = ctx->cfg.max_blocks_per_seq;
   if (ctx->staging_pending) {
     CK(cudaEventSynchronize(ctx->staging_ev), "cudaEventSynchronize(staging)");
     ctx->staging_pending = false;
   }
-  std::memcpy(ctx->staging, sl, sizeof(int32_t) * n);
-  std::memcpy(ctx->staging + Bmax, bt, sizeof(int32_t) * static_cast<size_t>(n) * mb);
-  const size_t count = static_cast<size_t>(Bmax) + static_cast<size_t>(n) * mb;
-  CK(cudaMemcpyAsync(ctx->tables_d, ctx->staging, count * sizeof(int32_t), cudaMemcpyHostToDevice, st),
-     "cudaMemcpyAsync(tables)");
+  const kvprm::AttnWorkHost& w = ctx->work_host;
+  int32_t* S = ctx->staging;
+  std::memcpy(S, sl, sizeof(int32_t) * n);
+  std::memcpy(S + Bmax, bt, sizeof(int32_t) * static_cast<size_t>(n) * mb);
+  std::memcpy(S + ctx->off_items, w.items.data(), sizeof(kvprm::AttnItem) * w.items.size());
+  std::memcpy(S + ctx->off_pages, w.pages.data(), sizeof(int32_t) * w.pages.size());
+  std::memcpy(S + ctx->off_cands, w.cands.data(), sizeof(int32_t) * w.cands.size());
+  std::memcpy(S + ctx->off_slots, w.slots.data(), sizeof(int32_t) * w.slots.size());
+  std::memcpy(S + ctx->off_nslots, w.nslots.data(), sizeof(int32_t) * w.nslots.size());
+  auto up = [&](size_t off, size_t ints) -> cudaError_t {
+    if (ints == 0) return cudaSuccess;
+    return cudaMemcpyAsync(ctx->tables_d + off, S + off, ints * sizeof(int32_t), cudaMemcpyHostToDevice, st);
+  };
+  CK(up(0, static_cast<size_t>(Bmax) + static_cast<size_t>(n) * mb), "cudaMemcpyAsync(tables)");
+  CK(up(ctx->off_items, w.items.size() * (sizeof(kvprm::AttnItem) / sizeof(int32_t))), "cudaMemcpyAsync(items)");
+  CK(up(ctx->off_pages, w.pages.size()), "cudaMemcpyAsync(pages)");
+  CK(up(ctx->off_cands, w.cands.size()), "cudaMemcpyAsync(cands)");
+  CK(up(ctx->off_slots, w.slots.size()), "cudaMemcpyAsync(slots)");
+  CK(up(ctx->off_nslots, w.nslots.size()), "cudaMemcpyAsync(nslots)");
   CK(cudaEventRecord(ctx->staging_ev, st), "cudaEventRecord(staging)");
   ctx->staging_pending = true;
   return KVPRM_OK;
+}
+
+kvprm::AttnWork device_work(kvprm_ctx* ctx) {
+  kvprm::AttnWork wk;
+  wk.items = reinterpret_cast<const kvprm::AttnItem*>(ctx->tables_d + ctx->off_items);
+  wk.pages = ctx->tables_d + ctx->off_pages;
+  wk.cands = ctx->tables_d + ctx->off_cands;
+  wk.slots = ctx->tables_d + ctx->off_slots;
+  wk.nslots = ctx->tables_d + ctx->off_nslots;
+  wk.n_items = static_cast<int>(ctx->work_host.items.size());
+  return wk;
 }
 
 int ensure_pool_map(kvprm_ctx* ctx, const void* pool, int64_t n_pages, int layers) {
@@ -302,7 +344,8 @@ CallPlan make_plan(kvprm_ctx* ctx, int n, int max_pages) {
   p.g_o = kvprm::plan_gemm(m.d, m.n_q * m.hd, p.n_pad, ctx->num_sms, true, false);
   p.g_gu = kvprm::plan_gemm(m.ff, m.d, p.n_pad, ctx->num_sms, true, true);
   p.g_down = kvprm::plan_gemm(m.d, m.ff, p.n_pad, ctx->num_sms, true, false);
-  p.attn = kvprm::plan_attention(ctx->as, n, max_pages, ctx->num_sms, kSplitCap);
+  p.n_items = static_cast<int>(ctx->work_host.items.size());
+  p.max_item_pages = ctx->work_host.max_item_pages;
   return p;
 }
 
@@ -356,7 +399,6 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
   const ModelDims& m = ctx->md;
   const int n = P.n, np = P.n_pad;
   const int32_t* sl = ctx->tables_d;
-  const int32_t* bt = ctx->tables_d + ctx->cfg.max_candidates;
   cudaStream_t st = E.st;
   const bool pdl = E.pdl;
   const int NL = ctx->cfg.n_layers;
@@ -409,9 +451,9 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
     float* dbg = (ctx->debug_flags & 1) ? ctx->dbg + static_cast<size_t>(l) * n * m.n_q * m.hd : nullptr;
     const kvprm::AttnMerge mg{ctx->q, ctx->kself, ctx->vself, ctx->attn_counter, O.hi, O.lo, nullptr, dbg};
     LAUNCH(KVPRM_PROF_ATTN,
-           kvprm::launch_attn_split(ctx->as, P.attn, &ctx->tm_pool, l, bt, sl, ctx->qhi, ctx->qlo, n, ctx->apart_o,
-                                    ctx->apart_ml, mg, ctx->err_d, st, pdl, TS),
-           "attn_split");
+           kvprm::launch_attention(ctx->as, device_work(ctx), P.max_item_pages, &ctx->tm_pool, l, ctx->qhi, ctx->qlo,
+                                   kSplitCap, ctx->apart_o, ctx->apart_ml, mg, ctx->err_d, st, pdl, TS),
+           "attention");
     LAUNCH(KVPRM_PROF_GEMM_O,
            kvprm::launch_gemm(P.g_o, &ctx->tm_o[l], &ctx->tm_ohi, &ctx->tm_olo, er, np, ctx->err_d, st, pdl, TS),
            "gemm_o");
@@ -486,6 +528,7 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   }
   if ((rc = ensure_pool_map(ctx, pool, pages, ctx->cfg.n_layers))) return rc;
   ctx->as.layer_rows = pages * 2 * ctx->cfg.n_kv_heads * 16;
+  if ((rc = plan_work(ctx, bt, sl, n))) return rc;
   const CallPlan P = make_plan(ctx, n, max_pages);
   if ((rc = ensure_x_maps(ctx, P.n_pad))) return rc;
   if ((rc = upload_tables(ctx, bt, sl, n, st))) return rc;
@@ -504,8 +547,8 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   GraphKey key;
   key.n = n;
   key.n_pad = P.n_pad;
-  key.n_split = P.attn.n_split;
-  key.pps = P.attn.pages_per_split;
+  key.n_items = P.n_items;
+  key.max_item_pages = P.max_item_pages;
   key.debug = ctx->debug_flags;
   key.profile = ctx->profile ? 1 : 0;
   key.pdl = ctx->use_pdl ? 1 : 0;
@@ -675,13 +718,26 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   CREATE_CK(dalloc(ctx, &ctx->apart_ml, static_cast<size_t>(Bmax) * m.n_q * kSplitCap * 2, "attn stats"));
   CREATE_CK(dalloc(ctx, &ctx->attn_counter, static_cast<size_t>(Bmax) * m.n_kv, "attn counters"));
   CREATE_CK(dalloc(ctx, &ctx->rope, static_cast<size_t>(Bmax) * (m.hd / 2), "rope table"));
-  CREATE_CK(dalloc(ctx, &ctx->tables_d, static_cast<size_t>(Bmax) * (1 + c.max_blocks_per_seq), "tables"));
+  {
+    const size_t tbl = static_cast<size_t>(Bmax) * (1 + c.max_blocks_per_seq);
+    auto al8 = [](size_t x) { return (x + 7) & ~static_cast<size_t>(7); };
+    ctx->cap_items = static_cast<size_t>(Bmax) * (kSplitCap + 1);
+    ctx->cap_pages = static_cast<size_t>(2) * Bmax * c.max_blocks_per_seq;
+    ctx->cap_cands = static_cast<size_t>(Bmax) * kSplitCap;
+    ctx->off_items = al8(tbl);
+    ctx->off_pages = al8(ctx->off_items + ctx->cap_items * (sizeof(kvprm::AttnItem) / sizeof(int32_t)));
+    ctx->off_cands = al8(ctx->off_pages + ctx->cap_pages);
+    ctx->off_slots = al8(ctx->off_cands + ctx->cap_cands);
+    ctx->off_nslots = al8(ctx->off_slots + ctx->cap_cands);
+    ctx->tables_ints = al8(ctx->off_nslots + Bmax);
+  }
+  CREATE_CK(dalloc(ctx, &ctx->tables_d, ctx->tables_ints, "tables and attention work"));
   CREATE_CK(dalloc(ctx, &ctx->rewards_d, static_cast<size_t>(Bmax), "rewards"));
   CREATE_CK(dalloc(ctx, &ctx->err_d, 1, "err"));
   CREATE_CK(dalloc(ctx, &ctx->dummy_pool, static_cast<size_t>(NL) * 2 * m.n_kv * 16 * m.hd, "dummy pool"));
   {
     cudaError_t e =
-        cudaMallocHost(reinterpret_cast<void**>(&ctx->staging), sizeof(int32_t) * Bmax * (1 + c.max_blocks_per_seq));
+        cudaMallocHost(reinterpret_cast<void**>(&ctx->staging), sizeof(int32_t) * ctx->tables_ints);
     if (e == cudaSuccess) e = cudaMallocHost(reinterpret_cast<void**>(&ctx->h_rewards), sizeof(float) * Bmax);
     if (e == cudaSuccess) e = cudaMallocHost(reinterpret_cast<void**>(&ctx->h_err), sizeof(int));
     if (e != cudaSuccess) {
@@ -694,6 +750,7 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   CREATE_CK(cu(cudaStreamCreateWithFlags(&ctx->cap_stream, cudaStreamNonBlocking), "cudaStreamCreate"));
   ctx->use_graph = !env_off("KVPRM_NO_GRAPH");
   ctx->use_pdl = !env_off("KVPRM_NO_PDL");
+  ctx->share_pages = !env_off("KVPRM_NO_SHARING");
   CREATE_CK(cu(cudaDeviceSynchronize(), "cudaDeviceSynchronize(create)"));
 #undef CREATE_CK
   *out = ctx;
@@ -786,12 +843,10 @@ int kvprm_attention(kvprm_ctx* ctx, const void* kv_layer, int64_t n_pages, const
     if (!aligned16(kv_layer)) return fail(ctx, KVPRM_EINVAL, "kv_layer is not 16-byte aligned");
   }
   if ((rc = ensure_pool_map(ctx, pool, pages, 1))) return rc;
+  if ((rc = plan_work(ctx, block_table, seq_lens, n))) return rc;
   if ((rc = upload_tables(ctx, block_table, seq_lens, n, st))) return rc;
   AttnShape as = ctx->as;
   as.layer_rows = pages * 2 * ctx->cfg.n_kv_heads * 16;
-  const AttnPlan P = kvprm::plan_attention(as, n, max_pages, ctx->num_sms, kSplitCap);
-  const int32_t* sl = ctx->tables_d;
-  const int32_t* bt = ctx->tables_d + ctx->cfg.max_candidates;
   Enq E{ctx, st, false, ctx->profile, &ctx->live_marks};
   LAUNCH(KVPRM_PROF_FUSED,
          kvprm::launch_split_hilo(static_cast<const float*>(q), static_cast<int64_t>(n) * ctx->md.n_q * ctx->md.hd, Q,
@@ -801,9 +856,9 @@ int kvprm_attention(kvprm_ctx* ctx, const void* kv_layer, int64_t n_pages, const
   const kvprm::AttnMerge mg{static_cast<const float*>(q), static_cast<const float*>(k_self),
                             static_cast<const float*>(v_self), ctx->attn_counter, ctx->ohi, ctx->olo, out, nullptr};
   LAUNCH(KVPRM_PROF_ATTN,
-         kvprm::launch_attn_split(as, P, &ctx->tm_pool, 0, bt, sl, Q.hi, Q.lo, n, ctx->apart_o, ctx->apart_ml, mg,
-                                  ctx->err_d, st, false),
-         "attn_split");
+         kvprm::launch_attention(as, device_work(ctx), ctx->work_host.max_item_pages, &ctx->tm_pool, 0, Q.hi, Q.lo,
+                                 kSplitCap, ctx->apart_o, ctx->apart_ml, mg, ctx->err_d, st, false),
+         "attention");
   ctx->last_n = n;
   ctx->last_stream = st;
   if (ctx->profile) {

@@ -3,9 +3,9 @@
 // all of its GPU memory up front and forbids allocations afterwards, or code
 // that runs inside another framework's memory-managed region where a
 // cudaMalloc would break the owner's accounting or stall on a device-wide
-// synchronisation.  It needs no context: its scratch (the copied block table
-// and lengths, the query split into bf16 hi/lo parts, the split-K partials and
-// an error word) lives in one file-scope device array, so every GPU that loads
+// synchronisation.  It needs no context: its scratch (the attention work list built
+// on the host from the block table and lengths, the query split into bf16
+// hi/lo parts, the split partials and an error word) lives in one file-scope device array, so every GPU that loads
 // this library holds that array until the process exits.
 //
 // Set-up: the first call on a device (with that device current) looks up the
@@ -70,33 +70,35 @@ int setup_current_device(unsigned char** scratch) {
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
 struct Carve {
-  size_t err, cnt, sl, bt, qhi, qlo, ohi, olo, pml, po, total;
+  size_t err, cnt, items, pages, cands, slots, nslots, qhi, qlo, ohi, olo, pml, po, total;
 };
 
-Carve carve(int n, int max_blocks, int n_q, int n_kv, int hd, int n_split) {
+// Layout of the scratch array for one call: the error word, the split-arrival
+// counters, the attention work list, the query's bf16 hi/lo parts, the
+// output's hi/lo parts (the kernel always writes them) and `stride` partial
+// slots per (candidate, query head).
+Carve carve(int n, int n_q, int n_kv, int hd, int stride, const kvprm::AttnWorkHost& w) {
   Carve c;
   size_t off = 0;
-  c.err = off;
-  off = align256(off + sizeof(int));
-  c.cnt = off;
-  off = align256(off + sizeof(int) * static_cast<size_t>(n) * n_kv);
-  c.sl = off;
-  off = align256(off + sizeof(int32_t) * n);
-  c.bt = off;
-  off = align256(off + sizeof(int32_t) * static_cast<size_t>(n) * max_blocks);
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = align256(off + bytes);
+    return at;
+  };
+  c.err = take(sizeof(int));
+  c.cnt = take(sizeof(int) * static_cast<size_t>(n) * n_kv);
+  c.items = take(sizeof(kvprm::AttnItem) * w.items.size());
+  c.pages = take(sizeof(int32_t) * w.pages.size());
+  c.cands = take(sizeof(int32_t) * w.cands.size());
+  c.slots = take(sizeof(int32_t) * w.slots.size());
+  c.nslots = take(sizeof(int32_t) * w.nslots.size());
   const size_t qe = static_cast<size_t>(n) * n_q * hd;
-  c.qhi = off;
-  off = align256(off + 2 * qe);
-  c.qlo = off;
-  off = align256(off + 2 * qe);
-  c.ohi = off;
-  off = align256(off + 2 * qe);
-  c.olo = off;
-  off = align256(off + 2 * qe);
-  c.pml = off;
-  off = align256(off + sizeof(float) * static_cast<size_t>(n) * n_q * n_split * 2);
-  c.po = off;
-  off = align256(off + sizeof(float) * qe * n_split);
+  c.qhi = take(2 * qe);
+  c.qlo = take(2 * qe);
+  c.ohi = take(2 * qe);
+  c.olo = take(2 * qe);
+  c.pml = take(sizeof(float) * static_cast<size_t>(n) * n_q * stride * 2);
+  c.po = take(sizeof(float) * qe * stride);
   c.total = off;
   return c;
 }
@@ -143,14 +145,18 @@ extern "C" int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, co
   int dev = 0, sms = 148;
   if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     return KVPRM_ECUDA;
-  // the largest split count (<= kSplitCapMax) whose partials fit in the array
-  kvprm::AttnPlan plan;
+  // the work list with the most partial slots per candidate (<= kSplitCapMax)
+  // whose list and partials fit in the array
+  thread_local kvprm::AttnWorkHost work;
   Carve cv;
-  for (int cap = kSplitCapMax;; cap /= 2) {
-    plan = kvprm::plan_attention(as, n, max_pages, sms, cap);
-    cv = carve(n, max_blocks_per_seq, n_q_heads, n_kv_heads, head_dim, plan.n_split);
-    if (cv.total <= static_cast<size_t>(KVPRM_NOALLOC_SCRATCH_BYTES)) break;
-    if (cap == 1) return KVPRM_ECAPACITY;   // even one split per sequence does not fit
+  int stride = kSplitCapMax;
+  for (;; stride /= 2) {
+    if (kvprm::build_attn_work(block_table, seq_lens, n, max_blocks_per_seq, n_kv_heads, head_dim, sms, stride, true,
+                               work)) {
+      cv = carve(n, n_q_heads, n_kv_heads, head_dim, stride, work);
+      if (cv.total <= static_cast<size_t>(KVPRM_NOALLOC_SCRATCH_BYTES)) break;
+    }
+    if (stride == 1) return KVPRM_ECAPACITY;   // does not fit even with one slot per candidate
   }
 
   // tensor map over this layer's pages (built on the host stack; no allocation)
@@ -177,29 +183,40 @@ extern "C" int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, co
 
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   int* err = reinterpret_cast<int*>(scratch + cv.err);
-  int32_t* d_sl = reinterpret_cast<int32_t*>(scratch + cv.sl);
-  int32_t* d_bt = reinterpret_cast<int32_t*>(scratch + cv.bt);
+  int* cnt = reinterpret_cast<int*>(scratch + cv.cnt);
   kvprm::HiLo Q{reinterpret_cast<__nv_bfloat16*>(scratch + cv.qhi), reinterpret_cast<__nv_bfloat16*>(scratch + cv.qlo)};
   __nv_bfloat16* ohi = reinterpret_cast<__nv_bfloat16*>(scratch + cv.ohi);
   __nv_bfloat16* olo = reinterpret_cast<__nv_bfloat16*>(scratch + cv.olo);
   float* pml = reinterpret_cast<float*>(scratch + cv.pml);
   float* po = reinterpret_cast<float*>(scratch + cv.po);
+  kvprm::AttnWork wk;
+  wk.items = reinterpret_cast<const kvprm::AttnItem*>(scratch + cv.items);
+  wk.pages = reinterpret_cast<const int32_t*>(scratch + cv.pages);
+  wk.cands = reinterpret_cast<const int32_t*>(scratch + cv.cands);
+  wk.slots = reinterpret_cast<const int32_t*>(scratch + cv.slots);
+  wk.nslots = reinterpret_cast<const int32_t*>(scratch + cv.nslots);
+  wk.n_items = static_cast<int>(work.items.size());
 
-  int* cnt = reinterpret_cast<int*>(scratch + cv.cnt);
   // the error word and the split-arrival counters must start at zero; everything
   // else is written before it is read
   if (cudaMemsetAsync(err, 0, sizeof(int), st) != cudaSuccess) return KVPRM_ECUDA;
   if (cudaMemsetAsync(cnt, 0, sizeof(int) * static_cast<size_t>(n) * n_kv_heads, st) != cudaSuccess)
     return KVPRM_ECUDA;
-  if (cudaMemcpyAsync(d_sl, seq_lens, sizeof(int32_t) * n, cudaMemcpyHostToDevice, st) != cudaSuccess)
-    return KVPRM_ECUDA;
-  if (cudaMemcpyAsync(d_bt, block_table, sizeof(int32_t) * static_cast<size_t>(n) * max_blocks_per_seq,
-                      cudaMemcpyHostToDevice, st) != cudaSuccess)
+  // pageable host sources: each copy is staged by the driver before it returns,
+  // so the thread-local work list may be rebuilt by the next call
+  auto up = [&](size_t off, const void* src, size_t bytes) {
+    return bytes == 0 || cudaMemcpyAsync(scratch + off, src, bytes, cudaMemcpyHostToDevice, st) == cudaSuccess;
+  };
+  if (!up(cv.items, work.items.data(), sizeof(kvprm::AttnItem) * work.items.size()) ||
+      !up(cv.pages, work.pages.data(), sizeof(int32_t) * work.pages.size()) ||
+      !up(cv.cands, work.cands.data(), sizeof(int32_t) * work.cands.size()) ||
+      !up(cv.slots, work.slots.data(), sizeof(int32_t) * work.slots.size()) ||
+      !up(cv.nslots, work.nslots.data(), sizeof(int32_t) * work.nslots.size()))
     return KVPRM_ECUDA;
   if (kvprm::launch_split_hilo(q, static_cast<int64_t>(n) * n_q_heads * head_dim, Q, st) != cudaSuccess)
     return KVPRM_ECUDA;
   const kvprm::AttnMerge mg{q, k_self, v_self, cnt, ohi, olo, out, nullptr};
-  if (kvprm::launch_attn_split(as, plan, &tm, 0, d_bt, d_sl, Q.hi, Q.lo, n, po, pml, mg, err, st, false) !=
+  if (kvprm::launch_attention(as, wk, work.max_item_pages, &tm, 0, Q.hi, Q.lo, stride, po, pml, mg, err, st, false) !=
       cudaSuccess)
     return KVPRM_ECUDA;
   return KVPRM_OK;
