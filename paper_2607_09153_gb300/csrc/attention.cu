@@ -3,20 +3,23 @@
 // split over the cache ("flash decoding"), with the splits merged together
 // with the verify token's own key/value.
 //
-// The work is a list of items built on the host from the block tables
-// (build_attn_work), one CTA per (item, kv head), 9 warps:
-//  - warp 8 (producer) copies the item's physical page ids to shared memory
-//    and streams K and V pages with TMA (tiled, 128-byte swizzle) into a
-//    3-stage ring of 8 pages (128 tokens) per stage -- starting before the
-//    query is ready, since the cache does not depend on it;
-//  - a *private* item holds pages of one candidate: consumer warp w scores
-//    page w of every stage, and the eight warps' (m, l, O) are merged in
-//    shared memory into one partial;
-//  - a *shared* item holds pages that several candidates reference (a beam
+// Persistent layout: one CTA per SM (9 warps) works through a host-built
+// schedule (build_attn_work).  The schedule lays every (run of pages, kv head)
+// end to end on a cost axis and cuts the axis into equal CTA ranges, so every
+// SM streams the same number of bytes whatever the mix of lengths; a run cut
+// by a range boundary simply yields one more partial.
+//  - warp 8 (producer) streams the K and V pages of the CTA's segments, one
+//    after the other, with TMA (one 5-D box per page and kv head: K and V,
+//    128-byte swizzle) through a 3-stage ring of 8 pages (128 tokens) per
+//    stage -- starting before the query is ready, since the cache does not
+//    depend on it -- and never drains the ring between segments;
+//  - a *private* segment holds pages of one candidate: consumer warp w scores
+//    page w of every stage;
+//  - a *shared* segment holds pages that several candidates reference (a beam
 //    prefix, an MCTS ancestor): each page is loaded once and consumer warp w
-//    scores it for candidate w (up to 8), writing its own partial.  Attention
-//    is invariant to the order of the keys, so shared pages need not sit at
-//    the same positions in the candidates' sequences;
+//    scores it for candidate w (up to 8).  Attention is invariant to the order
+//    of the keys, so shared pages need not sit at the same positions in the
+//    candidates' sequences;
 //  - per page and warp: S = Q K^T on the tensor cores (mma.m16n8k16), an
 //    online softmax in fp32 registers with quad shuffles, then O += P V.  The
 //    query and the probabilities enter the bf16 MMAs as (hi, lo) pairs so both
@@ -24,10 +27,14 @@
 //    rows 0..7 and the lo parts rows 8..15 of the same instruction (summed
 //    afterwards), so the split costs no extra MMAs; with 8 < G <= 16 hi and lo
 //    take one MMA each;
-//  - every partial lands in a slot of its candidate; the last arrival per
-//    (candidate, kv head) (an atomic counter, no waiting) merges the slots with
-//    the self entry and writes the attention output as a bf16 (hi, lo) pair
-//    for the O projection.
+//  - at the end of a private segment the consumer warps hand their (m, l, O)
+//    to warp 9 (the merger) through shared memory and go straight on to the
+//    next segment; the merger folds them into the segment's partial slot.  In
+//    a shared segment each warp writes its own candidate's slot.  No barrier,
+//    fence or atomic is involved;
+//  - a second small kernel (attn_combine_kernel) merges each (candidate, kv
+//    head)'s slots with the verify token's own entry and writes the attention
+//    output as a bf16 (hi, lo) pair for the O projection.
 // All scores are kept in log2 units (scaled by log2(e) / sqrt(hd)).
 #include <cuda_bf16.h>
 
@@ -45,8 +52,19 @@ namespace {
 constexpr int kPagesPerStage = 8;
 constexpr int kStages = 3;
 constexpr int kConsumerWarps = 8;
-constexpr int kThreads = (kConsumerWarps + 1) * 32;
+constexpr int kProducerWarp = kConsumerWarps;       // warp 8: TMA
+constexpr int kMergerWarp = kConsumerWarps + 1;     // warp 9: folds private segments' warp states
+constexpr int kThreads = (kConsumerWarps + 2) * 32;
 constexpr float kLog2e = 1.4426950408889634f;
+
+// Schedule costs per page and kv head.  A private page is read by one warp
+// while the other seven read the rest of its stage, so a private stage costs
+// the time to stream it (measured ~0.19 us per page per SM at full HBM rate).
+// A shared page is scored by one warp per candidate, and those warps compete
+// for the same SM pipelines: measured ~0.1 us per page and candidate, i.e. about
+// half a private page per candidate.
+constexpr int64_t kPrivateCost = 4;
+constexpr int64_t kSharedCostPerCand = 2;
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -56,64 +74,6 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
 // used by the resolve entry point, so indexing can be checked bit-exactly).
 __device__ __forceinline__ int32_t phys_page(const int32_t* __restrict__ bt, int b, int max_blocks, int j) {
   return bt[static_cast<int64_t>(b) * max_blocks + j];
-}
-
-// Merge the ns partial slots of every query head of group g of candidate b
-// with the verify token's own entry s_self = q . k_self / sqrt(hd):
-//   M = max(m_i, s_self), o = (sum_i 2^(m_i - M) o_i + 2^(s_self - M) v_self)
-//                             / (sum_i 2^(m_i - M) l_i + 2^(s_self - M)),
-// summed in slot order.  Warps w0, w0 + nw, ... take one head each.
-template <int HD>
-__device__ __forceinline__ void merge_group(int b, int g, int n_q, int n_kv, int group, int ns, int stride,
-                                            const float* __restrict__ part_o, const float* __restrict__ part_ml,
-                                            const AttnMerge& mg, int w0, int nw) {
-  constexpr int kPer = HD / 32;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t hk = static_cast<int64_t>(b) * n_kv + g;
-  for (int r = warp - w0; r < group; r += nw) {
-    const int64_t hq = static_cast<int64_t>(b) * n_q + static_cast<int64_t>(g) * group + r;
-    float qv[kPer], vv[kPer];
-    float dot = 0.f;
-#pragma unroll
-    for (int j = 0; j < kPer; ++j) {
-      const int d = lane + 32 * j;
-      qv[j] = mg.q[hq * HD + d];
-      dot += qv[j] * mg.kself[hk * HD + d];
-      vv[j] = mg.vself[hk * HD + d];
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
-    const float s_self = dot * (kLog2e * rsqrtf(static_cast<float>(HD)));
-    const float mi = lane < ns ? __ldcg(part_ml + (hq * stride + lane) * 2) : -INFINITY;
-    const float li = lane < ns ? __ldcg(part_ml + (hq * stride + lane) * 2 + 1) : 0.f;
-    float M = fmaxf(mi, s_self);
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, off));
-    const float wi = lane < ns ? exp2f(mi - M) : 0.f;
-    const float wself = exp2f(s_self - M);
-    float lsum = wself;
-    for (int i = 0; i < ns; ++i) lsum += __shfl_sync(0xffffffffu, wi * li, i);
-    const float inv = 1.0f / lsum;
-    float acc[kPer];
-#pragma unroll
-    for (int j = 0; j < kPer; ++j) acc[j] = wself * vv[j];
-    const float* po = part_o + hq * stride * HD + lane;
-    for (int i = 0; i < ns; ++i) {
-      const float w = __shfl_sync(0xffffffffu, wi, i);
-#pragma unroll
-      for (int j = 0; j < kPer; ++j) acc[j] += w * __ldcg(po + i * HD + 32 * j);
-    }
-#pragma unroll
-    for (int j = 0; j < kPer; ++j) {
-      const int d = lane + 32 * j;
-      const float out = acc[j] * inv;
-      const __nv_bfloat16 hi = __float2bfloat16_rn(out);
-      mg.o_hi[hq * HD + d] = hi;
-      mg.o_lo[hq * HD + d] = __float2bfloat16_rn(out - __bfloat162float(hi));
-      if (mg.out_f32) mg.out_f32[hq * HD + d] = out;
-      if (mg.dbg) mg.dbg[hq * HD + d] = out;
-    }
-  }
 }
 
 // A fragments of one warp's query rows.
@@ -152,33 +112,61 @@ __device__ __forceinline__ void load_q(WarpQ<HD>& q, const __nv_bfloat16* __rest
   }
 }
 
+// Online-softmax state of one warp: per thread rows gid (and gid + 8 when two
+// rows) of the running maximum, the running sum and O.
+template <int HD>
+struct WarpState {
+  float m[2], l[2];
+  float o[HD / 8][4];
+  __device__ __forceinline__ void reset() {
+    m[0] = m[1] = -INFINITY;
+    l[0] = l[1] = 0.f;
+#pragma unroll
+    for (int n = 0; n < HD / 8; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
+  }
+};
+
 // Score one page (16 tokens, `valid` of them real) for one warp's query rows
-// and fold it into the online softmax state.
+// and fold it into the online softmax state.  The K fragments of the whole
+// page are loaded first and S is accumulated in four independent chains; O is
+// rescaled only when some row's maximum grew (the factor is exactly 1
+// otherwise).
 template <int HD, bool TWO_ROWS>
 __device__ __forceinline__ void process_page(const WarpQ<HD>& q, uint32_t kbase, uint32_t vbase, int valid, int lane,
-                                             float (&m_run)[2], float (&l_run)[2], float (&o)[HD / 8][4]) {
+                                             WarpState<HD>& st) {
   const int tig = lane & 3;
   const float sl2 = kLog2e * rsqrtf(static_cast<float>(HD));
   // S = Q K^T for the page's 16 tokens (two n-tiles of 8 tokens)
   float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
+  float t0[4] = {0.f, 0.f, 0.f, 0.f}, t1[4] = {0.f, 0.f, 0.f, 0.f};
   {
     const int mi = lane >> 3, r = lane & 7;
     const int tok = (mi >> 1) * 8 + r;
+    uint32_t kb[HD / 16][4];
 #pragma unroll
     for (int ks = 0; ks < HD / 16; ++ks) {
       const int hdc = ks * 16 + (mi & 1) * 8;
       const uint32_t addr = kbase + (hdc >> 6) * 2048 + tok * 128 + ((((hdc & 63) >> 3) ^ (tok & 7)) << 4);
-      uint32_t b0, b1, b2, b3;
-      ldsm_x4(addr, b0, b1, b2, b3);
-      mma_bf16_16816(s0, q.a0[ks], q.a1[ks], q.a2[ks], q.a3[ks], b0, b1);
-      mma_bf16_16816(s1, q.a0[ks], q.a1[ks], q.a2[ks], q.a3[ks], b2, b3);
+      ldsm_x4(addr, kb[ks][0], kb[ks][1], kb[ks][2], kb[ks][3]);
+    }
+#pragma unroll
+    for (int ks = 0; ks < HD / 16; ++ks) {
+      float(&d0)[4] = (ks & 1) ? t0 : s0;
+      float(&d1)[4] = (ks & 1) ? t1 : s1;
+      mma_bf16_16816(d0, q.a0[ks], q.a1[ks], q.a2[ks], q.a3[ks], kb[ks][0], kb[ks][1]);
+      mma_bf16_16816(d1, q.a0[ks], q.a1[ks], q.a2[ks], q.a3[ks], kb[ks][2], kb[ks][3]);
       if (TWO_ROWS) {
-        mma_bf16_16816(s0, q.b0[ks], q.b1[ks], q.b2[ks], q.b3[ks], b0, b1);
-        mma_bf16_16816(s1, q.b0[ks], q.b1[ks], q.b2[ks], q.b3[ks], b2, b3);
+        mma_bf16_16816(d0, q.b0[ks], q.b1[ks], q.b2[ks], q.b3[ks], kb[ks][0], kb[ks][1]);
+        mma_bf16_16816(d1, q.b0[ks], q.b1[ks], q.b2[ks], q.b3[ks], kb[ks][2], kb[ks][3]);
       }
     }
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      s0[i] += t0[i];
+      s1[i] += t1[i];
+    }
   }
-  const int t0 = tig * 2, t1 = tig * 2 + 1, t2 = 8 + tig * 2, t3 = 9 + tig * 2;
+  const int c0 = tig * 2, c1 = tig * 2 + 1, c2 = 8 + tig * 2, c3 = 9 + tig * 2;
   float x[2][4];
   if (!TWO_ROWS) {   // hi (row gid) + lo (row gid + 8) parts of the same head
     x[0][0] = s0[0] + s0[2];
@@ -198,44 +186,50 @@ __device__ __forceinline__ void process_page(const WarpQ<HD>& q, uint32_t kbase,
   uint32_t ph[4], pl[4];   // A fragments of P: hi / lo
 #pragma unroll
   for (int r = 0; r < (TWO_ROWS ? 2 : 1); ++r) {
-    x[r][0] = t0 < valid ? x[r][0] * sl2 : -INFINITY;
-    x[r][1] = t1 < valid ? x[r][1] * sl2 : -INFINITY;
-    x[r][2] = t2 < valid ? x[r][2] * sl2 : -INFINITY;
-    x[r][3] = t3 < valid ? x[r][3] * sl2 : -INFINITY;
+    x[r][0] = c0 < valid ? x[r][0] * sl2 : -INFINITY;
+    x[r][1] = c1 < valid ? x[r][1] * sl2 : -INFINITY;
+    x[r][2] = c2 < valid ? x[r][2] * sl2 : -INFINITY;
+    x[r][3] = c3 < valid ? x[r][3] * sl2 : -INFINITY;
     float mx = fmaxf(fmaxf(x[r][0], x[r][1]), fmaxf(x[r][2], x[r][3]));
     mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
     mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-    const float m_new = fmaxf(m_run[r], mx);
-    const float alpha = exp2f(m_run[r] - m_new);
+    const float m_new = fmaxf(st.m[r], mx);
+    if (__any_sync(0xffffffffu, m_new > st.m[r])) {   // warp-uniform: rescale O by 2^(m_old - m_new)
+      const float alpha = exp2f(st.m[r] - m_new);
+      st.l[r] *= alpha;
+      if (!TWO_ROWS) {   // one head per thread row: both MMA row halves rescale together
+#pragma unroll
+        for (int n = 0; n < HD / 8; ++n) {
+          st.o[n][0] *= alpha;
+          st.o[n][1] *= alpha;
+          st.o[n][2] *= alpha;
+          st.o[n][3] *= alpha;
+        }
+      } else {
+#pragma unroll
+        for (int n = 0; n < HD / 8; ++n) {
+          st.o[n][2 * r] *= alpha;
+          st.o[n][2 * r + 1] *= alpha;
+        }
+      }
+      st.m[r] = m_new;
+    }
     float p[4];
 #pragma unroll
     for (int i2 = 0; i2 < 4; ++i2) p[i2] = exp2f(x[r][i2] - m_new);
-    l_run[r] = l_run[r] * alpha + ((p[0] + p[1]) + (p[2] + p[3]));
-    m_run[r] = m_new;
+    st.l[r] += (p[0] + p[1]) + (p[2] + p[3]);
     float hi[4], lo[4];
 #pragma unroll
     for (int i2 = 0; i2 < 4; ++i2) {
       hi[i2] = __bfloat162float(__float2bfloat16_rn(p[i2]));
       lo[i2] = p[i2] - hi[i2];
     }
-    if (!TWO_ROWS) {   // one head per thread row: both MMA row halves rescale together
-#pragma unroll
-      for (int n = 0; n < HD / 8; ++n) {
-        o[n][0] *= alpha;
-        o[n][1] *= alpha;
-        o[n][2] *= alpha;
-        o[n][3] *= alpha;
-      }
+    if (!TWO_ROWS) {
       ph[0] = pack_bf16(hi[0], hi[1]);   // row gid: P_hi
       ph[1] = pack_bf16(lo[0], lo[1]);   // row gid + 8: P_lo
       ph[2] = pack_bf16(hi[2], hi[3]);
       ph[3] = pack_bf16(lo[2], lo[3]);
     } else {
-#pragma unroll
-      for (int n = 0; n < HD / 8; ++n) {
-        o[n][2 * r] *= alpha;
-        o[n][2 * r + 1] *= alpha;
-      }
       ph[r] = pack_bf16(hi[0], hi[1]);
       ph[r + 2] = pack_bf16(hi[2], hi[3]);
       pl[r] = pack_bf16(lo[0], lo[1]);
@@ -246,236 +240,412 @@ __device__ __forceinline__ void process_page(const WarpQ<HD>& q, uint32_t kbase,
   {
     const int mi = lane >> 3;
     const int tok = (mi & 1) * 8 + (lane & 7);
+    uint32_t vb[HD / 16][4];
 #pragma unroll
     for (int j2 = 0; j2 < HD / 16; ++j2) {
       const int hdc = j2 * 16 + (mi >> 1) * 8;
       const uint32_t addr = vbase + (hdc >> 6) * 2048 + tok * 128 + ((((hdc & 63) >> 3) ^ (tok & 7)) << 4);
-      uint32_t b0, b1, b2, b3;
-      ldsm_x4_t(addr, b0, b1, b2, b3);
-      mma_bf16_16816(o[2 * j2], ph[0], ph[1], ph[2], ph[3], b0, b1);
-      mma_bf16_16816(o[2 * j2 + 1], ph[0], ph[1], ph[2], ph[3], b2, b3);
+      ldsm_x4_t(addr, vb[j2][0], vb[j2][1], vb[j2][2], vb[j2][3]);
+    }
+#pragma unroll
+    for (int j2 = 0; j2 < HD / 16; ++j2) {
+      mma_bf16_16816(st.o[2 * j2], ph[0], ph[1], ph[2], ph[3], vb[j2][0], vb[j2][1]);
+      mma_bf16_16816(st.o[2 * j2 + 1], ph[0], ph[1], ph[2], ph[3], vb[j2][2], vb[j2][3]);
       if (TWO_ROWS) {
-        mma_bf16_16816(o[2 * j2], pl[0], pl[1], pl[2], pl[3], b0, b1);
-        mma_bf16_16816(o[2 * j2 + 1], pl[0], pl[1], pl[2], pl[3], b2, b3);
+        mma_bf16_16816(st.o[2 * j2], pl[0], pl[1], pl[2], pl[3], vb[j2][0], vb[j2][1]);
+        mma_bf16_16816(st.o[2 * j2 + 1], pl[0], pl[1], pl[2], pl[3], vb[j2][2], vb[j2][3]);
       }
     }
   }
 }
 
+// Shared-memory layout of the kernel (offsets from the 1024-aligned base).
+template <int HD>
+struct AttnSmem {
+  static constexpr uint32_t kBlockBytes = (HD / 64) * 16 * 128;   // one K (or V) page of one kv head
+  static constexpr uint32_t kPageBytes = 2 * kBlockBytes;
+  static constexpr uint32_t kStageBytes = kPagesPerStage * kPageBytes;
+  static constexpr uint32_t kRing = 0;
+  static constexpr uint32_t kMergeO = kStages * kStageBytes;                  // [8 warps][8 rows][HD] fp32
+  static constexpr uint32_t kMergeM = kMergeO + kConsumerWarps * 8 * HD * 4;  // [8][8] running max
+  static constexpr uint32_t kMergeL = kMergeM + kConsumerWarps * 8 * 4;       // [8][8] running sum
+  static constexpr uint32_t kBars = kMergeL + kConsumerWarps * 8 * 4;   // full[kStages], empty[kStages], seg_full, seg_free
+  static constexpr uint32_t kEnd = kBars + (2 * kStages + 2) * 8;
+  static constexpr size_t kDynamic = kEnd + 1024;   // + alignment slack
+};
+static_assert(AttnSmem<128>::kDynamic <= 227 * 1024, "attention shared memory exceeds the per-block limit");
+
 template <int HD, bool TWO_ROWS>
 __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
-    const __grid_constant__ CUtensorMap tm_pool, int64_t layer_row0, AttnWork wk,
+    const __grid_constant__ CUtensorMap tm_pool, int64_t layer_page0, AttnWork wk,
     const __nv_bfloat16* __restrict__ q_hi, const __nv_bfloat16* __restrict__ q_lo, int n_q, int n_kv, int group,
-    int stride, float* __restrict__ part_o, float* __restrict__ part_ml, AttnMerge mg, int* err,
-    unsigned long long* ts) {
+    float* __restrict__ part_o, float* __restrict__ part_ml, int* err, unsigned long long* ts) {
+  using SM = AttnSmem<HD>;
   trace_begin(ts);
-  constexpr int kSub = HD / 64;                       // 64-column sub-tiles per row
-  constexpr uint32_t kBlockBytes = kSub * 16 * 128;   // one K (or V) page of one kv head
-  constexpr uint32_t kPageBytes = 2 * kBlockBytes;
-  constexpr uint32_t kStageBytes = kPagesPerStage * kPageBytes;
 
   extern __shared__ uint8_t smem_raw[];
-  uint8_t* ring = align1024(smem_raw);
-  uint64_t* full = reinterpret_cast<uint64_t*>(ring + kStages * kStageBytes);
+  uint8_t* base = align1024(smem_raw);
+  uint8_t* ring = base + SM::kRing;
+  float* mo = reinterpret_cast<float*>(base + SM::kMergeO);
+  float* mm = reinterpret_cast<float*>(base + SM::kMergeM);
+  float* ml = reinterpret_cast<float*>(base + SM::kMergeL);
+  uint64_t* full = reinterpret_cast<uint64_t*>(base + SM::kBars);
   uint64_t* empty = full + kStages;
-  // no static shared memory: the dynamic request alone reaches the 227 KiB limit
-  int* s_last_p = reinterpret_cast<int*>(empty + kStages);   // 16 B: merge decision of this CTA
-  int32_t* pages_s = s_last_p + 4;
+  uint64_t* seg_full = empty + kStages;   // the 8 consumer warps' states of a private segment are in mo / mm / ml
+  uint64_t* seg_free = seg_full + 1;      // the merger has read them
 
-  const AttnItem it = wk.items[blockIdx.x];
-  const int g = blockIdx.y;
-  const bool shared = it.kind == 1;
-  const int np = it.n_pages;
+  const int seg0 = wk.cta_seg[blockIdx.x], seg1 = wk.cta_seg[blockIdx.x + 1];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int gid = lane >> 2, tig = lane & 3;
-
-  if (np == 0) {   // a candidate with an empty cache: the verify token attends to itself only
-    grid_dep_launch();
-    grid_dep_wait();
-    merge_group<HD>(it.cand, g, n_q, n_kv, group, 0, stride, part_o, part_ml, mg, 0, kThreads / 32);
-    trace_end(ts);
-    return;
-  }
-  const int n_stages = (np + kPagesPerStage - 1) / kPagesPerStage;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], kConsumerWarps);
     }
+    mbar_init(seg_full, kConsumerWarps);
+    mbar_init(seg_free, 1);
     fence_mbar_init();
   }
-  if (warp == kConsumerWarps)
-    for (int i = lane; i < np; i += 32) pages_s[i] = wk.pages[it.page_off + i];
   __syncthreads();
   grid_dep_launch();   // the next kernel may start; it waits for this grid before reading its output
 
-  float m_run[2] = {-INFINITY, -INFINITY};
-  float l_run[2] = {0.f, 0.f};
-  float o[HD / 8][4];
-#pragma unroll
-  for (int n = 0; n < HD / 8; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
-  int cand = shared ? -1 : it.cand;   // the candidate this warp scores
-
-  if (warp == kConsumerWarps) {
+  if (warp == kProducerWarp) {
     // ------------------------------------------------ producer
+    // One TMA box per page: K and V of kv head g (coordinates: column 0,
+    // token 0, sub-tile 0, head g, 2 * (layer * n_pages + page)).
     if (lane == 0) {
       tma_prefetch_desc(&tm_pool);
       const uint64_t pol = policy_evict_first();
-      for (int u = 0; u < n_stages; ++u) {
-        const int slot = u % kStages;
-        const uint32_t use = static_cast<uint32_t>(u / kStages);
-        if (u >= kStages && !mbar_wait(&empty[slot], (use & 1u) ^ 1u, err)) break;
-        const int npg = min(kPagesPerStage, np - u * kPagesPerStage);
-        mbar_arrive_expect_tx(&full[slot], static_cast<uint32_t>(npg) * kPageBytes);
-        uint8_t* st = ring + slot * kStageBytes;
-        for (int pi = 0; pi < npg; ++pi) {
-          const int64_t phys = pages_s[u * kPagesPerStage + pi];
-          const int32_t row_k = static_cast<int32_t>(layer_row0 + (phys * 2 * n_kv + g) * 16);
-          const int32_t row_v = row_k + n_kv * 16;
+      uint32_t u = 0;   // stage sequence number over all segments
+      bool ok = true;
+      for (int si = seg0; si < seg1 && ok; ++si) {
+        const AttnSeg sg = wk.segs[si];
+        const int32_t* pg = wk.pages + sg.page_off;
+        for (int p0 = 0; p0 < sg.n_pages; p0 += kPagesPerStage, ++u) {
+          const int slot = static_cast<int>(u % kStages);
+          if (u >= static_cast<uint32_t>(kStages) &&
+              !mbar_wait(&empty[slot], ((u / kStages) & 1u) ^ 1u, err)) {
+            ok = false;
+            break;
+          }
+          const int npg = min(kPagesPerStage, sg.n_pages - p0);
+          mbar_arrive_expect_tx(&full[slot], static_cast<uint32_t>(npg) * SM::kPageBytes);
+          uint8_t* stg = ring + slot * SM::kStageBytes;
+          for (int pi = 0; pi < npg; ++pi) {
+            const int64_t phys = __ldg(pg + p0 + pi);
+            tma_load_5d(stg + pi * SM::kPageBytes, &tm_pool, &full[slot], 0, 0, 0, sg.g,
+                        static_cast<int32_t>(2 * (layer_page0 + phys)), pol);
+          }
+        }
+      }
+      // Every copy issued above has landed once the consumers released the
+      // last stages (each slot's latest phase); a lost arrival times out.
+      if (ok)
+        for (uint32_t v = u > static_cast<uint32_t>(kStages) ? u - kStages : 0; v < u; ++v)
+          if (!mbar_wait(&empty[v % kStages], (v / kStages) & 1u, err)) break;
+    }
+  } else if (warp < kConsumerWarps) {
+    // ------------------------------------------------ consumers
+    // Every warp waits for every stage before releasing it, busy or not, so
+    // no warp can arrive for a slot's next use early.
+    grid_dep_wait();   // q is written by the preceding kernel
+    bool ok = true;
+    uint32_t u = 0, n_priv = 0;
+    for (int si = seg0; si < seg1; ++si) {
+      const AttnSeg sg = wk.segs[si];
+      const bool shared = sg.kind == 1;
+      // the candidate this warp scores in this segment, -1 if none
+      const int cand = shared ? (warp < sg.n_cands ? wk.cands[sg.cand + warp] : -1)
+                              : (warp < sg.n_pages ? sg.cand : -1);
+      WarpQ<HD> q;
+      if (cand >= 0) {
+        const int64_t q0 = (static_cast<int64_t>(cand) * n_q + static_cast<int64_t>(sg.g) * group) * HD;
+        load_q<HD, TWO_ROWS>(q, q_hi + q0, q_lo + q0, group, lane);
+      }
+      WarpState<HD> st;
+      st.reset();
+      for (int p0 = 0; p0 < sg.n_pages; p0 += kPagesPerStage, ++u) {
+        const int slot = static_cast<int>(u % kStages);
+        if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&full[slot], (u / kStages) & 1u, err));
+        if (ok && cand >= 0) {
+          const uint32_t sbase = smem_u32(ring + slot * SM::kStageBytes);
+          const int npg = min(kPagesPerStage, sg.n_pages - p0);
+          if (!shared) {   // page `warp` of this stage
+            if (warp < npg) {
+              const int valid = p0 + warp == sg.n_pages - 1 ? sg.last_valid : 16;
+              const uint32_t kb = sbase + warp * SM::kPageBytes;
+              process_page<HD, TWO_ROWS>(q, kb, kb + SM::kBlockBytes, valid, lane, st);
+            }
+          } else {         // every page of this stage, for this warp's candidate
+            for (int pi = 0; pi < npg; ++pi) {
+              const int valid = p0 + pi == sg.n_pages - 1 ? sg.last_valid : 16;
+              const uint32_t kb = sbase + pi * SM::kPageBytes;
+              process_page<HD, TWO_ROWS>(q, kb, kb + SM::kBlockBytes, valid, lane, st);
+            }
+          }
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty[slot]);
+      }
+      if (cand >= 0 && ok) {
+        if (!TWO_ROWS) {   // fold the lo-part rows onto their heads
 #pragma unroll
-          for (int sub = 0; sub < kSub; ++sub) {
-            tma_load_2d(st + pi * kPageBytes + sub * 2048, &tm_pool, &full[slot], sub * 64, row_k, pol);
-            tma_load_2d(st + pi * kPageBytes + kBlockBytes + sub * 2048, &tm_pool, &full[slot], sub * 64, row_v,
-                        pol);
+          for (int n = 0; n < HD / 8; ++n) {
+            st.o[n][0] += st.o[n][2];
+            st.o[n][1] += st.o[n][3];
+          }
+        }
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {   // quad-reduce the row sums
+          st.l[r] += __shfl_xor_sync(0xffffffffu, st.l[r], 1);
+          st.l[r] += __shfl_xor_sync(0xffffffffu, st.l[r], 2);
+        }
+      }
+      if (!shared && !TWO_ROWS) {
+        // hand the warp's state to the merger warp (one slot per private
+        // segment); wait only until it has read the previous segment's states
+        if (n_priv > 0) ok = __all_sync(0xffffffffu, mbar_wait(seg_free, (n_priv - 1) & 1u, err)) && ok;
+        if (cand >= 0 && ok) {
+          if (gid < group) {
+#pragma unroll
+            for (int n = 0; n < HD / 8; ++n)
+              *reinterpret_cast<float2*>(mo + (warp * 8 + gid) * HD + n * 8 + tig * 2) =
+                  make_float2(st.o[n][0], st.o[n][1]);
+            if (tig == 0) {
+              mm[warp * 8 + gid] = st.m[0];
+              ml[warp * 8 + gid] = st.l[0];
+            }
+          }
+        } else if (lane < 8) {
+          mm[warp * 8 + lane] = -INFINITY;   // nothing scored by this warp
+          ml[warp * 8 + lane] = 0.f;
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(seg_full);
+        ++n_priv;
+      } else if (cand >= 0 && ok) {
+        // this warp's own partial slot
+        const int slot_id = shared ? wk.slots[sg.slot + warp] : sg.slot + warp;
+#pragma unroll
+        for (int r = 0; r < (TWO_ROWS ? 2 : 1); ++r) {
+          const int row = gid + 8 * r;
+          if (row < group) {
+            const int64_t pr = static_cast<int64_t>(slot_id) * group + row;
+            float* dst = part_o + pr * HD;
+#pragma unroll
+            for (int n = 0; n < HD / 8; ++n)
+              *reinterpret_cast<float2*>(dst + n * 8 + tig * 2) = make_float2(st.o[n][2 * r], st.o[n][2 * r + 1]);
+            if (tig == 0) *reinterpret_cast<float2*>(part_ml + pr * 2) = make_float2(st.m[r], st.l[r]);
           }
         }
       }
     }
-  } else {
-    // ------------------------------------------------ consumers
-    if (shared) cand = warp < it.n_cands ? wk.cands[it.cand + warp] : -1;
-    grid_dep_wait();   // q is written by the preceding kernel
-    WarpQ<HD> q;
-    if (cand >= 0) {
-      const int64_t q0 = (static_cast<int64_t>(cand) * n_q + static_cast<int64_t>(g) * group) * HD;
-      load_q<HD, TWO_ROWS>(q, q_hi + q0, q_lo + q0, group, lane);
-    }
-    for (int u = 0; u < n_stages; ++u) {
-      const int slot = u % kStages;
-      const uint32_t use = static_cast<uint32_t>(u / kStages);
-      if (!__all_sync(0xffffffffu, mbar_wait(&full[slot], use & 1u, err))) break;
-      const uint32_t sbase = smem_u32(ring + slot * kStageBytes);
-      const int npg = min(kPagesPerStage, np - u * kPagesPerStage);
-      if (!shared) {   // page `warp` of this stage
-        if (warp < npg) {
-          const int pg = u * kPagesPerStage + warp;
-          const int valid = pg == np - 1 ? it.last_valid : 16;
-          const uint32_t kb = sbase + warp * kPageBytes;
-          process_page<HD, TWO_ROWS>(q, kb, kb + kBlockBytes, valid, lane, m_run, l_run, o);
-        }
-      } else if (cand >= 0) {   // every page of this stage, for this warp's candidate
-        for (int pi = 0; pi < npg; ++pi) {
-          const int pg = u * kPagesPerStage + pi;
-          const int valid = pg == np - 1 ? it.last_valid : 16;
-          const uint32_t kb = sbase + pi * kPageBytes;
-          process_page<HD, TWO_ROWS>(q, kb, kb + kBlockBytes, valid, lane, m_run, l_run, o);
+  } else if (warp == kMergerWarp && !TWO_ROWS) {
+    // ------------------------------------------------ merger
+    // For every private segment, in order: fold the eight consumer warps'
+    // (m, l, O) into the segment's partial slot,
+    //   M = max_w m_w, L = sum_w 2^(m_w - M) l_w, O = sum_w 2^(m_w - M) O_w.
+    constexpr int kPer = HD / 32;
+    uint32_t k = 0;
+    bool ok = true;
+    for (int si = seg0; si < seg1; ++si) {
+      const AttnSeg sg = wk.segs[si];
+      if (sg.kind != 0) continue;
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(seg_full, k & 1u, err));
+      if (ok) {
+        for (int r = 0; r < group; ++r) {
+          float mw[kConsumerWarps], M = -INFINITY;
+#pragma unroll
+          for (int w = 0; w < kConsumerWarps; ++w) {
+            mw[w] = mm[w * 8 + r];
+            M = fmaxf(M, mw[w]);
+          }
+          float acc[kPer], L = 0.f;
+#pragma unroll
+          for (int j = 0; j < kPer; ++j) acc[j] = 0.f;
+#pragma unroll
+          for (int w = 0; w < kConsumerWarps; ++w) {
+            if (mw[w] == -INFINITY) continue;   // an idle warp: its O rows are not written
+            const float f = exp2f(mw[w] - M);
+            L += f * ml[w * 8 + r];
+#pragma unroll
+            for (int j = 0; j < kPer; ++j) acc[j] += f * mo[(w * 8 + r) * HD + lane + 32 * j];
+          }
+          const int64_t pr = static_cast<int64_t>(sg.slot) * group + r;
+#pragma unroll
+          for (int j = 0; j < kPer; ++j) part_o[pr * HD + lane + 32 * j] = acc[j];
+          if (lane == 0) *reinterpret_cast<float2*>(part_ml + pr * 2) = make_float2(M, L);
         }
       }
       __syncwarp();
-      if (lane == 0) mbar_arrive(&empty[slot]);
-    }
-    if (!TWO_ROWS) {   // fold the lo-part rows onto their heads
-#pragma unroll
-      for (int n = 0; n < HD / 8; ++n) {
-        o[n][0] += o[n][2];
-        o[n][1] += o[n][3];
-      }
-    }
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {   // quad-reduce the row sums
-      l_run[r] += __shfl_xor_sync(0xffffffffu, l_run[r], 1);
-      l_run[r] += __shfl_xor_sync(0xffffffffu, l_run[r], 2);
+      if (lane == 0) mbar_arrive(seg_free);
+      ++k;
     }
   }
-  // all stages consumed (every issued copy was waited for)
-  __syncthreads();
-  grid_dep_wait();
+  trace_end(ts);
+}
 
-  if (shared) {
-    // each consumer warp owns one candidate's partial
-    if (warp < kConsumerWarps && cand >= 0) {
-      const int slot_id = wk.slots[it.slot + warp];
+// The combine: one CTA per (candidate, kv head), W warps.  Warp w folds slots
+// w, w + W, ... (U at a time, every load of those issued before the first
+// use) into a running (M, L, O) per query head of the group; the warps' states
+// and the verify token's own entry are then merged through shared memory:
+//   M* = max(s_self, M_w), o = (2^(s_self - M*) v_self + sum_w 2^(M_w - M*) O_w)
+//                              / (2^(s_self - M*) + sum_w 2^(M_w - M*) L_w).
+// W and U keep the per-thread state within the register budget of W warps.
+template <int HD, int ROWS>
+struct CombineShape {
+  static constexpr int W = 8;                               // warps
+  static constexpr int U = HD * ROWS <= 512 ? 2 : 1;        // slots in flight per warp
+  static constexpr size_t kAcc = 0;                                         // [W][ROWS][HD]
+  static constexpr size_t kM = kAcc + sizeof(float) * W * ROWS * HD;        // [W][ROWS]
+  static constexpr size_t kL = kM + sizeof(float) * W * ROWS;               // [W][ROWS]
+  static constexpr size_t kSelf = kL + sizeof(float) * W * ROWS;            // [ROWS]
+  static constexpr size_t kBytes = kSelf + sizeof(float) * ROWS;
+};
+
+template <int HD, int ROWS>
+__global__ void __launch_bounds__(CombineShape<HD, ROWS>::W * 32) attn_combine_kernel(
+    const int32_t* __restrict__ slot_base, const int32_t* __restrict__ nslots, int n_q, int n_kv, int group,
+    const float* __restrict__ part_o, const float* __restrict__ part_ml, AttnMerge mg, unsigned long long* ts) {
+  using CS = CombineShape<HD, ROWS>;
+  constexpr int kPer = HD / 32, W = CS::W, U = CS::U;
+  constexpr int kOut = (ROWS * HD + W * 32 - 1) / (W * 32);   // outputs per thread in the final phase
+  trace_begin(ts);
+  grid_dep_launch();
+  extern __shared__ __align__(16) uint8_t csm[];
+  float* s_acc = reinterpret_cast<float*>(csm + CS::kAcc);
+  float* s_m = reinterpret_cast<float*>(csm + CS::kM);
+  float* s_l = reinterpret_cast<float*>(csm + CS::kL);
+  float* s_self = reinterpret_cast<float*>(csm + CS::kSelf);
+  const int cg = blockIdx.x, b = cg / n_kv, g = cg - b * n_kv;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int64_t hq0 = static_cast<int64_t>(b) * n_q + static_cast<int64_t>(g) * group;
+  const int64_t hk = static_cast<int64_t>(b) * n_kv + g;
+  const int first = slot_base[cg], ns = nslots[cg];   // host-uploaded before the call: no wait needed
+
+  grid_dep_wait();   // the partials (and q, k_self, v_self) are written by earlier kernels
+  // Every global load of the first round is issued before any is used: this
+  // warp's first U slots, the q / k_self rows of head `warp` and this thread's
+  // v_self values for the final phase.
+  float2 ml[U];
+  float v[U][ROWS][kPer];
 #pragma unroll
-      for (int r = 0; r < (TWO_ROWS ? 2 : 1); ++r) {
-        const int row = gid + 8 * r;
-        if (row < group) {
-          const int64_t hq = static_cast<int64_t>(cand) * n_q + static_cast<int64_t>(g) * group + row;
-          float* dst = part_o + (hq * stride + slot_id) * HD;
+  for (int k = 0; k < U; ++k) {
+    const int sk = warp + k * W;
+    const int64_t pr = (static_cast<int64_t>(first) + (sk < ns ? sk : 0)) * group;
+    ml[k] = (sk < ns && lane < group) ? __ldcg(reinterpret_cast<const float2*>(part_ml + (pr + lane) * 2))
+                                      : make_float2(-INFINITY, 0.f);
 #pragma unroll
-          for (int n = 0; n < HD / 8; ++n) {
-            dst[n * 8 + tig * 2] = o[n][2 * r];
-            dst[n * 8 + tig * 2 + 1] = o[n][2 * r + 1];
-          }
-          if (tig == 0) {
-            part_ml[(hq * stride + slot_id) * 2 + 0] = m_run[r];
-            part_ml[(hq * stride + slot_id) * 2 + 1] = l_run[r];
-          }
-        }
+    for (int r = 0; r < ROWS; ++r)
+#pragma unroll
+      for (int j = 0; j < kPer; ++j)
+        v[k][r][j] = (sk < ns && r < group) ? __ldcg(part_o + (pr + r) * HD + lane + 32 * j) : 0.f;
+  }
+  float qd[kPer], kd[kPer];
+#pragma unroll
+  for (int j = 0; j < kPer; ++j) {
+    qd[j] = warp < group ? mg.q[(hq0 + warp) * HD + lane + 32 * j] : 0.f;
+    kd[j] = warp < group ? mg.kself[hk * HD + lane + 32 * j] : 0.f;
+  }
+  float vsf[kOut];
+#pragma unroll
+  for (int i = 0; i < kOut; ++i) {
+    const int idx = threadIdx.x + i * W * 32;
+    vsf[i] = idx < group * HD ? mg.vself[hk * HD + idx % HD] : 0.f;
+  }
+  // the verify token's own score of head `warp`
+  if (warp < group) {
+    float dot = 0.f;
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) dot += qd[j] * kd[j];
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
+    if (lane == 0) s_self[warp] = dot * (kLog2e * rsqrtf(static_cast<float>(HD)));
+  }
+  for (int r = warp + W; r < group; r += W) {   // heads beyond the warp count (G > W; k_self is loaded by all)
+    float dot = 0.f;
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) dot += mg.q[(hq0 + r) * HD + lane + 32 * j] * kd[j];
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
+    if (lane == 0) s_self[r] = dot * (kLog2e * rsqrtf(static_cast<float>(HD)));
+  }
+  float M[ROWS], L[ROWS], acc[ROWS][kPer];
+#pragma unroll
+  for (int r = 0; r < ROWS; ++r) {
+    M[r] = -INFINITY;
+    L[r] = 0.f;
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) acc[r][j] = 0.f;
+  }
+  for (int s0 = warp;; s0 += U * W) {
+#pragma unroll
+    for (int k = 0; k < U; ++k)
+#pragma unroll
+      for (int r = 0; r < ROWS; ++r) {
+        const float mr = __shfl_sync(0xffffffffu, ml[k].x, r), lr = __shfl_sync(0xffffffffu, ml[k].y, r);
+        if (mr == -INFINITY) continue;   // past the last slot (warp-uniform)
+        const float Mn = fmaxf(M[r], mr);
+        const float sc = exp2f(M[r] - Mn), wv = exp2f(mr - Mn);
+        L[r] = L[r] * sc + wv * lr;
+#pragma unroll
+        for (int j = 0; j < kPer; ++j) acc[r][j] = acc[r][j] * sc + wv * v[k][r][j];
+        M[r] = Mn;
       }
-      __threadfence();
-      __syncwarp();
-      int last = 0;
-      if (lane == 0) last = atomicAdd(&mg.counter[cand * n_kv + g], 1) == wk.nslots[cand] - 1;
-      last = __shfl_sync(0xffffffffu, last, 0);
-      if (last) {
-        __threadfence();
-        merge_group<HD>(cand, g, n_q, n_kv, group, wk.nslots[cand], stride, part_o, part_ml, mg, warp, 1);
-        if (lane == 0) mg.counter[cand * n_kv + g] = 0;   // ready for the next layer
+    if (s0 + U * W >= ns) break;
+    // the next round of slots (more than U * W slots only)
+#pragma unroll
+    for (int k = 0; k < U; ++k) {
+      const int sk = s0 + U * W + k * W;
+      const int64_t pr = (static_cast<int64_t>(first) + (sk < ns ? sk : 0)) * group;
+      ml[k] = (sk < ns && lane < group) ? __ldcg(reinterpret_cast<const float2*>(part_ml + (pr + lane) * 2))
+                                        : make_float2(-INFINITY, 0.f);
+#pragma unroll
+      for (int r = 0; r < ROWS; ++r)
+#pragma unroll
+        for (int j = 0; j < kPer; ++j)
+          v[k][r][j] = (sk < ns && r < group) ? __ldcg(part_o + (pr + r) * HD + lane + 32 * j) : 0.f;
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < ROWS; ++r) {
+    if (r < group) {
+#pragma unroll
+      for (int j = 0; j < kPer; ++j) s_acc[(warp * ROWS + r) * HD + lane + 32 * j] = acc[r][j];
+      if (lane == 0) {
+        s_m[warp * ROWS + r] = M[r];
+        s_l[warp * ROWS + r] = L[r];
       }
     }
-  } else {
-    // merge the eight warps' states through shared memory into one partial
-    float* mo = reinterpret_cast<float*>(ring);                 // [8][16][HD]
-    float* mm = mo + kConsumerWarps * 16 * HD;                  // [8][16]
-    float* ml = mm + kConsumerWarps * 16;                       // [8][16]
-    if (warp < kConsumerWarps) {
+  }
+  __syncthreads();
 #pragma unroll
-      for (int r = 0; r < (TWO_ROWS ? 2 : 1); ++r) {
-        const int row = gid + 8 * r;
-        if (row < group) {
+  for (int i = 0; i < kOut; ++i) {
+    const int idx = threadIdx.x + i * W * 32;
+    if (idx >= group * HD) break;
+    const int r = idx / HD, d = idx - r * HD;
+    const float ss = s_self[r];
+    float Mt = ss;
 #pragma unroll
-          for (int n = 0; n < HD / 8; ++n) {
-            mo[(warp * 16 + row) * HD + n * 8 + tig * 2] = o[n][2 * r];
-            mo[(warp * 16 + row) * HD + n * 8 + tig * 2 + 1] = o[n][2 * r + 1];
-          }
-          if (tig == 0) {
-            mm[warp * 16 + row] = m_run[r];
-            ml[warp * 16 + row] = l_run[r];
-          }
-        }
-      }
+    for (int w = 0; w < W; ++w) Mt = fmaxf(Mt, s_m[w * ROWS + r]);
+    const float ws = exp2f(ss - Mt);
+    float num = ws * vsf[i], den = ws;
+#pragma unroll
+    for (int w = 0; w < W; ++w) {
+      const float mw = s_m[w * ROWS + r];
+      if (mw == -INFINITY) continue;
+      const float f = exp2f(mw - Mt);
+      num += f * s_acc[(w * ROWS + r) * HD + d];
+      den += f * s_l[w * ROWS + r];
     }
-    __syncthreads();
-    for (int idx = threadIdx.x; idx < group * HD; idx += kThreads) {
-      const int row = idx / HD, d = idx - row * HD;
-      float M = -INFINITY;
-#pragma unroll
-      for (int w = 0; w < kConsumerWarps; ++w) M = fmaxf(M, mm[w * 16 + row]);
-      float acc = 0.f, lsum = 0.f;
-#pragma unroll
-      for (int w = 0; w < kConsumerWarps; ++w) {
-        const float mw = mm[w * 16 + row];
-        const float f = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
-        acc += f * mo[(w * 16 + row) * HD + d];
-        lsum += f * ml[w * 16 + row];
-      }
-      const int64_t hq = static_cast<int64_t>(cand) * n_q + static_cast<int64_t>(g) * group + row;
-      part_o[(hq * stride + it.slot) * HD + d] = acc;
-      if (d == 0) {
-        part_ml[(hq * stride + it.slot) * 2 + 0] = M;
-        part_ml[(hq * stride + it.slot) * 2 + 1] = lsum;
-      }
-    }
-    __threadfence();
-    __syncthreads();
-    if (threadIdx.x == 0) *s_last_p = atomicAdd(&mg.counter[cand * n_kv + g], 1) == wk.nslots[cand] - 1;
-    __syncthreads();
-    if (*s_last_p) {
-      __threadfence();
-      merge_group<HD>(cand, g, n_q, n_kv, group, wk.nslots[cand], stride, part_o, part_ml, mg, 0, kThreads / 32);
-      if (threadIdx.x == 0) mg.counter[cand * n_kv + g] = 0;   // ready for the next layer
-    }
+    const float out = num / den;
+    const int64_t o = (hq0 + r) * HD + d;
+    const __nv_bfloat16 hi = __float2bfloat16_rn(out);
+    mg.o_hi[o] = hi;
+    mg.o_lo[o] = __float2bfloat16_rn(out - __bfloat162float(hi));
+    if (mg.out_f32) mg.out_f32[o] = out;
+    if (mg.dbg) mg.dbg[o] = out;
   }
   trace_end(ts);
 }
@@ -488,8 +658,8 @@ __global__ void resolve_kernel(const int32_t* __restrict__ bt, const int32_t* __
 }
 
 template <typename K>
-cudaError_t set_smem(K kernel) {
-  return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+cudaError_t set_smem(K kernel, size_t bytes) {
+  return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
 }
 
 uint64_t hash_list(const int32_t* v, int n) {
@@ -498,40 +668,84 @@ uint64_t hash_list(const int32_t* v, int n) {
     h ^= static_cast<uint32_t>(v[i]);
     h *= 1099511628211ull;
   }
-  return h ^ static_cast<uint64_t>(n);
+  return h;
 }
+
+// A run of pages scored together: one candidate's private pages, or pages
+// shared by one chunk (<= 8) of a candidate set.
+struct Run {
+  int kind;
+  int cand;        // kind 0: candidate; kind 1: offset into cands
+  int n_cands;
+  int page_off;    // offset into pages
+  int n_pages;
+  int last_valid;
+  int64_t cost;    // per page and kv head
+};
 
 }  // namespace
 
-size_t attention_smem_bytes(int hd, int max_item_pages) {
-  const size_t stage = static_cast<size_t>(kPagesPerStage) * 2 * (hd / 64) * 2048;
-  return kStages * stage + 1024 + 2 * kStages * 8 + 16 + static_cast<size_t>(max_item_pages) * 4 + 64;
+CUresult encode_pool_map(PFN_cuTensorMapEncodeTiled_v12000 encode, CUtensorMap* map, const void* pool,
+                         int64_t page_units, int n_kv, int hd) {
+  const cuuint64_t row = static_cast<cuuint64_t>(hd) * 2;   // bytes per token row
+  cuuint64_t dims[5] = {64, 16, static_cast<cuuint64_t>(hd / 64), static_cast<cuuint64_t>(n_kv),
+                        static_cast<cuuint64_t>(page_units) * 2};
+  cuuint64_t strides[4] = {row, 128, 16 * row, static_cast<cuuint64_t>(n_kv) * 16 * row};
+  cuuint32_t box[5] = {64, 16, static_cast<cuuint32_t>(hd / 64), 1, 2};
+  cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+  return encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(pool), dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
-int attention_max_item_pages(int hd) {
-  const size_t fixed = attention_smem_bytes(hd, 0);
-  return static_cast<int>((227 * 1024 - fixed) / 4);
+size_t attention_smem_bytes(int hd) {
+  return hd == 128 ? AttnSmem<128>::kDynamic : AttnSmem<64>::kDynamic;
 }
 
-// Host planner: split each candidate's private pages into items, and group the
-// full pages that several candidates reference (each exactly once) by their
-// exact candidate set into shared items of up to kConsumerWarps candidates.
-// Items are sized so that about two waves of CTAs (one per SM) cover the work,
-// counting a shared page as kConsumerWarps times the per-CTA work of a private
-// one (every warp scores every page of a shared item).  Returns false when some
-// candidate would need more than slot_cap partial slots at any item size.
-bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks, int n_kv, int hd, int num_sms,
-                     int slot_cap, bool share, AttnWorkHost& w) {
-  const int max_pages_item = attention_max_item_pages(hd);
+size_t attn_slot_capacity(int max_candidates, int n_kv, int num_sms) {
+  // private runs: at most B * n_kv + n_ctas segments of at most 8 slots each
+  return static_cast<size_t>(kConsumerWarps) * 2 * (static_cast<size_t>(max_candidates) * n_kv + num_sms);
+}
+
+// Host planner.
+//  1. Shared pages: full pages that >= 2 candidates reference, each exactly
+//     once, grouped by their exact candidate set; each set is cut into chunks
+//     of <= 8 candidates, one run per chunk.  Every other page of a candidate
+//     goes to its private run.
+//  2. The (run, kv head) pairs are laid end to end on a cost axis (a page
+//     costs kPrivateCost, or kSharedCostPerCand per candidate) and each page goes to the CTA whose
+//     equal share of the axis holds the page's midpoint; the pages of a pair
+//     that fall to one CTA form a segment.  A private segment adds one
+//     partial slot (with G > 8 one per warp that gets a page, page i going
+//     to warp i mod 8); a shared segment adds one per candidate.
+//  3. The slots of each (candidate, kv head) are numbered consecutively from
+//     slot_base.
+// Falls back to private runs when sharing would need more than slot_limit
+// slots; returns false if even those do not fit.
+bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks, int n_kv, int group, int n_ctas,
+                     size_t slot_limit, bool share, AttnWorkHost& w) {
+  w.segs.clear();
+  w.cta_seg.clear();
+  w.pages.clear();
+  w.cands.clear();
+  w.slots.clear();
+  w.slot_base.assign(static_cast<size_t>(n) * n_kv, 0);
+  w.nslots.assign(static_cast<size_t>(n) * n_kv, 0);
+  w.n_slots = 0;
+  w.n_ctas = 0;
+  if (n <= 0) {
+    w.cta_seg.push_back(0);
+    return true;
+  }
   std::vector<int> np(n);
   int64_t total_refs = 0;
   for (int b = 0; b < n; ++b) {
     np[b] = (sl[b] + 15) / 16;
     total_refs += np[b];
   }
-  // ---- shared pages: full pages referenced once each by >= 2 candidates
+  // ---- 1. runs
   std::vector<uint8_t> is_shared(static_cast<size_t>(n) * max_blocks, 0);
-  std::vector<std::vector<int32_t>> group_cands, group_pages;
+  std::vector<Run> runs;
   if (share && total_refs > 0) {
     std::unordered_map<int32_t, std::vector<int32_t>> refs;   // page -> candidates (full refs)
     refs.reserve(static_cast<size_t>(total_refs));
@@ -545,6 +759,7 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
       }
     }
     if (any_dup) {
+      std::vector<std::vector<int32_t>> group_cands, group_pages;
       std::unordered_map<uint64_t, int> gidx;
       std::unordered_map<int32_t, char> in_group;
       for (auto& kv : refs) {
@@ -575,154 +790,189 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
           if (in_group.count(bt[static_cast<int64_t>(b) * max_blocks + j]))
             is_shared[static_cast<size_t>(b) * max_blocks + j] = 1;
       }
-      for (auto& pgs : group_pages) std::sort(pgs.begin(), pgs.end());   // deterministic item contents
-      // deterministic group order (the hash map's iteration order is not)
-      std::vector<int> order(group_cands.size());
+      for (auto& pgs : group_pages) std::sort(pgs.begin(), pgs.end());   // deterministic contents
+      std::vector<int> order(group_cands.size());   // deterministic group order
       for (size_t i = 0; i < order.size(); ++i) order[i] = static_cast<int>(i);
-      std::sort(order.begin(), order.end(), [&](int a, int b2) {
-        return group_pages[a].front() < group_pages[b2].front();
-      });
-      std::vector<std::vector<int32_t>> gc, gp;
-      for (int i : order) {
-        gc.push_back(std::move(group_cands[i]));
-        gp.push_back(std::move(group_pages[i]));
-      }
-      group_cands.swap(gc);
-      group_pages.swap(gp);
-    }
-  }
-  // ---- cost model and item sizes
-  int64_t priv_pages = 0, shared_units = 0;
-  for (int b = 0; b < n; ++b)
-    for (int j = 0; j < np[b]; ++j) priv_pages += is_shared[static_cast<size_t>(b) * max_blocks + j] ? 0 : 1;
-  for (size_t gi = 0; gi < group_cands.size(); ++gi) {
-    const int64_t chunks = (static_cast<int64_t>(group_cands[gi].size()) + kConsumerWarps - 1) / kConsumerWarps;
-    shared_units += chunks * static_cast<int64_t>(group_pages[gi].size()) * kConsumerWarps;
-  }
-  const int64_t total = (priv_pages + shared_units) * n_kv;
-  const int64_t target_ctas = 2LL * num_sms;
-  int64_t unit = total / (target_ctas > 0 ? target_ctas : 1);   // private pages per item
-  if (unit < kPagesPerStage) unit = kPagesPerStage;
-  for (int attempt = 0; attempt < 20; ++attempt, unit *= 2) {
-    w.items.clear();
-    w.pages.clear();
-    w.cands.clear();
-    w.slots.clear();
-    w.nslots.assign(n, 0);
-    const int64_t priv_split =
-        std::min<int64_t>(max_pages_item, (unit + kPagesPerStage - 1) / kPagesPerStage * kPagesPerStage);
-    const int64_t shared_split = std::min<int64_t>(max_pages_item, std::max<int64_t>(1, unit / kConsumerWarps));
-    bool ok = true;
-    // shared items first: they are the longest per CTA
-    for (size_t gi = 0; gi < group_cands.size() && ok; ++gi) {
-      const auto& c = group_cands[gi];
-      const auto& pg = group_pages[gi];
-      for (size_t c0 = 0; c0 < c.size(); c0 += kConsumerWarps) {
-        const int nc = static_cast<int>(std::min<size_t>(kConsumerWarps, c.size() - c0));
-        for (size_t p0 = 0; p0 < pg.size(); p0 += static_cast<size_t>(shared_split)) {
-          const int npg = static_cast<int>(std::min<size_t>(static_cast<size_t>(shared_split), pg.size() - p0));
-          AttnItem it{};
-          it.kind = 1;
-          it.cand = static_cast<int32_t>(w.cands.size());
-          it.n_cands = nc;
-          it.page_off = static_cast<int32_t>(w.pages.size());
-          it.n_pages = npg;
-          it.last_valid = 16;
-          it.slot = static_cast<int32_t>(w.slots.size());
-          for (int k = 0; k < nc; ++k) {
-            const int b = c[c0 + k];
-            w.cands.push_back(b);
-            w.slots.push_back(w.nslots[b]++);
-            if (w.nslots[b] > slot_cap) ok = false;
-          }
-          w.pages.insert(w.pages.end(), pg.begin() + p0, pg.begin() + p0 + npg);
-          w.items.push_back(it);
+      std::sort(order.begin(), order.end(),
+                [&](int a, int b2) { return group_pages[a].front() < group_pages[b2].front(); });
+      for (int gi : order) {
+        const auto& c = group_cands[gi];
+        const auto& pg = group_pages[gi];
+        const int page_off = static_cast<int>(w.pages.size());
+        w.pages.insert(w.pages.end(), pg.begin(), pg.end());
+        for (size_t c0 = 0; c0 < c.size(); c0 += kConsumerWarps) {
+          Run r;
+          r.kind = 1;
+          r.cand = static_cast<int>(w.cands.size());
+          r.n_cands = static_cast<int>(std::min<size_t>(kConsumerWarps, c.size() - c0));
+          r.page_off = page_off;
+          r.n_pages = static_cast<int>(pg.size());
+          r.last_valid = 16;
+          r.cost = kSharedCostPerCand * r.n_cands;
+          w.cands.insert(w.cands.end(), c.begin() + c0, c.begin() + c0 + r.n_cands);
+          runs.push_back(r);
         }
       }
     }
-    for (int b = 0; b < n && ok; ++b) {
-      std::vector<int32_t> priv;
-      for (int j = 0; j < np[b]; ++j)
-        if (!is_shared[static_cast<size_t>(b) * max_blocks + j])
-          priv.push_back(bt[static_cast<int64_t>(b) * max_blocks + j]);
-      const int last_valid_b = np[b] > 0 ? sl[b] - 16 * (np[b] - 1) : 16;
-      const bool last_private = np[b] > 0 && !is_shared[static_cast<size_t>(b) * max_blocks + np[b] - 1];
-      if (priv.empty()) {
-        if (np[b] == 0) {   // empty cache: an item with no pages merges the self entry alone
-          AttnItem it{};
-          it.kind = 0;
-          it.cand = b;
-          it.n_cands = 1;
-          it.page_off = static_cast<int32_t>(w.pages.size());
-          it.n_pages = 0;
-          it.last_valid = 16;
-          it.slot = 0;
-          w.items.push_back(it);
+  }
+  for (int b = 0; b < n; ++b) {
+    Run r;
+    r.kind = 0;
+    r.cand = b;
+    r.n_cands = 1;
+    r.page_off = static_cast<int>(w.pages.size());
+    r.last_valid = 16;
+    for (int j = 0; j < np[b]; ++j)
+      if (!is_shared[static_cast<size_t>(b) * max_blocks + j]) {
+        w.pages.push_back(bt[static_cast<int64_t>(b) * max_blocks + j]);
+        if (j == np[b] - 1) r.last_valid = sl[b] - 16 * (np[b] - 1);
+      }
+    r.n_pages = static_cast<int>(w.pages.size()) - r.page_off;
+    if (r.n_pages == 0) continue;   // an empty cache, or every page shared
+    r.cost = kPrivateCost;
+    runs.push_back(r);
+  }
+  // ---- 2. cut the cost axis into C equal ranges (at least a stage of work each)
+  int64_t total = 0;
+  for (const Run& r : runs) total += static_cast<int64_t>(r.n_pages) * r.cost * n_kv;
+  if (total == 0) {   // no cached token anywhere: only the combine runs
+    w.cta_seg.push_back(0);
+    return true;
+  }
+  const int C = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(n_ctas, total / (kPagesPerStage * kPrivateCost))));
+  std::vector<int> seg_cta;
+  int64_t pos = 0;   // cost position of the current pair's first unit
+  for (const Run& r : runs) {
+    for (int g = 0; g < n_kv; ++g) {
+      const int units = r.n_pages;
+      const int64_t c = r.cost;
+      int i = 0;
+      while (i < units) {
+        // CTA of unit i: floor((2 pos + (2 i + 1) c) C / (2 total))
+        const int k = static_cast<int>(((2 * pos + (2 * static_cast<int64_t>(i) + 1) * c) * C) / (2 * total));
+        // first unit of a later CTA: the smallest e with (2 pos + (2 e + 1) c) C >= 2 total (k + 1)
+        const int64_t num = 2 * total * (k + 1) - (2 * pos + c) * C;
+        int64_t e = num <= 0 ? 0 : (num + 2 * c * C - 1) / (2 * c * C);
+        e = std::min<int64_t>(std::max<int64_t>(e, i + 1), units);
+        AttnSeg s;
+        s.kind = r.kind;
+        s.g = g;
+        s.cand = r.cand;
+        s.n_cands = r.n_cands;
+        s.page_off = r.page_off + i;
+        s.n_pages = static_cast<int>(e - i);
+        s.last_valid = e == units ? r.last_valid : 16;
+        if (r.kind == 0) {   // one slot (the merger's), or one per warp that gets a page when G > 8
+          int32_t& ns = w.nslots[static_cast<size_t>(r.cand) * n_kv + g];
+          s.slot = ns;
+          ns += group > 8 ? std::min(s.n_pages, kConsumerWarps) : 1;
+        } else {
+          s.slot = static_cast<int>(w.slots.size());
+          for (int k2 = 0; k2 < r.n_cands; ++k2)
+            w.slots.push_back(w.nslots[static_cast<size_t>(w.cands[r.cand + k2]) * n_kv + g]++);
         }
-        continue;
+        w.segs.push_back(s);
+        seg_cta.push_back(k);
+        i = static_cast<int>(e);
       }
-      for (size_t p0 = 0; p0 < priv.size(); p0 += static_cast<size_t>(priv_split)) {
-        const int npg = static_cast<int>(std::min<size_t>(static_cast<size_t>(priv_split), priv.size() - p0));
-        const bool ends = p0 + npg == priv.size();
-        AttnItem it{};
-        it.kind = 0;
-        it.cand = b;
-        it.n_cands = 1;
-        it.page_off = static_cast<int32_t>(w.pages.size());
-        it.n_pages = npg;
-        it.last_valid = (ends && last_private) ? last_valid_b : 16;
-        it.slot = w.nslots[b]++;
-        if (w.nslots[b] > slot_cap) ok = false;
-        w.pages.insert(w.pages.end(), priv.begin() + p0, priv.begin() + p0 + npg);
-        w.items.push_back(it);
-      }
-    }
-    if (ok) {
-      w.max_item_pages = 0;
-      for (const auto& it : w.items) w.max_item_pages = std::max(w.max_item_pages, it.n_pages);
-      return true;
+      pos += static_cast<int64_t>(units) * c;
     }
   }
-  return false;
+  // ---- 3. slot numbering
+  size_t next = 0;
+  for (size_t cg = 0; cg < w.nslots.size(); ++cg) {
+    w.slot_base[cg] = static_cast<int32_t>(next);
+    next += static_cast<size_t>(w.nslots[cg]);
+  }
+  if (next > slot_limit) {
+    if (share) return build_attn_work(bt, sl, n, max_blocks, n_kv, group, n_ctas, slot_limit, false, w);
+    return false;
+  }
+  w.n_slots = static_cast<int>(next);
+  for (AttnSeg& s : w.segs) {
+    if (s.kind == 0)
+      s.slot += w.slot_base[static_cast<size_t>(s.cand) * n_kv + s.g];
+    else
+      for (int k2 = 0; k2 < s.n_cands; ++k2)
+        w.slots[s.slot + k2] += w.slot_base[static_cast<size_t>(w.cands[s.cand + k2]) * n_kv + s.g];
+  }
+  w.n_ctas = C;
+  w.cta_seg.assign(C + 1, 0);
+  for (int k : seg_cta) w.cta_seg[k + 1]++;
+  for (int k = 0; k < C; ++k) w.cta_seg[k + 1] += w.cta_seg[k];
+  return true;
 }
 
 cudaError_t attention_configure() {
   cudaError_t e;
-  if ((e = set_smem(attn_kernel<64, false>)) != cudaSuccess) return e;
-  if ((e = set_smem(attn_kernel<64, true>)) != cudaSuccess) return e;
-  if ((e = set_smem(attn_kernel<128, false>)) != cudaSuccess) return e;
-  return set_smem(attn_kernel<128, true>);
+  if ((e = set_smem(attn_combine_kernel<64, 8>, CombineShape<64, 8>::kBytes)) != cudaSuccess) return e;
+  if ((e = set_smem(attn_combine_kernel<64, 16>, CombineShape<64, 16>::kBytes)) != cudaSuccess) return e;
+  if ((e = set_smem(attn_combine_kernel<128, 8>, CombineShape<128, 8>::kBytes)) != cudaSuccess) return e;
+  if ((e = set_smem(attn_combine_kernel<128, 16>, CombineShape<128, 16>::kBytes)) != cudaSuccess) return e;
+  if ((e = set_smem(attn_kernel<64, false>, AttnSmem<64>::kDynamic)) != cudaSuccess) return e;
+  if ((e = set_smem(attn_kernel<64, true>, AttnSmem<64>::kDynamic)) != cudaSuccess) return e;
+  if ((e = set_smem(attn_kernel<128, false>, AttnSmem<128>::kDynamic)) != cudaSuccess) return e;
+  return set_smem(attn_kernel<128, true>, AttnSmem<128>::kDynamic);
 }
 
-cudaError_t launch_attention(const AttnShape& s, const AttnWork& wk, int max_item_pages, const CUtensorMap* tm_pool,
-                             int layer, const __nv_bfloat16* q_hi, const __nv_bfloat16* q_lo, int stride,
-                             float* part_o, float* part_ml, const AttnMerge& mg, int* err, cudaStream_t stream,
-                             bool pdl, unsigned long long* ts) {
-  if (wk.n_items == 0) return cudaSuccess;
+cudaError_t launch_attention(const AttnShape& s, const AttnWork& wk, const CUtensorMap* tm_pool, int layer,
+                             const __nv_bfloat16* q_hi, const __nv_bfloat16* q_lo, float* part_o, float* part_ml,
+                             int* err, cudaStream_t stream, bool pdl, unsigned long long* ts) {
+  if (wk.n_ctas == 0) return cudaSuccess;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(wk.n_items, s.n_kv, 1);
+  cfg.gridDim = dim3(wk.n_ctas, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
-  cfg.dynamicSmemBytes = attention_smem_bytes(s.hd, max_item_pages);
+  cfg.dynamicSmemBytes = attention_smem_bytes(s.hd);
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
-  const int64_t row0 = static_cast<int64_t>(layer) * s.layer_rows;
+  const int64_t page0 = static_cast<int64_t>(layer) * s.layer_pages;
   const bool two = s.group > 8;
   if (s.hd == 128) {
     if (two)
-      return cudaLaunchKernelEx(&cfg, attn_kernel<128, true>, *tm_pool, row0, wk, q_hi, q_lo, s.n_q, s.n_kv, s.group,
-                                stride, part_o, part_ml, mg, err, ts);
-    return cudaLaunchKernelEx(&cfg, attn_kernel<128, false>, *tm_pool, row0, wk, q_hi, q_lo, s.n_q, s.n_kv, s.group,
-                              stride, part_o, part_ml, mg, err, ts);
+      return cudaLaunchKernelEx(&cfg, attn_kernel<128, true>, *tm_pool, page0, wk, q_hi, q_lo, s.n_q, s.n_kv, s.group,
+                                part_o, part_ml, err, ts);
+    return cudaLaunchKernelEx(&cfg, attn_kernel<128, false>, *tm_pool, page0, wk, q_hi, q_lo, s.n_q, s.n_kv, s.group,
+                              part_o, part_ml, err, ts);
   }
   if (two)
-    return cudaLaunchKernelEx(&cfg, attn_kernel<64, true>, *tm_pool, row0, wk, q_hi, q_lo, s.n_q, s.n_kv, s.group,
-                              stride, part_o, part_ml, mg, err, ts);
-  return cudaLaunchKernelEx(&cfg, attn_kernel<64, false>, *tm_pool, row0, wk, q_hi, q_lo, s.n_q, s.n_kv, s.group,
-                            stride, part_o, part_ml, mg, err, ts);
+    return cudaLaunchKernelEx(&cfg, attn_kernel<64, true>, *tm_pool, page0, wk, q_hi, q_lo, s.n_q, s.n_kv, s.group,
+                              part_o, part_ml, err, ts);
+  return cudaLaunchKernelEx(&cfg, attn_kernel<64, false>, *tm_pool, page0, wk, q_hi, q_lo, s.n_q, s.n_kv, s.group,
+                            part_o, part_ml, err, ts);
+}
+
+cudaError_t launch_attn_combine(const AttnShape& s, const AttnWork& wk, int n, const float* part_o,
+                                const float* part_ml, const AttnMerge& mg, cudaStream_t stream, bool pdl,
+                                unsigned long long* ts) {
+  if (n == 0) return cudaSuccess;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(n) * s.n_kv, 1, 1);
+
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  const bool two = s.group > 8;
+#define KVPRM_COMBINE(HD_, R_)                                                                                     \
+  do {                                                                                                           \
+    cfg.dynamicSmemBytes = CombineShape<HD_, R_>::kBytes;                                                        \
+    cfg.blockDim = dim3(32 * CombineShape<HD_, R_>::W, 1, 1);                                                    \
+    return cudaLaunchKernelEx(&cfg, attn_combine_kernel<HD_, R_>, wk.slot_base, wk.nslots, s.n_q, s.n_kv, s.group, \
+                              part_o, part_ml, mg, ts);                                                          \
+  } while (0)
+  if (s.hd == 128) {
+    if (two) KVPRM_COMBINE(128, 16);
+    KVPRM_COMBINE(128, 8);
+  }
+  if (two) KVPRM_COMBINE(64, 16);
+  KVPRM_COMBINE(64, 8);
+#undef KVPRM_COMBINE
 }
 
 cudaError_t launch_resolve(const int32_t* bt, const int32_t* seq_lens, int max_blocks, int b, int64_t* out,

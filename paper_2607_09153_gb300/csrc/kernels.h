@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -48,54 +49,72 @@ cudaError_t launch_gemm(const GemmPlan& p, const CUtensorMap* tmW, const CUtenso
 struct AttnShape {
   int n_q, n_kv, hd, group;     // group = n_q / n_kv
   int max_blocks;               // block-table row length
-  int64_t layer_rows;           // rows (of hd elements) per layer in the pool map: n_pages * 2 * n_kv * 16
+  int64_t layer_pages;          // pages per layer of the pool (n_pages)
 };
-// One unit of attention work (see attention.cu): a run of physical pages of one
-// candidate (kind 0) or pages shared by up to 8 candidates (kind 1).
-struct AttnItem {
+// Tensor map of a paged KV pool [layers][n_pages][2][n_kv][16][hd] (bf16) whose
+// box is one page of one kv head, K and V together: 5-D (column within a
+// 64-column sub-tile, token, sub-tile, kv head, 2 * (layer * n_pages + page) +
+// {0: K, 1: V}) with the 128-byte swizzle, landing in shared memory as
+// [K, V][sub-tile][token][64 columns].  page_units = layers * n_pages.
+CUresult encode_pool_map(PFN_cuTensorMapEncodeTiled_v12000 encode, CUtensorMap* map, const void* pool,
+                         int64_t page_units, int n_kv, int hd);
+// One segment of attention work (see attention.cu): a run of physical pages of
+// one kv head, scored for one candidate (kind 0) or for up to 8 candidates that
+// all reference those pages (kind 1).
+struct AttnSeg {
   int32_t kind;
+  int32_t g;           // kv head
   int32_t cand;        // kind 0: the candidate; kind 1: offset into AttnWork::cands
   int32_t n_cands;     // kind 1: candidates (<= 8)
   int32_t page_off;    // offset into AttnWork::pages
   int32_t n_pages;     // 0: an empty cache (self entry only)
-  int32_t last_valid;  // valid tokens in the item's last page (1..16)
-  int32_t slot;        // kind 0: the candidate's partial slot; kind 1: offset into AttnWork::slots
-  int32_t pad;
+  int32_t last_valid;  // valid tokens in the segment's last page (1..16)
+  int32_t slot;        // kind 0: the partial slot; kind 1: offset into AttnWork::slots
 };
-struct AttnWork {            // device arrays
-  const AttnItem* items;
-  const int32_t* pages;      // physical page ids
-  const int32_t* cands;      // candidates of shared items
-  const int32_t* slots;      // their partial slots
-  const int32_t* nslots;     // [B] partial slots of each candidate
-  int n_items;
+struct AttnWork {             // device arrays
+  const AttnSeg* segs;
+  const int32_t* cta_seg;     // [n_ctas + 1] first segment of each CTA
+  const int32_t* pages;       // physical page ids
+  const int32_t* cands;       // candidates of shared segments
+  const int32_t* slots;       // their partial slots
+  const int32_t* slot_base;   // [B][n_kv] first partial slot of each (candidate, kv head)
+  const int32_t* nslots;      // [B][n_kv] number of partial slots
+  int n_ctas;
 };
 struct AttnWorkHost {
-  std::vector<AttnItem> items;
-  std::vector<int32_t> pages, cands, slots, nslots;
-  int max_item_pages = 0;
+  std::vector<AttnSeg> segs;
+  std::vector<int32_t> cta_seg, pages, cands, slots, slot_base, nslots;
+  int n_slots = 0, n_ctas = 0;
 };
-bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks, int n_kv, int hd, int num_sms,
-                     int slot_cap, bool share, AttnWorkHost& w);
-size_t attention_smem_bytes(int hd, int max_item_pages);
+bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks, int n_kv, int group, int n_ctas,
+                     size_t slot_limit, bool share, AttnWorkHost& w);
+// partial slots a context sized for max_candidates provides (the planner falls
+// back to private runs, which always fit, when sharing needs more)
+size_t attn_slot_capacity(int max_candidates, int n_kv, int num_sms);
+size_t attention_smem_bytes(int hd);
 cudaError_t attention_configure();
-// Inputs and outputs of the split merge done by the last CTA of each (candidate, kv head).
+// Inputs and outputs of the combine (attn_combine_kernel).
 struct AttnMerge {
   const float* q;       // [B][n_q][hd] rotated query (fp32)
   const float* kself;   // [B][n_kv][hd]
   const float* vself;   // [B][n_kv][hd]
-  int* counter;         // [B][n_kv] arrival counters, zero between calls
   __nv_bfloat16* o_hi;  // [B][n_q][hd] attention output as a bf16 pair
   __nv_bfloat16* o_lo;
   float* out_f32;       // optional fp32 copy
   float* dbg;           // optional fp32 copy
 };
-// q_hi / q_lo: bf16 pair of the rotated query [B][n_q][hd]; partial slots
-// [B][n_q][stride][hd] (values) and [B][n_q][stride][2] (max in log2 units, sum)
-cudaError_t launch_attention(const AttnShape& s, const AttnWork& wk, int max_item_pages, const CUtensorMap* tm_pool,
-                             int layer, const __nv_bfloat16* q_hi, const __nv_bfloat16* q_lo, int stride,
-                             float* part_o, float* part_ml, const AttnMerge& mg, int* err, cudaStream_t stream,
-                             bool pdl, unsigned long long* ts = nullptr);
+// q_hi / q_lo: bf16 pair of the rotated query [B][n_q][hd]; partial slot s of
+// query row r of its group at part_o[(s * group + r) * hd] (values) and
+// part_ml[(s * group + r) * 2] (max in log2 units, sum).  One CTA per entry of
+// wk.cta_seg.
+cudaError_t launch_attention(const AttnShape& s, const AttnWork& wk, const CUtensorMap* tm_pool, int layer,
+                             const __nv_bfloat16* q_hi, const __nv_bfloat16* q_lo, float* part_o, float* part_ml,
+                             int* err, cudaStream_t stream, bool pdl, unsigned long long* ts = nullptr);
+// Merge every (candidate, kv head)'s slots (wk.slot_base / wk.nslots) of the
+// n candidates with the self entry into the attention output.
+cudaError_t launch_attn_combine(const AttnShape& s, const AttnWork& wk, int n, const float* part_o,
+                                const float* part_ml, const AttnMerge& mg, cudaStream_t stream, bool pdl,
+                                unsigned long long* ts = nullptr);
 cudaError_t launch_resolve(const int32_t* bt, const int32_t* seq_lens, int max_blocks, int b, int64_t* out,
                            cudaStream_t stream);
 

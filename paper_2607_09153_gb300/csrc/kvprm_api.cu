@@ -24,22 +24,18 @@ typedef __nv_bfloat16 bf16;
 
 namespace {
 
-constexpr int kSplitCap = 32;   // max split-K partials of the attention per (candidate, head)
-
 struct CallPlan {
   int n = 0, n_pad = 0, max_pages = 0;
   GemmPlan g_qkv, g_o, g_gu, g_down;
-  int n_items = 0, max_item_pages = 0;   // attention work list (see build_attn_work)
+  int attn_ctas = 0;   // grid of the attention (see build_attn_work)
 };
 
 struct GraphKey {
-  int n = -1, n_pad = -1, n_items = -1, max_item_pages = -1, debug = -1, profile = -1, pdl = -1, trace = -1;
+  int n = -1, n_pad = -1, attn_ctas = -1, debug = -1, profile = -1, pdl = -1, trace = -1;
   const void* pool = nullptr;
   int64_t n_pages = -1;
   bool operator==(const GraphKey& o) const {
-    return n == o.n && n_pad == o.n_pad && n_items == o.n_items && max_item_pages == o.max_item_pages &&
-           debug == o.debug &&
-           profile == o.profile && pdl == o.pdl && trace == o.trace && pool == o.pool && n_pages == o.n_pages;
+    return n == o.n && n_pad == o.n_pad && attn_ctas == o.attn_ctas && debug == o.debug && profile == o.profile && pdl == o.pdl && trace == o.trace && pool == o.pool && n_pages == o.n_pages;
   }
 };
 
@@ -68,14 +64,15 @@ struct kvprm_ctx {
   int d_tiles = 0;
   float *q = nullptr, *kself = nullptr, *vself = nullptr;
   bf16 *qhi = nullptr, *qlo = nullptr;
-  float *apart_o = nullptr, *apart_ml = nullptr;
-  int* attn_counter = nullptr;   // [Bmax][n_kv] split-arrival counters
+  float *apart_o = nullptr, *apart_ml = nullptr;   // [slot_cap][group][hd], [slot_cap][group][2]
+  size_t slot_cap = 0;
   float2* rope = nullptr;
   int32_t* tables_d = nullptr;   // [Bmax] seq_lens, [Bmax][max_blocks] block table, then the attention work
   // attention work list: host plan of the current call and fixed offsets (ints) in tables_d / staging
   kvprm::AttnWorkHost work_host;
-  size_t off_items = 0, off_pages = 0, off_cands = 0, off_slots = 0, off_nslots = 0, tables_ints = 0;
-  size_t cap_items = 0, cap_pages = 0, cap_cands = 0;
+  size_t off_segs = 0, off_cta = 0, off_pages = 0, off_cands = 0, off_slots = 0, off_base = 0, off_nslots = 0;
+  size_t tables_ints = 0;
+  size_t cap_segs = 0, cap_pages = 0, cap_cands = 0;
   bool share_pages = true;
   float* rewards_d = nullptr;
   int* err_d = nullptr;
@@ -97,7 +94,7 @@ struct kvprm_ctx {
   // pool tensor map (depends on the caller's pool)
   const void* pool_ptr = nullptr;
   int64_t pool_pages = -1;
-  int64_t pool_rows = -1;
+  int64_t pool_units = -1;
   CUtensorMap tm_pool{};
   // library-owned device pool for kvprm_score_host
   void* dev_pool = nullptr;
@@ -194,7 +191,6 @@ void free_ctx(kvprm_ctx* c) {
   cudaFree(c->vself);
   cudaFree(c->apart_o);
   cudaFree(c->apart_ml);
-  cudaFree(c->attn_counter);
   cudaFree(c->rope);
   cudaFree(c->tables_d);
   cudaFree(c->rewards_d);
@@ -251,13 +247,20 @@ int validate_tables(kvprm_ctx* ctx, int64_t n_pages, const int32_t* bt, const in
   return KVPRM_OK;
 }
 
-// Plan the attention work of this call on the host (build_attn_work).
+// Plan the attention work of this call on the host (build_attn_work); a
+// sharing plan that does not fit the context's work arrays falls back to
+// private runs, which always fit.
 int plan_work(kvprm_ctx* ctx, const int32_t* bt, const int32_t* sl, int32_t n) {
   kvprm::AttnWorkHost& w = ctx->work_host;
-  if (!kvprm::build_attn_work(bt, sl, n, ctx->cfg.max_blocks_per_seq, ctx->cfg.n_kv_heads, ctx->cfg.head_dim,
-                              ctx->num_sms, kSplitCap, ctx->share_pages, w))
-    return fail(ctx, KVPRM_EUNSUPPORTED, "attention work does not fit %d partial slots per candidate", kSplitCap);
-  if (w.items.size() > ctx->cap_items || w.pages.size() > ctx->cap_pages || w.cands.size() > ctx->cap_cands)
+  const int mb = ctx->cfg.max_blocks_per_seq, nkv = ctx->cfg.n_kv_heads;
+  auto fits = [&]() {
+    return w.segs.size() <= ctx->cap_segs && w.pages.size() <= ctx->cap_pages && w.cands.size() <= ctx->cap_cands &&
+           w.slots.size() <= ctx->slot_cap && static_cast<size_t>(w.n_ctas) <= static_cast<size_t>(ctx->num_sms);
+  };
+  bool ok = kvprm::build_attn_work(bt, sl, n, mb, nkv, ctx->md.n_q / nkv, ctx->num_sms, ctx->slot_cap, ctx->share_pages, w);
+  if (ok && !fits() && ctx->share_pages)
+    ok = kvprm::build_attn_work(bt, sl, n, mb, nkv, ctx->md.n_q / nkv, ctx->num_sms, ctx->slot_cap, false, w);
+  if (!ok || !fits())
     return fail(ctx, KVPRM_ECAPACITY, "attention work list exceeds the context's capacity");
   return KVPRM_OK;
 }
@@ -271,23 +274,30 @@ int upload_tables(kvprm_ctx* ctx, const int32_t* bt, const int32_t* sl, int32_t 
   }
   const kvprm::AttnWorkHost& w = ctx->work_host;
   int32_t* S = ctx->staging;
+  constexpr size_t kSegInts = sizeof(kvprm::AttnSeg) / sizeof(int32_t);
   std::memcpy(S, sl, sizeof(int32_t) * n);
   std::memcpy(S + Bmax, bt, sizeof(int32_t) * static_cast<size_t>(n) * mb);
-  std::memcpy(S + ctx->off_items, w.items.data(), sizeof(kvprm::AttnItem) * w.items.size());
-  std::memcpy(S + ctx->off_pages, w.pages.data(), sizeof(int32_t) * w.pages.size());
-  std::memcpy(S + ctx->off_cands, w.cands.data(), sizeof(int32_t) * w.cands.size());
-  std::memcpy(S + ctx->off_slots, w.slots.data(), sizeof(int32_t) * w.slots.size());
-  std::memcpy(S + ctx->off_nslots, w.nslots.data(), sizeof(int32_t) * w.nslots.size());
+  struct Part {
+    size_t off;
+    const void* src;
+    size_t ints;
+  } parts[] = {
+      {ctx->off_segs, w.segs.data(), w.segs.size() * kSegInts},
+      {ctx->off_cta, w.cta_seg.data(), w.cta_seg.size()},
+      {ctx->off_pages, w.pages.data(), w.pages.size()},
+      {ctx->off_cands, w.cands.data(), w.cands.size()},
+      {ctx->off_slots, w.slots.data(), w.slots.size()},
+      {ctx->off_base, w.slot_base.data(), w.slot_base.size()},
+      {ctx->off_nslots, w.nslots.data(), w.nslots.size()},
+  };
+  for (const Part& p : parts)
+    if (p.ints) std::memcpy(S + p.off, p.src, sizeof(int32_t) * p.ints);
   auto up = [&](size_t off, size_t ints) -> cudaError_t {
     if (ints == 0) return cudaSuccess;
     return cudaMemcpyAsync(ctx->tables_d + off, S + off, ints * sizeof(int32_t), cudaMemcpyHostToDevice, st);
   };
   CK(up(0, static_cast<size_t>(Bmax) + static_cast<size_t>(n) * mb), "cudaMemcpyAsync(tables)");
-  CK(up(ctx->off_items, w.items.size() * (sizeof(kvprm::AttnItem) / sizeof(int32_t))), "cudaMemcpyAsync(items)");
-  CK(up(ctx->off_pages, w.pages.size()), "cudaMemcpyAsync(pages)");
-  CK(up(ctx->off_cands, w.cands.size()), "cudaMemcpyAsync(cands)");
-  CK(up(ctx->off_slots, w.slots.size()), "cudaMemcpyAsync(slots)");
-  CK(up(ctx->off_nslots, w.nslots.size()), "cudaMemcpyAsync(nslots)");
+  for (const Part& p : parts) CK(up(p.off, p.ints), "cudaMemcpyAsync(attention work)");
   CK(cudaEventRecord(ctx->staging_ev, st), "cudaEventRecord(staging)");
   ctx->staging_pending = true;
   return KVPRM_OK;
@@ -295,28 +305,29 @@ int upload_tables(kvprm_ctx* ctx, const int32_t* bt, const int32_t* sl, int32_t 
 
 kvprm::AttnWork device_work(kvprm_ctx* ctx) {
   kvprm::AttnWork wk;
-  wk.items = reinterpret_cast<const kvprm::AttnItem*>(ctx->tables_d + ctx->off_items);
+  wk.segs = reinterpret_cast<const kvprm::AttnSeg*>(ctx->tables_d + ctx->off_segs);
+  wk.cta_seg = ctx->tables_d + ctx->off_cta;
   wk.pages = ctx->tables_d + ctx->off_pages;
   wk.cands = ctx->tables_d + ctx->off_cands;
   wk.slots = ctx->tables_d + ctx->off_slots;
+  wk.slot_base = ctx->tables_d + ctx->off_base;
   wk.nslots = ctx->tables_d + ctx->off_nslots;
-  wk.n_items = static_cast<int>(ctx->work_host.items.size());
+  wk.n_ctas = ctx->work_host.n_ctas;
   return wk;
 }
 
 int ensure_pool_map(kvprm_ctx* ctx, const void* pool, int64_t n_pages, int layers) {
-  if (ctx->pool_ptr == pool && ctx->pool_pages == n_pages && ctx->pool_rows >= 0 &&
-      ctx->pool_rows == static_cast<int64_t>(layers) * n_pages * 2 * ctx->cfg.n_kv_heads * 16)
-    return KVPRM_OK;
-  const int64_t rows = static_cast<int64_t>(layers) * n_pages * 2 * ctx->cfg.n_kv_heads * 16;
-  if (rows >= (static_cast<int64_t>(1) << 31))
-    return fail(ctx, KVPRM_EUNSUPPORTED, "pool of %lld rows exceeds the 2^31-row tensor-map limit",
-                static_cast<long long>(rows));
-  int rc = make_map(ctx, &ctx->tm_pool, pool, ctx->cfg.head_dim, rows, 64, 16, "kv pool");
-  if (rc) return rc;
+  const int64_t units = static_cast<int64_t>(layers) * n_pages;   // (layer, page) pairs
+  if (ctx->pool_ptr == pool && ctx->pool_pages == n_pages && ctx->pool_units == units) return KVPRM_OK;
+  if (2 * units >= (static_cast<int64_t>(1) << 31))
+    return fail(ctx, KVPRM_EUNSUPPORTED, "pool of %lld layer pages exceeds the 2^30 tensor-map coordinate limit",
+                static_cast<long long>(units));
+  const CUresult r = kvprm::encode_pool_map(ctx->encode, &ctx->tm_pool, pool, units, ctx->cfg.n_kv_heads,
+                                            ctx->cfg.head_dim);
+  if (r != CUDA_SUCCESS) return fail(ctx, KVPRM_ECUDA, "cuTensorMapEncodeTiled(kv pool) failed with %d", (int)r);
   ctx->pool_ptr = pool;
   ctx->pool_pages = n_pages;
-  ctx->pool_rows = rows;
+  ctx->pool_units = units;
   return KVPRM_OK;
 }
 
@@ -344,8 +355,7 @@ CallPlan make_plan(kvprm_ctx* ctx, int n, int max_pages) {
   p.g_o = kvprm::plan_gemm(m.d, m.n_q * m.hd, p.n_pad, ctx->num_sms, true, false);
   p.g_gu = kvprm::plan_gemm(m.ff, m.d, p.n_pad, ctx->num_sms, true, true);
   p.g_down = kvprm::plan_gemm(m.d, m.ff, p.n_pad, ctx->num_sms, true, false);
-  p.n_items = static_cast<int>(ctx->work_host.items.size());
-  p.max_item_pages = ctx->work_host.max_item_pages;
+  p.attn_ctas = ctx->work_host.n_ctas;
   return p;
 }
 
@@ -433,7 +443,6 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
   ctx->trace_cls.clear();
   if (ctx->trace)
     CK(cudaMemsetAsync(ctx->trace_d, 0xFF, sizeof(unsigned long long) * 2 * ctx->trace_cap, st), "trace reset");
-  CK(cudaMemsetAsync(ctx->attn_counter, 0, sizeof(int) * static_cast<size_t>(n) * m.n_kv, st), "counter reset");
   LAUNCH(KVPRM_PROF_FUSED, kvprm::launch_rope_table(sl, n, m.hd, ctx->cfg.rope_base, ctx->rope, st, false, TS), "rope");
   LAUNCH(KVPRM_PROF_FUSED,
          kvprm::launch_embed_norm(m, ctx->embed, ctx->attn_norm[0], n, ctx->h, ctx->sumsq, X, st, pdl, TS),
@@ -449,11 +458,14 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
       CK(cudaMemcpyAsync(ctx->dbg_v + l * nk, ctx->vself, nk * 4, cudaMemcpyDeviceToDevice, st), "debug v");
     }
     float* dbg = (ctx->debug_flags & 1) ? ctx->dbg + static_cast<size_t>(l) * n * m.n_q * m.hd : nullptr;
-    const kvprm::AttnMerge mg{ctx->q, ctx->kself, ctx->vself, ctx->attn_counter, O.hi, O.lo, nullptr, dbg};
+    const kvprm::AttnMerge mg{ctx->q, ctx->kself, ctx->vself, O.hi, O.lo, nullptr, dbg};
+    const kvprm::AttnWork wk = device_work(ctx);
     LAUNCH(KVPRM_PROF_ATTN,
-           kvprm::launch_attention(ctx->as, device_work(ctx), P.max_item_pages, &ctx->tm_pool, l, ctx->qhi, ctx->qlo,
-                                   kSplitCap, ctx->apart_o, ctx->apart_ml, mg, ctx->err_d, st, pdl, TS),
+           kvprm::launch_attention(ctx->as, wk, &ctx->tm_pool, l, ctx->qhi, ctx->qlo, ctx->apart_o, ctx->apart_ml,
+                                   ctx->err_d, st, pdl, TS),
            "attention");
+    LAUNCH(KVPRM_PROF_COMBINE,
+           kvprm::launch_attn_combine(ctx->as, wk, n, ctx->apart_o, ctx->apart_ml, mg, st, pdl, TS), "attn_combine");
     LAUNCH(KVPRM_PROF_GEMM_O,
            kvprm::launch_gemm(P.g_o, &ctx->tm_o[l], &ctx->tm_ohi, &ctx->tm_olo, er, np, ctx->err_d, st, pdl, TS),
            "gemm_o");
@@ -527,7 +539,7 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
     if (!aligned16(kv_pages)) return fail(ctx, KVPRM_EINVAL, "kv_pages is not 16-byte aligned");
   }
   if ((rc = ensure_pool_map(ctx, pool, pages, ctx->cfg.n_layers))) return rc;
-  ctx->as.layer_rows = pages * 2 * ctx->cfg.n_kv_heads * 16;
+  ctx->as.layer_pages = pages;
   if ((rc = plan_work(ctx, bt, sl, n))) return rc;
   const CallPlan P = make_plan(ctx, n, max_pages);
   if ((rc = ensure_x_maps(ctx, P.n_pad))) return rc;
@@ -547,8 +559,7 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   GraphKey key;
   key.n = n;
   key.n_pad = P.n_pad;
-  key.n_items = P.n_items;
-  key.max_item_pages = P.max_item_pages;
+  key.attn_ctas = P.attn_ctas;
   key.debug = ctx->debug_flags;
   key.profile = ctx->profile ? 1 : 0;
   key.pdl = ctx->use_pdl ? 1 : 0;
@@ -674,7 +685,7 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   as.hd = m.hd;
   as.group = m.n_q / m.n_kv;
   as.max_blocks = c.max_blocks_per_seq;
-  as.layer_rows = 0;   // set per call from the pool
+  as.layer_pages = 0;   // set per call from the pool
 
   ctx->embed = static_cast<const bf16*>(w->embed_verify);
   ctx->final_norm = static_cast<const bf16*>(w->final_norm);
@@ -714,22 +725,28 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   CREATE_CK(dalloc(ctx, &ctx->qlo, static_cast<size_t>(Bmax) * m.n_q * m.hd, "q_lo"));
   CREATE_CK(dalloc(ctx, &ctx->kself, static_cast<size_t>(Bmax) * m.n_kv * m.hd, "k_self"));
   CREATE_CK(dalloc(ctx, &ctx->vself, static_cast<size_t>(Bmax) * m.n_kv * m.hd, "v_self"));
-  CREATE_CK(dalloc(ctx, &ctx->apart_o, static_cast<size_t>(Bmax) * m.n_q * kSplitCap * m.hd, "attn partials"));
-  CREATE_CK(dalloc(ctx, &ctx->apart_ml, static_cast<size_t>(Bmax) * m.n_q * kSplitCap * 2, "attn stats"));
-  CREATE_CK(dalloc(ctx, &ctx->attn_counter, static_cast<size_t>(Bmax) * m.n_kv, "attn counters"));
+  ctx->slot_cap = kvprm::attn_slot_capacity(Bmax, m.n_kv, ctx->num_sms);
+  const size_t group = static_cast<size_t>(m.n_q / m.n_kv);
+  CREATE_CK(dalloc(ctx, &ctx->apart_o, ctx->slot_cap * group * m.hd, "attn partials"));
+  CREATE_CK(dalloc(ctx, &ctx->apart_ml, ctx->slot_cap * group * 2, "attn stats"));
   CREATE_CK(dalloc(ctx, &ctx->rope, static_cast<size_t>(Bmax) * (m.hd / 2), "rope table"));
   {
     const size_t tbl = static_cast<size_t>(Bmax) * (1 + c.max_blocks_per_seq);
     auto al8 = [](size_t x) { return (x + 7) & ~static_cast<size_t>(7); };
-    ctx->cap_items = static_cast<size_t>(Bmax) * (kSplitCap + 1);
-    ctx->cap_pages = static_cast<size_t>(2) * Bmax * c.max_blocks_per_seq;
-    ctx->cap_cands = static_cast<size_t>(Bmax) * kSplitCap;
-    ctx->off_items = al8(tbl);
-    ctx->off_pages = al8(ctx->off_items + ctx->cap_items * (sizeof(kvprm::AttnItem) / sizeof(int32_t)));
+    // private runs need at most Bmax * n_kv + n_ctas segments, Bmax * max_blocks
+    // pages and no candidate lists; sharing plans beyond these fall back to them
+    const size_t bkv = static_cast<size_t>(Bmax) * m.n_kv;
+    ctx->cap_segs = 4 * bkv + 2 * static_cast<size_t>(ctx->num_sms);
+    ctx->cap_pages = static_cast<size_t>(Bmax) * c.max_blocks_per_seq;
+    ctx->cap_cands = static_cast<size_t>(Bmax) * c.max_blocks_per_seq;
+    ctx->off_segs = al8(tbl);
+    ctx->off_cta = al8(ctx->off_segs + ctx->cap_segs * (sizeof(kvprm::AttnSeg) / sizeof(int32_t)));
+    ctx->off_pages = al8(ctx->off_cta + ctx->num_sms + 1);
     ctx->off_cands = al8(ctx->off_pages + ctx->cap_pages);
     ctx->off_slots = al8(ctx->off_cands + ctx->cap_cands);
-    ctx->off_nslots = al8(ctx->off_slots + ctx->cap_cands);
-    ctx->tables_ints = al8(ctx->off_nslots + Bmax);
+    ctx->off_base = al8(ctx->off_slots + ctx->slot_cap);
+    ctx->off_nslots = al8(ctx->off_base + bkv);
+    ctx->tables_ints = al8(ctx->off_nslots + bkv);
   }
   CREATE_CK(dalloc(ctx, &ctx->tables_d, ctx->tables_ints, "tables and attention work"));
   CREATE_CK(dalloc(ctx, &ctx->rewards_d, static_cast<size_t>(Bmax), "rewards"));
@@ -846,19 +863,21 @@ int kvprm_attention(kvprm_ctx* ctx, const void* kv_layer, int64_t n_pages, const
   if ((rc = plan_work(ctx, block_table, seq_lens, n))) return rc;
   if ((rc = upload_tables(ctx, block_table, seq_lens, n, st))) return rc;
   AttnShape as = ctx->as;
-  as.layer_rows = pages * 2 * ctx->cfg.n_kv_heads * 16;
+  as.layer_pages = pages;
   Enq E{ctx, st, false, ctx->profile, &ctx->live_marks};
   LAUNCH(KVPRM_PROF_FUSED,
          kvprm::launch_split_hilo(static_cast<const float*>(q), static_cast<int64_t>(n) * ctx->md.n_q * ctx->md.hd, Q,
                                   st),
          "split_hilo");
-  CK(cudaMemsetAsync(ctx->attn_counter, 0, sizeof(int) * static_cast<size_t>(n) * ctx->md.n_kv, st), "counter reset");
   const kvprm::AttnMerge mg{static_cast<const float*>(q), static_cast<const float*>(k_self),
-                            static_cast<const float*>(v_self), ctx->attn_counter, ctx->ohi, ctx->olo, out, nullptr};
+                            static_cast<const float*>(v_self), ctx->ohi, ctx->olo, out, nullptr};
+  const kvprm::AttnWork wk = device_work(ctx);
   LAUNCH(KVPRM_PROF_ATTN,
-         kvprm::launch_attention(as, device_work(ctx), ctx->work_host.max_item_pages, &ctx->tm_pool, 0, Q.hi, Q.lo,
-                                 kSplitCap, ctx->apart_o, ctx->apart_ml, mg, ctx->err_d, st, false),
+         kvprm::launch_attention(as, wk, &ctx->tm_pool, 0, Q.hi, Q.lo, ctx->apart_o, ctx->apart_ml, ctx->err_d, st,
+                                 false),
          "attention");
+  LAUNCH(KVPRM_PROF_COMBINE, kvprm::launch_attn_combine(as, wk, n, ctx->apart_o, ctx->apart_ml, mg, st, false),
+         "attn_combine");
   ctx->last_n = n;
   ctx->last_stream = st;
   if (ctx->profile) {

@@ -19,6 +19,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <cstdint>
 #include <cstring>
 #include <mutex>
 
@@ -30,7 +31,6 @@ namespace {
 static __device__ __align__(256) unsigned char g_scratch[KVPRM_NOALLOC_SCRATCH_BYTES];
 
 constexpr int kMaxDevices = 64;
-constexpr int kSplitCapMax = 32;
 
 struct DeviceState {
   bool ready = false;
@@ -70,14 +70,13 @@ int setup_current_device(unsigned char** scratch) {
 size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
 
 struct Carve {
-  size_t err, cnt, items, pages, cands, slots, nslots, qhi, qlo, ohi, olo, pml, po, total;
+  size_t err, segs, cta, pages, cands, slots, base, nslots, qhi, qlo, ohi, olo, pml, po, total;
 };
 
-// Layout of the scratch array for one call: the error word, the split-arrival
-// counters, the attention work list, the query's bf16 hi/lo parts, the
-// output's hi/lo parts (the kernel always writes them) and `stride` partial
-// slots per (candidate, query head).
-Carve carve(int n, int n_q, int n_kv, int hd, int stride, const kvprm::AttnWorkHost& w) {
+// Layout of the scratch array for one call: the error word, the attention
+// schedule, the query's bf16 hi/lo parts, the
+// output's hi/lo parts (the kernel always writes them) and the partial slots.
+Carve carve(int n, int n_q, int n_kv, int hd, const kvprm::AttnWorkHost& w) {
   Carve c;
   size_t off = 0;
   auto take = [&](size_t bytes) {
@@ -86,19 +85,21 @@ Carve carve(int n, int n_q, int n_kv, int hd, int stride, const kvprm::AttnWorkH
     return at;
   };
   c.err = take(sizeof(int));
-  c.cnt = take(sizeof(int) * static_cast<size_t>(n) * n_kv);
-  c.items = take(sizeof(kvprm::AttnItem) * w.items.size());
+  c.segs = take(sizeof(kvprm::AttnSeg) * w.segs.size());
+  c.cta = take(sizeof(int32_t) * w.cta_seg.size());
   c.pages = take(sizeof(int32_t) * w.pages.size());
   c.cands = take(sizeof(int32_t) * w.cands.size());
   c.slots = take(sizeof(int32_t) * w.slots.size());
+  c.base = take(sizeof(int32_t) * w.slot_base.size());
   c.nslots = take(sizeof(int32_t) * w.nslots.size());
   const size_t qe = static_cast<size_t>(n) * n_q * hd;
   c.qhi = take(2 * qe);
   c.qlo = take(2 * qe);
   c.ohi = take(2 * qe);
   c.olo = take(2 * qe);
-  c.pml = take(sizeof(float) * static_cast<size_t>(n) * n_q * stride * 2);
-  c.po = take(sizeof(float) * qe * stride);
+  const size_t group = static_cast<size_t>(n_q / n_kv);
+  c.pml = take(sizeof(float) * static_cast<size_t>(w.n_slots) * group * 2);
+  c.po = take(sizeof(float) * static_cast<size_t>(w.n_slots) * group * hd);
   c.total = off;
   return c;
 }
@@ -145,19 +146,20 @@ extern "C" int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, co
   int dev = 0, sms = 148;
   if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     return KVPRM_ECUDA;
-  // the work list with the most partial slots per candidate (<= kSplitCapMax)
-  // whose list and partials fit in the array
+  // the attention schedule, with shared-prefix runs if they fit the array,
+  // else with private runs only
   thread_local kvprm::AttnWorkHost work;
   Carve cv;
-  int stride = kSplitCapMax;
-  for (;; stride /= 2) {
-    if (kvprm::build_attn_work(block_table, seq_lens, n, max_blocks_per_seq, n_kv_heads, head_dim, sms, stride, true,
-                               work)) {
-      cv = carve(n, n_q_heads, n_kv_heads, head_dim, stride, work);
-      if (cv.total <= static_cast<size_t>(KVPRM_NOALLOC_SCRATCH_BYTES)) break;
-    }
-    if (stride == 1) return KVPRM_ECAPACITY;   // does not fit even with one slot per candidate
+  bool fits = false;
+  for (int share = 1; share >= 0 && !fits; --share) {
+    if (!kvprm::build_attn_work(block_table, seq_lens, n, max_blocks_per_seq, n_kv_heads, n_q_heads / n_kv_heads, sms,
+                                SIZE_MAX, share != 0,
+                                work))
+      continue;
+    cv = carve(n, n_q_heads, n_kv_heads, head_dim, work);
+    fits = cv.total <= static_cast<size_t>(KVPRM_NOALLOC_SCRATCH_BYTES);
   }
+  if (!fits) return KVPRM_ECAPACITY;
 
   // tensor map over this layer's pages (built on the host stack; no allocation)
   const void* pool = kv_layer;
@@ -166,58 +168,47 @@ extern "C" int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, co
     pool = scratch;
     pages = 1;
   }
-  const int64_t rows = pages * 2 * n_kv_heads * 16;
-  if (rows >= (static_cast<int64_t>(1) << 31)) return KVPRM_EUNSUPPORTED;
-  as.layer_rows = rows;
+  if (2 * pages >= (static_cast<int64_t>(1) << 31)) return KVPRM_EUNSUPPORTED;
+  as.layer_pages = pages;
   CUtensorMap tm;
-  {
-    cuuint64_t dims[2] = {static_cast<cuuint64_t>(head_dim), static_cast<cuuint64_t>(rows)};
-    cuuint64_t strides[1] = {static_cast<cuuint64_t>(head_dim) * 2};
-    cuuint32_t box[2] = {64, 16};
-    cuuint32_t estr[2] = {1, 1};
-    if (g_encode(&tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(pool), dims, strides, box, estr,
-                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-      return KVPRM_ECUDA;
-  }
+  if (kvprm::encode_pool_map(g_encode, &tm, pool, pages, n_kv_heads, head_dim) != CUDA_SUCCESS) return KVPRM_ECUDA;
 
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   int* err = reinterpret_cast<int*>(scratch + cv.err);
-  int* cnt = reinterpret_cast<int*>(scratch + cv.cnt);
   kvprm::HiLo Q{reinterpret_cast<__nv_bfloat16*>(scratch + cv.qhi), reinterpret_cast<__nv_bfloat16*>(scratch + cv.qlo)};
   __nv_bfloat16* ohi = reinterpret_cast<__nv_bfloat16*>(scratch + cv.ohi);
   __nv_bfloat16* olo = reinterpret_cast<__nv_bfloat16*>(scratch + cv.olo);
   float* pml = reinterpret_cast<float*>(scratch + cv.pml);
   float* po = reinterpret_cast<float*>(scratch + cv.po);
   kvprm::AttnWork wk;
-  wk.items = reinterpret_cast<const kvprm::AttnItem*>(scratch + cv.items);
+  wk.segs = reinterpret_cast<const kvprm::AttnSeg*>(scratch + cv.segs);
+  wk.cta_seg = reinterpret_cast<const int32_t*>(scratch + cv.cta);
   wk.pages = reinterpret_cast<const int32_t*>(scratch + cv.pages);
   wk.cands = reinterpret_cast<const int32_t*>(scratch + cv.cands);
   wk.slots = reinterpret_cast<const int32_t*>(scratch + cv.slots);
+  wk.slot_base = reinterpret_cast<const int32_t*>(scratch + cv.base);
   wk.nslots = reinterpret_cast<const int32_t*>(scratch + cv.nslots);
-  wk.n_items = static_cast<int>(work.items.size());
+  wk.n_ctas = work.n_ctas;
 
-  // the error word and the split-arrival counters must start at zero; everything
-  // else is written before it is read
+  // the error word must start at zero; everything else is written before it is read
   if (cudaMemsetAsync(err, 0, sizeof(int), st) != cudaSuccess) return KVPRM_ECUDA;
-  if (cudaMemsetAsync(cnt, 0, sizeof(int) * static_cast<size_t>(n) * n_kv_heads, st) != cudaSuccess)
-    return KVPRM_ECUDA;
   // pageable host sources: each copy is staged by the driver before it returns,
   // so the thread-local work list may be rebuilt by the next call
   auto up = [&](size_t off, const void* src, size_t bytes) {
     return bytes == 0 || cudaMemcpyAsync(scratch + off, src, bytes, cudaMemcpyHostToDevice, st) == cudaSuccess;
   };
-  if (!up(cv.items, work.items.data(), sizeof(kvprm::AttnItem) * work.items.size()) ||
+  if (!up(cv.segs, work.segs.data(), sizeof(kvprm::AttnSeg) * work.segs.size()) ||
+      !up(cv.cta, work.cta_seg.data(), sizeof(int32_t) * work.cta_seg.size()) ||
       !up(cv.pages, work.pages.data(), sizeof(int32_t) * work.pages.size()) ||
       !up(cv.cands, work.cands.data(), sizeof(int32_t) * work.cands.size()) ||
       !up(cv.slots, work.slots.data(), sizeof(int32_t) * work.slots.size()) ||
+      !up(cv.base, work.slot_base.data(), sizeof(int32_t) * work.slot_base.size()) ||
       !up(cv.nslots, work.nslots.data(), sizeof(int32_t) * work.nslots.size()))
     return KVPRM_ECUDA;
   if (kvprm::launch_split_hilo(q, static_cast<int64_t>(n) * n_q_heads * head_dim, Q, st) != cudaSuccess)
     return KVPRM_ECUDA;
-  const kvprm::AttnMerge mg{q, k_self, v_self, cnt, ohi, olo, out, nullptr};
-  if (kvprm::launch_attention(as, wk, work.max_item_pages, &tm, 0, Q.hi, Q.lo, stride, po, pml, mg, err, st, false) !=
-      cudaSuccess)
-    return KVPRM_ECUDA;
+  const kvprm::AttnMerge mg{q, k_self, v_self, ohi, olo, out, nullptr};
+  if (kvprm::launch_attention(as, wk, &tm, 0, Q.hi, Q.lo, po, pml, err, st, false) != cudaSuccess) return KVPRM_ECUDA;
+  if (kvprm::launch_attn_combine(as, wk, n, po, pml, mg, st, false) != cudaSuccess) return KVPRM_ECUDA;
   return KVPRM_OK;
 }
