@@ -213,6 +213,46 @@ KVPRM_API int kvprm_debug_layers(kvprm_ctx* ctx, int which, void* d_out);
  * Blocking. */
 KVPRM_API int kvprm_resolve(kvprm_ctx* ctx, int32_t b, int64_t* phys_row);
 
+/* The paged-attention schedule a scoring call builds (host only; no context,
+ * no GPU).  The paper's read-out (App. A.3) is split here into segments: a
+ * segment is a run of physical pages of one kv head scored for one candidate
+ * (kind 0) or, when pages are shared by several candidates (a beam prefix or
+ * MCTS ancestors), for up to 8 of them at once (kind 1).  Segments are cut so
+ * that each of n_ctas CTAs gets an equal share of the estimated cost; each
+ * segment writes partial softmax states ("slots") that are merged per
+ * (candidate, kv head) with the verify token's own entry.
+ * Inputs: block_table host int32 [n_candidates][max_blocks_per_seq], seq_lens
+ * host int32 [n_candidates], group = n_q_heads / n_kv_heads, n_ctas >= 1,
+ * share != 0 to form shared segments.  Outputs go to caller-owned arrays with
+ * the capacities given (elements); the counts are always written:
+ *  segs       [n_segs][8] int32: kind, kv head, candidate (kind 0) or offset
+ *             into cands (kind 1), candidates, offset into pages, pages, valid
+ *             tokens of the last page, slot (kind 0) or offset into slots
+ *  cta_seg    [n_ctas + 1] first segment of each CTA
+ *  pages      physical page ids referenced by segments
+ *  cands      candidates of kind-1 segments; slots: their partial slots
+ *  slot_base, nslots  [n_candidates][n_kv_heads] first slot and slot count
+ * Returns KVPRM_EINVAL for bad arguments and KVPRM_ECAPACITY if an array is
+ * too small (counts still reflect the full plan). */
+typedef struct {
+  int32_t n_segs, n_ctas, n_pages, n_cands, n_slot_refs, n_slots; /* out */
+  int32_t* segs;
+  int64_t segs_cap; /* segments (8 ints each) */
+  int32_t* cta_seg;
+  int64_t cta_cap;
+  int32_t* pages;
+  int64_t pages_cap;
+  int32_t* cands;
+  int64_t cands_cap;
+  int32_t* slots;
+  int64_t slots_cap;
+  int32_t* slot_base; /* [n_candidates * n_kv_heads] */
+  int32_t* nslots;    /* [n_candidates * n_kv_heads] */
+} kvprm_attn_plan;
+KVPRM_API int kvprm_plan_attention(const int32_t* block_table, int32_t max_blocks_per_seq, const int32_t* seq_lens,
+                                   int32_t n_candidates, int32_t n_kv_heads, int32_t group, int32_t n_ctas,
+                                   int32_t share, kvprm_attn_plan* plan);
+
 /* Device-side status: returns KVPRM_OK, or KVPRM_ETIMEOUT if an in-kernel
  * bounded wait gave up since the last check (the flag is then cleared).
  * Synchronises the context's last stream. */

@@ -998,6 +998,46 @@ int kvprm_resolve(kvprm_ctx* ctx, int32_t b, int64_t* phys_row) {
   return KVPRM_OK;
 }
 
+int kvprm_plan_attention(const int32_t* block_table, int32_t max_blocks_per_seq, const int32_t* seq_lens,
+                         int32_t n_candidates, int32_t n_kv_heads, int32_t group, int32_t n_ctas, int32_t share,
+                         kvprm_attn_plan* plan) {
+  if (!plan || n_candidates < 0 || max_blocks_per_seq < 1 || n_kv_heads < 1 || group < 1 || group > 16 ||
+      n_ctas < 1)
+    return KVPRM_EINVAL;
+  if (n_candidates > 0 && (!block_table || !seq_lens)) return KVPRM_EINVAL;
+  for (int b = 0; b < n_candidates; ++b)
+    if (seq_lens[b] < 0 || static_cast<int64_t>(seq_lens[b]) > static_cast<int64_t>(max_blocks_per_seq) * 16)
+      return KVPRM_EINVAL;
+  kvprm::AttnWorkHost w;
+  if (!kvprm::build_attn_work(block_table, seq_lens, n_candidates, max_blocks_per_seq, n_kv_heads, group, n_ctas,
+                              SIZE_MAX, share != 0, w))
+    return KVPRM_ECAPACITY;
+  plan->n_segs = static_cast<int32_t>(w.segs.size());
+  plan->n_ctas = w.n_ctas;
+  plan->n_pages = static_cast<int32_t>(w.pages.size());
+  plan->n_cands = static_cast<int32_t>(w.cands.size());
+  plan->n_slot_refs = static_cast<int32_t>(w.slots.size());
+  plan->n_slots = w.n_slots;
+  constexpr size_t kSegInts = sizeof(kvprm::AttnSeg) / sizeof(int32_t);
+  static_assert(kSegInts == 8, "segment layout");
+  auto fits = [](const int32_t* p, int64_t cap, size_t need) { return need == 0 || (p && cap >= static_cast<int64_t>(need)); };
+  if (!fits(plan->segs, plan->segs_cap, w.segs.size()) || !fits(plan->cta_seg, plan->cta_cap, w.cta_seg.size()) ||
+      !fits(plan->pages, plan->pages_cap, w.pages.size()) || !fits(plan->cands, plan->cands_cap, w.cands.size()) ||
+      !fits(plan->slots, plan->slots_cap, w.slots.size()) ||
+      (!w.slot_base.empty() && (!plan->slot_base || !plan->nslots)))
+    return KVPRM_ECAPACITY;
+  if (!w.segs.empty()) std::memcpy(plan->segs, w.segs.data(), sizeof(kvprm::AttnSeg) * w.segs.size());
+  if (!w.cta_seg.empty()) std::memcpy(plan->cta_seg, w.cta_seg.data(), sizeof(int32_t) * w.cta_seg.size());
+  if (!w.pages.empty()) std::memcpy(plan->pages, w.pages.data(), sizeof(int32_t) * w.pages.size());
+  if (!w.cands.empty()) std::memcpy(plan->cands, w.cands.data(), sizeof(int32_t) * w.cands.size());
+  if (!w.slots.empty()) std::memcpy(plan->slots, w.slots.data(), sizeof(int32_t) * w.slots.size());
+  if (!w.slot_base.empty()) {
+    std::memcpy(plan->slot_base, w.slot_base.data(), sizeof(int32_t) * w.slot_base.size());
+    std::memcpy(plan->nslots, w.nslots.data(), sizeof(int32_t) * w.nslots.size());
+  }
+  return KVPRM_OK;
+}
+
 int kvprm_check_device(kvprm_ctx* ctx) {
   if (!ctx) return KVPRM_EINVAL;
   CK(cudaStreamSynchronize(ctx->last_stream), "cudaStreamSynchronize");

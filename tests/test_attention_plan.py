@@ -1,0 +1,146 @@
+"""Host logic of the paged-attention schedule (kvprm_plan_attention; no GPU).
+
+The read-out of App. A.3 is split into segments of pages scored per kv head;
+whatever the split, every cached token of every candidate must be scored
+exactly once per kv head, every partial slot must belong to exactly one
+(candidate, kv head), and the CTAs must get equal shares of the work.  These
+checks recompute all of that from the block tables, independently of the
+planner."""
+import collections
+
+import numpy as np
+import pytest
+
+import kvsynth as ks
+import paper_2607_09153_gb300.kvprm as kp
+
+PRIVATE_COST, SHARED_COST_PER_CAND = 4, 2   # the planner's per-page cost model
+
+
+def check_plan(bt, sl, n_kv, group, n_ctas, share):
+    bt = np.asarray(bt, np.int32)
+    sl = np.asarray(sl, np.int32)
+    n = len(sl)
+    p = kp.kvprm_plan_attention(bt, sl, n_kv, group, n_ctas, share)
+    segs, cta = p["segs"], p["cta_seg"]
+    # expected multiset of (b, g, page, valid tokens)
+    want = collections.Counter()
+    for b in range(n):
+        npg = (int(sl[b]) + 15) // 16
+        for g in range(n_kv):
+            for j in range(npg):
+                want[(b, g, int(bt[b, j]), 16 if j < npg - 1 else int(sl[b]) - 16 * (npg - 1))] += 1
+    got = collections.Counter()
+    used = collections.defaultdict(list)   # (b, g) -> slots
+    assert p["n_ctas"] <= n_ctas
+    if p["n_ctas"]:
+        assert cta[0] == 0 and cta[-1] == len(segs) and np.all(np.diff(cta) >= 0)
+    cost = np.zeros(max(p["n_ctas"], 1))
+    for k in range(p["n_ctas"]):
+        for s in segs[cta[k]:cta[k + 1]]:
+            kind, g, c, nc, off, npg, last, slot = (int(x) for x in s)
+            assert 0 <= g < n_kv and npg >= 1 and 1 <= last <= 16
+            pages = p["pages"][off:off + npg]
+            if kind == 0:
+                cands = [c]
+                k_slots = 1 if group <= 8 else min(8, npg)
+                slots = [[slot + i for i in range(k_slots)]]
+                cost[k] += PRIVATE_COST * npg
+            else:
+                assert share and 1 <= nc <= 8 and last == 16
+                cands = [int(x) for x in p["cands"][c:c + nc]]
+                slots = [[int(x)] for x in p["slots"][slot:slot + nc]]
+                cost[k] += SHARED_COST_PER_CAND * nc * npg
+            for b, sls in zip(cands, slots):
+                used[(b, g)] += sls
+                for i, pg in enumerate(pages):
+                    got[(b, g, int(pg), last if i == npg - 1 else 16)] += 1
+    assert got == want, "every cached token scored exactly once per kv head"
+    for b in range(n):
+        for g in range(n_kv):
+            base, cnt = int(p["slot_base"][b * n_kv + g]), int(p["nslots"][b * n_kv + g])
+            assert sorted(used[(b, g)]) == list(range(base, base + cnt)), (b, g)
+    assert int(p["nslots"].sum()) == p["n_slots"]
+    if p["n_ctas"] > 1:
+        total = cost.sum()
+        unit = PRIVATE_COST if not share else max(PRIVATE_COST, SHARED_COST_PER_CAND * 8)
+        assert np.abs(cost - total / p["n_ctas"]).max() <= unit, "equal CTA shares up to one page"
+    return p
+
+
+@pytest.mark.parametrize("name", ["tiny", "qwen1p5b_b16_l2048", "beam7b_b64_p4096_s512", "long8b_b8_l32768",
+                                  "mcts7b_b256_d4"])
+@pytest.mark.parametrize("share", [True, False])
+def test_workload_plans(name, share):
+    w = ks.make_workload(name)
+    a = w.arch
+    p = check_plan(w.block_table, w.seq_lens, a.n_kv_heads, a.n_q_heads // a.n_kv_heads, 152, share)
+    if not share:
+        assert (p["segs"][:, 0] == 0).all()
+
+
+def test_shared_prefix_is_read_once_per_chunk():
+    # 20 candidates share a 10-page prefix, then own 3 pages each
+    n, pre, own = 20, 10, 3
+    bt = np.zeros((n, pre + own), np.int32)
+    for b in range(n):
+        bt[b, :pre] = np.arange(pre)
+        bt[b, pre:] = pre + own * b + np.arange(own)
+    sl = np.full(n, 16 * (pre + own) - 5, np.int32)
+    p = check_plan(bt, sl, 2, 4, 16, True)
+    shared = p["segs"][p["segs"][:, 0] == 1]
+    # the prefix pages go to shared segments of <= 8 candidates: ceil(20 / 8) = 3 chunks per head
+    per_head = collections.Counter()
+    for s in shared:
+        per_head[int(s[1])] += int(s[5])
+    assert per_head == {0: 3 * pre, 1: 3 * pre}
+
+
+def test_repeated_page_in_one_candidate_stays_private():
+    bt = np.array([[3, 3, 4], [3, 3, 5]], np.int32)   # page 3 listed twice by both candidates
+    sl = np.array([48, 48], np.int32)
+    p = check_plan(bt, sl, 1, 2, 4, True)
+    assert (p["segs"][:, 0] == 0).all()
+
+
+def test_partial_last_page_is_never_shared():
+    bt = np.array([[0, 1], [0, 1]], np.int32)
+    sl = np.array([20, 20], np.int32)   # page 1 is partial (4 tokens) for both
+    p = check_plan(bt, sl, 1, 1, 4, True)
+    for s in p["segs"]:
+        if s[0] == 1:
+            assert 1 not in set(p["pages"][s[4]:s[4] + s[5]].tolist())
+
+
+@pytest.mark.parametrize("lens", [[0], [0, 0, 0], [1], [16], [17], [0, 1, 15, 16, 17, 31, 33, 100, 257, 1000]])
+@pytest.mark.parametrize("n_ctas", [1, 3, 152])
+def test_edges(lens, n_ctas):
+    n = len(lens)
+    mb = max(1, max((L + 15) // 16 for L in lens))
+    bt = np.arange(n * mb, dtype=np.int32).reshape(n, mb)
+    p = check_plan(bt, lens, 2, 3, n_ctas, True)
+    for b, L in enumerate(lens):
+        if L == 0:
+            assert (p["nslots"][b * 2:(b + 1) * 2] == 0).all(), "an empty cache has no partial: self entry only"
+
+
+def test_two_row_groups_count_one_slot_per_busy_warp():
+    bt = np.arange(3 * 40, dtype=np.int32).reshape(3, 40)
+    sl = np.array([5, 100, 640], np.int32)
+    check_plan(bt, sl, 1, 16, 7, True)
+
+
+def test_deterministic():
+    w = ks.make_workload("mcts7b_b256_d4")
+    a = w.arch
+    p1 = kp.kvprm_plan_attention(w.block_table, w.seq_lens, a.n_kv_heads, a.n_q_heads // a.n_kv_heads, 152)
+    p2 = kp.kvprm_plan_attention(w.block_table, w.seq_lens, a.n_kv_heads, a.n_q_heads // a.n_kv_heads, 152)
+    for k in ("segs", "cta_seg", "pages", "cands", "slots", "slot_base", "nslots"):
+        assert np.array_equal(p1[k], p2[k]), k
+
+
+def test_bad_arguments():
+    with pytest.raises(kp.KvprmError):
+        kp.kvprm_plan_attention(np.zeros((1, 1), np.int32), [17], 1, 1, 4)   # 17 tokens > 16 * 1 block
+    with pytest.raises(kp.KvprmError):
+        kp.kvprm_plan_attention(np.zeros((1, 1), np.int32), [1], 1, 17, 4)   # G > 16
