@@ -380,6 +380,76 @@ def run_gpu(args, world, rank, local):
         print(json.dumps(line), flush=True)
 
 
+def run_attention_only(args, world, rank, local):
+    """The paged attention read-out alone (kvprm_attention: split-K attention
+    plus combine) on ONE layer of the workload's cache, timed per kernel with
+    CUDA events; a few-GB footprint, the case ncu captures use."""
+    import dataclasses
+
+    import torch
+
+    import kvsynth as ks
+    import paper_2607_09153_gb300 as kp
+
+    torch.cuda.set_device(local)
+    w = ks.make_workload(args.workload)
+    a = w.arch
+    # the workload's heads and cache on a one-layer scorer (its projections are never run here)
+    w1 = dataclasses.replace(w, arch=ks.Arch(1, 256, a.n_q_heads, a.n_kv_heads, a.head_dim, 256, a.rope_base,
+                                             a.rms_eps))
+    dev = ks.DeviceInputs(w1, ks.Tables.make())
+    B = w.n_candidates
+    sc = make_scorer(dev, B, w.max_blocks)
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(7)
+    q = torch.randn(B, a.n_q_heads, a.head_dim, device="cuda", generator=gen)
+    kself = torch.randn(B, a.n_kv_heads, a.head_dim, device="cuda", generator=gen)
+    vself = torch.randn(B, a.n_kv_heads, a.head_dim, device="cuda", generator=gen)
+    out = torch.empty_like(q)
+    stream = torch.cuda.Stream()
+    bt, sl = np.ascontiguousarray(w.block_table), np.ascontiguousarray(w.seq_lens)
+
+    def step():
+        kp.kvprm_attention(sc.ctx, dev.pool[0].data_ptr(), dev.n_pages, bt, sl, B, q.data_ptr(), kself.data_ptr(),
+                           vself.data_ptr(), out.data_ptr(), stream.cuda_stream)
+
+    for _ in range(args.warmup):
+        step()
+    stream.synchronize()
+    clocks = ClockSampler(local)
+    clocks.start()
+    kp.kvprm_set_profile(sc.ctx, True)
+    for _ in range(args.steps):
+        step()
+    prof = kp.kvprm_get_profile(sc.ctx)
+    kp.kvprm_set_profile(sc.ctx, False)
+    clk = clocks.stop()
+    kp.kvprm_check_device(sc.ctx)
+    n_at, t_at = prof["attention"]
+    n_cb, t_cb = prof["combine"]
+    kv_bytes = w.unique_kv_bytes() // a.n_layers   # one layer, each distinct page once
+    at_s = t_at / n_at / 1000.0
+    peaks = load_peaks()
+    ach = kv_bytes / at_s / 1e9
+    line = {
+        "metric": "paged attention HBM GB/s (one layer, kernel time)", "value": round(ach, 1), "unit": "GB/s",
+        "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "higher_is_better": True, "dtype": "bf16",
+        "data": "synthetic (seeded K/V N(0,1); random fp32 q / self k / self v)",
+        "config": dict(workload_config(w, args), layers=1,
+                       l2="one layer's cache; inputs larger than L2 except small workloads, no flush"),
+        "roofline": {"bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                     "frac": round(ach / peaks["hbm_gbs"], 4), "peak_src": peaks["src"],
+                     "frac_of_8tbs": round(ach / HBM_NOMINAL_GBS, 4), "traffic": ncu_traffic("attention", w.name),
+                     "kernel": "attention", "algorithmic_bytes_per_launch": int(kv_bytes),
+                     "avg_launch_us": round(at_s * 1e6, 3)},
+        "combine_avg_us": round(1000 * t_cb / max(n_cb, 1), 3),
+        "clocks": clk,
+    }
+    sc.close()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
 def main():
     import kvsynth as ks
     ap = argparse.ArgumentParser()
@@ -391,12 +461,16 @@ def main():
     ap.add_argument("--profile-steps", type=int, default=50)
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--attention-only", action="store_true",
+                    help="time the paged attention alone on one layer of the workload's cache")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
     world, rank, local = dist_setup()
     if args.impl == "reference":
         run_reference(args, world, rank)
+    elif args.attention_only:
+        run_attention_only(args, world, rank, local)
     else:
         run_gpu(args, world, rank, local)
     if world > 1:
