@@ -5,12 +5,13 @@
 // hi = bf16(x), lo = bf16(x - hi), so no bf16 rounding of the activation
 // itself enters the result.
 //   rope_table   cos/sin of p * base^(-2i/hd) at p = L_b (fp64 angles)
-//   embed_norm   h = e_v ; per-tile sums of squares of h ; x = RMSNorm(h) * g
-//   norm         x = h * r * g with r = 1/sqrt(mean(h^2) + eps), mean(h^2)
-//                from the per-128-row-tile sums of squares the residual
-//                GEMM epilogue wrote (summed in tile order: deterministic)
-//   head         x = RMSNorm(h) * g_final ; P(+) = 1/(1 + exp(w_minus.x - w_plus.x))
-//                (Eq. score, App. B.2)
+//   embed_norm   h = e_v ; per-tile sums of squares of h ; x = h ⊙ g (the
+//                RMSNorm's per-candidate factor 1/sqrt(mean(h^2) + eps) is
+//                applied by the QKV epilogue, as between all projections)
+//   head         x = RMSNorm(h) * g_final with mean(h^2) from the per-tile
+//                sums of squares the last residual epilogue wrote (summed in
+//                tile order: deterministic);
+//                P(+) = 1/(1 + exp(w_minus.x - w_plus.x)) (Eq. score, App. B.2)
 #include <cuda_bf16.h>
 
 #include "kernels.h"
@@ -67,21 +68,13 @@ __global__ void rope_table_kernel(const int32_t* __restrict__ seq_lens, int hd, 
 
 // One CTA per candidate: h = e_v, its per-tile sums of squares, and x.
 __global__ void embed_norm_kernel(const __nv_bfloat16* __restrict__ e_v, const __nv_bfloat16* __restrict__ gain,
-                                  int d, float eps, int n_cand, float* __restrict__ h, float* __restrict__ sumsq,
-                                  HiLo x, unsigned long long* ts) {
+                                  int d, int n_cand, float* __restrict__ h, float* __restrict__ sumsq, HiLo x,
+                                  unsigned long long* ts) {
   trace_begin(ts);
-  __shared__ float red[32];
   grid_dep_launch();
   grid_dep_wait();
   const int b = blockIdx.x;
-  float ss = 0.f;
-  for (int c = threadIdx.x; c < d; c += blockDim.x) {
-    const float v = __bfloat162float(e_v[c]);
-    h[static_cast<int64_t>(b) * d + c] = v;
-    ss += v * v;
-  }
-  const float total = block_sum(ss, red);
-  // per-tile partial sums, as the residual GEMM epilogue writes them (only their sum is used)
+  // per-tile sums of squares of h, as the residual GEMM epilogue writes them
   const int m_tiles = (d + 127) / 128;
   if (threadIdx.x < m_tiles) {
     float t = 0.f;
@@ -91,26 +84,12 @@ __global__ void embed_norm_kernel(const __nv_bfloat16* __restrict__ e_v, const _
     }
     sumsq[static_cast<int64_t>(threadIdx.x) * n_cand + b] = t;
   }
-  const float r = 1.0f / sqrtf(total / d + eps);
-  for (int c = threadIdx.x; c < d; c += blockDim.x)
-    store_hilo(x, static_cast<int64_t>(b) * d + c, __bfloat162float(e_v[c]) * r * __bfloat162float(gain[c]));
-  trace_end(ts);
-}
-
-// grid (n_cand, ceil(d / blockDim)): elementwise RMSNorm from the tile sums.
-__global__ void norm_kernel(const float* __restrict__ h, const float* __restrict__ sumsq, int m_tiles, int n_cand,
-                            int d, float eps, const __nv_bfloat16* __restrict__ gain, HiLo x,
-                            unsigned long long* ts) {
-  trace_begin(ts);
-  __shared__ float slot;
-  grid_dep_launch();
-  grid_dep_wait();
-  const int b = blockIdx.x;
-  const float r = row_rscale(sumsq, m_tiles, n_cand, b, d, eps, &slot);
-  const int c = blockIdx.y * blockDim.x + threadIdx.x;
-  if (c < d) {
-    const int64_t i = static_cast<int64_t>(b) * d + c;
-    store_hilo(x, i, h[i] * r * __bfloat162float(gain[c]));
+  // h = e_v, and the QKV projection's input h ⊙ g before the RMSNorm's
+  // per-candidate factor, which its epilogue applies from the tile sums
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    const float v = __bfloat162float(e_v[c]);
+    h[static_cast<int64_t>(b) * d + c] = v;
+    store_hilo(x, static_cast<int64_t>(b) * d + c, v * __bfloat162float(gain[c]));
   }
   trace_end(ts);
 }
@@ -171,15 +150,7 @@ cudaError_t launch_embed_norm(const ModelDims& m, const __nv_bfloat16* e_v, cons
                               unsigned long long* ts) {
   cudaLaunchAttribute attr[1];
   cudaLaunchConfig_t cfg = make_cfg(dim3(n_cand), dim3(256), stream, attr, pdl);
-  return cudaLaunchKernelEx(&cfg, embed_norm_kernel, e_v, gain, m.d, m.eps, n_cand, h, sumsq, x, ts);
-}
-
-cudaError_t launch_norm(const ModelDims& m, const float* h, const float* sumsq, int m_tiles, int n_cand,
-                        const __nv_bfloat16* gain, HiLo x, cudaStream_t stream, bool pdl, unsigned long long* ts) {
-  cudaLaunchAttribute attr[1];
-  const int threads = 256;
-  cudaLaunchConfig_t cfg = make_cfg(dim3(n_cand, (m.d + threads - 1) / threads), dim3(threads), stream, attr, pdl);
-  return cudaLaunchKernelEx(&cfg, norm_kernel, h, sumsq, m_tiles, n_cand, m.d, m.eps, gain, x, ts);
+  return cudaLaunchKernelEx(&cfg, embed_norm_kernel, e_v, gain, m.d, n_cand, h, sumsq, x, ts);
 }
 
 cudaError_t launch_head(const ModelDims& m, const float* h, const float* sumsq, int m_tiles, int n_cand,

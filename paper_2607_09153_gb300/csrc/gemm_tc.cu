@@ -20,10 +20,17 @@
 //   PLAIN  out[n][m] = y
 //   QKV    RoPE on the q and k rows (rotate-half pairs inside a head) -> q
 //          (fp32 and bf16 hi/lo), self k, self v (fp32)
-//   RESID  h[n][m] += y, and the tile's sum of squares of the new h per
-//          candidate (the next RMSNorm reads these partial sums)
+//   RESID  h[n][m] += y, the tile's sum of squares of the new h per
+//          candidate, and h ⊙ g (g = the next RMSNorm's gain) as the next
+//          projection's bf16 hi/lo input
 //   SILU   rows are 64 gate rows and the matching 64 up rows (two TMA boxes
 //          per stage); a = SiLU(gate) * up as a bf16 hi/lo pair
+// An RMSNorm x = g ⊙ h / sqrt(mean(h^2) + eps) between two projections is
+// thereby split: the per-candidate factor r = 1/sqrt(mean(h^2) + eps) is a
+// scalar of the column, so W x = r (W (h ⊙ g)); the residual epilogue writes
+// h ⊙ g and the per-tile sums of squares, and the QKV and SILU epilogues scale
+// their accumulators by r before RoPE / SiLU.  No normalisation kernel runs
+// between the projections.
 #include "kernels.h"
 #include "ptx.cuh"
 
@@ -34,6 +41,9 @@ namespace {
 constexpr int kBM = 128;
 constexpr int kBK = 64;
 constexpr uint32_t kWTileBytes = kBM * kBK * 2;   // 16 KB
+// after the ring: barriers, TMEM slot and 64 block-sum floats (512 B), then 256
+// per-column RMSNorm factors (1 KB)
+constexpr size_t kTailBytes = 512 + 1024;
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -78,6 +88,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
   uint64_t* done = empty + stages;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
   float* red = reinterpret_cast<float*>(tmem_slot + 4);   // 64 floats for per-column block sums
+  float* rsc = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full) + 512);   // RMSNorm factor per column
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int m_tile = blockIdx.x / cs;
@@ -227,6 +238,14 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       }
     }
   }
+  // the RMSNorm factor of each of this rank's columns (QKV, SILU)
+  if (ep.rs_sumsq)
+    for (int t0 = threadIdx.x; t0 < nc; t0 += blockDim.x) {   // nc <= 256 columns
+      const int c = cbeg + t0;
+      float ssum = 0.f;
+      for (int t = 0; t < ep.rs_tiles; ++t) ssum += ep.rs_sumsq[static_cast<int64_t>(t) * ep.n_valid + c];
+      rsc[t0] = 1.0f / sqrtf(ssum / ep.rs_d + ep.rs_eps);
+    }
   __syncthreads();
   // Step 2: the epilogue over (row, column) pairs, all threads in parallel
   if (ep.mode == GemmEpilogue::PLAIN) {
@@ -244,6 +263,8 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
           float* hp = ep.h + static_cast<int64_t>(c) * ep.M + gm;
           hv = *hp + acc[c * kBM + m];
           *hp = hv;
+          if (ep.gain_next)
+            store_hilo(ep.x_hi, ep.x_lo, static_cast<int64_t>(c) * ep.M + gm, hv * __bfloat162float(ep.gain_next[gm]));
         }
         float sq = hv * hv;
 #pragma unroll
@@ -262,7 +283,8 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     const int j = m_tile * 64 + r;
     if (j < ep.ff)
       for (int c = cbeg + half_sel; c < cend; c += 2) {
-        const float g = acc[c * kBM + r], u = acc[c * kBM + 64 + r];
+        const float rs = ep.rs_sumsq ? rsc[c - cbeg] : 1.f;
+        const float g = acc[c * kBM + r] * rs, u = acc[c * kBM + 64 + r] * rs;
         store_hilo(ep.a_hi, ep.a_lo, static_cast<int64_t>(c) * ep.ff + j, g / (1.0f + expf(-g)) * u);
       }
   } else {   // QKV: pair p = m & 63 of this tile, two column groups of 64 threads
@@ -273,7 +295,8 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     const int grow = m_tile * kBM + row_a;              // row of W_qkv
     const int head = grow / hd, i = grow % hd;          // i < half
     for (int c = cbeg + half_sel; c < cend; c += 2) {
-      float a = acc[c * kBM + row_a], b = acc[c * kBM + row_b];
+      const float rs = ep.rs_sumsq ? rsc[c - cbeg] : 1.f;
+      float a = acc[c * kBM + row_a] * rs, b = acc[c * kBM + row_b] * rs;
       if (head < ep.n_q + ep.n_kv) {
         const float2 cs2 = ep.rope[c * half + i];
         const float a2 = a * cs2.x - b * cs2.y;
@@ -317,7 +340,7 @@ GemmPlan plan_gemm(int M, int K, int n_pad, int num_sms, bool has_lo, bool gate_
   size_t ring = static_cast<size_t>(p.stages) * stage_bytes;
   const size_t acc = static_cast<size_t>(n_pad) * kBM * 4;
   if (ring < acc) ring = acc;
-  p.smem_bytes = ring + 1024 /*align*/ + 512 /*barriers, TMEM slot, block sums*/;
+  p.smem_bytes = ring + 1024 /*align*/ + kTailBytes;
   // cluster size: the largest power of two <= 16 that keeps the CTA count within
   // two per SM and gives every rank at least two K tiles
   int cs = 1;
@@ -330,7 +353,7 @@ GemmPlan plan_gemm(int M, int K, int n_pad, int num_sms, bool has_lo, bool gate_
   if (p.stages > p.kt_per_split) p.stages = p.kt_per_split < 2 ? 2 : p.kt_per_split;
   ring = static_cast<size_t>(p.stages) * stage_bytes;
   if (ring < acc) ring = acc;
-  p.smem_bytes = ring + 1024 /*align*/ + 512 /*barriers, TMEM slot, block sums*/;
+  p.smem_bytes = ring + 1024 /*align*/ + kTailBytes;
   uint32_t cols = 32;
   while (cols < static_cast<uint32_t>(n_pad)) cols <<= 1;
   p.tmem_cols = cols;

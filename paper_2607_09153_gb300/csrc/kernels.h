@@ -28,6 +28,16 @@ struct GemmEpilogue {
   float* out = nullptr;  // PLAIN: [n][M]
   float* h = nullptr;    // RESID: [n][M], updated in place
   float* sumsq = nullptr;  // RESID: [m_tiles][n] sum of squares of the new h per tile
+  // RESID: when set, also x = h ⊙ gain (the next RMSNorm's input before its
+  // per-candidate scale) as a bf16 hi/lo pair [n][M] for the next projection
+  const __nv_bfloat16* gain_next = nullptr;
+  __nv_bfloat16* x_hi = nullptr;
+  __nv_bfloat16* x_lo = nullptr;
+  // QKV, SILU: when set, the input was h ⊙ gain and the accumulator is scaled
+  // per candidate by the RMSNorm factor 1/sqrt(sum_t rs_sumsq[t][n] / rs_d + rs_eps)
+  const float* rs_sumsq = nullptr;
+  int rs_tiles = 0, rs_d = 0;
+  float rs_eps = 0.f;
   const float2* rope = nullptr;  // QKV: [n][hd/2] (cos, sin)
   int n_q = 0, n_kv = 0, hd = 0;
   float* q = nullptr;
@@ -133,10 +143,6 @@ struct HiLo {
 cudaError_t launch_embed_norm(const ModelDims& m, const __nv_bfloat16* e_v, const __nv_bfloat16* gain,
                               int n_cand, float* h, float* sumsq, HiLo x, cudaStream_t stream, bool pdl,
                               unsigned long long* ts = nullptr);
-// x = h * r * gain as a hi/lo pair, r = 1/sqrt(sum of the m_tiles partial sums of squares / d + eps)
-cudaError_t launch_norm(const ModelDims& m, const float* h, const float* sumsq, int m_tiles, int n_cand,
-                        const __nv_bfloat16* gain, HiLo x, cudaStream_t stream, bool pdl,
-                        unsigned long long* ts = nullptr);
 // rewards = P(+) from the final RMSNorm of h and the two head rows
 cudaError_t launch_head(const ModelDims& m, const float* h, const float* sumsq, int m_tiles, int n_cand,
                         const __nv_bfloat16* gain, const __nv_bfloat16* w_plus, const __nv_bfloat16* w_minus,

@@ -426,12 +426,19 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
   eq.q_lo = ctx->qlo;
   eq.kself = ctx->kself;
   eq.vself = ctx->vself;
+  // the pre-attention RMSNorm's per-candidate factor, from the residual stream's tile sums of squares
+  eq.rs_sumsq = ctx->sumsq;
+  eq.rs_tiles = ctx->d_tiles;
+  eq.rs_d = m.d;
+  eq.rs_eps = m.eps;
   kvprm::GemmEpilogue er;   // O and down projections -> residual stream + tile sums of squares
   er.mode = kvprm::GemmEpilogue::RESID;
   er.M = m.d;
   er.n_valid = n;
   er.h = ctx->h;
   er.sumsq = ctx->sumsq;
+  er.x_hi = X.hi;   // h ⊙ (next RMSNorm gain): the next projection's input
+  er.x_lo = X.lo;
   kvprm::GemmEpilogue es;   // gate/up projection -> SiLU(gate) * up
   es.mode = kvprm::GemmEpilogue::SILU;
   es.M = m.ff;
@@ -439,6 +446,10 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
   es.ff = m.ff;
   es.a_hi = ctx->ahi;
   es.a_lo = ctx->alo;
+  es.rs_sumsq = ctx->sumsq;   // the pre-MLP RMSNorm's per-candidate factor
+  es.rs_tiles = ctx->d_tiles;
+  es.rs_d = m.d;
+  es.rs_eps = m.eps;
   ctx->trace_n = 0;
   ctx->trace_cls.clear();
   if (ctx->trace)
@@ -466,23 +477,21 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
            "attention");
     LAUNCH(KVPRM_PROF_COMBINE,
            kvprm::launch_attn_combine(ctx->as, wk, n, ctx->apart_o, ctx->apart_ml, mg, st, pdl, TS), "attn_combine");
+    kvprm::GemmEpilogue er_o = er;   // h += W_o o; x = h ⊙ g_mlp for the gate/up projection
+    er_o.gain_next = ctx->mlp_norm[l];
     LAUNCH(KVPRM_PROF_GEMM_O,
-           kvprm::launch_gemm(P.g_o, &ctx->tm_o[l], &ctx->tm_ohi, &ctx->tm_olo, er, np, ctx->err_d, st, pdl, TS),
+           kvprm::launch_gemm(P.g_o, &ctx->tm_o[l], &ctx->tm_ohi, &ctx->tm_olo, er_o, np, ctx->err_d, st, pdl, TS),
            "gemm_o");
-    LAUNCH(KVPRM_PROF_FUSED,
-           kvprm::launch_norm(m, ctx->h, ctx->sumsq, ctx->d_tiles, n, ctx->mlp_norm[l], X, st, pdl, TS),
-           "norm_mlp");
     LAUNCH(KVPRM_PROF_GEMM_GATE_UP,
            kvprm::launch_gemm(P.g_gu, &ctx->tm_gu[l], &ctx->tm_xhi, &ctx->tm_xlo, es, np, ctx->err_d, st, pdl, TS),
            "gemm_gate_up");
+    kvprm::GemmEpilogue er_d = er;   // h += W_down a; x = h ⊙ g_attn of the next layer
+    er_d.gain_next = l + 1 < NL ? ctx->attn_norm[l + 1] : nullptr;
     LAUNCH(KVPRM_PROF_GEMM_DOWN,
-           kvprm::launch_gemm(P.g_down, &ctx->tm_down[l], &ctx->tm_ahi, &ctx->tm_alo, er, np, ctx->err_d, st, pdl, TS),
+           kvprm::launch_gemm(P.g_down, &ctx->tm_down[l], &ctx->tm_ahi, &ctx->tm_alo, er_d, np, ctx->err_d, st, pdl,
+                              TS),
            "gemm_down");
-    if (l + 1 < NL) {
-      LAUNCH(KVPRM_PROF_FUSED,
-             kvprm::launch_norm(m, ctx->h, ctx->sumsq, ctx->d_tiles, n, ctx->attn_norm[l + 1], X, st, pdl, TS),
-             "norm_attn");
-    } else {
+    if (l + 1 == NL) {
       LAUNCH(KVPRM_PROF_FUSED,
              kvprm::launch_head(m, ctx->h, ctx->sumsq, ctx->d_tiles, n, ctx->final_norm, ctx->w_plus, ctx->w_minus,
                                 ctx->rewards_d, st, pdl, TS),
