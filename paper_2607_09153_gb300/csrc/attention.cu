@@ -42,6 +42,7 @@
 #include <unordered_map>
 #include <vector>
 
+#include "attn_core.cuh"
 #include "kernels.h"
 #include "ptx.cuh"
 
@@ -49,13 +50,14 @@ namespace kvprm {
 
 namespace {
 
+using namespace ac;
+
 constexpr int kPagesPerStage = 8;
 constexpr int kStages = 3;
 constexpr int kConsumerWarps = 8;
 constexpr int kProducerWarp = kConsumerWarps;       // warp 8: TMA
 constexpr int kMergerWarp = kConsumerWarps + 1;     // warp 9: folds private segments' warp states
 constexpr int kThreads = (kConsumerWarps + 2) * 32;
-constexpr float kLog2e = 1.4426950408889634f;
 
 // Schedule costs per page and kv head.  A private page is read by one warp
 // while the other seven read the rest of its stage, so a private stage costs
@@ -74,189 +76,6 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
 // used by the resolve entry point, so indexing can be checked bit-exactly).
 __device__ __forceinline__ int32_t phys_page(const int32_t* __restrict__ bt, int b, int max_blocks, int j) {
   return bt[static_cast<int64_t>(b) * max_blocks + j];
-}
-
-// A fragments of one warp's query rows.
-template <int HD>
-struct WarpQ {
-  uint32_t a0[HD / 16], a1[HD / 16], a2[HD / 16], a3[HD / 16];   // packed: rows hi / lo; two-row: hi
-  uint32_t b0[HD / 16], b1[HD / 16], b2[HD / 16], b3[HD / 16];   // two-row: lo
-};
-
-template <int HD, bool TWO_ROWS>
-__device__ __forceinline__ void load_q(WarpQ<HD>& q, const __nv_bfloat16* __restrict__ qh,
-                                       const __nv_bfloat16* __restrict__ ql, int group, int lane) {
-  const int gid = lane >> 2, tig = lane & 3;
-  auto ldq = [&](const __nv_bfloat16* base, int row, int col) -> uint32_t {
-    return row < group ? *reinterpret_cast<const uint32_t*>(base + row * HD + col) : 0u;
-  };
-#pragma unroll
-  for (int ks = 0; ks < HD / 16; ++ks) {
-    const int c = ks * 16 + tig * 2;
-    if (!TWO_ROWS) {   // rows 0..7 = hi, rows 8..15 = lo of the same heads
-      q.a0[ks] = ldq(qh, gid, c);
-      q.a1[ks] = ldq(ql, gid, c);
-      q.a2[ks] = ldq(qh, gid, c + 8);
-      q.a3[ks] = ldq(ql, gid, c + 8);
-      q.b0[ks] = q.b1[ks] = q.b2[ks] = q.b3[ks] = 0u;
-    } else {           // a hi and a lo fragment over 16 heads
-      q.a0[ks] = ldq(qh, gid, c);
-      q.a1[ks] = ldq(qh, gid + 8, c);
-      q.a2[ks] = ldq(qh, gid, c + 8);
-      q.a3[ks] = ldq(qh, gid + 8, c + 8);
-      q.b0[ks] = ldq(ql, gid, c);
-      q.b1[ks] = ldq(ql, gid + 8, c);
-      q.b2[ks] = ldq(ql, gid, c + 8);
-      q.b3[ks] = ldq(ql, gid + 8, c + 8);
-    }
-  }
-}
-
-// Online-softmax state of one warp: per thread rows gid (and gid + 8 when two
-// rows) of the running maximum, the running sum and O.
-template <int HD>
-struct WarpState {
-  float m[2], l[2];
-  float o[HD / 8][4];
-  __device__ __forceinline__ void reset() {
-    m[0] = m[1] = -INFINITY;
-    l[0] = l[1] = 0.f;
-#pragma unroll
-    for (int n = 0; n < HD / 8; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
-  }
-};
-
-// Score one page (16 tokens, `valid` of them real) for one warp's query rows
-// and fold it into the online softmax state.  The K fragments of the whole
-// page are loaded first and S is accumulated in four independent chains; O is
-// rescaled only when some row's maximum grew (the factor is exactly 1
-// otherwise).
-template <int HD, bool TWO_ROWS>
-__device__ __forceinline__ void process_page(const WarpQ<HD>& q, uint32_t kbase, uint32_t vbase, int valid, int lane,
-                                             WarpState<HD>& st) {
-  const int tig = lane & 3;
-  const float sl2 = kLog2e * rsqrtf(static_cast<float>(HD));
-  // S = Q K^T for the page's 16 tokens (two n-tiles of 8 tokens)
-  float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
-  float t0[4] = {0.f, 0.f, 0.f, 0.f}, t1[4] = {0.f, 0.f, 0.f, 0.f};
-  {
-    const int mi = lane >> 3, r = lane & 7;
-    const int tok = (mi >> 1) * 8 + r;
-    uint32_t kb[HD / 16][4];
-#pragma unroll
-    for (int ks = 0; ks < HD / 16; ++ks) {
-      const int hdc = ks * 16 + (mi & 1) * 8;
-      const uint32_t addr = kbase + (hdc >> 6) * 2048 + tok * 128 + ((((hdc & 63) >> 3) ^ (tok & 7)) << 4);
-      ldsm_x4(addr, kb[ks][0], kb[ks][1], kb[ks][2], kb[ks][3]);
-    }
-#pragma unroll
-    for (int ks = 0; ks < HD / 16; ++ks) {
-      float(&d0)[4] = (ks & 1) ? t0 : s0;
-      float(&d1)[4] = (ks & 1) ? t1 : s1;
-      mma_bf16_16816(d0, q.a0[ks], q.a1[ks], q.a2[ks], q.a3[ks], kb[ks][0], kb[ks][1]);
-      mma_bf16_16816(d1, q.a0[ks], q.a1[ks], q.a2[ks], q.a3[ks], kb[ks][2], kb[ks][3]);
-      if (TWO_ROWS) {
-        mma_bf16_16816(d0, q.b0[ks], q.b1[ks], q.b2[ks], q.b3[ks], kb[ks][0], kb[ks][1]);
-        mma_bf16_16816(d1, q.b0[ks], q.b1[ks], q.b2[ks], q.b3[ks], kb[ks][2], kb[ks][3]);
-      }
-    }
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      s0[i] += t0[i];
-      s1[i] += t1[i];
-    }
-  }
-  const int c0 = tig * 2, c1 = tig * 2 + 1, c2 = 8 + tig * 2, c3 = 9 + tig * 2;
-  float x[2][4];
-  if (!TWO_ROWS) {   // hi (row gid) + lo (row gid + 8) parts of the same head
-    x[0][0] = s0[0] + s0[2];
-    x[0][1] = s0[1] + s0[3];
-    x[0][2] = s1[0] + s1[2];
-    x[0][3] = s1[1] + s1[3];
-  } else {
-    x[0][0] = s0[0];
-    x[0][1] = s0[1];
-    x[0][2] = s1[0];
-    x[0][3] = s1[1];
-    x[1][0] = s0[2];
-    x[1][1] = s0[3];
-    x[1][2] = s1[2];
-    x[1][3] = s1[3];
-  }
-  uint32_t ph[4], pl[4];   // A fragments of P: hi / lo
-#pragma unroll
-  for (int r = 0; r < (TWO_ROWS ? 2 : 1); ++r) {
-    x[r][0] = c0 < valid ? x[r][0] * sl2 : -INFINITY;
-    x[r][1] = c1 < valid ? x[r][1] * sl2 : -INFINITY;
-    x[r][2] = c2 < valid ? x[r][2] * sl2 : -INFINITY;
-    x[r][3] = c3 < valid ? x[r][3] * sl2 : -INFINITY;
-    float mx = fmaxf(fmaxf(x[r][0], x[r][1]), fmaxf(x[r][2], x[r][3]));
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-    const float m_new = fmaxf(st.m[r], mx);
-    if (__any_sync(0xffffffffu, m_new > st.m[r])) {   // warp-uniform: rescale O by 2^(m_old - m_new)
-      const float alpha = exp2f(st.m[r] - m_new);
-      st.l[r] *= alpha;
-      if (!TWO_ROWS) {   // one head per thread row: both MMA row halves rescale together
-#pragma unroll
-        for (int n = 0; n < HD / 8; ++n) {
-          st.o[n][0] *= alpha;
-          st.o[n][1] *= alpha;
-          st.o[n][2] *= alpha;
-          st.o[n][3] *= alpha;
-        }
-      } else {
-#pragma unroll
-        for (int n = 0; n < HD / 8; ++n) {
-          st.o[n][2 * r] *= alpha;
-          st.o[n][2 * r + 1] *= alpha;
-        }
-      }
-      st.m[r] = m_new;
-    }
-    float p[4];
-#pragma unroll
-    for (int i2 = 0; i2 < 4; ++i2) p[i2] = exp2f(x[r][i2] - m_new);
-    st.l[r] += (p[0] + p[1]) + (p[2] + p[3]);
-    float hi[4], lo[4];
-#pragma unroll
-    for (int i2 = 0; i2 < 4; ++i2) {
-      hi[i2] = __bfloat162float(__float2bfloat16_rn(p[i2]));
-      lo[i2] = p[i2] - hi[i2];
-    }
-    if (!TWO_ROWS) {
-      ph[0] = pack_bf16(hi[0], hi[1]);   // row gid: P_hi
-      ph[1] = pack_bf16(lo[0], lo[1]);   // row gid + 8: P_lo
-      ph[2] = pack_bf16(hi[2], hi[3]);
-      ph[3] = pack_bf16(lo[2], lo[3]);
-    } else {
-      ph[r] = pack_bf16(hi[0], hi[1]);
-      ph[r + 2] = pack_bf16(hi[2], hi[3]);
-      pl[r] = pack_bf16(lo[0], lo[1]);
-      pl[r + 2] = pack_bf16(lo[2], lo[3]);
-    }
-  }
-  // O += P V  (V^T fragments through ldmatrix.trans)
-  {
-    const int mi = lane >> 3;
-    const int tok = (mi & 1) * 8 + (lane & 7);
-    uint32_t vb[HD / 16][4];
-#pragma unroll
-    for (int j2 = 0; j2 < HD / 16; ++j2) {
-      const int hdc = j2 * 16 + (mi >> 1) * 8;
-      const uint32_t addr = vbase + (hdc >> 6) * 2048 + tok * 128 + ((((hdc & 63) >> 3) ^ (tok & 7)) << 4);
-      ldsm_x4_t(addr, vb[j2][0], vb[j2][1], vb[j2][2], vb[j2][3]);
-    }
-#pragma unroll
-    for (int j2 = 0; j2 < HD / 16; ++j2) {
-      mma_bf16_16816(st.o[2 * j2], ph[0], ph[1], ph[2], ph[3], vb[j2][0], vb[j2][1]);
-      mma_bf16_16816(st.o[2 * j2 + 1], ph[0], ph[1], ph[2], ph[3], vb[j2][2], vb[j2][3]);
-      if (TWO_ROWS) {
-        mma_bf16_16816(st.o[2 * j2], pl[0], pl[1], pl[2], pl[3], vb[j2][0], vb[j2][1]);
-        mma_bf16_16816(st.o[2 * j2 + 1], pl[0], pl[1], pl[2], pl[3], vb[j2][2], vb[j2][3]);
-      }
-    }
-  }
 }
 
 // Shared-memory layout of the kernel (offsets from the 1024-aligned base).
@@ -296,7 +115,6 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
 
   const int seg0 = wk.cta_seg[blockIdx.x], seg1 = wk.cta_seg[blockIdx.x + 1];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int gid = lane >> 2, tig = lane & 3;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -388,57 +206,19 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
         __syncwarp();
         if (lane == 0) mbar_arrive(&empty[slot]);
       }
-      if (cand >= 0 && ok) {
-        if (!TWO_ROWS) {   // fold the lo-part rows onto their heads
-#pragma unroll
-          for (int n = 0; n < HD / 8; ++n) {
-            st.o[n][0] += st.o[n][2];
-            st.o[n][1] += st.o[n][3];
-          }
-        }
-#pragma unroll
-        for (int r = 0; r < 2; ++r) {   // quad-reduce the row sums
-          st.l[r] += __shfl_xor_sync(0xffffffffu, st.l[r], 1);
-          st.l[r] += __shfl_xor_sync(0xffffffffu, st.l[r], 2);
-        }
-      }
+      if (cand >= 0 && ok) finish_state<HD, TWO_ROWS>(st);
       if (!shared && !TWO_ROWS) {
         // hand the warp's state to the merger warp (one slot per private
         // segment); wait only until it has read the previous segment's states
         if (n_priv > 0) ok = __all_sync(0xffffffffu, mbar_wait(seg_free, (n_priv - 1) & 1u, err)) && ok;
-        if (cand >= 0 && ok) {
-          if (gid < group) {
-#pragma unroll
-            for (int n = 0; n < HD / 8; ++n)
-              *reinterpret_cast<float2*>(mo + (warp * 8 + gid) * HD + n * 8 + tig * 2) =
-                  make_float2(st.o[n][0], st.o[n][1]);
-            if (tig == 0) {
-              mm[warp * 8 + gid] = st.m[0];
-              ml[warp * 8 + gid] = st.l[0];
-            }
-          }
-        } else if (lane < 8) {
-          mm[warp * 8 + lane] = -INFINITY;   // nothing scored by this warp
-          ml[warp * 8 + lane] = 0.f;
-        }
+        stash_state<HD>(st, cand >= 0 && ok, warp, group, lane, mo, mm, ml);
         __syncwarp();
         if (lane == 0) mbar_arrive(seg_full);
         ++n_priv;
       } else if (cand >= 0 && ok) {
         // this warp's own partial slot
         const int slot_id = shared ? wk.slots[sg.slot + warp] : sg.slot + warp;
-#pragma unroll
-        for (int r = 0; r < (TWO_ROWS ? 2 : 1); ++r) {
-          const int row = gid + 8 * r;
-          if (row < group) {
-            const int64_t pr = static_cast<int64_t>(slot_id) * group + row;
-            float* dst = part_o + pr * HD;
-#pragma unroll
-            for (int n = 0; n < HD / 8; ++n)
-              *reinterpret_cast<float2*>(dst + n * 8 + tig * 2) = make_float2(st.o[n][2 * r], st.o[n][2 * r + 1]);
-            if (tig == 0) *reinterpret_cast<float2*>(part_ml + pr * 2) = make_float2(st.m[r], st.l[r]);
-          }
-        }
+        store_state_slot<HD, TWO_ROWS>(st, slot_id, group, lane, part_o, part_ml);
       }
     }
   } else if (warp == kMergerWarp && !TWO_ROWS) {
@@ -446,38 +226,13 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
     // For every private segment, in order: fold the eight consumer warps'
     // (m, l, O) into the segment's partial slot,
     //   M = max_w m_w, L = sum_w 2^(m_w - M) l_w, O = sum_w 2^(m_w - M) O_w.
-    constexpr int kPer = HD / 32;
     uint32_t k = 0;
     bool ok = true;
     for (int si = seg0; si < seg1; ++si) {
       const AttnSeg sg = wk.segs[si];
       if (sg.kind != 0) continue;
       if (ok) ok = __all_sync(0xffffffffu, mbar_wait(seg_full, k & 1u, err));
-      if (ok) {
-        for (int r = 0; r < group; ++r) {
-          float mw[kConsumerWarps], M = -INFINITY;
-#pragma unroll
-          for (int w = 0; w < kConsumerWarps; ++w) {
-            mw[w] = mm[w * 8 + r];
-            M = fmaxf(M, mw[w]);
-          }
-          float acc[kPer], L = 0.f;
-#pragma unroll
-          for (int j = 0; j < kPer; ++j) acc[j] = 0.f;
-#pragma unroll
-          for (int w = 0; w < kConsumerWarps; ++w) {
-            if (mw[w] == -INFINITY) continue;   // an idle warp: its O rows are not written
-            const float f = exp2f(mw[w] - M);
-            L += f * ml[w * 8 + r];
-#pragma unroll
-            for (int j = 0; j < kPer; ++j) acc[j] += f * mo[(w * 8 + r) * HD + lane + 32 * j];
-          }
-          const int64_t pr = static_cast<int64_t>(sg.slot) * group + r;
-#pragma unroll
-          for (int j = 0; j < kPer; ++j) part_o[pr * HD + lane + 32 * j] = acc[j];
-          if (lane == 0) *reinterpret_cast<float2*>(part_ml + pr * 2) = make_float2(M, L);
-        }
-      }
+      if (ok) merge_warp_states<HD>(group, mo, mm, ml, sg.slot, lane, part_o, part_ml);
       __syncwarp();
       if (lane == 0) mbar_arrive(seg_free);
       ++k;
@@ -486,167 +241,19 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
   trace_end(ts);
 }
 
-// The combine: one CTA per (candidate, kv head), W warps.  Warp w folds slots
-// w, w + W, ... (U at a time, every load of those issued before the first
-// use) into a running (M, L, O) per query head of the group; the warps' states
-// and the verify token's own entry are then merged through shared memory:
-//   M* = max(s_self, M_w), o = (2^(s_self - M*) v_self + sum_w 2^(M_w - M*) O_w)
-//                              / (2^(s_self - M*) + sum_w 2^(M_w - M*) L_w).
-// W and U keep the per-thread state within the register budget of W warps.
-template <int HD, int ROWS>
-struct CombineShape {
-  static constexpr int W = 8;                               // warps
-  static constexpr int U = HD * ROWS <= 512 ? 2 : 1;        // slots in flight per warp
-  static constexpr size_t kAcc = 0;                                         // [W][ROWS][HD]
-  static constexpr size_t kM = kAcc + sizeof(float) * W * ROWS * HD;        // [W][ROWS]
-  static constexpr size_t kL = kM + sizeof(float) * W * ROWS;               // [W][ROWS]
-  static constexpr size_t kSelf = kL + sizeof(float) * W * ROWS;            // [ROWS]
-  static constexpr size_t kBytes = kSelf + sizeof(float) * ROWS;
-};
-
+// The combine: one CTA per (candidate, kv head) running combine_group.
 template <int HD, int ROWS>
 __global__ void __launch_bounds__(CombineShape<HD, ROWS>::W * 32) attn_combine_kernel(
     const int32_t* __restrict__ slot_base, const int32_t* __restrict__ nslots, int n_q, int n_kv, int group,
     const float* __restrict__ part_o, const float* __restrict__ part_ml, AttnMerge mg, unsigned long long* ts) {
-  using CS = CombineShape<HD, ROWS>;
-  constexpr int kPer = HD / 32, W = CS::W, U = CS::U;
-  constexpr int kOut = (ROWS * HD + W * 32 - 1) / (W * 32);   // outputs per thread in the final phase
   trace_begin(ts);
   grid_dep_launch();
   extern __shared__ __align__(16) uint8_t csm[];
-  float* s_acc = reinterpret_cast<float*>(csm + CS::kAcc);
-  float* s_m = reinterpret_cast<float*>(csm + CS::kM);
-  float* s_l = reinterpret_cast<float*>(csm + CS::kL);
-  float* s_self = reinterpret_cast<float*>(csm + CS::kSelf);
   const int cg = blockIdx.x, b = cg / n_kv, g = cg - b * n_kv;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int64_t hq0 = static_cast<int64_t>(b) * n_q + static_cast<int64_t>(g) * group;
-  const int64_t hk = static_cast<int64_t>(b) * n_kv + g;
   const int first = slot_base[cg], ns = nslots[cg];   // host-uploaded before the call: no wait needed
-
   grid_dep_wait();   // the partials (and q, k_self, v_self) are written by earlier kernels
-  // Every global load of the first round is issued before any is used: this
-  // warp's first U slots, the q / k_self rows of head `warp` and this thread's
-  // v_self values for the final phase.
-  float2 ml[U];
-  float v[U][ROWS][kPer];
-#pragma unroll
-  for (int k = 0; k < U; ++k) {
-    const int sk = warp + k * W;
-    const int64_t pr = (static_cast<int64_t>(first) + (sk < ns ? sk : 0)) * group;
-    ml[k] = (sk < ns && lane < group) ? __ldcg(reinterpret_cast<const float2*>(part_ml + (pr + lane) * 2))
-                                      : make_float2(-INFINITY, 0.f);
-#pragma unroll
-    for (int r = 0; r < ROWS; ++r)
-#pragma unroll
-      for (int j = 0; j < kPer; ++j)
-        v[k][r][j] = (sk < ns && r < group) ? __ldcg(part_o + (pr + r) * HD + lane + 32 * j) : 0.f;
-  }
-  float qd[kPer], kd[kPer];
-#pragma unroll
-  for (int j = 0; j < kPer; ++j) {
-    qd[j] = warp < group ? mg.q[(hq0 + warp) * HD + lane + 32 * j] : 0.f;
-    kd[j] = warp < group ? mg.kself[hk * HD + lane + 32 * j] : 0.f;
-  }
-  float vsf[kOut];
-#pragma unroll
-  for (int i = 0; i < kOut; ++i) {
-    const int idx = threadIdx.x + i * W * 32;
-    vsf[i] = idx < group * HD ? mg.vself[hk * HD + idx % HD] : 0.f;
-  }
-  // the verify token's own score of head `warp`
-  if (warp < group) {
-    float dot = 0.f;
-#pragma unroll
-    for (int j = 0; j < kPer; ++j) dot += qd[j] * kd[j];
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
-    if (lane == 0) s_self[warp] = dot * (kLog2e * rsqrtf(static_cast<float>(HD)));
-  }
-  for (int r = warp + W; r < group; r += W) {   // heads beyond the warp count (G > W; k_self is loaded by all)
-    float dot = 0.f;
-#pragma unroll
-    for (int j = 0; j < kPer; ++j) dot += mg.q[(hq0 + r) * HD + lane + 32 * j] * kd[j];
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
-    if (lane == 0) s_self[r] = dot * (kLog2e * rsqrtf(static_cast<float>(HD)));
-  }
-  float M[ROWS], L[ROWS], acc[ROWS][kPer];
-#pragma unroll
-  for (int r = 0; r < ROWS; ++r) {
-    M[r] = -INFINITY;
-    L[r] = 0.f;
-#pragma unroll
-    for (int j = 0; j < kPer; ++j) acc[r][j] = 0.f;
-  }
-  for (int s0 = warp;; s0 += U * W) {
-#pragma unroll
-    for (int k = 0; k < U; ++k)
-#pragma unroll
-      for (int r = 0; r < ROWS; ++r) {
-        const float mr = __shfl_sync(0xffffffffu, ml[k].x, r), lr = __shfl_sync(0xffffffffu, ml[k].y, r);
-        if (mr == -INFINITY) continue;   // past the last slot (warp-uniform)
-        const float Mn = fmaxf(M[r], mr);
-        const float sc = exp2f(M[r] - Mn), wv = exp2f(mr - Mn);
-        L[r] = L[r] * sc + wv * lr;
-#pragma unroll
-        for (int j = 0; j < kPer; ++j) acc[r][j] = acc[r][j] * sc + wv * v[k][r][j];
-        M[r] = Mn;
-      }
-    if (s0 + U * W >= ns) break;
-    // the next round of slots (more than U * W slots only)
-#pragma unroll
-    for (int k = 0; k < U; ++k) {
-      const int sk = s0 + U * W + k * W;
-      const int64_t pr = (static_cast<int64_t>(first) + (sk < ns ? sk : 0)) * group;
-      ml[k] = (sk < ns && lane < group) ? __ldcg(reinterpret_cast<const float2*>(part_ml + (pr + lane) * 2))
-                                        : make_float2(-INFINITY, 0.f);
-#pragma unroll
-      for (int r = 0; r < ROWS; ++r)
-#pragma unroll
-        for (int j = 0; j < kPer; ++j)
-          v[k][r][j] = (sk < ns && r < group) ? __ldcg(part_o + (pr + r) * HD + lane + 32 * j) : 0.f;
-    }
-  }
-#pragma unroll
-  for (int r = 0; r < ROWS; ++r) {
-    if (r < group) {
-#pragma unroll
-      for (int j = 0; j < kPer; ++j) s_acc[(warp * ROWS + r) * HD + lane + 32 * j] = acc[r][j];
-      if (lane == 0) {
-        s_m[warp * ROWS + r] = M[r];
-        s_l[warp * ROWS + r] = L[r];
-      }
-    }
-  }
-  __syncthreads();
-#pragma unroll
-  for (int i = 0; i < kOut; ++i) {
-    const int idx = threadIdx.x + i * W * 32;
-    if (idx >= group * HD) break;
-    const int r = idx / HD, d = idx - r * HD;
-    const float ss = s_self[r];
-    float Mt = ss;
-#pragma unroll
-    for (int w = 0; w < W; ++w) Mt = fmaxf(Mt, s_m[w * ROWS + r]);
-    const float ws = exp2f(ss - Mt);
-    float num = ws * vsf[i], den = ws;
-#pragma unroll
-    for (int w = 0; w < W; ++w) {
-      const float mw = s_m[w * ROWS + r];
-      if (mw == -INFINITY) continue;
-      const float f = exp2f(mw - Mt);
-      num += f * s_acc[(w * ROWS + r) * HD + d];
-      den += f * s_l[w * ROWS + r];
-    }
-    const float out = num / den;
-    const int64_t o = (hq0 + r) * HD + d;
-    const __nv_bfloat16 hi = __float2bfloat16_rn(out);
-    mg.o_hi[o] = hi;
-    mg.o_lo[o] = __float2bfloat16_rn(out - __bfloat162float(hi));
-    if (mg.out_f32) mg.out_f32[o] = out;
-    if (mg.dbg) mg.dbg[o] = out;
-  }
+  combine_group<HD, ROWS>(threadIdx.x, b, g, first, ns, n_q, n_kv, group, part_o, part_ml, mg, csm,
+                          [] { __syncthreads(); });
   trace_end(ts);
 }
 

@@ -1,8 +1,9 @@
 // Inline-PTX building blocks for sm_103a: shared-memory mbarriers, TMA tiled
 // bulk copies, tcgen05 tensor-core MMA with TMEM accumulators, and bounded
 // waits.  Every wait in this library is bounded: after kWaitTimeoutNs of
-// global time it records KVPRM_DEV_TIMEOUT in a device error word and gives
-// up, so a lost arrival can never hang the GPU.
+// global time it records a nonzero code (the wait site, where the caller names
+// one) in a device error word and gives up, so a lost arrival can never hang
+// the GPU.
 #pragma once
 
 #include <cuda.h>
@@ -64,7 +65,7 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 // Wait until the phase with the given parity has completed.  Returns false
 // (after flagging *err) if that takes longer than kWaitTimeoutNs, or at once
 // if another thread already flagged an error.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err) {
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err, int site = kDevTimeout) {
   const uint32_t a = smem_u32(bar);
   if (mbar_try_wait(a, parity)) return true;
   const uint64_t t0 = global_timer_ns();
@@ -74,7 +75,7 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* e
       if (mbar_try_wait(a, parity)) return true;
     if (*(volatile int*)err != 0) return false;
     if (global_timer_ns() - t0 > kWaitTimeoutNs) {
-      atomicExch(err, kDevTimeout);
+      atomicCAS(err, 0, site);
       return false;
     }
   }
@@ -162,6 +163,69 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Each thread of a warp reads 8 consecutive fp32 columns of its own TMEM lane.
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, float (&v)[8]) {
+  uint32_t r[8];
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+               : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// ---------------------------------------------------------------- inter-CTA flags (persistent kernels)
+__device__ __forceinline__ int ld_acquire_gpu(const int* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+// Order this thread's generic-proxy global accesses with later async-proxy
+// (TMA) accesses: data written by ordinary stores and read by TMA.
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+// Wait until *cnt >= target (acquire).  Bounded like mbar_wait: false after
+// kWaitTimeoutNs (flagging *err), or at once when *err is already set.
+__device__ __forceinline__ bool wait_counter(const int* cnt, int target, int* err, int site = kDevTimeout) {
+  if (ld_acquire_gpu(cnt) >= target) return true;
+  const uint64_t t0 = global_timer_ns();
+  for (;;) {
+#pragma unroll 1
+    for (int i = 0; i < 16; ++i)
+      if (ld_acquire_gpu(cnt) >= target) return true;
+    if (*(volatile int*)err != 0) return false;
+    if (global_timer_ns() - t0 > kWaitTimeoutNs) {
+      atomicCAS(err, 0, site);
+      return false;
+    }
+  }
+}
+
+// ---------------------------------------------------------------- cp.async (LSU path, L2 only)
+__device__ __forceinline__ void cp_async16_cg(uint32_t dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+// Wait until at most n (0..7) committed groups of this thread are pending.
+__device__ __forceinline__ void cp_async_wait_pending(int n) {
+  switch (n) {
+    case 0: asm volatile("cp.async.wait_group 0;" ::: "memory"); break;
+    case 1: asm volatile("cp.async.wait_group 1;" ::: "memory"); break;
+    case 2: asm volatile("cp.async.wait_group 2;" ::: "memory"); break;
+    case 3: asm volatile("cp.async.wait_group 3;" ::: "memory"); break;
+    case 4: asm volatile("cp.async.wait_group 4;" ::: "memory"); break;
+    case 5: asm volatile("cp.async.wait_group 5;" ::: "memory"); break;
+    case 6: asm volatile("cp.async.wait_group 6;" ::: "memory"); break;
+    default: asm volatile("cp.async.wait_group 7;" ::: "memory"); break;
+  }
+}
+// Make this thread's completed generic-proxy shared-memory writes visible to
+// the async proxy (tcgen05.mma operand reads).
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
 // Shared-memory matrix descriptor (tcgen05 "matrix descriptor") for a K-major
