@@ -202,17 +202,7 @@ KVPRM_API int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, con
  * the last call's stream).  Bit 1: keep every layer's rotated q, self k and
  * self v (float); bit 2: keep the residual stream after every layer (float).
  * kvprm_debug_layers copies them: which = 1 q [N_L][n][n_q*hd], 2 k_self
- * [N_L][n][n_kv*hd], 3 v_self (same), 4 h [N_L][n][d_model].  Bit 3: event
- * timeline of the persistent forward kernel; which = 5 copies uint64
- * [n_SM][N_L][32] per CTA and layer.  Entries 0..15 are global-timer stamps
- * (ns): for projection k (0 QKV, 1 O, 2 gate/up, 3 down) entry 3k its
- * activations became ready, 3k + 1 its last MMA was issued, 3k + 2 its drains
- * and epilogues ended; 12 the query became ready, 13 attention ended, 14 the
- * combine could start, 15 the combine ended (0 where the CTA had no such
- * work).  Entries 16..31 are durations (ns) summed over the step: 16 + k the
- * MMA issuer's waits for weight tiles of projection k, 20 + k its waits for
- * activation tiles, 24 + k the release fences after the partial-sum
- * reductions, 28 + k the tile-arrival atomics. */
+ * [N_L][n][n_kv*hd], 3 v_self (same), 4 h [N_L][n][d_model]. */
 KVPRM_API int kvprm_set_debug(kvprm_ctx* ctx, int flags);
 KVPRM_API int kvprm_debug_attn_out(kvprm_ctx* ctx, float* d_out);
 KVPRM_API int kvprm_debug_layers(kvprm_ctx* ctx, int which, void* d_out);
@@ -272,9 +262,7 @@ KVPRM_API int kvprm_check_device(kvprm_ctx* ctx);
  * the scoring stream while enabled (one event pair per launch; programmatic
  * launch overlap is switched off meanwhile, so each launch is timed alone).
  * Classes: 0..3 the QKV, O, gate/up and down projections, 4 paged attention
- * (split-K), 5 attention combine, 6 the small RoPE-table / embedding / head
- * kernels, 7 the persistent all-layer forward kernel (the default schedule, in
- * which classes 0..5 do not occur: those steps run inside it).
+ * (split-K), 5 attention combine, 6 fused norm / RoPE / SiLU / head kernels.
  * Profiled calls synchronise the stream.  kvprm_get_profile returns per class
  * the launch count and total milliseconds since profiling was enabled. */
 enum {
@@ -285,8 +273,7 @@ enum {
   KVPRM_PROF_ATTN = 4,
   KVPRM_PROF_COMBINE = 5,
   KVPRM_PROF_FUSED = 6,
-  KVPRM_PROF_FORWARD = 7,
-  KVPRM_PROF_N = 8
+  KVPRM_PROF_N = 7
 };
 KVPRM_API int kvprm_set_profile(kvprm_ctx* ctx, int enable);
 
@@ -298,16 +285,18 @@ KVPRM_API int kvprm_set_profile(kvprm_ctx* ctx, int enable);
  * number of records written, or a negative KVPRM_E* code. */
 KVPRM_API int kvprm_set_trace(kvprm_ctx* ctx, int enable);
 KVPRM_API int kvprm_get_trace(kvprm_ctx* ctx, int32_t max_records, int32_t* cls, double* start_us, double* end_us);
+/* As kvprm_get_trace, plus the critical path inside each projection launch:
+ * events_us [max_records][8] (may be NULL) holds, per launch, the time at
+ * which the LAST CTA passed each milestone -- 0 the preceding kernel had
+ * completed (programmatic-launch wait returned), 1 the first weight and
+ * activation tiles landed, 2 all MMAs completed, 3 the accumulators were
+ * parked in shared memory cluster-wide, 4 the split-K reduction over the
+ * cluster was done, 5 the RMSNorm factors were ready, 6 the epilogue was
+ * written, 7 the cluster released -- or -1 where a launch has no such
+ * milestone (attention, combine and the small kernels record none). */
+KVPRM_API int kvprm_get_trace_events(kvprm_ctx* ctx, int32_t max_records, int32_t* cls, double* start_us,
+                                     double* end_us, double* events_us);
 KVPRM_API int kvprm_get_profile(kvprm_ctx* ctx, int64_t* launches, double* total_ms);
-
-/* Step timeline inside the persistent forward kernel of the last traced call
- * (kvprm_set_trace on): for layer l and step s (0 QKV projection, 1 attention,
- * 2 combine, 3 O projection, 4 gate/up projection, 5 down projection),
- * end_us[6 l + s] is the time, in microseconds after the kernel's first CTA
- * started, at which the last CTA finished its share of that step.  Returns the
- * number of values written (0 when the call did not run the persistent
- * kernel), or a negative KVPRM_E* code.  Synchronises the last call's stream. */
-KVPRM_API int kvprm_get_phase_trace(kvprm_ctx* ctx, int32_t max_records, double* end_us);
 
 #ifdef __cplusplus
 }

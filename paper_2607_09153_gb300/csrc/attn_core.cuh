@@ -1,7 +1,6 @@
 // Warp-level building blocks of the paged decode attention (App. A.3 read-out,
-// head = softmax(q^T K / sqrt(d_k)) V for the verify token's query), shared by
-// the stand-alone attention kernels (attention.cu) and the persistent forward
-// kernel (forward.cu):
+// head = softmax(q^T K / sqrt(d_k)) V for the verify token's query), used by
+// the attention kernels (attention.cu):
 //  - WarpQ / load_q: one warp's query rows as mma.m16n8k16 A fragments, hi and
 //    lo bf16 parts of the fp32 query (packed into the two 8-row halves of one
 //    MMA when the group has <= 8 heads, two MMAs otherwise);
@@ -36,8 +35,7 @@ __device__ __forceinline__ void load_q(WarpQ<HD>& q, const __nv_bfloat16* __rest
                                        const __nv_bfloat16* __restrict__ ql, int group, int lane) {
   const int gid = lane >> 2, tig = lane & 3;
   auto ldq = [&](const __nv_bfloat16* base, int row, int col) -> uint32_t {
-    // L2 load: in the persistent kernel the query is rewritten by other CTAs every layer
-    return row < group ? __ldcg(reinterpret_cast<const unsigned int*>(base + row * HD + col)) : 0u;
+    return row < group ? *reinterpret_cast<const uint32_t*>(base + row * HD + col) : 0u;
   };
 #pragma unroll
   for (int ks = 0; ks < HD / 16; ++ks) {

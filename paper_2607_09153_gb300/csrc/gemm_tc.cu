@@ -7,9 +7,12 @@
 // producer thread streams W and X tiles with TMA (128-byte swizzle) through a
 // multi-stage mbarrier ring; one thread issues tcgen05.mma (kind::f16, bf16 x
 // bf16 -> fp32) into a TMEM accumulator.  The activation X arrives as a bf16
-// (hi, lo) pair, X = hi + lo to ~2^-17 relative, and each K step issues two
-// MMAs (W*hi, W*lo) into the same accumulator, so the contraction sees the
-// fp32 activation (the weights are bf16 by definition).
+// (hi, lo) pair, X = hi + lo to ~2^-17 relative, so the contraction sees the
+// fp32 activation (the weights are bf16 by definition).  The hi and lo tiles
+// sit back to back in shared memory and one MMA of N = 2 n_pad covers both
+// (each weight K slice is read from shared memory once -- the MMA issue rate
+// is bounded by those reads at this small N); the two accumulator halves are
+// added when TMEM is read.  Beyond N = 256 each half takes its own MMA.
 //
 // K is split across the CTAs of a thread-block cluster (one cluster per
 // 128-row tile) so that every SM streams weights.  The splits are reduced
@@ -143,6 +146,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       load_w(smem + i * stage_bytes, kt0 + i, &full[i]);
     }
     grid_dep_wait();
+    trace_event(ts, 0);   // the preceding kernel has completed
     for (int i = 0; i < pre; ++i) {
       tma_load_2d(smem + i * stage_bytes + kWTileBytes, &tmX, &full[i], (kt0 + i) * kBK, 0, pol_x);
       if (has_lo)
@@ -160,11 +164,18 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     }
   } else if (warp == 1 && lane == 0 && nk > 0) {
     // ---------------- MMA issuer
-    const uint32_t idesc = idesc_bf16_f32(kBM, n_pad);
+    // With the hi and lo activation tiles stored back to back (2 n_pad rows
+    // under the same swizzle), one MMA of N = 2 n_pad reads each weight K
+    // slice from shared memory once: columns [0, n_pad) accumulate W hi,
+    // [n_pad, 2 n_pad) accumulate W lo, summed when the accumulator is read.
+    // Beyond N = 256 the two halves take one MMA each into the same columns.
+    const bool merged = has_lo && 2 * n_pad <= 256;
+    const uint32_t idesc = idesc_bf16_f32(kBM, merged ? 2 * n_pad : n_pad);
     for (int i = 0; i < nk; ++i) {
       const int s = i % stages;
       const uint32_t use = static_cast<uint32_t>(i / stages);
       if (!mbar_wait(&full[s], use & 1u, err)) break;
+      if (i == 0) trace_event(ts, 1);   // first weight and activation tiles landed
       tc_fence_after();
       const uint32_t a_base = smem_u32(smem + s * stage_bytes);
       const uint32_t b_base = a_base + kWTileBytes;
@@ -172,7 +183,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       for (int kk = 0; kk < kBK / 16; ++kk) {
         const uint64_t a_desc = desc_sw128(a_base + kk * 32);
         umma_bf16(tmem, a_desc, desc_sw128(b_base + kk * 32), idesc, (i > 0 || kk > 0) ? 1u : 0u);
-        if (has_lo) umma_bf16(tmem, a_desc, desc_sw128(b_base + x_bytes + kk * 32), idesc, 1u);
+        if (has_lo && !merged) umma_bf16(tmem, a_desc, desc_sw128(b_base + x_bytes + kk * 32), idesc, 1u);
       }
       umma_commit(&empty[s]);
     }
@@ -182,13 +193,22 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
 
   // ---------------- accumulator -> own shared memory, acc[c][m] (fp32, c < n_pad, m < 128)
   const bool have = nk > 0 ? __all_sync(0xffffffffu, mbar_wait(done, 0, err)) : true;
+  if (threadIdx.x == 0) trace_event(ts, 2);   // all MMAs of this CTA completed
   tc_fence_after();
   float* acc = reinterpret_cast<float*>(smem);   // the ring is idle once `done` has fired
   const int m = warp * 32 + lane;
+  const bool merged = has_lo && 2 * n_pad <= 256;
   for (int c0 = 0; c0 < n_pad; c0 += 16) {
     float v[16];
     if (nk > 0 && have) {
-      tmem_ld16(tmem + (static_cast<uint32_t>(warp * 32) << 16) + static_cast<uint32_t>(c0), v);
+      const uint32_t t = tmem + (static_cast<uint32_t>(warp * 32) << 16) + static_cast<uint32_t>(c0);
+      tmem_ld16(t, v);
+      if (merged) {
+        float w[16];
+        tmem_ld16(t + static_cast<uint32_t>(n_pad), w);
+#pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] += w[j];
+      }
     } else {
 #pragma unroll
       for (int j = 0; j < 16; ++j) v[j] = 0.f;
@@ -198,6 +218,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
   }
   tc_fence_before();
   cluster_sync();   // every rank's partial is parked
+  if (threadIdx.x == 0) trace_event(ts, 3);
 
   // ---------------- reduce this rank's candidate columns over the cluster, then the epilogue
   grid_dep_wait();   // outputs may still be read by kernels that precede this one
@@ -238,6 +259,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       }
     }
   }
+  if (threadIdx.x == 0) trace_event(ts, 4);   // this rank's columns are reduced over the cluster
   // the RMSNorm factor of each of this rank's columns (QKV, SILU)
   if (ep.rs_sumsq)
     for (int t0 = threadIdx.x; t0 < nc; t0 += blockDim.x) {   // nc <= 256 columns
@@ -247,6 +269,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       rsc[t0] = 1.0f / sqrtf(ssum / ep.rs_d + ep.rs_eps);
     }
   __syncthreads();
+  if (threadIdx.x == 0) trace_event(ts, 5);
   // Step 2: the epilogue over (row, column) pairs, all threads in parallel
   if (ep.mode == GemmEpilogue::PLAIN) {
     const int gm = m_tile * kBM + m;
@@ -320,7 +343,10 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     }
   }
   (void)nc;
+  __syncthreads();
+  if (threadIdx.x == 0) trace_event(ts, 6);   // epilogue written
   cluster_sync();   // peers have finished reading this CTA's partial
+  if (threadIdx.x == 0) trace_event(ts, 7);
   if (warp == 1) tmem_dealloc(tmem, tmem_cols);
   trace_end(ts);
 }
@@ -355,7 +381,8 @@ GemmPlan plan_gemm(int M, int K, int n_pad, int num_sms, bool has_lo, bool gate_
   if (ring < acc) ring = acc;
   p.smem_bytes = ring + 1024 /*align*/ + kTailBytes;
   uint32_t cols = 32;
-  while (cols < static_cast<uint32_t>(n_pad)) cols <<= 1;
+  const int need = (has_lo && 2 * n_pad <= 256) ? 2 * n_pad : n_pad;   // merged hi/lo accumulator halves
+  while (cols < static_cast<uint32_t>(need)) cols <<= 1;
   p.tmem_cols = cols;
   return p;
 }

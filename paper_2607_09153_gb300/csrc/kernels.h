@@ -11,6 +11,12 @@
 
 namespace kvprm {
 
+// Launch trace record (ptx.cuh: trace_begin / trace_end / trace_event): u64
+// [0] earliest CTA start, [1] ~latest CTA end, [2 + e] ~time the last CTA
+// passed milestone e of the kernel.
+constexpr int kTraceEvents = 8;
+constexpr int kTraceStride = 2 + kTraceEvents;
+
 // ---------------------------------------------------------------- projection GEMM
 struct GemmPlan {
   bool has_lo = true;    // activation given as a bf16 (hi, lo) pair
@@ -149,79 +155,5 @@ cudaError_t launch_head(const ModelDims& m, const float* h, const float* sumsq, 
                         float* rewards, cudaStream_t stream, bool pdl, unsigned long long* ts = nullptr);
 cudaError_t launch_split_hilo(const float* in, int64_t count, HiLo out, cudaStream_t stream);
 
-
-// ---------------------------------------------------------------- persistent forward (forward.cu)
-// The projections are split over the persistent CTAs "stream-K" style: the
-// (128-row tile, 64-wide K tile) units of one projection are laid out tile by
-// tile and cut into one equal range per CTA; the part of a range inside one
-// tile is a piece, whose fp32 partial product is added into the tile's
-// accumulator in global memory; the last piece of a tile to arrive applies the
-// step's epilogue.
-enum FwdKind : int { FWD_QKV = 0, FWD_O = 1, FWD_GU = 2, FWD_DOWN = 3, FWD_KINDS = 4 };
-struct FwdPiece {
-  int32_t tile, kt0, kt1, pad;
-};
-struct FwdGemmHost {
-  int tiles = 0, ktiles = 0;
-  int resident = 0;                  // 1: every CTA's pieces lie in one K range that is loaded once per step
-  std::vector<FwdPiece> pieces;      // CTA by CTA
-  std::vector<int32_t> cta_piece;    // [P + 1] first piece of each CTA
-  std::vector<int32_t> tile_np;      // [tiles] pieces of each tile
-};
-// resident_kt = 0: plain stream-K over all (tile, K tile) units.  resident_kt
-// > 0: the K axis is cut into groups of at most resident_kt K tiles, each group
-// gets CTAs in proportion to its width and its units are cut stream-K among
-// them, so a CTA's activation slice is one group's K range.  Returns false if
-// some group would get no CTA.
-bool split_gemm(int tiles, int ktiles, int n_ctas, int resident_kt, FwdGemmHost& g);
-struct FwdGemmDev {
-  const FwdPiece* pieces;
-  const int32_t* cta_piece;
-  const int32_t* tile_np;
-  int tiles, ktiles, resident;
-};
-// Tensor maps passed as kernel parameters: activations (bf16 hi / lo pairs
-// [n_pad][K], box {64, n_pad}) and the KV pool (see encode_pool_map).
-struct FwdMaps {
-  CUtensorMap xhi, xlo, ohi, olo, ahi, alo, pool;
-};
-struct FwdArgs {
-  int n_layers, d, n_q, n_kv, hd, group, ff, n, n_pad, d_tiles;
-  float eps;
-  int64_t layer_pages;
-  // shared-memory plan (see plan_forward)
-  int ring_slots, x_stages;
-  uint32_t x_bytes, tmem_cols;
-  uint32_t aux_off, misc_off;
-  const CUtensorMap* wmaps;   // device [n_layers][FWD_KINDS] weight maps (box {64, 128}; gate/up {64, 64})
-  FwdGemmDev gemm[FWD_KINDS];
-  AttnWork wk;
-  const __nv_bfloat16* const* attn_norm;   // device [n_layers] gain pointers
-  const __nv_bfloat16* const* mlp_norm;
-  float* h;
-  float* sumsq;   // [d_tiles][n]
-  __nv_bfloat16 *x_hi, *x_lo, *o_hi, *o_lo, *a_hi, *a_lo, *q_hi, *q_lo;
-  float *q, *kself, *vself;
-  const float2* rope;
-  float* acc;              // tile accumulators [tiles][128][n_pad], zero between steps
-  unsigned long long* probe;   // optional per-CTA event timeline [grid][n_layers][16]
-  float *apart_o, *apart_ml;
-  int* counters;           // zeroed per call: per-tile arrivals of each kind, then done[4], attn_done, comb_done
-  int tile_cnt_off[FWD_KINDS];
-  int done_off, attn_done_off, comb_done_off;
-  int* err;
-  float *dbg_attn, *dbg_q, *dbg_k, *dbg_v, *dbg_h;   // optional per-layer captures
-  unsigned long long* phase_ts;   // optional: [0] earliest CTA start, [1 + 6 l + phase] latest CTA end
-};
-struct FwdPlan {
-  int ring_slots = 0, x_stages = 0;
-  int resident_kt = 0;   // > 0: activation slices of up to this many K tiles are loaded once per step
-  uint32_t x_bytes = 0, tmem_cols = 0, aux_off = 0, misc_off = 0;
-  size_t smem_bytes = 0;
-};
-bool plan_forward(int hd, int group, int n_pad, FwdPlan& p);
-cudaError_t forward_configure();
-cudaError_t launch_forward(const FwdMaps& maps, const FwdArgs& a, int grid, cudaStream_t stream, bool cooperative,
-                           unsigned long long* ts = nullptr);
 
 }  // namespace kvprm

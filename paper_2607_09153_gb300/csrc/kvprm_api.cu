@@ -7,7 +7,6 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
-#include <algorithm>
 #include <cstdarg>
 #include <cstdio>
 #include <cstdlib>
@@ -112,24 +111,6 @@ struct kvprm_ctx {
   unsigned long long* trace_d = nullptr;
   int trace_cap = 0, trace_n = 0;
   std::vector<int> trace_cls;
-  // persistent forward (forward.cu): the projections' splits over the CTAs,
-  // their device copies, the GEMM partials and the step counters
-  bool fused = true;
-  bool coop = true;
-  kvprm::FwdGemmHost fwd_split[kvprm::FWD_KINDS];
-  int32_t* fwd_tables_d = nullptr;
-  size_t fwd_off[kvprm::FWD_KINDS][3] = {};   // ints: pieces, cta_piece, tile_np
-  size_t fwd_tables_cap = 0;
-  int fwd_split_npad = -1;                     // n_pad the splits were built for
-  float* fwd_part = nullptr;                   // tile accumulators [max tiles][128][n_pad]
-  int fwd_max_tiles = 0;
-  unsigned long long* fwd_probe = nullptr;     // per-CTA event timeline (debug flag 8)
-  int* fwd_counters = nullptr;
-  int fwd_tile_cnt_off[kvprm::FWD_KINDS] = {};
-  int fwd_done_off = 0, fwd_n_counters = 0;
-  CUtensorMap* wmaps_d = nullptr;              // [NL][FWD_KINDS]
-  const bf16** norms_d = nullptr;              // attn_norm[NL], then mlp_norm[NL]
-  unsigned long long* phase_d = nullptr;       // phase timeline of the last traced call
   // profiling
   bool profile = false;
   std::vector<ProfMark> live_marks;   // marks recorded in the current (non-graph) capture
@@ -221,13 +202,6 @@ void free_ctx(kvprm_ctx* c) {
   cudaFree(c->dbg_h);
   cudaFree(c->dummy_pool);
   cudaFree(c->dev_pool);
-  cudaFree(c->fwd_tables_d);
-  cudaFree(c->fwd_part);
-  cudaFree(c->fwd_probe);
-  cudaFree(c->fwd_counters);
-  cudaFree(c->wmaps_d);
-  cudaFree(c->norms_d);
-  cudaFree(c->phase_d);
   if (c->staging) cudaFreeHost(c->staging);
   if (c->h_rewards) cudaFreeHost(c->h_rewards);
   if (c->h_err) cudaFreeHost(c->h_err);
@@ -409,7 +383,7 @@ struct Enq {
   unsigned long long* trace_slot(int cls) {
     if (!ctx->trace || ctx->trace_n >= ctx->trace_cap) return nullptr;
     ctx->trace_cls.push_back(cls);
-    return ctx->trace_d + 2 * static_cast<size_t>(ctx->trace_n++);
+    return ctx->trace_d + kvprm::kTraceStride * static_cast<size_t>(ctx->trace_n++);
   }
   int end(cudaEvent_t ev_b) {
     if (!prof) return KVPRM_OK;
@@ -479,7 +453,8 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
   ctx->trace_n = 0;
   ctx->trace_cls.clear();
   if (ctx->trace)
-    CK(cudaMemsetAsync(ctx->trace_d, 0xFF, sizeof(unsigned long long) * 2 * ctx->trace_cap, st), "trace reset");
+    CK(cudaMemsetAsync(ctx->trace_d, 0xFF, sizeof(unsigned long long) * kvprm::kTraceStride * ctx->trace_cap, st),
+       "trace reset");
   LAUNCH(KVPRM_PROF_FUSED, kvprm::launch_rope_table(sl, n, m.hd, ctx->cfg.rope_base, ctx->rope, st, false, TS), "rope");
   LAUNCH(KVPRM_PROF_FUSED,
          kvprm::launch_embed_norm(m, ctx->embed, ctx->attn_norm[0], n, ctx->h, ctx->sumsq, X, st, pdl, TS),
@@ -531,116 +506,6 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
   return KVPRM_OK;
 }
 
-// The persistent schedule: RoPE table and verify-token embedding, ONE kernel
-// for every layer (forward.cu), then the reward head.
-int enqueue_fused(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
-  const ModelDims& m = ctx->md;
-  const int n = P.n, NL = ctx->cfg.n_layers;
-  cudaStream_t st = E.st;
-  const bool pdl = E.pdl;
-  const kvprm::HiLo X{ctx->xhi, ctx->xlo};
-  ctx->trace_n = 0;
-  ctx->trace_cls.clear();
-  if (ctx->trace) {
-    CK(cudaMemsetAsync(ctx->trace_d, 0xFF, sizeof(unsigned long long) * 2 * ctx->trace_cap, st), "trace reset");
-    CK(cudaMemsetAsync(ctx->phase_d, 0, sizeof(unsigned long long) * (1 + 6 * static_cast<size_t>(NL)), st),
-       "phase trace reset");
-    CK(cudaMemsetAsync(ctx->phase_d, 0xFF, sizeof(unsigned long long), st), "phase trace reset");
-  }
-  CK(cudaMemsetAsync(ctx->fwd_counters, 0, sizeof(int) * ctx->fwd_n_counters, st), "step counters reset");
-  if (ctx->debug_flags & 8)
-    CK(cudaMemsetAsync(ctx->fwd_probe, 0, sizeof(unsigned long long) * ctx->num_sms * NL * 48, st), "probe reset");
-  CK(cudaMemsetAsync(ctx->fwd_part, 0, sizeof(float) * ctx->fwd_max_tiles * 128 * P.n_pad, st),
-     "tile accumulators reset");
-  LAUNCH(KVPRM_PROF_FUSED, kvprm::launch_rope_table(ctx->tables_d, n, m.hd, ctx->cfg.rope_base, ctx->rope, st, false, TS),
-         "rope");
-  LAUNCH(KVPRM_PROF_FUSED,
-         kvprm::launch_embed_norm(m, ctx->embed, ctx->attn_norm[0], n, ctx->h, ctx->sumsq, X, st, pdl, TS),
-         "embed_norm");
-  kvprm::FwdMaps maps;
-  maps.xhi = ctx->tm_xhi;
-  maps.xlo = ctx->tm_xlo;
-  maps.ohi = ctx->tm_ohi;
-  maps.olo = ctx->tm_olo;
-  maps.ahi = ctx->tm_ahi;
-  maps.alo = ctx->tm_alo;
-  maps.pool = ctx->tm_pool;
-  kvprm::FwdArgs a{};
-  a.n_layers = NL;
-  a.d = m.d;
-  a.n_q = m.n_q;
-  a.n_kv = m.n_kv;
-  a.hd = m.hd;
-  a.group = m.n_q / m.n_kv;
-  a.ff = m.ff;
-  a.n = n;
-  a.n_pad = P.n_pad;
-  a.d_tiles = ctx->d_tiles;
-  a.eps = m.eps;
-  a.layer_pages = ctx->as.layer_pages;
-  kvprm::FwdPlan fp;
-  if (!kvprm::plan_forward(m.hd, a.group, P.n_pad, fp))
-    return fail(ctx, KVPRM_EUNSUPPORTED, "no shared-memory plan for the persistent forward at n_pad = %d", P.n_pad);
-  a.ring_slots = fp.ring_slots;
-  a.x_stages = fp.x_stages;
-  a.x_bytes = fp.x_bytes;
-  a.tmem_cols = fp.tmem_cols;
-  a.aux_off = fp.aux_off;
-  a.misc_off = fp.misc_off;
-  a.wmaps = ctx->wmaps_d;
-  for (int k = 0; k < kvprm::FWD_KINDS; ++k) {
-    a.gemm[k].pieces = reinterpret_cast<const kvprm::FwdPiece*>(ctx->fwd_tables_d + ctx->fwd_off[k][0]);
-    a.gemm[k].cta_piece = ctx->fwd_tables_d + ctx->fwd_off[k][1];
-    a.gemm[k].tile_np = ctx->fwd_tables_d + ctx->fwd_off[k][2];
-    a.gemm[k].tiles = ctx->fwd_split[k].tiles;
-    a.gemm[k].ktiles = ctx->fwd_split[k].ktiles;
-    a.gemm[k].resident = ctx->fwd_split[k].resident;
-    a.tile_cnt_off[k] = ctx->fwd_tile_cnt_off[k];
-  }
-  a.wk = device_work(ctx);
-  a.attn_norm = ctx->norms_d;
-  a.mlp_norm = ctx->norms_d + NL;
-  a.h = ctx->h;
-  a.sumsq = ctx->sumsq;
-  a.x_hi = ctx->xhi;
-  a.x_lo = ctx->xlo;
-  a.o_hi = ctx->ohi;
-  a.o_lo = ctx->olo;
-  a.a_hi = ctx->ahi;
-  a.a_lo = ctx->alo;
-  a.q_hi = ctx->qhi;
-  a.q_lo = ctx->qlo;
-  a.q = ctx->q;
-  a.kself = ctx->kself;
-  a.vself = ctx->vself;
-  a.rope = ctx->rope;
-  a.acc = ctx->fwd_part;
-  a.probe = (ctx->debug_flags & 8) ? ctx->fwd_probe : nullptr;
-  a.apart_o = ctx->apart_o;
-  a.apart_ml = ctx->apart_ml;
-  a.counters = ctx->fwd_counters;
-  a.done_off = ctx->fwd_done_off;
-  a.attn_done_off = ctx->fwd_done_off + kvprm::FWD_KINDS;
-  a.comb_done_off = a.attn_done_off + 1;
-  a.err = ctx->err_d;
-  a.dbg_attn = (ctx->debug_flags & 1) ? ctx->dbg : nullptr;
-  a.dbg_q = (ctx->debug_flags & 2) ? ctx->dbg_q : nullptr;
-  a.dbg_k = (ctx->debug_flags & 2) ? ctx->dbg_k : nullptr;
-  a.dbg_v = (ctx->debug_flags & 2) ? ctx->dbg_v : nullptr;
-  a.dbg_h = (ctx->debug_flags & 4) ? ctx->dbg_h : nullptr;
-  a.phase_ts = ctx->trace ? ctx->phase_d : nullptr;
-  LAUNCH(KVPRM_PROF_FORWARD, kvprm::launch_forward(maps, a, ctx->num_sms, st, ctx->coop, TS), "forward");
-  LAUNCH(KVPRM_PROF_FUSED,
-         kvprm::launch_head(m, ctx->h, ctx->sumsq, ctx->d_tiles, n, ctx->final_norm, ctx->w_plus, ctx->w_minus,
-                            ctx->rewards_d, st, false, TS),
-         "reward_head");
-  return KVPRM_OK;
-}
-
-int enqueue_call(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
-  return ctx->fused ? enqueue_fused(ctx, P, E) : enqueue_forward(ctx, P, E);
-}
-
 int accumulate_marks(kvprm_ctx* ctx, std::vector<ProfMark>& marks, bool destroy) {
   for (auto& mk : marks) {
     float ms = 0.f;
@@ -667,8 +532,6 @@ void drop_graph(kvprm_ctx* ctx) {
   ctx->gkey = GraphKey();
 }
 
-int ensure_fwd_split(kvprm_ctx* ctx, int n_pad);
-
 // Score into ctx->rewards_d on stream `st` (stream-ordered).
 int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const int32_t* bt, const int32_t* sl, int32_t n,
                  cudaStream_t st) {
@@ -690,14 +553,13 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   if ((rc = plan_work(ctx, bt, sl, n))) return rc;
   const CallPlan P = make_plan(ctx, n, max_pages);
   if ((rc = ensure_x_maps(ctx, P.n_pad))) return rc;
-  if (ctx->fused && (rc = ensure_fwd_split(ctx, P.n_pad))) return rc;
   if ((rc = upload_tables(ctx, bt, sl, n, st))) return rc;
   ctx->last_n = n;
   ctx->last_stream = st;
 
   if (!ctx->use_graph) {
     Enq E{ctx, st, ctx->use_pdl && !ctx->profile, ctx->profile, &ctx->live_marks};
-    if ((rc = enqueue_call(ctx, P, E))) return rc;
+    if ((rc = enqueue_forward(ctx, P, E))) return rc;
     if (ctx->profile) {
       CK(cudaStreamSynchronize(st), "cudaStreamSynchronize(profile)");
       if ((rc = accumulate_marks(ctx, ctx->live_marks, true))) return rc;
@@ -719,7 +581,7 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
     CK(cudaStreamBeginCapture(ctx->cap_stream, cudaStreamCaptureModeThreadLocal), "cudaStreamBeginCapture");
     Enq E{ctx, ctx->cap_stream, ctx->use_pdl && !ctx->profile, ctx->profile, &ctx->graph_marks};
     E.capturing = true;
-    rc = enqueue_call(ctx, P, E);
+    rc = enqueue_forward(ctx, P, E);
     cudaGraph_t graph = nullptr;
     cudaError_t e = cudaStreamEndCapture(ctx->cap_stream, &graph);
     if (rc) {
@@ -752,7 +614,7 @@ int finish_blocking(kvprm_ctx* ctx, int32_t n, float* rewards, cudaStream_t st) 
   if (*ctx->h_err) {
     const int site = *ctx->h_err;
     cudaMemsetAsync(ctx->err_d, 0, sizeof(int), st);
-    return fail(ctx, KVPRM_ETIMEOUT, "a bounded device wait timed out (wait site %d); results are invalid", site);
+    return fail(ctx, KVPRM_ETIMEOUT, "a bounded device wait timed out (code %d); results are invalid", site);
   }
   std::memcpy(rewards, ctx->h_rewards, sizeof(float) * n);
   return KVPRM_OK;
@@ -762,110 +624,7 @@ bool env_off(const char* name) {
   const char* v = std::getenv(name);
   return v && v[0] == '1';
 }
-bool env_on(const char* name) { return env_off(name); }
 
-}  // namespace
-
-namespace {
-// Persistent-forward tables: the split of every projection over the CTAs, the
-// per-layer weight maps and gain pointers in device memory, the partial buffer
-// and the step counters.
-// The projections' shapes in (128-row tile, 64-wide K tile) units.
-void fwd_shapes(const kvprm_ctx* ctx, int* tiles, int* ktiles) {
-  const ModelDims& m = ctx->md;
-  const int t[kvprm::FWD_KINDS] = {(m.qkv_rows + 127) / 128, (m.d + 127) / 128, m.ff / 64, (m.d + 127) / 128};
-  const int k[kvprm::FWD_KINDS] = {m.d / 64, m.n_q * m.hd / 64, m.d / 64, m.ff / 64};
-  for (int i = 0; i < kvprm::FWD_KINDS; ++i) {
-    tiles[i] = t[i];
-    ktiles[i] = k[i];
-  }
-}
-
-// Split every projection over the CTAs for a padded batch of n_pad (the
-// activation slice budget depends on it) and upload the tables.  Resident
-// slices for every projection, or pipelined activations for every projection:
-// one call never mixes the two.
-int ensure_fwd_split(kvprm_ctx* ctx, int n_pad) {
-  if (ctx->fwd_split_npad == n_pad) return KVPRM_OK;
-  kvprm::FwdPlan fp;
-  if (!kvprm::plan_forward(ctx->md.hd, ctx->md.n_q / ctx->md.n_kv, n_pad, fp))
-    return fail(ctx, KVPRM_EUNSUPPORTED, "no shared-memory plan for the persistent forward at n_pad = %d", n_pad);
-  int tiles[kvprm::FWD_KINDS], ktiles[kvprm::FWD_KINDS];
-  fwd_shapes(ctx, tiles, ktiles);
-  const int P = ctx->num_sms;
-  bool ok = true;
-  for (int k = 0; k < kvprm::FWD_KINDS && ok; ++k)
-    ok = kvprm::split_gemm(tiles[k], ktiles[k], P, fp.resident_kt, ctx->fwd_split[k]);
-  if (!ok)
-    for (int k = 0; k < kvprm::FWD_KINDS; ++k) kvprm::split_gemm(tiles[k], ktiles[k], P, 0, ctx->fwd_split[k]);
-  std::vector<int32_t> tab;
-  for (int k = 0; k < kvprm::FWD_KINDS; ++k) {
-    const kvprm::FwdGemmHost& g = ctx->fwd_split[k];
-    ctx->fwd_off[k][0] = tab.size();
-    for (const kvprm::FwdPiece& pc : g.pieces) tab.insert(tab.end(), {pc.tile, pc.kt0, pc.kt1, pc.pad});
-    ctx->fwd_off[k][1] = tab.size();
-    tab.insert(tab.end(), g.cta_piece.begin(), g.cta_piece.end());
-    ctx->fwd_off[k][2] = tab.size();
-    tab.insert(tab.end(), g.tile_np.begin(), g.tile_np.end());
-    while (tab.size() % 4) tab.push_back(0);   // keep every piece array 16-byte aligned
-  }
-  if (tab.size() > ctx->fwd_tables_cap) {
-    cudaFree(ctx->fwd_tables_d);
-    ctx->fwd_tables_d = nullptr;
-    ctx->fwd_tables_cap = 0;
-    int rc = dalloc(ctx, &ctx->fwd_tables_d, tab.size(), "forward tables");
-    if (rc) return rc;
-    ctx->fwd_tables_cap = tab.size();
-  }
-  CK(cudaMemcpy(ctx->fwd_tables_d, tab.data(), tab.size() * sizeof(int32_t), cudaMemcpyHostToDevice),
-     "cudaMemcpy(forward tables)");
-  ctx->fwd_split_npad = n_pad;
-  drop_graph(ctx);
-  return KVPRM_OK;
-}
-
-// Persistent-forward state that does not depend on the batch: per-layer weight
-// maps and gain pointers in device memory, the tile accumulators and the step
-// counters.
-int setup_forward(kvprm_ctx* ctx, const kvprm_weights* w) {
-  const int NL = ctx->cfg.n_layers;
-  int tiles[kvprm::FWD_KINDS], ktiles[kvprm::FWD_KINDS];
-  fwd_shapes(ctx, tiles, ktiles);
-  int max_tiles = 0;
-  int cnt = 0;
-  for (int k = 0; k < kvprm::FWD_KINDS; ++k) {
-    max_tiles = std::max(max_tiles, tiles[k]);
-    ctx->fwd_tile_cnt_off[k] = cnt;
-    cnt += tiles[k];
-  }
-  ctx->fwd_done_off = cnt;
-  ctx->fwd_n_counters = cnt + kvprm::FWD_KINDS + 2;
-  int rc;
-  ctx->fwd_max_tiles = max_tiles;
-  if ((rc = dalloc(ctx, &ctx->fwd_part, static_cast<size_t>(max_tiles) * 128 * ctx->npad_max, "tile accumulators")))
-    return rc;
-  if ((rc = dalloc(ctx, &ctx->fwd_counters, static_cast<size_t>(ctx->fwd_n_counters), "step counters"))) return rc;
-  std::vector<CUtensorMap> maps(static_cast<size_t>(NL) * kvprm::FWD_KINDS);
-  for (int l = 0; l < NL; ++l) {
-    maps[l * kvprm::FWD_KINDS + kvprm::FWD_QKV] = ctx->tm_qkv[l];
-    maps[l * kvprm::FWD_KINDS + kvprm::FWD_O] = ctx->tm_o[l];
-    maps[l * kvprm::FWD_KINDS + kvprm::FWD_GU] = ctx->tm_gu[l];
-    maps[l * kvprm::FWD_KINDS + kvprm::FWD_DOWN] = ctx->tm_down[l];
-  }
-  CK(cudaMalloc(reinterpret_cast<void**>(&ctx->wmaps_d), maps.size() * sizeof(CUtensorMap)), "cudaMalloc(maps)");
-  CK(cudaMemcpy(ctx->wmaps_d, maps.data(), maps.size() * sizeof(CUtensorMap), cudaMemcpyHostToDevice),
-     "cudaMemcpy(maps)");
-  std::vector<const bf16*> norms(2 * static_cast<size_t>(NL));
-  for (int l = 0; l < NL; ++l) {
-    norms[l] = static_cast<const bf16*>(w->attn_norm[l]);
-    norms[NL + l] = static_cast<const bf16*>(w->mlp_norm[l]);
-  }
-  CK(cudaMalloc(reinterpret_cast<void**>(&ctx->norms_d), norms.size() * sizeof(bf16*)), "cudaMalloc(norms)");
-  CK(cudaMemcpy(ctx->norms_d, norms.data(), norms.size() * sizeof(bf16*), cudaMemcpyHostToDevice),
-     "cudaMemcpy(norms)");
-  ctx->coop = !env_off("KVPRM_NO_COOP");
-  return KVPRM_OK;
-}
 }  // namespace
 
 // ======================================================================== C ABI
@@ -922,7 +681,6 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   }
   CREATE_CK(cu(kvprm::gemm_configure(), "gemm_configure"));
   CREATE_CK(cu(kvprm::attention_configure(), "attention_configure"));
-  CREATE_CK(cu(kvprm::forward_configure(), "forward_configure"));
 
   ModelDims& m = ctx->md;
   m.d = c.d_model;
@@ -1016,13 +774,6 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
       return KVPRM_ENOMEM;
     }
   }
-  ctx->fused = env_on("KVPRM_FUSED");
-  if (ctx->fused) {
-    kvprm::FwdPlan fp;
-    for (int np = 16; np <= ctx->npad_max; np += 16)
-      if (!kvprm::plan_forward(m.hd, m.n_q / m.n_kv, np, fp)) ctx->fused = false;
-  }
-  if (ctx->fused) CREATE_CK(setup_forward(ctx, w));
   CREATE_CK(cu(cudaEventCreateWithFlags(&ctx->staging_ev, cudaEventDisableTiming), "cudaEventCreate"));
   CREATE_CK(cu(cudaStreamCreateWithFlags(&ctx->cap_stream, cudaStreamNonBlocking), "cudaStreamCreate"));
   ctx->use_graph = !env_off("KVPRM_NO_GRAPH");
@@ -1206,10 +957,6 @@ int kvprm_set_debug(kvprm_ctx* ctx, int flags) {
     int rc = dalloc(ctx, &ctx->dbg_h, NB * ctx->md.d, "debug h");
     if (rc) return rc;
   }
-  if ((flags & 8) && !ctx->fwd_probe) {
-    int rc = dalloc(ctx, &ctx->fwd_probe, static_cast<size_t>(ctx->num_sms) * ctx->cfg.n_layers * 48, "event probe");
-    if (rc) return rc;
-  }
   ctx->debug_flags = flags;
   return KVPRM_OK;
 }
@@ -1227,11 +974,6 @@ int kvprm_debug_layers(kvprm_ctx* ctx, int which, void* d_out) {
     if (!(ctx->debug_flags & 4)) return fail(ctx, KVPRM_EINVAL, "hidden-state capture (flag 4) is not enabled");
     src = ctx->dbg_h;
     bytes = L * ctx->md.d * 4;
-  } else if (which == 5) {
-    if (!(ctx->debug_flags & 8) || !ctx->fwd_probe)
-      return fail(ctx, KVPRM_EINVAL, "event probe (flag 8) is not enabled");
-    src = ctx->fwd_probe;
-    bytes = static_cast<size_t>(ctx->num_sms) * ctx->cfg.n_layers * 48 * sizeof(unsigned long long);
   } else {
     return fail(ctx, KVPRM_EINVAL, "unknown capture %d", which);
   }
@@ -1314,7 +1056,7 @@ int kvprm_check_device(kvprm_ctx* ctx) {
   if (*ctx->h_err) {
     const int site = *ctx->h_err;
     CK(cudaMemset(ctx->err_d, 0, sizeof(int)), "cudaMemset(err)");
-    return fail(ctx, KVPRM_ETIMEOUT, "a bounded device wait timed out (wait site %d)", site);
+    return fail(ctx, KVPRM_ETIMEOUT, "a bounded device wait timed out (code %d)", site);
   }
   return KVPRM_OK;
 }
@@ -1323,9 +1065,7 @@ int kvprm_set_trace(kvprm_ctx* ctx, int enable) {
   if (!ctx) return KVPRM_EINVAL;
   if (enable && !ctx->trace_d) {
     ctx->trace_cap = 2 + 8 * ctx->cfg.n_layers + 8;
-    int rc = dalloc(ctx, &ctx->trace_d, static_cast<size_t>(2) * ctx->trace_cap, "trace");
-    if (rc) return rc;
-    rc = dalloc(ctx, &ctx->phase_d, 1 + 6 * static_cast<size_t>(ctx->cfg.n_layers), "phase trace");
+    int rc = dalloc(ctx, &ctx->trace_d, static_cast<size_t>(kvprm::kTraceStride) * ctx->trace_cap, "trace");
     if (rc) return rc;
   }
   ctx->trace = enable != 0;
@@ -1333,38 +1073,34 @@ int kvprm_set_trace(kvprm_ctx* ctx, int enable) {
 }
 
 int kvprm_get_trace(kvprm_ctx* ctx, int32_t max_records, int32_t* cls, double* start_us, double* end_us) {
+  return kvprm_get_trace_events(ctx, max_records, cls, start_us, end_us, nullptr);
+}
+
+int kvprm_get_trace_events(kvprm_ctx* ctx, int32_t max_records, int32_t* cls, double* start_us, double* end_us,
+                           double* events_us) {
   if (!ctx || max_records < 0 || (max_records > 0 && (!cls || !start_us || !end_us))) return -KVPRM_EINVAL;
   if (!ctx->trace_d || ctx->trace_n == 0) return 0;
   if (cudaStreamSynchronize(ctx->last_stream) != cudaSuccess) return -KVPRM_ECUDA;
-  std::vector<unsigned long long> raw(2 * static_cast<size_t>(ctx->trace_n));
+  constexpr int R = kvprm::kTraceStride;
+  std::vector<unsigned long long> raw(static_cast<size_t>(R) * ctx->trace_n);
   if (cudaMemcpy(raw.data(), ctx->trace_d, raw.size() * sizeof(unsigned long long), cudaMemcpyDeviceToHost) !=
       cudaSuccess)
     return -KVPRM_ECUDA;
   unsigned long long t0 = ~0ull;
   for (int i = 0; i < ctx->trace_n; ++i)
-    if (raw[2 * i] < t0) t0 = raw[2 * i];
+    if (raw[R * i] < t0) t0 = raw[R * i];
+  auto rel = [&](unsigned long long v, bool complemented) {
+    if (v == ~0ull) return -1.0;
+    return 1e-3 * static_cast<double>((complemented ? ~v : v) - t0);
+  };
   const int n = ctx->trace_n < max_records ? ctx->trace_n : max_records;
   for (int i = 0; i < n; ++i) {
     cls[i] = ctx->trace_cls[i];
-    start_us[i] = (raw[2 * i] == ~0ull) ? -1.0 : 1e-3 * static_cast<double>(raw[2 * i] - t0);
-    const unsigned long long e = ~raw[2 * i + 1];
-    end_us[i] = (raw[2 * i + 1] == ~0ull) ? -1.0 : 1e-3 * static_cast<double>(e - t0);
+    start_us[i] = rel(raw[R * i], false);
+    end_us[i] = rel(raw[R * i + 1], true);
+    if (events_us)
+      for (int e = 0; e < kvprm::kTraceEvents; ++e) events_us[i * kvprm::kTraceEvents + e] = rel(raw[R * i + 2 + e], true);
   }
-  return n;
-}
-
-int kvprm_get_phase_trace(kvprm_ctx* ctx, int32_t max_records, double* end_us) {
-  if (!ctx || max_records < 0 || (max_records > 0 && !end_us)) return -KVPRM_EINVAL;
-  if (!ctx->fused || !ctx->phase_d || ctx->trace_n == 0) return 0;
-  if (cudaStreamSynchronize(ctx->last_stream) != cudaSuccess) return -KVPRM_ECUDA;
-  const size_t nrec = 6 * static_cast<size_t>(ctx->cfg.n_layers);
-  std::vector<unsigned long long> raw(1 + nrec);
-  if (cudaMemcpy(raw.data(), ctx->phase_d, raw.size() * sizeof(unsigned long long), cudaMemcpyDeviceToHost) !=
-      cudaSuccess)
-    return -KVPRM_ECUDA;
-  const int n = static_cast<int>(std::min<size_t>(nrec, static_cast<size_t>(max_records)));
-  for (int i = 0; i < n; ++i)
-    end_us[i] = raw[1 + i] == 0 ? -1.0 : 1e-3 * static_cast<double>(static_cast<long long>(raw[1 + i] - raw[0]));
   return n;
 }
 

@@ -11,6 +11,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "kernels.h"
+
 namespace kvprm {
 
 constexpr int kDevTimeout = 1;                          // value written to the device error word
@@ -35,6 +37,12 @@ __device__ __forceinline__ void trace_begin(unsigned long long* ts) {
 }
 __device__ __forceinline__ void trace_end(unsigned long long* ts) {
   if (ts && threadIdx.x == 0) atomicMin(&ts[1], ~static_cast<unsigned long long>(global_timer_ns()));
+}
+// Kernels with internal milestones also record, in ts[2 + e] (e < kTraceEvents,
+// complemented like ts[1]), when the LAST CTA reached milestone e: the
+// launch's critical path.  Called by the one thread that passes the milestone.
+__device__ __forceinline__ void trace_event(unsigned long long* ts, int e) {
+  if (ts) atomicMin(&ts[2 + e], ~static_cast<unsigned long long>(global_timer_ns()));
 }
 
 // ---------------------------------------------------------------- mbarrier
@@ -163,69 +171,6 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
   for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
-}
-
-// Each thread of a warp reads 8 consecutive fp32 columns of its own TMEM lane.
-__device__ __forceinline__ void tmem_ld8(uint32_t taddr, float (&v)[8]) {
-  uint32_t r[8];
-  asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0, %1, %2, %3, %4, %5, %6, %7}, [%8];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
-               : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int i = 0; i < 8; ++i) v[i] = __uint_as_float(r[i]);
-}
-
-// ---------------------------------------------------------------- inter-CTA flags (persistent kernels)
-__device__ __forceinline__ int ld_acquire_gpu(const int* p) {
-  int v;
-  asm volatile("ld.acquire.gpu.global.s32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
-  return v;
-}
-// Order this thread's generic-proxy global accesses with later async-proxy
-// (TMA) accesses: data written by ordinary stores and read by TMA.
-__device__ __forceinline__ void fence_proxy_async_global() {
-  asm volatile("fence.proxy.async.global;" ::: "memory");
-}
-// Wait until *cnt >= target (acquire).  Bounded like mbar_wait: false after
-// kWaitTimeoutNs (flagging *err), or at once when *err is already set.
-__device__ __forceinline__ bool wait_counter(const int* cnt, int target, int* err, int site = kDevTimeout) {
-  if (ld_acquire_gpu(cnt) >= target) return true;
-  const uint64_t t0 = global_timer_ns();
-  for (;;) {
-#pragma unroll 1
-    for (int i = 0; i < 16; ++i)
-      if (ld_acquire_gpu(cnt) >= target) return true;
-    if (*(volatile int*)err != 0) return false;
-    if (global_timer_ns() - t0 > kWaitTimeoutNs) {
-      atomicCAS(err, 0, site);
-      return false;
-    }
-  }
-}
-
-// ---------------------------------------------------------------- cp.async (LSU path, L2 only)
-__device__ __forceinline__ void cp_async16_cg(uint32_t dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-// Wait until at most n (0..7) committed groups of this thread are pending.
-__device__ __forceinline__ void cp_async_wait_pending(int n) {
-  switch (n) {
-    case 0: asm volatile("cp.async.wait_group 0;" ::: "memory"); break;
-    case 1: asm volatile("cp.async.wait_group 1;" ::: "memory"); break;
-    case 2: asm volatile("cp.async.wait_group 2;" ::: "memory"); break;
-    case 3: asm volatile("cp.async.wait_group 3;" ::: "memory"); break;
-    case 4: asm volatile("cp.async.wait_group 4;" ::: "memory"); break;
-    case 5: asm volatile("cp.async.wait_group 5;" ::: "memory"); break;
-    case 6: asm volatile("cp.async.wait_group 6;" ::: "memory"); break;
-    default: asm volatile("cp.async.wait_group 7;" ::: "memory"); break;
-  }
-}
-// Make this thread's completed generic-proxy shared-memory writes visible to
-// the async proxy (tcgen05.mma operand reads).
-__device__ __forceinline__ void fence_proxy_async_smem() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
 // Shared-memory matrix descriptor (tcgen05 "matrix descriptor") for a K-major

@@ -17,7 +17,7 @@ from . import build as _build
 
 KVPRM_OK, KVPRM_EINVAL, KVPRM_ECAPACITY, KVPRM_EINDEX, KVPRM_ECUDA, KVPRM_ENOMEM, KVPRM_ETIMEOUT, \
     KVPRM_EUNSUPPORTED = range(8)
-PROF_NAMES = ("gemm_qkv", "gemm_o", "gemm_gate_up", "gemm_down", "attention", "combine", "fused", "forward")
+PROF_NAMES = ("gemm_qkv", "gemm_o", "gemm_gate_up", "gemm_down", "attention", "combine", "fused")
 
 
 class KvprmError(RuntimeError):
@@ -84,8 +84,9 @@ def lib() -> ctypes.CDLL:
         L.kvprm_set_profile.argtypes = [vp, ctypes.c_int]
         L.kvprm_set_trace.argtypes = [vp, ctypes.c_int]
         L.kvprm_get_trace.argtypes = [vp, i32, i32p, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)]
+        L.kvprm_get_trace_events.argtypes = [vp, i32, i32p, ctypes.POINTER(ctypes.c_double),
+                                             ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)]
         L.kvprm_get_profile.argtypes = [vp, i64p, ctypes.POINTER(ctypes.c_double)]
-        L.kvprm_get_phase_trace.argtypes = [vp, i32, ctypes.POINTER(ctypes.c_double)]
         L.kvprm_plan_attention.argtypes = [i32p, i32, i32p, i32, i32, i32, i32, i32, ctypes.POINTER(KvprmAttnPlan)]
         _lib = L
     return _lib
@@ -250,14 +251,18 @@ def kvprm_get_trace(ctx, max_records: int = 4096) -> list:
     return [(PROF_NAMES[cls[i]], float(t0[i]), float(t1[i])) for i in range(n)]
 
 
-def kvprm_get_phase_trace(ctx, max_records: int = 6 * 256) -> np.ndarray:
-    """[n_layers][6] end times (us after the kernel start) of the persistent kernel's steps
-    (QKV, attention, combine, O, gate/up, down) in the last traced call; empty if none."""
-    end = np.zeros(max_records, np.float64)
-    n = lib().kvprm_get_phase_trace(ctx, max_records, end.ctypes.data_as(ctypes.POINTER(ctypes.c_double)))
+def kvprm_get_trace_events(ctx, max_records: int = 4096) -> list:
+    """[(class name, start us, end us, [8 milestone us or -1])] of the last call's launches, in issue order."""
+    dp = ctypes.POINTER(ctypes.c_double)
+    cls = np.zeros(max_records, np.int32)
+    t0 = np.zeros(max_records, np.float64)
+    t1 = np.zeros(max_records, np.float64)
+    ev = np.zeros((max_records, 8), np.float64)
+    n = lib().kvprm_get_trace_events(ctx, max_records, _p(cls, ctypes.c_int32), t0.ctypes.data_as(dp),
+                                     t1.ctypes.data_as(dp), ev.ctypes.data_as(dp))
     if n < 0:
         _check(ctx, -n)
-    return end[:n].reshape(-1, 6)
+    return [(PROF_NAMES[cls[i]], float(t0[i]), float(t1[i]), ev[i].tolist()) for i in range(n)]
 
 
 def kvprm_get_profile(ctx) -> dict:
