@@ -292,8 +292,11 @@ KVPRM_API int kvprm_get_trace(kvprm_ctx* ctx, int32_t max_records, int32_t* cls,
  * activation tiles landed, 2 all MMAs completed, 3 the accumulators were
  * parked in shared memory cluster-wide, 4 the split-K reduction over the
  * cluster was done, 5 the RMSNorm factors were ready, 6 the epilogue was
- * written, 7 the cluster released -- or -1 where a launch has no such
- * milestone (attention, combine and the small kernels record none). */
+ * written, 7 the cluster released.  Attention launches record 0 the query
+ * was ready, 1 the consumer warps had scored every page, 2 the private runs
+ * were merged into their partial slots; combine launches 0 the partials were
+ * ready, 1 the outputs were written.  -1 where a launch has no such
+ * milestone. */
 KVPRM_API int kvprm_get_trace_events(kvprm_ctx* ctx, int32_t max_records, int32_t* cls, double* start_us,
                                      double* end_us, double* events_us);
 KVPRM_API int kvprm_get_profile(kvprm_ctx* ctx, int64_t* launches, double* total_ms);

@@ -168,6 +168,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
     // Every warp waits for every stage before releasing it, busy or not, so
     // no warp can arrive for a slot's next use early.
     grid_dep_wait();   // q is written by the preceding kernel
+    if (warp == 0 && lane == 0) trace_event(ts, 0);   // the query is ready
     bool ok = true;
     uint32_t u = 0, n_priv = 0;
     for (int si = seg0; si < seg1; ++si) {
@@ -221,6 +222,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
         store_state_slot<HD, TWO_ROWS>(st, slot_id, group, lane, part_o, part_ml);
       }
     }
+    if (lane == 0) trace_event(ts, 1);   // this warp has scored every page of its CTA
   } else if (warp == kMergerWarp && !TWO_ROWS) {
     // ------------------------------------------------ merger
     // For every private segment, in order: fold the eight consumer warps'
@@ -237,6 +239,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
       if (lane == 0) mbar_arrive(seg_free);
       ++k;
     }
+    if (lane == 0) trace_event(ts, 2);   // every private run of this CTA is merged
   }
   trace_end(ts);
 }
@@ -252,8 +255,10 @@ __global__ void __launch_bounds__(CombineShape<HD, ROWS>::W * 32) attn_combine_k
   const int cg = blockIdx.x, b = cg / n_kv, g = cg - b * n_kv;
   const int first = slot_base[cg], ns = nslots[cg];   // host-uploaded before the call: no wait needed
   grid_dep_wait();   // the partials (and q, k_self, v_self) are written by earlier kernels
+  if (threadIdx.x == 0) trace_event(ts, 0);
   combine_group<HD, ROWS>(threadIdx.x, b, g, first, ns, n_q, n_kv, group, part_o, part_ml, mg, csm,
                           [] { __syncthreads(); });
+  if (threadIdx.x == 0) trace_event(ts, 1);
   trace_end(ts);
 }
 
