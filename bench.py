@@ -158,8 +158,10 @@ def source_hash(files: list[str]) -> str:
 
 
 KERNEL_SOURCES = {
-    "gemm": ["paper_2607_09153_gb300/csrc/gemm_tc.cu", "paper_2607_09153_gb300/csrc/ptx.cuh"],
-    "attention": ["paper_2607_09153_gb300/csrc/attention.cu", "paper_2607_09153_gb300/csrc/ptx.cuh"],
+    "gemm": ["paper_2607_09153_gb300/csrc/gemm_tc.cu", "paper_2607_09153_gb300/csrc/ptx.cuh",
+             "paper_2607_09153_gb300/csrc/kernels.h"],
+    "attention": ["paper_2607_09153_gb300/csrc/attention.cu", "paper_2607_09153_gb300/csrc/attn_core.cuh",
+                  "paper_2607_09153_gb300/csrc/ptx.cuh", "paper_2607_09153_gb300/csrc/kernels.h"],
 }
 
 
