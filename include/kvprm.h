@@ -202,7 +202,21 @@ KVPRM_API int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, con
  * the last call's stream).  Bit 1: keep every layer's rotated q, self k and
  * self v (float); bit 2: keep the residual stream after every layer (float).
  * kvprm_debug_layers copies them: which = 1 q [N_L][n][n_q*hd], 2 k_self
- * [N_L][n][n_kv*hd], 3 v_self (same), 4 h [N_L][n][d_model]. */
+ * [N_L][n][n_kv*hd], 3 v_self (same), 4 h [N_L][n][d_model].  Bit 4: the
+ * tensor-core attention of shared pages rescales its running state on every
+ * new row maximum instead of only beyond a margin of 2^8 (same result up to
+ * rounding; exercises the rescale path).  Bit 5: the tensor-core attention
+ * accumulates a wait profile; which = 5 copies uint64 [1024 + n_SM * 16]:
+ * first CTA 0's event log of the last launch, [8][128] SM-clock stamps -- per
+ * chunk 0 S issued, 1 O issued, 2 S seen by the softmax, 3 P written, 4
+ * values requested, 5 keys requested; per segment 6 Q loaded, 7 O written
+ * out ([7][127] holds the CTA's start) -- then [n_SM][16] SM-clock cycles per
+ * CTA, summed over every launch since the flag was set: 0 the MMA issuer
+ * waiting for keys, 1 for the S buffer (the O MMAs four chunks back), 2 for
+ * P, 3 for values; 4 the softmax waiting for S, 5 for the previous O before a
+ * rescale; 6 the loader waiting for a free key stage, 7 for a free value
+ * stage; 8 reading S, 9 computing and storing P, 10 a segment's O read-out,
+ * 11 loading Q; 12 chunks scored; 13 the CTA's lifetime. */
 KVPRM_API int kvprm_set_debug(kvprm_ctx* ctx, int flags);
 KVPRM_API int kvprm_debug_attn_out(kvprm_ctx* ctx, float* d_out);
 KVPRM_API int kvprm_debug_layers(kvprm_ctx* ctx, int which, void* d_out);
@@ -223,15 +237,24 @@ KVPRM_API int kvprm_resolve(kvprm_ctx* ctx, int32_t b, int64_t* phys_row);
  * (candidate, kv head) with the verify token's own entry.
  * Inputs: block_table host int32 [n_candidates][max_blocks_per_seq], seq_lens
  * host int32 [n_candidates], group = n_q_heads / n_kv_heads, n_ctas >= 1,
- * share != 0 to form shared segments.  Outputs go to caller-owned arrays with
- * the capacities given (elements); the counts are always written:
+ * share: 0 no sharing, 1 shared segments (kind 1) on the persistent CTAs, 2
+ * shared pages scored on the tensor cores (kind 2; what scoring contexts with
+ * head_dim 128 use): tiles of up to 128 / group candidates whose 4-page
+ * chunks are cut into equal ranges, one per CTA of a separate launch (at most
+ * n_ctas of them); kind-2 segments follow the persistent CTAs' segments
+ * (segs[cta_seg[n_ctas]] on), and tensor-core CTA k scores segments
+ * segs[tc_cta[k]] .. segs[tc_cta[k + 1] - 1].
+ * Outputs go to caller-owned arrays with the capacities given (elements); the
+ * counts are always written:
  *  segs       [n_segs][8] int32: kind, kv head, candidate (kind 0) or offset
- *             into cands (kind 1), candidates, offset into pages, pages, valid
- *             tokens of the last page, slot (kind 0) or offset into slots
- *  cta_seg    [n_ctas + 1] first segment of each CTA
+ *             into cands (kinds 1, 2), candidates, offset into pages, pages,
+ *             valid tokens of the last page, slot (kind 0) or offset into slots
+ *  cta_seg    [n_ctas + 1] first segment of each persistent CTA
  *  pages      physical page ids referenced by segments
- *  cands      candidates of kind-1 segments; slots: their partial slots
+ *  cands      candidates of kind-1 and kind-2 segments; slots: their partial slots
  *  slot_base, nslots  [n_candidates][n_kv_heads] first slot and slot count
+ *  tc_cta     [n_tc_ctas + 1] first segment (index into segs) of each
+ *             tensor-core CTA
  * Returns KVPRM_EINVAL for bad arguments and KVPRM_ECAPACITY if an array is
  * too small (counts still reflect the full plan). */
 typedef struct {
@@ -248,6 +271,9 @@ typedef struct {
   int64_t slots_cap;
   int32_t* slot_base; /* [n_candidates * n_kv_heads] */
   int32_t* nslots;    /* [n_candidates * n_kv_heads] */
+  int32_t n_tc_ctas;  /* out */
+  int32_t* tc_cta;
+  int64_t tc_cta_cap;
 } kvprm_attn_plan;
 KVPRM_API int kvprm_plan_attention(const int32_t* block_table, int32_t max_blocks_per_seq, const int32_t* seq_lens,
                                    int32_t n_candidates, int32_t n_kv_heads, int32_t group, int32_t n_ctas,

@@ -67,6 +67,10 @@ constexpr int kThreads = (kConsumerWarps + 2) * 32;
 // half a private page per candidate.
 constexpr int64_t kPrivateCost = 4;
 constexpr int64_t kSharedCostPerCand = 2;
+// Tensor-core scoring of shared pages (attn_tc_kernel): query rows per tile
+// and pages per 64-token chunk.
+constexpr int kTcRows = 128;
+constexpr int kTcChunkPages = 4;
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -262,6 +266,420 @@ __global__ void __launch_bounds__(CombineShape<HD, ROWS>::W * 32) attn_combine_k
   trace_end(ts);
 }
 
+// ---------------------------------------------------------------- shared pages on the tensor cores
+// attn_tc_kernel: persistent CTAs, each scoring its range of kind-2 segments
+// (wk.tc_cta).  A segment is a tile of <= 128 / G candidates that all
+// reference its pages, for one kv head; the tile's query rows (candidate,
+// head) are the M = 128 side of tcgen05 MMAs whose A operands live in tensor
+// memory:
+//   S = Q K^T   per 64-token chunk (4 pages): A = Q as bf16 hi and lo (two
+//               MMAs, so S sees the fp32 query), B = the chunk's keys in
+//               shared memory; S in TMEM, two 64-column buffers;
+//   softmax     one thread per query row reads its S row; the running
+//               maximum m only moves when a chunk's scores exceed it by more
+//               than `margin` (log2 units; then the row's O is rescaled in
+//               TMEM), so P = 2^(s - m) stays below 2^margin and rescales are
+//               rare; P goes back as bf16 hi and lo (truncations by bit mask,
+//               |P - hi - lo| < 2^-14 P) over the S buffer it came from;
+//   O += P V    A = P (hi, lo) from TMEM, B = the chunk's values in shared
+//               memory as TMA left them (token rows of 128 bytes): an
+//               MN-major operand, so nothing is transposed; O in TMEM (128
+//               columns).
+// Warp 0 streams K with TMA (one 2 KB box per page and 64-column sub-tile,
+// so a chunk's 64 tokens land contiguously; a segment's missing tail pages
+// are read at an out-of-range page and arrive as zeros) through a 6-stage
+// ring released by the S MMAs that read it; warp 10 streams V the same way
+// through a ring released by the O MMAs, so neither waits for the other.
+// Warp 1 issues the MMAs (S two chunks ahead of O within a segment, four S/P
+// buffers); warps 2..9 run the softmax, two threads per query row (each 32 of
+// a chunk's 64 columns; the half maxima meet in shared memory) and, at each
+// segment's end, write every live row's (m, l, O) into its candidate's
+// partial slot.
+struct TcSmem {
+  static constexpr int kStages = 6;
+  static constexpr uint32_t kKVTile = 2 * 64 * 128;          // [2 sub-tiles][64 tokens][128 B] = 16 KB
+  static constexpr uint32_t kK = 0;                          // key stages
+  static constexpr uint32_t kV = kK + kStages * kKVTile;     // value stages
+  static constexpr uint32_t kBars = kV + kStages * kKVTile;
+  static constexpr uint32_t kXch = kBars + 512;               // softmax exchange: half maxima [2][128], l [128]
+  static constexpr uint32_t kEnd = kXch + 3 * 128 * 4;
+  static constexpr size_t kDynamic = kEnd + 1024;
+};
+static_assert(TcSmem::kDynamic <= 227 * 1024, "tensor-core attention shared memory exceeds the per-block limit");
+constexpr int kTcThreads = 352;   // warp 0 key TMA, 1 MMA, 2..9 softmax (two threads per row), 10 value TMA
+constexpr uint32_t kTcTmemCols = 512;
+// TMEM columns: four S/P buffers at 0, 64, 128, 192; O at 256..383; Q hi at 384..447, Q lo at 448..511.
+// With four S buffers the MMA warp issues S two chunks ahead of the softmax without waiting for
+// the O MMAs that read the P it overwrites (those completed two chunks earlier).
+constexpr int kTcSBufs = 4;
+constexpr uint32_t kColO = 256, kColQhi = 384, kColQlo = 448;
+
+__global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(
+    const __grid_constant__ CUtensorMap tm_pool_tc, int64_t layer_page0, AttnWork wk,
+    const __nv_bfloat16* __restrict__ q_hi, const __nv_bfloat16* __restrict__ q_lo, int n_q, int group,
+    float* __restrict__ part_o, float* __restrict__ part_ml, float margin, int* err, unsigned long long* ts,
+    unsigned long long* prof) {
+  using SM = TcSmem;
+  trace_begin(ts);
+  // optional wait profile (SM clock cycles per CTA, accumulated with reductions so that the
+  // measured warps never wait on a load) and CTA 0's per-chunk event log: see kvprm_set_debug, flag 32
+  unsigned long long* pr = prof ? prof + kTcEventLog + static_cast<int64_t>(blockIdx.x) * 16 : nullptr;
+  unsigned long long* ev = (prof && blockIdx.x == 0) ? prof : nullptr;
+  auto tic = [&]() -> long long { return pr ? clock64() : 0; };
+  auto toc = [&](int slot, long long t0) {
+    if (pr) atomicAdd(pr + slot, static_cast<unsigned long long>(clock64() - t0));
+  };
+  auto event = [&](int kind, uint32_t i) {
+    if (ev && i < 128) ev[kind * 128 + i] = static_cast<unsigned long long>(clock64());
+  };
+  const long long t_start = tic();
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base = align1024(smem_raw);
+  uint64_t* k_full = reinterpret_cast<uint64_t*>(base + SM::kBars);    // [6] keys landed
+  uint64_t* k_empty = k_full + SM::kStages;                           // [6] the S MMAs read the keys
+  uint64_t* v_full = k_empty + SM::kStages;                           // [6] values landed
+  uint64_t* v_empty = v_full + SM::kStages;                           // [6] the O MMAs read the values
+  uint64_t* s_full = v_empty + SM::kStages;                           // [4] S in TMEM
+  uint64_t* p_full = s_full + kTcSBufs;                               // [4] P in TMEM
+  uint64_t* pv_done = p_full + kTcSBufs;                              // [4] the O MMAs of a chunk completed
+  uint64_t* q_ready = pv_done + kTcSBufs;                             // Q of the current segment in TMEM
+  uint64_t* o_free = q_ready + 1;                                     // O of the previous segment read out
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(o_free + 1);
+  const int seg0 = wk.tc_cta[blockIdx.x], seg1 = wk.tc_cta[blockIdx.x + 1];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  auto chunks = [](const AttnSeg& sg) { return (sg.n_pages + kTcChunkPages - 1) / kTcChunkPages; };
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < SM::kStages; ++s) {
+      mbar_init(&k_full[s], 1);
+      mbar_init(&k_empty[s], 1);
+      mbar_init(&v_full[s], 1);
+      mbar_init(&v_empty[s], 1);
+    }
+    for (int b = 0; b < kTcSBufs; ++b) {
+      mbar_init(&s_full[b], 1);
+      mbar_init(&p_full[b], 8);
+      mbar_init(&pv_done[b], 1);
+    }
+    mbar_init(q_ready, 8);
+    mbar_init(o_free, 8);
+    fence_mbar_init();
+    tma_prefetch_desc(&tm_pool_tc);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kTcTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  grid_dep_launch();
+
+  if (warp == 0 || warp == 10) {
+    // ------------------------------------------------ loaders: warp 0 the keys, warp 10 the values
+    // (the cache does not depend on q; each ring runs ahead of its own consumer)
+    if (lane == 0) {
+      const bool keys = warp == 0;
+      const uint64_t pol = policy_evict_normal();   // the group's other tiles read the same pages
+      // one ring (keys or values): wait for the stage, then all four pages of the chunk, a page
+      // past the segment's end at unit -1 (out of range: TMA writes zeros and counts the bytes)
+      auto load = [&](uint64_t* full, uint64_t* empty, uint32_t off, int slot, uint32_t u, const int32_t* pg, int npg,
+                      int g, int kv) -> bool {
+        const int st = static_cast<int>(u % SM::kStages);
+        const long long t0 = tic();
+        if (u >= static_cast<uint32_t>(SM::kStages) && !mbar_wait(&empty[st], ((u / SM::kStages) - 1) & 1u, err))
+          return false;
+        toc(slot, t0);
+        mbar_arrive_expect_tx(&full[st], SM::kKVTile);
+        uint8_t* dst = base + off + st * SM::kKVTile;
+#pragma unroll
+        for (int i = 0; i < kTcChunkPages; ++i) {
+          const int32_t unit = i < npg ? static_cast<int32_t>(2 * (layer_page0 + __ldg(pg + i))) + kv : -1;
+#pragma unroll
+          for (int sub = 0; sub < 2; ++sub)
+            tma_load_5d(dst + sub * 8192 + i * 2048, &tm_pool_tc, &full[st], 0, 0, sub, g, unit, pol);
+        }
+        return true;
+      };
+      uint64_t* full = keys ? k_full : v_full;
+      uint64_t* empty = keys ? k_empty : v_empty;
+      uint32_t u = 0;
+      bool ok = true;
+      for (int si = seg0; si < seg1 && ok; ++si) {
+        const AttnSeg sg = wk.segs[si];
+        const int32_t* pg = wk.pages + sg.page_off;
+        for (int c = 0; c < chunks(sg) && ok; ++c, ++u) {
+          const int npg = min(kTcChunkPages, sg.n_pages - c * kTcChunkPages);
+          event(keys ? 5 : 4, u);
+          ok = load(full, empty, keys ? SM::kK : SM::kV, keys ? 6 : 7, u, pg + c * kTcChunkPages, npg, sg.g,
+                    keys ? 0 : 1);
+        }
+      }
+      for (uint32_t v = u > static_cast<uint32_t>(SM::kStages) ? u - SM::kStages : 0; v < u; ++v)   // all landed
+        if (!mbar_wait(&full[v % SM::kStages], (v / SM::kStages) & 1u, err)) break;
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer (the whole warp; one elected lane issues)
+    // O MMAs take V as an MN-major B operand (instruction descriptor bit 16)
+    const uint32_t id_s = idesc_bf16_f32(128, 64), id_o = idesc_bf16_f32(128, 128) | (1u << 16);
+    auto wait_all = [&](uint64_t* bar, uint32_t parity) { return __all_sync(0xffffffffu, mbar_wait(bar, parity, err)); };
+    auto issue_s = [&](uint32_t v) -> bool {
+      const int st = static_cast<int>(v % SM::kStages);
+      const uint32_t b = v % kTcSBufs;
+      long long t0 = tic();
+      if (!wait_all(&k_full[st], (v / SM::kStages) & 1u)) return false;
+      if (lane == 0) toc(0, t0);
+      t0 = tic();
+      if (v >= kTcSBufs && !wait_all(&pv_done[b], ((v / kTcSBufs) - 1) & 1u)) return false;   // P of v - 4 consumed
+      if (lane == 0) toc(1, t0);
+      tc_fence_after();
+      // keys: two 64-column sub-tiles of 8 KB; K step kk at sub-tile kk / 4, 32 bytes per step inside it
+      const uint64_t k0 = desc_sw128(smem_u32(base + SM::kK + st * SM::kKVTile));
+      const uint32_t d = tmem + b * 64;
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk) {
+        const uint64_t kdesc = k0 + (((kk >> 2) * 8192 + (kk & 3) * 32) >> 4);
+        umma_bf16_ta_w(d, tmem + kColQhi + kk * 8, kdesc, id_s, kk > 0 ? 1u : 0u);
+        umma_bf16_ta_w(d, tmem + kColQlo + kk * 8, kdesc, id_s, 1u);
+      }
+      umma_commit_w(&s_full[b]);
+      umma_commit_w(&k_empty[st]);
+      if (lane == 0) event(0, v);
+      return true;
+    };
+    auto issue_o = [&](uint32_t v, bool first) -> bool {
+      const int st = static_cast<int>(v % SM::kStages);
+      const uint32_t b = v % kTcSBufs;
+      long long t0 = tic();
+      if (!wait_all(&p_full[b], (v / kTcSBufs) & 1u)) return false;
+      if (lane == 0) toc(2, t0);
+      t0 = tic();
+      if (!wait_all(&v_full[st], (v / SM::kStages) & 1u)) return false;
+      if (lane == 0) toc(3, t0);
+      tc_fence_after();
+      // values: N = head dim over the two 64-column sub-tiles (8 KB apart), K = tokens in groups
+      // of 8 rows (1 KB apart); K step kk starts 16 rows (2 KB) further
+      const uint64_t v0 = desc_sw128_mn(smem_u32(base + SM::kV + st * SM::kKVTile), 8192);
+      const uint32_t p = tmem + b * 64;
+      const uint32_t acc0 = first ? 0u : 1u;
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk) {   // the chunk's 64 tokens in steps of 16
+        umma_bf16_ta_w(tmem + kColO, p + kk * 8, v0 + 128 * kk, id_o, kk > 0 ? 1u : acc0);
+        umma_bf16_ta_w(tmem + kColO, p + 32 + kk * 8, v0 + 128 * kk, id_o, 1u);
+      }
+      umma_commit_w(&pv_done[b]);
+      umma_commit_w(&v_empty[st]);
+      if (lane == 0) event(1, v);
+      return true;
+    };
+    uint32_t u = 0, k = 0;
+    bool ok = true;
+    for (int si = seg0; si < seg1 && ok; ++si, ++k) {
+      const int nch = chunks(wk.segs[si]);
+      ok = wait_all(q_ready, k & 1u) && (k == 0 || wait_all(o_free, (k - 1) & 1u));
+      if (ok) ok = issue_s(u);
+      if (ok && nch > 1) ok = issue_s(u + 1);
+      for (int c = 0; c < nch && ok; ++c, ++u) {   // S two chunks ahead of O
+        if (c + 2 < nch) ok = issue_s(u + 2);
+        if (ok) ok = issue_o(u, c == 0);
+      }
+    }
+  } else if (warp < 10) {
+    // ------------------------------------------------ softmax: two threads per query row (columns 0..31 / 32..63)
+    const int w4 = warp & 3;              // TMEM lane quadrant of this warp
+    const int hsel = (warp - 2) >> 2;     // which half of the chunk's columns (and of Q, O) this thread owns
+    const int r = w4 * 32 + lane;
+    const uint32_t trow = tmem + (static_cast<uint32_t>(w4 * 32) << 16);
+    float* s_hmax = reinterpret_cast<float*>(base + SM::kXch);   // [2 halves][128 rows]
+    float* s_l = s_hmax + 256;                                   // [128 rows]
+    const float sl2 = kLog2e * rsqrtf(128.f);
+    grid_dep_wait();   // q is written by the preceding kernel
+    if (threadIdx.x == 64) trace_event(ts, 0);
+    uint32_t u = 0, k = 0;
+    bool ok = true;
+    for (int si = seg0; si < seg1; ++si, ++k) {
+      const AttnSeg sg = wk.segs[si];
+      const int nch = chunks(sg);
+      const int ci = r / group, hr = r - ci * group;
+      const bool live = ci < sg.n_cands;
+      // Q of this row into TMEM: half 0 the hi part, half 1 the lo part (every MMA of the
+      // previous segment has completed)
+      const long long tq = tic();
+      {
+        const int64_t row0 =
+            live ? (static_cast<int64_t>(wk.cands[sg.cand + ci]) * n_q + static_cast<int64_t>(sg.g) * group + hr) * 128
+                 : 0;
+        const __nv_bfloat16* src = hsel ? q_lo : q_hi;
+        uint4 w[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e) w[e] = live ? *reinterpret_cast<const uint4*>(src + row0 + e * 8) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {   // 32 head-dim elements = 16 columns per store
+          float v[16];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            v[4 * e] = __uint_as_float(w[4 * j + e].x);
+            v[4 * e + 1] = __uint_as_float(w[4 * j + e].y);
+            v[4 * e + 2] = __uint_as_float(w[4 * j + e].z);
+            v[4 * e + 3] = __uint_as_float(w[4 * j + e].w);
+          }
+          tmem_st16(trow + (hsel ? kColQlo : kColQhi) + j * 16, v);
+        }
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(q_ready);
+      }
+      if (lane == 0 && warp == 2) {
+        toc(11, tq);
+        event(6, k);
+      }
+      float m = -INFINITY, l = 0.f;
+      for (int c = 0; c < nch; ++c, ++u) {
+        const uint32_t b = u % kTcSBufs;
+        long long t0 = tic();
+        if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&s_full[b], (u / kTcSBufs) & 1u, err));
+        // tokens of my 32 that exist (none after a timeout: x is then never read)
+        const int valid = ok ? min(kTcChunkPages, sg.n_pages - c * kTcChunkPages) * 16 - 32 * hsel : 0;
+        tc_fence_after();
+        if (lane == 0 && warp == 2) {
+          toc(4, t0);
+          event(2, u);
+        }
+        t0 = tic();
+        float x[32];
+        if (ok) {
+          float v0[16], v1[16];
+          tmem_ld16_nowait(trow + b * 64 + hsel * 32, v0);
+          tmem_ld16_nowait(trow + b * 64 + hsel * 32 + 16, v1);
+          tmem_wait_ld();
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            x[j] = v0[j];
+            x[16 + j] = v1[j];
+          }
+        }
+        if (lane == 0 && warp == 2) toc(8, t0);
+        t0 = tic();
+        float hm = -INFINITY;   // my half's maximum of the raw scores, then in log2 units
+        if (valid >= 32) {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) hm = fmaxf(hm, x[j]);
+        } else {
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            x[j] = j < valid ? x[j] : -INFINITY;
+            hm = fmaxf(hm, x[j]);
+          }
+        }
+        hm *= sl2;
+        s_hmax[hsel * 128 + r] = hm;
+        tc_fence_before();   // my S loads are done before the other half may write P over them
+        named_bar_sync(1, 256);
+        const float mx = fmaxf(hm, s_hmax[(hsel ^ 1) * 128 + r]);
+        named_bar_sync(1, 256);   // both halves have read before the next chunk overwrites
+        tc_fence_after();
+        const bool grow = mx > m + margin;   // else keep the stale maximum: 2^(s - m) <= 2^margin
+        if (c > 0 && ok && __any_sync(0xffffffffu, grow)) {   // move my half of O to the new maximum
+          const uint32_t pb = (u - 1) % kTcSBufs;
+          const long long tr = tic();
+          ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[pb], ((u - 1) / kTcSBufs) & 1u, err));
+          if (lane == 0 && warp == 2) toc(5, tr);
+          tc_fence_after();
+          const float alpha = grow ? exp2f(m - mx) : 1.f;
+          if (ok) {
+#pragma unroll 1
+            for (int c0 = 0; c0 < 64; c0 += 16) {
+              float v[16];
+              tmem_ld16(trow + kColO + hsel * 64 + c0, v);
+#pragma unroll
+              for (int j = 0; j < 16; ++j) v[j] *= alpha;
+              tmem_st16(trow + kColO + hsel * 64 + c0, v);
+            }
+            tmem_wait_st();
+          }
+        }
+        if (grow) {
+          l *= exp2f(m - mx);
+          m = mx;
+        }
+        // P = 2^(s - m) for my 32 tokens as bf16 hi (columns hsel*16 ..) and lo (32 + hsel*16 ..):
+        // hi = p truncated to bf16, lo = (p - hi) truncated, by bit masks: |p - hi - lo| < 2^-14 p
+        float hv[16], lv[16];
+        const float nm = -m;
+#pragma unroll
+        for (int e = 0; e < 16; ++e) {
+          const float p0 = ex2_ftz(fmaf(x[2 * e], sl2, nm)), p1 = ex2_ftz(fmaf(x[2 * e + 1], sl2, nm));
+          l += p0 + p1;
+          const uint32_t h0 = __float_as_uint(p0) & 0xFFFF0000u, h1 = __float_as_uint(p1) & 0xFFFF0000u;
+          const uint32_t l0 = __float_as_uint(p0 - __uint_as_float(h0));
+          const uint32_t l1 = __float_as_uint(p1 - __uint_as_float(h1));
+          hv[e] = __uint_as_float(__byte_perm(h0, h1, 0x7632));   // upper halves: (h0, h1)
+          lv[e] = __uint_as_float(__byte_perm(l0, l1, 0x7632));
+        }
+        tmem_st16(trow + b * 64 + hsel * 16, hv);
+        tmem_st16(trow + b * 64 + 32 + hsel * 16, lv);
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&p_full[b]);
+        if (lane == 0 && warp == 2) {
+          toc(9, t0);
+          if (pr) atomicAdd(pr + 12, 1ull);
+          event(3, u);
+        }
+      }
+      if (threadIdx.x == 64 && si == seg1 - 1) trace_event(ts, 1);
+      // the segment's partial slots: (m, l) and the unnormalised O of every live row, my half of O
+      const uint32_t lb = (u - 1) % kTcSBufs;
+      const long long to = tic();
+      if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&pv_done[lb], ((u - 1) / kTcSBufs) & 1u, err));
+      tc_fence_after();
+      if (hsel) s_l[r] = l;
+      named_bar_sync(1, 256);
+      if (ok) {
+        const int slot = live ? wk.slots[sg.slot + ci] : 0;
+        float* dst = part_o + (static_cast<int64_t>(slot) * group + hr) * 128 + hsel * 64;
+        float v[4][16];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) tmem_ld16_nowait(trow + kColO + hsel * 64 + q * 16, v[q]);
+        tmem_wait_ld();
+        if (live) {
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+#pragma unroll
+            for (int j = 0; j < 16; j += 4)
+              *reinterpret_cast<float4*>(dst + q * 16 + j) = make_float4(v[q][j], v[q][j + 1], v[q][j + 2], v[q][j + 3]);
+          if (!hsel)
+            *reinterpret_cast<float2*>(part_ml + (static_cast<int64_t>(slot) * group + hr) * 2) = make_float2(m, l + s_l[r]);
+        }
+      }
+      named_bar_sync(1, 256);   // s_l is read before the next segment writes it
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(o_free);
+      if (lane == 0 && warp == 2) {
+        toc(10, to);
+        event(7, k);
+      }
+    }
+    if (threadIdx.x == 64) trace_event(ts, 2);
+  }
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTcTmemCols);
+  }
+  if (threadIdx.x == 0) {
+    toc(13, t_start);
+    if (ev) ev[7 * 128 + 127] = static_cast<unsigned long long>(t_start);
+  }
+  trace_end(ts);
+}
+
 __global__ void resolve_kernel(const int32_t* __restrict__ bt, const int32_t* __restrict__ seq_lens, int max_blocks,
                                int b, int64_t* __restrict__ out) {
   const int L = seq_lens[b];
@@ -322,20 +740,31 @@ size_t attn_slot_capacity(int max_candidates, int n_kv, int num_sms) {
 // Host planner.
 //  1. Shared pages: full pages that >= 2 candidates reference, each exactly
 //     once, grouped by their exact candidate set; each set is cut into chunks
-//     of <= 8 candidates, one run per chunk.  Every other page of a candidate
-//     goes to its private run.
+//     of <= 8 candidates (share = 1: scored by the persistent kernel, one
+//     warp per candidate) or of <= 128 / G candidates (share = 2: one
+//     tensor-core tile of up to 128 query rows, see attn_tc_kernel), one run
+//     per chunk.  Every other page of a candidate goes to its private run.
 //  2. The (run, kv head) pairs are laid end to end on a cost axis (a page
 //     costs kPrivateCost, or kSharedCostPerCand per candidate) and each page goes to the CTA whose
 //     equal share of the axis holds the page's midpoint; the pages of a pair
 //     that fall to one CTA form a segment.  A private segment adds one
 //     partial slot (with G > 8 one per warp that gets a page, page i going
 //     to warp i mod 8); a shared segment adds one per candidate.
+//     Tensor-core runs (kind 2) stay off that axis: their (run, kv head)
+//     pairs' 4-page chunks are laid end to end and cut into equal ranges, one
+//     per CTA of the tensor-core launch (at most n_ctas); the chunks of a pair
+//     falling to one CTA form a segment, stored after the persistent CTAs'
+//     segments, with one slot per candidate.
 //  3. The slots of each (candidate, kv head) are numbered consecutively from
 //     slot_base.
 // Falls back to private runs when sharing would need more than slot_limit
 // slots; returns false if even those do not fit.
 bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks, int n_kv, int group, int n_ctas,
-                     size_t slot_limit, bool share, AttnWorkHost& w) {
+                     size_t slot_limit, int share, AttnWorkHost& w) {
+  w.tc_seg0 = 0;
+  w.n_tc = 0;
+  w.n_tc_ctas = 0;
+  w.tc_cta.clear();
   w.segs.clear();
   w.cta_seg.clear();
   w.pages.clear();
@@ -412,17 +841,22 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
         const auto& pg = group_pages[gi];
         const int page_off = static_cast<int>(w.pages.size());
         w.pages.insert(w.pages.end(), pg.begin(), pg.end());
-        for (size_t c0 = 0; c0 < c.size(); c0 += kConsumerWarps) {
+        // tensor-core tiles: as few as possible, with the candidates spread evenly over them
+        const size_t per = share == 2 ? static_cast<size_t>(kTcRows / group) : static_cast<size_t>(kConsumerWarps);
+        const size_t n_chunks = (c.size() + per - 1) / per;
+        for (size_t k = 0, c0 = 0; k < n_chunks; ++k) {
+          const size_t c1 = share == 2 ? c.size() * (k + 1) / n_chunks : std::min(c.size(), c0 + per);
           Run r;
-          r.kind = 1;
+          r.kind = share == 2 ? 2 : 1;
           r.cand = static_cast<int>(w.cands.size());
-          r.n_cands = static_cast<int>(std::min<size_t>(kConsumerWarps, c.size() - c0));
+          r.n_cands = static_cast<int>(c1 - c0);
           r.page_off = page_off;
           r.n_pages = static_cast<int>(pg.size());
           r.last_valid = 16;
           r.cost = kSharedCostPerCand * r.n_cands;
-          w.cands.insert(w.cands.end(), c.begin() + c0, c.begin() + c0 + r.n_cands);
+          w.cands.insert(w.cands.end(), c.begin() + c0, c.begin() + c1);
           runs.push_back(r);
+          c0 = c1;
         }
       }
     }
@@ -445,16 +879,20 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
     runs.push_back(r);
   }
   // ---- 2. cut the cost axis into C equal ranges (at least a stage of work each)
-  int64_t total = 0;
-  for (const Run& r : runs) total += static_cast<int64_t>(r.n_pages) * r.cost * n_kv;
-  if (total == 0) {   // no cached token anywhere: only the combine runs
-    w.cta_seg.push_back(0);
-    return true;
+  int64_t total = 0, tc_units = 0;
+  for (const Run& r : runs) {
+    if (r.kind == 2)
+      tc_units += static_cast<int64_t>(r.n_pages) * n_kv;
+    else
+      total += static_cast<int64_t>(r.n_pages) * r.cost * n_kv;
   }
-  const int C = static_cast<int>(std::max<int64_t>(1, std::min<int64_t>(n_ctas, total / (kPagesPerStage * kPrivateCost))));
+  const int C = total == 0 ? 0
+                           : static_cast<int>(std::max<int64_t>(
+                                 1, std::min<int64_t>(n_ctas, total / (kPagesPerStage * kPrivateCost))));
   std::vector<int> seg_cta;
   int64_t pos = 0;   // cost position of the current pair's first unit
   for (const Run& r : runs) {
+    if (r.kind == 2) continue;
     for (int g = 0; g < n_kv; ++g) {
       const int units = r.n_pages;
       const int64_t c = r.cost;
@@ -490,6 +928,52 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
       pos += static_cast<int64_t>(units) * c;
     }
   }
+  // tensor-core work: the (run, kv head) pairs' 4-page chunks laid end to end
+  // and cut into equal ranges, one per CTA of the tensor-core launch; a pair's
+  // chunks falling to one CTA form a segment (one slot per candidate)
+  w.tc_seg0 = static_cast<int>(w.segs.size());
+  w.tc_cta.clear();
+  w.n_tc_ctas = 0;
+  if (tc_units > 0) {
+    int64_t T = 0;
+    for (const Run& r : runs)
+      if (r.kind == 2) T += static_cast<int64_t>((r.n_pages + kTcChunkPages - 1) / kTcChunkPages) * n_kv;
+    const int Ct = static_cast<int>(std::min<int64_t>(n_ctas, T));
+    std::vector<int> tc_seg_cta;
+    int64_t at = 0;   // chunk position of the current pair's first chunk
+    for (const Run& r : runs) {
+      if (r.kind != 2) continue;
+      const int nch = (r.n_pages + kTcChunkPages - 1) / kTcChunkPages;
+      for (int g = 0; g < n_kv; ++g) {
+        for (int i = 0; i < nch;) {
+          const int k = static_cast<int>((at + i) * Ct / T);                 // CTA of chunk i
+          const int64_t next = ((k + 1) * T + Ct - 1) / Ct;                  // first chunk of CTA k + 1
+          const int e = static_cast<int>(std::min<int64_t>(nch, std::max<int64_t>(i + 1, next - at)));
+          AttnSeg sg;
+          sg.kind = 2;
+          sg.g = g;
+          sg.cand = r.cand;
+          sg.n_cands = r.n_cands;
+          sg.page_off = r.page_off + i * kTcChunkPages;
+          sg.n_pages = std::min(r.n_pages, e * kTcChunkPages) - i * kTcChunkPages;
+          sg.last_valid = 16;
+          sg.slot = static_cast<int>(w.slots.size());
+          for (int k2 = 0; k2 < r.n_cands; ++k2)
+            w.slots.push_back(w.nslots[static_cast<size_t>(w.cands[r.cand + k2]) * n_kv + g]++);
+          w.segs.push_back(sg);
+          tc_seg_cta.push_back(k);
+          i = e;
+        }
+        at += nch;
+      }
+    }
+    w.n_tc_ctas = Ct;
+    w.tc_cta.assign(Ct + 1, 0);
+    for (int k : tc_seg_cta) w.tc_cta[k + 1]++;
+    for (int k = 0; k < Ct; ++k) w.tc_cta[k + 1] += w.tc_cta[k];
+    for (int32_t& v : w.tc_cta) v += w.tc_seg0;   // indices into segs
+  }
+  w.n_tc = static_cast<int>(w.segs.size()) - w.tc_seg0;
   // ---- 3. slot numbering
   size_t next = 0;
   for (size_t cg = 0; cg < w.nslots.size(); ++cg) {
@@ -497,7 +981,7 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
     next += static_cast<size_t>(w.nslots[cg]);
   }
   if (next > slot_limit) {
-    if (share) return build_attn_work(bt, sl, n, max_blocks, n_kv, group, n_ctas, slot_limit, false, w);
+    if (share) return build_attn_work(bt, sl, n, max_blocks, n_kv, group, n_ctas, slot_limit, 0, w);
     return false;
   }
   w.n_slots = static_cast<int>(next);
@@ -524,6 +1008,7 @@ cudaError_t attention_configure() {
   if ((e = set_smem(attn_kernel<64, false>, AttnSmem<64>::kDynamic)) != cudaSuccess) return e;
   if ((e = set_smem(attn_kernel<64, true>, AttnSmem<64>::kDynamic)) != cudaSuccess) return e;
   if ((e = set_smem(attn_kernel<128, false>, AttnSmem<128>::kDynamic)) != cudaSuccess) return e;
+  if ((e = set_smem(attn_tc_kernel, TcSmem::kDynamic)) != cudaSuccess) return e;
   return set_smem(attn_kernel<128, true>, AttnSmem<128>::kDynamic);
 }
 
@@ -555,6 +1040,40 @@ cudaError_t launch_attention(const AttnShape& s, const AttnWork& wk, const CUten
                               part_o, part_ml, err, ts);
   return cudaLaunchKernelEx(&cfg, attn_kernel<64, false>, *tm_pool, page0, wk, q_hi, q_lo, s.n_q, s.n_kv, s.group,
                             part_o, part_ml, err, ts);
+}
+
+CUresult encode_pool_map_tc(PFN_cuTensorMapEncodeTiled_v12000 encode, CUtensorMap* map, const void* pool,
+                            int64_t page_units, int n_kv, int hd) {
+  const cuuint64_t row = static_cast<cuuint64_t>(hd) * 2;   // bytes per token row
+  cuuint64_t dims[5] = {64, 16, static_cast<cuuint64_t>(hd / 64), static_cast<cuuint64_t>(n_kv),
+                        static_cast<cuuint64_t>(page_units) * 2};
+  cuuint64_t strides[4] = {row, 128, 16 * row, static_cast<cuuint64_t>(n_kv) * 16 * row};
+  cuuint32_t box[5] = {64, 16, 1, 1, 1};
+  cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+  return encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(pool), dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
+cudaError_t launch_attention_tc(const AttnShape& s, const AttnWork& wk, const CUtensorMap* tm_pool_tc, int layer,
+                                const __nv_bfloat16* q_hi, const __nv_bfloat16* q_lo, float* part_o, float* part_ml,
+                                float margin, int* err, cudaStream_t stream, bool pdl, unsigned long long* ts,
+                                unsigned long long* prof) {
+  if (wk.n_tc == 0 || wk.n_tc_ctas == 0) return cudaSuccess;
+  if (s.hd != 128) return cudaErrorInvalidValue;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(wk.n_tc_ctas, 1, 1);
+  cfg.blockDim = dim3(kTcThreads, 1, 1);
+  cfg.dynamicSmemBytes = TcSmem::kDynamic;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  const int64_t page0 = static_cast<int64_t>(layer) * s.layer_pages;
+  return cudaLaunchKernelEx(&cfg, attn_tc_kernel, *tm_pool_tc, page0, wk, q_hi, q_lo, s.n_q, s.group, part_o, part_ml,
+                            margin, err, ts, prof);
 }
 
 cudaError_t launch_attn_combine(const AttnShape& s, const AttnWork& wk, int n, const float* part_o,

@@ -162,32 +162,39 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       tma_load_2d(st + kWTileBytes, &tmX, &full[s], (kt0 + i) * kBK, 0, pol_x);
       if (has_lo) tma_load_2d(st + kWTileBytes + x_bytes, &tmXlo, &full[s], (kt0 + i) * kBK, 0, pol_x);
     }
-  } else if (warp == 1 && lane == 0 && nk > 0) {
-    // ---------------- MMA issuer
+  } else if (warp == 1 && nk > 0) {
+    // ---------------- MMA issuer (the whole warp; one elected lane issues)
     // With the hi and lo activation tiles stored back to back (2 n_pad rows
     // under the same swizzle), one MMA of N = 2 n_pad reads each weight K
     // slice from shared memory once: columns [0, n_pad) accumulate W hi,
     // [n_pad, 2 n_pad) accumulate W lo, summed when the accumulator is read.
     // Beyond N = 256 the two halves take one MMA each into the same columns.
     const bool merged = has_lo && 2 * n_pad <= 256;
+    const bool two = has_lo && !merged;
     const uint32_t idesc = idesc_bf16_f32(kBM, merged ? 2 * n_pad : n_pad);
     for (int i = 0; i < nk; ++i) {
       const int s = i % stages;
       const uint32_t use = static_cast<uint32_t>(i / stages);
-      if (!mbar_wait(&full[s], use & 1u, err)) break;
-      if (i == 0) trace_event(ts, 1);   // first weight and activation tiles landed
+      if (!__all_sync(0xffffffffu, mbar_wait(&full[s], use & 1u, err))) break;
+      if (i == 0 && lane == 0) trace_event(ts, 1);   // first weight and activation tiles landed
       tc_fence_after();
-      const uint32_t a_base = smem_u32(smem + s * stage_bytes);
-      const uint32_t b_base = a_base + kWTileBytes;
+      const uint64_t a0 = desc_sw128(smem_u32(smem + s * stage_bytes));   // K step kk: + 2 kk (32 bytes)
+      const uint64_t b0 = a0 + (kWTileBytes >> 4);
+      const uint64_t l0 = b0 + static_cast<uint64_t>(x_bytes >> 4);
+      const uint32_t acc0 = i > 0 ? 1u : 0u;
+      if (two) {
 #pragma unroll
-      for (int kk = 0; kk < kBK / 16; ++kk) {
-        const uint64_t a_desc = desc_sw128(a_base + kk * 32);
-        umma_bf16(tmem, a_desc, desc_sw128(b_base + kk * 32), idesc, (i > 0 || kk > 0) ? 1u : 0u);
-        if (has_lo && !merged) umma_bf16(tmem, a_desc, desc_sw128(b_base + x_bytes + kk * 32), idesc, 1u);
+        for (int kk = 0; kk < kBK / 16; ++kk) {
+          umma_bf16_w(tmem, a0 + 2 * kk, b0 + 2 * kk, idesc, kk > 0 ? 1u : acc0);
+          umma_bf16_w(tmem, a0 + 2 * kk, l0 + 2 * kk, idesc, 1u);
+        }
+      } else {
+#pragma unroll
+        for (int kk = 0; kk < kBK / 16; ++kk) umma_bf16_w(tmem, a0 + 2 * kk, b0 + 2 * kk, idesc, kk > 0 ? 1u : acc0);
       }
-      umma_commit(&empty[s]);
+      umma_commit_w(&empty[s]);
     }
-    umma_commit(done);
+    umma_commit_w(done);
   }
   __syncwarp();
 

@@ -96,17 +96,30 @@ struct AttnWork {             // device arrays
   const int32_t* slot_base;   // [B][n_kv] first partial slot of each (candidate, kv head)
   const int32_t* nslots;      // [B][n_kv] number of partial slots
   int n_ctas;
+  int tc_seg0, n_tc;          // tensor-core segments (kind 2)
+  const int32_t* tc_cta;      // [n_tc_ctas + 1] first tensor-core segment of each CTA of attn_tc_kernel
+  int n_tc_ctas;
 };
 struct AttnWorkHost {
   std::vector<AttnSeg> segs;
   std::vector<int32_t> cta_seg, pages, cands, slots, slot_base, nslots;
   int n_slots = 0, n_ctas = 0;
+  int tc_seg0 = 0, n_tc = 0;   // tensor-core segments (kind 2): segs[tc_seg0, tc_seg0 + n_tc)
+  int n_tc_ctas = 0;
+  std::vector<int32_t> tc_cta;   // [n_tc_ctas + 1] first segment (index into segs) of each tensor-core CTA
 };
+// share: 0 every page scored per candidate; 1 shared pages scored once per run
+// of <= 8 candidates by the persistent kernel; 2 shared pages scored on the
+// tensor cores (head_dim 128 only), tiles of <= 128 / group candidates.
 bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks, int n_kv, int group, int n_ctas,
-                     size_t slot_limit, bool share, AttnWorkHost& w);
+                     size_t slot_limit, int share, AttnWorkHost& w);
 // partial slots a context sized for max_candidates provides (the planner falls
 // back to private runs, which always fit, when sharing needs more)
 size_t attn_slot_capacity(int max_candidates, int n_kv, int num_sms);
+// The same pool with a box of one 64-column sub-tile of one page, K or V
+// (2 KB): the tensor-core attention lays a 4-page chunk's tokens contiguously.
+CUresult encode_pool_map_tc(PFN_cuTensorMapEncodeTiled_v12000 encode, CUtensorMap* map, const void* pool,
+                            int64_t page_units, int n_kv, int hd);
 size_t attention_smem_bytes(int hd);
 cudaError_t attention_configure();
 // Inputs and outputs of the combine (attn_combine_kernel).
@@ -126,6 +139,18 @@ struct AttnMerge {
 cudaError_t launch_attention(const AttnShape& s, const AttnWork& wk, const CUtensorMap* tm_pool, int layer,
                              const __nv_bfloat16* q_hi, const __nv_bfloat16* q_lo, float* part_o, float* part_ml,
                              int* err, cudaStream_t stream, bool pdl, unsigned long long* ts = nullptr);
+// The kind-2 segments (wk.tc_seg0 .., wk.n_tc of them; head_dim 128): shared
+// pages scored on the tensor cores, one CTA per segment.  Writes the same
+// partial slots as launch_attention.  margin: the running row maximum moves
+// only when a chunk's scores exceed it by more than this (log2 units; 8 in
+// production, 0 to rescale on every new maximum).
+// Debug profile of the tensor-core attention (flag 32): an event log of CTA 0
+// ([8][128] clock64 stamps) followed by [n_SM][16] per-CTA accumulators.
+constexpr int kTcEventLog = 8 * 128;
+cudaError_t launch_attention_tc(const AttnShape& s, const AttnWork& wk, const CUtensorMap* tm_pool_tc, int layer,
+                                const __nv_bfloat16* q_hi, const __nv_bfloat16* q_lo, float* part_o, float* part_ml,
+                                float margin, int* err, cudaStream_t stream, bool pdl,
+                                unsigned long long* ts = nullptr, unsigned long long* prof = nullptr);
 // Merge every (candidate, kv head)'s slots (wk.slot_base / wk.nslots) of the
 // n candidates with the self entry into the attention output.
 cudaError_t launch_attn_combine(const AttnShape& s, const AttnWork& wk, int n, const float* part_o,

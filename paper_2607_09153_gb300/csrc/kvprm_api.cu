@@ -31,11 +31,13 @@ struct CallPlan {
 };
 
 struct GraphKey {
-  int n = -1, n_pad = -1, attn_ctas = -1, debug = -1, profile = -1, pdl = -1, trace = -1;
+  int n = -1, n_pad = -1, attn_ctas = -1, tc_ctas = -1, n_tc = -1, debug = -1, profile = -1, pdl = -1, trace = -1;
   const void* pool = nullptr;
   int64_t n_pages = -1;
   bool operator==(const GraphKey& o) const {
-    return n == o.n && n_pad == o.n_pad && attn_ctas == o.attn_ctas && debug == o.debug && profile == o.profile && pdl == o.pdl && trace == o.trace && pool == o.pool && n_pages == o.n_pages;
+    return n == o.n && n_pad == o.n_pad && attn_ctas == o.attn_ctas && tc_ctas == o.tc_ctas && n_tc == o.n_tc &&
+           debug == o.debug && profile == o.profile && pdl == o.pdl && trace == o.trace && pool == o.pool &&
+           n_pages == o.n_pages;
   }
 };
 
@@ -70,15 +72,17 @@ struct kvprm_ctx {
   int32_t* tables_d = nullptr;   // [Bmax] seq_lens, [Bmax][max_blocks] block table, then the attention work
   // attention work list: host plan of the current call and fixed offsets (ints) in tables_d / staging
   kvprm::AttnWorkHost work_host;
-  size_t off_segs = 0, off_cta = 0, off_pages = 0, off_cands = 0, off_slots = 0, off_base = 0, off_nslots = 0;
+  size_t off_segs = 0, off_cta = 0, off_pages = 0, off_cands = 0, off_slots = 0, off_base = 0, off_nslots = 0,
+         off_tc_cta = 0;
   size_t tables_ints = 0;
   size_t cap_segs = 0, cap_pages = 0, cap_cands = 0;
-  bool share_pages = true;
+  int share_mode = 2;   // sharing of pages referenced by several candidates (build_attn_work)
   float* rewards_d = nullptr;
   int* err_d = nullptr;
   float* dbg = nullptr;
   float *dbg_q = nullptr, *dbg_k = nullptr, *dbg_v = nullptr;
   float* dbg_h = nullptr;
+  unsigned long long* tc_prof = nullptr;   // tensor-core attention wait profile (debug flag 32)
   bf16* dummy_pool = nullptr;
   int debug_flags = 0;
   int last_n = 0;
@@ -95,7 +99,7 @@ struct kvprm_ctx {
   const void* pool_ptr = nullptr;
   int64_t pool_pages = -1;
   int64_t pool_units = -1;
-  CUtensorMap tm_pool{};
+  CUtensorMap tm_pool{}, tm_pool_tc{};
   // library-owned device pool for kvprm_score_host
   void* dev_pool = nullptr;
   size_t dev_pool_bytes = 0;
@@ -200,6 +204,7 @@ void free_ctx(kvprm_ctx* c) {
   cudaFree(c->dbg_k);
   cudaFree(c->dbg_v);
   cudaFree(c->dbg_h);
+  cudaFree(c->tc_prof);
   cudaFree(c->dummy_pool);
   cudaFree(c->dev_pool);
   if (c->staging) cudaFreeHost(c->staging);
@@ -255,11 +260,12 @@ int plan_work(kvprm_ctx* ctx, const int32_t* bt, const int32_t* sl, int32_t n) {
   const int mb = ctx->cfg.max_blocks_per_seq, nkv = ctx->cfg.n_kv_heads;
   auto fits = [&]() {
     return w.segs.size() <= ctx->cap_segs && w.pages.size() <= ctx->cap_pages && w.cands.size() <= ctx->cap_cands &&
-           w.slots.size() <= ctx->slot_cap && static_cast<size_t>(w.n_ctas) <= static_cast<size_t>(ctx->num_sms);
+           w.slots.size() <= ctx->slot_cap && static_cast<size_t>(w.n_ctas) <= static_cast<size_t>(ctx->num_sms) &&
+           static_cast<size_t>(w.n_tc_ctas) <= static_cast<size_t>(ctx->num_sms);
   };
-  bool ok = kvprm::build_attn_work(bt, sl, n, mb, nkv, ctx->md.n_q / nkv, ctx->num_sms, ctx->slot_cap, ctx->share_pages, w);
-  if (ok && !fits() && ctx->share_pages)
-    ok = kvprm::build_attn_work(bt, sl, n, mb, nkv, ctx->md.n_q / nkv, ctx->num_sms, ctx->slot_cap, false, w);
+  bool ok = kvprm::build_attn_work(bt, sl, n, mb, nkv, ctx->md.n_q / nkv, ctx->num_sms, ctx->slot_cap, ctx->share_mode, w);
+  if (ok && !fits() && ctx->share_mode)
+    ok = kvprm::build_attn_work(bt, sl, n, mb, nkv, ctx->md.n_q / nkv, ctx->num_sms, ctx->slot_cap, 0, w);
   if (!ok || !fits())
     return fail(ctx, KVPRM_ECAPACITY, "attention work list exceeds the context's capacity");
   return KVPRM_OK;
@@ -289,6 +295,7 @@ int upload_tables(kvprm_ctx* ctx, const int32_t* bt, const int32_t* sl, int32_t 
       {ctx->off_slots, w.slots.data(), w.slots.size()},
       {ctx->off_base, w.slot_base.data(), w.slot_base.size()},
       {ctx->off_nslots, w.nslots.data(), w.nslots.size()},
+      {ctx->off_tc_cta, w.tc_cta.data(), w.tc_cta.size()},
   };
   for (const Part& p : parts)
     if (p.ints) std::memcpy(S + p.off, p.src, sizeof(int32_t) * p.ints);
@@ -303,6 +310,10 @@ int upload_tables(kvprm_ctx* ctx, const int32_t* bt, const int32_t* sl, int32_t 
   return KVPRM_OK;
 }
 
+// Stale-maximum margin of the tensor-core attention (debug flag 16: rescale on
+// every new maximum, which exercises the rescale path).
+float tc_margin(const kvprm_ctx* ctx) { return (ctx->debug_flags & 16) ? 0.f : 8.f; }
+
 kvprm::AttnWork device_work(kvprm_ctx* ctx) {
   kvprm::AttnWork wk;
   wk.segs = reinterpret_cast<const kvprm::AttnSeg*>(ctx->tables_d + ctx->off_segs);
@@ -313,6 +324,10 @@ kvprm::AttnWork device_work(kvprm_ctx* ctx) {
   wk.slot_base = ctx->tables_d + ctx->off_base;
   wk.nslots = ctx->tables_d + ctx->off_nslots;
   wk.n_ctas = ctx->work_host.n_ctas;
+  wk.tc_seg0 = ctx->work_host.tc_seg0;
+  wk.n_tc = ctx->work_host.n_tc;
+  wk.tc_cta = ctx->tables_d + ctx->off_tc_cta;
+  wk.n_tc_ctas = ctx->work_host.n_tc_ctas;
   return wk;
 }
 
@@ -322,9 +337,11 @@ int ensure_pool_map(kvprm_ctx* ctx, const void* pool, int64_t n_pages, int layer
   if (2 * units >= (static_cast<int64_t>(1) << 31))
     return fail(ctx, KVPRM_EUNSUPPORTED, "pool of %lld layer pages exceeds the 2^30 tensor-map coordinate limit",
                 static_cast<long long>(units));
-  const CUresult r = kvprm::encode_pool_map(ctx->encode, &ctx->tm_pool, pool, units, ctx->cfg.n_kv_heads,
-                                            ctx->cfg.head_dim);
+  CUresult r = kvprm::encode_pool_map(ctx->encode, &ctx->tm_pool, pool, units, ctx->cfg.n_kv_heads,
+                                      ctx->cfg.head_dim);
   if (r != CUDA_SUCCESS) return fail(ctx, KVPRM_ECUDA, "cuTensorMapEncodeTiled(kv pool) failed with %d", (int)r);
+  r = kvprm::encode_pool_map_tc(ctx->encode, &ctx->tm_pool_tc, pool, units, ctx->cfg.n_kv_heads, ctx->cfg.head_dim);
+  if (r != CUDA_SUCCESS) return fail(ctx, KVPRM_ECUDA, "cuTensorMapEncodeTiled(kv pool, 2 KB box) failed with %d", (int)r);
   ctx->pool_ptr = pool;
   ctx->pool_pages = n_pages;
   ctx->pool_units = units;
@@ -472,6 +489,12 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
     float* dbg = (ctx->debug_flags & 1) ? ctx->dbg + static_cast<size_t>(l) * n * m.n_q * m.hd : nullptr;
     const kvprm::AttnMerge mg{ctx->q, ctx->kself, ctx->vself, O.hi, O.lo, nullptr, dbg};
     const kvprm::AttnWork wk = device_work(ctx);
+    if (wk.n_tc > 0)   // shared pages on the tensor cores
+      LAUNCH(KVPRM_PROF_ATTN,
+             kvprm::launch_attention_tc(ctx->as, wk, &ctx->tm_pool_tc, l, ctx->qhi, ctx->qlo, ctx->apart_o,
+                                        ctx->apart_ml, tc_margin(ctx), ctx->err_d, st, pdl, TS,
+                                        (ctx->debug_flags & 32) ? ctx->tc_prof : nullptr),
+             "attention_tc");
     LAUNCH(KVPRM_PROF_ATTN,
            kvprm::launch_attention(ctx->as, wk, &ctx->tm_pool, l, ctx->qhi, ctx->qlo, ctx->apart_o, ctx->apart_ml,
                                    ctx->err_d, st, pdl, TS),
@@ -570,6 +593,8 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   key.n = n;
   key.n_pad = P.n_pad;
   key.attn_ctas = P.attn_ctas;
+  key.tc_ctas = ctx->work_host.n_tc_ctas;
+  key.n_tc = ctx->work_host.n_tc > 0 ? 1 : 0;
   key.debug = ctx->debug_flags;
   key.profile = ctx->profile ? 1 : 0;
   key.pdl = ctx->use_pdl ? 1 : 0;
@@ -747,7 +772,7 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
     // private runs need at most Bmax * n_kv + n_ctas segments, Bmax * max_blocks
     // pages and no candidate lists; sharing plans beyond these fall back to them
     const size_t bkv = static_cast<size_t>(Bmax) * m.n_kv;
-    ctx->cap_segs = 4 * bkv + 2 * static_cast<size_t>(ctx->num_sms);
+    ctx->cap_segs = 8 * bkv + 4 * static_cast<size_t>(ctx->num_sms);
     ctx->cap_pages = static_cast<size_t>(Bmax) * c.max_blocks_per_seq;
     ctx->cap_cands = static_cast<size_t>(Bmax) * c.max_blocks_per_seq;
     ctx->off_segs = al8(tbl);
@@ -757,7 +782,8 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
     ctx->off_slots = al8(ctx->off_cands + ctx->cap_cands);
     ctx->off_base = al8(ctx->off_slots + ctx->slot_cap);
     ctx->off_nslots = al8(ctx->off_base + bkv);
-    ctx->tables_ints = al8(ctx->off_nslots + bkv);
+    ctx->off_tc_cta = al8(ctx->off_nslots + bkv);
+    ctx->tables_ints = al8(ctx->off_tc_cta + ctx->num_sms + 1);
   }
   CREATE_CK(dalloc(ctx, &ctx->tables_d, ctx->tables_ints, "tables and attention work"));
   CREATE_CK(dalloc(ctx, &ctx->rewards_d, static_cast<size_t>(Bmax), "rewards"));
@@ -778,7 +804,8 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   CREATE_CK(cu(cudaStreamCreateWithFlags(&ctx->cap_stream, cudaStreamNonBlocking), "cudaStreamCreate"));
   ctx->use_graph = !env_off("KVPRM_NO_GRAPH");
   ctx->use_pdl = !env_off("KVPRM_NO_PDL");
-  ctx->share_pages = !env_off("KVPRM_NO_SHARING");
+  // shared pages: on the tensor cores at head_dim 128, else one warp per candidate
+  ctx->share_mode = env_off("KVPRM_NO_SHARING") ? 0 : ((c.head_dim == 128 && !env_off("KVPRM_NO_TC_SHARING")) ? 2 : 1);
   CREATE_CK(cu(cudaDeviceSynchronize(), "cudaDeviceSynchronize(create)"));
 #undef CREATE_CK
   *out = ctx;
@@ -883,6 +910,11 @@ int kvprm_attention(kvprm_ctx* ctx, const void* kv_layer, int64_t n_pages, const
   const kvprm::AttnMerge mg{static_cast<const float*>(q), static_cast<const float*>(k_self),
                             static_cast<const float*>(v_self), ctx->ohi, ctx->olo, out, nullptr};
   const kvprm::AttnWork wk = device_work(ctx);
+  if (wk.n_tc > 0)
+    LAUNCH(KVPRM_PROF_ATTN,
+           kvprm::launch_attention_tc(as, wk, &ctx->tm_pool_tc, 0, Q.hi, Q.lo, ctx->apart_o, ctx->apart_ml,
+                                      tc_margin(ctx), ctx->err_d, st, false),
+           "attention_tc");
   LAUNCH(KVPRM_PROF_ATTN,
          kvprm::launch_attention(as, wk, &ctx->tm_pool, 0, Q.hi, Q.lo, ctx->apart_o, ctx->apart_ml, ctx->err_d, st,
                                  false),
@@ -957,6 +989,11 @@ int kvprm_set_debug(kvprm_ctx* ctx, int flags) {
     int rc = dalloc(ctx, &ctx->dbg_h, NB * ctx->md.d, "debug h");
     if (rc) return rc;
   }
+  if ((flags & 32) && !ctx->tc_prof) {
+    int rc = dalloc(ctx, &ctx->tc_prof, kvprm::kTcEventLog + static_cast<size_t>(ctx->num_sms) * 16,
+                    "tensor-core attention profile");
+    if (rc) return rc;
+  }
   ctx->debug_flags = flags;
   return KVPRM_OK;
 }
@@ -974,6 +1011,11 @@ int kvprm_debug_layers(kvprm_ctx* ctx, int which, void* d_out) {
     if (!(ctx->debug_flags & 4)) return fail(ctx, KVPRM_EINVAL, "hidden-state capture (flag 4) is not enabled");
     src = ctx->dbg_h;
     bytes = L * ctx->md.d * 4;
+  } else if (which == 5) {
+    if (!(ctx->debug_flags & 32) || !ctx->tc_prof)
+      return fail(ctx, KVPRM_EINVAL, "tensor-core attention profile (flag 32) is not enabled");
+    src = ctx->tc_prof;
+    bytes = (kvprm::kTcEventLog + static_cast<size_t>(ctx->num_sms) * 16) * sizeof(unsigned long long);
   } else {
     return fail(ctx, KVPRM_EINVAL, "unknown capture %d", which);
   }
@@ -1021,7 +1063,7 @@ int kvprm_plan_attention(const int32_t* block_table, int32_t max_blocks_per_seq,
       return KVPRM_EINVAL;
   kvprm::AttnWorkHost w;
   if (!kvprm::build_attn_work(block_table, seq_lens, n_candidates, max_blocks_per_seq, n_kv_heads, group, n_ctas,
-                              SIZE_MAX, share != 0, w))
+                              SIZE_MAX, share < 0 ? 0 : (share > 2 ? 2 : share), w))
     return KVPRM_ECAPACITY;
   plan->n_segs = static_cast<int32_t>(w.segs.size());
   plan->n_ctas = w.n_ctas;
@@ -1029,12 +1071,13 @@ int kvprm_plan_attention(const int32_t* block_table, int32_t max_blocks_per_seq,
   plan->n_cands = static_cast<int32_t>(w.cands.size());
   plan->n_slot_refs = static_cast<int32_t>(w.slots.size());
   plan->n_slots = w.n_slots;
+  plan->n_tc_ctas = w.n_tc_ctas;
   constexpr size_t kSegInts = sizeof(kvprm::AttnSeg) / sizeof(int32_t);
   static_assert(kSegInts == 8, "segment layout");
   auto fits = [](const int32_t* p, int64_t cap, size_t need) { return need == 0 || (p && cap >= static_cast<int64_t>(need)); };
   if (!fits(plan->segs, plan->segs_cap, w.segs.size()) || !fits(plan->cta_seg, plan->cta_cap, w.cta_seg.size()) ||
       !fits(plan->pages, plan->pages_cap, w.pages.size()) || !fits(plan->cands, plan->cands_cap, w.cands.size()) ||
-      !fits(plan->slots, plan->slots_cap, w.slots.size()) ||
+      !fits(plan->slots, plan->slots_cap, w.slots.size()) || !fits(plan->tc_cta, plan->tc_cta_cap, w.tc_cta.size()) ||
       (!w.slot_base.empty() && (!plan->slot_base || !plan->nslots)))
     return KVPRM_ECAPACITY;
   if (!w.segs.empty()) std::memcpy(plan->segs, w.segs.data(), sizeof(kvprm::AttnSeg) * w.segs.size());
@@ -1042,6 +1085,7 @@ int kvprm_plan_attention(const int32_t* block_table, int32_t max_blocks_per_seq,
   if (!w.pages.empty()) std::memcpy(plan->pages, w.pages.data(), sizeof(int32_t) * w.pages.size());
   if (!w.cands.empty()) std::memcpy(plan->cands, w.cands.data(), sizeof(int32_t) * w.cands.size());
   if (!w.slots.empty()) std::memcpy(plan->slots, w.slots.data(), sizeof(int32_t) * w.slots.size());
+  if (!w.tc_cta.empty()) std::memcpy(plan->tc_cta, w.tc_cta.data(), sizeof(int32_t) * w.tc_cta.size());
   if (!w.slot_base.empty()) {
     std::memcpy(plan->slot_base, w.slot_base.data(), sizeof(int32_t) * w.slot_base.size());
     std::memcpy(plan->nslots, w.nslots.data(), sizeof(int32_t) * w.nslots.size());

@@ -189,6 +189,10 @@ extern "C" int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, co
   wk.slot_base = reinterpret_cast<const int32_t*>(scratch + cv.base);
   wk.nslots = reinterpret_cast<const int32_t*>(scratch + cv.nslots);
   wk.n_ctas = work.n_ctas;
+  wk.tc_seg0 = work.tc_seg0;
+  wk.n_tc = work.n_tc;   // 0: this entry point schedules shared pages on the persistent kernel only
+  wk.tc_cta = nullptr;
+  wk.n_tc_ctas = 0;
 
   // the error word must start at zero; everything else is written before it is read
   if (cudaMemsetAsync(err, 0, sizeof(int), st) != cudaSuccess) return KVPRM_ECUDA;

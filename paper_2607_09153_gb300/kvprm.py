@@ -50,7 +50,8 @@ class KvprmAttnPlan(ctypes.Structure):
                 ("pages", ctypes.POINTER(ctypes.c_int32)), ("pages_cap", ctypes.c_int64),
                 ("cands", ctypes.POINTER(ctypes.c_int32)), ("cands_cap", ctypes.c_int64),
                 ("slots", ctypes.POINTER(ctypes.c_int32)), ("slots_cap", ctypes.c_int64),
-                ("slot_base", ctypes.POINTER(ctypes.c_int32)), ("nslots", ctypes.POINTER(ctypes.c_int32))]
+                ("slot_base", ctypes.POINTER(ctypes.c_int32)), ("nslots", ctypes.POINTER(ctypes.c_int32)),
+                ("n_tc_ctas", ctypes.c_int32), ("tc_cta", ctypes.POINTER(ctypes.c_int32)), ("tc_cta_cap", ctypes.c_int64)]
 
 
 _lib = None
@@ -176,36 +177,41 @@ def kvprm_attention_noalloc(kv_layer_ptr: int, n_pages: int, block_table, seq_le
         raise KvprmError(rc, "kvprm_attention_noalloc failed")
 
 
-def kvprm_plan_attention(block_table, seq_lens, n_kv_heads: int, group: int, n_ctas: int, share: bool = True) -> dict:
+def kvprm_plan_attention(block_table, seq_lens, n_kv_heads: int, group: int, n_ctas: int, share: int = 1) -> dict:
     """The attention schedule of a call (host only): dict of numpy arrays
-    segs [n_segs][8], cta_seg, pages, cands, slots, slot_base, nslots."""
+    segs [n_segs][8], cta_seg, pages, cands, slots, slot_base, nslots.  share: 0 none,
+    1 shared runs on the persistent CTAs, 2 shared pages on the tensor cores."""
     bt, sl = _i32(block_table), _i32(seq_lens)
     n = len(sl)
     mb = bt.shape[1] if bt.ndim == 2 and bt.shape[1] > 0 else 1
     bt = bt.reshape(max(n, 1) if n else 1, -1) if n else np.zeros((1, 1), np.int32)
     plan = KvprmAttnPlan()
     rc = lib().kvprm_plan_attention(_p(bt, ctypes.c_int32), mb, _p(sl, ctypes.c_int32), n, n_kv_heads, group, n_ctas,
-                                    int(bool(share)), ctypes.byref(plan))
+                                    int(share), ctypes.byref(plan))
     if rc not in (KVPRM_OK, KVPRM_ECAPACITY):
         raise KvprmError(rc, "kvprm_plan_attention failed")
     bufs = {"segs": np.zeros((max(plan.n_segs, 1), 8), np.int32), "cta_seg": np.zeros(max(plan.n_ctas + 1, 1), np.int32),
             "pages": np.zeros(max(plan.n_pages, 1), np.int32), "cands": np.zeros(max(plan.n_cands, 1), np.int32),
             "slots": np.zeros(max(plan.n_slot_refs, 1), np.int32),
-            "slot_base": np.zeros(max(n * n_kv_heads, 1), np.int32), "nslots": np.zeros(max(n * n_kv_heads, 1), np.int32)}
+            "slot_base": np.zeros(max(n * n_kv_heads, 1), np.int32), "nslots": np.zeros(max(n * n_kv_heads, 1), np.int32),
+            "tc_cta": np.zeros(max(plan.n_tc_ctas + 1, 1), np.int32)}
     plan.segs, plan.segs_cap = _p(bufs["segs"], ctypes.c_int32), bufs["segs"].shape[0]
     plan.cta_seg, plan.cta_cap = _p(bufs["cta_seg"], ctypes.c_int32), bufs["cta_seg"].size
     plan.pages, plan.pages_cap = _p(bufs["pages"], ctypes.c_int32), bufs["pages"].size
     plan.cands, plan.cands_cap = _p(bufs["cands"], ctypes.c_int32), bufs["cands"].size
     plan.slots, plan.slots_cap = _p(bufs["slots"], ctypes.c_int32), bufs["slots"].size
     plan.slot_base, plan.nslots = _p(bufs["slot_base"], ctypes.c_int32), _p(bufs["nslots"], ctypes.c_int32)
+    plan.tc_cta, plan.tc_cta_cap = _p(bufs["tc_cta"], ctypes.c_int32), bufs["tc_cta"].size
     rc = lib().kvprm_plan_attention(_p(bt, ctypes.c_int32), mb, _p(sl, ctypes.c_int32), n, n_kv_heads, group, n_ctas,
-                                    int(bool(share)), ctypes.byref(plan))
+                                    int(share), ctypes.byref(plan))
     if rc != KVPRM_OK:
         raise KvprmError(rc, "kvprm_plan_attention failed")
     return {"segs": bufs["segs"][:plan.n_segs], "cta_seg": bufs["cta_seg"][:plan.n_ctas + 1] if plan.n_ctas else
             np.zeros(1, np.int32), "pages": bufs["pages"][:plan.n_pages], "cands": bufs["cands"][:plan.n_cands],
             "slots": bufs["slots"][:plan.n_slot_refs], "slot_base": bufs["slot_base"][:n * n_kv_heads],
-            "nslots": bufs["nslots"][:n * n_kv_heads], "n_ctas": plan.n_ctas, "n_slots": plan.n_slots}
+            "nslots": bufs["nslots"][:n * n_kv_heads], "n_ctas": plan.n_ctas, "n_slots": plan.n_slots,
+            "tc_cta": bufs["tc_cta"][:plan.n_tc_ctas + 1] if plan.n_tc_ctas else np.zeros(1, np.int32),
+            "n_tc_ctas": plan.n_tc_ctas}
 
 
 def kvprm_set_debug(ctx, flags: int) -> None:

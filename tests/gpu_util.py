@@ -30,15 +30,16 @@ def make_scorer(dev: ks.DeviceInputs, max_candidates: int, max_blocks: int):
                   a.rope_base, a.rms_eps)
 
 
-def run_gpu(w: ks.Workload, tables: ks.Tables, debug: bool = True, dev=None, scorer=None):
-    """Score every candidate on the GPU; returns (rewards [B], attn [N_L][B][nq*hd] or None)."""
+def run_gpu(w: ks.Workload, tables: ks.Tables, debug: bool = True, dev=None, scorer=None, extra_flags: int = 0):
+    """Score every candidate on the GPU; returns (rewards [B], attn [N_L][B][nq*hd] or None).
+    extra_flags: further kvprm_set_debug bits (16: rescale on every new attention row maximum)."""
     torch = require_gpu()
     import paper_2607_09153_gb300 as kp
     dev = dev or ks.DeviceInputs(w, tables)
     sc = scorer or make_scorer(dev, max(1, w.n_candidates), w.max_blocks)
     a = w.arch
-    if debug:
-        kp.kvprm_set_debug(sc.ctx, 1)
+    if debug or extra_flags:
+        kp.kvprm_set_debug(sc.ctx, (1 if debug else 0) | extra_flags)
     r = sc.score(dev.pool, w.block_table, w.seq_lens)
     attn = None
     if debug:

@@ -18,6 +18,7 @@ PRIVATE_COST, SHARED_COST_PER_CAND = 4, 2   # the planner's per-page cost model
 
 
 def check_plan(bt, sl, n_kv, group, n_ctas, share):
+    share = int(share)
     bt = np.asarray(bt, np.int32)
     sl = np.asarray(sl, np.int32)
     n = len(sl)
@@ -34,7 +35,8 @@ def check_plan(bt, sl, n_kv, group, n_ctas, share):
     used = collections.defaultdict(list)   # (b, g) -> slots
     assert p["n_ctas"] <= n_ctas
     if p["n_ctas"]:
-        assert cta[0] == 0 and cta[-1] == len(segs) and np.all(np.diff(cta) >= 0)
+        assert cta[0] == 0 and np.all(np.diff(cta) >= 0)
+        assert cta[-1] == len(segs) if share != 2 else cta[-1] <= len(segs)
     cost = np.zeros(max(p["n_ctas"], 1))
     for k in range(p["n_ctas"]):
         for s in segs[cta[k]:cta[k + 1]]:
@@ -47,7 +49,7 @@ def check_plan(bt, sl, n_kv, group, n_ctas, share):
                 slots = [[slot + i for i in range(k_slots)]]
                 cost[k] += PRIVATE_COST * npg
             else:
-                assert share and 1 <= nc <= 8 and last == 16
+                assert kind == 1 and share == 1 and 1 <= nc <= 8 and last == 16
                 cands = [int(x) for x in p["cands"][c:c + nc]]
                 slots = [[int(x)] for x in p["slots"][slot:slot + nc]]
                 cost[k] += SHARED_COST_PER_CAND * nc * npg
@@ -55,6 +57,16 @@ def check_plan(bt, sl, n_kv, group, n_ctas, share):
                 used[(b, g)] += sls
                 for i, pg in enumerate(pages):
                     got[(b, g, int(pg), last if i == npg - 1 else 16)] += 1
+    # tensor-core segments (share = 2) follow the persistent CTAs' segments
+    tc0 = int(cta[-1]) if p["n_ctas"] else 0
+    for s in segs[tc0:]:
+        kind, g, c, nc, off, npg, last, slot = (int(x) for x in s)
+        assert kind == 2 and share == 2 and 0 <= g < n_kv and npg >= 1 and last == 16
+        assert 1 <= nc <= 128 // group, "a tile holds at most 128 query rows"
+        for b, sl_ in zip(p["cands"][c:c + nc], p["slots"][slot:slot + nc]):
+            used[(int(b), g)].append(int(sl_))
+            for pg in p["pages"][off:off + npg]:
+                got[(int(b), g, int(pg), 16)] += 1
     assert got == want, "every cached token scored exactly once per kv head"
     for b in range(n):
         for g in range(n_kv):
@@ -63,20 +75,35 @@ def check_plan(bt, sl, n_kv, group, n_ctas, share):
     assert int(p["nslots"].sum()) == p["n_slots"]
     if p["n_ctas"] > 1:
         total = cost.sum()
-        unit = PRIVATE_COST if not share else max(PRIVATE_COST, SHARED_COST_PER_CAND * 8)
+        unit = PRIVATE_COST if share != 1 else max(PRIVATE_COST, SHARED_COST_PER_CAND * 8)
         assert np.abs(cost - total / p["n_ctas"]).max() <= unit, "equal CTA shares up to one page"
     return p
 
 
 @pytest.mark.parametrize("name", ["tiny", "qwen1p5b_b16_l2048", "beam7b_b64_p4096_s512", "long8b_b8_l32768",
                                   "mcts7b_b256_d4"])
-@pytest.mark.parametrize("share", [True, False])
+@pytest.mark.parametrize("share", [0, 1, 2])
 def test_workload_plans(name, share):
     w = ks.make_workload(name)
     a = w.arch
     p = check_plan(w.block_table, w.seq_lens, a.n_kv_heads, a.n_q_heads // a.n_kv_heads, 152, share)
     if not share:
         assert (p["segs"][:, 0] == 0).all()
+    if share == 2 and name in ("beam7b_b64_p4096_s512", "mcts7b_b256_d4"):
+        tc = p["segs"][p["segs"][:, 0] == 2]
+        # at most one tensor-core CTA per SM, equal chunk counts up to one, every kind-2 segment owned once;
+        # within a (tile, kv head) every piece but the last is whole 4-page chunks
+        tcc, nt = p["tc_cta"], p["n_tc_ctas"]
+        assert 1 <= nt <= 152 and tcc[0] == len(p["segs"]) - len(tc) and tcc[-1] == len(p["segs"])
+        per_cta = [sum((int(x[5]) + 3) // 4 for x in p["segs"][tcc[k]:tcc[k + 1]]) for k in range(nt)]
+        assert max(per_cta) - min(per_cta) <= 1
+        parts = collections.defaultdict(list)
+        for s in tc:
+            parts[(int(s[2]), int(s[1]))].append((int(s[4]), int(s[5])))
+        for lst in parts.values():
+            lst.sort()
+            assert all(npg % 4 == 0 for _, npg in lst[:-1])
+            assert all(o0 + n0 == o1 for (o0, n0), (o1, _) in zip(lst, lst[1:])), "parts tile the run's pages"
 
 
 def test_shared_prefix_is_read_once_per_chunk():
@@ -94,6 +121,23 @@ def test_shared_prefix_is_read_once_per_chunk():
     for s in shared:
         per_head[int(s[1])] += int(s[5])
     assert per_head == {0: 3 * pre, 1: 3 * pre}
+
+
+def test_shared_prefix_tensor_core_tiles():
+    # 40 candidates share a 33-page prefix (G = 7: tiles of <= 18 candidates -> 3 tiles of 13-14)
+    n, pre, own = 40, 33, 2
+    bt = np.zeros((n, pre + own), np.int32)
+    for b in range(n):
+        bt[b, :pre] = np.arange(pre)
+        bt[b, pre:] = pre + own * b + np.arange(own)
+    sl = np.full(n, 16 * (pre + own) - 3, np.int32)
+    p = check_plan(bt, sl, 2, 7, 24, 2)
+    tc = p["segs"][p["segs"][:, 0] == 2]
+    assert sorted(set(tc[:, 3].tolist())) == [13, 14], "candidates spread evenly over the fewest tiles"
+    per_tile_head = collections.Counter()
+    for s in tc:
+        per_tile_head[(int(s[2]), int(s[1]))] += int(s[5])
+    assert len(per_tile_head) == 3 * 2 and set(per_tile_head.values()) == {pre}, "each tile reads the prefix once"
 
 
 def test_repeated_page_in_one_candidate_stays_private():
@@ -114,11 +158,12 @@ def test_partial_last_page_is_never_shared():
 
 @pytest.mark.parametrize("lens", [[0], [0, 0, 0], [1], [16], [17], [0, 1, 15, 16, 17, 31, 33, 100, 257, 1000]])
 @pytest.mark.parametrize("n_ctas", [1, 3, 152])
-def test_edges(lens, n_ctas):
+@pytest.mark.parametrize("share", [1, 2])
+def test_edges(lens, n_ctas, share):
     n = len(lens)
     mb = max(1, max((L + 15) // 16 for L in lens))
     bt = np.arange(n * mb, dtype=np.int32).reshape(n, mb)
-    p = check_plan(bt, lens, 2, 3, n_ctas, True)
+    p = check_plan(bt, lens, 2, 3, n_ctas, share)
     for b, L in enumerate(lens):
         if L == 0:
             assert (p["nslots"][b * 2:(b + 1) * 2] == 0).all(), "an empty cache has no partial: self entry only"

@@ -41,6 +41,37 @@ def test_shared_pages_tree():
     compare(w, t, gpu_rewards=r, gpu_attn=attn, label="tree")
 
 
+# head_dim 128 with G = 7: pages shared by several candidates are scored on the
+# tensor cores (tiles of <= 18 candidates x 7 heads) instead of per warp
+ARCH_G7 = ks.Arch(2, 256, 14, 2, 128, 512)
+
+
+@pytest.mark.parametrize("B,prefix,suffix", [(40, 528, 37), (3, 64, 1), (18, 16, 5), (20, 530, 40)])
+def test_tc_shared_prefix(B, prefix, suffix):
+    t = ks.Tables.make(0.2)
+    w = ks.shared_prefix("tc_prefix", ARCH_G7, 31 + B, B, prefix, suffix, gain_std=0.2)
+    r, attn, _, _ = run_gpu(w, t)
+    compare(w, t, gpu_rewards=r, gpu_attn=attn, label=f"tensor-core prefix B={B} prefix={prefix}")
+
+
+@pytest.mark.parametrize("rescale_always", [False, True])
+def test_tc_long_prefix(rescale_always):
+    # 36 candidates (two tiles) share 11,200 tokens: every tensor-core part spans >= 5
+    # chunks, so K/V stages are reused and S buffers alternate; flag 16 forces the
+    # running-maximum rescale of O in TMEM on every new maximum
+    t = ks.Tables.make(0.2)
+    w = ks.shared_prefix("tc_long", ARCH_G7, 37, 36, 11200, 23, gain_std=0.2)
+    r, attn, _, _ = run_gpu(w, t, extra_flags=16 if rescale_always else 0)
+    compare(w, t, gpu_rewards=r, gpu_attn=attn, label=f"tensor-core long prefix rescale_always={rescale_always}")
+
+
+def test_tc_tree():
+    t = ks.Tables.make(0.2)
+    w = ks.mcts_tree("tc_tree", ARCH_G7, 41, branching=3, depth=3, lo=5, hi=90, gain_std=0.2)
+    r, attn, _, _ = run_gpu(w, t)
+    compare(w, t, gpu_rewards=r, gpu_attn=attn, label="tensor-core tree")
+
+
 @pytest.mark.parametrize("B", [1, 17, 40])
 def test_batch_padding(B):
     t = ks.Tables.make(0.2)
