@@ -288,7 +288,8 @@ KVPRM_API int kvprm_check_device(kvprm_ctx* ctx);
  * the scoring stream while enabled (one event pair per launch; programmatic
  * launch overlap is switched off meanwhile, so each launch is timed alone).
  * Classes: 0..3 the QKV, O, gate/up and down projections, 4 paged attention
- * (split-K), 5 attention combine, 6 fused norm / RoPE / SiLU / head kernels.
+ * (split-K, CUDA cores), 5 attention combine, 6 fused norm / RoPE / SiLU /
+ * head kernels, 7 paged attention of shared pages on the tensor cores.
  * Profiled calls synchronise the stream.  kvprm_get_profile returns per class
  * the launch count and total milliseconds since profiling was enabled. */
 enum {
@@ -299,7 +300,8 @@ enum {
   KVPRM_PROF_ATTN = 4,
   KVPRM_PROF_COMBINE = 5,
   KVPRM_PROF_FUSED = 6,
-  KVPRM_PROF_N = 7
+  KVPRM_PROF_ATTN_TC = 7,
+  KVPRM_PROF_N = 8
 };
 KVPRM_API int kvprm_set_profile(kvprm_ctx* ctx, int enable);
 

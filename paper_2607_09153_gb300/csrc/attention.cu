@@ -290,8 +290,9 @@ __global__ void __launch_bounds__(CombineShape<HD, ROWS>::W * 32) attn_combine_k
 // are read at an out-of-range page and arrive as zeros) through a 6-stage
 // ring released by the S MMAs that read it; warp 10 streams V the same way
 // through a ring released by the O MMAs, so neither waits for the other.
-// Warp 1 issues the MMAs (S two chunks ahead of O within a segment, four S/P
-// buffers); warps 2..9 run the softmax, two threads per query row (each 32 of
+// Warp 1 issues the S MMAs (up to four chunks ahead: four S/P buffers) and
+// warp 11 the O MMAs, so neither stream waits behind the other's bookkeeping;
+// warps 2..9 run the softmax, two threads per query row (each 32 of
 // a chunk's 64 columns; the half maxima meet in shared memory) and, at each
 // segment's end, write every live row's (m, l, O) into its candidate's
 // partial slot.
@@ -306,7 +307,8 @@ struct TcSmem {
   static constexpr size_t kDynamic = kEnd + 1024;
 };
 static_assert(TcSmem::kDynamic <= 227 * 1024, "tensor-core attention shared memory exceeds the per-block limit");
-constexpr int kTcThreads = 352;   // warp 0 key TMA, 1 MMA, 2..9 softmax (two threads per row), 10 value TMA
+constexpr int kTcThreads = 384;   // warp 0 key TMA, 1 S MMAs, 2..9 softmax (two threads per row), 10 value TMA,
+                                  // 11 O MMAs
 constexpr uint32_t kTcTmemCols = 512;
 // TMEM columns: four S/P buffers at 0, 64, 128, 192; O at 256..383; Q hi at 384..447, Q lo at 448..511.
 // With four S buffers the MMA warp issues S two chunks ahead of the softmax without waiting for
@@ -419,8 +421,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(
       for (uint32_t v = u > static_cast<uint32_t>(SM::kStages) ? u - SM::kStages : 0; v < u; ++v)   // all landed
         if (!mbar_wait(&full[v % SM::kStages], (v / SM::kStages) & 1u, err)) break;
     }
-  } else if (warp == 1) {
-    // ------------------------------------------------ MMA issuer (the whole warp; one elected lane issues)
+  } else if (warp == 1 || warp == 11) {
+    // ------------------------------------------------ MMA issuers: warp 1 the S MMAs, warp 11 the O MMAs
+    // (each the whole warp; one elected lane issues, and its commits track only its own MMAs)
     // O MMAs take V as an MN-major B operand (instruction descriptor bit 16)
     const uint32_t id_s = idesc_bf16_f32(128, 64), id_o = idesc_bf16_f32(128, 128) | (1u << 16);
     auto wait_all = [&](uint64_t* bar, uint32_t parity) { return __all_sync(0xffffffffu, mbar_wait(bar, parity, err)); };
@@ -477,12 +480,12 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(
     bool ok = true;
     for (int si = seg0; si < seg1 && ok; ++si, ++k) {
       const int nch = chunks(wk.segs[si]);
-      ok = wait_all(q_ready, k & 1u) && (k == 0 || wait_all(o_free, (k - 1) & 1u));
-      if (ok) ok = issue_s(u);
-      if (ok && nch > 1) ok = issue_s(u + 1);
-      for (int c = 0; c < nch && ok; ++c, ++u) {   // S two chunks ahead of O
-        if (c + 2 < nch) ok = issue_s(u + 2);
-        if (ok) ok = issue_o(u, c == 0);
+      if (warp == 1) {   // S of a segment once its Q is in TMEM; up to four chunks ahead of O
+        ok = wait_all(q_ready, k & 1u);
+        for (int c = 0; c < nch && ok; ++c, ++u) ok = issue_s(u);
+      } else {           // O of a segment once the previous segment's O is read out
+        ok = k == 0 || wait_all(o_free, (k - 1) & 1u);
+        for (int c = 0; c < nch && ok; ++c, ++u) ok = issue_o(u, c == 0);
       }
     }
   } else if (warp < 10) {

@@ -490,7 +490,7 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
     const kvprm::AttnMerge mg{ctx->q, ctx->kself, ctx->vself, O.hi, O.lo, nullptr, dbg};
     const kvprm::AttnWork wk = device_work(ctx);
     if (wk.n_tc > 0)   // shared pages on the tensor cores
-      LAUNCH(KVPRM_PROF_ATTN,
+      LAUNCH(KVPRM_PROF_ATTN_TC,
              kvprm::launch_attention_tc(ctx->as, wk, &ctx->tm_pool_tc, l, ctx->qhi, ctx->qlo, ctx->apart_o,
                                         ctx->apart_ml, tc_margin(ctx), ctx->err_d, st, pdl, TS,
                                         (ctx->debug_flags & 32) ? ctx->tc_prof : nullptr),
@@ -911,7 +911,7 @@ int kvprm_attention(kvprm_ctx* ctx, const void* kv_layer, int64_t n_pages, const
                             static_cast<const float*>(v_self), ctx->ohi, ctx->olo, out, nullptr};
   const kvprm::AttnWork wk = device_work(ctx);
   if (wk.n_tc > 0)
-    LAUNCH(KVPRM_PROF_ATTN,
+    LAUNCH(KVPRM_PROF_ATTN_TC,
            kvprm::launch_attention_tc(as, wk, &ctx->tm_pool_tc, 0, Q.hi, Q.lo, ctx->apart_o, ctx->apart_ml,
                                       tc_margin(ctx), ctx->err_d, st, false),
            "attention_tc");

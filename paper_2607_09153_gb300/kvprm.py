@@ -17,7 +17,7 @@ from . import build as _build
 
 KVPRM_OK, KVPRM_EINVAL, KVPRM_ECAPACITY, KVPRM_EINDEX, KVPRM_ECUDA, KVPRM_ENOMEM, KVPRM_ETIMEOUT, \
     KVPRM_EUNSUPPORTED = range(8)
-PROF_NAMES = ("gemm_qkv", "gemm_o", "gemm_gate_up", "gemm_down", "attention", "combine", "fused")
+PROF_NAMES = ("gemm_qkv", "gemm_o", "gemm_gate_up", "gemm_down", "attention", "combine", "fused", "attention_tc")
 
 
 class KvprmError(RuntimeError):
