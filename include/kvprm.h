@@ -238,12 +238,14 @@ KVPRM_API int kvprm_resolve(kvprm_ctx* ctx, int32_t b, int64_t* phys_row);
  * Inputs: block_table host int32 [n_candidates][max_blocks_per_seq], seq_lens
  * host int32 [n_candidates], group = n_q_heads / n_kv_heads, n_ctas >= 1,
  * share: 0 no sharing, 1 shared segments (kind 1) on the persistent CTAs, 2
- * shared pages scored on the tensor cores (kind 2; what scoring contexts with
- * head_dim 128 use): tiles of up to 128 / group candidates whose 4-page
- * chunks are cut into equal ranges, one per CTA of a separate launch (at most
- * n_ctas of them); kind-2 segments follow the persistent CTAs' segments
- * (segs[cta_seg[n_ctas]] on), and tensor-core CTA k scores segments
- * segs[tc_cta[k]] .. segs[tc_cta[k + 1] - 1].
+ * shared pages scored on the tensor cores (kind 2): tiles of up to
+ * 128 / group candidates whose 4-page chunks are cut into equal ranges, one
+ * per CTA of a separate launch (at most n_ctas of them); 3 (what scoring
+ * contexts with head_dim 128 use) as 2, with the n_ctas SMs split between the
+ * two launches in proportion to their estimated time (n_ctas + n_tc_ctas <=
+ * the given n_ctas), so that they run side by side.  Kind-2 segments follow
+ * the persistent CTAs' segments (segs[cta_seg[n_ctas]] on), and tensor-core
+ * CTA k scores segments segs[tc_cta[k]] .. segs[tc_cta[k + 1] - 1].
  * Outputs go to caller-owned arrays with the capacities given (elements); the
  * counts are always written:
  *  segs       [n_segs][8] int32: kind, kv head, candidate (kind 0) or offset

@@ -67,6 +67,13 @@ constexpr int kThreads = (kConsumerWarps + 2) * 32;
 // half a private page per candidate.
 constexpr int64_t kPrivateCost = 4;
 constexpr int64_t kSharedCostPerCand = 2;
+// a 64-token chunk of the tensor-core attention on one SM, in the same units, when it runs beside
+// the private pages' launch (measured: 1.5-2.1 us per chunk then, against ~0.17 us per private
+// page; ~0.86 us per chunk alone)
+constexpr int64_t kTcChunkCost = 40;
+// pages shared by fewer candidates go to the persistent kernel as kind-1 runs: 2 units per page
+// and candidate there against kTcChunkCost / 4 per page on the tensor cores, whatever the tile's rows
+constexpr size_t kTcMinCands = 6;
 // Tensor-core scoring of shared pages (attn_tc_kernel): query rows per tile
 // and pages per 64-token chunk.
 constexpr int kTcRows = 128;
@@ -767,6 +774,7 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
   w.tc_seg0 = 0;
   w.n_tc = 0;
   w.n_tc_ctas = 0;
+  w.tc_concurrent = false;
   w.tc_cta.clear();
   w.segs.clear();
   w.cta_seg.clear();
@@ -845,12 +853,13 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
         const int page_off = static_cast<int>(w.pages.size());
         w.pages.insert(w.pages.end(), pg.begin(), pg.end());
         // tensor-core tiles: as few as possible, with the candidates spread evenly over them
-        const size_t per = share == 2 ? static_cast<size_t>(kTcRows / group) : static_cast<size_t>(kConsumerWarps);
+        const bool tc = share >= 2 && c.size() >= kTcMinCands;
+        const size_t per = tc ? static_cast<size_t>(kTcRows / group) : static_cast<size_t>(kConsumerWarps);
         const size_t n_chunks = (c.size() + per - 1) / per;
         for (size_t k = 0, c0 = 0; k < n_chunks; ++k) {
-          const size_t c1 = share == 2 ? c.size() * (k + 1) / n_chunks : std::min(c.size(), c0 + per);
+          const size_t c1 = tc ? c.size() * (k + 1) / n_chunks : std::min(c.size(), c0 + per);
           Run r;
-          r.kind = share == 2 ? 2 : 1;
+          r.kind = tc ? 2 : 1;
           r.cand = static_cast<int>(w.cands.size());
           r.n_cands = static_cast<int>(c1 - c0);
           r.page_off = page_off;
@@ -882,16 +891,26 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
     runs.push_back(r);
   }
   // ---- 2. cut the cost axis into C equal ranges (at least a stage of work each)
-  int64_t total = 0, tc_units = 0;
+  int64_t total = 0, tc_chunks = 0;
   for (const Run& r : runs) {
     if (r.kind == 2)
-      tc_units += static_cast<int64_t>(r.n_pages) * n_kv;
+      tc_chunks += static_cast<int64_t>((r.n_pages + kTcChunkPages - 1) / kTcChunkPages) * n_kv;
     else
       total += static_cast<int64_t>(r.n_pages) * r.cost * n_kv;
   }
+  // SMs for the private launch: all of them, or (share 3, both kinds of work) the share that makes
+  // both launches end together when they run side by side
+  int priv_ctas = n_ctas, tc_ctas = n_ctas;
+  if (share == 3 && total > 0 && tc_chunks > 0 && n_ctas >= 2) {
+    const int64_t wt = tc_chunks * kTcChunkCost;
+    tc_ctas = static_cast<int>(std::min<int64_t>(n_ctas - 1, std::max<int64_t>(1, (n_ctas * wt + (wt + total) / 2) /
+                                                                                        (wt + total))));
+    priv_ctas = n_ctas - tc_ctas;
+    w.tc_concurrent = true;
+  }
   const int C = total == 0 ? 0
                            : static_cast<int>(std::max<int64_t>(
-                                 1, std::min<int64_t>(n_ctas, total / (kPagesPerStage * kPrivateCost))));
+                                 1, std::min<int64_t>(priv_ctas, total / (kPagesPerStage * kPrivateCost))));
   std::vector<int> seg_cta;
   int64_t pos = 0;   // cost position of the current pair's first unit
   for (const Run& r : runs) {
@@ -937,11 +956,9 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
   w.tc_seg0 = static_cast<int>(w.segs.size());
   w.tc_cta.clear();
   w.n_tc_ctas = 0;
-  if (tc_units > 0) {
-    int64_t T = 0;
-    for (const Run& r : runs)
-      if (r.kind == 2) T += static_cast<int64_t>((r.n_pages + kTcChunkPages - 1) / kTcChunkPages) * n_kv;
-    const int Ct = static_cast<int>(std::min<int64_t>(n_ctas, T));
+  if (tc_chunks > 0) {
+    const int64_t T = tc_chunks;
+    const int Ct = static_cast<int>(std::min<int64_t>(tc_ctas, T));
     std::vector<int> tc_seg_cta;
     int64_t at = 0;   // chunk position of the current pair's first chunk
     for (const Run& r : runs) {

@@ -107,10 +107,14 @@ struct AttnWorkHost {
   int tc_seg0 = 0, n_tc = 0;   // tensor-core segments (kind 2): segs[tc_seg0, tc_seg0 + n_tc)
   int n_tc_ctas = 0;
   std::vector<int32_t> tc_cta;   // [n_tc_ctas + 1] first segment (index into segs) of each tensor-core CTA
+  bool tc_concurrent = false;    // the two attention launches have disjoint SMs and may run at once
 };
 // share: 0 every page scored per candidate; 1 shared pages scored once per run
 // of <= 8 candidates by the persistent kernel; 2 shared pages scored on the
-// tensor cores (head_dim 128 only), tiles of <= 128 / group candidates.
+// tensor cores (head_dim 128 only), tiles of <= 128 / group candidates, each
+// launch planned over all n_ctas SMs; 3 as 2, with the SMs split between the
+// tensor-core and the private launch in proportion to their estimated time,
+// so the two can run concurrently.
 bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks, int n_kv, int group, int n_ctas,
                      size_t slot_limit, int share, AttnWorkHost& w);
 // partial slots a context sized for max_candidates provides (the planner falls

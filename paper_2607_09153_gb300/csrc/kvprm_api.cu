@@ -105,6 +105,9 @@ struct kvprm_ctx {
   size_t dev_pool_bytes = 0;
   // graph replay
   cudaStream_t cap_stream = nullptr;
+  // the tensor-core attention's stream when it runs beside the private pages' launch
+  cudaStream_t side_stream = nullptr;
+  cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
 
   bool use_graph = true, use_pdl = true;
   GraphKey gkey;
@@ -213,14 +216,17 @@ void free_ctx(kvprm_ctx* c) {
   if (c->staging_ev) cudaEventDestroy(c->staging_ev);
   if (c->gexec) cudaGraphExecDestroy(c->gexec);
   for (auto& m : c->graph_marks) {
-    cudaEventDestroy(m.a);
-    cudaEventDestroy(m.b);
+    if (m.a) cudaEventDestroy(m.a);
+    if (m.b) cudaEventDestroy(m.b);
   }
   for (auto& m : c->live_marks) {
     cudaEventDestroy(m.a);
     cudaEventDestroy(m.b);
   }
   if (c->cap_stream) cudaStreamDestroy(c->cap_stream);
+  if (c->side_stream) cudaStreamDestroy(c->side_stream);
+  if (c->ev_fork) cudaEventDestroy(c->ev_fork);
+  if (c->ev_join) cudaEventDestroy(c->ev_join);
 
   delete c;
 }
@@ -397,6 +403,10 @@ struct Enq {
     *ev_b = m.b;
     return KVPRM_OK;
   }
+  // count a launch whose time is part of an enclosing mark (no events of its own)
+  void count(int cls) {
+    if (prof) marks->push_back(ProfMark{cls, nullptr, nullptr});
+  }
   unsigned long long* trace_slot(int cls) {
     if (!ctx->trace || ctx->trace_n >= ctx->trace_cap) return nullptr;
     ctx->trace_cls.push_back(cls);
@@ -421,6 +431,51 @@ struct Enq {
     rc_ = E.end(evb_);                             \
     if (rc_) return rc_;                           \
   } while (0)
+
+// The attention step of one layer: shared pages on the tensor cores (when the
+// plan has any) and the private pages, into partial slots.  When the plan gave
+// the two launches disjoint SMs (share mode 3) the tensor-core launch runs on
+// the side stream, forked here and joined before returning, so both read
+// their pages at once; a profiled call then times the pair as one step.
+int enqueue_attention(kvprm_ctx* ctx, Enq& E, const kvprm::AttnShape& as, const kvprm::AttnWork& wk, int layer,
+                      const kvprm::HiLo& Q, bool pdl) {
+  cudaStream_t st = E.st;
+  unsigned long long* tc_prof = (ctx->debug_flags & 32) ? ctx->tc_prof : nullptr;
+  if (wk.n_tc > 0 && ctx->work_host.tc_concurrent) {
+    cudaEvent_t evb = nullptr;
+    int rc = E.begin(KVPRM_PROF_ATTN, &evb);
+    if (rc) return rc;
+    CK(cudaEventRecord(ctx->ev_fork, st), "cudaEventRecord(fork)");
+    CK(cudaStreamWaitEvent(ctx->side_stream, ctx->ev_fork, 0), "cudaStreamWaitEvent(fork)");
+    {
+      unsigned long long* TS = E.trace_slot(KVPRM_PROF_ATTN_TC);
+      cudaError_t e = kvprm::launch_attention_tc(as, wk, &ctx->tm_pool_tc, layer, Q.hi, Q.lo, ctx->apart_o,
+                                                 ctx->apart_ml, tc_margin(ctx), ctx->err_d, ctx->side_stream, false,
+                                                 TS, tc_prof);
+      if (e != cudaSuccess) return cuda_fail(ctx, e, "attention_tc");
+      E.count(KVPRM_PROF_ATTN_TC);
+    }
+    CK(cudaEventRecord(ctx->ev_join, ctx->side_stream), "cudaEventRecord(join)");
+    {
+      unsigned long long* TS = E.trace_slot(KVPRM_PROF_ATTN);
+      cudaError_t e = kvprm::launch_attention(as, wk, &ctx->tm_pool, layer, Q.hi, Q.lo, ctx->apart_o, ctx->apart_ml,
+                                              ctx->err_d, st, pdl, TS);
+      if (e != cudaSuccess) return cuda_fail(ctx, e, "attention");
+    }
+    CK(cudaStreamWaitEvent(st, ctx->ev_join, 0), "cudaStreamWaitEvent(join)");
+    return E.end(evb);
+  }
+  if (wk.n_tc > 0)
+    LAUNCH(KVPRM_PROF_ATTN_TC,
+           kvprm::launch_attention_tc(as, wk, &ctx->tm_pool_tc, layer, Q.hi, Q.lo, ctx->apart_o, ctx->apart_ml,
+                                      tc_margin(ctx), ctx->err_d, st, pdl, TS, tc_prof),
+           "attention_tc");
+  LAUNCH(KVPRM_PROF_ATTN,
+         kvprm::launch_attention(as, wk, &ctx->tm_pool, layer, Q.hi, Q.lo, ctx->apart_o, ctx->apart_ml, ctx->err_d,
+                                 st, pdl, TS),
+         "attention");
+  return KVPRM_OK;
+}
 
 int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
   const ModelDims& m = ctx->md;
@@ -489,16 +544,10 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
     float* dbg = (ctx->debug_flags & 1) ? ctx->dbg + static_cast<size_t>(l) * n * m.n_q * m.hd : nullptr;
     const kvprm::AttnMerge mg{ctx->q, ctx->kself, ctx->vself, O.hi, O.lo, nullptr, dbg};
     const kvprm::AttnWork wk = device_work(ctx);
-    if (wk.n_tc > 0)   // shared pages on the tensor cores
-      LAUNCH(KVPRM_PROF_ATTN_TC,
-             kvprm::launch_attention_tc(ctx->as, wk, &ctx->tm_pool_tc, l, ctx->qhi, ctx->qlo, ctx->apart_o,
-                                        ctx->apart_ml, tc_margin(ctx), ctx->err_d, st, pdl, TS,
-                                        (ctx->debug_flags & 32) ? ctx->tc_prof : nullptr),
-             "attention_tc");
-    LAUNCH(KVPRM_PROF_ATTN,
-           kvprm::launch_attention(ctx->as, wk, &ctx->tm_pool, l, ctx->qhi, ctx->qlo, ctx->apart_o, ctx->apart_ml,
-                                   ctx->err_d, st, pdl, TS),
-           "attention");
+    {
+      const int rc = enqueue_attention(ctx, E, ctx->as, wk, l, kvprm::HiLo{ctx->qhi, ctx->qlo}, pdl);
+      if (rc) return rc;
+    }
     LAUNCH(KVPRM_PROF_COMBINE,
            kvprm::launch_attn_combine(ctx->as, wk, n, ctx->apart_o, ctx->apart_ml, mg, st, pdl, TS), "attn_combine");
     kvprm::GemmEpilogue er_o = er;   // h += W_o o; x = h ⊙ g_mlp for the gate/up projection
@@ -532,10 +581,10 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
 int accumulate_marks(kvprm_ctx* ctx, std::vector<ProfMark>& marks, bool destroy) {
   for (auto& mk : marks) {
     float ms = 0.f;
-    CK(cudaEventElapsedTime(&ms, mk.a, mk.b), "cudaEventElapsedTime");
+    if (mk.a) CK(cudaEventElapsedTime(&ms, mk.a, mk.b), "cudaEventElapsedTime");
     ctx->prof_launches[mk.cls] += 1;
     ctx->prof_ms[mk.cls] += ms;
-    if (destroy) {
+    if (destroy && mk.a) {
       cudaEventDestroy(mk.a);
       cudaEventDestroy(mk.b);
     }
@@ -548,8 +597,8 @@ void drop_graph(kvprm_ctx* ctx) {
   if (ctx->gexec) cudaGraphExecDestroy(ctx->gexec);
   ctx->gexec = nullptr;
   for (auto& m : ctx->graph_marks) {
-    cudaEventDestroy(m.a);
-    cudaEventDestroy(m.b);
+    if (m.a) cudaEventDestroy(m.a);
+    if (m.b) cudaEventDestroy(m.b);
   }
   ctx->graph_marks.clear();
   ctx->gkey = GraphKey();
@@ -593,7 +642,7 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   key.n = n;
   key.n_pad = P.n_pad;
   key.attn_ctas = P.attn_ctas;
-  key.tc_ctas = ctx->work_host.n_tc_ctas;
+  key.tc_ctas = ctx->work_host.n_tc_ctas * (ctx->work_host.tc_concurrent ? -1 : 1);
   key.n_tc = ctx->work_host.n_tc > 0 ? 1 : 0;
   key.debug = ctx->debug_flags;
   key.profile = ctx->profile ? 1 : 0;
@@ -802,10 +851,16 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   }
   CREATE_CK(cu(cudaEventCreateWithFlags(&ctx->staging_ev, cudaEventDisableTiming), "cudaEventCreate"));
   CREATE_CK(cu(cudaStreamCreateWithFlags(&ctx->cap_stream, cudaStreamNonBlocking), "cudaStreamCreate"));
+  CREATE_CK(cu(cudaStreamCreateWithFlags(&ctx->side_stream, cudaStreamNonBlocking), "cudaStreamCreate"));
+  CREATE_CK(cu(cudaEventCreateWithFlags(&ctx->ev_fork, cudaEventDisableTiming), "cudaEventCreate"));
+  CREATE_CK(cu(cudaEventCreateWithFlags(&ctx->ev_join, cudaEventDisableTiming), "cudaEventCreate"));
   ctx->use_graph = !env_off("KVPRM_NO_GRAPH");
   ctx->use_pdl = !env_off("KVPRM_NO_PDL");
   // shared pages: on the tensor cores at head_dim 128, else one warp per candidate
-  ctx->share_mode = env_off("KVPRM_NO_SHARING") ? 0 : ((c.head_dim == 128 && !env_off("KVPRM_NO_TC_SHARING")) ? 2 : 1);
+  ctx->share_mode = env_off("KVPRM_NO_SHARING")
+                        ? 0
+                        : ((c.head_dim == 128 && !env_off("KVPRM_NO_TC_SHARING")) ? (env_off("KVPRM_TC_SERIAL") ? 2 : 3)
+                                                                                   : 1);
   CREATE_CK(cu(cudaDeviceSynchronize(), "cudaDeviceSynchronize(create)"));
 #undef CREATE_CK
   *out = ctx;
@@ -910,15 +965,7 @@ int kvprm_attention(kvprm_ctx* ctx, const void* kv_layer, int64_t n_pages, const
   const kvprm::AttnMerge mg{static_cast<const float*>(q), static_cast<const float*>(k_self),
                             static_cast<const float*>(v_self), ctx->ohi, ctx->olo, out, nullptr};
   const kvprm::AttnWork wk = device_work(ctx);
-  if (wk.n_tc > 0)
-    LAUNCH(KVPRM_PROF_ATTN_TC,
-           kvprm::launch_attention_tc(as, wk, &ctx->tm_pool_tc, 0, Q.hi, Q.lo, ctx->apart_o, ctx->apart_ml,
-                                      tc_margin(ctx), ctx->err_d, st, false),
-           "attention_tc");
-  LAUNCH(KVPRM_PROF_ATTN,
-         kvprm::launch_attention(as, wk, &ctx->tm_pool, 0, Q.hi, Q.lo, ctx->apart_o, ctx->apart_ml, ctx->err_d, st,
-                                 false),
-         "attention");
+  if ((rc = enqueue_attention(ctx, E, as, wk, 0, Q, false))) return rc;
   LAUNCH(KVPRM_PROF_COMBINE, kvprm::launch_attn_combine(as, wk, n, ctx->apart_o, ctx->apart_ml, mg, st, false),
          "attn_combine");
   ctx->last_n = n;
@@ -1063,7 +1110,7 @@ int kvprm_plan_attention(const int32_t* block_table, int32_t max_blocks_per_seq,
       return KVPRM_EINVAL;
   kvprm::AttnWorkHost w;
   if (!kvprm::build_attn_work(block_table, seq_lens, n_candidates, max_blocks_per_seq, n_kv_heads, group, n_ctas,
-                              SIZE_MAX, share < 0 ? 0 : (share > 2 ? 2 : share), w))
+                              SIZE_MAX, share < 0 ? 0 : (share > 3 ? 3 : share), w))
     return KVPRM_ECAPACITY;
   plan->n_segs = static_cast<int32_t>(w.segs.size());
   plan->n_ctas = w.n_ctas;

@@ -36,7 +36,7 @@ def check_plan(bt, sl, n_kv, group, n_ctas, share):
     assert p["n_ctas"] <= n_ctas
     if p["n_ctas"]:
         assert cta[0] == 0 and np.all(np.diff(cta) >= 0)
-        assert cta[-1] == len(segs) if share != 2 else cta[-1] <= len(segs)
+        assert cta[-1] == len(segs) if share < 2 else cta[-1] <= len(segs)
     cost = np.zeros(max(p["n_ctas"], 1))
     for k in range(p["n_ctas"]):
         for s in segs[cta[k]:cta[k + 1]]:
@@ -49,7 +49,9 @@ def check_plan(bt, sl, n_kv, group, n_ctas, share):
                 slots = [[slot + i for i in range(k_slots)]]
                 cost[k] += PRIVATE_COST * npg
             else:
-                assert kind == 1 and share == 1 and 1 <= nc <= 8 and last == 16
+                # kind 1: shared runs on the persistent CTAs (share 1, or share >= 2 for pages
+                # shared by fewer candidates than a tensor-core tile is worth)
+                assert kind == 1 and share >= 1 and 1 <= nc <= 8 and last == 16
                 cands = [int(x) for x in p["cands"][c:c + nc]]
                 slots = [[int(x)] for x in p["slots"][slot:slot + nc]]
                 cost[k] += SHARED_COST_PER_CAND * nc * npg
@@ -57,11 +59,11 @@ def check_plan(bt, sl, n_kv, group, n_ctas, share):
                 used[(b, g)] += sls
                 for i, pg in enumerate(pages):
                     got[(b, g, int(pg), last if i == npg - 1 else 16)] += 1
-    # tensor-core segments (share = 2) follow the persistent CTAs' segments
+    # tensor-core segments (share >= 2) follow the persistent CTAs' segments
     tc0 = int(cta[-1]) if p["n_ctas"] else 0
     for s in segs[tc0:]:
         kind, g, c, nc, off, npg, last, slot = (int(x) for x in s)
-        assert kind == 2 and share == 2 and 0 <= g < n_kv and npg >= 1 and last == 16
+        assert kind == 2 and share >= 2 and 0 <= g < n_kv and npg >= 1 and last == 16
         assert 1 <= nc <= 128 // group, "a tile holds at most 128 query rows"
         for b, sl_ in zip(p["cands"][c:c + nc], p["slots"][slot:slot + nc]):
             used[(int(b), g)].append(int(sl_))
@@ -75,21 +77,23 @@ def check_plan(bt, sl, n_kv, group, n_ctas, share):
     assert int(p["nslots"].sum()) == p["n_slots"]
     if p["n_ctas"] > 1:
         total = cost.sum()
-        unit = PRIVATE_COST if share != 1 else max(PRIVATE_COST, SHARED_COST_PER_CAND * 8)
+        unit = PRIVATE_COST if share == 0 else max(PRIVATE_COST, SHARED_COST_PER_CAND * 8)
         assert np.abs(cost - total / p["n_ctas"]).max() <= unit, "equal CTA shares up to one page"
     return p
 
 
 @pytest.mark.parametrize("name", ["tiny", "qwen1p5b_b16_l2048", "beam7b_b64_p4096_s512", "long8b_b8_l32768",
                                   "mcts7b_b256_d4"])
-@pytest.mark.parametrize("share", [0, 1, 2])
+@pytest.mark.parametrize("share", [0, 1, 2, 3])
 def test_workload_plans(name, share):
     w = ks.make_workload(name)
     a = w.arch
     p = check_plan(w.block_table, w.seq_lens, a.n_kv_heads, a.n_q_heads // a.n_kv_heads, 152, share)
     if not share:
         assert (p["segs"][:, 0] == 0).all()
-    if share == 2 and name in ("beam7b_b64_p4096_s512", "mcts7b_b256_d4"):
+    if share == 3 and p["n_tc_ctas"] and p["n_ctas"]:
+        assert p["n_ctas"] + p["n_tc_ctas"] <= 152, "side by side, the two launches share the SMs"
+    if share >= 2 and name in ("beam7b_b64_p4096_s512", "mcts7b_b256_d4"):
         tc = p["segs"][p["segs"][:, 0] == 2]
         # at most one tensor-core CTA per SM, equal chunk counts up to one, every kind-2 segment owned once;
         # within a (tile, kv head) every piece but the last is whole 4-page chunks
@@ -140,6 +144,35 @@ def test_shared_prefix_tensor_core_tiles():
     assert len(per_tile_head) == 3 * 2 and set(per_tile_head.values()) == {pre}, "each tile reads the prefix once"
 
 
+@pytest.mark.parametrize("n_share, kind", [(4, 1), (5, 1), (6, 2), (9, 2)])
+def test_small_shared_groups_stay_on_the_persistent_kernel(n_share, kind):
+    # pages shared by fewer than 6 candidates are scored as kind-1 runs even in the tensor-core modes
+    n, pre, own = 12, 9, 2
+    bt = np.zeros((n, pre + own), np.int32)
+    for b in range(n):
+        bt[b, :pre] = np.arange(pre) if b < n_share else 100 + pre * b + np.arange(pre)
+        bt[b, pre:] = 1000 + own * b + np.arange(own)
+    sl = np.full(n, 16 * (pre + own), np.int32)
+    for share in (2, 3):
+        p = check_plan(bt, sl, 2, 7, 24, share)
+        shared = p["segs"][p["segs"][:, 0] != 0]
+        assert len(shared) and set(shared[:, 0].tolist()) == {kind}
+
+
+def test_concurrent_split_shares_the_sms():
+    # a shared prefix (tensor cores) and private suffixes (persistent kernel) side by side
+    n, pre, own = 40, 64, 24
+    bt = np.zeros((n, pre + own), np.int32)
+    for b in range(n):
+        bt[b, :pre] = np.arange(pre)
+        bt[b, pre:] = pre + own * b + np.arange(own)
+    sl = np.full(n, 16 * (pre + own), np.int32)
+    p3 = check_plan(bt, sl, 2, 7, 64, 3)
+    assert p3["n_tc_ctas"] >= 1 and p3["n_ctas"] >= 1 and p3["n_tc_ctas"] + p3["n_ctas"] <= 64
+    p2 = check_plan(bt, sl, 2, 7, 64, 2)   # serial: each launch planned over all SMs
+    assert p2["n_ctas"] == 64 and p2["n_tc_ctas"] == 64
+
+
 def test_repeated_page_in_one_candidate_stays_private():
     bt = np.array([[3, 3, 4], [3, 3, 5]], np.int32)   # page 3 listed twice by both candidates
     sl = np.array([48, 48], np.int32)
@@ -158,7 +191,7 @@ def test_partial_last_page_is_never_shared():
 
 @pytest.mark.parametrize("lens", [[0], [0, 0, 0], [1], [16], [17], [0, 1, 15, 16, 17, 31, 33, 100, 257, 1000]])
 @pytest.mark.parametrize("n_ctas", [1, 3, 152])
-@pytest.mark.parametrize("share", [1, 2])
+@pytest.mark.parametrize("share", [1, 2, 3])
 def test_edges(lens, n_ctas, share):
     n = len(lens)
     mb = max(1, max((L + 15) // 16 for L in lens))
