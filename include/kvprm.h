@@ -276,7 +276,18 @@ typedef struct {
   int32_t n_tc_ctas;  /* out */
   int32_t* tc_cta;
   int64_t tc_cta_cap;
+  int32_t fuse_cs;    /* out: 0, or the cluster size of a fused-combine plan */
 } kvprm_attn_plan;
+/* share | KVPRM_PLAN_FUSE: first try the fused-combine plan (what scoring
+ * contexts do): when every candidate has about the same number of pages (the
+ * longest at most 5/4 of the shortest), no page is referenced twice and
+ * group <= 8, (candidate, kv head) pair p = b * n_kv_heads + g is scored by the
+ * fuse_cs CTAs fuse_cs * p .. fuse_cs * p + fuse_cs - 1 (one thread-block
+ * cluster; fuse_cs a power of two <= 8 with pairs * fuse_cs <= n_ctas, at most
+ * 64 pages per CTA), rank r taking pages [r L / fuse_cs, (r + 1) L / fuse_cs) of
+ * the candidate's L and partial slot fuse_cs * p + r; rank 0 merges the
+ * pair's slots in the same launch, so no combine launch follows. */
+#define KVPRM_PLAN_FUSE 16
 KVPRM_API int kvprm_plan_attention(const int32_t* block_table, int32_t max_blocks_per_seq, const int32_t* seq_lens,
                                    int32_t n_candidates, int32_t n_kv_heads, int32_t group, int32_t n_ctas,
                                    int32_t share, kvprm_attn_plan* plan);

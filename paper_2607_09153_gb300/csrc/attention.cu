@@ -39,6 +39,7 @@
 #include <cuda_bf16.h>
 
 #include <algorithm>
+#include <climits>
 #include <unordered_map>
 #include <vector>
 
@@ -109,7 +110,7 @@ template <int HD, bool TWO_ROWS>
 __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
     const __grid_constant__ CUtensorMap tm_pool, int64_t layer_page0, AttnWork wk,
     const __nv_bfloat16* __restrict__ q_hi, const __nv_bfloat16* __restrict__ q_lo, int n_q, int n_kv, int group,
-    float* __restrict__ part_o, float* __restrict__ part_ml, int* err, unsigned long long* ts) {
+    float* __restrict__ part_o, float* __restrict__ part_ml, AttnMerge mg, int* err, unsigned long long* ts) {
   using SM = AttnSmem<HD>;
   trace_begin(ts);
 
@@ -251,6 +252,21 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
       ++k;
     }
     if (lane == 0) trace_event(ts, 2);   // every private run of this CTA is merged
+  }
+  if (!TWO_ROWS && wk.fuse_cs > 0) {   // fused plans have group <= 8
+    // The cluster scored one (candidate, kv head): once every rank's partial slot is written
+    // (the cluster barrier releases them), rank 0 merges the slots with the verify token's own
+    // entry, as the combine launch would.  Its ring is idle by now and holds the merge scratch;
+    // warps 0..7 passed the grid-dependency wait, so q and the self k / v are visible to them.
+    __syncwarp();
+    cluster_sync();
+    if (cluster_rank() == 0 && warp < kConsumerWarps) {
+      const int pr = blockIdx.x / wk.fuse_cs, b = pr / n_kv, g = pr - b * n_kv;
+      combine_group<HD, 8>(threadIdx.x, b, g, wk.slot_base[pr], wk.nslots[pr], n_q, n_kv, group,
+                                           part_o, part_ml, mg, base,
+                                           [] { named_bar_sync(2, kConsumerWarps * 32); });
+      if (threadIdx.x == 0) trace_event(ts, 3);   // the pair's output is written
+    }
   }
   trace_end(ts);
 }
@@ -1019,6 +1035,67 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
   return true;
 }
 
+bool build_attn_work_fused(const int32_t* bt, const int32_t* sl, int n, int max_blocks, int n_kv, int group,
+                           int n_ctas, size_t slot_limit, AttnWorkHost& w) {
+  if (n <= 0 || group > 8 || n_kv < 1) return false;
+  int lo = INT32_MAX, hi = 0;
+  for (int b = 0; b < n; ++b) {
+    const int np = (sl[b] + 15) / 16;
+    lo = std::min(lo, np);
+    hi = std::max(hi, np);
+  }
+  if (lo < 1 || 4 * hi > 5 * lo) return false;   // equal ranges need about equal lengths
+  const int64_t pairs = static_cast<int64_t>(n) * n_kv;
+  int cs = 0;
+  for (int c = 8; c >= 1; c >>= 1)
+    if (pairs * c <= n_ctas && c <= lo) {
+      cs = c;
+      break;
+    }
+  if (cs == 0 || (hi + cs - 1) / cs > kFuseMaxPages) return false;
+  if (static_cast<size_t>(pairs) * cs > slot_limit) return false;
+  {   // a page referenced twice (sharing, or a repeat) is left to the persistent plan
+    std::unordered_map<int32_t, char> seen;
+    seen.reserve(static_cast<size_t>(n) * hi);
+    for (int b = 0; b < n; ++b)
+      for (int j = 0, np = (sl[b] + 15) / 16; j < np; ++j)
+        if (!seen.emplace(bt[static_cast<int64_t>(b) * max_blocks + j], 1).second) return false;
+  }
+  w = AttnWorkHost();
+  w.fuse_cs = cs;
+  w.slot_base.assign(static_cast<size_t>(pairs), 0);
+  w.nslots.assign(static_cast<size_t>(pairs), cs);
+  w.cta_seg.reserve(static_cast<size_t>(pairs) * cs + 1);
+  w.cta_seg.push_back(0);
+  for (int b = 0; b < n; ++b) {
+    const int np = (sl[b] + 15) / 16;
+    const int page_off = static_cast<int>(w.pages.size());
+    for (int j = 0; j < np; ++j) w.pages.push_back(bt[static_cast<int64_t>(b) * max_blocks + j]);
+    for (int g = 0; g < n_kv; ++g) {
+      const int pr = b * n_kv + g;
+      w.slot_base[pr] = pr * cs;
+      for (int r = 0; r < cs; ++r) {   // rank r: pages [r np / cs, (r + 1) np / cs)
+        const int p0 = r * np / cs, p1 = (r + 1) * np / cs;
+        AttnSeg sg;
+        sg.kind = 0;
+        sg.g = g;
+        sg.cand = b;
+        sg.n_cands = 1;
+        sg.page_off = page_off + p0;
+        sg.n_pages = p1 - p0;
+        sg.last_valid = p1 == np ? sl[b] - 16 * (np - 1) : 16;
+        sg.slot = pr * cs + r;
+        w.segs.push_back(sg);
+        w.cta_seg.push_back(static_cast<int32_t>(w.segs.size()));
+      }
+    }
+  }
+  w.n_ctas = static_cast<int>(pairs * cs);
+  w.n_slots = static_cast<int>(pairs * cs);
+  w.tc_seg0 = static_cast<int>(w.segs.size());
+  return true;
+}
+
 cudaError_t attention_configure() {
   cudaError_t e;
   if ((e = set_smem(attn_combine_kernel<64, 8>, CombineShape<64, 8>::kBytes)) != cudaSuccess) return e;
@@ -1034,32 +1111,44 @@ cudaError_t attention_configure() {
 
 cudaError_t launch_attention(const AttnShape& s, const AttnWork& wk, const CUtensorMap* tm_pool, int layer,
                              const __nv_bfloat16* q_hi, const __nv_bfloat16* q_lo, float* part_o, float* part_ml,
-                             int* err, cudaStream_t stream, bool pdl, unsigned long long* ts) {
+                             const AttnMerge& mg, int* err, cudaStream_t stream, bool pdl, unsigned long long* ts) {
   if (wk.n_ctas == 0) return cudaSuccess;
+  if (wk.fuse_cs > 0 && (wk.n_ctas % wk.fuse_cs != 0 || wk.fuse_cs > 8)) return cudaErrorInvalidValue;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(wk.n_ctas, 1, 1);
   cfg.blockDim = dim3(kThreads, 1, 1);
   cfg.dynamicSmemBytes = attention_smem_bytes(s.hd);
   cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cudaLaunchAttribute attr[2];
+  int na = 0;
+  if (pdl) {
+    attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[na].val.programmaticStreamSerializationAllowed = 1;
+    ++na;
+  }
+  if (wk.fuse_cs > 0) {
+    attr[na].id = cudaLaunchAttributeClusterDimension;
+    attr[na].val.clusterDim.x = static_cast<unsigned>(wk.fuse_cs);
+    attr[na].val.clusterDim.y = 1;
+    attr[na].val.clusterDim.z = 1;
+    ++na;
+  }
   cfg.attrs = attr;
-  cfg.numAttrs = pdl ? 1 : 0;
+  cfg.numAttrs = na;
   const int64_t page0 = static_cast<int64_t>(layer) * s.layer_pages;
   const bool two = s.group > 8;
   if (s.hd == 128) {
     if (two)
       return cudaLaunchKernelEx(&cfg, attn_kernel<128, true>, *tm_pool, page0, wk, q_hi, q_lo, s.n_q, s.n_kv, s.group,
-                                part_o, part_ml, err, ts);
+                                part_o, part_ml, mg, err, ts);
     return cudaLaunchKernelEx(&cfg, attn_kernel<128, false>, *tm_pool, page0, wk, q_hi, q_lo, s.n_q, s.n_kv, s.group,
-                              part_o, part_ml, err, ts);
+                              part_o, part_ml, mg, err, ts);
   }
   if (two)
     return cudaLaunchKernelEx(&cfg, attn_kernel<64, true>, *tm_pool, page0, wk, q_hi, q_lo, s.n_q, s.n_kv, s.group,
-                              part_o, part_ml, err, ts);
+                              part_o, part_ml, mg, err, ts);
   return cudaLaunchKernelEx(&cfg, attn_kernel<64, false>, *tm_pool, page0, wk, q_hi, q_lo, s.n_q, s.n_kv, s.group,
-                            part_o, part_ml, err, ts);
+                            part_o, part_ml, mg, err, ts);
 }
 
 CUresult encode_pool_map_tc(PFN_cuTensorMapEncodeTiled_v12000 encode, CUtensorMap* map, const void* pool,

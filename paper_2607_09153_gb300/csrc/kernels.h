@@ -99,6 +99,8 @@ struct AttnWork {             // device arrays
   int tc_seg0, n_tc;          // tensor-core segments (kind 2)
   const int32_t* tc_cta;      // [n_tc_ctas + 1] first tensor-core segment of each CTA of attn_tc_kernel
   int n_tc_ctas;
+  int fuse_cs;                // > 0: CTAs fuse_cs p .. fuse_cs p + fuse_cs - 1 (one cluster) score pair p and
+                              // its rank 0 merges the pair's slots (no combine launch)
 };
 struct AttnWorkHost {
   std::vector<AttnSeg> segs;
@@ -108,6 +110,7 @@ struct AttnWorkHost {
   int n_tc_ctas = 0;
   std::vector<int32_t> tc_cta;   // [n_tc_ctas + 1] first segment (index into segs) of each tensor-core CTA
   bool tc_concurrent = false;    // the two attention launches have disjoint SMs and may run at once
+  int fuse_cs = 0;               // see AttnWork::fuse_cs
 };
 // share: 0 every page scored per candidate; 1 shared pages scored once per run
 // of <= 8 candidates by the persistent kernel; 2 shared pages scored on the
@@ -117,6 +120,16 @@ struct AttnWorkHost {
 // so the two can run concurrently.
 bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks, int n_kv, int group, int n_ctas,
                      size_t slot_limit, int share, AttnWorkHost& w);
+// The plan with the combine fused into the attention launch, for calls where
+// every candidate has about the same number of pages, no page is shared and
+// group <= 8: (candidate, kv head) pair p = b n_kv + g is scored by the fuse_cs
+// CTAs of cluster p, one equal page range and one partial slot each, and the
+// cluster's rank 0 merges the slots once all are written.  Returns false (and
+// leaves w untouched) when the call does not qualify or the plan would leave
+// more than kFuseMaxPages pages per CTA (then the persistent plan is better).
+constexpr int kFuseMaxPages = 64;
+bool build_attn_work_fused(const int32_t* bt, const int32_t* sl, int n, int max_blocks, int n_kv, int group,
+                           int n_ctas, size_t slot_limit, AttnWorkHost& w);
 // partial slots a context sized for max_candidates provides (the planner falls
 // back to private runs, which always fit, when sharing needs more)
 size_t attn_slot_capacity(int max_candidates, int n_kv, int num_sms);
@@ -139,10 +152,12 @@ struct AttnMerge {
 // q_hi / q_lo: bf16 pair of the rotated query [B][n_q][hd]; partial slot s of
 // query row r of its group at part_o[(s * group + r) * hd] (values) and
 // part_ml[(s * group + r) * 2] (max in log2 units, sum).  One CTA per entry of
-// wk.cta_seg.
+// wk.cta_seg.  With wk.fuse_cs > 0 the launch is made of clusters of fuse_cs
+// CTAs and also does the combine (mg: its inputs and outputs).
 cudaError_t launch_attention(const AttnShape& s, const AttnWork& wk, const CUtensorMap* tm_pool, int layer,
                              const __nv_bfloat16* q_hi, const __nv_bfloat16* q_lo, float* part_o, float* part_ml,
-                             int* err, cudaStream_t stream, bool pdl, unsigned long long* ts = nullptr);
+                             const AttnMerge& mg, int* err, cudaStream_t stream, bool pdl,
+                             unsigned long long* ts = nullptr);
 // The kind-2 segments (wk.tc_seg0 .., wk.n_tc of them; head_dim 128): shared
 // pages scored on the tensor cores, one CTA per segment.  Writes the same
 // partial slots as launch_attention.  margin: the running row maximum moves

@@ -32,10 +32,12 @@ struct CallPlan {
 
 struct GraphKey {
   int n = -1, n_pad = -1, attn_ctas = -1, tc_ctas = -1, n_tc = -1, debug = -1, profile = -1, pdl = -1, trace = -1;
+  int fuse_cs = -1;
   const void* pool = nullptr;
   int64_t n_pages = -1;
   bool operator==(const GraphKey& o) const {
     return n == o.n && n_pad == o.n_pad && attn_ctas == o.attn_ctas && tc_ctas == o.tc_ctas && n_tc == o.n_tc &&
+           fuse_cs == o.fuse_cs &&
            debug == o.debug && profile == o.profile && pdl == o.pdl && trace == o.trace && pool == o.pool &&
            n_pages == o.n_pages;
   }
@@ -76,7 +78,8 @@ struct kvprm_ctx {
          off_tc_cta = 0;
   size_t tables_ints = 0;
   size_t cap_segs = 0, cap_pages = 0, cap_cands = 0;
-  int share_mode = 2;   // sharing of pages referenced by several candidates (build_attn_work)
+  int share_mode = 3;   // sharing of pages referenced by several candidates (build_attn_work)
+  bool fuse_combine = true;   // the combine inside the attention launch where the call qualifies
   float* rewards_d = nullptr;
   int* err_d = nullptr;
   float* dbg = nullptr;
@@ -269,6 +272,9 @@ int plan_work(kvprm_ctx* ctx, const int32_t* bt, const int32_t* sl, int32_t n) {
            w.slots.size() <= ctx->slot_cap && static_cast<size_t>(w.n_ctas) <= static_cast<size_t>(ctx->num_sms) &&
            static_cast<size_t>(w.n_tc_ctas) <= static_cast<size_t>(ctx->num_sms);
   };
+  if (ctx->fuse_combine &&
+      kvprm::build_attn_work_fused(bt, sl, n, mb, nkv, ctx->md.n_q / nkv, ctx->num_sms, ctx->slot_cap, w) && fits())
+    return KVPRM_OK;
   bool ok = kvprm::build_attn_work(bt, sl, n, mb, nkv, ctx->md.n_q / nkv, ctx->num_sms, ctx->slot_cap, ctx->share_mode, w);
   if (ok && !fits() && ctx->share_mode)
     ok = kvprm::build_attn_work(bt, sl, n, mb, nkv, ctx->md.n_q / nkv, ctx->num_sms, ctx->slot_cap, 0, w);
@@ -334,6 +340,7 @@ kvprm::AttnWork device_work(kvprm_ctx* ctx) {
   wk.n_tc = ctx->work_host.n_tc;
   wk.tc_cta = ctx->tables_d + ctx->off_tc_cta;
   wk.n_tc_ctas = ctx->work_host.n_tc_ctas;
+  wk.fuse_cs = ctx->work_host.fuse_cs;
   return wk;
 }
 
@@ -438,7 +445,7 @@ struct Enq {
 // the side stream, forked here and joined before returning, so both read
 // their pages at once; a profiled call then times the pair as one step.
 int enqueue_attention(kvprm_ctx* ctx, Enq& E, const kvprm::AttnShape& as, const kvprm::AttnWork& wk, int layer,
-                      const kvprm::HiLo& Q, bool pdl) {
+                      const kvprm::HiLo& Q, const kvprm::AttnMerge& mg, bool pdl) {
   cudaStream_t st = E.st;
   unsigned long long* tc_prof = (ctx->debug_flags & 32) ? ctx->tc_prof : nullptr;
   if (wk.n_tc > 0 && ctx->work_host.tc_concurrent) {
@@ -459,7 +466,7 @@ int enqueue_attention(kvprm_ctx* ctx, Enq& E, const kvprm::AttnShape& as, const 
     {
       unsigned long long* TS = E.trace_slot(KVPRM_PROF_ATTN);
       cudaError_t e = kvprm::launch_attention(as, wk, &ctx->tm_pool, layer, Q.hi, Q.lo, ctx->apart_o, ctx->apart_ml,
-                                              ctx->err_d, st, pdl, TS);
+                                              mg, ctx->err_d, st, pdl, TS);
       if (e != cudaSuccess) return cuda_fail(ctx, e, "attention");
     }
     CK(cudaStreamWaitEvent(st, ctx->ev_join, 0), "cudaStreamWaitEvent(join)");
@@ -471,8 +478,8 @@ int enqueue_attention(kvprm_ctx* ctx, Enq& E, const kvprm::AttnShape& as, const 
                                       tc_margin(ctx), ctx->err_d, st, pdl, TS, tc_prof),
            "attention_tc");
   LAUNCH(KVPRM_PROF_ATTN,
-         kvprm::launch_attention(as, wk, &ctx->tm_pool, layer, Q.hi, Q.lo, ctx->apart_o, ctx->apart_ml, ctx->err_d,
-                                 st, pdl, TS),
+         kvprm::launch_attention(as, wk, &ctx->tm_pool, layer, Q.hi, Q.lo, ctx->apart_o, ctx->apart_ml, mg,
+                                 ctx->err_d, st, pdl, TS),
          "attention");
   return KVPRM_OK;
 }
@@ -545,11 +552,13 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
     const kvprm::AttnMerge mg{ctx->q, ctx->kself, ctx->vself, O.hi, O.lo, nullptr, dbg};
     const kvprm::AttnWork wk = device_work(ctx);
     {
-      const int rc = enqueue_attention(ctx, E, ctx->as, wk, l, kvprm::HiLo{ctx->qhi, ctx->qlo}, pdl);
+      const int rc = enqueue_attention(ctx, E, ctx->as, wk, l, kvprm::HiLo{ctx->qhi, ctx->qlo}, mg, pdl);
       if (rc) return rc;
     }
-    LAUNCH(KVPRM_PROF_COMBINE,
-           kvprm::launch_attn_combine(ctx->as, wk, n, ctx->apart_o, ctx->apart_ml, mg, st, pdl, TS), "attn_combine");
+    if (wk.fuse_cs == 0)   // else the attention launch merged the slots itself
+      LAUNCH(KVPRM_PROF_COMBINE,
+             kvprm::launch_attn_combine(ctx->as, wk, n, ctx->apart_o, ctx->apart_ml, mg, st, pdl, TS),
+             "attn_combine");
     kvprm::GemmEpilogue er_o = er;   // h += W_o o; x = h ⊙ g_mlp for the gate/up projection
     er_o.gain_next = ctx->mlp_norm[l];
     LAUNCH(KVPRM_PROF_GEMM_O,
@@ -643,6 +652,7 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   key.n_pad = P.n_pad;
   key.attn_ctas = P.attn_ctas;
   key.tc_ctas = ctx->work_host.n_tc_ctas * (ctx->work_host.tc_concurrent ? -1 : 1);
+  key.fuse_cs = ctx->work_host.fuse_cs;
   key.n_tc = ctx->work_host.n_tc > 0 ? 1 : 0;
   key.debug = ctx->debug_flags;
   key.profile = ctx->profile ? 1 : 0;
@@ -857,6 +867,7 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   ctx->use_graph = !env_off("KVPRM_NO_GRAPH");
   ctx->use_pdl = !env_off("KVPRM_NO_PDL");
   // shared pages: on the tensor cores at head_dim 128, else one warp per candidate
+  ctx->fuse_combine = !env_off("KVPRM_NO_FUSED_COMBINE");
   ctx->share_mode = env_off("KVPRM_NO_SHARING")
                         ? 0
                         : ((c.head_dim == 128 && !env_off("KVPRM_NO_TC_SHARING")) ? (env_off("KVPRM_TC_SERIAL") ? 2 : 3)
@@ -965,9 +976,10 @@ int kvprm_attention(kvprm_ctx* ctx, const void* kv_layer, int64_t n_pages, const
   const kvprm::AttnMerge mg{static_cast<const float*>(q), static_cast<const float*>(k_self),
                             static_cast<const float*>(v_self), ctx->ohi, ctx->olo, out, nullptr};
   const kvprm::AttnWork wk = device_work(ctx);
-  if ((rc = enqueue_attention(ctx, E, as, wk, 0, Q, false))) return rc;
-  LAUNCH(KVPRM_PROF_COMBINE, kvprm::launch_attn_combine(as, wk, n, ctx->apart_o, ctx->apart_ml, mg, st, false),
-         "attn_combine");
+  if ((rc = enqueue_attention(ctx, E, as, wk, 0, Q, mg, false))) return rc;
+  if (wk.fuse_cs == 0)
+    LAUNCH(KVPRM_PROF_COMBINE, kvprm::launch_attn_combine(as, wk, n, ctx->apart_o, ctx->apart_ml, mg, st, false),
+           "attn_combine");
   ctx->last_n = n;
   ctx->last_stream = st;
   if (ctx->profile) {
@@ -1109,9 +1121,14 @@ int kvprm_plan_attention(const int32_t* block_table, int32_t max_blocks_per_seq,
     if (seq_lens[b] < 0 || static_cast<int64_t>(seq_lens[b]) > static_cast<int64_t>(max_blocks_per_seq) * 16)
       return KVPRM_EINVAL;
   kvprm::AttnWorkHost w;
-  if (!kvprm::build_attn_work(block_table, seq_lens, n_candidates, max_blocks_per_seq, n_kv_heads, group, n_ctas,
-                              SIZE_MAX, share < 0 ? 0 : (share > 3 ? 3 : share), w))
+  const bool fuse = share >= 0 && (share & KVPRM_PLAN_FUSE) != 0;
+  share = share < 0 ? 0 : (share & ~KVPRM_PLAN_FUSE);
+  if (!(fuse && kvprm::build_attn_work_fused(block_table, seq_lens, n_candidates, max_blocks_per_seq, n_kv_heads,
+                                             group, n_ctas, SIZE_MAX, w)) &&
+      !kvprm::build_attn_work(block_table, seq_lens, n_candidates, max_blocks_per_seq, n_kv_heads, group, n_ctas,
+                              SIZE_MAX, share > 3 ? 3 : share, w))
     return KVPRM_ECAPACITY;
+  plan->fuse_cs = w.fuse_cs;
   plan->n_segs = static_cast<int32_t>(w.segs.size());
   plan->n_ctas = w.n_ctas;
   plan->n_pages = static_cast<int32_t>(w.pages.size());

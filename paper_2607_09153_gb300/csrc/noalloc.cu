@@ -193,6 +193,7 @@ extern "C" int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, co
   wk.n_tc = work.n_tc;   // 0: this entry point schedules shared pages on the persistent kernel only
   wk.tc_cta = nullptr;
   wk.n_tc_ctas = 0;
+  wk.fuse_cs = 0;   // the persistent plan and a combine launch
 
   // the error word must start at zero; everything else is written before it is read
   if (cudaMemsetAsync(err, 0, sizeof(int), st) != cudaSuccess) return KVPRM_ECUDA;
@@ -212,7 +213,8 @@ extern "C" int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, co
   if (kvprm::launch_split_hilo(q, static_cast<int64_t>(n) * n_q_heads * head_dim, Q, st) != cudaSuccess)
     return KVPRM_ECUDA;
   const kvprm::AttnMerge mg{q, k_self, v_self, ohi, olo, out, nullptr};
-  if (kvprm::launch_attention(as, wk, &tm, 0, Q.hi, Q.lo, po, pml, err, st, false) != cudaSuccess) return KVPRM_ECUDA;
+  if (kvprm::launch_attention(as, wk, &tm, 0, Q.hi, Q.lo, po, pml, mg, err, st, false) != cudaSuccess)
+    return KVPRM_ECUDA;
   if (kvprm::launch_attn_combine(as, wk, n, po, pml, mg, st, false) != cudaSuccess) return KVPRM_ECUDA;
   return KVPRM_OK;
 }

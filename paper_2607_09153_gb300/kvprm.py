@@ -51,7 +51,10 @@ class KvprmAttnPlan(ctypes.Structure):
                 ("cands", ctypes.POINTER(ctypes.c_int32)), ("cands_cap", ctypes.c_int64),
                 ("slots", ctypes.POINTER(ctypes.c_int32)), ("slots_cap", ctypes.c_int64),
                 ("slot_base", ctypes.POINTER(ctypes.c_int32)), ("nslots", ctypes.POINTER(ctypes.c_int32)),
-                ("n_tc_ctas", ctypes.c_int32), ("tc_cta", ctypes.POINTER(ctypes.c_int32)), ("tc_cta_cap", ctypes.c_int64)]
+                ("n_tc_ctas", ctypes.c_int32), ("tc_cta", ctypes.POINTER(ctypes.c_int32)), ("tc_cta_cap", ctypes.c_int64),
+                ("fuse_cs", ctypes.c_int32)]
+
+KVPRM_PLAN_FUSE = 16
 
 
 _lib = None
@@ -179,8 +182,9 @@ def kvprm_attention_noalloc(kv_layer_ptr: int, n_pages: int, block_table, seq_le
 
 def kvprm_plan_attention(block_table, seq_lens, n_kv_heads: int, group: int, n_ctas: int, share: int = 1) -> dict:
     """The attention schedule of a call (host only): dict of numpy arrays
-    segs [n_segs][8], cta_seg, pages, cands, slots, slot_base, nslots.  share: 0 none,
-    1 shared runs on the persistent CTAs, 2 shared pages on the tensor cores."""
+    segs [n_segs][8], cta_seg, pages, cands, slots, slot_base, nslots, fuse_cs.  share: 0 none,
+    1 shared runs on the persistent CTAs, 2 shared pages on the tensor cores, 3 as 2 with the SMs
+    split between the two launches; | KVPRM_PLAN_FUSE tries the fused-combine plan first."""
     bt, sl = _i32(block_table), _i32(seq_lens)
     n = len(sl)
     mb = bt.shape[1] if bt.ndim == 2 and bt.shape[1] > 0 else 1
@@ -211,7 +215,7 @@ def kvprm_plan_attention(block_table, seq_lens, n_kv_heads: int, group: int, n_c
             "slots": bufs["slots"][:plan.n_slot_refs], "slot_base": bufs["slot_base"][:n * n_kv_heads],
             "nslots": bufs["nslots"][:n * n_kv_heads], "n_ctas": plan.n_ctas, "n_slots": plan.n_slots,
             "tc_cta": bufs["tc_cta"][:plan.n_tc_ctas + 1] if plan.n_tc_ctas else np.zeros(1, np.int32),
-            "n_tc_ctas": plan.n_tc_ctas}
+            "n_tc_ctas": plan.n_tc_ctas, "fuse_cs": plan.fuse_cs}
 
 
 def kvprm_set_debug(ctx, flags: int) -> None:

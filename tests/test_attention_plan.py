@@ -19,10 +19,12 @@ PRIVATE_COST, SHARED_COST_PER_CAND = 4, 2   # the planner's per-page cost model
 
 def check_plan(bt, sl, n_kv, group, n_ctas, share):
     share = int(share)
+    flags = share & kp.KVPRM_PLAN_FUSE
     bt = np.asarray(bt, np.int32)
     sl = np.asarray(sl, np.int32)
     n = len(sl)
     p = kp.kvprm_plan_attention(bt, sl, n_kv, group, n_ctas, share)
+    share &= ~flags
     segs, cta = p["segs"], p["cta_seg"]
     # expected multiset of (b, g, page, valid tokens)
     want = collections.Counter()
@@ -171,6 +173,49 @@ def test_concurrent_split_shares_the_sms():
     assert p3["n_tc_ctas"] >= 1 and p3["n_ctas"] >= 1 and p3["n_tc_ctas"] + p3["n_ctas"] <= 64
     p2 = check_plan(bt, sl, 2, 7, 64, 2)   # serial: each launch planned over all SMs
     assert p2["n_ctas"] == 64 and p2["n_tc_ctas"] == 64
+
+
+@pytest.mark.parametrize("name, cs", [("tiny", 8), ("qwen1p5b_b16_l2048", 4), ("long8b_b8_l32768", 0),
+                                      ("beam7b_b64_p4096_s512", 0), ("mcts7b_b256_d4", 0)])
+def test_fused_combine_plan(name, cs):
+    # equal lengths, no sharing, group <= 8 and few pages per CTA: pair p on cluster p, one slot per rank
+    w = ks.make_workload(name)
+    a = w.arch
+    n_kv, group = a.n_kv_heads, a.n_q_heads // a.n_kv_heads
+    p = check_plan(w.block_table, w.seq_lens, n_kv, group, 152, 3 | kp.KVPRM_PLAN_FUSE)
+    assert p["fuse_cs"] == cs
+    if not cs:
+        return
+    n = len(w.seq_lens)
+    assert p["n_ctas"] == n * n_kv * cs <= 152 and len(p["segs"]) == p["n_ctas"]
+    for k in range(p["n_ctas"]):
+        (seg,) = p["segs"][p["cta_seg"][k]:p["cta_seg"][k + 1]]
+        pr, r = divmod(k, cs)
+        b, g = divmod(pr, n_kv)
+        assert seg[0] == 0 and seg[2] == b and seg[1] == g and seg[7] == pr * cs + r
+        npg = (int(w.seq_lens[b]) + 15) // 16
+        assert seg[5] == (r + 1) * npg // cs - r * npg // cs and seg[5] <= 64
+    assert (p["slot_base"] == np.arange(n * n_kv) * cs).all() and (p["nslots"] == cs).all()
+
+
+@pytest.mark.parametrize("case", ["ragged", "shared", "repeat", "empty", "wide_group"])
+def test_fused_combine_plan_declines(case):
+    n, npg = 6, 8
+    bt = np.arange(n * npg, dtype=np.int32).reshape(n, npg)
+    sl = np.full(n, 16 * npg, np.int32)
+    group = 4
+    if case == "ragged":
+        sl[0] = 16 * 4   # 4 pages against 8
+    elif case == "shared":
+        bt[1, 0] = bt[0, 0]
+    elif case == "repeat":
+        bt[2, 3] = bt[2, 2]
+    elif case == "empty":
+        sl[3] = 0
+    else:
+        group = 12
+    p = check_plan(bt, sl, 2, group, 152, 1 | kp.KVPRM_PLAN_FUSE)
+    assert p["fuse_cs"] == 0
 
 
 def test_repeated_page_in_one_candidate_stays_private():

@@ -94,6 +94,22 @@ def test_layer_shapes(arch, lens):
     compare(w, t, gpu_rewards=r, gpu_attn=attn, label=f"arch {arch.d_model}/{arch.n_q_heads}/{arch.n_kv_heads}")
 
 
+@pytest.mark.parametrize("lens", [[16 * 9] * 4,            # 8 (candidate, kv head) pairs: clusters of 8
+                                  [16 * 33 - 5] * 20,       # 40 pairs: clusters of 2
+                                  [40] * 76,                # 152 pairs: one CTA each
+                                  [100, 110, 120, 125]])    # about equal lengths, ragged last pages
+@pytest.mark.parametrize("fused", [True, False])
+def test_fused_combine(lens, fused, monkeypatch):
+    # the combine merged by each cluster's rank 0 inside the attention launch, and the same calls
+    # with the persistent plan and a combine launch
+    if not fused:
+        monkeypatch.setenv("KVPRM_NO_FUSED_COMBINE", "1")
+    t = ks.Tables.make(0.2)
+    w = ks.distinct("fused", ks.ARCH_TINY, 41 + len(lens), lens, gain_std=0.2)
+    r, attn, _, _ = run_gpu(w, t)
+    compare(w, t, gpu_rewards=r, gpu_attn=attn, label=f"fused={fused} lens={lens[:2]}x{len(lens)}")
+
+
 def test_attention_teacher_forced():
     """kvprm_attention on given fp32 q / self k / self v against the oracle's read-out."""
     torch = require_gpu()
