@@ -101,7 +101,8 @@ struct AttnSmem {
   static constexpr uint32_t kMergeM = kMergeO + kConsumerWarps * 8 * HD * 4;  // [8][8] running max
   static constexpr uint32_t kMergeL = kMergeM + kConsumerWarps * 8 * 4;       // [8][8] running sum
   static constexpr uint32_t kBars = kMergeL + kConsumerWarps * 8 * 4;   // full[kStages], empty[kStages], seg_full, seg_free
-  static constexpr uint32_t kEnd = kBars + (2 * kStages + 2) * 8;
+  static constexpr uint32_t kSelf = kBars + (2 * kStages + 2) * 8;   // fused combine: [8] own logits
+  static constexpr uint32_t kEnd = kSelf + 8 * 4;
   static constexpr size_t kDynamic = kEnd + 1024;   // + alignment slack
 };
 static_assert(AttnSmem<128>::kDynamic <= 227 * 1024, "attention shared memory exceeds the per-block limit");
@@ -235,6 +236,27 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
       }
     }
     if (lane == 0) trace_event(ts, 1);   // this warp has scored every page of its CTA
+    if (!TWO_ROWS && wk.fuse_cs > 0) {
+      // fused combine (one private run per CTA): once every consumer warp has stashed its state and
+      // read its last stage, warp r folds query row r of the eight states into the idle ring
+      named_bar_sync(3, kConsumerWarps * 32);
+      if (warp < group) {
+        float* st_o = reinterpret_cast<float*>(ring);
+        merge_row<HD>(warp, mo, mm, ml, lane, st_o + warp * HD, st_o + 8 * HD + 2 * warp);
+      }
+    }
+    if (!TWO_ROWS && wk.fuse_cs > 0 && warp < group) {
+      // and the verify token's own logit of head `warp` (q . k_self / sqrt(hd), log2 units)
+      const int pr = blockIdx.x / wk.fuse_cs, b = pr / n_kv, g = pr - b * n_kv;
+      const float* qr = mg.q + (static_cast<int64_t>(b) * n_q + g * group + warp) * HD;
+      const float* kr = mg.kself + (static_cast<int64_t>(b) * n_kv + g) * HD;
+      float dot = 0.f;
+#pragma unroll
+      for (int j = 0; j < HD / 32; ++j) dot += __ldcg(qr + lane + 32 * j) * __ldcg(kr + lane + 32 * j);
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
+      if (lane == 0) reinterpret_cast<float*>(base + SM::kSelf)[warp] = dot * (kLog2e * rsqrtf(static_cast<float>(HD)));
+    }
   } else if (warp == kMergerWarp && !TWO_ROWS) {
     // ------------------------------------------------ merger
     // For every private segment, in order: fold the eight consumer warps'
@@ -242,7 +264,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
     //   M = max_w m_w, L = sum_w 2^(m_w - M) l_w, O = sum_w 2^(m_w - M) O_w.
     uint32_t k = 0;
     bool ok = true;
-    for (int si = seg0; si < seg1; ++si) {
+    for (int si = wk.fuse_cs > 0 ? seg1 : seg0; si < seg1; ++si) {   // fused plans: the consumers merge
       const AttnSeg sg = wk.segs[si];
       if (sg.kind != 0) continue;
       if (ok) ok = __all_sync(0xffffffffu, mbar_wait(seg_full, k & 1u, err));
@@ -254,19 +276,74 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
     if (lane == 0) trace_event(ts, 2);   // every private run of this CTA is merged
   }
   if (!TWO_ROWS && wk.fuse_cs > 0) {   // fused plans have group <= 8
-    // The cluster scored one (candidate, kv head): once every rank's partial slot is written
-    // (the cluster barrier releases them), rank 0 merges the slots with the verify token's own
-    // entry, as the combine launch would.  Its ring is idle by now and holds the merge scratch;
-    // warps 0..7 passed the grid-dependency wait, so q and the self k / v are visible to them.
+    // The cluster scored one (candidate, kv head); every rank left its (M, L, O) per query row at
+    // the start of its ring and the verify token's own logits in kSelf.  Rank k then produces
+    // head-dimension slice k of every row, reading the ranks' states through distributed shared
+    // memory and merging them with the verify token's own entry:
+    //   M* = max(s_self, M_j), o = (2^(s_self - M*) v_self + sum_j 2^(M_j - M*) O_j)
+    //                              / (2^(s_self - M*) + sum_j 2^(M_j - M*) L_j).
+    // The second cluster barrier keeps every rank's shared memory until all have read it.  Only
+    // the consumer warps passed the grid-dependency wait (v_self is written by the preceding
+    // kernel), so they alone produce the outputs.
+    constexpr int kMergeThreads = kConsumerWarps * 32;
+    constexpr int kOut = (8 * HD + kMergeThreads - 1) / kMergeThreads;
+    const int cs = wk.fuse_cs, pr = blockIdx.x / cs, b = pr / n_kv, g = pr - b * n_kv;
+    const int slice = HD / cs, d0 = static_cast<int>(cluster_rank()) * slice;
+    const bool mine = warp < kConsumerWarps;
+    const int64_t hq0 = static_cast<int64_t>(b) * n_q + static_cast<int64_t>(g) * group;
+    float vsf[kOut];
+#pragma unroll
+    for (int i = 0; i < kOut; ++i) {   // v_self of this thread's outputs, loaded before the barrier
+      const int idx = threadIdx.x + i * kMergeThreads;
+      vsf[i] = (mine && idx < group * slice)
+                   ? __ldcg(mg.vself + (static_cast<int64_t>(b) * n_kv + g) * HD + d0 + idx % slice)
+                   : 0.f;
+    }
     __syncwarp();
     cluster_sync();
-    if (cluster_rank() == 0 && warp < kConsumerWarps) {
-      const int pr = blockIdx.x / wk.fuse_cs, b = pr / n_kv, g = pr - b * n_kv;
-      combine_group<HD, 8>(threadIdx.x, b, g, wk.slot_base[pr], wk.nslots[pr], n_q, n_kv, group,
-                                           part_o, part_ml, mg, base,
-                                           [] { named_bar_sync(2, kConsumerWarps * 32); });
-      if (threadIdx.x == 0) trace_event(ts, 3);   // the pair's output is written
+    if (mine) {
+      const float* st_o = reinterpret_cast<const float*>(ring);
+      const float* st_ml = st_o + 8 * HD;
+      const float* s_self = reinterpret_cast<const float*>(base + SM::kSelf);
+#pragma unroll
+      for (int i = 0; i < kOut; ++i) {
+        const int idx = threadIdx.x + i * kMergeThreads;
+        if (idx >= group * slice) break;
+        const int r = idx / slice, d = d0 + idx - r * slice;
+        const float ss = s_self[r];
+        float Mk[8], Lk[8], Ok[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          if (k >= cs) break;
+          Mk[k] = ld_cluster(st_ml + 2 * r, k);
+          Lk[k] = ld_cluster(st_ml + 2 * r + 1, k);
+          Ok[k] = ld_cluster(st_o + r * HD + d, k);
+        }
+        float Mt = ss;
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+          if (k < cs) Mt = fmaxf(Mt, Mk[k]);
+        const float ws = exp2f(ss - Mt);
+        float num = ws * vsf[i], den = ws;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          if (k >= cs || Mk[k] == -INFINITY) continue;   // a rank with no pages
+          const float f = exp2f(Mk[k] - Mt);
+          num += f * Ok[k];
+          den += f * Lk[k];
+        }
+        const float out = num / den;
+        const int64_t o = (hq0 + r) * HD + d;
+        const __nv_bfloat16 hi = __float2bfloat16_rn(out);
+        mg.o_hi[o] = hi;
+        mg.o_lo[o] = __float2bfloat16_rn(out - __bfloat162float(hi));
+        if (mg.out_f32) mg.out_f32[o] = out;
+        if (mg.dbg) mg.dbg[o] = out;
+      }
+      if (threadIdx.x == 0) trace_event(ts, 3);   // this rank's outputs are written
     }
+    __syncwarp();
+    cluster_sync();
   }
   trace_end(ts);
 }

@@ -267,34 +267,42 @@ __device__ __forceinline__ void store_state_slot(const WarpState<HD>& st, int sl
   }
 }
 
-// One warp folds the eight stashed warp states of a private run into partial
-// slot `slot`:  M = max_w m_w, L = sum_w 2^(m_w - M) l_w, O = sum_w 2^(m_w - M) O_w.
+// One warp folds query row r of the eight stashed warp states of a private run:
+//   M = max_w m_w, L = sum_w 2^(m_w - M) l_w, O = sum_w 2^(m_w - M) O_w
+// into dst_o[0 .. HD) and dst_ml[0 .. 2) = (M, L).
+template <int HD>
+__device__ __forceinline__ void merge_row(int r, const float* mo, const float* mm, const float* ml, int lane,
+                                          float* dst_o, float* dst_ml) {
+  constexpr int kPer = HD / 32;
+  float mw[kStateWarps], M = -INFINITY;
+#pragma unroll
+  for (int w = 0; w < kStateWarps; ++w) {
+    mw[w] = mm[w * 8 + r];
+    M = fmaxf(M, mw[w]);
+  }
+  float acc[kPer], L = 0.f;
+#pragma unroll
+  for (int j = 0; j < kPer; ++j) acc[j] = 0.f;
+#pragma unroll
+  for (int w = 0; w < kStateWarps; ++w) {
+    if (mw[w] == -INFINITY) continue;   // an idle warp: its O rows are not written
+    const float f = exp2f(mw[w] - M);
+    L += f * ml[w * 8 + r];
+#pragma unroll
+    for (int j = 0; j < kPer; ++j) acc[j] += f * mo[(w * 8 + r) * HD + lane + 32 * j];
+  }
+#pragma unroll
+  for (int j = 0; j < kPer; ++j) dst_o[lane + 32 * j] = acc[j];
+  if (lane == 0) *reinterpret_cast<float2*>(dst_ml) = make_float2(M, L);
+}
+
+// One warp folds the eight stashed warp states of a private run into partial slot `slot`, row by row.
 template <int HD>
 __device__ __forceinline__ void merge_warp_states(int group, const float* mo, const float* mm, const float* ml,
                                                   int slot, int lane, float* part_o, float* part_ml) {
-  constexpr int kPer = HD / 32;
   for (int r = 0; r < group; ++r) {
-    float mw[kStateWarps], M = -INFINITY;
-#pragma unroll
-    for (int w = 0; w < kStateWarps; ++w) {
-      mw[w] = mm[w * 8 + r];
-      M = fmaxf(M, mw[w]);
-    }
-    float acc[kPer], L = 0.f;
-#pragma unroll
-    for (int j = 0; j < kPer; ++j) acc[j] = 0.f;
-#pragma unroll
-    for (int w = 0; w < kStateWarps; ++w) {
-      if (mw[w] == -INFINITY) continue;   // an idle warp: its O rows are not written
-      const float f = exp2f(mw[w] - M);
-      L += f * ml[w * 8 + r];
-#pragma unroll
-      for (int j = 0; j < kPer; ++j) acc[j] += f * mo[(w * 8 + r) * HD + lane + 32 * j];
-    }
     const int64_t pr = static_cast<int64_t>(slot) * group + r;
-#pragma unroll
-    for (int j = 0; j < kPer; ++j) part_o[pr * HD + lane + 32 * j] = acc[j];
-    if (lane == 0) *reinterpret_cast<float2*>(part_ml + pr * 2) = make_float2(M, L);
+    merge_row<HD>(r, mo, mm, ml, lane, part_o + pr * HD, part_ml + pr * 2);
   }
 }
 

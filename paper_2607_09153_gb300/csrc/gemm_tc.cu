@@ -52,14 +52,6 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~static_cast<uintptr_t>(1023));
 }
 
-// Load a float at the same shared-memory offset in cluster CTA `rank`.
-__device__ __forceinline__ float ld_peer(const float* local, uint32_t rank) {
-  uint32_t a;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(smem_u32(local)), "r"(rank));
-  float v;
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(a) : "memory");
-  return v;
-}
 __device__ __forceinline__ void store_hilo(__nv_bfloat16* hi, __nv_bfloat16* lo, int64_t i, float x) {
   const __nv_bfloat16 h = __float2bfloat16_rn(x);
   hi[i] = h;
@@ -238,7 +230,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
         const int r = step == 2 ? (k & 7) : k;
         const int cc = (step == 2 && k >= 8) ? c + 1 : c;
         const bool use = r < cs && (cc == c || two);
-        v[k] = use ? ld_peer(acc + cc * kBM + m, static_cast<uint32_t>(r)) : 0.f;
+        v[k] = use ? ld_cluster(acc + cc * kBM + m, static_cast<uint32_t>(r)) : 0.f;
       }
       if (step == 2) {
         float s0 = 0.f, s1 = 0.f;

@@ -310,6 +310,15 @@ __device__ __forceinline__ void cluster_sync() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
+// Load a float at the same shared-memory address in cluster CTA `rank` (distributed shared memory).
+__device__ __forceinline__ float ld_cluster(const float* local, uint32_t rank) {
+  uint32_t a;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(smem_u32(local)), "r"(rank));
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(a) : "memory");
+  return v;
+}
+
 // ---------------------------------------------------------------- PDL
 // Programmatic dependent launch: wait for the preceding grid's completion
 // (and memory flush) / allow the next grid to begin launching.
