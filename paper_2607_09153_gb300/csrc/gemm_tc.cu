@@ -85,6 +85,11 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
   const int kt1 = min(k_tiles, kt0 + kps);
   const int nk = kt1 > kt0 ? kt1 - kt0 : 0;
   const bool silu = ep.mode == GemmEpilogue::SILU;
+  // this rank's candidate columns in the reduction and the epilogue
+  const int cols = n_pad / cs;
+  const int cbeg = static_cast<int>(rank) * cols;
+  const int cend = min(cbeg + cols, ep.n_valid);
+  const int nc = cend > cbeg ? cend - cbeg : 0;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < stages; ++s) {
@@ -146,6 +151,18 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       tma_load_2d(st + kWTileBytes, &tmX, &full[s], (kt0 + i) * kBK, 0, pol_x);
       if (has_lo) tma_load_2d(st + kWTileBytes + x_bytes, &tmXlo, &full[s], (kt0 + i) * kBK, 0, pol_x);
     }
+  } else if (warp >= 2) {
+    // ---------------- while the weights stream: the RMSNorm factor of each of this rank's columns
+    // (QKV, SILU), from the residual stream's tile sums of squares the preceding kernel wrote; the
+    // parking barrier below orders these writes before the epilogue reads them
+    grid_dep_wait();
+    if (ep.rs_sumsq)
+      for (int t0 = threadIdx.x - 64; t0 < nc; t0 += blockDim.x - 64) {   // nc <= 256 columns
+        const int c = cbeg + t0;
+        float ssum = 0.f;
+        for (int t = 0; t < ep.rs_tiles; ++t) ssum += ep.rs_sumsq[static_cast<int64_t>(t) * ep.n_valid + c];
+        rsc[t0] = 1.0f / sqrtf(ssum / ep.rs_d + ep.rs_eps);
+      }
   } else if (warp == 1 && nk > 0) {
     // ---------------- MMA issuer (the whole warp; one elected lane issues)
     // With the hi and lo activation tiles stored back to back (2 n_pad rows
@@ -213,10 +230,6 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
 
   // ---------------- reduce this rank's candidate columns over the cluster, then the epilogue
   grid_dep_wait();   // outputs may still be read by kernels that precede this one
-  const int cols = n_pad / cs;
-  const int cbeg = static_cast<int>(rank) * cols;
-  const int cend = min(cbeg + cols, ep.n_valid);
-  const int nc = cend > cbeg ? cend - cbeg : 0;
   // Step 1: acc[c][m] <- sum over ranks of acc_r[c][m] for this rank's columns
   // (only this rank reads them, so it may overwrite its own copy).  Two columns
   // per round trip when the cluster has <= 8 ranks, all peer loads in flight.
@@ -251,15 +264,11 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     }
   }
   if (threadIdx.x == 0) trace_event(ts, 4);   // this rank's columns are reduced over the cluster
-  // the RMSNorm factor of each of this rank's columns (QKV, SILU)
-  if (ep.rs_sumsq)
-    for (int t0 = threadIdx.x; t0 < nc; t0 += blockDim.x) {   // nc <= 256 columns
-      const int c = cbeg + t0;
-      float ssum = 0.f;
-      for (int t = 0; t < ep.rs_tiles; ++t) ssum += ep.rs_sumsq[static_cast<int64_t>(t) * ep.n_valid + c];
-      rsc[t0] = 1.0f / sqrtf(ssum / ep.rs_d + ep.rs_eps);
-    }
-  __syncthreads();
+  // no peer reads this CTA's shared memory any more: arrive on the exit barrier now and wait for the
+  // peers only before exiting, so the barrier's latency hides behind the epilogue
+  __syncwarp();
+  cluster_arrive();
+  __syncthreads();   // every warp's reduced columns are in acc
   if (threadIdx.x == 0) trace_event(ts, 5);
   // Step 2: the epilogue over (row, column) pairs, all threads in parallel
   if (ep.mode == GemmEpilogue::PLAIN) {
@@ -334,9 +343,9 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     }
   }
   (void)nc;
-  __syncthreads();
-  if (threadIdx.x == 0) trace_event(ts, 6);   // epilogue written
-  cluster_sync();   // peers have finished reading this CTA's partial
+  if (threadIdx.x == 0) trace_event(ts, 6);   // this thread's epilogue written
+  __syncwarp();
+  cluster_wait();   // peers have finished reading this CTA's partial
   if (threadIdx.x == 0) trace_event(ts, 7);
   if (warp == 1) tmem_dealloc(tmem, tmem_cols);
   trace_end(ts);
