@@ -101,8 +101,8 @@ struct AttnSmem {
   static constexpr uint32_t kMergeM = kMergeO + kConsumerWarps * 8 * HD * 4;  // [8][8] running max
   static constexpr uint32_t kMergeL = kMergeM + kConsumerWarps * 8 * 4;       // [8][8] running sum
   static constexpr uint32_t kBars = kMergeL + kConsumerWarps * 8 * 4;   // full[kStages], empty[kStages], seg_full, seg_free
-  static constexpr uint32_t kSelf = kBars + (2 * kStages + 2) * 8;   // fused combine: [8] own logits
-  static constexpr uint32_t kEnd = kSelf + 8 * 4;
+  static constexpr uint32_t kSelf = kBars + (2 * kStages + 2) * 8;   // fused combine: [8] own logits,
+  static constexpr uint32_t kEnd = kSelf + (8 + HD) * 4;                // then v_self [HD]
   static constexpr size_t kDynamic = kEnd + 1024;   // + alignment slack
 };
 static_assert(AttnSmem<128>::kDynamic <= 227 * 1024, "attention shared memory exceeds the per-block limit");
@@ -182,6 +182,24 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
     // no warp can arrive for a slot's next use early.
     grid_dep_wait();   // q is written by the preceding kernel
     if (warp == 0 && lane == 0) trace_event(ts, 0);   // the query is ready
+    if (!TWO_ROWS && wk.fuse_cs > 0) {
+      // fused combine, before the pages: the verify token's own logit of head `warp`
+      // (q . k_self / sqrt(hd), log2 units) and the pair's v_self, into shared memory
+      const int pr = blockIdx.x / wk.fuse_cs, b = pr / n_kv, g = pr - b * n_kv;
+      const float* kr = mg.kself + (static_cast<int64_t>(b) * n_kv + g) * HD;
+      float* s_self = reinterpret_cast<float*>(base + SM::kSelf);
+      if (warp < group) {
+        const float* qr = mg.q + (static_cast<int64_t>(b) * n_q + g * group + warp) * HD;
+        float dot = 0.f;
+#pragma unroll
+        for (int j = 0; j < HD / 32; ++j) dot += __ldcg(qr + lane + 32 * j) * __ldcg(kr + lane + 32 * j);
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
+        if (lane == 0) s_self[warp] = dot * (kLog2e * rsqrtf(static_cast<float>(HD)));
+      }
+      for (int d = threadIdx.x; d < HD; d += kConsumerWarps * 32)
+        s_self[8 + d] = __ldcg(mg.vself + (static_cast<int64_t>(b) * n_kv + g) * HD + d);
+    }
     bool ok = true;
     uint32_t u = 0, n_priv = 0;
     for (int si = seg0; si < seg1; ++si) {
@@ -245,18 +263,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
         merge_row<HD>(warp, mo, mm, ml, lane, st_o + warp * HD, st_o + 8 * HD + 2 * warp);
       }
     }
-    if (!TWO_ROWS && wk.fuse_cs > 0 && warp < group) {
-      // and the verify token's own logit of head `warp` (q . k_self / sqrt(hd), log2 units)
-      const int pr = blockIdx.x / wk.fuse_cs, b = pr / n_kv, g = pr - b * n_kv;
-      const float* qr = mg.q + (static_cast<int64_t>(b) * n_q + g * group + warp) * HD;
-      const float* kr = mg.kself + (static_cast<int64_t>(b) * n_kv + g) * HD;
-      float dot = 0.f;
-#pragma unroll
-      for (int j = 0; j < HD / 32; ++j) dot += __ldcg(qr + lane + 32 * j) * __ldcg(kr + lane + 32 * j);
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
-      if (lane == 0) reinterpret_cast<float*>(base + SM::kSelf)[warp] = dot * (kLog2e * rsqrtf(static_cast<float>(HD)));
-    }
+
   } else if (warp == kMergerWarp && !TWO_ROWS) {
     // ------------------------------------------------ merger
     // For every private segment, in order: fold the eight consumer warps'
@@ -282,23 +289,15 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
     // memory and merging them with the verify token's own entry:
     //   M* = max(s_self, M_j), o = (2^(s_self - M*) v_self + sum_j 2^(M_j - M*) O_j)
     //                              / (2^(s_self - M*) + sum_j 2^(M_j - M*) L_j).
-    // The second cluster barrier keeps every rank's shared memory until all have read it.  Only
-    // the consumer warps passed the grid-dependency wait (v_self is written by the preceding
-    // kernel), so they alone produce the outputs.
+    // The second cluster barrier keeps every rank's shared memory until all have read it.  The
+    // consumer warps produce the outputs (they wrote the logits and v_self, after the
+    // grid-dependency wait).
     constexpr int kMergeThreads = kConsumerWarps * 32;
     constexpr int kOut = (8 * HD + kMergeThreads - 1) / kMergeThreads;
     const int cs = wk.fuse_cs, pr = blockIdx.x / cs, b = pr / n_kv, g = pr - b * n_kv;
     const int slice = HD / cs, d0 = static_cast<int>(cluster_rank()) * slice;
     const bool mine = warp < kConsumerWarps;
     const int64_t hq0 = static_cast<int64_t>(b) * n_q + static_cast<int64_t>(g) * group;
-    float vsf[kOut];
-#pragma unroll
-    for (int i = 0; i < kOut; ++i) {   // v_self of this thread's outputs, loaded before the barrier
-      const int idx = threadIdx.x + i * kMergeThreads;
-      vsf[i] = (mine && idx < group * slice)
-                   ? __ldcg(mg.vself + (static_cast<int64_t>(b) * n_kv + g) * HD + d0 + idx % slice)
-                   : 0.f;
-    }
     __syncwarp();
     cluster_sync();
     if (mine) {
@@ -324,7 +323,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
         for (int k = 0; k < 8; ++k)
           if (k < cs) Mt = fmaxf(Mt, Mk[k]);
         const float ws = exp2f(ss - Mt);
-        float num = ws * vsf[i], den = ws;
+        float num = ws * s_self[8 + d], den = ws;
 #pragma unroll
         for (int k = 0; k < 8; ++k) {
           if (k >= cs || Mk[k] == -INFINITY) continue;   // a rank with no pages
