@@ -46,7 +46,8 @@ constexpr int kBK = 64;
 constexpr uint32_t kWTileBytes = kBM * kBK * 2;   // 16 KB
 // after the ring: barriers, TMEM slot and 64 block-sum floats (512 B), then 256
 // per-column RMSNorm factors (1 KB)
-constexpr size_t kTailBytes = 512 + 1024;
+constexpr size_t kTailBytes = 512 + 1024 + 4096;   // barriers, RMSNorm factors, preloaded residual
+constexpr int kHPreCols = 8;                        // residual columns preloaded per rank (128 rows each)
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -76,6 +77,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(done + 1);
   float* red = reinterpret_cast<float*>(tmem_slot + 4);   // 64 floats for per-column block sums
   float* rsc = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full) + 512);   // RMSNorm factor per column
+  float* hpre = rsc + 256;   // RESID: this rank's columns of h for the tile's rows, [c - cbeg][128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int m_tile = blockIdx.x / cs;
@@ -90,6 +92,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
   const int cbeg = static_cast<int>(rank) * cols;
   const int cend = min(cbeg + cols, ep.n_valid);
   const int nc = cend > cbeg ? cend - cbeg : 0;
+  const bool hpreload = ep.mode == GemmEpilogue::RESID && nc <= kHPreCols;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < stages; ++s) {
@@ -111,9 +114,9 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
   // Let the next kernel in the stream start its own independent prologue and
-  // streaming now; it waits for this grid's completion before touching what
-  // this grid writes.
-  grid_dep_launch();
+  // streaming now (or, with late_trigger, once the partials are parked); it
+  // waits for this grid's completion before touching what this grid writes.
+  if (!ep.late_trigger) grid_dep_launch();
 
   if (warp == 0 && lane == 0 && nk > 0) {
     // ---------------- TMA producer
@@ -162,6 +165,13 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
         float ssum = 0.f;
         for (int t = 0; t < ep.rs_tiles; ++t) ssum += ep.rs_sumsq[static_cast<int64_t>(t) * ep.n_valid + c];
         rsc[t0] = 1.0f / sqrtf(ssum / ep.rs_d + ep.rs_eps);
+      }
+    // RESID: the residual values the epilogue adds to, read now rather than after the MMAs, when
+    // the next kernel's weight stream may be competing for the memory system
+    if (hpreload)
+      for (int idx = threadIdx.x - 64; idx < nc * kBM; idx += blockDim.x - 64) {
+        const int c = cbeg + idx / kBM, gm = m_tile * kBM + idx % kBM;
+        hpre[idx] = gm < ep.M ? ep.h[static_cast<int64_t>(c) * ep.M + gm] : 0.f;
       }
   } else if (warp == 1 && nk > 0) {
     // ---------------- MMA issuer (the whole warp; one elected lane issues)
@@ -227,6 +237,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
   tc_fence_before();
   cluster_sync();   // every rank's partial is parked
   if (threadIdx.x == 0) trace_event(ts, 3);
+  if (ep.late_trigger) grid_dep_launch();
 
   // ---------------- reduce this rank's candidate columns over the cluster, then the epilogue
   grid_dep_wait();   // outputs may still be read by kernels that precede this one
@@ -284,7 +295,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
         float hv = 0.f;
         if (gm < ep.M) {
           float* hp = ep.h + static_cast<int64_t>(c) * ep.M + gm;
-          hv = *hp + acc[c * kBM + m];
+          hv = (hpreload ? hpre[(c - cbeg) * kBM + m] : *hp) + acc[c * kBM + m];
           *hp = hv;
           if (ep.gain_next)
             store_hilo(ep.x_hi, ep.x_lo, static_cast<int64_t>(c) * ep.M + gm, hv * __bfloat162float(ep.gain_next[gm]));

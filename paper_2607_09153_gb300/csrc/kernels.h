@@ -54,6 +54,10 @@ struct GemmEpilogue {
   int ff = 0;            // SILU: output width; up rows start at row ff of W
   __nv_bfloat16* a_hi = nullptr;
   __nv_bfloat16* a_lo = nullptr;
+  // let the next kernel in the stream launch only once this one's partials are parked (after its
+  // first cluster barrier) instead of at entry: a next kernel whose CTAs fit beside this one's on
+  // an SM otherwise slows that barrier by ~2.5 us (measured for the O projection before gate/up)
+  bool late_trigger = false;
 };
 GemmPlan plan_gemm(int M, int K, int n_pad, int num_sms, bool has_lo, bool gate_up);
 cudaError_t gemm_configure();

@@ -561,6 +561,7 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
              "attn_combine");
     kvprm::GemmEpilogue er_o = er;   // h += W_o o; x = h ⊙ g_mlp for the gate/up projection
     er_o.gain_next = ctx->mlp_norm[l];
+    er_o.late_trigger = true;   // gate/up CTAs fit beside the O projection's
     LAUNCH(KVPRM_PROF_GEMM_O,
            kvprm::launch_gemm(P.g_o, &ctx->tm_o[l], &ctx->tm_ohi, &ctx->tm_olo, er_o, np, ctx->err_d, st, pdl, TS),
            "gemm_o");
