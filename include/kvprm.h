@@ -97,6 +97,25 @@ typedef struct kvprm_ctx kvprm_ctx;
  * without a context).  Sec. 4.1 "Architecture". */
 KVPRM_API int kvprm_create(const kvprm_config* cfg, const kvprm_weights* weights, kvprm_ctx** out);
 
+/* How a context schedules the attention of each call (fixed at kvprm_create;
+ * every choice gives the same result up to fp32 rounding order):
+ *  - calls whose candidates all have about the same number of pages (longest
+ *    <= 5/4 of the shortest), share no page and have group <= 8 use the
+ *    fused-combine plan when it leaves <= 64 pages per CTA: one thread-block
+ *    cluster per (candidate, kv head), whose CTAs merge their partial states
+ *    through distributed shared memory, so no combine launch follows
+ *    (KVPRM_PLAN_FUSE below; environment KVPRM_NO_FUSED_COMBINE=1 turns it off);
+ *  - otherwise the persistent plan (kvprm_plan_attention): pages referenced by
+ *    several candidates are scored once per group; with head_dim 128, groups of
+ *    >= 6 candidates go to a tensor-core launch on a share of the SMs that runs
+ *    beside the private pages' launch (a second stream forked and joined inside
+ *    the call; share mode 3), smaller groups to the persistent kernel.
+ *    Environment: KVPRM_NO_SHARING=1 (every page per candidate),
+ *    KVPRM_NO_TC_SHARING=1 (shared groups on the persistent kernel),
+ *    KVPRM_TC_SERIAL=1 (the two launches one after the other, all SMs each).
+ * KVPRM_NO_GRAPH=1 and KVPRM_NO_PDL=1 switch off graph capture and programmatic
+ * dependent launch (for debugging). */
+
 /* Free the workspace.  Waits for work the context enqueued.  NULL is a no-op. */
 KVPRM_API void kvprm_destroy(kvprm_ctx* ctx);
 
