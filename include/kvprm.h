@@ -272,7 +272,11 @@ KVPRM_API int kvprm_resolve(kvprm_ctx* ctx, int32_t b, int64_t* phys_row);
  *             valid tokens of the last page, slot (kind 0) or offset into slots
  *  cta_seg    [n_ctas + 1] first segment of each persistent CTA
  *  pages      physical page ids referenced by segments
- *  cands      candidates of kind-1 and kind-2 segments; slots: their partial slots
+ *  cands      candidates of kind-1 and kind-2 segments; slots: their partial
+ *             slots -- a kind-1 segment of n candidates has (8 / n) * n, slot w
+ *             written by the warp that scores candidate w % n on every
+ *             (8 / n)-th page of each stage (all 8 warps busy for n <= 4); a
+ *             kind-2 segment one per candidate
  *  slot_base, nslots  [n_candidates][n_kv_heads] first slot and slot count
  *  tc_cta     [n_tc_ctas + 1] first segment (index into segs) of each
  *             tensor-core CTA

@@ -68,10 +68,14 @@ constexpr int kThreads = (kConsumerWarps + 2) * 32;
 // half a private page per candidate.
 constexpr int64_t kPrivateCost = 4;
 constexpr int64_t kSharedCostPerCand = 2;
+// A shared run of n candidates is scored by (8 / n) warps per candidate, each taking every
+// (8 / n)-th page of a stage and writing its own partial slot: warp w scores candidate w % n,
+// pages p with p % (8 / n) == w / n, into slot w of the segment.  (n <= 4 keeps every warp busy.)
+__host__ __device__ constexpr int shared_reps(int n_cands) { return kConsumerWarps / n_cands; }
 // a 64-token chunk of the tensor-core attention on one SM, in the same units, when it runs beside
-// the private pages' launch (measured: 1.5-2.1 us per chunk then, against ~0.17 us per private
-// page; ~0.86 us per chunk alone)
-constexpr int64_t kTcChunkCost = 40;
+// the private pages' launch (measured: ~1.8 us per chunk beside the beam suffixes, ~2.2 us beside
+// the MCTS leaves, against ~0.043 us per unit on the private side; ~0.86 us per chunk alone)
+constexpr int64_t kTcChunkCost = 48;
 // pages shared by fewer candidates go to the persistent kernel as kind-1 runs: 2 units per page
 // and candidate there against kTcChunkCost / 4 per page on the tensor cores, whatever the tile's rows
 constexpr size_t kTcMinCands = 6;
@@ -205,9 +209,12 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
     for (int si = seg0; si < seg1; ++si) {
       const AttnSeg sg = wk.segs[si];
       const bool shared = sg.kind == 1;
-      // the candidate this warp scores in this segment, -1 if none
-      const int cand = shared ? (warp < sg.n_cands ? wk.cands[sg.cand + warp] : -1)
+      // the candidate this warp scores in this segment, -1 if none (and, in a shared run, which of the
+      // candidate's replica warps it is)
+      const int reps = shared ? shared_reps(sg.n_cands) : 1;
+      const int cand = shared ? (warp < reps * sg.n_cands ? wk.cands[sg.cand + warp % sg.n_cands] : -1)
                               : (warp < sg.n_pages ? sg.cand : -1);
+      const int part = shared ? warp / sg.n_cands : 0;
       WarpQ<HD> q;
       if (cand >= 0) {
         const int64_t q0 = (static_cast<int64_t>(cand) * n_q + static_cast<int64_t>(sg.g) * group) * HD;
@@ -227,8 +234,8 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
               const uint32_t kb = sbase + warp * SM::kPageBytes;
               process_page<HD, TWO_ROWS>(q, kb, kb + SM::kBlockBytes, valid, lane, st);
             }
-          } else {         // every page of this stage, for this warp's candidate
-            for (int pi = 0; pi < npg; ++pi) {
+          } else {         // this replica's pages of this stage, for this warp's candidate
+            for (int pi = part; pi < npg; pi += reps) {
               const int valid = p0 + pi == sg.n_pages - 1 ? sg.last_valid : 16;
               const uint32_t kb = sbase + pi * SM::kPageBytes;
               process_page<HD, TWO_ROWS>(q, kb, kb + SM::kBlockBytes, valid, lane, st);
@@ -347,9 +354,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
   trace_end(ts);
 }
 
-// The combine: one CTA per (candidate, kv head) running combine_group.
-template <int HD, int ROWS>
-__global__ void __launch_bounds__(CombineShape<HD, ROWS>::W * 32) attn_combine_kernel(
+// The combine: one CTA of W warps per (candidate, kv head) running combine_group.
+template <int HD, int ROWS, int W>
+__global__ void __launch_bounds__(W * 32) attn_combine_kernel(
     const int32_t* __restrict__ slot_base, const int32_t* __restrict__ nslots, int n_q, int n_kv, int group,
     const float* __restrict__ part_o, const float* __restrict__ part_ml, AttnMerge mg, unsigned long long* ts) {
   trace_begin(ts);
@@ -359,8 +366,8 @@ __global__ void __launch_bounds__(CombineShape<HD, ROWS>::W * 32) attn_combine_k
   const int first = slot_base[cg], ns = nslots[cg];   // host-uploaded before the call: no wait needed
   grid_dep_wait();   // the partials (and q, k_self, v_self) are written by earlier kernels
   if (threadIdx.x == 0) trace_event(ts, 0);
-  combine_group<HD, ROWS>(threadIdx.x, b, g, first, ns, n_q, n_kv, group, part_o, part_ml, mg, csm,
-                          [] { __syncthreads(); });
+  combine_group<HD, ROWS, W>(threadIdx.x, b, g, first, ns, n_q, n_kv, group, part_o, part_ml, mg, csm,
+                             [] { __syncthreads(); });
   if (threadIdx.x == 0) trace_event(ts, 1);
   trace_end(ts);
 }
@@ -1031,9 +1038,9 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
           s.slot = ns;
           ns += group > 8 ? std::min(s.n_pages, kConsumerWarps) : 1;
         } else {
-          s.slot = static_cast<int>(w.slots.size());
-          for (int k2 = 0; k2 < r.n_cands; ++k2)
-            w.slots.push_back(w.nslots[static_cast<size_t>(w.cands[r.cand + k2]) * n_kv + g]++);
+          s.slot = static_cast<int>(w.slots.size());   // slot w of the segment: warp w (shared_reps)
+          for (int w2 = 0; w2 < shared_reps(r.n_cands) * r.n_cands; ++w2)
+            w.slots.push_back(w.nslots[static_cast<size_t>(w.cands[r.cand + w2 % r.n_cands]) * n_kv + g]++);
         }
         w.segs.push_back(s);
         seg_cta.push_back(k);
@@ -1100,9 +1107,9 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
   for (AttnSeg& s : w.segs) {
     if (s.kind == 0)
       s.slot += w.slot_base[static_cast<size_t>(s.cand) * n_kv + s.g];
-    else
-      for (int k2 = 0; k2 < s.n_cands; ++k2)
-        w.slots[s.slot + k2] += w.slot_base[static_cast<size_t>(w.cands[s.cand + k2]) * n_kv + s.g];
+    else   // kind 1: shared_reps(n) * n slots, slot w for candidate w % n; kind 2: one per candidate
+      for (int k2 = 0; k2 < (s.kind == 1 ? shared_reps(s.n_cands) : 1) * s.n_cands; ++k2)
+        w.slots[s.slot + k2] += w.slot_base[static_cast<size_t>(w.cands[s.cand + k2 % s.n_cands]) * n_kv + s.g];
   }
   w.n_ctas = C;
   w.cta_seg.assign(C + 1, 0);
@@ -1174,10 +1181,14 @@ bool build_attn_work_fused(const int32_t* bt, const int32_t* sl, int n, int max_
 
 cudaError_t attention_configure() {
   cudaError_t e;
-  if ((e = set_smem(attn_combine_kernel<64, 8>, CombineShape<64, 8>::kBytes)) != cudaSuccess) return e;
-  if ((e = set_smem(attn_combine_kernel<64, 16>, CombineShape<64, 16>::kBytes)) != cudaSuccess) return e;
-  if ((e = set_smem(attn_combine_kernel<128, 8>, CombineShape<128, 8>::kBytes)) != cudaSuccess) return e;
-  if ((e = set_smem(attn_combine_kernel<128, 16>, CombineShape<128, 16>::kBytes)) != cudaSuccess) return e;
+  if ((e = set_smem(attn_combine_kernel<64, 8, 8>, CombineShape<64, 8, 8>::kBytes)) != cudaSuccess) return e;
+  if ((e = set_smem(attn_combine_kernel<64, 16, 8>, CombineShape<64, 16, 8>::kBytes)) != cudaSuccess) return e;
+  if ((e = set_smem(attn_combine_kernel<128, 8, 8>, CombineShape<128, 8, 8>::kBytes)) != cudaSuccess) return e;
+  if ((e = set_smem(attn_combine_kernel<128, 16, 8>, CombineShape<128, 16, 8>::kBytes)) != cudaSuccess) return e;
+  if ((e = set_smem(attn_combine_kernel<64, 8, 4>, CombineShape<64, 8, 4>::kBytes)) != cudaSuccess) return e;
+  if ((e = set_smem(attn_combine_kernel<64, 16, 4>, CombineShape<64, 16, 4>::kBytes)) != cudaSuccess) return e;
+  if ((e = set_smem(attn_combine_kernel<128, 8, 4>, CombineShape<128, 8, 4>::kBytes)) != cudaSuccess) return e;
+  if ((e = set_smem(attn_combine_kernel<128, 16, 4>, CombineShape<128, 16, 4>::kBytes)) != cudaSuccess) return e;
   if ((e = set_smem(attn_kernel<64, false>, AttnSmem<64>::kDynamic)) != cudaSuccess) return e;
   if ((e = set_smem(attn_kernel<64, true>, AttnSmem<64>::kDynamic)) != cudaSuccess) return e;
   if ((e = set_smem(attn_kernel<128, false>, AttnSmem<128>::kDynamic)) != cudaSuccess) return e;
@@ -1275,12 +1286,27 @@ cudaError_t launch_attn_combine(const AttnShape& s, const AttnWork& wk, int n, c
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 1 : 0;
   const bool two = s.group > 8;
-#define KVPRM_COMBINE(HD_, R_)                                                                                     \
+  // 8 warps per (candidate, kv head) while the launch fits one wave (<= 6 CTAs of 256 threads per SM),
+  // else 4 (half the shared memory and threads: one wave up to ~12 per SM)
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) !=
+                                                 cudaSuccess)
+      sms = 1;
+  }
+  const bool narrow = static_cast<int64_t>(n) * s.n_kv > 6 * static_cast<int64_t>(sms);
+#define KVPRM_COMBINE_W(HD_, R_, W_)                                                                               \
   do {                                                                                                           \
-    cfg.dynamicSmemBytes = CombineShape<HD_, R_>::kBytes;                                                        \
-    cfg.blockDim = dim3(32 * CombineShape<HD_, R_>::W, 1, 1);                                                    \
-    return cudaLaunchKernelEx(&cfg, attn_combine_kernel<HD_, R_>, wk.slot_base, wk.nslots, s.n_q, s.n_kv, s.group, \
-                              part_o, part_ml, mg, ts);                                                          \
+    cfg.dynamicSmemBytes = CombineShape<HD_, R_, W_>::kBytes;                                                    \
+    cfg.blockDim = dim3(32 * W_, 1, 1);                                                                          \
+    return cudaLaunchKernelEx(&cfg, attn_combine_kernel<HD_, R_, W_>, wk.slot_base, wk.nslots, s.n_q, s.n_kv,    \
+                              s.group, part_o, part_ml, mg, ts);                                                 \
+  } while (0)
+#define KVPRM_COMBINE(HD_, R_)             \
+  do {                                     \
+    if (narrow) KVPRM_COMBINE_W(HD_, R_, 4); \
+    KVPRM_COMBINE_W(HD_, R_, 8);           \
   } while (0)
   if (s.hd == 128) {
     if (two) KVPRM_COMBINE(128, 16);
@@ -1289,6 +1315,7 @@ cudaError_t launch_attn_combine(const AttnShape& s, const AttnWork& wk, int n, c
   if (two) KVPRM_COMBINE(64, 16);
   KVPRM_COMBINE(64, 8);
 #undef KVPRM_COMBINE
+#undef KVPRM_COMBINE_W
 }
 
 cudaError_t launch_resolve(const int32_t* bt, const int32_t* seq_lens, int max_blocks, int b, int64_t* out,

@@ -306,7 +306,7 @@ __device__ __forceinline__ void merge_warp_states(int group, const float* mo, co
   }
 }
 
-// Combine of one (candidate b, kv head g): W = 8 warps (threads tid < 256)
+// Combine of one (candidate b, kv head g): W warps (8 or 4; threads tid < 32 W)
 // fold its partial slots [first, first + ns), U at a time per warp with every
 // load of a round issued before the first use, into a running (M, L, O) per
 // query head of the group; the warps' states and the verify token's own entry
@@ -314,11 +314,11 @@ __device__ __forceinline__ void merge_warp_states(int group, const float* mo, co
 //   M* = max(s_self, M_w), o = (2^(s_self - M*) v_self + sum_w 2^(M_w - M*) O_w)
 //                              / (2^(s_self - M*) + sum_w 2^(M_w - M*) L_w),
 // written as a bf16 (hi, lo) pair (and optional fp32 copies).  `smem` holds
-// CombineShape::kBytes; sync() is a barrier over exactly the 256 threads.  A
+// CombineShape::kBytes; sync() is a barrier over exactly the 32 W threads.  A
 // caller running several groups back to back syncs between them.
-template <int HD, int ROWS>
+template <int HD, int ROWS, int W_ = 8>
 struct CombineShape {
-  static constexpr int W = 8;                               // warps
+  static constexpr int W = W_;                              // warps
   static constexpr int U = HD * ROWS <= 512 ? 2 : 1;        // slots in flight per warp
   static constexpr size_t kAcc = 0;                                         // [W][ROWS][HD]
   static constexpr size_t kM = kAcc + sizeof(float) * W * ROWS * HD;        // [W][ROWS]
@@ -327,11 +327,11 @@ struct CombineShape {
   static constexpr size_t kBytes = kSelf + sizeof(float) * ROWS;
 };
 
-template <int HD, int ROWS, typename Sync>
+template <int HD, int ROWS, int W_ = 8, typename Sync>
 __device__ __forceinline__ void combine_group(int tid, int b, int g, int first, int ns, int n_q, int n_kv, int group,
                                               const float* __restrict__ part_o, const float* __restrict__ part_ml,
                                               const AttnMerge& mg, uint8_t* smem, Sync sync) {
-  using CS = CombineShape<HD, ROWS>;
+  using CS = CombineShape<HD, ROWS, W_>;
   constexpr int kPer = HD / 32, W = CS::W, U = CS::U;
   constexpr int kOut = (ROWS * HD + W * 32 - 1) / (W * 32);   // outputs per thread in the final phase
   float* s_acc = reinterpret_cast<float*>(smem + CS::kAcc);

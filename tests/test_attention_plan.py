@@ -55,7 +55,9 @@ def check_plan(bt, sl, n_kv, group, n_ctas, share):
                 # shared by fewer candidates than a tensor-core tile is worth)
                 assert kind == 1 and share >= 1 and 1 <= nc <= 8 and last == 16
                 cands = [int(x) for x in p["cands"][c:c + nc]]
-                slots = [[int(x)] for x in p["slots"][slot:slot + nc]]
+                # (8 // nc) replica warps per candidate, slot w of the segment for warp w (candidate w % nc)
+                reps = 8 // nc
+                slots = [[int(p["slots"][slot + w]) for w in range(reps * nc) if w % nc == k2] for k2 in range(nc)]
                 cost[k] += SHARED_COST_PER_CAND * nc * npg
             for b, sls in zip(cands, slots):
                 used[(b, g)] += sls

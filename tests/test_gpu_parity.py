@@ -110,6 +110,16 @@ def test_fused_combine(lens, fused, monkeypatch):
     compare(w, t, gpu_rewards=r, gpu_attn=attn, label=f"fused={fused} lens={lens[:2]}x{len(lens)}")
 
 
+def test_narrow_combine():
+    # more (candidate, kv head) pairs than six per SM: the combine runs with four warps per pair
+    # (240 candidates x 4 kv heads = 960 > 6 x 152; a context holds at most 256 candidates)
+    t = ks.Tables.make(0.2)
+    lens = [int(x) for x in np.random.default_rng(47).integers(0, 60, size=240)]
+    w = ks.distinct("narrow", ks.Arch(2, 256, 8, 4, 64, 512), 47, lens, gain_std=0.2)
+    r, attn, _, _ = run_gpu(w, t)
+    compare(w, t, gpu_rewards=r, gpu_attn=attn, label="narrow combine, 240 candidates x 4 kv heads")
+
+
 def test_attention_teacher_forced():
     """kvprm_attention on given fp32 q / self k / self v against the oracle's read-out."""
     torch = require_gpu()
