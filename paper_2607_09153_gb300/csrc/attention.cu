@@ -73,9 +73,13 @@ constexpr int64_t kSharedCostPerCand = 2;
 // pages p with p % (8 / n) == w / n, into slot w of the segment.  (n <= 4 keeps every warp busy.)
 __host__ __device__ constexpr int shared_reps(int n_cands) { return kConsumerWarps / n_cands; }
 // a 64-token chunk of the tensor-core attention on one SM, in the same units, when it runs beside
-// the private pages' launch (measured: ~1.8 us per chunk beside the beam suffixes, ~2.2 us beside
-// the MCTS leaves, against ~0.043 us per unit on the private side; ~0.86 us per chunk alone)
-constexpr int64_t kTcChunkCost = 48;
+// the private pages' launch: kTcChunkCost, plus up to kTcContention as the private side's work
+// grows to 3x the tensor-core side's (its page stream takes HBM bandwidth and raises the chunks'
+// load latency).  Measured: ~1.8 us per chunk beside the beam suffixes (private work ~0.8x),
+// ~2.2 us beside the MCTS leaves (~6x), against ~0.043 us per unit on the private side; ~0.86 us
+// per chunk alone.
+constexpr int64_t kTcChunkCost = 40;
+constexpr int64_t kTcContention = 12;
 // pages shared by fewer candidates go to the persistent kernel as kind-1 runs: 2 units per page
 // and candidate there against kTcChunkCost / 4 per page on the tensor cores, whatever the tile's rows
 constexpr size_t kTcMinCands = 6;
@@ -1001,7 +1005,8 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
   // both launches end together when they run side by side
   int priv_ctas = n_ctas, tc_ctas = n_ctas;
   if (share == 3 && total > 0 && tc_chunks > 0 && n_ctas >= 2) {
-    const int64_t wt = tc_chunks * kTcChunkCost;
+    const int64_t base = tc_chunks * kTcChunkCost;
+    const int64_t wt = base + tc_chunks * kTcContention * std::min<int64_t>(total, 3 * base) / (3 * base);
     tc_ctas = static_cast<int>(std::min<int64_t>(n_ctas - 1, std::max<int64_t>(1, (n_ctas * wt + (wt + total) / 2) /
                                                                                         (wt + total))));
     priv_ctas = n_ctas - tc_ctas;
