@@ -244,7 +244,8 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
   // Step 1: acc[c][m] <- sum over ranks of acc_r[c][m] for this rank's columns
   // (only this rank reads them, so it may overwrite its own copy).  Two columns
   // per round trip when the cluster has <= 8 ranks, all peer loads in flight.
-  {
+  // Without split K (cs = 1) the parked accumulator is already the sum.
+  if (cs > 1) {
     const int step = cs <= 8 ? 2 : 1;
     for (int c = cbeg; c < cend; c += step) {
       const bool two = step == 2 && c + 1 < cend;
