@@ -59,6 +59,10 @@ __device__ __forceinline__ void store_hilo(__nv_bfloat16* hi, __nv_bfloat16* lo,
   lo[i] = __float2bfloat16_rn(x - __bfloat162float(h));
 }
 
+// LARGE (n_pad > 64, one kernel image per batch class so that the small-batch code keeps its own
+// register allocation): the residual epilogue issues a 16-column group's residual loads before
+// using any, and clusters of 4 reduce four columns per DSMEM round trip.
+template <bool LARGE>
 __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant__ CUtensorMap tmW,
                                                            const __grid_constant__ CUtensorMap tmX,
                                                            const __grid_constant__ CUtensorMap tmXlo, int has_lo,
@@ -245,7 +249,20 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
   // (only this rank reads them, so it may overwrite its own copy).  Two columns
   // per round trip when the cluster has <= 8 ranks, all peer loads in flight.
   // Without split K (cs = 1) the parked accumulator is already the sum.
-  if (cs > 1) {
+  if (LARGE && cs == 4) {
+    for (int c = cbeg; c < cend; c += 4) {
+      float v[16];
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {   // rank k % 4 of column c + k / 4
+        const int cc = c + k / 4;
+        v[k] = cc < cend ? ld_cluster(acc + cc * kBM + m, static_cast<uint32_t>(k % 4)) : 0.f;
+      }
+      __syncwarp();
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (c + j < cend) acc[(c + j) * kBM + m] = (v[4 * j] + v[4 * j + 1]) + (v[4 * j + 2] + v[4 * j + 3]);
+    }
+  } else if (cs > 1) {
     const int step = cs <= 8 ? 2 : 1;
     for (int c = cbeg; c < cend; c += step) {
       const bool two = step == 2 && c + 1 < cend;
@@ -292,19 +309,45 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     float* sq_s = red;   // [16 columns][4 warps]
     for (int c0 = cbeg; c0 < cend; c0 += 16) {
       const int c1 = min(cend, c0 + 16);
-      for (int c = c0; c < c1; ++c) {
-        float hv = 0.f;
-        if (gm < ep.M) {
-          float* hp = ep.h + static_cast<int64_t>(c) * ep.M + gm;
-          hv = (hpreload ? hpre[(c - cbeg) * kBM + m] : *hp) + acc[c * kBM + m];
-          *hp = hv;
-          if (ep.gain_next)
-            store_hilo(ep.x_hi, ep.x_lo, static_cast<int64_t>(c) * ep.M + gm, hv * __bfloat162float(ep.gain_next[gm]));
-        }
-        float sq = hv * hv;
+      if constexpr (LARGE) {   // the group's residual values, all 16 loads in flight before the first use
+        float h_in[16];
 #pragma unroll
-        for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
-        if (lane == 0) sq_s[(c - c0) * 4 + warp] = sq;
+        for (int j = 0; j < 16; ++j) {
+          const int c = c0 + j;
+          h_in[j] = (c < c1 && gm < ep.M) ? ep.h[static_cast<int64_t>(c) * ep.M + gm] : 0.f;
+        }
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const int c = c0 + j;
+          if (c >= c1) break;
+          float hv = 0.f;
+          if (gm < ep.M) {
+            hv = h_in[j] + acc[c * kBM + m];
+            ep.h[static_cast<int64_t>(c) * ep.M + gm] = hv;
+            if (ep.gain_next)
+              store_hilo(ep.x_hi, ep.x_lo, static_cast<int64_t>(c) * ep.M + gm,
+                         hv * __bfloat162float(ep.gain_next[gm]));
+          }
+          float sq = hv * hv;
+#pragma unroll
+          for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
+          if (lane == 0) sq_s[j * 4 + warp] = sq;
+        }
+      } else {
+        for (int c = c0; c < c1; ++c) {
+          float hv = 0.f;
+          if (gm < ep.M) {
+            float* hp = ep.h + static_cast<int64_t>(c) * ep.M + gm;
+            hv = (hpreload ? hpre[(c - cbeg) * kBM + m] : *hp) + acc[c * kBM + m];
+            *hp = hv;
+            if (ep.gain_next)
+              store_hilo(ep.x_hi, ep.x_lo, static_cast<int64_t>(c) * ep.M + gm, hv * __bfloat162float(ep.gain_next[gm]));
+          }
+          float sq = hv * hv;
+  #pragma unroll
+          for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
+          if (lane == 0) sq_s[(c - c0) * 4 + warp] = sq;
+        }
       }
       __syncthreads();
       if (threadIdx.x < c1 - c0) {
@@ -379,10 +422,12 @@ GemmPlan plan_gemm(int M, int K, int n_pad, int num_sms, bool has_lo, bool gate_
   const size_t acc = static_cast<size_t>(n_pad) * kBM * 4;
   if (ring < acc) ring = acc;
   p.smem_bytes = ring + 1024 /*align*/ + kTailBytes;
-  // cluster size: the largest power of two <= 16 that keeps the CTA count within
-  // two per SM and gives every rank at least two K tiles
+  // cluster size: the largest power of two <= 16 that keeps the CTA count within what fits on the
+  // SMs at once (two per SM when two CTAs' shared memory fits, else one: at B = 256 a stage holds
+  // 64 KB of activations) and gives every rank at least two K tiles
+  const int per_sm = p.smem_bytes + 1024 <= 228u * 1024u / 2 ? 2 : 1;
   int cs = 1;
-  while (cs < 16 && p.m_tiles * cs * 2 <= 2 * num_sms && cs * 4 <= p.k_tiles && cs * 2 <= n_pad) cs *= 2;
+  while (cs < 16 && p.m_tiles * cs * 2 <= per_sm * num_sms && cs * 4 <= p.k_tiles && cs * 2 <= n_pad) cs *= 2;
   p.cluster = cs;
   p.splits = cs;
   p.kt_per_split = (p.k_tiles + cs - 1) / cs;
@@ -400,9 +445,14 @@ GemmPlan plan_gemm(int M, int K, int n_pad, int num_sms, bool has_lo, bool gate_
 }
 
 cudaError_t gemm_configure() {
-  cudaError_t e = cudaFuncSetAttribute(gemm_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+  cudaError_t e = cudaFuncSetAttribute(gemm_cluster_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       200 * 1024);
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(gemm_cluster_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  e = cudaFuncSetAttribute(gemm_cluster_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(gemm_cluster_kernel<false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(gemm_cluster_kernel<true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
 }
 
 cudaError_t launch_gemm(const GemmPlan& p, const CUtensorMap* tmW, const CUtensorMap* tmX, const CUtensorMap* tmXlo,
@@ -422,7 +472,10 @@ cudaError_t launch_gemm(const GemmPlan& p, const CUtensorMap* tmW, const CUtenso
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 2 : 1;
-  return cudaLaunchKernelEx(&cfg, gemm_cluster_kernel, *tmW, *tmX, p.has_lo ? *tmXlo : *tmX, p.has_lo ? 1 : 0,
+  if (n_pad > 64)
+    return cudaLaunchKernelEx(&cfg, gemm_cluster_kernel<true>, *tmW, *tmX, p.has_lo ? *tmXlo : *tmX,
+                              p.has_lo ? 1 : 0, p.k_tiles, p.cluster, p.stages, p.tmem_cols, n_pad, ep, err, ts);
+  return cudaLaunchKernelEx(&cfg, gemm_cluster_kernel<false>, *tmW, *tmX, p.has_lo ? *tmXlo : *tmX, p.has_lo ? 1 : 0,
                             p.k_tiles, p.cluster, p.stages, p.tmem_cols, n_pad, ep, err, ts);
 }
 
