@@ -363,8 +363,13 @@ def run_gpu(args, world, rank, local):
     dominant = max((k for k in kernels if k in alg), key=lambda k: kernels[k]["total_ms"]
                    + (kernels.get("attention_tc", {}).get("total_ms", 0.0) if k == "attention" else 0.0))
     attn = roof("attention")
+    # unique bytes (each referenced page once) are the roofline; logical bytes (each candidate's whole
+    # cache) are what a reader without page sharing would stream, for context on shared workloads
+    logical = w.logical_kv_bytes()
     attention_obj = {"achieved_gbs": attn["achieved"], "frac_of_8tbs": round(attn["achieved"] / HBM_NOMINAL_GBS, 4),
                      "frac_of_measured": attn["frac"], "unique_kv_bytes_per_step": alg["attention"],
+                     "logical_kv_bytes_per_step": int(logical),
+                     "logical_gbs": round(logical / a.n_layers / (attn["time_per_layer_us"] * 1e-6) / 1e9, 1),
                      "time_per_layer_us": attn["time_per_layer_us"], "kernels": attn["kernel"]}
     step_bytes = alg["call_total"]
     line = {
