@@ -33,11 +33,12 @@ struct CallPlan {
 struct GraphKey {
   int n = -1, n_pad = -1, attn_ctas = -1, tc_ctas = -1, n_tc = -1, debug = -1, profile = -1, pdl = -1, trace = -1;
   int fuse_cs = -1;
+  int layer_waits = -1;
   const void* pool = nullptr;
   int64_t n_pages = -1;
   bool operator==(const GraphKey& o) const {
     return n == o.n && n_pad == o.n_pad && attn_ctas == o.attn_ctas && tc_ctas == o.tc_ctas && n_tc == o.n_tc &&
-           fuse_cs == o.fuse_cs &&
+           fuse_cs == o.fuse_cs && layer_waits == o.layer_waits &&
            debug == o.debug && profile == o.profile && pdl == o.pdl && trace == o.trace && pool == o.pool &&
            n_pages == o.n_pages;
   }
@@ -111,6 +112,15 @@ struct kvprm_ctx {
   // the tensor-core attention's stream when it runs beside the private pages' launch
   cudaStream_t side_stream = nullptr;
   cudaEvent_t ev_fork = nullptr, ev_join = nullptr;
+  // kvprm_score_host: the cache is copied layer by layer on one copy stream, one event per layer;
+  // while layer_waits is set, the forward being enqueued waits for layer l's event before layer l's
+  // attention, so scoring overlaps the copy of the later layers
+  cudaStream_t copy_stream = nullptr;
+  std::vector<cudaEvent_t> layer_ready;
+  cudaEvent_t pool_free = nullptr;
+  bool layer_waits = false;
+  const void* host_pool = nullptr;   // source of those copies, set for the duration of the call
+  size_t host_pool_bytes = 0;
 
   bool use_graph = true, use_pdl = true;
   GraphKey gkey;
@@ -230,6 +240,10 @@ void free_ctx(kvprm_ctx* c) {
   if (c->side_stream) cudaStreamDestroy(c->side_stream);
   if (c->ev_fork) cudaEventDestroy(c->ev_fork);
   if (c->ev_join) cudaEventDestroy(c->ev_join);
+  if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
+  for (cudaEvent_t ev : c->layer_ready)
+    if (ev) cudaEventDestroy(ev);
+  if (c->pool_free) cudaEventDestroy(c->pool_free);
 
   delete c;
 }
@@ -551,6 +565,9 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
     float* dbg = (ctx->debug_flags & 1) ? ctx->dbg + static_cast<size_t>(l) * n * m.n_q * m.hd : nullptr;
     const kvprm::AttnMerge mg{ctx->q, ctx->kself, ctx->vself, O.hi, O.lo, nullptr, dbg};
     const kvprm::AttnWork wk = device_work(ctx);
+    if (ctx->layer_waits)   // this layer's pages are still being copied in (kvprm_score_host)
+      CK(cudaStreamWaitEvent(st, ctx->layer_ready[l], E.capturing ? cudaEventWaitExternal : cudaEventWaitDefault),
+         "cudaStreamWaitEvent(layer pages)");
     {
       const int rc = enqueue_attention(ctx, E, ctx->as, wk, l, kvprm::HiLo{ctx->qhi, ctx->qlo}, mg, pdl);
       if (rc) return rc;
@@ -615,6 +632,26 @@ void drop_graph(kvprm_ctx* ctx) {
 }
 
 // Score into ctx->rewards_d on stream `st` (stream-ordered).
+// kvprm_score_host's cache copy: layer by layer, in layer order on ONE copy stream (the copy engine
+// drains one stream's queue before the next, so layers spread over several streams arrive out of
+// order), after the work already on `st` (an earlier call may still read the pool, and this call's
+// tables go first, so that the small table copies do not queue behind the cache); layer l's event
+// gates layer l's attention.
+int enqueue_pool_copy(kvprm_ctx* ctx, cudaStream_t st) {
+  CK(cudaEventRecord(ctx->pool_free, st), "cudaEventRecord(pool free)");
+  const size_t layer_bytes = ctx->host_pool_bytes / static_cast<size_t>(ctx->cfg.n_layers);
+  cudaStream_t cs = ctx->copy_stream;
+  CK(cudaStreamWaitEvent(cs, ctx->pool_free, 0), "cudaStreamWaitEvent(pool)");
+  for (int l = 0; l < ctx->cfg.n_layers; ++l) {
+    CK(cudaMemcpyAsync(static_cast<uint8_t*>(ctx->dev_pool) + l * layer_bytes,
+                       static_cast<const uint8_t*>(ctx->host_pool) + l * layer_bytes, layer_bytes,
+                       cudaMemcpyHostToDevice, cs),
+       "cudaMemcpyAsync(pool layer)");
+    CK(cudaEventRecord(ctx->layer_ready[l], cs), "cudaEventRecord(layer ready)");
+  }
+  return KVPRM_OK;
+}
+
 int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const int32_t* bt, const int32_t* sl, int32_t n,
                  cudaStream_t st) {
   int max_pages = 0;
@@ -636,6 +673,7 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   const CallPlan P = make_plan(ctx, n, max_pages);
   if ((rc = ensure_x_maps(ctx, P.n_pad))) return rc;
   if ((rc = upload_tables(ctx, bt, sl, n, st))) return rc;
+  if (ctx->layer_waits && (rc = enqueue_pool_copy(ctx, st))) return rc;
   ctx->last_n = n;
   ctx->last_stream = st;
 
@@ -654,6 +692,7 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   key.attn_ctas = P.attn_ctas;
   key.tc_ctas = ctx->work_host.n_tc_ctas * (ctx->work_host.tc_concurrent ? -1 : 1);
   key.fuse_cs = ctx->work_host.fuse_cs;
+  key.layer_waits = ctx->layer_waits ? 1 : 0;
   key.n_tc = ctx->work_host.n_tc > 0 ? 1 : 0;
   key.debug = ctx->debug_flags;
   key.profile = ctx->profile ? 1 : 0;
@@ -865,6 +904,11 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   CREATE_CK(cu(cudaStreamCreateWithFlags(&ctx->side_stream, cudaStreamNonBlocking), "cudaStreamCreate"));
   CREATE_CK(cu(cudaEventCreateWithFlags(&ctx->ev_fork, cudaEventDisableTiming), "cudaEventCreate"));
   CREATE_CK(cu(cudaEventCreateWithFlags(&ctx->ev_join, cudaEventDisableTiming), "cudaEventCreate"));
+  CREATE_CK(cu(cudaStreamCreateWithFlags(&ctx->copy_stream, cudaStreamNonBlocking), "cudaStreamCreate"));
+  ctx->layer_ready.assign(static_cast<size_t>(c.n_layers), nullptr);
+  for (cudaEvent_t& ev : ctx->layer_ready)
+    CREATE_CK(cu(cudaEventCreateWithFlags(&ev, cudaEventDisableTiming), "cudaEventCreate"));
+  CREATE_CK(cu(cudaEventCreateWithFlags(&ctx->pool_free, cudaEventDisableTiming), "cudaEventCreate"));
   ctx->use_graph = !env_off("KVPRM_NO_GRAPH");
   ctx->use_pdl = !env_off("KVPRM_NO_PDL");
   // shared pages: on the tensor cores at head_dim 128, else one warp per candidate
@@ -934,10 +978,15 @@ int kvprm_score_host(kvprm_ctx* ctx, const void* h_kv_pages, int64_t n_pages, co
       }
       ctx->dev_pool_bytes = bytes;
     }
-    CK(cudaMemcpyAsync(ctx->dev_pool, h_kv_pages, bytes, cudaMemcpyHostToDevice, st), "cudaMemcpyAsync(pool)");
     pool = ctx->dev_pool;
   }
+  ctx->layer_waits = bytes > 0;
+  ctx->host_pool = h_kv_pages;
+  ctx->host_pool_bytes = bytes;
   int rc = score_device(ctx, pool, n_pages, block_table, seq_lens, n, st);
+  ctx->layer_waits = false;
+  ctx->host_pool = nullptr;
+  ctx->host_pool_bytes = 0;
   if (rc) return rc;
   return finish_blocking(ctx, n, rewards, st);
 }
