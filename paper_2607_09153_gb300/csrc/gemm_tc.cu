@@ -48,6 +48,7 @@ constexpr uint32_t kWTileBytes = kBM * kBK * 2;   // 16 KB
 // per-column RMSNorm factors (1 KB)
 constexpr size_t kTailBytes = 512 + 1024 + 4096;   // barriers, RMSNorm factors, preloaded residual
 constexpr int kHPreCols = 8;                        // residual columns preloaded per rank (128 rows each)
+constexpr size_t kGemmMaxSmem = 200 * 1024;         // dynamic shared memory the kernel is configured for
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -61,18 +62,25 @@ __device__ __forceinline__ void store_hilo(__nv_bfloat16* hi, __nv_bfloat16* lo,
 
 // LARGE (n_pad > 64, one kernel image per batch class so that the small-batch code keeps its own
 // register allocation): the residual epilogue issues a 16-column group's residual loads before
-// using any, and clusters of 4 reduce four columns per DSMEM round trip.
+// using any and sums each column's squares in one pass over the parked tile, and clusters of 4
+// reduce eight columns per DSMEM round trip. The SiLU and QKV epilogues read kEpiBatch columns'
+// operands before the batch's first store (the 4-warp CTA is otherwise bound by one load latency
+// per column).
 template <bool LARGE>
 __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant__ CUtensorMap tmW,
                                                            const __grid_constant__ CUtensorMap tmX,
                                                            const __grid_constant__ CUtensorMap tmXlo, int has_lo,
                                                            int k_tiles, int cs, int stages, uint32_t tmem_cols,
-                                                           int n_pad, GemmEpilogue ep, int* err, unsigned long long* ts) {
+                                                           int n_pad, int mt_arg, GemmEpilogue ep, int* err,
+                                                           unsigned long long* ts) {
   trace_begin(ts);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = align1024(smem_raw);
+  // m-tiles of this CTA (LARGE only): a stage holds mt weight tiles, then the activation tile(s)
+  const int mt = LARGE ? mt_arg : 1;
   const uint32_t x_bytes = static_cast<uint32_t>(n_pad) * kBK * 2;
-  const uint32_t stage_bytes = kWTileBytes + x_bytes * (has_lo ? 2u : 1u);
+  const uint32_t w_bytes = kWTileBytes * static_cast<uint32_t>(mt);
+  const uint32_t stage_bytes = w_bytes + x_bytes * (has_lo ? 2u : 1u);
   const uint32_t acc_bytes = static_cast<uint32_t>(n_pad) * kBM * 4;
   const uint32_t ring_bytes = stages * stage_bytes > acc_bytes ? stages * stage_bytes : acc_bytes;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + ring_bytes);
@@ -84,7 +92,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
   float* hpre = rsc + 256;   // RESID: this rank's columns of h for the tile's rows, [c - cbeg][128]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int m_tile = blockIdx.x / cs;
+  const int m_tile0 = blockIdx.x / cs * mt;   // first m-tile of this CTA
   const uint32_t rank = cluster_rank();
   const int kps = (k_tiles + cs - 1) / cs;
   const int kt0 = static_cast<int>(rank) * kps;
@@ -97,6 +105,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
   const int cend = min(cbeg + cols, ep.n_valid);
   const int nc = cend > cbeg ? cend - cbeg : 0;
   const bool hpreload = ep.mode == GemmEpilogue::RESID && nc <= kHPreCols;
+  constexpr int kEpiBatch = LARGE ? 8 : 1;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < stages; ++s) {
@@ -127,11 +136,15 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     const uint64_t pol_w = policy_evict_first();
     const uint64_t pol_x = policy_evict_last();
     auto load_w = [&](uint8_t* st, int kt, uint64_t* bar) {
-      if (!silu) {
-        tma_load_2d(st, &tmW, bar, kt * kBK, m_tile * kBM, pol_w);
-      } else {   // 64 gate rows, then the matching 64 up rows
-        tma_load_2d(st, &tmW, bar, kt * kBK, m_tile * 64, pol_w);
-        tma_load_2d(st + kWTileBytes / 2, &tmW, bar, kt * kBK, ep.ff + m_tile * 64, pol_w);
+      for (int t = 0; t < mt; ++t) {
+        const int m_tile = m_tile0 + t;
+        uint8_t* wt = st + t * kWTileBytes;
+        if (!silu) {
+          tma_load_2d(wt, &tmW, bar, kt * kBK, m_tile * kBM, pol_w);
+        } else {   // 64 gate rows, then the matching 64 up rows
+          tma_load_2d(wt, &tmW, bar, kt * kBK, m_tile * 64, pol_w);
+          tma_load_2d(wt + kWTileBytes / 2, &tmW, bar, kt * kBK, ep.ff + m_tile * 64, pol_w);
+        }
       }
     };
     // Weights do not depend on the preceding kernel: start streaming the first
@@ -144,9 +157,9 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     grid_dep_wait();
     trace_event(ts, 0);   // the preceding kernel has completed
     for (int i = 0; i < pre; ++i) {
-      tma_load_2d(smem + i * stage_bytes + kWTileBytes, &tmX, &full[i], (kt0 + i) * kBK, 0, pol_x);
+      tma_load_2d(smem + i * stage_bytes + w_bytes, &tmX, &full[i], (kt0 + i) * kBK, 0, pol_x);
       if (has_lo)
-        tma_load_2d(smem + i * stage_bytes + kWTileBytes + x_bytes, &tmXlo, &full[i], (kt0 + i) * kBK, 0, pol_x);
+        tma_load_2d(smem + i * stage_bytes + w_bytes + x_bytes, &tmXlo, &full[i], (kt0 + i) * kBK, 0, pol_x);
     }
     for (int i = pre; i < nk; ++i) {
       const int s = i % stages;
@@ -155,8 +168,8 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       uint8_t* st = smem + s * stage_bytes;
       mbar_arrive_expect_tx(&full[s], stage_bytes);
       load_w(st, kt0 + i, &full[s]);
-      tma_load_2d(st + kWTileBytes, &tmX, &full[s], (kt0 + i) * kBK, 0, pol_x);
-      if (has_lo) tma_load_2d(st + kWTileBytes + x_bytes, &tmXlo, &full[s], (kt0 + i) * kBK, 0, pol_x);
+      tma_load_2d(st + w_bytes, &tmX, &full[s], (kt0 + i) * kBK, 0, pol_x);
+      if (has_lo) tma_load_2d(st + w_bytes + x_bytes, &tmXlo, &full[s], (kt0 + i) * kBK, 0, pol_x);
     }
   } else if (warp >= 2) {
     // ---------------- while the weights stream: the RMSNorm factor of each of this rank's columns
@@ -174,7 +187,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     // the next kernel's weight stream may be competing for the memory system
     if (hpreload)
       for (int idx = threadIdx.x - 64; idx < nc * kBM; idx += blockDim.x - 64) {
-        const int c = cbeg + idx / kBM, gm = m_tile * kBM + idx % kBM;
+        const int c = cbeg + idx / kBM, gm = m_tile0 * kBM + idx % kBM;
         hpre[idx] = gm < ep.M ? ep.h[static_cast<int64_t>(c) * ep.M + gm] : 0.f;
       }
   } else if (warp == 1 && nk > 0) {
@@ -184,9 +197,12 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     // slice from shared memory once: columns [0, n_pad) accumulate W hi,
     // [n_pad, 2 n_pad) accumulate W lo, summed when the accumulator is read.
     // Beyond N = 256 the two halves take one MMA each into the same columns.
+    // With two m-tiles per CTA, tile t accumulates from TMEM column t tile_cols (half the
+    // allocation, a power of two).
     const bool merged = has_lo && 2 * n_pad <= 256;
     const bool two = has_lo && !merged;
     const uint32_t idesc = idesc_bf16_f32(kBM, merged ? 2 * n_pad : n_pad);
+    const uint32_t tile_cols = tmem_cols / static_cast<uint32_t>(mt);
     for (int i = 0; i < nk; ++i) {
       const int s = i % stages;
       const uint32_t use = static_cast<uint32_t>(i / stages);
@@ -194,18 +210,22 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       if (i == 0 && lane == 0) trace_event(ts, 1);   // first weight and activation tiles landed
       tc_fence_after();
       const uint64_t a0 = desc_sw128(smem_u32(smem + s * stage_bytes));   // K step kk: + 2 kk (32 bytes)
-      const uint64_t b0 = a0 + (kWTileBytes >> 4);
+      const uint64_t b0 = a0 + (w_bytes >> 4);
       const uint64_t l0 = b0 + static_cast<uint64_t>(x_bytes >> 4);
       const uint32_t acc0 = i > 0 ? 1u : 0u;
-      if (two) {
+      for (int t = 0; t < mt; ++t) {
+        const uint32_t d = tmem + static_cast<uint32_t>(t) * tile_cols;
+        const uint64_t at = a0 + static_cast<uint64_t>(t) * (kWTileBytes >> 4);
+        if (two) {
 #pragma unroll
-        for (int kk = 0; kk < kBK / 16; ++kk) {
-          umma_bf16_w(tmem, a0 + 2 * kk, b0 + 2 * kk, idesc, kk > 0 ? 1u : acc0);
-          umma_bf16_w(tmem, a0 + 2 * kk, l0 + 2 * kk, idesc, 1u);
+          for (int kk = 0; kk < kBK / 16; ++kk) {
+            umma_bf16_w(d, at + 2 * kk, b0 + 2 * kk, idesc, kk > 0 ? 1u : acc0);
+            umma_bf16_w(d, at + 2 * kk, l0 + 2 * kk, idesc, 1u);
+          }
+        } else {
+#pragma unroll
+          for (int kk = 0; kk < kBK / 16; ++kk) umma_bf16_w(d, at + 2 * kk, b0 + 2 * kk, idesc, kk > 0 ? 1u : acc0);
         }
-      } else {
-#pragma unroll
-        for (int kk = 0; kk < kBK / 16; ++kk) umma_bf16_w(tmem, a0 + 2 * kk, b0 + 2 * kk, idesc, kk > 0 ? 1u : acc0);
       }
       umma_commit_w(&empty[s]);
     }
@@ -220,182 +240,328 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
   float* acc = reinterpret_cast<float*>(smem);   // the ring is idle once `done` has fired
   const int m = warp * 32 + lane;
   const bool merged = has_lo && 2 * n_pad <= 256;
-  for (int c0 = 0; c0 < n_pad; c0 += 16) {
-    float v[16];
-    if (nk > 0 && have) {
-      const uint32_t t = tmem + (static_cast<uint32_t>(warp * 32) << 16) + static_cast<uint32_t>(c0);
-      tmem_ld16(t, v);
-      if (merged) {
-        float w[16];
-        tmem_ld16(t + static_cast<uint32_t>(n_pad), w);
+  const uint32_t tile_cols = tmem_cols / static_cast<uint32_t>(mt);
+  // one m-tile at a time: park it, reduce it over the cluster (split K only: never with two
+  // tiles), write its epilogue
+  for (int tt = 0; tt < mt; ++tt) {
+    const int m_tile = m_tile0 + tt;
+    const uint32_t tcol = static_cast<uint32_t>(tt) * tile_cols;
+    for (int c0 = 0; c0 < n_pad; c0 += 16) {
+      float v[16];
+      if (nk > 0 && have) {
+        const uint32_t t = tmem + (static_cast<uint32_t>(warp * 32) << 16) + tcol + static_cast<uint32_t>(c0);
+        tmem_ld16(t, v);
+        if (merged) {
+          float w[16];
+          tmem_ld16(t + static_cast<uint32_t>(n_pad), w);
 #pragma unroll
-        for (int j = 0; j < 16; ++j) v[j] += w[j];
+          for (int j = 0; j < 16; ++j) v[j] += w[j];
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) v[j] = 0.f;
       }
-    } else {
 #pragma unroll
-      for (int j = 0; j < 16; ++j) v[j] = 0.f;
+      for (int j = 0; j < 16; ++j) acc[(c0 + j) * kBM + m] = v[j];
     }
-#pragma unroll
-    for (int j = 0; j < 16; ++j) acc[(c0 + j) * kBM + m] = v[j];
-  }
-  tc_fence_before();
-  cluster_sync();   // every rank's partial is parked
-  if (threadIdx.x == 0) trace_event(ts, 3);
-  if (ep.late_trigger) grid_dep_launch();
+    tc_fence_before();
+    if (tt == 0) {
+      cluster_sync();   // every rank's partial is parked
+      if (threadIdx.x == 0) trace_event(ts, 3);
+      if (ep.late_trigger) grid_dep_launch();
 
-  // ---------------- reduce this rank's candidate columns over the cluster, then the epilogue
-  grid_dep_wait();   // outputs may still be read by kernels that precede this one
-  // Step 1: acc[c][m] <- sum over ranks of acc_r[c][m] for this rank's columns
-  // (only this rank reads them, so it may overwrite its own copy).  Two columns
-  // per round trip when the cluster has <= 8 ranks, all peer loads in flight.
-  // Without split K (cs = 1) the parked accumulator is already the sum.
-  if (LARGE && cs == 4) {
-    for (int c = cbeg; c < cend; c += 4) {
-      float v[16];
+      // ---------------- reduce this rank's candidate columns over the cluster, then the epilogue
+      grid_dep_wait();   // outputs may still be read by kernels that precede this one
+      // Step 1: acc[c][m] <- sum over ranks of acc_r[c][m] for this rank's columns
+      // (only this rank reads them, so it may overwrite its own copy).  Two columns
+      // per round trip when the cluster has <= 8 ranks, all peer loads in flight.
+      // Without split K (cs = 1) the parked accumulator is already the sum.
+      if (LARGE && cs == 4) {
+        for (int c = cbeg; c < cend; c += 8) {
+          float v[32];
 #pragma unroll
-      for (int k = 0; k < 16; ++k) {   // rank k % 4 of column c + k / 4
-        const int cc = c + k / 4;
-        v[k] = cc < cend ? ld_cluster(acc + cc * kBM + m, static_cast<uint32_t>(k % 4)) : 0.f;
+          for (int k = 0; k < 32; ++k) {   // rank k % 4 of column c + k / 4
+            const int cc = c + k / 4;
+            v[k] = cc < cend ? ld_cluster(acc + cc * kBM + m, static_cast<uint32_t>(k % 4)) : 0.f;
+          }
+          __syncwarp();
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            if (c + j < cend) acc[(c + j) * kBM + m] = (v[4 * j] + v[4 * j + 1]) + (v[4 * j + 2] + v[4 * j + 3]);
+        }
+      } else if (cs > 1) {
+        const int step = cs <= 8 ? 2 : 1;
+        for (int c = cbeg; c < cend; c += step) {
+          const bool two = step == 2 && c + 1 < cend;
+          float v[16];
+#pragma unroll
+          for (int k = 0; k < 16; ++k) {
+            const int r = step == 2 ? (k & 7) : k;
+            const int cc = (step == 2 && k >= 8) ? c + 1 : c;
+            const bool use = r < cs && (cc == c || two);
+            v[k] = use ? ld_cluster(acc + cc * kBM + m, static_cast<uint32_t>(r)) : 0.f;
+          }
+          if (step == 2) {
+            float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+              s0 += v[k];
+              s1 += v[8 + k];
+            }
+            __syncwarp();
+            acc[c * kBM + m] = s0;
+            if (two) acc[(c + 1) * kBM + m] = s1;
+          } else {
+            float s0 = 0.f;
+#pragma unroll
+            for (int k = 0; k < 16; ++k) s0 += v[k];
+            acc[c * kBM + m] = s0;
+          }
+        }
       }
+      if (threadIdx.x == 0) trace_event(ts, 4);   // this rank's columns are reduced over the cluster
+      // no peer reads this CTA's shared memory any more: arrive on the exit barrier now and wait for the
+      // peers only before exiting, so the barrier's latency hides behind the epilogue
       __syncwarp();
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if (c + j < cend) acc[(c + j) * kBM + m] = (v[4 * j] + v[4 * j + 1]) + (v[4 * j + 2] + v[4 * j + 3]);
+      cluster_arrive();
     }
-  } else if (cs > 1) {
-    const int step = cs <= 8 ? 2 : 1;
-    for (int c = cbeg; c < cend; c += step) {
-      const bool two = step == 2 && c + 1 < cend;
-      float v[16];
-#pragma unroll
-      for (int k = 0; k < 16; ++k) {
-        const int r = step == 2 ? (k & 7) : k;
-        const int cc = (step == 2 && k >= 8) ? c + 1 : c;
-        const bool use = r < cs && (cc == c || two);
-        v[k] = use ? ld_cluster(acc + cc * kBM + m, static_cast<uint32_t>(r)) : 0.f;
-      }
-      if (step == 2) {
-        float s0 = 0.f, s1 = 0.f;
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-          s0 += v[k];
-          s1 += v[8 + k];
+    __syncthreads();   // every warp's reduced columns are in acc
+    if (threadIdx.x == 0) trace_event(ts, 5);
+    // Step 2: the epilogue over (row, column) pairs, all threads in parallel
+    if (ep.mode == GemmEpilogue::PLAIN) {
+      const int gm = m_tile * kBM + m;
+      if (gm < ep.M)
+        for (int c = cbeg; c < cend; ++c) ep.out[static_cast<int64_t>(c) * ep.M + gm] = acc[c * kBM + m];
+    } else if (ep.mode == GemmEpilogue::RESID && LARGE) {
+      // pass 1, 16 columns at a time with the group's residual loads in flight before the first use:
+      // h += acc, the next projection's input, and hv^2 parked in place of acc (each (column, row)
+      // slot is this thread's own)
+      const int gm = m_tile * kBM + m;
+      const float gain = (ep.gain_next && gm < ep.M) ? __bfloat162float(ep.gain_next[gm]) : 0.f;
+      if ((ep.M & 3) == 0) {
+        // four consecutive rows of one column per thread (a warp covers one column's 128 rows):
+        // 16-byte residual loads and stores, 8-byte hi/lo stores; eight columns' loads in flight
+        const int rq = static_cast<int>(threadIdx.x) & 31, cg = static_cast<int>(threadIdx.x) >> 5;
+        const int gm0 = m_tile * kBM + 4 * rq;
+        const bool rows_ok = gm0 < ep.M;   // M % 4 == 0: the four rows are all valid or all past M
+        float g4[4] = {0.f, 0.f, 0.f, 0.f};
+        if (ep.gain_next && rows_ok) {
+          const uint2 gb = *reinterpret_cast<const uint2*>(ep.gain_next + gm0);
+          const float2 ga = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&gb.x));
+          const float2 gc = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&gb.y));
+          g4[0] = ga.x;
+          g4[1] = ga.y;
+          g4[2] = gc.x;
+          g4[3] = gc.y;
         }
-        __syncwarp();
-        acc[c * kBM + m] = s0;
-        if (two) acc[(c + 1) * kBM + m] = s1;
-      } else {
-        float s0 = 0.f;
+        for (int c0 = cbeg + cg; c0 < cend; c0 += 4 * 8) {
+          float4 h_in[8];
 #pragma unroll
-        for (int k = 0; k < 16; ++k) s0 += v[k];
-        acc[c * kBM + m] = s0;
-      }
-    }
-  }
-  if (threadIdx.x == 0) trace_event(ts, 4);   // this rank's columns are reduced over the cluster
-  // no peer reads this CTA's shared memory any more: arrive on the exit barrier now and wait for the
-  // peers only before exiting, so the barrier's latency hides behind the epilogue
-  __syncwarp();
-  cluster_arrive();
-  __syncthreads();   // every warp's reduced columns are in acc
-  if (threadIdx.x == 0) trace_event(ts, 5);
-  // Step 2: the epilogue over (row, column) pairs, all threads in parallel
-  if (ep.mode == GemmEpilogue::PLAIN) {
-    const int gm = m_tile * kBM + m;
-    if (gm < ep.M)
-      for (int c = cbeg; c < cend; ++c) ep.out[static_cast<int64_t>(c) * ep.M + gm] = acc[c * kBM + m];
-  } else if (ep.mode == GemmEpilogue::RESID) {
-    const int gm = m_tile * kBM + m;
-    float* sq_s = red;   // [16 columns][4 warps]
-    for (int c0 = cbeg; c0 < cend; c0 += 16) {
-      const int c1 = min(cend, c0 + 16);
-      if constexpr (LARGE) {   // the group's residual values, all 16 loads in flight before the first use
-        float h_in[16];
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          const int c = c0 + j;
-          h_in[j] = (c < c1 && gm < ep.M) ? ep.h[static_cast<int64_t>(c) * ep.M + gm] : 0.f;
-        }
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          const int c = c0 + j;
-          if (c >= c1) break;
-          float hv = 0.f;
-          if (gm < ep.M) {
-            hv = h_in[j] + acc[c * kBM + m];
-            ep.h[static_cast<int64_t>(c) * ep.M + gm] = hv;
-            if (ep.gain_next)
-              store_hilo(ep.x_hi, ep.x_lo, static_cast<int64_t>(c) * ep.M + gm,
-                         hv * __bfloat162float(ep.gain_next[gm]));
+          for (int k = 0; k < 8; ++k) {
+            const int c = c0 + 4 * k;
+            h_in[k] = (c < cend && rows_ok) ? *reinterpret_cast<const float4*>(ep.h + static_cast<int64_t>(c) * ep.M + gm0)
+                                            : make_float4(0.f, 0.f, 0.f, 0.f);
           }
-          float sq = hv * hv;
 #pragma unroll
-          for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
-          if (lane == 0) sq_s[j * 4 + warp] = sq;
+          for (int k = 0; k < 8; ++k) {
+            const int c = c0 + 4 * k;
+            if (c >= cend) break;
+            float4* ap = reinterpret_cast<float4*>(acc + c * kBM + 4 * rq);
+            const float4 a = *ap;
+            float4 hv = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (rows_ok) {
+              hv = make_float4(h_in[k].x + a.x, h_in[k].y + a.y, h_in[k].z + a.z, h_in[k].w + a.w);
+              const int64_t o = static_cast<int64_t>(c) * ep.M + gm0;
+              *reinterpret_cast<float4*>(ep.h + o) = hv;
+              if (ep.gain_next) {
+                const float x[4] = {hv.x * g4[0], hv.y * g4[1], hv.z * g4[2], hv.w * g4[3]};
+                uint32_t hi[2], lo[2];
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                  const __nv_bfloat162 h2 = __floats2bfloat162_rn(x[2 * e], x[2 * e + 1]);
+                  const float2 hf = __bfloat1622float2(h2);
+                  const __nv_bfloat162 l2 = __floats2bfloat162_rn(x[2 * e] - hf.x, x[2 * e + 1] - hf.y);
+                  hi[e] = *reinterpret_cast<const uint32_t*>(&h2);
+                  lo[e] = *reinterpret_cast<const uint32_t*>(&l2);
+                }
+                *reinterpret_cast<uint2*>(ep.x_hi + o) = make_uint2(hi[0], hi[1]);
+                *reinterpret_cast<uint2*>(ep.x_lo + o) = make_uint2(lo[0], lo[1]);
+              }
+            }
+            *ap = make_float4(hv.x * hv.x, hv.y * hv.y, hv.z * hv.z, hv.w * hv.w);
+          }
         }
       } else {
-        for (int c = c0; c < c1; ++c) {
-          float hv = 0.f;
-          if (gm < ep.M) {
-            float* hp = ep.h + static_cast<int64_t>(c) * ep.M + gm;
-            hv = (hpreload ? hpre[(c - cbeg) * kBM + m] : *hp) + acc[c * kBM + m];
-            *hp = hv;
-            if (ep.gain_next)
-              store_hilo(ep.x_hi, ep.x_lo, static_cast<int64_t>(c) * ep.M + gm, hv * __bfloat162float(ep.gain_next[gm]));
+        for (int c0 = cbeg; c0 < cend; c0 += 16) {
+          float h_in[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const int c = c0 + j;
+            h_in[j] = (c < cend && gm < ep.M) ? ep.h[static_cast<int64_t>(c) * ep.M + gm] : 0.f;
           }
-          float sq = hv * hv;
-  #pragma unroll
-          for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
-          if (lane == 0) sq_s[(c - c0) * 4 + warp] = sq;
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const int c = c0 + j;
+            if (c >= cend) break;
+            float hv = 0.f;
+            if (gm < ep.M) {
+              hv = h_in[j] + acc[c * kBM + m];
+              ep.h[static_cast<int64_t>(c) * ep.M + gm] = hv;
+              if (ep.gain_next) store_hilo(ep.x_hi, ep.x_lo, static_cast<int64_t>(c) * ep.M + gm, hv * gain);
+            }
+            acc[c * kBM + m] = hv * hv;
+          }
         }
       }
       __syncthreads();
-      if (threadIdx.x < c1 - c0) {
-        const float* q4 = sq_s + threadIdx.x * 4;
-        ep.sumsq[static_cast<int64_t>(m_tile) * ep.n_valid + c0 + threadIdx.x] = (q4[0] + q4[1]) + (q4[2] + q4[3]);
+      // pass 2: each column's sum of squares over the tile's 128 rows, eight threads per column
+      // (rows part + 8 q, the start of q rotated per column so that a warp's four columns hit
+      // different banks), warp-uniform trip count for the shuffles
+      for (int t0 = 0; t0 < nc * 8; t0 += blockDim.x) {
+        const int t = t0 + static_cast<int>(threadIdx.x);
+        const int cl = t >> 3, part = t & 7;
+        float sq = 0.f;
+        if (t < nc * 8) {
+          const float* col = acc + (cbeg + cl) * kBM + part;
+#pragma unroll
+          for (int q = 0; q < 16; ++q) sq += col[8 * ((q + (cl & 3)) & 15)];
+        }
+        sq += __shfl_xor_sync(0xffffffffu, sq, 1);
+        sq += __shfl_xor_sync(0xffffffffu, sq, 2);
+        sq += __shfl_xor_sync(0xffffffffu, sq, 4);
+        if (t < nc * 8 && part == 0) ep.sumsq[static_cast<int64_t>(m_tile) * ep.n_valid + cbeg + cl] = sq;
       }
-      __syncthreads();
+    } else if (ep.mode == GemmEpilogue::RESID) {
+      const int gm = m_tile * kBM + m;
+      float* sq_s = red;   // [16 columns][4 warps]
+      for (int c0 = cbeg; c0 < cend; c0 += 16) {
+        const int c1 = min(cend, c0 + 16);
+        {
+          for (int c = c0; c < c1; ++c) {
+            float hv = 0.f;
+            if (gm < ep.M) {
+              float* hp = ep.h + static_cast<int64_t>(c) * ep.M + gm;
+              hv = (hpreload ? hpre[(c - cbeg) * kBM + m] : *hp) + acc[c * kBM + m];
+              *hp = hv;
+              if (ep.gain_next)
+                store_hilo(ep.x_hi, ep.x_lo, static_cast<int64_t>(c) * ep.M + gm, hv * __bfloat162float(ep.gain_next[gm]));
+            }
+            float sq = hv * hv;
+#pragma unroll
+            for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
+            if (lane == 0) sq_s[(c - c0) * 4 + warp] = sq;
+          }
+        }
+        __syncthreads();
+        if (threadIdx.x < c1 - c0) {
+          const float* q4 = sq_s + threadIdx.x * 4;
+          ep.sumsq[static_cast<int64_t>(m_tile) * ep.n_valid + c0 + threadIdx.x] = (q4[0] + q4[1]) + (q4[2] + q4[3]);
+        }
+        __syncthreads();
+      }
+    } else if (ep.mode == GemmEpilogue::SILU && LARGE && (ep.ff & 7) == 0) {
+      // eight consecutive rows of one column per thread (8 row groups x 16 column groups): 16-byte
+      // loads from the parked tile and one 16-byte store for each of the hi and lo halves (2-byte
+      // stores, 256 per warp and tile at B = 256, bound the scalar form); the exponential and the
+      // divide take the fast intrinsics
+      const int rg = static_cast<int>(threadIdx.x) & 7, cg = static_cast<int>(threadIdx.x) >> 3;
+      const int j0 = m_tile * 64 + 8 * rg;   // ff % 8 == 0: a row group is all valid or all past ff
+      if (j0 < ep.ff) {
+#pragma unroll 2
+        for (int c = cbeg + cg; c < cend; c += 16) {
+          const float rs = ep.rs_sumsq ? rsc[c - cbeg] : 1.f;
+          const float4* gp = reinterpret_cast<const float4*>(acc + c * kBM + 8 * rg);
+          const float4* up = reinterpret_cast<const float4*>(acc + c * kBM + 64 + 8 * rg);
+          const float4 g0 = gp[0], g1 = gp[1], u0 = up[0], u1 = up[1];
+          const float g[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+          const float u[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+          uint32_t hi[4], lo[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float ga = g[2 * e] * rs, gb = g[2 * e + 1] * rs;
+            const float a = __fdividef(ga, 1.0f + __expf(-ga)) * (u[2 * e] * rs);
+            const float b = __fdividef(gb, 1.0f + __expf(-gb)) * (u[2 * e + 1] * rs);
+            const __nv_bfloat162 h2 = __floats2bfloat162_rn(a, b);
+            const float2 hf = __bfloat1622float2(h2);
+            const __nv_bfloat162 l2 = __floats2bfloat162_rn(a - hf.x, b - hf.y);
+            hi[e] = *reinterpret_cast<const uint32_t*>(&h2);
+            lo[e] = *reinterpret_cast<const uint32_t*>(&l2);
+          }
+          const int64_t o = static_cast<int64_t>(c) * ep.ff + j0;
+          *reinterpret_cast<uint4*>(ep.a_hi + o) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+          *reinterpret_cast<uint4*>(ep.a_lo + o) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+        }
+      }
+    } else if (ep.mode == GemmEpilogue::SILU) {
+      const int r = m & 63, half_sel = m >> 6;   // two column groups of 64 threads
+      const int j = m_tile * 64 + r;
+      if (j < ep.ff)
+        for (int c0 = cbeg + half_sel; c0 < cend; c0 += 2 * kEpiBatch) {
+          float g[kEpiBatch], u[kEpiBatch];   // a batch's operands, read before its first store
+#pragma unroll
+          for (int k = 0; k < kEpiBatch; ++k) {
+            const int c = c0 + 2 * k;
+            const bool ok = c < cend;
+            const float rs = (ok && ep.rs_sumsq) ? rsc[c - cbeg] : 1.f;
+            g[k] = ok ? acc[c * kBM + r] * rs : 0.f;
+            u[k] = ok ? acc[c * kBM + 64 + r] * rs : 0.f;
+          }
+#pragma unroll
+          for (int k = 0; k < kEpiBatch; ++k) {
+            const int c = c0 + 2 * k;
+            if (c < cend)
+            store_hilo(ep.a_hi, ep.a_lo, static_cast<int64_t>(c) * ep.ff + j, g[k] / (1.0f + expf(-g[k])) * u[k]);
+          }
+        }
+    } else {   // QKV: pair p = m & 63 of this tile, two column groups of 64 threads
+      const int p = m & 63, half_sel = m >> 6;
+      const int hd = ep.hd, half = hd / 2;
+      const int row_a = (p / half) * hd + (p % half);   // first element of the pair, within the tile
+      const int row_b = row_a + half;
+      const int grow = m_tile * kBM + row_a;              // row of W_qkv
+      const int head = grow / hd, i = grow % hd;          // i < half
+      const bool rot = head < ep.n_q + ep.n_kv;   // q and k rows take RoPE, v rows do not
+      for (int c0 = cbeg + half_sel; c0 < cend; c0 += 2 * kEpiBatch) {
+        // a batch's operands (accumulator pair and rotation), read before its first store
+        float av[kEpiBatch], bv[kEpiBatch];
+        float2 cs2[kEpiBatch];
+#pragma unroll
+        for (int k = 0; k < kEpiBatch; ++k) {
+          const int c = c0 + 2 * k;
+          const bool ok = c < cend;
+          const float rs = (ok && ep.rs_sumsq) ? rsc[c - cbeg] : 1.f;
+          av[k] = ok ? acc[c * kBM + row_a] * rs : 0.f;
+          bv[k] = ok ? acc[c * kBM + row_b] * rs : 0.f;
+          cs2[k] = (ok && rot) ? ep.rope[c * half + i] : make_float2(1.f, 0.f);
+        }
+#pragma unroll
+        for (int k = 0; k < kEpiBatch; ++k) {
+          const int c = c0 + 2 * k;
+          if (c >= cend) break;
+          float a = av[k], b = bv[k];
+          if (rot) {
+            const float a2 = a * cs2[k].x - b * cs2[k].y;
+            const float b2 = b * cs2[k].x + a * cs2[k].y;
+            a = a2;
+            b = b2;
+          }
+          if (head < ep.n_q) {
+            const int64_t o = (static_cast<int64_t>(c) * ep.n_q + head) * hd + i;
+            ep.q[o] = a;
+            ep.q[o + half] = b;
+            store_hilo(ep.q_hi, ep.q_lo, o, a);
+            store_hilo(ep.q_hi, ep.q_lo, o + half, b);
+          } else if (head < ep.n_q + 2 * ep.n_kv) {
+            const bool is_k = head < ep.n_q + ep.n_kv;
+            const int kvh = is_k ? head - ep.n_q : head - ep.n_q - ep.n_kv;
+            float* dst = (is_k ? ep.kself : ep.vself) + (static_cast<int64_t>(c) * ep.n_kv + kvh) * hd + i;
+            dst[0] = a;
+            dst[half] = b;
+          }
+        }
+      }
     }
-  } else if (ep.mode == GemmEpilogue::SILU) {
-    const int r = m & 63, half_sel = m >> 6;   // two column groups of 64 threads
-    const int j = m_tile * 64 + r;
-    if (j < ep.ff)
-      for (int c = cbeg + half_sel; c < cend; c += 2) {
-        const float rs = ep.rs_sumsq ? rsc[c - cbeg] : 1.f;
-        const float g = acc[c * kBM + r] * rs, u = acc[c * kBM + 64 + r] * rs;
-        store_hilo(ep.a_hi, ep.a_lo, static_cast<int64_t>(c) * ep.ff + j, g / (1.0f + expf(-g)) * u);
-      }
-  } else {   // QKV: pair p = m & 63 of this tile, two column groups of 64 threads
-    const int p = m & 63, half_sel = m >> 6;
-    const int hd = ep.hd, half = hd / 2;
-    const int row_a = (p / half) * hd + (p % half);   // first element of the pair, within the tile
-    const int row_b = row_a + half;
-    const int grow = m_tile * kBM + row_a;              // row of W_qkv
-    const int head = grow / hd, i = grow % hd;          // i < half
-    for (int c = cbeg + half_sel; c < cend; c += 2) {
-      const float rs = ep.rs_sumsq ? rsc[c - cbeg] : 1.f;
-      float a = acc[c * kBM + row_a] * rs, b = acc[c * kBM + row_b] * rs;
-      if (head < ep.n_q + ep.n_kv) {
-        const float2 cs2 = ep.rope[c * half + i];
-        const float a2 = a * cs2.x - b * cs2.y;
-        const float b2 = b * cs2.x + a * cs2.y;
-        a = a2;
-        b = b2;
-      }
-      if (head < ep.n_q) {
-        const int64_t o = (static_cast<int64_t>(c) * ep.n_q + head) * hd + i;
-        ep.q[o] = a;
-        ep.q[o + half] = b;
-        store_hilo(ep.q_hi, ep.q_lo, o, a);
-        store_hilo(ep.q_hi, ep.q_lo, o + half, b);
-      } else if (head < ep.n_q + 2 * ep.n_kv) {
-        const bool is_k = head < ep.n_q + ep.n_kv;
-        const int kvh = is_k ? head - ep.n_q : head - ep.n_q - ep.n_kv;
-        float* dst = (is_k ? ep.kself : ep.vself) + (static_cast<int64_t>(c) * ep.n_kv + kvh) * hd + i;
-        dst[0] = a;
-        dst[half] = b;
-      }
-    }
+    if (tt + 1 < mt) __syncthreads();   // every thread is done with acc before the next tile is parked
   }
   (void)nc;
   if (threadIdx.x == 0) trace_event(ts, 6);   // this thread's epilogue written
@@ -441,14 +607,33 @@ GemmPlan plan_gemm(int M, int K, int n_pad, int num_sms, bool has_lo, bool gate_
   const int need = (has_lo && 2 * n_pad <= 256) ? 2 * n_pad : n_pad;   // merged hi/lo accumulator halves
   while (cols < static_cast<uint32_t>(need)) cols <<= 1;
   p.tmem_cols = cols;
+  // gate/up at large batches without split K: when one-tile CTAs would need two waves, a CTA takes
+  // two m-tiles, so that every stage's activation tile (four times the weight tile at B = 256 with
+  // the lo half) serves both, and the grid fits on the SMs at once
+  if (gate_up && n_pad > 64 && cs == 1 && p.m_tiles % 2 == 0 && p.m_tiles > per_sm * num_sms) {
+    const uint32_t st2 = 2 * kWTileBytes + static_cast<uint32_t>(n_pad) * kBK * 2 * (has_lo ? 2u : 1u);
+    int stages2 = static_cast<int>((192u * 1024u) / st2);
+    if (stages2 > 8) stages2 = 8;
+    if (stages2 > p.kt_per_split) stages2 = p.kt_per_split;
+    size_t ring2 = static_cast<size_t>(stages2) * st2;
+    if (ring2 < acc) ring2 = acc;
+    const size_t smem2 = ring2 + 1024 + kTailBytes;
+    if (stages2 >= 2 && 2 * cols <= 512 && smem2 <= kGemmMaxSmem && (p.m_tiles / 2) <= num_sms) {
+      p.mt = 2;
+      p.stages = stages2;
+      p.smem_bytes = smem2;
+      p.tmem_cols = 2 * cols;
+    }
+  }
   return p;
 }
 
 cudaError_t gemm_configure() {
   cudaError_t e = cudaFuncSetAttribute(gemm_cluster_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       200 * 1024);
+                                       static_cast<int>(kGemmMaxSmem));
   if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(gemm_cluster_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024);
+  e = cudaFuncSetAttribute(gemm_cluster_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(kGemmMaxSmem));
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(gemm_cluster_kernel<false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   if (e != cudaSuccess) return e;
@@ -459,7 +644,7 @@ cudaError_t launch_gemm(const GemmPlan& p, const CUtensorMap* tmW, const CUtenso
                         const GemmEpilogue& ep, int n_pad, int* err, cudaStream_t stream, bool pdl,
                         unsigned long long* ts) {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(p.m_tiles * p.cluster, 1, 1);
+  cfg.gridDim = dim3((p.m_tiles + p.mt - 1) / p.mt * p.cluster, 1, 1);
   cfg.blockDim = dim3(128, 1, 1);
   cfg.dynamicSmemBytes = p.smem_bytes;
   cfg.stream = stream;
@@ -474,9 +659,11 @@ cudaError_t launch_gemm(const GemmPlan& p, const CUtensorMap* tmW, const CUtenso
   cfg.numAttrs = pdl ? 2 : 1;
   if (n_pad > 64)
     return cudaLaunchKernelEx(&cfg, gemm_cluster_kernel<true>, *tmW, *tmX, p.has_lo ? *tmXlo : *tmX,
-                              p.has_lo ? 1 : 0, p.k_tiles, p.cluster, p.stages, p.tmem_cols, n_pad, ep, err, ts);
+                              p.has_lo ? 1 : 0, p.k_tiles, p.cluster, p.stages, p.tmem_cols, n_pad, p.mt, ep, err,
+                              ts);
+  if (p.mt != 1) return cudaErrorInvalidValue;   // two m-tiles per CTA exist in the large-batch image only
   return cudaLaunchKernelEx(&cfg, gemm_cluster_kernel<false>, *tmW, *tmX, p.has_lo ? *tmXlo : *tmX, p.has_lo ? 1 : 0,
-                            p.k_tiles, p.cluster, p.stages, p.tmem_cols, n_pad, ep, err, ts);
+                            p.k_tiles, p.cluster, p.stages, p.tmem_cols, n_pad, 1, ep, err, ts);
 }
 
 }  // namespace kvprm

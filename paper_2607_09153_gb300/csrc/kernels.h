@@ -22,6 +22,9 @@ struct GemmPlan {
   bool has_lo = true;    // activation given as a bf16 (hi, lo) pair
   bool gate_up = false;  // tiles of 64 gate rows + the matching 64 up rows
   int m_tiles = 0, k_tiles = 0, kt_per_split = 0, splits = 0, stages = 0, cluster = 1;
+  // m-tiles per CTA: 2 for a gate/up projection without split K whose one-tile CTAs would need two
+  // waves (large batches); the CTA's stage then holds both weight tiles and one activation tile
+  int mt = 1;
   uint32_t tmem_cols = 32;
   size_t smem_bytes = 0;
 };

@@ -94,6 +94,20 @@ def test_layer_shapes(arch, lens):
     compare(w, t, gpu_rewards=r, gpu_attn=attn, label=f"arch {arch.d_model}/{arch.n_q_heads}/{arch.n_kv_heads}")
 
 
+def test_two_tile_gate_up():
+    """7B layer shapes at 200 candidates (padded to 208): the gate/up projection's one-tile CTAs
+    would not fit on the SMs at once, so each CTA takes two m-tiles (two accumulators of N = 208
+    side by side in TMEM, one activation stage for both); sampled candidates against the oracle."""
+    t = ks.Tables.make(0.2)
+    lens = [(53 * b) % 257 for b in range(200)]
+    w = ks.distinct("two_tile", ks.Arch(2, 3584, 28, 4, 128, 18944), 57, lens, gain_std=0.2)
+    r, attn, dev, sc = run_gpu(w, t)
+    assert np.isfinite(r).all()
+    ids = [0, 1, 100, 127, 128, 199]
+    compare(w, t, cand_ids=ids, gpu_rewards=r, gpu_attn=attn, label="two-tile gate/up")
+    sc.close()
+
+
 @pytest.mark.parametrize("lens", [[16 * 9] * 4,            # 8 (candidate, kv head) pairs: clusters of 8
                                   [16 * 33 - 5] * 20,       # 40 pairs: clusters of 2
                                   [40] * 76,                # 152 pairs: one CTA each
