@@ -62,10 +62,10 @@ __device__ __forceinline__ void store_hilo(__nv_bfloat16* hi, __nv_bfloat16* lo,
 
 // LARGE (n_pad > 64, one kernel image per batch class so that the small-batch code keeps its own
 // register allocation): the residual epilogue issues a 16-column group's residual loads before
-// using any and sums each column's squares in one pass over the parked tile, and clusters of 4
-// reduce eight columns per DSMEM round trip. The SiLU and QKV epilogues read kEpiBatch columns'
-// operands before the batch's first store (the 4-warp CTA is otherwise bound by one load latency
-// per column).
+// using any and sums each column's squares in one pass over the parked tile, clusters of 4 reduce
+// with 16-byte DSMEM loads, and the epilogues move 4 or 8 consecutive rows of a column per thread
+// with 16-byte accesses (the 4-warp CTA is otherwise bound by 2- and 4-byte stores and by one load
+// latency per column).
 template <bool LARGE>
 __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant__ CUtensorMap tmW,
                                                            const __grid_constant__ CUtensorMap tmX,
@@ -274,20 +274,31 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       grid_dep_wait();   // outputs may still be read by kernels that precede this one
       // Step 1: acc[c][m] <- sum over ranks of acc_r[c][m] for this rank's columns
       // (only this rank reads them, so it may overwrite its own copy).  Two columns
-      // per round trip when the cluster has <= 8 ranks, all peer loads in flight.
+      // per round trip when the cluster has <= 8 ranks (four with 16-byte loads in
+      // the large-batch image's clusters of 4), all peer loads in flight.
       // Without split K (cs = 1) the parked accumulator is already the sum.
       if (LARGE && cs == 4) {
-        for (int c = cbeg; c < cend; c += 8) {
-          float v[32];
+        // four consecutive rows of one column per thread (a warp covers a column's 128 rows), four
+        // columns per round: 16 loads of 16 bytes in flight, the four ranks' copies of each
+        const int rq = static_cast<int>(threadIdx.x) & 31, cg = static_cast<int>(threadIdx.x) >> 5;
+        for (int c0 = cbeg + cg; c0 < cend; c0 += 4 * 4) {
+          float4 v[16];
 #pragma unroll
-          for (int k = 0; k < 32; ++k) {   // rank k % 4 of column c + k / 4
-            const int cc = c + k / 4;
-            v[k] = cc < cend ? ld_cluster(acc + cc * kBM + m, static_cast<uint32_t>(k % 4)) : 0.f;
+          for (int k = 0; k < 16; ++k) {   // rank k % 4 of column c0 + 4 (k / 4)
+            const int cc = c0 + 4 * (k / 4);
+            v[k] = cc < cend ? ld_cluster4(acc + cc * kBM + 4 * rq, static_cast<uint32_t>(k % 4))
+                             : make_float4(0.f, 0.f, 0.f, 0.f);
           }
-          __syncwarp();
 #pragma unroll
-          for (int j = 0; j < 8; ++j)
-            if (c + j < cend) acc[(c + j) * kBM + m] = (v[4 * j] + v[4 * j + 1]) + (v[4 * j + 2] + v[4 * j + 3]);
+          for (int j = 0; j < 4; ++j) {
+            const int cc = c0 + 4 * j;
+            if (cc < cend) {
+              const float4 a = v[4 * j], b = v[4 * j + 1], c = v[4 * j + 2], d = v[4 * j + 3];
+              *reinterpret_cast<float4*>(acc + cc * kBM + 4 * rq) =
+                  make_float4((a.x + b.x) + (c.x + d.x), (a.y + b.y) + (c.y + d.y), (a.z + b.z) + (c.z + d.z),
+                              (a.w + b.w) + (c.w + d.w));
+            }
+          }
         }
       } else if (cs > 1) {
         const int step = cs <= 8 ? 2 : 1;
@@ -513,6 +524,73 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
             store_hilo(ep.a_hi, ep.a_lo, static_cast<int64_t>(c) * ep.ff + j, g[k] / (1.0f + expf(-g[k])) * u[k]);
           }
         }
+    } else if (LARGE && (ep.hd & 7) == 0) {
+      // QKV, four consecutive RoPE pairs (i .. i + 3, partners i + half ..) of one column per
+      // thread (16 pair groups x 8 column groups): 16-byte loads of the parked tile and the
+      // rotation, 16-byte fp32 and 8-byte hi/lo stores; two columns' operands in flight
+      const int pq = 4 * (static_cast<int>(threadIdx.x) & 15), cg = static_cast<int>(threadIdx.x) >> 4;
+      const int hd = ep.hd, half = hd / 2;
+      const int row_a = (pq / half) * hd + (pq % half);   // half % 4 == 0: the four pairs share a head
+      const int row_b = row_a + half;
+      const int grow = m_tile * kBM + row_a;
+      const int head = grow / hd, i = grow % hd;
+      const bool rot = head < ep.n_q + ep.n_kv;
+      auto store4 = [&](float* dst, __nv_bfloat16* dhi, __nv_bfloat16* dlo, int64_t o, const float (&x)[4]) {
+        *reinterpret_cast<float4*>(dst + o) = make_float4(x[0], x[1], x[2], x[3]);
+        if (dhi) {
+          uint32_t hi[2], lo[2];
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const __nv_bfloat162 h2 = __floats2bfloat162_rn(x[2 * e], x[2 * e + 1]);
+            const float2 hf = __bfloat1622float2(h2);
+            const __nv_bfloat162 l2 = __floats2bfloat162_rn(x[2 * e] - hf.x, x[2 * e + 1] - hf.y);
+            hi[e] = *reinterpret_cast<const uint32_t*>(&h2);
+            lo[e] = *reinterpret_cast<const uint32_t*>(&l2);
+          }
+          *reinterpret_cast<uint2*>(dhi + o) = make_uint2(hi[0], hi[1]);
+          *reinterpret_cast<uint2*>(dlo + o) = make_uint2(lo[0], lo[1]);
+        }
+      };
+      if (head < ep.n_q + 2 * ep.n_kv) {
+#pragma unroll 2
+        for (int c = cbeg + cg; c < cend; c += 8) {
+          const float rs = ep.rs_sumsq ? rsc[c - cbeg] : 1.f;
+          const float4 a4 = *reinterpret_cast<const float4*>(acc + c * kBM + row_a);
+          const float4 b4 = *reinterpret_cast<const float4*>(acc + c * kBM + row_b);
+          float4 r0 = make_float4(1.f, 0.f, 1.f, 0.f), r1 = r0;   // (cos, sin) of pairs i, i+1 / i+2, i+3
+          if (rot) {
+            const float4* rp = reinterpret_cast<const float4*>(ep.rope + c * half + i);
+            r0 = rp[0];
+            r1 = rp[1];
+          }
+          const float cs_[4] = {r0.x, r0.z, r1.x, r1.z}, sn_[4] = {r0.y, r0.w, r1.y, r1.w};
+          const float av[4] = {a4.x * rs, a4.y * rs, a4.z * rs, a4.w * rs};
+          const float bv[4] = {b4.x * rs, b4.y * rs, b4.z * rs, b4.w * rs};
+          float oa[4], ob[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            if (rot) {
+              oa[e] = av[e] * cs_[e] - bv[e] * sn_[e];
+              ob[e] = bv[e] * cs_[e] + av[e] * sn_[e];
+            } else {
+              oa[e] = av[e];
+              ob[e] = bv[e];
+            }
+          }
+          if (head < ep.n_q) {
+            const int64_t o = (static_cast<int64_t>(c) * ep.n_q + head) * hd + i;
+            store4(ep.q, ep.q_hi, ep.q_lo, o, oa);
+            store4(ep.q, ep.q_hi, ep.q_lo, o + half, ob);
+          } else {
+            const bool is_k = head < ep.n_q + ep.n_kv;
+            const int kvh = is_k ? head - ep.n_q : head - ep.n_q - ep.n_kv;
+            float* dst = is_k ? ep.kself : ep.vself;
+            const int64_t o = (static_cast<int64_t>(c) * ep.n_kv + kvh) * hd + i;
+            store4(dst, nullptr, nullptr, o, oa);
+            store4(dst, nullptr, nullptr, o + half, ob);
+          }
+        }
+      }
     } else {   // QKV: pair p = m & 63 of this tile, two column groups of 64 threads
       const int p = m & 63, half_sel = m >> 6;
       const int hd = ep.hd, half = hd / 2;

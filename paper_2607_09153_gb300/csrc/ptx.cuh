@@ -324,6 +324,18 @@ __device__ __forceinline__ float ld_cluster(const float* local, uint32_t rank) {
   return v;
 }
 
+// 16 bytes of a cluster peer's shared memory (16-byte aligned), same offset as `local`.
+__device__ __forceinline__ float4 ld_cluster4(const float* local, uint32_t rank) {
+  uint32_t a;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(smem_u32(local)), "r"(rank));
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(a)
+               : "memory");
+  return v;
+}
+
 // ---------------------------------------------------------------- PDL
 // Programmatic dependent launch: wait for the preceding grid's completion
 // (and memory flush) / allow the next grid to begin launching.
