@@ -60,7 +60,7 @@ __device__ __forceinline__ void store_hilo(__nv_bfloat16* hi, __nv_bfloat16* lo,
   lo[i] = __float2bfloat16_rn(x - __bfloat162float(h));
 }
 
-// LARGE (n_pad > 64, one kernel image per batch class so that the small-batch code keeps its own
+// LARGE (n_pad >= 64, one kernel image per batch class so that the small-batch code keeps its own
 // register allocation): the residual epilogue issues a 16-column group's residual loads before
 // using any and sums each column's squares in one pass over the parked tile, clusters of 4 reduce
 // with 16-byte DSMEM loads, and the epilogues move 4 or 8 consecutive rows of a column per thread
@@ -735,7 +735,7 @@ cudaError_t launch_gemm(const GemmPlan& p, const CUtensorMap* tmW, const CUtenso
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 2 : 1;
-  if (n_pad > 64)
+  if (n_pad >= 64)
     return cudaLaunchKernelEx(&cfg, gemm_cluster_kernel<true>, *tmW, *tmX, p.has_lo ? *tmXlo : *tmX,
                               p.has_lo ? 1 : 0, p.k_tiles, p.cluster, p.stages, p.tmem_cols, n_pad, p.mt, ep, err,
                               ts);
