@@ -29,6 +29,11 @@ DEV_LIB = os.path.join(_BUILD, "libkvsynth_dev.so")
 
 # weight kinds (same numbering the oracle's provider interface uses)
 EMBED, FINAL_NORM, W_PLUS, W_MINUS, ATTN_NORM, W_QKV, W_O, MLP_NORM, W_GATE_UP, W_DOWN = range(10)
+# low-rank adapter factors of each projection (y = W x + scale B (A x)): A [r][in], B [out][r]
+(LORA_A_QKV, LORA_B_QKV, LORA_A_O, LORA_B_O, LORA_A_GATE_UP, LORA_B_GATE_UP, LORA_A_DOWN,
+ LORA_B_DOWN) = range(10, 18)
+LORA_KINDS = tuple(range(10, 18))
+LAYER_KINDS = (ATTN_NORM, W_QKV, W_O, MLP_NORM, W_GATE_UP, W_DOWN)
 GAIN_KINDS = (FINAL_NORM, ATTN_NORM, MLP_NORM)
 
 
@@ -146,21 +151,33 @@ class Arch:
     rope_base: float = 1e4
     rms_eps: float = 1e-6
     page_size: int = 16
+    lora_rank: int = 0          # 0: merged scorer weights; else an adapter of this rank on every projection
+    lora_alpha: float = 32.0    # adapter scale alpha / rank
+
+    @property
+    def lora_scale(self) -> float:
+        return self.lora_alpha / self.lora_rank if self.lora_rank else 0.0
+
+    def layer_kinds(self) -> tuple[int, ...]:
+        return LAYER_KINDS + (LORA_KINDS if self.lora_rank else ())
 
     @property
     def qkv_rows(self) -> int:
         return (self.n_q_heads + 2 * self.n_kv_heads) * self.head_dim
 
     def weight_shape(self, kind: int) -> tuple[int, ...]:
-        d, hd = self.d_model, self.head_dim
+        d, hd, r = self.d_model, self.head_dim, self.lora_rank
         return {
             EMBED: (d,), FINAL_NORM: (d,), W_PLUS: (d,), W_MINUS: (d,), ATTN_NORM: (d,),
             W_QKV: (self.qkv_rows, d), W_O: (d, self.n_q_heads * hd), MLP_NORM: (d,),
             W_GATE_UP: (2 * self.d_ff, d), W_DOWN: (d, self.d_ff),
+            LORA_A_QKV: (r, d), LORA_B_QKV: (self.qkv_rows, r), LORA_A_O: (r, self.n_q_heads * hd), LORA_B_O: (d, r),
+            LORA_A_GATE_UP: (r, d), LORA_B_GATE_UP: (2 * self.d_ff, r), LORA_A_DOWN: (r, self.d_ff),
+            LORA_B_DOWN: (d, r),
         }[kind]
 
     def weight_bytes(self) -> int:
-        per_layer = sum(int(np.prod(self.weight_shape(k))) for k in (ATTN_NORM, W_QKV, W_O, MLP_NORM, W_GATE_UP, W_DOWN))
+        per_layer = sum(int(np.prod(self.weight_shape(k))) for k in self.layer_kinds())
         top = sum(int(np.prod(self.weight_shape(k))) for k in (EMBED, FINAL_NORM, W_PLUS, W_MINUS))
         return 2 * (self.n_layers * per_layer + top)
 
@@ -351,8 +368,7 @@ def host_weight(arch: Arch, kind: int, layer: int, seed: int, tables: Tables) ->
 def host_weights(arch: Arch, seed: int, tables: Tables) -> dict:
     """All weights as bf16 bit arrays: {'top': {kind: arr}, 'layers': [{kind: arr}]}"""
     top = {k: host_weight(arch, k, 0, seed, tables) for k in (EMBED, FINAL_NORM, W_PLUS, W_MINUS)}
-    layers = [{k: host_weight(arch, k, l, seed, tables) for k in (ATTN_NORM, W_QKV, W_O, MLP_NORM, W_GATE_UP, W_DOWN)}
-              for l in range(arch.n_layers)]
+    layers = [{k: host_weight(arch, k, l, seed, tables) for k in arch.layer_kinds()} for l in range(arch.n_layers)]
     return {"top": top, "layers": layers}
 
 
@@ -410,8 +426,7 @@ class DeviceInputs:
             return t
 
         self.top = {k: fill(k, 0) for k in (EMBED, FINAL_NORM, W_PLUS, W_MINUS)}
-        self.layers = [{k: fill(k, l) for k in (ATTN_NORM, W_QKV, W_O, MLP_NORM, W_GATE_UP, W_DOWN)}
-                       for l in range(a.n_layers)]
+        self.layers = [{k: fill(k, l) for k in a.layer_kinds()} for l in range(a.n_layers)]
         P = a.page_size
         self.n_pages = w.n_pages + pool_slack_pages
         self.pool = torch.empty((a.n_layers, self.n_pages, 2, a.n_kv_heads, P, a.head_dim), dtype=torch.bfloat16,

@@ -48,17 +48,19 @@ class OracleCfg(ctypes.Structure):
     _fields_ = [("n_layers", ctypes.c_int), ("d_model", ctypes.c_int), ("n_q_heads", ctypes.c_int),
                 ("n_kv_heads", ctypes.c_int), ("head_dim", ctypes.c_int), ("d_ff", ctypes.c_int),
                 ("rope_base", ctypes.c_double), ("rms_eps", ctypes.c_double), ("mirror", ctypes.c_int),
-                ("nthreads", ctypes.c_int)]
+                ("nthreads", ctypes.c_int), ("lora_rank", ctypes.c_int), ("lora_scale", ctypes.c_double)]
 
     @staticmethod
     def from_arch(arch, mirror: bool = True, nthreads: int | None = None) -> "OracleCfg":
+        rank = int(getattr(arch, "lora_rank", 0))
         return OracleCfg(arch.n_layers, arch.d_model, arch.n_q_heads, arch.n_kv_heads, arch.head_dim, arch.d_ff,
                          float(arch.rope_base), float(arch.rms_eps), int(mirror),
-                         int(nthreads or max(1, os.cpu_count() or 1)))
+                         int(nthreads or max(1, os.cpu_count() or 1)), rank,
+                         float(arch.lora_alpha) / rank if rank else 0.0)
 
 
 class DenseWeights(ctypes.Structure):
-    _fields_ = [("top", _u16p * 4), ("layer", ctypes.POINTER(_u16p) * 6)]
+    _fields_ = [("top", _u16p * 4), ("layer", ctypes.POINTER(_u16p) * 14)]
 
 
 class DenseKV(ctypes.Structure):
@@ -181,7 +183,8 @@ def score_synth(w, tables, cand_ids=None, mirror: bool = True, want_attn: bool =
 
 def score_dense(arch, weights: dict, kv: list, mirror: bool = True, want_attn: bool = True, want_hidden: bool = False,
                 nthreads: int | None = None, mutant: int = 0) -> Result:
-    """Score from explicit arrays.  weights = {'top': {kind: bits}, 'layers': [{kind: bits}]};
+    """Score from explicit arrays.  weights = {'top': {kind: bits}, 'layers': [{kind: bits}]} (kinds 4..9, and
+    the adapter factors 10..17 when arch.lora_rank > 0);
     kv[l][b] = (K_bits [L_b][nkv][hd], V_bits [L_b][nkv][hd])."""
     keep = []
     dw = DenseWeights()
@@ -189,7 +192,9 @@ def score_dense(arch, weights: dict, kv: list, mirror: bool = True, want_attn: b
         a, ap = _u16(weights["top"][k])
         keep.append(a)
         dw.top[k] = ap
-    for j, kind in enumerate(range(4, 10)):
+    kinds = range(4, 18) if getattr(arch, "lora_rank", 0) else range(4, 10)   # with an adapter: its factors too
+    for kind in kinds:
+        j = kind - 4
         ptrs = (_u16p * arch.n_layers)()
         for l in range(arch.n_layers):
             a, ap = _u16(weights["layers"][l][kind])

@@ -34,6 +34,13 @@
  *     h  += W_down (SiLU(W_gate x) * (W_up x))      W_gate_up rows: [gate | up]
  *   then x = RMSNorm(h) * g_final, z_+ = w_plus . x, z_- = w_minus . x.
  *
+ *   Scorer adapter, Sec. 4.1 (f_{theta + Delta theta}, a LoRA adapter) and App.
+ *   B.1 (rank r = 256, alpha = 32): when lora_rank > 0 each of the four
+ *   projections y = W x above becomes y = W x + s B (A x) with its own factors
+ *   A [r][in] and B [out][r] and s = lora_scale (alpha / r); A x is a
+ *   projection input like x (rounded to bf16 in mirror mode).  With
+ *   lora_rank = 0 the weights are the merged scorer's.
+ *
  * Precision.  The paper trains and serves in bf16 (App. B.1), so weights and
  * cached K/V are bf16 values.  "exact" mode (mirror = 0) computes everything
  * else exactly (double) on those bf16 inputs; it is the reference the CUDA
@@ -57,7 +64,9 @@
 #include <string.h>
 
 /* weight kinds, as asked of the weight provider */
-enum { K_EMBED = 0, K_FINAL_NORM, K_W_PLUS, K_W_MINUS, K_ATTN_NORM, K_W_QKV, K_W_O, K_MLP_NORM, K_W_GATE_UP, K_W_DOWN };
+enum { K_EMBED = 0, K_FINAL_NORM, K_W_PLUS, K_W_MINUS, K_ATTN_NORM, K_W_QKV, K_W_O, K_MLP_NORM, K_W_GATE_UP, K_W_DOWN,
+       K_LORA_A_QKV, K_LORA_B_QKV, K_LORA_A_O, K_LORA_B_O, K_LORA_A_GATE_UP, K_LORA_B_GATE_UP, K_LORA_A_DOWN,
+       K_LORA_B_DOWN };
 
 typedef int (*oracle_weight_fn)(void* user, int kind, int layer, uint16_t* out, int64_t n);
 typedef int (*oracle_kv_fn)(void* user, int layer, int cand, uint16_t* K, uint16_t* V, int64_t L);
@@ -67,6 +76,8 @@ typedef struct {
     double rope_base, rms_eps;
     int mirror;   /* 1: bf16 rounding at the precision contract's points; 0: exact */
     int nthreads;
+    int lora_rank;       /* 0: no adapter */
+    double lora_scale;   /* s in y = W x + s B (A x) */
 } oracle_cfg;
 
 /* ------------------------------------------------------------------ numbers */
@@ -225,6 +236,27 @@ static void project(const oracle_cfg* cfg, const uint16_t* W, int rows, int cols
     par_for(rows, cfg->nthreads, proj_row, &c);
 }
 
+/* The adapter term of one projection: y[i][r] += s * sum_j B[r][j] t[i][j], t = A x (t and tmp are
+ * scratch of n * lora_rank and n * rows doubles). */
+static void lora_add(const oracle_cfg* cfg, const uint16_t* A, const uint16_t* B, int rows, int cols,
+                     const double* x, double* y, int n, double* t, double* tmp) {
+    const int r = cfg->lora_rank;
+    project(cfg, A, r, cols, x, t, n, 0, 0);
+    for (int64_t e = 0; e < (int64_t)n * r; ++e) t[e] = rnd(cfg, t[e]);
+    project(cfg, B, rows, r, t, tmp, n, 0, 0);
+#if ORACLE_MUTANT == 15 /* planted mistake: adapter scale left out */
+    const double s = 1.0;
+#else
+    const double s = cfg->lora_scale;
+#endif
+    for (int64_t e = 0; e < (int64_t)n * rows; ++e)
+#if ORACLE_MUTANT == 16 /* planted mistake: adapter term subtracted */
+        y[e] -= s * tmp[e];
+#else
+        y[e] += s * tmp[e];
+#endif
+}
+
 /* ------------------------------------------------------------- attention */
 typedef struct {
     const oracle_cfg* cfg;
@@ -288,6 +320,25 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
     double *gu = calloc((size_t)n * 2 * ff, 8), *a = calloc((size_t)n * ff, 8);
     uint16_t** K = calloc((size_t)n, sizeof(uint16_t*));
     uint16_t** V = calloc((size_t)n, sizeof(uint16_t*));
+    /* adapter factors of the four projections (A [r][in], B [out][r]) and scratch */
+    const int r = cfg->lora_rank;
+    const int64_t in_of[4] = { d, (int64_t)nq * hd, d, ff }, out_of[4] = { qkv_rows, d, 2 * (int64_t)ff, d };
+    uint16_t* LA[4] = { NULL, NULL, NULL, NULL };
+    uint16_t* LB[4] = { NULL, NULL, NULL, NULL };
+    double *lt = NULL, *ltmp = NULL;
+    if (r < 0) { rc = -1; goto done; }
+    if (r > 0) {
+        int64_t most = qkv_rows > 2 * (int64_t)ff ? qkv_rows : 2 * (int64_t)ff;
+        if (d > most) most = d;
+        for (int j = 0; j < 4; ++j) {
+            LA[j] = malloc(2 * (size_t)r * in_of[j]);
+            LB[j] = malloc(2 * (size_t)out_of[j] * r);
+            if (!LA[j] || !LB[j]) { rc = -2; goto done; }
+        }
+        lt = calloc((size_t)n * r, 8);
+        ltmp = calloc((size_t)n * most, 8);
+        if (!lt || !ltmp) { rc = -2; goto done; }
+    }
     if (!embed || !gfin || !wp || !wm || !gattn || !gmlp || !Wqkv || !Wo || !Wgu || !Wd || !h || !x || !qkv || !q ||
         !ks || !vs || !o || !gu || !a || !K || !V) {
         rc = -2;
@@ -313,6 +364,12 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
             rc = -3;
             goto done;
         }
+        for (int j = 0; j < 4 && r > 0; ++j)
+            if (wfn(wuser, K_LORA_A_QKV + 2 * j, l, LA[j], (int64_t)r * in_of[j]) ||
+                wfn(wuser, K_LORA_B_QKV + 2 * j, l, LB[j], out_of[j] * r)) {
+                rc = -3;
+                goto done;
+            }
         for (int i = 0; i < n; ++i)
             if (lens[i] > 0 && kvfn(kvuser, l, cand_ids[i], K[i], V[i], lens[i])) { rc = -4; goto done; }
 
@@ -327,6 +384,7 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
             for (int c = 0; c < d; ++c) xi[c] = rnd(cfg, xi[c]);
         }
         project(cfg, Wqkv, qkv_rows, d, x, qkv, n, 0, 0);
+        if (r > 0) lora_add(cfg, LA[0], LB[0], qkv_rows, d, x, qkv, n, lt, ltmp);
         for (int i = 0; i < n; ++i) {
             const double* r = qkv + (int64_t)i * qkv_rows;
 #if ORACLE_MUTANT == 8 /* planted mistake: verify token placed on the last cached position */
@@ -372,6 +430,7 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
 #else
         project(cfg, Wo, d, nq * hd, o, h, n, 1, 0);
 #endif
+        if (r > 0) lora_add(cfg, LA[1], LB[1], d, nq * hd, o, h, n, lt, ltmp);
 
         /* feed-forward block */
         for (int i = 0; i < n; ++i) {
@@ -380,6 +439,7 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
             for (int c = 0; c < d; ++c) xi[c] = rnd(cfg, xi[c]);
         }
         project(cfg, Wgu, 2 * ff, d, x, gu, n, 0, 0);
+        if (r > 0) lora_add(cfg, LA[2], LB[2], 2 * ff, d, x, gu, n, lt, ltmp);
         for (int i = 0; i < n; ++i)
             for (int j = 0; j < ff; ++j) {
                 double gt = gu[(int64_t)i * 2 * ff + j], up = gu[(int64_t)i * 2 * ff + ff + j];
@@ -397,6 +457,7 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
 #else
         project(cfg, Wd, d, ff, a, h, n, 1, 0);
 #endif
+        if (r > 0) lora_add(cfg, LA[3], LB[3], d, ff, a, h, n, lt, ltmp);
         if (h_layers_out) memcpy(h_layers_out + (int64_t)l * n * d, h, 8 * (size_t)n * d);
     }
 
@@ -417,6 +478,8 @@ done:
     free(K); free(V);
     free(embed); free(gfin); free(wp); free(wm); free(gattn); free(gmlp);
     free(Wqkv); free(Wo); free(Wgu); free(Wd);
+    for (int j = 0; j < 4; ++j) { free(LA[j]); free(LB[j]); }
+    free(lt); free(ltmp);
     free(h); free(x); free(qkv); free(q); free(ks); free(vs); free(o); free(gu); free(a);
     return rc;
 }
@@ -425,7 +488,7 @@ done:
 /* Weights held in caller arrays: top[kind] for kinds 0..3, layer[kind-4][l] otherwise. */
 typedef struct {
     const uint16_t* top[4];
-    const uint16_t* const* layer[6];
+    const uint16_t* const* layer[14];   /* kinds 4 .. 17 (the adapter factors may be NULL without an adapter) */
 } oracle_dense_weights;
 
 int oracle_dense_weight_provider(void* user, int kind, int layer, uint16_t* out, int64_t n) {

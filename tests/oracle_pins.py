@@ -126,4 +126,52 @@ def pin_reencode(m=0, lens=(0, 1, 5, 16, 17, 40), mirror=True, arch=None):
         np.testing.assert_allclose(r.attn[:, 0], attn, rtol=1e-9, atol=1e-12)
 
 
-ALL_PINS = [pin_bf16_round, pin_rmsnorm, pin_rope, pin_attend, pin_reward, pin_reencode]
+def pin_lora_merged(m=0):
+    """The scorer adapter (Sec. 4.1 f_{theta + Delta theta}; App. B.1 r, alpha) equals its merged weights:
+    W x + s B (A x) = (W + s B A) x.  With A a column selection (one 1 per row) and W and s B on a grid of
+    2^-10 below 256 steps, W + s B A is exactly a bf16 matrix, so the unmerged scorer (rank 64, s = 1/2)
+    and the merged one must agree to fp64 rounding on every projection, in both modes."""
+    import dataclasses
+    base = ks.ARCH_TINY
+    arch = dataclasses.replace(base, lora_rank=64)
+    s, r = arch.lora_scale, arch.lora_rank
+    assert s == 0.5
+    rng = np.random.default_rng(515)
+    W = ks.host_weights(base, 78, ks.Tables.make(0.2))
+    proj = [(ks.W_QKV, ks.LORA_A_QKV, ks.LORA_B_QKV), (ks.W_O, ks.LORA_A_O, ks.LORA_B_O),
+            (ks.W_GATE_UP, ks.LORA_A_GATE_UP, ks.LORA_B_GATE_UP), (ks.W_DOWN, ks.LORA_A_DOWN, ks.LORA_B_DOWN)]
+    unmerged = {"top": W["top"], "layers": []}
+    merged = {"top": W["top"], "layers": []}
+    for l in range(arch.n_layers):
+        lu, lm = dict(W["layers"][l]), dict(W["layers"][l])
+        for kw, ka, kb in proj:
+            rows, cols = base.weight_shape(kw)
+            w0 = rng.integers(-100, 101, (rows, cols)) * 2.0 ** -10
+            b = rng.integers(-100, 101, (rows, r)) * 2.0 ** -10 / s
+            sel = rng.choice(cols, r, replace=False)
+            a = np.zeros((r, cols))
+            a[np.arange(r), sel] = 1.0
+            wm = w0.copy()
+            wm[:, sel] += s * b
+            for v in (w0, a, b, wm):   # every value is a bf16 number
+                assert np.array_equal(ks.bf16_bits_to_f64(_bits(v)), v)
+            lu[kw], lu[ka], lu[kb] = _bits(w0), _bits(a), _bits(b)
+            lm[kw] = _bits(wm)
+        unmerged["layers"].append(lu)
+        merged["layers"].append(lm)
+    kv_rng = np.random.default_rng(516)
+    lens = (0, 7, 33)
+    kv = [[tuple(_bits(kv_rng.normal(0, 1, (L, base.n_kv_heads, base.head_dim))) for _ in range(2)) for L in lens]
+          for _ in range(base.n_layers)]
+    for mirror in (False, True):
+        ru = oracle.score_dense(arch, unmerged, kv, mirror=mirror, mutant=m)
+        rm = oracle.score_dense(base, merged, kv, mirror=mirror, mutant=m)
+        assert np.abs(ru.p_plus - rm.p_plus).max() < 1e-12, (mirror, ru.p_plus, rm.p_plus)
+        np.testing.assert_allclose(ru.attn, rm.attn, rtol=1e-9, atol=1e-12)
+    # and the adapter is not a no-op on these weights
+    rb = oracle.score_dense(base, {"top": W["top"], "layers": [
+        {k: v for k, v in lu.items() if k < ks.LORA_A_QKV} for lu in unmerged["layers"]]}, kv, mirror=False, mutant=m)
+    assert np.abs(rb.p_plus - rm.p_plus).max() > 1e-6
+
+
+ALL_PINS = [pin_bf16_round, pin_rmsnorm, pin_rope, pin_attend, pin_reward, pin_reencode, pin_lora_merged]

@@ -17,6 +17,8 @@ MUTANTS = {
     10: "gate not passed through SiLU",
     12: "all query heads read kv head 0",
     14: "gate and up exchanged",
+    15: "adapter scale left out",
+    16: "adapter term subtracted",
 }
 
 

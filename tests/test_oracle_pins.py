@@ -28,6 +28,25 @@ def test_reward():
     P.pin_reward()
 
 
+def test_lora_equals_merged():
+    P.pin_lora_merged()
+
+
+def test_lora_synth_provider():
+    """The seeded generator supplies the adapter factors: with rank 64 the scores move away from the
+    merged scorer's, and a zero-scale adapter (alpha = 0) gives the merged scorer's scores exactly."""
+    import dataclasses
+    t = ks.Tables.make(0.2)
+    w = ks.distinct("lora", ks.ARCH_TINY, 11, [0, 20, 70], gain_std=0.2)
+    r0 = oracle.score_synth(w, t, mirror=False)
+    w.arch = dataclasses.replace(ks.ARCH_TINY, lora_rank=64)
+    r1 = oracle.score_synth(w, t, mirror=False)
+    assert np.abs(r1.p_plus - r0.p_plus).max() > 1e-4
+    w.arch = dataclasses.replace(ks.ARCH_TINY, lora_rank=64, lora_alpha=0.0)
+    r2 = oracle.score_synth(w, t, mirror=False)
+    assert np.array_equal(r2.p_plus, r0.p_plus)
+
+
 @pytest.mark.parametrize("mirror", [True, False])
 def test_reencode_tiny(mirror):
     P.pin_reencode(mirror=mirror)
