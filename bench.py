@@ -143,6 +143,13 @@ def algorithmic_bytes(w) -> dict:
         "gemm_down": a.n_layers * 2 * a.d_model * a.d_ff,
         "attention": w.unique_kv_bytes(),
     }
+    r = a.lora_rank
+    if r:   # scorer adapter: each projection also streams B [out][r]; the A x launches stream A [r][in]
+        per["gemm_qkv"] += a.n_layers * 2 * a.qkv_rows * r
+        per["gemm_o"] += a.n_layers * 2 * a.d_model * r
+        per["gemm_gate_up"] += a.n_layers * 2 * 2 * a.d_ff * r
+        per["gemm_down"] += a.n_layers * 2 * a.d_model * r
+        per["adapter"] = a.n_layers * 2 * r * (2 * a.d_model + a.n_q_heads * a.head_dim + a.d_ff)
     per["weights_total"] = a.weight_bytes()
     per["call_total"] = per["weights_total"] + per["attention"]
     del ks
@@ -216,7 +223,7 @@ def run_reference(args, world, rank):
     if rank != 0:
         return
     import kvsynth as ks
-    w = ks.make_workload(args.workload)
+    w = make_workload(args)
     t = ks.Tables.make()
     samples = []
     budget = max(5.0, 60.0 / max(1, args.steps + args.warmup))
@@ -235,6 +242,17 @@ def run_reference(args, world, rank):
     print(json.dumps(line), flush=True)
 
 
+def make_workload(args):
+    """The named workload; with --lora R its scorer carries an adapter of rank R (alpha 32) apart from
+    the merged weights (every projection y = W x + (alpha / R) B (A x))."""
+    import dataclasses
+    import kvsynth as ks
+    w = ks.make_workload(args.workload)
+    if args.lora:
+        w.arch = dataclasses.replace(w.arch, lora_rank=args.lora)
+    return w
+
+
 def workload_config(w, args) -> dict:
     a = w.arch
     return {"workload": w.name, "layers": a.n_layers, "d_model": a.d_model, "n_q_heads": a.n_q_heads,
@@ -242,7 +260,8 @@ def workload_config(w, args) -> dict:
             "seq_len_min": int(w.seq_lens.min()), "seq_len_max": int(w.seq_lens.max()), "page_size": a.page_size,
             "unique_pages": int(len(set(np.concatenate([w.block_table[b, :(int(w.seq_lens[b]) + 15) // 16]
                                                         for b in range(w.n_candidates)]).tolist()))),
-            "l2": "inputs exceed L2 (weights + cache >> 129 MB); no flush", "parallelism": f"replicas{args.gpus}"}
+            "l2": "inputs exceed L2 (weights + cache >> 129 MB); no flush", "parallelism": f"replicas{args.gpus}",
+            **({"lora_rank": a.lora_rank, "lora_alpha": a.lora_alpha} if a.lora_rank else {})}
 
 
 # ---------------------------------------------------------------- GPU arm
@@ -254,8 +273,12 @@ def make_scorer(dev, max_candidates: int, max_blocks: int):
           "w_minus": dev.top[ks.W_MINUS],
           "layers": [{"attn_norm": L[ks.ATTN_NORM], "w_qkv": L[ks.W_QKV], "w_o": L[ks.W_O], "mlp_norm": L[ks.MLP_NORM],
                       "w_gate_up": L[ks.W_GATE_UP], "w_down": L[ks.W_DOWN]} for L in dev.layers]}
-    return Scorer(a.n_layers, a.d_model, a.n_q_heads, a.n_kv_heads, a.head_dim, a.d_ff, wt, max_candidates, max_blocks,
-                  a.rope_base, a.rms_eps)
+    sc = Scorer(a.n_layers, a.d_model, a.n_q_heads, a.n_kv_heads, a.head_dim, a.d_ff, wt, max_candidates, max_blocks,
+                a.rope_base, a.rms_eps)
+    if a.lora_rank:   # the scorer adapter, kept apart from the base weights
+        names = dict(zip(ks.LORA_KINDS, ("a_qkv", "b_qkv", "a_o", "b_o", "a_gate_up", "b_gate_up", "a_down", "b_down")))
+        sc.set_lora(a.lora_rank, a.lora_alpha, [{names[k]: L[k] for k in ks.LORA_KINDS} for L in dev.layers])
+    return sc
 
 
 def run_gpu(args, world, rank, local):
@@ -265,7 +288,7 @@ def run_gpu(args, world, rank, local):
     import paper_2607_09153_gb300 as kp
 
     torch.cuda.set_device(local)
-    w = ks.make_workload(args.workload)
+    w = make_workload(args)
     tables = ks.Tables.make()
     dev = ks.DeviceInputs(w, tables)
     a = w.arch
@@ -408,7 +431,7 @@ def run_attention_only(args, world, rank, local):
     import paper_2607_09153_gb300 as kp
 
     torch.cuda.set_device(local)
-    w = ks.make_workload(args.workload)
+    w = make_workload(args)
     a = w.arch
     # the workload's heads and cache on a one-layer scorer (its projections are never run here)
     w1 = dataclasses.replace(w, arch=ks.Arch(1, 256, a.n_q_heads, a.n_kv_heads, a.head_dim, 256, a.rope_base,
@@ -477,6 +500,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="qwen1p5b_b16_l2048", choices=list(ks.WORKLOAD_NAMES))
+    ap.add_argument("--lora", type=int, default=0,
+                    help="scorer adapter rank kept apart from the weights (0: merged weights, the default)")
     ap.add_argument("--profile-steps", type=int, default=50)
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")

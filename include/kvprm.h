@@ -116,6 +116,39 @@ KVPRM_API int kvprm_create(const kvprm_config* cfg, const kvprm_weights* weights
  * KVPRM_NO_GRAPH=1 and KVPRM_NO_PDL=1 switch off graph capture and programmatic
  * dependent launch (for debugging). */
 
+/* Scorer adapter kept apart from the base weights (Sec. 4.1: the scorer is
+ * f_{theta + Delta theta}, the base model with a LoRA adapter; App. B.1: rank
+ * r = 256, alpha = 32): every projection y = W x of every layer becomes
+ * y = W x + scale * B (A x), so one copy of the base weights serves both the
+ * generator and the scorer.  Factors are device bf16, row-major, borrowed like
+ * the weights (must outlive the context or the next kvprm_set_lora); each
+ * member is a HOST array of N_L device pointers, read during this call only:
+ *  a_qkv[l] [r][d]        b_qkv[l]     [(n_q + 2 n_kv) hd][r]
+ *  a_o[l]   [r][n_q hd]   b_o[l]       [d][r]
+ *  a_gate_up[l] [r][d]    b_gate_up[l] [2 d_ff][r]  rows: gate, then up
+ *  a_down[l] [r][d_ff]    b_down[l]    [d][r]
+ * A per-module adapter on q, k and v (or gate and up) is this form with the
+ * modules' A stacked and B block-diagonal.  Each projection then takes two
+ * launches: t = scale * (A x), kept at fp32 precision as a bf16 hi/lo pair,
+ * then W x + B t as one K loop over the columns of W followed by those of B.
+ *  rank   a multiple of 64 in [64, 1024], or 0 to go back to the merged
+ *         weights alone (lora is then ignored and may be NULL).
+ *  scale  alpha / r in the usual LoRA parameterisation.
+ * Errors: KVPRM_EINVAL (bad rank, NULL or unaligned factor; nothing changes),
+ * KVPRM_ENOMEM.  Takes effect for the next scoring call (the captured graph
+ * is rebuilt). */
+typedef struct {
+  const void* const* a_qkv;
+  const void* const* b_qkv;
+  const void* const* a_o;
+  const void* const* b_o;
+  const void* const* a_gate_up;
+  const void* const* b_gate_up;
+  const void* const* a_down;
+  const void* const* b_down;
+} kvprm_lora;
+KVPRM_API int kvprm_set_lora(kvprm_ctx* ctx, int32_t rank, float scale, const kvprm_lora* lora);
+
 /* Free the workspace.  Waits for work the context enqueued.  NULL is a no-op. */
 KVPRM_API void kvprm_destroy(kvprm_ctx* ctx);
 
@@ -325,7 +358,8 @@ KVPRM_API int kvprm_check_device(kvprm_ctx* ctx);
  * launch overlap is switched off meanwhile, so each launch is timed alone).
  * Classes: 0..3 the QKV, O, gate/up and down projections, 4 paged attention
  * (split-K, CUDA cores), 5 attention combine, 6 fused norm / RoPE / SiLU /
- * head kernels, 7 paged attention of shared pages on the tensor cores.
+ * head kernels, 7 paged attention of shared pages on the tensor cores, 8 the
+ * scorer adapter's A x products (kvprm_set_lora).
  * Profiled calls synchronise the stream.  kvprm_get_profile returns per class
  * the launch count and total milliseconds since profiling was enabled. */
 enum {
@@ -337,7 +371,8 @@ enum {
   KVPRM_PROF_COMBINE = 5,
   KVPRM_PROF_FUSED = 6,
   KVPRM_PROF_ATTN_TC = 7,
-  KVPRM_PROF_N = 8
+  KVPRM_PROF_LORA = 8,
+  KVPRM_PROF_N = 9
 };
 KVPRM_API int kvprm_set_profile(kvprm_ctx* ctx, int enable);
 

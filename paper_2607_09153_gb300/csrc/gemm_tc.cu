@@ -70,6 +70,9 @@ template <bool LARGE>
 __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant__ CUtensorMap tmW,
                                                            const __grid_constant__ CUtensorMap tmX,
                                                            const __grid_constant__ CUtensorMap tmXlo, int has_lo,
+                                                           const __grid_constant__ CUtensorMap tmB,
+                                                           const __grid_constant__ CUtensorMap tmT,
+                                                           const __grid_constant__ CUtensorMap tmTlo, int k_main,
                                                            int k_tiles, int cs, int stages, uint32_t tmem_cols,
                                                            int n_pad, int mt_arg, GemmEpilogue ep, int* err,
                                                            unsigned long long* ts) {
@@ -117,6 +120,11 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     tma_prefetch_desc(&tmW);
     tma_prefetch_desc(&tmX);
     if (has_lo) tma_prefetch_desc(&tmXlo);
+    if (k_main < k_tiles) {
+      tma_prefetch_desc(&tmB);
+      tma_prefetch_desc(&tmT);
+      if (has_lo) tma_prefetch_desc(&tmTlo);
+    }
   }
   if (warp == 1) {
     tmem_alloc(tmem_slot, tmem_cols);
@@ -135,17 +143,26 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     // ---------------- TMA producer
     const uint64_t pol_w = policy_evict_first();
     const uint64_t pol_x = policy_evict_last();
+    // K tiles [0, k_main) come from W and x; a scorer adapter's tiles after them from B and t
     auto load_w = [&](uint8_t* st, int kt, uint64_t* bar) {
+      const CUtensorMap* wm = kt < k_main ? &tmW : &tmB;
+      const int kx = (kt < k_main ? kt : kt - k_main) * kBK;
       for (int t = 0; t < mt; ++t) {
         const int m_tile = m_tile0 + t;
         uint8_t* wt = st + t * kWTileBytes;
         if (!silu) {
-          tma_load_2d(wt, &tmW, bar, kt * kBK, m_tile * kBM, pol_w);
+          tma_load_2d(wt, wm, bar, kx, m_tile * kBM, pol_w);
         } else {   // 64 gate rows, then the matching 64 up rows
-          tma_load_2d(wt, &tmW, bar, kt * kBK, m_tile * 64, pol_w);
-          tma_load_2d(wt + kWTileBytes / 2, &tmW, bar, kt * kBK, ep.ff + m_tile * 64, pol_w);
+          tma_load_2d(wt, wm, bar, kx, m_tile * 64, pol_w);
+          tma_load_2d(wt + kWTileBytes / 2, wm, bar, kx, ep.ff + m_tile * 64, pol_w);
         }
       }
+    };
+    auto load_x = [&](uint8_t* st, int kt, uint64_t* bar) {
+      const bool main = kt < k_main;
+      const int kx = (main ? kt : kt - k_main) * kBK;
+      tma_load_2d(st + w_bytes, main ? &tmX : &tmT, bar, kx, 0, pol_x);
+      if (has_lo) tma_load_2d(st + w_bytes + x_bytes, main ? &tmXlo : &tmTlo, bar, kx, 0, pol_x);
     };
     // Weights do not depend on the preceding kernel: start streaming the first
     // ring's worth of W before waiting for the activations it produces.
@@ -156,11 +173,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     }
     grid_dep_wait();
     trace_event(ts, 0);   // the preceding kernel has completed
-    for (int i = 0; i < pre; ++i) {
-      tma_load_2d(smem + i * stage_bytes + w_bytes, &tmX, &full[i], (kt0 + i) * kBK, 0, pol_x);
-      if (has_lo)
-        tma_load_2d(smem + i * stage_bytes + w_bytes + x_bytes, &tmXlo, &full[i], (kt0 + i) * kBK, 0, pol_x);
-    }
+    for (int i = 0; i < pre; ++i) load_x(smem + i * stage_bytes, kt0 + i, &full[i]);
     for (int i = pre; i < nk; ++i) {
       const int s = i % stages;
       const uint32_t use = static_cast<uint32_t>(i / stages);
@@ -168,8 +181,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       uint8_t* st = smem + s * stage_bytes;
       mbar_arrive_expect_tx(&full[s], stage_bytes);
       load_w(st, kt0 + i, &full[s]);
-      tma_load_2d(st + w_bytes, &tmX, &full[s], (kt0 + i) * kBK, 0, pol_x);
-      if (has_lo) tma_load_2d(st + w_bytes + x_bytes, &tmXlo, &full[s], (kt0 + i) * kBK, 0, pol_x);
+      load_x(st, kt0 + i, &full[s]);
     }
   } else if (warp >= 2) {
     // ---------------- while the weights stream: the RMSNorm factor of each of this rank's columns
@@ -343,6 +355,11 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       const int gm = m_tile * kBM + m;
       if (gm < ep.M)
         for (int c = cbeg; c < cend; ++c) ep.out[static_cast<int64_t>(c) * ep.M + gm] = acc[c * kBM + m];
+    } else if (LARGE && ep.mode == GemmEpilogue::LOWRANK) {   // t = s (A x), hi/lo [n][r]; large image only
+      const int gm = m_tile * kBM + m;
+      if (gm < ep.M)
+        for (int c = cbeg; c < cend; ++c)
+          store_hilo(ep.t_hi, ep.t_lo, static_cast<int64_t>(c) * ep.M + gm, ep.lr_scale * acc[c * kBM + m]);
     } else if (ep.mode == GemmEpilogue::RESID && LARGE) {
       // pass 1, 16 columns at a time with the group's residual loads in flight before the first use:
       // h += acc, the next projection's input, and hv^2 parked in place of acc (each (column, row)
@@ -720,7 +737,7 @@ cudaError_t gemm_configure() {
 
 cudaError_t launch_gemm(const GemmPlan& p, const CUtensorMap* tmW, const CUtensorMap* tmX, const CUtensorMap* tmXlo,
                         const GemmEpilogue& ep, int n_pad, int* err, cudaStream_t stream, bool pdl,
-                        unsigned long long* ts) {
+                        unsigned long long* ts, const GemmLowRank* lr) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((p.m_tiles + p.mt - 1) / p.mt * p.cluster, 1, 1);
   cfg.blockDim = dim3(128, 1, 1);
@@ -735,12 +752,21 @@ cudaError_t launch_gemm(const GemmPlan& p, const CUtensorMap* tmW, const CUtenso
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = pdl ? 2 : 1;
-  if (n_pad >= 64)
-    return cudaLaunchKernelEx(&cfg, gemm_cluster_kernel<true>, *tmW, *tmX, p.has_lo ? *tmXlo : *tmX,
-                              p.has_lo ? 1 : 0, p.k_tiles, p.cluster, p.stages, p.tmem_cols, n_pad, p.mt, ep, err,
-                              ts);
+  const CUtensorMap& xlo = p.has_lo ? *tmXlo : *tmX;
+  // without an adapter every K tile is W's and x's (the extra maps are never read)
+  const bool with_lr = lr && lr->b && lr->t_hi && (!p.has_lo || lr->t_lo);
+  if (with_lr && (lr->k_main < 1 || lr->k_main >= p.k_tiles)) return cudaErrorInvalidValue;
+  const CUtensorMap& mb = with_lr ? *lr->b : *tmW;
+  const CUtensorMap& mt = with_lr ? *lr->t_hi : *tmX;
+  const CUtensorMap& mtl = with_lr ? (p.has_lo ? *lr->t_lo : *lr->t_hi) : xlo;
+  const int k_main = with_lr ? lr->k_main : p.k_tiles;
+  // the adapter's A x (LOWRANK) runs on the large-batch image at every batch size, so that the
+  // small-batch image keeps its register allocation
+  if (n_pad >= 64 || ep.mode == GemmEpilogue::LOWRANK)
+    return cudaLaunchKernelEx(&cfg, gemm_cluster_kernel<true>, *tmW, *tmX, xlo, p.has_lo ? 1 : 0, mb, mt, mtl, k_main,
+                              p.k_tiles, p.cluster, p.stages, p.tmem_cols, n_pad, p.mt, ep, err, ts);
   if (p.mt != 1) return cudaErrorInvalidValue;   // two m-tiles per CTA exist in the large-batch image only
-  return cudaLaunchKernelEx(&cfg, gemm_cluster_kernel<false>, *tmW, *tmX, p.has_lo ? *tmXlo : *tmX, p.has_lo ? 1 : 0,
+  return cudaLaunchKernelEx(&cfg, gemm_cluster_kernel<false>, *tmW, *tmX, xlo, p.has_lo ? 1 : 0, mb, mt, mtl, k_main,
                             p.k_tiles, p.cluster, p.stages, p.tmem_cols, n_pad, 1, ep, err, ts);
 }
 

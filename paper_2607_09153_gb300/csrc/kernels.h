@@ -30,7 +30,7 @@ struct GemmPlan {
 };
 // What the cluster does with the reduced tile (see gemm_tc.cu).
 struct GemmEpilogue {
-  enum Mode : int { PLAIN = 0, QKV = 1, RESID = 2, SILU = 3 };
+  enum Mode : int { PLAIN = 0, QKV = 1, RESID = 2, SILU = 3, LOWRANK = 4 };
   int mode = PLAIN;
   int M = 0;             // rows of the full output (PLAIN, RESID: row stride of out / h)
   int n_valid = 0;       // candidates
@@ -57,16 +57,30 @@ struct GemmEpilogue {
   int ff = 0;            // SILU: output width; up rows start at row ff of W
   __nv_bfloat16* a_hi = nullptr;
   __nv_bfloat16* a_lo = nullptr;
+  // LOWRANK: t = lr_scale * (A x) as a bf16 hi/lo pair [n][M] (M = the adapter's rank), the extra K
+  // columns of the projection that follows (GemmLowRank)
+  float lr_scale = 0.f;
+  __nv_bfloat16* t_hi = nullptr;
+  __nv_bfloat16* t_lo = nullptr;
   // let the next kernel in the stream launch only once this one's partials are parked (after its
   // first cluster barrier) instead of at entry: a next kernel whose CTAs fit beside this one's on
   // an SM otherwise slows that barrier by ~2.5 us (measured for the O projection before gate/up)
   bool late_trigger = false;
 };
 GemmPlan plan_gemm(int M, int K, int n_pad, int num_sms, bool has_lo, bool gate_up);
+// A scorer adapter's term of a projection, y = W x + B t with t = s A x already computed (LOWRANK):
+// after its k_main K tiles of W and x the projection streams B [out][r] against t [n][r] as further
+// K tiles (the plan counts both: plan_gemm(M, 64 k_main + r, ...)).
+struct GemmLowRank {
+  const CUtensorMap* b = nullptr;      // B, box of the projection's weight tile
+  const CUtensorMap* t_hi = nullptr;   // t hi / lo, box of its activation tile
+  const CUtensorMap* t_lo = nullptr;
+  int k_main = 0;
+};
 cudaError_t gemm_configure();
 cudaError_t launch_gemm(const GemmPlan& p, const CUtensorMap* tmW, const CUtensorMap* tmX, const CUtensorMap* tmXlo,
                         const GemmEpilogue& ep, int n_pad, int* err, cudaStream_t stream, bool pdl,
-                        unsigned long long* ts = nullptr);
+                        unsigned long long* ts = nullptr, const GemmLowRank* lr = nullptr);
 
 // ---------------------------------------------------------------- paged attention
 struct AttnShape {

@@ -7,6 +7,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <cmath>
 #include <cstdarg>
 #include <cstdio>
 #include <cstdlib>
@@ -27,6 +28,9 @@ namespace {
 struct CallPlan {
   int n = 0, n_pad = 0, max_pages = 0;
   GemmPlan g_qkv, g_o, g_gu, g_down;
+  // scorer adapter: the A x launches, and each projection's K tiles of W (the rest are B's)
+  GemmPlan l_qkv, l_o, l_gu, l_down;
+  int k_qkv = 0, k_o = 0, k_gu = 0, k_down = 0;
   int attn_ctas = 0;   // grid of the attention (see build_attn_work)
 };
 
@@ -34,11 +38,12 @@ struct GraphKey {
   int n = -1, n_pad = -1, attn_ctas = -1, tc_ctas = -1, n_tc = -1, debug = -1, profile = -1, pdl = -1, trace = -1;
   int fuse_cs = -1;
   int layer_waits = -1;
+  int lora_rank = -1;
   const void* pool = nullptr;
   int64_t n_pages = -1;
   bool operator==(const GraphKey& o) const {
     return n == o.n && n_pad == o.n_pad && attn_ctas == o.attn_ctas && tc_ctas == o.tc_ctas && n_tc == o.n_tc &&
-           fuse_cs == o.fuse_cs && layer_waits == o.layer_waits &&
+           fuse_cs == o.fuse_cs && layer_waits == o.layer_waits && lora_rank == o.lora_rank &&
            debug == o.debug && profile == o.profile && pdl == o.pdl && trace == o.trace && pool == o.pool &&
            n_pages == o.n_pages;
   }
@@ -61,6 +66,15 @@ struct kvprm_ctx {
   const bf16 *embed = nullptr, *final_norm = nullptr, *w_plus = nullptr, *w_minus = nullptr;
   std::vector<const bf16*> attn_norm, mlp_norm;
   std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_down;
+  // scorer adapter (kvprm_set_lora; rank 0: the merged weights alone): per projection (QKV, O,
+  // gate/up, down) and layer the maps of A and B, and t = scale (A x) as hi/lo [npad_max][rank]
+  int lora_rank = 0;
+  float lora_scale = 0.f;
+  std::vector<CUtensorMap> tm_la[4], tm_lb[4];
+  bf16 *thi = nullptr, *tlo = nullptr;
+  size_t t_cap = 0;
+  int tm_t_npad = -1;
+  CUtensorMap tm_thi{}, tm_tlo{};
   // workspace
   int npad_max = 16;
   float* h = nullptr;
@@ -202,6 +216,8 @@ void free_ctx(kvprm_ctx* c) {
   cudaFree(c->olo);
   cudaFree(c->ahi);
   cudaFree(c->alo);
+  cudaFree(c->thi);
+  cudaFree(c->tlo);
   cudaFree(c->qhi);
   cudaFree(c->qlo);
   cudaFree(c->sumsq);
@@ -389,16 +405,41 @@ int ensure_x_maps(kvprm_ctx* ctx, int n_pad) {
   return KVPRM_OK;
 }
 
+// the adapter's t = scale (A x) buffer as the K-extension operand of a batch padded to n_pad
+int ensure_t_maps(kvprm_ctx* ctx, int n_pad) {
+  if (ctx->lora_rank == 0 || ctx->tm_t_npad == n_pad) return KVPRM_OK;
+  int rc;
+  const uint64_t r = static_cast<uint64_t>(ctx->lora_rank);
+  if ((rc = make_map(ctx, &ctx->tm_thi, ctx->thi, r, n_pad, 64, n_pad, "t_hi"))) return rc;
+  if ((rc = make_map(ctx, &ctx->tm_tlo, ctx->tlo, r, n_pad, 64, n_pad, "t_lo"))) return rc;
+  ctx->tm_t_npad = n_pad;
+  return KVPRM_OK;
+}
+
 CallPlan make_plan(kvprm_ctx* ctx, int n, int max_pages) {
   CallPlan p;
   p.n = n;
   p.n_pad = (n + 15) / 16 * 16;
   p.max_pages = max_pages;
   const ModelDims& m = ctx->md;
-  p.g_qkv = kvprm::plan_gemm(m.qkv_rows, m.d, p.n_pad, ctx->num_sms, true, false);
-  p.g_o = kvprm::plan_gemm(m.d, m.n_q * m.hd, p.n_pad, ctx->num_sms, true, false);
-  p.g_gu = kvprm::plan_gemm(m.ff, m.d, p.n_pad, ctx->num_sms, true, true);
-  p.g_down = kvprm::plan_gemm(m.d, m.ff, p.n_pad, ctx->num_sms, true, false);
+  // with an adapter each projection's K loop runs on over B's r columns (W's last tile zero-padded)
+  const int r = ctx->lora_rank;
+  auto kt = [](int K) { return (K + 63) / 64; };
+  auto keff = [&](int K) { return r ? 64 * kt(K) + r : K; };
+  p.g_qkv = kvprm::plan_gemm(m.qkv_rows, keff(m.d), p.n_pad, ctx->num_sms, true, false);
+  p.g_o = kvprm::plan_gemm(m.d, keff(m.n_q * m.hd), p.n_pad, ctx->num_sms, true, false);
+  p.g_gu = kvprm::plan_gemm(m.ff, keff(m.d), p.n_pad, ctx->num_sms, true, true);
+  p.g_down = kvprm::plan_gemm(m.d, keff(m.ff), p.n_pad, ctx->num_sms, true, false);
+  if (r) {
+    p.l_qkv = kvprm::plan_gemm(r, m.d, p.n_pad, ctx->num_sms, true, false);
+    p.l_o = kvprm::plan_gemm(r, m.n_q * m.hd, p.n_pad, ctx->num_sms, true, false);
+    p.l_gu = kvprm::plan_gemm(r, m.d, p.n_pad, ctx->num_sms, true, false);
+    p.l_down = kvprm::plan_gemm(r, m.ff, p.n_pad, ctx->num_sms, true, false);
+    p.k_qkv = kt(m.d);
+    p.k_o = kt(m.n_q * m.hd);
+    p.k_gu = kt(m.d);
+    p.k_down = kt(m.ff);
+  }
   p.attn_ctas = ctx->work_host.n_ctas;
   return p;
 }
@@ -543,6 +584,26 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
   es.rs_tiles = ctx->d_tiles;
   es.rs_d = m.d;
   es.rs_eps = m.eps;
+  kvprm::GemmEpilogue et;   // scorer adapter: t = scale (A x), the K extension of the projection after it
+  et.mode = kvprm::GemmEpilogue::LOWRANK;
+  et.M = ctx->lora_rank;
+  et.n_valid = n;
+  et.lr_scale = ctx->lora_scale;
+  et.t_hi = ctx->thi;
+  et.t_lo = ctx->tlo;
+  const bool lora = ctx->lora_rank > 0;
+  // launch A x of projection j (0 QKV, 1 O, 2 gate/up, 3 down) of layer l on the projection's input
+  // maps; returns the K extension the projection itself then takes
+  auto adapter = [&](int j, int l, const GemmPlan& g, const CUtensorMap* xh, const CUtensorMap* xl, int k_main,
+                     kvprm::GemmLowRank* lr) -> int {
+    static const char* what[4] = {"adapter_qkv", "adapter_o", "adapter_gate_up", "adapter_down"};
+    LAUNCH(KVPRM_PROF_LORA, kvprm::launch_gemm(g, &ctx->tm_la[j][l], xh, xl, et, np, ctx->err_d, st, pdl, TS), what[j]);
+    lr->b = &ctx->tm_lb[j][l];
+    lr->t_hi = &ctx->tm_thi;
+    lr->t_lo = &ctx->tm_tlo;
+    lr->k_main = k_main;
+    return KVPRM_OK;
+  };
   ctx->trace_n = 0;
   ctx->trace_cls.clear();
   if (ctx->trace)
@@ -553,8 +614,12 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
          kvprm::launch_embed_norm(m, ctx->embed, ctx->attn_norm[0], n, ctx->h, ctx->sumsq, X, st, pdl, TS),
          "embed_norm");
   for (int l = 0; l < NL; ++l) {
+    kvprm::GemmLowRank lr_qkv, lr_o, lr_gu, lr_down;
+    int arc;
+    if (lora && (arc = adapter(0, l, P.l_qkv, &ctx->tm_xhi, &ctx->tm_xlo, P.k_qkv, &lr_qkv))) return arc;
     LAUNCH(KVPRM_PROF_GEMM_QKV,
-           kvprm::launch_gemm(P.g_qkv, &ctx->tm_qkv[l], &ctx->tm_xhi, &ctx->tm_xlo, eq, np, ctx->err_d, st, pdl, TS),
+           kvprm::launch_gemm(P.g_qkv, &ctx->tm_qkv[l], &ctx->tm_xhi, &ctx->tm_xlo, eq, np, ctx->err_d, st, pdl, TS,
+                              lora ? &lr_qkv : nullptr),
            "gemm_qkv");
     if (ctx->debug_flags & 2) {
       const size_t nq = static_cast<size_t>(n) * m.n_q * m.hd, nk = static_cast<size_t>(n) * m.n_kv * m.hd;
@@ -579,17 +644,22 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
     kvprm::GemmEpilogue er_o = er;   // h += W_o o; x = h ⊙ g_mlp for the gate/up projection
     er_o.gain_next = ctx->mlp_norm[l];
     er_o.late_trigger = true;   // gate/up CTAs fit beside the O projection's
+    if (lora && (arc = adapter(1, l, P.l_o, &ctx->tm_ohi, &ctx->tm_olo, P.k_o, &lr_o))) return arc;
     LAUNCH(KVPRM_PROF_GEMM_O,
-           kvprm::launch_gemm(P.g_o, &ctx->tm_o[l], &ctx->tm_ohi, &ctx->tm_olo, er_o, np, ctx->err_d, st, pdl, TS),
+           kvprm::launch_gemm(P.g_o, &ctx->tm_o[l], &ctx->tm_ohi, &ctx->tm_olo, er_o, np, ctx->err_d, st, pdl, TS,
+                              lora ? &lr_o : nullptr),
            "gemm_o");
+    if (lora && (arc = adapter(2, l, P.l_gu, &ctx->tm_xhi, &ctx->tm_xlo, P.k_gu, &lr_gu))) return arc;
     LAUNCH(KVPRM_PROF_GEMM_GATE_UP,
-           kvprm::launch_gemm(P.g_gu, &ctx->tm_gu[l], &ctx->tm_xhi, &ctx->tm_xlo, es, np, ctx->err_d, st, pdl, TS),
+           kvprm::launch_gemm(P.g_gu, &ctx->tm_gu[l], &ctx->tm_xhi, &ctx->tm_xlo, es, np, ctx->err_d, st, pdl, TS,
+                              lora ? &lr_gu : nullptr),
            "gemm_gate_up");
     kvprm::GemmEpilogue er_d = er;   // h += W_down a; x = h ⊙ g_attn of the next layer
     er_d.gain_next = l + 1 < NL ? ctx->attn_norm[l + 1] : nullptr;
+    if (lora && (arc = adapter(3, l, P.l_down, &ctx->tm_ahi, &ctx->tm_alo, P.k_down, &lr_down))) return arc;
     LAUNCH(KVPRM_PROF_GEMM_DOWN,
            kvprm::launch_gemm(P.g_down, &ctx->tm_down[l], &ctx->tm_ahi, &ctx->tm_alo, er_d, np, ctx->err_d, st, pdl,
-                              TS),
+                              TS, lora ? &lr_down : nullptr),
            "gemm_down");
     if (l + 1 == NL) {
       LAUNCH(KVPRM_PROF_FUSED,
@@ -672,6 +742,7 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   if ((rc = plan_work(ctx, bt, sl, n))) return rc;
   const CallPlan P = make_plan(ctx, n, max_pages);
   if ((rc = ensure_x_maps(ctx, P.n_pad))) return rc;
+  if ((rc = ensure_t_maps(ctx, P.n_pad))) return rc;
   if ((rc = upload_tables(ctx, bt, sl, n, st))) return rc;
   if (ctx->layer_waits && (rc = enqueue_pool_copy(ctx, st))) return rc;
   ctx->last_n = n;
@@ -693,6 +764,7 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   key.tc_ctas = ctx->work_host.n_tc_ctas * (ctx->work_host.tc_concurrent ? -1 : 1);
   key.fuse_cs = ctx->work_host.fuse_cs;
   key.layer_waits = ctx->layer_waits ? 1 : 0;
+  key.lora_rank = ctx->lora_rank;
   key.n_tc = ctx->work_host.n_tc > 0 ? 1 : 0;
   key.debug = ctx->debug_flags;
   key.profile = ctx->profile ? 1 : 0;
@@ -920,6 +992,78 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   CREATE_CK(cu(cudaDeviceSynchronize(), "cudaDeviceSynchronize(create)"));
 #undef CREATE_CK
   *out = ctx;
+  return KVPRM_OK;
+}
+
+int kvprm_set_lora(kvprm_ctx* ctx, int32_t rank, float scale, const kvprm_lora* lora) {
+  if (!ctx) return KVPRM_EINVAL;
+  if (rank == 0) {   // back to the merged weights alone
+    if (ctx->lora_rank != 0) drop_graph(ctx);
+    ctx->lora_rank = 0;
+    ctx->lora_scale = 0.f;
+    return KVPRM_OK;
+  }
+  if (rank < 64 || rank > 1024 || rank % 64)
+    return fail(ctx, KVPRM_EINVAL, "adapter rank %d: a multiple of 64 in [64, 1024], or 0", rank);
+  if (!lora) return fail(ctx, KVPRM_EINVAL, "kvprm_lora is NULL");
+  if (!std::isfinite(scale)) return fail(ctx, KVPRM_EINVAL, "adapter scale is not finite");
+  const ModelDims& m = ctx->md;
+  const int NL = ctx->cfg.n_layers;
+  const void* const* a_of[4] = {lora->a_qkv, lora->a_o, lora->a_gate_up, lora->a_down};
+  const void* const* b_of[4] = {lora->b_qkv, lora->b_o, lora->b_gate_up, lora->b_down};
+  const uint64_t in_of[4] = {static_cast<uint64_t>(m.d), static_cast<uint64_t>(m.n_q) * m.hd,
+                             static_cast<uint64_t>(m.d), static_cast<uint64_t>(m.ff)};
+  const uint64_t out_of[4] = {static_cast<uint64_t>(m.qkv_rows), static_cast<uint64_t>(m.d),
+                              2 * static_cast<uint64_t>(m.ff), static_cast<uint64_t>(m.d)};
+  static const char* nm[4] = {"qkv", "o", "gate_up", "down"};
+  for (int j = 0; j < 4; ++j) {
+    if (!a_of[j] || !b_of[j]) return fail(ctx, KVPRM_EINVAL, "adapter factor arrays of %s are NULL", nm[j]);
+    for (int l = 0; l < NL; ++l)
+      if (!a_of[j][l] || !b_of[j][l] || !aligned16(a_of[j][l]) || !aligned16(b_of[j][l]))
+        return fail(ctx, KVPRM_EINVAL, "adapter factor of %s, layer %d, is NULL or not 16-byte aligned", nm[j], l);
+  }
+  // every map first, so that a failure leaves the context as it was
+  std::vector<CUtensorMap> la[4], lb[4];
+  int rc;
+  for (int j = 0; j < 4; ++j) {
+    la[j].resize(NL);
+    lb[j].resize(NL);
+    for (int l = 0; l < NL; ++l) {
+      // A [r][in]: 128-row tiles of the A x launch; B [out][r]: the projection's own weight tile rows
+      if ((rc = make_map(ctx, &la[j][l], a_of[j][l], in_of[j], static_cast<uint64_t>(rank), 64, 128, "adapter A")))
+        return rc;
+      if ((rc = make_map(ctx, &lb[j][l], b_of[j][l], static_cast<uint64_t>(rank), out_of[j], 64, j == 2 ? 64 : 128,
+                         "adapter B")))
+        return rc;
+    }
+  }
+  const size_t need = static_cast<size_t>(ctx->npad_max) * rank;
+  if (need > ctx->t_cap) {
+    bf16 *th = nullptr, *tl = nullptr;
+    if ((rc = dalloc(ctx, &th, need, "adapter t_hi"))) return rc;
+    if ((rc = dalloc(ctx, &tl, need, "adapter t_lo"))) {
+      cudaFree(th);
+      return rc;
+    }
+    CK(cudaDeviceSynchronize(), "cudaDeviceSynchronize(adapter buffers)");
+    cudaFree(ctx->thi);
+    cudaFree(ctx->tlo);
+    ctx->thi = th;
+    ctx->tlo = tl;
+    ctx->t_cap = need;
+  } else if (rank != ctx->lora_rank) {
+    // padding rows of t (candidates >= n) are read as K-extension columns: keep them zero
+    CK(cudaMemset(ctx->thi, 0, sizeof(bf16) * ctx->t_cap), "cudaMemset(t_hi)");
+    CK(cudaMemset(ctx->tlo, 0, sizeof(bf16) * ctx->t_cap), "cudaMemset(t_lo)");
+  }
+  for (int j = 0; j < 4; ++j) {
+    ctx->tm_la[j] = std::move(la[j]);
+    ctx->tm_lb[j] = std::move(lb[j]);
+  }
+  ctx->lora_rank = rank;
+  ctx->lora_scale = scale;
+  ctx->tm_t_npad = -1;
+  drop_graph(ctx);
   return KVPRM_OK;
 }
 

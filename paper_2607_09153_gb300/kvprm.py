@@ -17,7 +17,8 @@ from . import build as _build
 
 KVPRM_OK, KVPRM_EINVAL, KVPRM_ECAPACITY, KVPRM_EINDEX, KVPRM_ECUDA, KVPRM_ENOMEM, KVPRM_ETIMEOUT, \
     KVPRM_EUNSUPPORTED = range(8)
-PROF_NAMES = ("gemm_qkv", "gemm_o", "gemm_gate_up", "gemm_down", "attention", "combine", "fused", "attention_tc")
+PROF_NAMES = ("gemm_qkv", "gemm_o", "gemm_gate_up", "gemm_down", "attention", "combine", "fused", "attention_tc",
+              "adapter")
 
 
 class KvprmError(RuntimeError):
@@ -40,6 +41,13 @@ class KvprmWeights(ctypes.Structure):
     _fields_ = [("embed_verify", ctypes.c_void_p), ("final_norm", ctypes.c_void_p), ("w_plus", ctypes.c_void_p),
                 ("w_minus", ctypes.c_void_p), ("attn_norm", _VPP), ("w_qkv", _VPP), ("w_o", _VPP),
                 ("mlp_norm", _VPP), ("w_gate_up", _VPP), ("w_down", _VPP)]
+
+
+class KvprmLora(ctypes.Structure):
+    _fields_ = [(k, _VPP) for k in ("a_qkv", "b_qkv", "a_o", "b_o", "a_gate_up", "b_gate_up", "a_down", "b_down")]
+
+
+LORA_FACTORS = ("a_qkv", "b_qkv", "a_o", "b_o", "a_gate_up", "b_gate_up", "a_down", "b_down")
 
 
 class KvprmAttnPlan(ctypes.Structure):
@@ -78,6 +86,7 @@ def lib() -> ctypes.CDLL:
         L.kvprm_score_host.argtypes = [vp, vp, i64, i32p, i32p, i32, f32p, vp]
         L.kvprm_attention.argtypes = [vp, vp, i64, i32p, i32p, i32, vp, vp, vp, vp, vp]
         L.kvprm_projection.argtypes = [vp, vp, i32, i32, vp, i32, vp, vp]
+        L.kvprm_set_lora.argtypes = [vp, i32, ctypes.c_float, ctypes.POINTER(KvprmLora)]
         L.kvprm_debug_hidden.argtypes = [vp, vp]
         L.kvprm_attention_noalloc.argtypes = [vp, i64, i32p, i32, i32p, i32, i32, i32, i32, vp, vp, vp, vp, vp]
         L.kvprm_set_debug.argtypes = [vp, ctypes.c_int]
@@ -161,6 +170,10 @@ def kvprm_attention(ctx, kv_layer_ptr: int, n_pages: int, block_table, seq_lens,
 
 def kvprm_projection(ctx, W_ptr: int, M: int, K: int, X_ptr: int, n: int, Y_ptr: int, stream_ptr: int = 0) -> None:
     _check(ctx, lib().kvprm_projection(ctx, W_ptr, M, K, X_ptr, n, Y_ptr, stream_ptr))
+
+
+def kvprm_set_lora(ctx, rank: int, scale: float, lora: KvprmLora | None) -> None:
+    _check(ctx, lib().kvprm_set_lora(ctx, int(rank), float(scale), ctypes.byref(lora) if lora is not None else None))
 
 
 def kvprm_debug_hidden(ctx, d_out_ptr: int) -> None:
@@ -307,6 +320,19 @@ class Scorer:
                               cast(self._arrays["mlp_norm"]), cast(self._arrays["w_gate_up"]),
                               cast(self._arrays["w_down"]))
         self.ctx = kvprm_create(self.cfg, self.w)
+
+    def set_lora(self, rank: int, alpha: float = 32.0, factors: list | None = None) -> None:
+        """Scorer adapter on every projection (rank 0: merged weights alone); factors[l] holds
+        {'a_qkv', 'b_qkv', 'a_o', 'b_o', 'a_gate_up', 'b_gate_up', 'a_down', 'b_down'} bf16 tensors."""
+        if rank == 0:
+            kvprm_set_lora(self.ctx, 0, 0.0, None)
+            return
+        n = self.cfg.n_layers
+        arr = ctypes.c_void_p * n
+        self._lora_arrays = {k: arr(*[factors[l][k].data_ptr() for l in range(n)]) for k in LORA_FACTORS}
+        self._lora_factors = factors   # keep the tensors alive
+        lo = KvprmLora(*[ctypes.cast(self._lora_arrays[k], _VPP) for k in LORA_FACTORS])
+        kvprm_set_lora(self.ctx, rank, alpha / rank, lo)
 
     def close(self):
         if self.ctx:

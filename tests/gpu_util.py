@@ -26,8 +26,12 @@ def make_scorer(dev: ks.DeviceInputs, max_candidates: int, max_blocks: int):
           "w_minus": dev.top[ks.W_MINUS],
           "layers": [{"attn_norm": L[ks.ATTN_NORM], "w_qkv": L[ks.W_QKV], "w_o": L[ks.W_O], "mlp_norm": L[ks.MLP_NORM],
                       "w_gate_up": L[ks.W_GATE_UP], "w_down": L[ks.W_DOWN]} for L in dev.layers]}
-    return Scorer(a.n_layers, a.d_model, a.n_q_heads, a.n_kv_heads, a.head_dim, a.d_ff, wt, max_candidates, max_blocks,
-                  a.rope_base, a.rms_eps)
+    sc = Scorer(a.n_layers, a.d_model, a.n_q_heads, a.n_kv_heads, a.head_dim, a.d_ff, wt, max_candidates, max_blocks,
+                a.rope_base, a.rms_eps)
+    if a.lora_rank:   # the scorer adapter, kept apart from the weights
+        names = dict(zip(ks.LORA_KINDS, ("a_qkv", "b_qkv", "a_o", "b_o", "a_gate_up", "b_gate_up", "a_down", "b_down")))
+        sc.set_lora(a.lora_rank, a.lora_alpha, [{names[k]: L[k] for k in ks.LORA_KINDS} for L in dev.layers])
+    return sc
 
 
 def run_gpu(w: ks.Workload, tables: ks.Tables, debug: bool = True, dev=None, scorer=None, extra_flags: int = 0):

@@ -227,3 +227,52 @@ def test_host_side_errors():
         sc.score(dev.pool, w.block_table, np.array([20, -1], np.int32))
     assert e.value.code == 1
     assert kp.kvprm_score(sc.ctx, 0, 0, np.zeros((0, 1), np.int32), np.zeros(0, np.int32), 0).size == 0
+
+
+# ---------------------------------------------------------------- scorer adapter (kvprm_set_lora)
+def _lora_arch(arch, rank):
+    import dataclasses
+    return dataclasses.replace(arch, lora_rank=rank)
+
+
+@pytest.mark.parametrize("arch,rank,lens,sample", [
+    (ks.ARCH_TINY, 64, [0, 50, 129, 200], None),                                    # r = 64: half an A tile
+    (ks.Arch(2, 1536, 12, 2, 128, 8960), 256, [2048] * 16, None),                   # 1.5B layers, small image
+    (ks.Arch(2, 3584, 28, 4, 128, 18944), 256, [(37 * b) % 300 for b in range(64)],  # 7B layers, B = 64
+     [0, 1, 31, 63]),
+    (ks.Arch(2, 3584, 28, 4, 128, 18944), 128, [(53 * b) % 257 for b in range(200)],  # two m-tiles per gate/up CTA
+     [0, 100, 199]),
+])
+def test_lora(arch, rank, lens, sample):
+    """Every projection y = W x + (alpha / r) B (A x) with the factors kept apart (Sec. 4.1, App. B.1):
+    t = s A x on its own launch, then W x + B t as one K loop; against the oracle's fp64 adapter."""
+    t = ks.Tables.make(0.2)
+    w = ks.distinct("lora", _lora_arch(arch, rank), 61 + rank, lens, gain_std=0.2)
+    r, attn, dev, sc = run_gpu(w, t)
+    compare(w, t, cand_ids=sample, gpu_rewards=r, gpu_attn=attn, label=f"adapter r={rank} d={arch.d_model}")
+    sc.close()
+
+
+def test_lora_switch_and_errors():
+    """Rank 0 restores the merged scorer bit for bit; bad arguments leave the context as it was."""
+    import paper_2607_09153_gb300 as kp
+    t = ks.Tables.make(0.2)
+    w = ks.distinct("lora_sw", _lora_arch(ks.ARCH_TINY, 64), 71, [3, 40, 100], gain_std=0.2)
+    dev = ks.DeviceInputs(w, t)
+    sc = make_scorer(dev, 8, w.max_blocks)
+    with_lora = sc.score(dev.pool, w.block_table, w.seq_lens)
+    sc.set_lora(0)
+    merged = sc.score(dev.pool, w.block_table, w.seq_lens)
+    w0 = ks.distinct("lora_sw", ks.ARCH_TINY, 71, [3, 40, 100], gain_std=0.2)
+    fresh = make_scorer(ks.DeviceInputs(w0, t), 8, w0.max_blocks)
+    base = fresh.score(ks.DeviceInputs(w0, t).pool, w0.block_table, w0.seq_lens)
+    assert np.array_equal(merged, base)
+    assert np.abs(with_lora - merged).max() > 1e-5
+    for bad in (32, 100, 2048, -64):
+        with pytest.raises(kp.KvprmError):
+            kp.kvprm_set_lora(sc.ctx, bad, 0.5, None)
+    with pytest.raises(kp.KvprmError):
+        kp.kvprm_set_lora(sc.ctx, 64, 0.5, None)
+    assert np.array_equal(sc.score(dev.pool, w.block_table, w.seq_lens), merged)
+    fresh.close()
+    sc.close()
