@@ -48,15 +48,16 @@ class OracleCfg(ctypes.Structure):
     _fields_ = [("n_layers", ctypes.c_int), ("d_model", ctypes.c_int), ("n_q_heads", ctypes.c_int),
                 ("n_kv_heads", ctypes.c_int), ("head_dim", ctypes.c_int), ("d_ff", ctypes.c_int),
                 ("rope_base", ctypes.c_double), ("rms_eps", ctypes.c_double), ("mirror", ctypes.c_int),
-                ("nthreads", ctypes.c_int), ("lora_rank", ctypes.c_int), ("lora_scale", ctypes.c_double)]
+                ("nthreads", ctypes.c_int), ("lora_rank", ctypes.c_int), ("lora_scale", ctypes.c_double),
+                ("depth", ctypes.c_int)]
 
     @staticmethod
-    def from_arch(arch, mirror: bool = True, nthreads: int | None = None) -> "OracleCfg":
+    def from_arch(arch, mirror: bool = True, nthreads: int | None = None, depth: int = 1) -> "OracleCfg":
         rank = int(getattr(arch, "lora_rank", 0))
         return OracleCfg(arch.n_layers, arch.d_model, arch.n_q_heads, arch.n_kv_heads, arch.head_dim, arch.d_ff,
                          float(arch.rope_base), float(arch.rms_eps), int(mirror),
                          int(nthreads or max(1, os.cpu_count() or 1)), rank,
-                         float(arch.lora_alpha) / rank if rank else 0.0)
+                         float(arch.lora_alpha) / rank if rank else 0.0, int(depth))
 
 
 class DenseWeights(ctypes.Structure):
@@ -148,16 +149,17 @@ class Result:
 
 
 def _score(arch, wfn, wuser, kvfn, kvuser, cand_ids, lens, mirror, want_attn, want_hidden, nthreads, mutant,
-           want_layers=False):
+           want_layers=False, depth: int = 1):
     n = len(cand_ids)
+    rows = n * depth   # per-row outputs: candidate i's verify tokens are rows i depth .. i depth + depth - 1
     ids = np.ascontiguousarray(cand_ids, np.int32)
     lens = np.ascontiguousarray(lens, np.int64)
     p = np.empty(n)
-    attn = np.empty((arch.n_layers, n, arch.n_q_heads * arch.head_dim)) if want_attn else None
+    attn = np.empty((arch.n_layers, rows, arch.n_q_heads * arch.head_dim)) if want_attn else None
     hid = np.empty((n, arch.d_model)) if want_hidden else None
-    qkv = np.empty((arch.n_layers, n, arch.qkv_rows)) if want_layers else None
-    hl = np.empty((arch.n_layers, n, arch.d_model)) if want_layers else None
-    cfg = OracleCfg.from_arch(arch, mirror, nthreads)
+    qkv = np.empty((arch.n_layers, rows, arch.qkv_rows)) if want_layers else None
+    hl = np.empty((arch.n_layers, rows, arch.d_model)) if want_layers else None
+    cfg = OracleCfg.from_arch(arch, mirror, nthreads, depth)
     rc = lib(mutant).oracle_score(ctypes.byref(cfg), wfn, wuser, kvfn, kvuser, n,
                                   ids.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)),
                                   lens.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)), p.ctypes.data_as(_f64p),
@@ -171,18 +173,19 @@ def _score(arch, wfn, wuser, kvfn, kvuser, cand_ids, lens, mirror, want_attn, wa
 
 
 def score_synth(w, tables, cand_ids=None, mirror: bool = True, want_attn: bool = True, want_hidden: bool = False,
-                nthreads: int | None = None, mutant: int = 0, want_layers: bool = False) -> Result:
-    """Score candidates of a kvsynth workload; K/V come from their logical token identities."""
+                nthreads: int | None = None, mutant: int = 0, want_layers: bool = False, depth: int = 1) -> Result:
+    """Score candidates of a kvsynth workload; K/V come from their logical token identities.  depth > 1:
+    a depth-k readout (k verify tokens, causal among themselves; per-row outputs have len(ids) * k rows)."""
     import kvsynth
     prov = kvsynth.Providers(w, tables, nthreads)
     ids = list(range(w.n_candidates)) if cand_ids is None else list(cand_ids)
     lens = [len(w.cand_seg[i]) for i in ids]
     return _score(w.arch, prov.weight_fn, prov.user, prov.kv_fn, prov.user, ids, lens, mirror, want_attn, want_hidden,
-                  nthreads, mutant, want_layers)
+                  nthreads, mutant, want_layers, depth)
 
 
 def score_dense(arch, weights: dict, kv: list, mirror: bool = True, want_attn: bool = True, want_hidden: bool = False,
-                nthreads: int | None = None, mutant: int = 0) -> Result:
+                nthreads: int | None = None, mutant: int = 0, depth: int = 1) -> Result:
     """Score from explicit arrays.  weights = {'top': {kind: bits}, 'layers': [{kind: bits}]} (kinds 4..9, and
     the adapter factors 10..17 when arch.lora_rank > 0);
     kv[l][b] = (K_bits [L_b][nkv][hd], V_bits [L_b][nkv][hd])."""
@@ -220,4 +223,4 @@ def score_dense(arch, weights: dict, kv: list, mirror: bool = True, want_attn: b
     kvfn = ctypes.cast(L.oracle_dense_kv_provider, ctypes.c_void_p).value
     return _score(arch, wfn, ctypes.cast(ctypes.pointer(dw), ctypes.c_void_p).value, kvfn,
                   ctypes.cast(ctypes.pointer(dk), ctypes.c_void_p).value, list(range(n)), lens, mirror, want_attn,
-                  want_hidden, nthreads, mutant)
+                  want_hidden, nthreads, mutant, False, depth)

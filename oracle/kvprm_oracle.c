@@ -34,6 +34,12 @@
  *     h  += W_down (SiLU(W_gate x) * (W_up x))      W_gate_up rows: [gate | up]
  *   then x = RMSNorm(h) * g_final, z_+ = w_plus . x, z_- = w_minus . x.
  *
+ *   Depth-k readout (Sec. 3, definition of R_k; Sec. 5 "more verify tokens"): with
+ *   depth = k > 1, k verify tokens follow the trajectory at positions
+ *   L_b .. L_b + k - 1 and run causally among themselves: token t attends to the
+ *   cache and to tokens 0 .. t; the reward is read at the last one.  Internally
+ *   candidate b is k rows b k + t.
+ *
  *   Scorer adapter, Sec. 4.1 (f_{theta + Delta theta}, a LoRA adapter) and App.
  *   B.1 (rank r = 256, alpha = 32): when lora_rank > 0 each of the four
  *   projections y = W x above becomes y = W x + s B (A x) with its own factors
@@ -78,6 +84,7 @@ typedef struct {
     int nthreads;
     int lora_rank;       /* 0: no adapter */
     double lora_scale;   /* s in y = W x + s B (A x) */
+    int depth;           /* verify tokens per candidate (depth-k readout); 0 or 1: one */
 } oracle_cfg;
 
 /* ------------------------------------------------------------------ numbers */
@@ -153,34 +160,38 @@ void oracle_rope(double* x, int hd, double pos, double base) {
     }
 }
 
-/* Attention read-out of one query head (App. A.3), with the verify token's own
- * key/value as the last entry:
- *   s_j = q . K_j / sqrt(hd) for j < L,   s_L = q . k_self / sqrt(hd)
- *   w = softmax(s),  o = sum_j w_j V_j + w_L v_self.
- * K and V are bf16 rows with `stride` elements between consecutive tokens.
- * If `weights` is non-NULL it receives the L + 1 softmax weights. */
-void oracle_attend(const double* q, const uint16_t* K, const uint16_t* V, int64_t L, int64_t stride,
-                   const double* k_self, const double* v_self, int hd, double* o, double* weights) {
+/* Attention read-out of one query head (App. A.3) over the L cached entries and
+ * n_self verify-token entries (their own keys/values, the last one being the
+ * token's own; one entry except in a depth-k readout):
+ *   s_j = q . K_j / sqrt(hd) for j < L,   s_{L+t} = q . k_self[t] / sqrt(hd)
+ *   w = softmax(s),  o = sum_j w_j V_j + sum_t w_{L+t} v_self[t].
+ * K and V are bf16 rows with `stride` elements between consecutive tokens;
+ * self entry t starts at k_self + t * self_stride (likewise v_self).  If
+ * `weights` is non-NULL it receives the L + n_self softmax weights. */
+void oracle_attend_multi(const double* q, const uint16_t* K, const uint16_t* V, int64_t L, int64_t stride,
+                         const double* k_self, const double* v_self, int64_t self_stride, int n_self, int hd,
+                         double* o, double* weights) {
     double scale = 1.0 / sqrt((double)hd);
-    double* s = (double*)malloc(sizeof(double) * (size_t)(L + 1));
+    const int64_t N = L + n_self;
+    double* s = (double*)malloc(sizeof(double) * (size_t)N);
     for (int64_t j = 0; j < L; ++j) {
         double acc = 0.0;
         for (int d = 0; d < hd; ++d) acc += q[d] * bf16_to_f64(K[j * stride + d]);
         s[j] = acc * scale;
     }
-    {
+    for (int t = 0; t < n_self; ++t) {
         double acc = 0.0;
-        for (int d = 0; d < hd; ++d) acc += q[d] * k_self[d];
-        s[L] = acc * scale;
+        for (int d = 0; d < hd; ++d) acc += q[d] * k_self[t * self_stride + d];
+        s[L + t] = acc * scale;
     }
 #if ORACLE_MUTANT == 1 /* planted mistake: the verify token ignores itself */
-    if (L > 0) s[L] = -INFINITY;
+    if (L > 0) s[N - 1] = -INFINITY;
 #endif
     double m = s[0];
-    for (int64_t j = 1; j <= L; ++j)
+    for (int64_t j = 1; j < N; ++j)
         if (s[j] > m) m = s[j];
     double l = 0.0;
-    for (int64_t j = 0; j <= L; ++j) {
+    for (int64_t j = 0; j < N; ++j) {
         s[j] = exp(s[j] - m);
         l += s[j];
     }
@@ -189,13 +200,19 @@ void oracle_attend(const double* q, const uint16_t* K, const uint16_t* V, int64_
         double w = s[j] / l;
         for (int d = 0; d < hd; ++d) o[d] += w * bf16_to_f64(V[j * stride + d]);
     }
-    {
-        double w = s[L] / l;
-        for (int d = 0; d < hd; ++d) o[d] += w * v_self[d];
+    for (int t = 0; t < n_self; ++t) {
+        double w = s[L + t] / l;
+        for (int d = 0; d < hd; ++d) o[d] += w * v_self[t * self_stride + d];
     }
     if (weights)
-        for (int64_t j = 0; j <= L; ++j) weights[j] = s[j] / l;
+        for (int64_t j = 0; j < N; ++j) weights[j] = s[j] / l;
     free(s);
+}
+
+/* The single-verify-token read-out: the token's own key/value as the last entry. */
+void oracle_attend(const double* q, const uint16_t* K, const uint16_t* V, int64_t L, int64_t stride,
+                   const double* k_self, const double* v_self, int hd, double* o, double* weights) {
+    oracle_attend_multi(q, K, V, L, stride, k_self, v_self, 0, 1, hd, o, weights);
 }
 
 /* Reward head (Eq. score): P(+) = softmax([z_-, z_+]) at "+" = 1/(1+exp(z_- - z_+)). */
@@ -260,19 +277,21 @@ static void lora_add(const oracle_cfg* cfg, const uint16_t* A, const uint16_t* B
 /* ------------------------------------------------------------- attention */
 typedef struct {
     const oracle_cfg* cfg;
-    const double* q;        /* [n][nq][hd]   rotated (and rounded in mirror mode) */
-    const double* kself;    /* [n][nkv][hd] */
-    const double* vself;    /* [n][nkv][hd] */
+    const double* q;        /* [rows][nq][hd]   rotated (and rounded in mirror mode) */
+    const double* kself;    /* [rows][nkv][hd] */
+    const double* vself;    /* [rows][nkv][hd] */
     uint16_t* const* K;     /* per candidate [L][nkv][hd] */
     uint16_t* const* V;
-    const int64_t* lens;
-    double* o;              /* [n][nq][hd] */
+    const int64_t* lens;    /* per candidate */
+    int depth;              /* rows per candidate (verify tokens) */
+    double* o;              /* [rows][nq][hd] */
 } attn_ctx;
 static void attn_item(void* p, int64_t it) {
     const attn_ctx* c = (const attn_ctx*)p;
     const oracle_cfg* cfg = c->cfg;
     int nq = cfg->n_q_heads, nkv = cfg->n_kv_heads, hd = cfg->head_dim, G = nq / nkv;
-    int i = (int)(it / nq), h = (int)(it % nq);
+    int row = (int)(it / nq), h = (int)(it % nq);
+    int i = row / c->depth, t = row % c->depth;   /* candidate, verify token */
 #if ORACLE_MUTANT == 3 /* planted mistake: interleaved instead of contiguous head groups */
     int g = h % nkv;
 #elif ORACLE_MUTANT == 12 /* planted mistake: every query head reads kv head 0 */
@@ -281,22 +300,32 @@ static void attn_item(void* p, int64_t it) {
 #else
     int g = h / G;
 #endif
-    const double* q = c->q + ((int64_t)i * nq + h) * hd;
+    const double* q = c->q + ((int64_t)row * nq + h) * hd;
     double qs[1024];
 #if ORACLE_MUTANT == 4 /* planted mistake: scores not divided by sqrt(hd) */
     for (int d = 0; d < hd; ++d) qs[d] = q[d] * sqrt((double)hd);
 #else
     for (int d = 0; d < hd; ++d) qs[d] = q[d];
 #endif
-    oracle_attend(qs, c->K[i] + (int64_t)g * hd, c->V[i] + (int64_t)g * hd, c->lens[i], (int64_t)nkv * hd,
-                  c->kself + ((int64_t)i * nkv + g) * hd, c->vself + ((int64_t)i * nkv + g) * hd, hd,
-                  c->o + ((int64_t)i * nq + h) * hd, NULL);
+    /* token t sees the candidate's verify tokens 0 .. t (causal) */
+    const int64_t first = (int64_t)i * c->depth;
+#if ORACLE_MUTANT == 17 /* planted mistake: every verify token also sees the ones after it */
+    const int n_self = c->depth;
+    (void)t;
+#else
+    const int n_self = t + 1;
+#endif
+    oracle_attend_multi(qs, c->K[i] + (int64_t)g * hd, c->V[i] + (int64_t)g * hd, c->lens[i], (int64_t)nkv * hd,
+                        c->kself + (first * nkv + g) * hd, c->vself + (first * nkv + g) * hd, (int64_t)nkv * hd,
+                        n_self, hd, c->o + ((int64_t)row * nq + h) * hd, NULL);
 }
 
 /* ------------------------------------------------------------------ scorer */
 /*
  * Score n candidates.  cand_ids[i] is passed to the kv provider; lens[i] is its
- * cached length L.  Outputs: p_plus[n]; if non-NULL, attn_out[N_L][n][nq*hd]
+ * cached length L.  With depth D > 1 the per-row outputs below have n D rows
+ * (candidate i's tokens are rows i D .. i D + D - 1) and h_out is each
+ * candidate's last row.  Outputs: p_plus[n]; if non-NULL, attn_out[N_L][n][nq*hd]
  * (each layer's attention output o before rounding), h_out[n][d] (final
  * residual stream), qkv_out[N_L][n][(nq+2nkv)*hd] (each layer's rotated q,
  * self k and self v as the attention consumes them) and
@@ -310,14 +339,17 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
     const int ff = cfg->d_ff, qkv_rows = (nq + 2 * nkv) * hd;
     if (hd > 1024 || hd % 2 || nq % nkv) return -1;
     int rc = 0;
+    /* rows: candidate i's verify tokens are rows i D .. i D + D - 1 (one row each without depth-k) */
+    const int D = cfg->depth > 1 ? cfg->depth : 1;
+    const int nr = n * D;
     uint16_t *embed = malloc(2 * (size_t)d), *gfin = malloc(2 * (size_t)d), *wp = malloc(2 * (size_t)d),
              *wm = malloc(2 * (size_t)d), *gattn = malloc(2 * (size_t)d), *gmlp = malloc(2 * (size_t)d);
     uint16_t *Wqkv = malloc(2 * (size_t)qkv_rows * d), *Wo = malloc(2 * (size_t)d * nq * hd),
              *Wgu = malloc(2 * (size_t)2 * ff * d), *Wd = malloc(2 * (size_t)d * ff);
-    double *h = calloc((size_t)n * d, 8), *x = calloc((size_t)n * d, 8), *qkv = calloc((size_t)n * qkv_rows, 8);
-    double *q = calloc((size_t)n * nq * hd, 8), *ks = calloc((size_t)n * nkv * hd, 8),
-           *vs = calloc((size_t)n * nkv * hd, 8), *o = calloc((size_t)n * nq * hd, 8);
-    double *gu = calloc((size_t)n * 2 * ff, 8), *a = calloc((size_t)n * ff, 8);
+    double *h = calloc((size_t)nr * d, 8), *x = calloc((size_t)nr * d, 8), *qkv = calloc((size_t)nr * qkv_rows, 8);
+    double *q = calloc((size_t)nr * nq * hd, 8), *ks = calloc((size_t)nr * nkv * hd, 8),
+           *vs = calloc((size_t)nr * nkv * hd, 8), *o = calloc((size_t)nr * nq * hd, 8);
+    double *gu = calloc((size_t)nr * 2 * ff, 8), *a = calloc((size_t)nr * ff, 8);
     uint16_t** K = calloc((size_t)n, sizeof(uint16_t*));
     uint16_t** V = calloc((size_t)n, sizeof(uint16_t*));
     /* adapter factors of the four projections (A [r][in], B [out][r]) and scratch */
@@ -335,8 +367,8 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
             LB[j] = malloc(2 * (size_t)out_of[j] * r);
             if (!LA[j] || !LB[j]) { rc = -2; goto done; }
         }
-        lt = calloc((size_t)n * r, 8);
-        ltmp = calloc((size_t)n * most, 8);
+        lt = calloc((size_t)nr * r, 8);
+        ltmp = calloc((size_t)nr * most, 8);
         if (!lt || !ltmp) { rc = -2; goto done; }
     }
     if (!embed || !gfin || !wp || !wm || !gattn || !gmlp || !Wqkv || !Wo || !Wgu || !Wd || !h || !x || !qkv || !q ||
@@ -353,8 +385,8 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
     if (wfn(wuser, K_EMBED, 0, embed, d) || wfn(wuser, K_FINAL_NORM, 0, gfin, d) || wfn(wuser, K_W_PLUS, 0, wp, d) ||
         wfn(wuser, K_W_MINUS, 0, wm, d)) { rc = -3; goto done; }
 
-    /* the verify token's embedding starts every candidate's residual stream */
-    for (int i = 0; i < n; ++i)
+    /* the verify token's embedding starts every row's residual stream */
+    for (int i = 0; i < nr; ++i)
         for (int c = 0; c < d; ++c) h[(int64_t)i * d + c] = bf16_to_f64(embed[c]);
 
     for (int l = 0; l < NL; ++l) {
@@ -374,7 +406,7 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
             if (lens[i] > 0 && kvfn(kvuser, l, cand_ids[i], K[i], V[i], lens[i])) { rc = -4; goto done; }
 
         /* attention block */
-        for (int i = 0; i < n; ++i) {
+        for (int i = 0; i < nr; ++i) {
             double* xi = x + (int64_t)i * d;
 #if ORACLE_MUTANT == 9 /* planted mistake: eps left out of the norm */
             oracle_rmsnorm(h + (int64_t)i * d, gattn, d, 0.0, xi);
@@ -383,18 +415,19 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
 #endif
             for (int c = 0; c < d; ++c) xi[c] = rnd(cfg, xi[c]);
         }
-        project(cfg, Wqkv, qkv_rows, d, x, qkv, n, 0, 0);
-        if (r > 0) lora_add(cfg, LA[0], LB[0], qkv_rows, d, x, qkv, n, lt, ltmp);
-        for (int i = 0; i < n; ++i) {
-            const double* r = qkv + (int64_t)i * qkv_rows;
+        project(cfg, Wqkv, qkv_rows, d, x, qkv, nr, 0, 0);
+        if (r > 0) lora_add(cfg, LA[0], LB[0], qkv_rows, d, x, qkv, nr, lt, ltmp);
+        for (int i = 0; i < nr; ++i) {
+            const double* qr = qkv + (int64_t)i * qkv_rows;
+            /* verify token t of candidate i / D sits at position L + t */
 #if ORACLE_MUTANT == 8 /* planted mistake: verify token placed on the last cached position */
-            double pos = (double)lens[i] - 1.0;
+            double pos = (double)lens[i / D] - 1.0 + (double)(i % D);
 #else
-            double pos = (double)lens[i];
+            double pos = (double)lens[i / D] + (double)(i % D);
 #endif
             for (int hh = 0; hh < nq; ++hh) {
                 double* qh = q + ((int64_t)i * nq + hh) * hd;
-                memcpy(qh, r + (int64_t)hh * hd, 8 * (size_t)hd);
+                memcpy(qh, qr + (int64_t)hh * hd, 8 * (size_t)hd);
 #if ORACLE_MUTANT == 2 /* planted mistake: rotation in the wrong direction */
                 oracle_rope(qh, hd, -pos, cfg->rope_base);
 #else
@@ -405,8 +438,8 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
             for (int g = 0; g < nkv; ++g) {
                 double* kh = ks + ((int64_t)i * nkv + g) * hd;
                 double* vh = vs + ((int64_t)i * nkv + g) * hd;
-                memcpy(kh, r + (int64_t)(nq + g) * hd, 8 * (size_t)hd);
-                memcpy(vh, r + (int64_t)(nq + nkv + g) * hd, 8 * (size_t)hd);
+                memcpy(kh, qr + (int64_t)(nq + g) * hd, 8 * (size_t)hd);
+                memcpy(vh, qr + (int64_t)(nq + nkv + g) * hd, 8 * (size_t)hd);
                 oracle_rope(kh, hd, pos, cfg->rope_base);
                 for (int c = 0; c < hd; ++c) {
                     kh[c] = rnd(cfg, kh[c]);
@@ -415,32 +448,32 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
             }
         }
         if (qkv_out)
-            for (int i = 0; i < n; ++i) {
-                double* dst = qkv_out + ((int64_t)l * n + i) * qkv_rows;
+            for (int i = 0; i < nr; ++i) {
+                double* dst = qkv_out + ((int64_t)l * nr + i) * qkv_rows;
                 memcpy(dst, q + (int64_t)i * nq * hd, 8 * (size_t)nq * hd);
                 memcpy(dst + (int64_t)nq * hd, ks + (int64_t)i * nkv * hd, 8 * (size_t)nkv * hd);
                 memcpy(dst + (int64_t)(nq + nkv) * hd, vs + (int64_t)i * nkv * hd, 8 * (size_t)nkv * hd);
             }
-        attn_ctx ac = { cfg, q, ks, vs, K, V, lens, o };
-        par_for((int64_t)n * nq, cfg->nthreads, attn_item, &ac);
-        if (attn_out) memcpy(attn_out + (int64_t)l * n * nq * hd, o, 8 * (size_t)n * nq * hd);
-        for (int64_t e = 0; e < (int64_t)n * nq * hd; ++e) o[e] = rnd(cfg, o[e]);
+        attn_ctx ac = { cfg, q, ks, vs, K, V, lens, D, o };
+        par_for((int64_t)nr * nq, cfg->nthreads, attn_item, &ac);
+        if (attn_out) memcpy(attn_out + (int64_t)l * nr * nq * hd, o, 8 * (size_t)nr * nq * hd);
+        for (int64_t e = 0; e < (int64_t)nr * nq * hd; ++e) o[e] = rnd(cfg, o[e]);
 #if ORACLE_MUTANT == 5 /* planted mistake: output projection applied transposed */
-        project(cfg, Wo, d, nq * hd, o, h, n, 1, 1);
+        project(cfg, Wo, d, nq * hd, o, h, nr, 1, 1);
 #else
-        project(cfg, Wo, d, nq * hd, o, h, n, 1, 0);
+        project(cfg, Wo, d, nq * hd, o, h, nr, 1, 0);
 #endif
-        if (r > 0) lora_add(cfg, LA[1], LB[1], d, nq * hd, o, h, n, lt, ltmp);
+        if (r > 0) lora_add(cfg, LA[1], LB[1], d, nq * hd, o, h, nr, lt, ltmp);
 
         /* feed-forward block */
-        for (int i = 0; i < n; ++i) {
+        for (int i = 0; i < nr; ++i) {
             double* xi = x + (int64_t)i * d;
             oracle_rmsnorm(h + (int64_t)i * d, gmlp, d, cfg->rms_eps, xi);
             for (int c = 0; c < d; ++c) xi[c] = rnd(cfg, xi[c]);
         }
-        project(cfg, Wgu, 2 * ff, d, x, gu, n, 0, 0);
-        if (r > 0) lora_add(cfg, LA[2], LB[2], 2 * ff, d, x, gu, n, lt, ltmp);
-        for (int i = 0; i < n; ++i)
+        project(cfg, Wgu, 2 * ff, d, x, gu, nr, 0, 0);
+        if (r > 0) lora_add(cfg, LA[2], LB[2], 2 * ff, d, x, gu, nr, lt, ltmp);
+        for (int i = 0; i < nr; ++i)
             for (int j = 0; j < ff; ++j) {
                 double gt = gu[(int64_t)i * 2 * ff + j], up = gu[(int64_t)i * 2 * ff + ff + j];
 #if ORACLE_MUTANT == 10 /* planted mistake: gate not passed through SiLU */
@@ -453,22 +486,23 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
                 a[(int64_t)i * ff + j] = rnd(cfg, act);
             }
 #if ORACLE_MUTANT == 6 /* planted mistake: feed-forward output replaces the residual stream */
-        project(cfg, Wd, d, ff, a, h, n, 0, 0);
+        project(cfg, Wd, d, ff, a, h, nr, 0, 0);
 #else
-        project(cfg, Wd, d, ff, a, h, n, 1, 0);
+        project(cfg, Wd, d, ff, a, h, nr, 1, 0);
 #endif
-        if (r > 0) lora_add(cfg, LA[3], LB[3], d, ff, a, h, n, lt, ltmp);
-        if (h_layers_out) memcpy(h_layers_out + (int64_t)l * n * d, h, 8 * (size_t)n * d);
+        if (r > 0) lora_add(cfg, LA[3], LB[3], d, ff, a, h, nr, lt, ltmp);
+        if (h_layers_out) memcpy(h_layers_out + (int64_t)l * nr * d, h, 8 * (size_t)nr * d);
     }
 
-    /* reward head on the final-normed stream */
+    /* reward head on the final-normed stream of each candidate's last verify token */
     for (int i = 0; i < n; ++i) {
-        double* xi = x + (int64_t)i * d;
-        oracle_rmsnorm(h + (int64_t)i * d, gfin, d, cfg->rms_eps, xi);
+        const int64_t row = (int64_t)i * D + D - 1;
+        double* xi = x + row * d;
+        oracle_rmsnorm(h + row * d, gfin, d, cfg->rms_eps, xi);
         for (int c = 0; c < d; ++c) xi[c] = rnd(cfg, xi[c]);
         p_plus[i] = oracle_reward(xi, wp, wm, d);
+        if (h_out) memcpy(h_out + (int64_t)i * d, h + row * d, 8 * (size_t)d);
     }
-    if (h_out) memcpy(h_out, h, 8 * (size_t)n * d);
 
 done:
     if (K)

@@ -52,17 +52,19 @@ def _rotate_half(x: torch.Tensor) -> torch.Tensor:
     return torch.cat([-x[..., h:], x[..., :h]], dim=-1)
 
 
-def reencode(arch, weights: dict, xs: np.ndarray, mirror: bool = True):
-    """Causal forward over [xs; e_v].  xs: [L, d] float64 hidden inputs of the trajectory.
+def reencode(arch, weights: dict, xs: np.ndarray, mirror: bool = True, depth: int = 1):
+    """Causal forward over [xs; e_v x depth] (depth verify tokens, the depth-k readout).  xs: [L, d]
+    float64 hidden inputs of the trajectory.
 
-    Returns (p_plus, attn_last [N_L, nq*hd], cache) where cache[l] = (K_bits, V_bits),
-    each [L, nkv, hd] uint16 (post-RoPE keys)."""
+    Returns (p_plus of the last position, attn, cache): attn [N_L, nq*hd] at the last position for
+    depth 1, else [N_L, depth, nq*hd] at the verify positions; cache[l] = (K_bits, V_bits), each
+    [L, nkv, hd] uint16 (post-RoPE keys)."""
     d, nq, nkv, hd, ff = arch.d_model, arch.n_q_heads, arch.n_kv_heads, arch.head_dim, arch.d_ff
     L = xs.shape[0]
-    T = L + 1
+    T = L + depth
     top = weights["top"]
     e_v = _bits_to_f64(top[0])
-    h = torch.cat([torch.as_tensor(xs, dtype=torch.float64).reshape(L, d), e_v[None, :]], dim=0)
+    h = torch.cat([torch.as_tensor(xs, dtype=torch.float64).reshape(L, d), e_v[None, :].expand(depth, d)], dim=0)
     cos, sin = _rope_tables(T, hd, arch.rope_base)
     rb = round_bf16 if mirror else (lambda t: t)
     cache, attn_last = [], []
@@ -90,13 +92,13 @@ def reencode(arch, weights: dict, xs: np.ndarray, mirror: bool = True):
         o = F.scaled_dot_product_attention(q.transpose(0, 1)[None], k.transpose(0, 1)[None],
                                            v.transpose(0, 1)[None], is_causal=True, enable_gqa=True)
         o = o[0].transpose(0, 1).reshape(T, nq * hd)
-        attn_last.append(o[L].clone())
+        attn_last.append(o[L].clone() if depth == 1 else o[L:].clone())
         h = h + rb(o) @ W_o.T
         x = rb(F.rms_norm(h, (d,), weight=g_mlp, eps=arch.rms_eps))
         gu = x @ W_gu.T
         a = rb(F.silu(gu[:, :ff]) * gu[:, ff:])
         h = h + a @ W_d.T
-    x = rb(F.rms_norm(h[L:L + 1], (d,), weight=_bits_to_f64(top[1]), eps=arch.rms_eps))[0]
+    x = rb(F.rms_norm(h[T - 1:T], (d,), weight=_bits_to_f64(top[1]), eps=arch.rms_eps))[0]
     z = torch.stack([x @ _bits_to_f64(top[3]), x @ _bits_to_f64(top[2])])     # [z_-, z_+]
     p_plus = torch.softmax(z, dim=0)[1].item()
     return p_plus, torch.stack(attn_last).numpy(), cache

@@ -174,4 +174,21 @@ def pin_lora_merged(m=0):
     assert np.abs(rb.p_plus - rm.p_plus).max() > 1e-6
 
 
-ALL_PINS = [pin_bf16_round, pin_rmsnorm, pin_rope, pin_attend, pin_reward, pin_reencode, pin_lora_merged]
+def pin_depth_reencode(m=0, depth=3, lens=(0, 5, 17)):
+    """Depth-k readout (Sec. 3 R_k; Sec. 5, k > 1 verify tokens) == the last k positions of a full causal
+    forward over [x; v, .., v]: verify token t sits at position L + t and sees the cache and tokens 0..t."""
+    arch = ks.ARCH_TINY
+    t = ks.Tables.make(0.2)
+    W = ks.host_weights(arch, 79, t)
+    for mirror in (True, False):
+        for L in lens:
+            xs = np.random.default_rng(2000 + L).normal(0, 1, (L, arch.d_model))
+            p, attn, cache = reencode(arch, W, xs, mirror, depth=depth)
+            r = oracle.score_dense(arch, W, [[cache[l]] for l in range(arch.n_layers)], mirror=mirror, mutant=m,
+                                   depth=depth)
+            assert abs(p - r.p_plus[0]) < 1e-12, (L, mirror, p, r.p_plus[0])
+            np.testing.assert_allclose(r.attn, attn, rtol=1e-9, atol=1e-12)
+
+
+ALL_PINS = [pin_bf16_round, pin_rmsnorm, pin_rope, pin_attend, pin_reward, pin_reencode, pin_lora_merged,
+            pin_depth_reencode]

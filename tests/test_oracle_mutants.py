@@ -19,6 +19,7 @@ MUTANTS = {
     14: "gate and up exchanged",
     15: "adapter scale left out",
     16: "adapter term subtracted",
+    17: "a verify token of a depth-k readout also sees the tokens after it",
 }
 
 

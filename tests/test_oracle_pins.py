@@ -28,6 +28,11 @@ def test_reward():
     P.pin_reward()
 
 
+@pytest.mark.parametrize("depth", [2, 4])
+def test_depth_readout_reencode(depth):
+    P.pin_depth_reencode(depth=depth)
+
+
 def test_lora_equals_merged():
     P.pin_lora_merged()
 
