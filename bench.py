@@ -189,7 +189,7 @@ def ncu_traffic(kernel: str, workload: str):
 
 
 # ---------------------------------------------------------------- CPU oracle
-def cpu_oracle_time(w, tables, budget_s: float = 12.0, max_cands: int | None = None):
+def cpu_oracle_time(w, tables, budget_s: float = 12.0, max_cands: int | None = None, depth: int = 1):
     """Time the oracle (exact mode) on a bounded sample of the workload's candidates."""
     import kvsynth as ks
     import oracle
@@ -203,7 +203,7 @@ def cpu_oracle_time(w, tables, budget_s: float = 12.0, max_cands: int | None = N
     def run(ids):
         kv = [[ks.host_kv_logical(w, l, b, tables) for b in ids] for l in range(a.n_layers)]
         t = time.perf_counter()
-        oracle.score_dense(a, W, kv, mirror=False, want_attn=False, nthreads=nthreads)
+        oracle.score_dense(a, W, kv, mirror=False, want_attn=False, nthreads=nthreads, depth=depth)
         return time.perf_counter() - t
 
     t1 = run([0])
@@ -228,7 +228,7 @@ def run_reference(args, world, rank):
     samples = []
     budget = max(5.0, 60.0 / max(1, args.steps + args.warmup))
     for i in range(args.warmup + args.steps):
-        r = cpu_oracle_time(w, t, budget_s=budget, max_cands=4)
+        r = cpu_oracle_time(w, t, budget_s=budget, max_cands=4, depth=args.depth)
         if i >= args.warmup:
             samples.append(r)
     val = float(np.mean([s["value"] for s in samples]))
@@ -261,7 +261,8 @@ def workload_config(w, args) -> dict:
             "unique_pages": int(len(set(np.concatenate([w.block_table[b, :(int(w.seq_lens[b]) + 15) // 16]
                                                         for b in range(w.n_candidates)]).tolist()))),
             "l2": "inputs exceed L2 (weights + cache >> 129 MB); no flush", "parallelism": f"replicas{args.gpus}",
-            **({"lora_rank": a.lora_rank, "lora_alpha": a.lora_alpha} if a.lora_rank else {})}
+            **({"lora_rank": a.lora_rank, "lora_alpha": a.lora_alpha} if a.lora_rank else {}),
+            **({"readout_depth": args.depth} if args.depth > 1 else {})}
 
 
 # ---------------------------------------------------------------- GPU arm
@@ -293,7 +294,9 @@ def run_gpu(args, world, rank, local):
     dev = ks.DeviceInputs(w, tables)
     a = w.arch
     B = w.n_candidates
-    sc = make_scorer(dev, B, w.max_blocks)
+    sc = make_scorer(dev, B * args.depth, w.max_blocks)
+    if args.depth > 1:   # depth-k readout: k verify tokens per candidate, rows of the same batch
+        sc.set_depth(args.depth)
     stream = torch.cuda.Stream()
     sp = stream.cuda_stream
     d_rewards = torch.empty(B, dtype=torch.float32, device="cuda")
@@ -414,7 +417,7 @@ def run_gpu(args, world, rank, local):
     }
     sc.close()
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_oracle_time(w, tables, budget_s=args.cpu_budget)
+        line["cpu_baseline"] = cpu_oracle_time(w, tables, budget_s=args.cpu_budget, depth=args.depth)
     if rank == 0:
         print(json.dumps(line), flush=True)
 
@@ -500,6 +503,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="qwen1p5b_b16_l2048", choices=list(ks.WORKLOAD_NAMES))
+    ap.add_argument("--depth", type=int, default=1,
+                    help="verify tokens per candidate (depth-k readout; 1, the default: one)")
     ap.add_argument("--lora", type=int, default=0,
                     help="scorer adapter rank kept apart from the weights (0: merged weights, the default)")
     ap.add_argument("--profile-steps", type=int, default=50)

@@ -116,6 +116,20 @@ KVPRM_API int kvprm_create(const kvprm_config* cfg, const kvprm_weights* weights
  * KVPRM_NO_GRAPH=1 and KVPRM_NO_PDL=1 switch off graph capture and programmatic
  * dependent launch (for debugging). */
 
+/* Depth-k readout (Sec. 3, Definition "Depth-k Readout": k query vectors
+ * against the cache; Sec. 5, "more verify tokens"): every scoring call then
+ * appends k verify tokens to each candidate, at positions L_b .. L_b + k - 1,
+ * run causally among themselves (token t attends to the cache and to tokens
+ * 0 .. t), and reads P(+) at the last one.  Candidate b becomes k rows of the
+ * batch that share its pages (each page is still read once per candidate), so
+ * n_candidates * k <= max_candidates.  Debug captures (kvprm_debug_attn_out,
+ * ...) then hold n_candidates * k rows, candidate b's tokens at rows b k + t.
+ * kvprm_attention is not affected.
+ *  depth  1 .. 8 (1, the default: one verify token).
+ * Errors: KVPRM_EINVAL (depth out of range; nothing changes).  Takes effect for
+ * the next scoring call. */
+KVPRM_API int kvprm_set_readout_depth(kvprm_ctx* ctx, int32_t depth);
+
 /* Scorer adapter kept apart from the base weights (Sec. 4.1: the scorer is
  * f_{theta + Delta theta}, the base model with a LoRA adapter; App. B.1: rank
  * r = 256, alpha = 32): every projection y = W x of every layer becomes

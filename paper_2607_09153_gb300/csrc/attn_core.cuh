@@ -306,13 +306,16 @@ __device__ __forceinline__ void merge_warp_states(int group, const float* mo, co
   }
 }
 
-// Combine of one (candidate b, kv head g): W warps (8 or 4; threads tid < 32 W)
+// Combine of one (candidate row b, kv head g): W warps (8 or 4; threads tid < 32 W)
 // fold its partial slots [first, first + ns), U at a time per warp with every
 // load of a round issued before the first use, into a running (M, L, O) per
 // query head of the group; the warps' states and the verify token's own entry
 // (s_self = q . k_self, value v_self) are then merged through shared memory:
 //   M* = max(s_self, M_w), o = (2^(s_self - M*) v_self + sum_w 2^(M_w - M*) O_w)
-//                              / (2^(s_self - M*) + sum_w 2^(M_w - M*) L_w),
+//                              / (2^(s_self - M*) + sum_w 2^(M_w - M*) L_w).
+// In a depth-k readout (mg.depth > 1) row b is verify token t = b % depth and the
+// self entries are its candidate's tokens 0 .. t (rows b - t .. b), each a term
+// 2^(s_j - M*) v_j of the same sums;
 // written as a bf16 (hi, lo) pair (and optional fp32 copies).  `smem` holds
 // CombineShape::kBytes; sync() is a barrier over exactly the 32 W threads.  A
 // caller running several groups back to back syncs between them.
@@ -323,8 +326,8 @@ struct CombineShape {
   static constexpr size_t kAcc = 0;                                         // [W][ROWS][HD]
   static constexpr size_t kM = kAcc + sizeof(float) * W * ROWS * HD;        // [W][ROWS]
   static constexpr size_t kL = kM + sizeof(float) * W * ROWS;               // [W][ROWS]
-  static constexpr size_t kSelf = kL + sizeof(float) * W * ROWS;            // [ROWS]
-  static constexpr size_t kBytes = kSelf + sizeof(float) * ROWS;
+  static constexpr size_t kSelf = kL + sizeof(float) * W * ROWS;            // [ROWS][kMaxReadoutDepth]
+  static constexpr size_t kBytes = kSelf + sizeof(float) * ROWS * kMaxReadoutDepth;
 };
 
 template <int HD, int ROWS, int W_ = 8, typename Sync>
@@ -370,22 +373,32 @@ __device__ __forceinline__ void combine_group(int tid, int b, int g, int first, 
     const int idx = tid + i * W * 32;
     vsf[i] = idx < group * HD ? __ldcg(mg.vself + hk * HD + idx % HD) : 0.f;
   }
-  // the verify token's own score of head `warp`
+  // the self entries' scores of head `warp`: token t's own (k_self already loaded) and, in a
+  // depth-k readout, its candidate's earlier tokens (rows b - t .. b - 1)
+  const int t_self = b % mg.depth, n_self = t_self + 1;
+  const int64_t hk0 = hk - static_cast<int64_t>(t_self) * n_kv;
   if (warp < group) {
-    float dot = 0.f;
+    for (int e = 0; e < n_self; ++e) {
+      float dot = 0.f;
 #pragma unroll
-    for (int j = 0; j < kPer; ++j) dot += qd[j] * kd[j];
+      for (int j = 0; j < kPer; ++j)
+        dot += qd[j] * (e == t_self ? kd[j] : __ldcg(mg.kself + (hk0 + e * n_kv) * HD + lane + 32 * j));
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
-    if (lane == 0) s_self[warp] = dot * (kLog2e * rsqrtf(static_cast<float>(HD)));
+      for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
+      if (lane == 0) s_self[warp * kMaxReadoutDepth + e] = dot * (kLog2e * rsqrtf(static_cast<float>(HD)));
+    }
   }
   for (int r = warp + W; r < group; r += W) {   // heads beyond the warp count (G > W; k_self is loaded by all)
-    float dot = 0.f;
+    for (int e = 0; e < n_self; ++e) {
+      float dot = 0.f;
 #pragma unroll
-    for (int j = 0; j < kPer; ++j) dot += __ldcg(mg.q + (hq0 + r) * HD + lane + 32 * j) * kd[j];
+      for (int j = 0; j < kPer; ++j)
+        dot += __ldcg(mg.q + (hq0 + r) * HD + lane + 32 * j) *
+               (e == t_self ? kd[j] : __ldcg(mg.kself + (hk0 + e * n_kv) * HD + lane + 32 * j));
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
-    if (lane == 0) s_self[r] = dot * (kLog2e * rsqrtf(static_cast<float>(HD)));
+      for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
+      if (lane == 0) s_self[r * kMaxReadoutDepth + e] = dot * (kLog2e * rsqrtf(static_cast<float>(HD)));
+    }
   }
   float M[ROWS], L[ROWS], acc[ROWS][kPer];
 #pragma unroll
@@ -441,12 +454,17 @@ __device__ __forceinline__ void combine_group(int tid, int b, int g, int first, 
     const int idx = tid + i * W * 32;
     if (idx >= group * HD) break;
     const int r = idx / HD, d = idx - r * HD;
-    const float ss = s_self[r];
-    float Mt = ss;
+    const float* ss = s_self + r * kMaxReadoutDepth;
+    float Mt = ss[0];
+    for (int e = 1; e < n_self; ++e) Mt = fmaxf(Mt, ss[e]);
 #pragma unroll
     for (int w = 0; w < W; ++w) Mt = fmaxf(Mt, s_m[w * ROWS + r]);
-    const float ws = exp2f(ss - Mt);
-    float num = ws * vsf[i], den = ws;
+    float num = 0.f, den = 0.f;
+    for (int e = 0; e < n_self; ++e) {   // the self entries (one without a depth-k readout)
+      const float ws = exp2f(ss[e] - Mt);
+      num += ws * (e == t_self ? vsf[i] : __ldcg(mg.vself + (hk0 + e * n_kv) * HD + d));
+      den += ws;
+    }
 #pragma unroll
     for (int w = 0; w < W; ++w) {
       const float mw = s_m[w * ROWS + r];

@@ -53,14 +53,15 @@ __device__ __forceinline__ float row_rscale(const float* __restrict__ sumsq, int
   return *slot;
 }
 
-__global__ void rope_table_kernel(const int32_t* __restrict__ seq_lens, int hd, double base, float2* __restrict__ tab,
-                                  unsigned long long* ts) {
+__global__ void rope_table_kernel(const int32_t* __restrict__ seq_lens, int hd, double base, int depth,
+                                  float2* __restrict__ tab, unsigned long long* ts) {
   trace_begin(ts);
   grid_dep_launch();
   grid_dep_wait();
   const int b = blockIdx.x, i = threadIdx.x;
   if (i < hd / 2) {
-    const double ang = static_cast<double>(seq_lens[b]) * pow(base, -2.0 * i / hd);
+    // row b is verify token b % depth of its candidate: position L + b % depth
+    const double ang = static_cast<double>(seq_lens[b] + b % depth) * pow(base, -2.0 * i / hd);
     tab[b * (hd / 2) + i] = make_float2(static_cast<float>(cos(ang)), static_cast<float>(sin(ang)));
   }
   trace_end(ts);
@@ -94,8 +95,10 @@ __global__ void embed_norm_kernel(const __nv_bfloat16* __restrict__ e_v, const _
   trace_end(ts);
 }
 
-__global__ void head_kernel(const float* __restrict__ h, const float* __restrict__ sumsq, int m_tiles, int n_cand,
-                            int d, float eps, const __nv_bfloat16* __restrict__ gain,
+// One CTA per candidate: the reward of its last row (its last verify token; one row per candidate
+// except in a depth-k readout).
+__global__ void head_kernel(const float* __restrict__ h, const float* __restrict__ sumsq, int m_tiles, int n_rows,
+                            int depth, int d, float eps, const __nv_bfloat16* __restrict__ gain,
                             const __nv_bfloat16* __restrict__ w_plus, const __nv_bfloat16* __restrict__ w_minus,
                             float* __restrict__ rewards, unsigned long long* ts) {
   trace_begin(ts);
@@ -103,11 +106,11 @@ __global__ void head_kernel(const float* __restrict__ h, const float* __restrict
   __shared__ float slot;
   grid_dep_launch();
   grid_dep_wait();
-  const int b = blockIdx.x;
-  const float r = row_rscale(sumsq, m_tiles, n_cand, b, d, eps, &slot);
+  const int b = blockIdx.x, row = b * depth + depth - 1;
+  const float r = row_rscale(sumsq, m_tiles, n_rows, row, d, eps, &slot);
   float zp = 0.f, zm = 0.f;
   for (int c = threadIdx.x; c < d; c += blockDim.x) {
-    const float xf = h[static_cast<int64_t>(b) * d + c] * r * __bfloat162float(gain[c]);
+    const float xf = h[static_cast<int64_t>(row) * d + c] * r * __bfloat162float(gain[c]);
     zp += xf * __bfloat162float(w_plus[c]);
     zm += xf * __bfloat162float(w_minus[c]);
   }
@@ -138,11 +141,11 @@ cudaLaunchConfig_t make_cfg(dim3 grid, dim3 block, cudaStream_t st, cudaLaunchAt
 
 }  // namespace
 
-cudaError_t launch_rope_table(const int32_t* seq_lens, int n_cand, int hd, double base, float2* table,
+cudaError_t launch_rope_table(const int32_t* seq_lens, int n_rows, int hd, double base, int depth, float2* table,
                               cudaStream_t stream, bool pdl, unsigned long long* ts) {
   cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = make_cfg(dim3(n_cand), dim3(64), stream, attr, pdl);
-  return cudaLaunchKernelEx(&cfg, rope_table_kernel, seq_lens, hd, base, table, ts);
+  cudaLaunchConfig_t cfg = make_cfg(dim3(n_rows), dim3(64), stream, attr, pdl);
+  return cudaLaunchKernelEx(&cfg, rope_table_kernel, seq_lens, hd, base, depth, table, ts);
 }
 
 cudaError_t launch_embed_norm(const ModelDims& m, const __nv_bfloat16* e_v, const __nv_bfloat16* gain, int n_cand,
@@ -153,12 +156,12 @@ cudaError_t launch_embed_norm(const ModelDims& m, const __nv_bfloat16* e_v, cons
   return cudaLaunchKernelEx(&cfg, embed_norm_kernel, e_v, gain, m.d, n_cand, h, sumsq, x, ts);
 }
 
-cudaError_t launch_head(const ModelDims& m, const float* h, const float* sumsq, int m_tiles, int n_cand,
+cudaError_t launch_head(const ModelDims& m, const float* h, const float* sumsq, int m_tiles, int n_rows, int depth,
                         const __nv_bfloat16* gain, const __nv_bfloat16* w_plus, const __nv_bfloat16* w_minus,
                         float* rewards, cudaStream_t stream, bool pdl, unsigned long long* ts) {
   cudaLaunchAttribute attr[1];
-  cudaLaunchConfig_t cfg = make_cfg(dim3(n_cand), dim3(256), stream, attr, pdl);
-  return cudaLaunchKernelEx(&cfg, head_kernel, h, sumsq, m_tiles, n_cand, m.d, m.eps, gain, w_plus, w_minus,
+  cudaLaunchConfig_t cfg = make_cfg(dim3(n_rows / depth), dim3(256), stream, attr, pdl);
+  return cudaLaunchKernelEx(&cfg, head_kernel, h, sumsq, m_tiles, n_rows, depth, m.d, m.eps, gain, w_plus, w_minus,
                             rewards, ts);
 }
 

@@ -169,7 +169,11 @@ struct AttnMerge {
   __nv_bfloat16* o_lo;
   float* out_f32;       // optional fp32 copy
   float* dbg;           // optional fp32 copy
+  // depth-k readout: row b is verify token b % depth of its candidate and also attends to the
+  // candidate's earlier tokens (rows b - b % depth .. b - 1); 1: each row its own entry only
+  int depth = 1;
 };
+constexpr int kMaxReadoutDepth = 8;
 // q_hi / q_lo: bf16 pair of the rotated query [B][n_q][hd]; partial slot s of
 // query row r of its group at part_o[(s * group + r) * hd] (values) and
 // part_ml[(s * group + r) * 2] (max in log2 units, sum).  One CTA per entry of
@@ -204,7 +208,8 @@ struct ModelDims {
   int d, n_q, n_kv, hd, ff, qkv_rows;
   float eps;
 };
-cudaError_t launch_rope_table(const int32_t* seq_lens, int n_cand, int hd, double base, float2* table,
+// rows b: verify token b % depth of candidate b / depth, at position seq_lens[b] + b % depth
+cudaError_t launch_rope_table(const int32_t* seq_lens, int n_rows, int hd, double base, int depth, float2* table,
                               cudaStream_t stream, bool pdl, unsigned long long* ts = nullptr);
 // Activations handed to a projection are stored as a bf16 (hi, lo) pair.
 struct HiLo {
@@ -215,7 +220,8 @@ cudaError_t launch_embed_norm(const ModelDims& m, const __nv_bfloat16* e_v, cons
                               int n_cand, float* h, float* sumsq, HiLo x, cudaStream_t stream, bool pdl,
                               unsigned long long* ts = nullptr);
 // rewards = P(+) from the final RMSNorm of h and the two head rows
-cudaError_t launch_head(const ModelDims& m, const float* h, const float* sumsq, int m_tiles, int n_cand,
+// rewards[b] from row b depth + depth - 1 (each candidate's last verify token)
+cudaError_t launch_head(const ModelDims& m, const float* h, const float* sumsq, int m_tiles, int n_rows, int depth,
                         const __nv_bfloat16* gain, const __nv_bfloat16* w_plus, const __nv_bfloat16* w_minus,
                         float* rewards, cudaStream_t stream, bool pdl, unsigned long long* ts = nullptr);
 cudaError_t launch_split_hilo(const float* in, int64_t count, HiLo out, cudaStream_t stream);

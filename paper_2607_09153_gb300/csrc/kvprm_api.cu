@@ -39,11 +39,12 @@ struct GraphKey {
   int fuse_cs = -1;
   int layer_waits = -1;
   int lora_rank = -1;
+  int depth = -1;
   const void* pool = nullptr;
   int64_t n_pages = -1;
   bool operator==(const GraphKey& o) const {
     return n == o.n && n_pad == o.n_pad && attn_ctas == o.attn_ctas && tc_ctas == o.tc_ctas && n_tc == o.n_tc &&
-           fuse_cs == o.fuse_cs && layer_waits == o.layer_waits && lora_rank == o.lora_rank &&
+           fuse_cs == o.fuse_cs && layer_waits == o.layer_waits && lora_rank == o.lora_rank && depth == o.depth &&
            debug == o.debug && profile == o.profile && pdl == o.pdl && trace == o.trace && pool == o.pool &&
            n_pages == o.n_pages;
   }
@@ -66,6 +67,10 @@ struct kvprm_ctx {
   const bf16 *embed = nullptr, *final_norm = nullptr, *w_plus = nullptr, *w_minus = nullptr;
   std::vector<const bf16*> attn_norm, mlp_norm;
   std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_down;
+  // depth-k readout (kvprm_set_readout_depth): verify tokens per candidate; candidate b of a call is
+  // rows b depth .. b depth + depth - 1 of the batch (expanded tables below)
+  int depth = 1;
+  std::vector<int32_t> row_bt, row_sl;
   // scorer adapter (kvprm_set_lora; rank 0: the merged weights alone): per projection (QKV, O,
   // gate/up, down) and layer the maps of A and B, and t = scale (A x) as hi/lo [npad_max][rank]
   int lora_rank = 0;
@@ -294,7 +299,7 @@ int validate_tables(kvprm_ctx* ctx, int64_t n_pages, const int32_t* bt, const in
 // Plan the attention work of this call on the host (build_attn_work); a
 // sharing plan that does not fit the context's work arrays falls back to
 // private runs, which always fit.
-int plan_work(kvprm_ctx* ctx, const int32_t* bt, const int32_t* sl, int32_t n) {
+int plan_work(kvprm_ctx* ctx, const int32_t* bt, const int32_t* sl, int32_t n, bool allow_fused) {
   kvprm::AttnWorkHost& w = ctx->work_host;
   const int mb = ctx->cfg.max_blocks_per_seq, nkv = ctx->cfg.n_kv_heads;
   auto fits = [&]() {
@@ -302,7 +307,7 @@ int plan_work(kvprm_ctx* ctx, const int32_t* bt, const int32_t* sl, int32_t n) {
            w.slots.size() <= ctx->slot_cap && static_cast<size_t>(w.n_ctas) <= static_cast<size_t>(ctx->num_sms) &&
            static_cast<size_t>(w.n_tc_ctas) <= static_cast<size_t>(ctx->num_sms);
   };
-  if (ctx->fuse_combine &&
+  if (ctx->fuse_combine && allow_fused &&
       kvprm::build_attn_work_fused(bt, sl, n, mb, nkv, ctx->md.n_q / nkv, ctx->num_sms, ctx->slot_cap, w) && fits())
     return KVPRM_OK;
   bool ok = kvprm::build_attn_work(bt, sl, n, mb, nkv, ctx->md.n_q / nkv, ctx->num_sms, ctx->slot_cap, ctx->share_mode, w);
@@ -609,7 +614,8 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
   if (ctx->trace)
     CK(cudaMemsetAsync(ctx->trace_d, 0xFF, sizeof(unsigned long long) * kvprm::kTraceStride * ctx->trace_cap, st),
        "trace reset");
-  LAUNCH(KVPRM_PROF_FUSED, kvprm::launch_rope_table(sl, n, m.hd, ctx->cfg.rope_base, ctx->rope, st, false, TS), "rope");
+  LAUNCH(KVPRM_PROF_FUSED,
+         kvprm::launch_rope_table(sl, n, m.hd, ctx->cfg.rope_base, ctx->depth, ctx->rope, st, false, TS), "rope");
   LAUNCH(KVPRM_PROF_FUSED,
          kvprm::launch_embed_norm(m, ctx->embed, ctx->attn_norm[0], n, ctx->h, ctx->sumsq, X, st, pdl, TS),
          "embed_norm");
@@ -628,7 +634,7 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
       CK(cudaMemcpyAsync(ctx->dbg_v + l * nk, ctx->vself, nk * 4, cudaMemcpyDeviceToDevice, st), "debug v");
     }
     float* dbg = (ctx->debug_flags & 1) ? ctx->dbg + static_cast<size_t>(l) * n * m.n_q * m.hd : nullptr;
-    const kvprm::AttnMerge mg{ctx->q, ctx->kself, ctx->vself, O.hi, O.lo, nullptr, dbg};
+    const kvprm::AttnMerge mg{ctx->q, ctx->kself, ctx->vself, O.hi, O.lo, nullptr, dbg, ctx->depth};
     const kvprm::AttnWork wk = device_work(ctx);
     if (ctx->layer_waits)   // this layer's pages are still being copied in (kvprm_score_host)
       CK(cudaStreamWaitEvent(st, ctx->layer_ready[l], E.capturing ? cudaEventWaitExternal : cudaEventWaitDefault),
@@ -663,8 +669,8 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
            "gemm_down");
     if (l + 1 == NL) {
       LAUNCH(KVPRM_PROF_FUSED,
-             kvprm::launch_head(m, ctx->h, ctx->sumsq, ctx->d_tiles, n, ctx->final_norm, ctx->w_plus, ctx->w_minus,
-                                ctx->rewards_d, st, pdl, TS),
+             kvprm::launch_head(m, ctx->h, ctx->sumsq, ctx->d_tiles, n, ctx->depth, ctx->final_norm, ctx->w_plus,
+                                ctx->w_minus, ctx->rewards_d, st, pdl, TS),
              "reward_head");
     }
     if (ctx->debug_flags & 4) {
@@ -728,6 +734,25 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   int rc = validate_tables(ctx, n_pages, bt, sl, n, &max_pages);
   if (rc) return rc;
   if (n == 0) return KVPRM_OK;
+  // depth-k readout: each candidate's verify tokens are rows of the batch over the candidate's pages
+  const int D = ctx->depth;
+  if (D > 1) {
+    if (static_cast<int64_t>(n) * D > ctx->cfg.max_candidates)
+      return fail(ctx, KVPRM_ECAPACITY, "n_candidates x readout depth = %lld exceeds max_candidates = %d",
+                  static_cast<long long>(n) * D, ctx->cfg.max_candidates);
+    const int mb = ctx->cfg.max_blocks_per_seq;
+    ctx->row_bt.resize(static_cast<size_t>(n) * D * mb);
+    ctx->row_sl.resize(static_cast<size_t>(n) * D);
+    for (int b = 0; b < n; ++b)
+      for (int t = 0; t < D; ++t) {
+        const size_t row = static_cast<size_t>(b) * D + t;
+        ctx->row_sl[row] = sl[b];
+        std::memcpy(ctx->row_bt.data() + row * mb, bt + static_cast<size_t>(b) * mb, sizeof(int32_t) * mb);
+      }
+    bt = ctx->row_bt.data();
+    sl = ctx->row_sl.data();
+    n *= D;
+  }
   const void* pool = kv_pages;
   int64_t pages = n_pages;
   if (max_pages == 0) {   // no cached token anywhere: the pool is never read
@@ -739,7 +764,9 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   }
   if ((rc = ensure_pool_map(ctx, pool, pages, ctx->cfg.n_layers))) return rc;
   ctx->as.layer_pages = pages;
-  if ((rc = plan_work(ctx, bt, sl, n))) return rc;
+  // a depth-k readout's rows share their candidate's pages: the persistent plan scores each page once
+  // per candidate, and its combine adds the causal verify-token entries
+  if ((rc = plan_work(ctx, bt, sl, n, D == 1))) return rc;
   const CallPlan P = make_plan(ctx, n, max_pages);
   if ((rc = ensure_x_maps(ctx, P.n_pad))) return rc;
   if ((rc = ensure_t_maps(ctx, P.n_pad))) return rc;
@@ -765,6 +792,7 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   key.fuse_cs = ctx->work_host.fuse_cs;
   key.layer_waits = ctx->layer_waits ? 1 : 0;
   key.lora_rank = ctx->lora_rank;
+  key.depth = ctx->depth;
   key.n_tc = ctx->work_host.n_tc > 0 ? 1 : 0;
   key.debug = ctx->debug_flags;
   key.profile = ctx->profile ? 1 : 0;
@@ -995,6 +1023,15 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   return KVPRM_OK;
 }
 
+int kvprm_set_readout_depth(kvprm_ctx* ctx, int32_t depth) {
+  if (!ctx) return KVPRM_EINVAL;
+  if (depth < 1 || depth > kvprm::kMaxReadoutDepth)
+    return fail(ctx, KVPRM_EINVAL, "readout depth %d outside [1, %d]", depth, kvprm::kMaxReadoutDepth);
+  if (depth != ctx->depth) drop_graph(ctx);
+  ctx->depth = depth;
+  return KVPRM_OK;
+}
+
 int kvprm_set_lora(kvprm_ctx* ctx, int32_t rank, float scale, const kvprm_lora* lora) {
   if (!ctx) return KVPRM_EINVAL;
   if (rank == 0) {   // back to the merged weights alone
@@ -1158,7 +1195,7 @@ int kvprm_attention(kvprm_ctx* ctx, const void* kv_layer, int64_t n_pages, const
     if (!aligned16(kv_layer)) return fail(ctx, KVPRM_EINVAL, "kv_layer is not 16-byte aligned");
   }
   if ((rc = ensure_pool_map(ctx, pool, pages, 1))) return rc;
-  if ((rc = plan_work(ctx, block_table, seq_lens, n))) return rc;
+  if ((rc = plan_work(ctx, block_table, seq_lens, n, true))) return rc;
   if ((rc = upload_tables(ctx, block_table, seq_lens, n, st))) return rc;
   AttnShape as = ctx->as;
   as.layer_pages = pages;

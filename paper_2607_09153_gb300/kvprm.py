@@ -87,6 +87,7 @@ def lib() -> ctypes.CDLL:
         L.kvprm_attention.argtypes = [vp, vp, i64, i32p, i32p, i32, vp, vp, vp, vp, vp]
         L.kvprm_projection.argtypes = [vp, vp, i32, i32, vp, i32, vp, vp]
         L.kvprm_set_lora.argtypes = [vp, i32, ctypes.c_float, ctypes.POINTER(KvprmLora)]
+        L.kvprm_set_readout_depth.argtypes = [vp, i32]
         L.kvprm_debug_hidden.argtypes = [vp, vp]
         L.kvprm_attention_noalloc.argtypes = [vp, i64, i32p, i32, i32p, i32, i32, i32, i32, vp, vp, vp, vp, vp]
         L.kvprm_set_debug.argtypes = [vp, ctypes.c_int]
@@ -170,6 +171,10 @@ def kvprm_attention(ctx, kv_layer_ptr: int, n_pages: int, block_table, seq_lens,
 
 def kvprm_projection(ctx, W_ptr: int, M: int, K: int, X_ptr: int, n: int, Y_ptr: int, stream_ptr: int = 0) -> None:
     _check(ctx, lib().kvprm_projection(ctx, W_ptr, M, K, X_ptr, n, Y_ptr, stream_ptr))
+
+
+def kvprm_set_readout_depth(ctx, depth: int) -> None:
+    _check(ctx, lib().kvprm_set_readout_depth(ctx, int(depth)))
 
 
 def kvprm_set_lora(ctx, rank: int, scale: float, lora: KvprmLora | None) -> None:
@@ -320,6 +325,10 @@ class Scorer:
                               cast(self._arrays["mlp_norm"]), cast(self._arrays["w_gate_up"]),
                               cast(self._arrays["w_down"]))
         self.ctx = kvprm_create(self.cfg, self.w)
+
+    def set_depth(self, depth: int) -> None:
+        """Depth-k readout: k verify tokens per candidate, the reward read at the last one."""
+        kvprm_set_readout_depth(self.ctx, depth)
 
     def set_lora(self, rank: int, alpha: float = 32.0, factors: list | None = None) -> None:
         """Scorer adapter on every projection (rank 0: merged weights alone); factors[l] holds

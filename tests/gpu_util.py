@@ -34,20 +34,25 @@ def make_scorer(dev: ks.DeviceInputs, max_candidates: int, max_blocks: int):
     return sc
 
 
-def run_gpu(w: ks.Workload, tables: ks.Tables, debug: bool = True, dev=None, scorer=None, extra_flags: int = 0):
-    """Score every candidate on the GPU; returns (rewards [B], attn [N_L][B][nq*hd] or None).
-    extra_flags: further kvprm_set_debug bits (16: rescale on every new attention row maximum)."""
+def run_gpu(w: ks.Workload, tables: ks.Tables, debug: bool = True, dev=None, scorer=None, extra_flags: int = 0,
+            depth: int = 1):
+    """Score every candidate on the GPU; returns (rewards [B], attn [N_L][B depth][nq*hd] or None).
+    extra_flags: further kvprm_set_debug bits (16: rescale on every new attention row maximum);
+    depth > 1: a depth-k readout (candidate b's verify tokens are attention rows b depth + t)."""
     torch = require_gpu()
     import paper_2607_09153_gb300 as kp
     dev = dev or ks.DeviceInputs(w, tables)
-    sc = scorer or make_scorer(dev, max(1, w.n_candidates), w.max_blocks)
+    sc = scorer or make_scorer(dev, max(1, w.n_candidates * depth), w.max_blocks)
     a = w.arch
+    if depth > 1:
+        sc.set_depth(depth)
     if debug or extra_flags:
         kp.kvprm_set_debug(sc.ctx, (1 if debug else 0) | extra_flags)
     r = sc.score(dev.pool, w.block_table, w.seq_lens)
     attn = None
     if debug:
-        out = torch.empty((a.n_layers, w.n_candidates, a.n_q_heads * a.head_dim), dtype=torch.float32, device="cuda")
+        out = torch.empty((a.n_layers, w.n_candidates * depth, a.n_q_heads * a.head_dim), dtype=torch.float32,
+                          device="cuda")
         kp.kvprm_debug_attn_out(sc.ctx, out.data_ptr())
         torch.cuda.synchronize()
         attn = out.cpu().numpy().astype(np.float64)
@@ -62,14 +67,15 @@ def attn_rel_err(gpu: np.ndarray, ref: np.ndarray) -> np.ndarray:
     return num / np.maximum(den, 1e-30)
 
 
-def compare(w, tables, cand_ids=None, gpu_rewards=None, gpu_attn=None, label=""):
+def compare(w, tables, cand_ids=None, gpu_rewards=None, gpu_attn=None, label="", depth: int = 1):
     """Against the oracle in exact mode: bf16 weights and cache, every activation exact."""
     ids = list(range(w.n_candidates)) if cand_ids is None else list(cand_ids)
-    ref = oracle.score_synth(w, tables, ids, mirror=False)
+    ref = oracle.score_synth(w, tables, ids, mirror=False, depth=depth)
     dp = np.abs(gpu_rewards[ids] - ref.p_plus)
     msg = f"{label}: max |dP| = {dp.max():.3e}"
     if gpu_attn is not None:
-        e = attn_rel_err(gpu_attn[:, ids], ref.attn)
+        rows = [i * depth + t for i in ids for t in range(depth)]   # the oracle's rows, in the same order
+        e = attn_rel_err(gpu_attn[:, rows], ref.attn)
         msg += f", max attn rel err = {e.max():.3e}"
         assert e.max() <= ATTN_RTOL, msg + f" (worst layer/cand {np.unravel_index(e.argmax(), e.shape)})"
     assert dp.max() <= P_PLUS_ATOL, msg

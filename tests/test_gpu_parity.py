@@ -276,3 +276,43 @@ def test_lora_switch_and_errors():
     assert np.array_equal(sc.score(dev.pool, w.block_table, w.seq_lens), merged)
     fresh.close()
     sc.close()
+
+
+# ---------------------------------------------------------------- depth-k readout (kvprm_set_readout_depth)
+@pytest.mark.parametrize("arch,depth,make", [
+    (ks.ARCH_TINY, 3, lambda a: ks.distinct("depth", a, 81, [0, 17, 100, 250], gain_std=0.2)),
+    (ks.Arch(2, 1536, 12, 2, 128, 8960), 4, lambda a: ks.distinct("depth", a, 82, [2048] * 4, gain_std=0.2)),
+    # 8 rows per candidate on the tensor-core path for a 64-row shared prefix group (G = 7)
+    (ks.Arch(2, 3584, 28, 4, 128, 18944), 2, lambda a: ks.shared_prefix("depth", a, 83, 8, 256, 40, gain_std=0.2)),
+])
+def test_depth_readout(arch, depth, make):
+    """k verify tokens per candidate, causal among themselves, reward at the last (Sec. 3 R_k, Sec. 5):
+    every token's attention output per layer and P(+) against the oracle's depth-k readout."""
+    t = ks.Tables.make(0.2)
+    w = make(arch)
+    r, attn, dev, sc = run_gpu(w, t, depth=depth)
+    compare(w, t, gpu_rewards=r, gpu_attn=attn, label=f"depth {depth} d={arch.d_model}", depth=depth)
+    # depth 1 on the same context gives the single-token scores
+    sc.set_depth(1)
+    r1 = sc.score(dev.pool, w.block_table, w.seq_lens)
+    ref1 = oracle.score_synth(w, t, mirror=False)
+    assert np.abs(r1 - ref1.p_plus).max() <= 1e-3
+    sc.close()
+
+
+def test_depth_errors():
+    import paper_2607_09153_gb300 as kp
+    t = ks.Tables.make(0.2)
+    w = ks.distinct("depth_err", ks.ARCH_TINY, 84, [5, 9, 30], gain_std=0.2)
+    dev = ks.DeviceInputs(w, t)
+    sc = make_scorer(dev, 4, w.max_blocks)   # room for 4 rows
+    for bad in (0, 9, -1):
+        with pytest.raises(kp.KvprmError):
+            sc.set_depth(bad)
+    sc.set_depth(2)   # 3 candidates x 2 rows > 4
+    with pytest.raises(kp.KvprmError):
+        sc.score(dev.pool, w.block_table, w.seq_lens)
+    sc.set_depth(1)
+    r = sc.score(dev.pool, w.block_table, w.seq_lens)
+    assert np.isfinite(r).all()
+    sc.close()
