@@ -358,8 +358,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
   trace_end(ts);
 }
 
-// The combine: one CTA of W warps per (candidate, kv head) running combine_group.
-template <int HD, int ROWS, int W>
+// The combine: one CTA of W warps per (candidate, kv head) running combine_group (DEEP: a depth-k
+// readout's causal verify-token entries).
+template <int HD, int ROWS, int W, bool DEEP>
 __global__ void __launch_bounds__(W * 32) attn_combine_kernel(
     const int32_t* __restrict__ slot_base, const int32_t* __restrict__ nslots, int n_q, int n_kv, int group,
     const float* __restrict__ part_o, const float* __restrict__ part_ml, AttnMerge mg, unsigned long long* ts) {
@@ -370,8 +371,8 @@ __global__ void __launch_bounds__(W * 32) attn_combine_kernel(
   const int first = slot_base[cg], ns = nslots[cg];   // host-uploaded before the call: no wait needed
   grid_dep_wait();   // the partials (and q, k_self, v_self) are written by earlier kernels
   if (threadIdx.x == 0) trace_event(ts, 0);
-  combine_group<HD, ROWS, W>(threadIdx.x, b, g, first, ns, n_q, n_kv, group, part_o, part_ml, mg, csm,
-                             [] { __syncthreads(); });
+  combine_group<HD, ROWS, W, DEEP>(threadIdx.x, b, g, first, ns, n_q, n_kv, group, part_o, part_ml, mg, csm,
+                                   [] { __syncthreads(); });
   if (threadIdx.x == 0) trace_event(ts, 1);
   trace_end(ts);
 }
@@ -1186,14 +1187,20 @@ bool build_attn_work_fused(const int32_t* bt, const int32_t* sl, int n, int max_
 
 cudaError_t attention_configure() {
   cudaError_t e;
-  if ((e = set_smem(attn_combine_kernel<64, 8, 8>, CombineShape<64, 8, 8>::kBytes)) != cudaSuccess) return e;
-  if ((e = set_smem(attn_combine_kernel<64, 16, 8>, CombineShape<64, 16, 8>::kBytes)) != cudaSuccess) return e;
-  if ((e = set_smem(attn_combine_kernel<128, 8, 8>, CombineShape<128, 8, 8>::kBytes)) != cudaSuccess) return e;
-  if ((e = set_smem(attn_combine_kernel<128, 16, 8>, CombineShape<128, 16, 8>::kBytes)) != cudaSuccess) return e;
-  if ((e = set_smem(attn_combine_kernel<64, 8, 4>, CombineShape<64, 8, 4>::kBytes)) != cudaSuccess) return e;
-  if ((e = set_smem(attn_combine_kernel<64, 16, 4>, CombineShape<64, 16, 4>::kBytes)) != cudaSuccess) return e;
-  if ((e = set_smem(attn_combine_kernel<128, 8, 4>, CombineShape<128, 8, 4>::kBytes)) != cudaSuccess) return e;
-  if ((e = set_smem(attn_combine_kernel<128, 16, 4>, CombineShape<128, 16, 4>::kBytes)) != cudaSuccess) return e;
+#define KVPRM_COMBINE_SMEM(HD_, R_, W_)                                                                           \
+  if ((e = set_smem(attn_combine_kernel<HD_, R_, W_, false>, CombineShape<HD_, R_, W_>::kBytes)) != cudaSuccess) \
+    return e;                                                                                                    \
+  if ((e = set_smem(attn_combine_kernel<HD_, R_, W_, true>, CombineShape<HD_, R_, W_>::kBytes)) != cudaSuccess)  \
+    return e;
+  KVPRM_COMBINE_SMEM(64, 8, 8)
+  KVPRM_COMBINE_SMEM(64, 16, 8)
+  KVPRM_COMBINE_SMEM(128, 8, 8)
+  KVPRM_COMBINE_SMEM(128, 16, 8)
+  KVPRM_COMBINE_SMEM(64, 8, 4)
+  KVPRM_COMBINE_SMEM(64, 16, 4)
+  KVPRM_COMBINE_SMEM(128, 8, 4)
+  KVPRM_COMBINE_SMEM(128, 16, 4)
+#undef KVPRM_COMBINE_SMEM
   if ((e = set_smem(attn_kernel<64, false>, AttnSmem<64>::kDynamic)) != cudaSuccess) return e;
   if ((e = set_smem(attn_kernel<64, true>, AttnSmem<64>::kDynamic)) != cudaSuccess) return e;
   if ((e = set_smem(attn_kernel<128, false>, AttnSmem<128>::kDynamic)) != cudaSuccess) return e;
@@ -1305,8 +1312,11 @@ cudaError_t launch_attn_combine(const AttnShape& s, const AttnWork& wk, int n, c
   do {                                                                                                           \
     cfg.dynamicSmemBytes = CombineShape<HD_, R_, W_>::kBytes;                                                    \
     cfg.blockDim = dim3(32 * W_, 1, 1);                                                                          \
-    return cudaLaunchKernelEx(&cfg, attn_combine_kernel<HD_, R_, W_>, wk.slot_base, wk.nslots, s.n_q, s.n_kv,    \
-                              s.group, part_o, part_ml, mg, ts);                                                 \
+    if (mg.depth > 1)                                                                                            \
+      return cudaLaunchKernelEx(&cfg, attn_combine_kernel<HD_, R_, W_, true>, wk.slot_base, wk.nslots, s.n_q,    \
+                                s.n_kv, s.group, part_o, part_ml, mg, ts);                                       \
+    return cudaLaunchKernelEx(&cfg, attn_combine_kernel<HD_, R_, W_, false>, wk.slot_base, wk.nslots, s.n_q,     \
+                              s.n_kv, s.group, part_o, part_ml, mg, ts);                                         \
   } while (0)
 #define KVPRM_COMBINE(HD_, R_)             \
   do {                                     \

@@ -315,7 +315,7 @@ __device__ __forceinline__ void merge_warp_states(int group, const float* mo, co
 //                              / (2^(s_self - M*) + sum_w 2^(M_w - M*) L_w).
 // In a depth-k readout (mg.depth > 1) row b is verify token t = b % depth and the
 // self entries are its candidate's tokens 0 .. t (rows b - t .. b), each a term
-// 2^(s_j - M*) v_j of the same sums;
+// 2^(s_j - M*) v_j of the same sums (the DEEP variant);
 // written as a bf16 (hi, lo) pair (and optional fp32 copies).  `smem` holds
 // CombineShape::kBytes; sync() is a barrier over exactly the 32 W threads.  A
 // caller running several groups back to back syncs between them.
@@ -330,7 +330,7 @@ struct CombineShape {
   static constexpr size_t kBytes = kSelf + sizeof(float) * ROWS * kMaxReadoutDepth;
 };
 
-template <int HD, int ROWS, int W_ = 8, typename Sync>
+template <int HD, int ROWS, int W_ = 8, bool DEEP = false, typename Sync>
 __device__ __forceinline__ void combine_group(int tid, int b, int g, int first, int ns, int n_q, int n_kv, int group,
                                               const float* __restrict__ part_o, const float* __restrict__ part_ml,
                                               const AttnMerge& mg, uint8_t* smem, Sync sync) {
@@ -375,7 +375,8 @@ __device__ __forceinline__ void combine_group(int tid, int b, int g, int first, 
   }
   // the self entries' scores of head `warp`: token t's own (k_self already loaded) and, in a
   // depth-k readout, its candidate's earlier tokens (rows b - t .. b - 1)
-  const int t_self = b % mg.depth, n_self = t_self + 1;
+  // DEEP (a depth-k readout): a compiled variant of its own, so that the single-entry form keeps its code
+  const int t_self = DEEP ? b % mg.depth : 0, n_self = DEEP ? t_self + 1 : 1;
   const int64_t hk0 = hk - static_cast<int64_t>(t_self) * n_kv;
   if (warp < group) {
     for (int e = 0; e < n_self; ++e) {
