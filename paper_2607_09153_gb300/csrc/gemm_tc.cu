@@ -34,6 +34,7 @@
 // h ⊙ g and the per-tile sums of squares, and the QKV and SILU epilogues scale
 // their accumulators by r before RoPE / SiLU.  No normalisation kernel runs
 // between the projections.
+#include <type_traits>
 #include "kernels.h"
 #include "ptx.cuh"
 
@@ -107,7 +108,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
   const int cbeg = static_cast<int>(rank) * cols;
   const int cend = min(cbeg + cols, ep.n_valid);
   const int nc = cend > cbeg ? cend - cbeg : 0;
-  const bool hpreload = ep.mode == GemmEpilogue::RESID && nc <= kHPreCols;
+  const bool hpreload = ep.mode == GemmEpilogue::RESID && nc <= kHPreCols && mt == 1;
   constexpr int kEpiBatch = LARGE ? 8 : 1;
 
   if (threadIdx.x == 0) {
@@ -253,11 +254,12 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
   const int m = warp * 32 + lane;
   const bool merged = has_lo && 2 * n_pad <= 256;
   const uint32_t tile_cols = tmem_cols / static_cast<uint32_t>(mt);
-  // one m-tile at a time: park it, reduce it over the cluster (split K only: never with two
-  // tiles), write its epilogue
+  // one m-tile at a time: park it, reduce it over the cluster (split K), write its epilogue; with two
+  // tiles and split K the second is parked once every peer has read this CTA's first partial
   for (int tt = 0; tt < mt; ++tt) {
     const int m_tile = m_tile0 + tt;
     const uint32_t tcol = static_cast<uint32_t>(tt) * tile_cols;
+    if (tt > 0 && cs > 1) cluster_wait();   // matches the arrive after the previous tile's reduction
     for (int c0 = 0; c0 < n_pad; c0 += 16) {
       float v[16];
       if (nk > 0 && have) {
@@ -277,41 +279,49 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       for (int j = 0; j < 16; ++j) acc[(c0 + j) * kBM + m] = v[j];
     }
     tc_fence_before();
-    if (tt == 0) {
+    if (tt == 0 || cs > 1) {
       cluster_sync();   // every rank's partial is parked
-      if (threadIdx.x == 0) trace_event(ts, 3);
-      if (ep.late_trigger) grid_dep_launch();
-
-      // ---------------- reduce this rank's candidate columns over the cluster, then the epilogue
-      grid_dep_wait();   // outputs may still be read by kernels that precede this one
+      if (tt == 0) {
+        if (threadIdx.x == 0) trace_event(ts, 3);
+        if (ep.late_trigger) grid_dep_launch();
+        // ---------------- reduce this rank's candidate columns over the cluster, then the epilogue
+        grid_dep_wait();   // outputs may still be read by kernels that precede this one
+      }
       // Step 1: acc[c][m] <- sum over ranks of acc_r[c][m] for this rank's columns
       // (only this rank reads them, so it may overwrite its own copy).  Two columns
       // per round trip when the cluster has <= 8 ranks (four with 16-byte loads in
       // the large-batch image's clusters of 4), all peer loads in flight.
       // Without split K (cs = 1) the parked accumulator is already the sum.
-      if (LARGE && cs == 4) {
-        // four consecutive rows of one column per thread (a warp covers a column's 128 rows), four
-        // columns per round: 16 loads of 16 bytes in flight, the four ranks' copies of each
-        const int rq = static_cast<int>(threadIdx.x) & 31, cg = static_cast<int>(threadIdx.x) >> 5;
-        for (int c0 = cbeg + cg; c0 < cend; c0 += 4 * 4) {
-          float4 v[16];
+      if (LARGE && (cs == 4 || cs == 8)) {
+        // four consecutive rows of one column per thread (a warp covers a column's 128 rows), 16 / CS
+        // columns per round: 16 loads of 16 bytes in flight, the CS ranks' copies of each
+        auto vreduce = [&](auto cs_c) {
+          constexpr int CS = decltype(cs_c)::value, PER = 16 / CS;
+          const int rq = static_cast<int>(threadIdx.x) & 31, cg = static_cast<int>(threadIdx.x) >> 5;
+          for (int c0 = cbeg + cg; c0 < cend; c0 += 4 * PER) {
+            float4 v[16];
 #pragma unroll
-          for (int k = 0; k < 16; ++k) {   // rank k % 4 of column c0 + 4 (k / 4)
-            const int cc = c0 + 4 * (k / 4);
-            v[k] = cc < cend ? ld_cluster4(acc + cc * kBM + 4 * rq, static_cast<uint32_t>(k % 4))
-                             : make_float4(0.f, 0.f, 0.f, 0.f);
-          }
+            for (int k = 0; k < 16; ++k) {   // rank k % CS of column c0 + 4 (k / CS)
+              const int cc = c0 + 4 * (k / CS);
+              v[k] = cc < cend ? ld_cluster4(acc + cc * kBM + 4 * rq, static_cast<uint32_t>(k % CS))
+                               : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const int cc = c0 + 4 * j;
-            if (cc < cend) {
-              const float4 a = v[4 * j], b = v[4 * j + 1], c = v[4 * j + 2], d = v[4 * j + 3];
-              *reinterpret_cast<float4*>(acc + cc * kBM + 4 * rq) =
-                  make_float4((a.x + b.x) + (c.x + d.x), (a.y + b.y) + (c.y + d.y), (a.z + b.z) + (c.z + d.z),
-                              (a.w + b.w) + (c.w + d.w));
+            for (int j = 0; j < PER; ++j) {
+              const int cc = c0 + 4 * j;
+              if (cc >= cend) continue;
+              const float4* u = v + CS * j;
+              auto add = [](float4 x, float4 y) { return make_float4(x.x + y.x, x.y + y.y, x.z + y.z, x.w + y.w); };
+              float4 r = add(add(u[0], u[1]), add(u[2], u[3]));
+              if constexpr (CS == 8) r = add(r, add(add(u[4], u[5]), add(u[6], u[7])));
+              *reinterpret_cast<float4*>(acc + cc * kBM + 4 * rq) = r;
             }
           }
-        }
+        };
+        if (cs == 4)
+          vreduce(std::integral_constant<int, 4>{});
+        else
+          vreduce(std::integral_constant<int, 8>{});
       } else if (cs > 1) {
         const int step = cs <= 8 ? 2 : 1;
         for (int c = cbeg; c < cend; c += step) {
@@ -343,8 +353,9 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
         }
       }
       if (threadIdx.x == 0) trace_event(ts, 4);   // this rank's columns are reduced over the cluster
-      // no peer reads this CTA's shared memory any more: arrive on the exit barrier now and wait for the
-      // peers only before exiting, so the barrier's latency hides behind the epilogue
+      // no peer reads this tile's partial any more once every rank has arrived here: arrive now and
+      // wait only before this shared memory is reused (the next tile's parking, or the exit), so the
+      // barrier's latency hides behind the epilogue
       __syncwarp();
       cluster_arrive();
     }
@@ -718,6 +729,33 @@ GemmPlan plan_gemm(int M, int K, int n_pad, int num_sms, bool has_lo, bool gate_
       p.stages = stages2;
       p.smem_bytes = smem2;
       p.tmem_cols = 2 * cols;
+    }
+  }
+  // long split-K loops at large batches (the 7B down projection at B = 256: 74 K tiles per rank): two
+  // m-tiles per CTA over twice the ranks, the same CTA count.  A 96 KB stage then carries 16 MMAs
+  // (~1 us), enough to cover its own loading (~0.8 us), where one tile's 8 MMAs left the tensor pipe
+  // waiting a third of the time; the second tile's parking and cluster reduction cost less than those
+  // stalls once the K loop is long
+  if (!gate_up && n_pad >= 128 && per_sm == 1 && p.mt == 1 && cs >= 2 && cs * 2 <= 8 && p.m_tiles % 2 == 0 &&
+      p.kt_per_split >= 32) {
+    const int cs2 = cs * 2;
+    const uint32_t st2 = 2 * kWTileBytes + static_cast<uint32_t>(n_pad) * kBK * 2 * (has_lo ? 2u : 1u);
+    const int kps2 = (p.k_tiles + cs2 - 1) / cs2;
+    int stages2 = static_cast<int>((192u * 1024u) / st2);
+    if (stages2 > 8) stages2 = 8;
+    if (stages2 > kps2) stages2 = kps2;
+    size_t ring2 = static_cast<size_t>(stages2) * st2;
+    if (ring2 < acc) ring2 = acc;
+    const size_t smem2 = ring2 + 1024 + kTailBytes;
+    if (stages2 >= 2 && 2 * p.tmem_cols <= 512 && smem2 <= kGemmMaxSmem && (p.m_tiles / 2) * cs2 <= num_sms &&
+        cs2 * 4 <= p.k_tiles && n_pad % cs2 == 0) {
+      p.mt = 2;
+      p.cluster = cs2;
+      p.splits = cs2;
+      p.kt_per_split = kps2;
+      p.stages = stages2;
+      p.smem_bytes = smem2;
+      p.tmem_cols = 2 * p.tmem_cols;
     }
   }
   return p;
