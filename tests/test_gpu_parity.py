@@ -316,3 +316,12 @@ def test_depth_errors():
     r = sc.score(dev.pool, w.block_table, w.seq_lens)
     assert np.isfinite(r).all()
     sc.close()
+
+
+def test_lora_with_depth_readout():
+    """Both extensions at once: a rank-64 adapter on every projection and 3 verify tokens per candidate."""
+    t = ks.Tables.make(0.2)
+    w = ks.distinct("lora_depth", _lora_arch(ks.ARCH_TINY, 64), 91, [0, 33, 140], gain_std=0.2)
+    r, attn, dev, sc = run_gpu(w, t, depth=3)
+    compare(w, t, gpu_rewards=r, gpu_attn=attn, label="adapter r=64 with depth 3", depth=3)
+    sc.close()
