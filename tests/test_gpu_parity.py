@@ -263,9 +263,10 @@ def test_lora_switch_and_errors():
     with_lora = sc.score(dev.pool, w.block_table, w.seq_lens)
     sc.set_lora(0)
     merged = sc.score(dev.pool, w.block_table, w.seq_lens)
-    w0 = ks.distinct("lora_sw", ks.ARCH_TINY, 71, [3, 40, 100], gain_std=0.2)
-    fresh = make_scorer(ks.DeviceInputs(w0, t), 8, w0.max_blocks)
-    base = fresh.score(ks.DeviceInputs(w0, t).pool, w0.block_table, w0.seq_lens)
+    w0 = ks.distinct("lora_sw", ks.ARCH_TINY, 71, [3, 40, 100], gain_std=0.2)   # same seed: same weights and cache
+    dev0 = ks.DeviceInputs(w0, t)
+    fresh = make_scorer(dev0, 8, w0.max_blocks)
+    base = fresh.score(dev0.pool, w0.block_table, w0.seq_lens)
     assert np.array_equal(merged, base)
     assert np.abs(with_lora - merged).max() > 1e-5
     for bad in (32, 100, 2048, -64):
