@@ -250,6 +250,8 @@ def make_workload(args):
     w = ks.make_workload(args.workload)
     if args.lora:
         w.arch = dataclasses.replace(w.arch, lora_rank=args.lora)
+    if args.layers:   # the same shapes with fewer layers: small profiler captures of one layer's kernels
+        w.arch = dataclasses.replace(w.arch, n_layers=args.layers)
     return w
 
 
@@ -505,6 +507,8 @@ def main():
     ap.add_argument("--workload", default="qwen1p5b_b16_l2048", choices=list(ks.WORKLOAD_NAMES))
     ap.add_argument("--depth", type=int, default=1,
                     help="verify tokens per candidate (depth-k readout; 1, the default: one)")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="run the workload's shapes with this many layers (0: all; for small profiler captures)")
     ap.add_argument("--lora", type=int, default=0,
                     help="scorer adapter rank kept apart from the weights (0: merged weights, the default)")
     ap.add_argument("--profile-steps", type=int, default=50)
