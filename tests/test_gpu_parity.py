@@ -237,6 +237,7 @@ def _lora_arch(arch, rank):
 
 @pytest.mark.parametrize("arch,rank,lens,sample", [
     (ks.ARCH_TINY, 64, [0, 50, 129, 200], None),                                    # r = 64: half an A tile
+    (ks.ARCH_TINY, 1024, [7, 90], None),                                             # the largest rank
     (ks.Arch(2, 1536, 12, 2, 128, 8960), 256, [2048] * 16, None),                   # 1.5B layers, small image
     (ks.Arch(2, 3584, 28, 4, 128, 18944), 256, [(37 * b) % 300 for b in range(64)],  # 7B layers, B = 64
      [0, 1, 31, 63]),
