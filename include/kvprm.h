@@ -45,7 +45,7 @@ enum {
   KVPRM_ECUDA = 4,        /* a CUDA runtime/driver call failed */
   KVPRM_ENOMEM = 5,       /* device or pinned-host allocation failed */
   KVPRM_ETIMEOUT = 6,     /* a bounded in-kernel wait gave up (blocking calls, kvprm_check_device) */
-  KVPRM_EUNSUPPORTED = 7  /* a shape this build does not implement */
+  KVPRM_EUNSUPPORTED = 7  /* a shape the library does not implement */
 };
 
 /* Scorer shape and context capacity.
