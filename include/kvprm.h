@@ -362,6 +362,23 @@ KVPRM_API int kvprm_plan_attention(const int32_t* block_table, int32_t max_block
                                    int32_t n_candidates, int32_t n_kv_heads, int32_t group, int32_t n_ctas,
                                    int32_t share, kvprm_attn_plan* plan);
 
+/* The launch plan a scoring context uses for one projection GEMM y = W x (W [M][K] bf16, x a bf16
+ * hi/lo pair when has_lo, batch padded to n_pad, a multiple of 16), computed on the host only (no
+ * device call), so that its invariants can be checked without a GPU.  gate_up: W holds the gate rows
+ * then the up rows (M = d_ff pairs, 64 of each per tile).
+ *  m_tiles       128-row tiles (gate/up: 64-pair tiles)
+ *  k_tiles       64-wide K tiles; kt_per_split per rank of a split-K cluster
+ *  cluster       CTAs per thread-block cluster (split-K ranks)
+ *  tiles_per_cta m-tiles each CTA takes (1, or 2 for large batches)
+ *  stages        shared-memory ring stages; tmem_cols tensor-memory columns; smem_bytes per CTA
+ * Errors: KVPRM_EINVAL (M, K or num_sms < 1, n_pad not a positive multiple of 16, out NULL). */
+typedef struct {
+  int32_t m_tiles, k_tiles, kt_per_split, cluster, tiles_per_cta, stages, tmem_cols;
+  int64_t smem_bytes;
+} kvprm_projection_plan;
+KVPRM_API int kvprm_plan_projection(int32_t M, int32_t K, int32_t n_pad, int32_t num_sms, int32_t has_lo,
+                                    int32_t gate_up, kvprm_projection_plan* out);
+
 /* Device-side status: returns KVPRM_OK, or KVPRM_ETIMEOUT if an in-kernel
  * bounded wait gave up since the last check (the flag is then cleared).
  * Synchronises the context's last stream. */

@@ -1341,6 +1341,21 @@ int kvprm_resolve(kvprm_ctx* ctx, int32_t b, int64_t* phys_row) {
   return KVPRM_OK;
 }
 
+int kvprm_plan_projection(int32_t M, int32_t K, int32_t n_pad, int32_t num_sms, int32_t has_lo, int32_t gate_up,
+                          kvprm_projection_plan* out) {
+  if (!out || M < 1 || K < 1 || num_sms < 1 || n_pad < 16 || n_pad % 16) return KVPRM_EINVAL;
+  const GemmPlan g = kvprm::plan_gemm(M, K, n_pad, num_sms, has_lo != 0, gate_up != 0);
+  out->m_tiles = g.m_tiles;
+  out->k_tiles = g.k_tiles;
+  out->kt_per_split = g.kt_per_split;
+  out->cluster = g.cluster;
+  out->tiles_per_cta = g.mt;
+  out->stages = g.stages;
+  out->tmem_cols = static_cast<int32_t>(g.tmem_cols);
+  out->smem_bytes = static_cast<int64_t>(g.smem_bytes);
+  return KVPRM_OK;
+}
+
 int kvprm_plan_attention(const int32_t* block_table, int32_t max_blocks_per_seq, const int32_t* seq_lens,
                          int32_t n_candidates, int32_t n_kv_heads, int32_t group, int32_t n_ctas, int32_t share,
                          kvprm_attn_plan* plan) {

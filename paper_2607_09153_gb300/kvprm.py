@@ -43,6 +43,11 @@ class KvprmWeights(ctypes.Structure):
                 ("mlp_norm", _VPP), ("w_gate_up", _VPP), ("w_down", _VPP)]
 
 
+class KvprmProjectionPlan(ctypes.Structure):
+    _fields_ = [(k, ctypes.c_int32) for k in ("m_tiles", "k_tiles", "kt_per_split", "cluster", "tiles_per_cta",
+                                               "stages", "tmem_cols")] + [("smem_bytes", ctypes.c_int64)]
+
+
 class KvprmLora(ctypes.Structure):
     _fields_ = [(k, _VPP) for k in ("a_qkv", "b_qkv", "a_o", "b_o", "a_gate_up", "b_gate_up", "a_down", "b_down")]
 
@@ -88,6 +93,7 @@ def lib() -> ctypes.CDLL:
         L.kvprm_projection.argtypes = [vp, vp, i32, i32, vp, i32, vp, vp]
         L.kvprm_set_lora.argtypes = [vp, i32, ctypes.c_float, ctypes.POINTER(KvprmLora)]
         L.kvprm_set_readout_depth.argtypes = [vp, i32]
+        L.kvprm_plan_projection.argtypes = [i32, i32, i32, i32, i32, i32, ctypes.POINTER(KvprmProjectionPlan)]
         L.kvprm_debug_hidden.argtypes = [vp, vp]
         L.kvprm_attention_noalloc.argtypes = [vp, i64, i32p, i32, i32p, i32, i32, i32, i32, vp, vp, vp, vp, vp]
         L.kvprm_set_debug.argtypes = [vp, ctypes.c_int]
@@ -171,6 +177,17 @@ def kvprm_attention(ctx, kv_layer_ptr: int, n_pages: int, block_table, seq_lens,
 
 def kvprm_projection(ctx, W_ptr: int, M: int, K: int, X_ptr: int, n: int, Y_ptr: int, stream_ptr: int = 0) -> None:
     _check(ctx, lib().kvprm_projection(ctx, W_ptr, M, K, X_ptr, n, Y_ptr, stream_ptr))
+
+
+def kvprm_plan_projection(M: int, K: int, n_pad: int, num_sms: int, has_lo: bool = True,
+                          gate_up: bool = False) -> dict:
+    """The projection GEMM's launch plan (host only)."""
+    out = KvprmProjectionPlan()
+    rc = lib().kvprm_plan_projection(int(M), int(K), int(n_pad), int(num_sms), int(has_lo), int(gate_up),
+                                     ctypes.byref(out))
+    if rc != 0:
+        raise KvprmError(rc, "kvprm_plan_projection: bad arguments")
+    return {k: getattr(out, k) for k, _ in KvprmProjectionPlan._fields_}
 
 
 def kvprm_set_readout_depth(ctx, depth: int) -> None:
