@@ -269,3 +269,21 @@ def test_bad_arguments():
         kp.kvprm_plan_attention(np.zeros((1, 1), np.int32), [17], 1, 1, 4)   # 17 tokens > 16 * 1 block
     with pytest.raises(kp.KvprmError):
         kp.kvprm_plan_attention(np.zeros((1, 1), np.int32), [1], 1, 17, 4)   # G > 16
+
+
+@pytest.mark.parametrize("k", [2, 4, 8])
+def test_depth_rows_stream_each_page_once(k):
+    """A depth-k readout expands each candidate into k rows over the same pages (kvprm_set_readout_depth):
+    the schedule must score every token for every row, yet stream each (page, kv head) once, the k rows
+    forming one sharing group (shared runs below 6 rows, the tensor-core path from 6)."""
+    w = ks.make_workload("qwen1p5b_b16_l2048")
+    bt = np.repeat(np.asarray(w.block_table, np.int32), k, axis=0)
+    sl = np.repeat(np.asarray(w.seq_lens, np.int32), k)
+    p = check_plan(bt, sl, 2, 6, 152, 3)
+    streams = collections.Counter()
+    for s in p["segs"]:
+        kind, g, c, nc, off, npg, last, slot = (int(x) for x in s)
+        assert kind != 0, "a row of a depth-k candidate was planned as private pages"
+        for pg in p["pages"][off:off + npg]:
+            streams[(int(pg), g)] += 1
+    assert set(streams.values()) == {1}
