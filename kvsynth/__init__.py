@@ -33,8 +33,11 @@ EMBED, FINAL_NORM, W_PLUS, W_MINUS, ATTN_NORM, W_QKV, W_O, MLP_NORM, W_GATE_UP, 
 (LORA_A_QKV, LORA_B_QKV, LORA_A_O, LORA_B_O, LORA_A_GATE_UP, LORA_B_GATE_UP, LORA_A_DOWN,
  LORA_B_DOWN) = range(10, 18)
 LORA_KINDS = tuple(range(10, 18))
+# per-head RMSNorm gains of q and k (Qwen3-style q/k norm), [head_dim] per layer
+Q_NORM, K_NORM = 18, 19
+QK_NORM_KINDS = (Q_NORM, K_NORM)
 LAYER_KINDS = (ATTN_NORM, W_QKV, W_O, MLP_NORM, W_GATE_UP, W_DOWN)
-GAIN_KINDS = (FINAL_NORM, ATTN_NORM, MLP_NORM)
+GAIN_KINDS = (FINAL_NORM, ATTN_NORM, MLP_NORM, Q_NORM, K_NORM)
 
 
 # --------------------------------------------------------------------------- build
@@ -130,13 +133,24 @@ class Tables:
     kv: np.ndarray      # N(0, 1)
     w: np.ndarray       # N(0, 0.02)
     g: np.ndarray       # 1 + gain_std * N(0, 1)
+    qkv: np.ndarray | None = None   # W_qkv draws when set (N(0, qkv_std)), else those of `w`
 
     @staticmethod
-    def make(gain_std: float = 0.0) -> "Tables":
+    def make(gain_std: float = 0.0, qkv_std: float | None = None) -> "Tables":
+        """qkv_std: draw W_qkv at this std instead of 0.02.  Wider query/key projections give scores
+        q.k / sqrt(hd) tens of units apart, the peaked attention of a trained scorer."""
         kv = quantile_table(1.0)
         w = quantile_table(0.02)
         g = quantile_table(gain_std, 1.0) if gain_std > 0 else np.full(65536, 0x3F80, dtype=np.uint16)
-        return Tables(kv, w, g)
+        qkv = quantile_table(qkv_std) if qkv_std is not None else None
+        return Tables(kv, w, g, qkv)
+
+    def for_kind(self, kind: int) -> np.ndarray:
+        if kind in GAIN_KINDS:
+            return self.g
+        if kind == W_QKV and self.qkv is not None:
+            return self.qkv
+        return self.w
 
 
 # --------------------------------------------------------------------------- architectures
@@ -153,13 +167,14 @@ class Arch:
     page_size: int = 16
     lora_rank: int = 0          # 0: merged scorer weights; else an adapter of this rank on every projection
     lora_alpha: float = 32.0    # adapter scale alpha / rank
+    qk_norm: bool = False       # per-head RMSNorm of q and k (gains [head_dim] per layer) before RoPE
 
     @property
     def lora_scale(self) -> float:
         return self.lora_alpha / self.lora_rank if self.lora_rank else 0.0
 
     def layer_kinds(self) -> tuple[int, ...]:
-        return LAYER_KINDS + (LORA_KINDS if self.lora_rank else ())
+        return LAYER_KINDS + (LORA_KINDS if self.lora_rank else ()) + (QK_NORM_KINDS if self.qk_norm else ())
 
     @property
     def qkv_rows(self) -> int:
@@ -173,7 +188,7 @@ class Arch:
             W_GATE_UP: (2 * self.d_ff, d), W_DOWN: (d, self.d_ff),
             LORA_A_QKV: (r, d), LORA_B_QKV: (self.qkv_rows, r), LORA_A_O: (r, self.n_q_heads * hd), LORA_B_O: (d, r),
             LORA_A_GATE_UP: (r, d), LORA_B_GATE_UP: (2 * self.d_ff, r), LORA_A_DOWN: (r, self.d_ff),
-            LORA_B_DOWN: (d, r),
+            LORA_B_DOWN: (d, r), Q_NORM: (hd,), K_NORM: (hd,),
         }[kind]
 
     def weight_bytes(self) -> int:
@@ -360,7 +375,7 @@ def host_weight(arch: Arch, kind: int, layer: int, seed: int, tables: Tables) ->
     out = np.empty(int(np.prod(shape)), np.uint16)
     lib = host_lib()
     tid = lib.synth_weight_tid(kind, layer if kind >= ATTN_NORM else 0)
-    table = tables.g if kind in GAIN_KINDS else tables.w
+    table = tables.for_kind(kind)
     lib.synth_fill(_p(out, ctypes.c_uint16), out.size, seed, tid, _p(table, ctypes.c_uint16), _nthreads())
     return out.reshape(shape)
 
@@ -414,13 +429,14 @@ class DeviceInputs:
         t_kv = torch.from_numpy(tables.kv.view(np.int16)).to(dev)
         t_w = torch.from_numpy(tables.w.view(np.int16)).to(dev)
         t_g = torch.from_numpy(tables.g.view(np.int16)).to(dev)
+        t_q = torch.from_numpy(tables.qkv.view(np.int16)).to(dev) if tables.qkv is not None else t_w
         hl = host_lib()
 
         def fill(kind, layer):
             shape = a.weight_shape(kind)
             t = torch.empty(shape, dtype=torch.bfloat16, device=dev)
             tid = hl.synth_weight_tid(kind, layer if kind >= ATTN_NORM else 0)
-            table = t_g if kind in GAIN_KINDS else t_w
+            table = t_g if kind in GAIN_KINDS else (t_q if kind == W_QKV else t_w)
             rc = lib.synth_dev_fill(t.data_ptr(), t.numel(), w.seed, tid, table.data_ptr(), sp)
             assert rc == 0, rc
             return t
@@ -443,7 +459,7 @@ class DeviceInputs:
                                              t_kv.data_ptr(), sp)
             assert rc == 0, rc
         self.stream.synchronize()
-        del d_seg, d_off, t_kv, t_w, t_g
+        del d_seg, d_off, t_kv, t_w, t_g, t_q
 
 
 # --------------------------------------------------------------------------- oracle providers
@@ -461,6 +477,7 @@ class SynthModel(ctypes.Structure):
         ("cand_len", ctypes.POINTER(ctypes.c_int64)),
         ("cand_seg", ctypes.POINTER(ctypes.POINTER(ctypes.c_int32))),
         ("cand_off", ctypes.POINTER(ctypes.POINTER(ctypes.c_int32))),
+        ("table_qkv", ctypes.POINTER(ctypes.c_uint16)),
     ]
 
 
@@ -471,7 +488,7 @@ class Providers:
     def __init__(self, w: Workload, tables: Tables, nthreads: int | None = None):
         lib = host_lib()
         a = w.arch
-        self._keep = [tables.w, tables.g, tables.kv]
+        self._keep = [tables.w, tables.g, tables.kv, tables.qkv]
         segs = [np.ascontiguousarray(s, np.int32) for s in w.cand_seg]
         offs = [np.ascontiguousarray(o, np.int32) for o in w.cand_off]
         self._keep += segs + offs
@@ -482,7 +499,8 @@ class Providers:
         self._keep += [seg_arr, off_arr, lens]
         self.model = SynthModel(w.seed, _p(tables.w, ctypes.c_uint16), _p(tables.g, ctypes.c_uint16),
                                 _p(tables.kv, ctypes.c_uint16), nthreads or _nthreads(), a.n_kv_heads, a.head_dim,
-                                len(segs), _p(lens, ctypes.c_int64), seg_arr, off_arr)
+                                len(segs), _p(lens, ctypes.c_int64), seg_arr, off_arr,
+                                _p(tables.qkv, ctypes.c_uint16) if tables.qkv is not None else None)
         self.weight_fn = ctypes.cast(lib.synth_weight_provider, ctypes.c_void_p).value
         self.kv_fn = ctypes.cast(lib.synth_kv_provider, ctypes.c_void_p).value
         self.user = ctypes.cast(ctypes.pointer(self.model), ctypes.c_void_p).value

@@ -124,7 +124,8 @@ void synth_kv_pool_layer(uint16_t* pool_layer, int64_t n_pages, const int32_t* p
 /* Weight kinds, in the order the oracle asks for them:
  *   0 embed_verify [d], 1 final_norm [d], 2 w_plus [d], 3 w_minus [d],
  *   4 attn_norm [d], 5 w_qkv [(nq+2nkv)hd][d], 6 w_o [d][nq hd],
- *   7 mlp_norm [d], 8 w_gate_up [2ff][d], 9 w_down [d][ff]                */
+ *   7 mlp_norm [d], 8 w_gate_up [2ff][d], 9 w_down [d][ff],
+ *   10 .. 17 low-rank adapter factors, 18 q_norm [hd], 19 k_norm [hd]        */
 typedef struct {
     uint64_t seed;
     const uint16_t* table_w;   /* weights: bf16(0.02 * quantile) */
@@ -137,13 +138,15 @@ typedef struct {
     const int64_t* cand_len;
     const int32_t* const* cand_seg;
     const int32_t* const* cand_off;
+    const uint16_t* table_qkv; /* W_qkv when non-NULL (a wider draw for peaked attention), else table_w */
 } synth_model;
 
 int synth_weight_provider(void* user, int kind, int layer, uint16_t* out, int64_t n) {
     const synth_model* m = (const synth_model*)user;
-    int is_gain = (kind == 1 || kind == 4 || kind == 7);
+    int is_gain = (kind == 1 || kind == 4 || kind == 7 || kind == 18 || kind == 19);
     int lay = (kind >= 4) ? layer : 0;
-    synth_fill(out, n, m->seed, synth_weight_tid(kind, lay), is_gain ? m->table_g : m->table_w, m->nthreads);
+    const uint16_t* table = is_gain ? m->table_g : ((kind == 5 && m->table_qkv) ? m->table_qkv : m->table_w);
+    synth_fill(out, n, m->seed, synth_weight_tid(kind, lay), table, m->nthreads);
     return 0;
 }
 

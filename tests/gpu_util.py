@@ -81,3 +81,108 @@ def compare(w, tables, cand_ids=None, gpu_rewards=None, gpu_attn=None, label="",
     assert dp.max() <= P_PLUS_ATOL, msg
     print(msg)
     return ref
+
+
+# ---------------------------------------------------------------- peaked attention inputs
+class PlantedCase:
+    """One layer's paged cache with planted keys, and queries aimed at them, so that the softmax of
+    the attention read-out is peaked: scores q.k / sqrt(hd) tens of units apart, one key (or a run of
+    identical keys) dominating, the largest score arriving late in the sequence.
+
+    The plant is keyed by token identity (segment, offset) and applied twice, independently: to the
+    paged pool (through page_seg / page_off) and to each candidate's logical K/V (through cand_seg /
+    cand_off), so the block-table walk is still checked against the logical sequence."""
+
+    def __init__(self, w: ks.Workload, tables: ks.Tables, seed: int, needles: list, runs: list = (),
+                 broad_std: float = 15.0):
+        a = w.arch
+        self.w, self.arch = w, a
+        rng = np.random.default_rng(seed)
+        nkv, hd, G = a.n_kv_heads, a.head_dim, a.n_q_heads // a.n_kv_heads
+        self.pool = ks.host_kv_pool(w, tables, layers=[0])[0]          # [pages][2][nkv][16][hd]
+        self.K, self.V = [], []
+        for b in range(w.n_candidates):
+            K, V = ks.host_kv_logical(w, 0, b, tables)
+            self.K.append(K)
+            self.V.append(V)
+        keys = {}
+
+        def plant(seg, off, g, key_bits):
+            hit = (w.page_seg == seg) & (w.page_off == off)
+            pg, slot = np.nonzero(hit)
+            self.pool[pg, 0, g, slot, :] = key_bits
+            for b in range(w.n_candidates):
+                j = np.nonzero((w.cand_seg[b] == seg) & (w.cand_off[b] == off))[0]
+                self.K[b][j, g, :] = key_bits
+
+        # needles: (seg, off) -> one key per kv head, drawn N(0, 1) and rounded to bf16
+        for seg, off in needles:
+            kb = ks.f64_to_bf16_bits(rng.normal(0, 1, (nkv, hd)))
+            keys[(seg, off)] = kb
+            for g in range(nkv):
+                plant(seg, off, g, kb[g])
+        # identical-key runs: (seg, off0, count) all carry the same key per kv head
+        for seg, off0, count in runs:
+            kb = ks.f64_to_bf16_bits(rng.normal(0, 1, (nkv, hd)))
+            keys[(seg, off0)] = kb
+            for off in range(off0, off0 + count):
+                for g in range(nkv):
+                    plant(seg, off, g, kb[g])
+        # queries: per candidate the key of its latest planted identity, scaled per head so that the
+        # top score is ~10 .. ~70 units above the rest; every fourth head a broad N(0, broad_std)
+        # query (scores spread over tens of units without a planted target)
+        B, nq = w.n_candidates, a.n_q_heads
+        self.q = np.empty((B, nq, hd), np.float32)
+        alphas = np.array([1.0, 2.5, 4.5, 6.0])
+        for b in range(B):
+            pos = {ident: max(np.nonzero((w.cand_seg[b] == ident[0]) & (w.cand_off[b] == ident[1]))[0], default=-1)
+                   for ident in keys}
+            target = max(pos, key=pos.get) if pos and max(pos.values()) >= 0 else None
+            for h in range(nq):
+                g = h // G
+                if target is None or h % 4 == 3:
+                    self.q[b, h] = rng.normal(0, broad_std, hd).astype(np.float32)
+                else:
+                    kf = ks.bf16_bits_to_f64(keys[target][g])
+                    self.q[b, h] = (alphas[h % 4] * kf + rng.normal(0, 0.05, hd)).astype(np.float32)
+        self.kself = rng.normal(0, 1, (B, nkv, hd)).astype(np.float32)
+        self.vself = rng.normal(0, 1, (B, nkv, hd)).astype(np.float32)
+
+    def expected(self) -> np.ndarray:
+        """The oracle's read-out o [B][nq][hd] (fp64) of every (candidate, head)."""
+        a = self.arch
+        G = a.n_q_heads // a.n_kv_heads
+        out = np.empty((self.w.n_candidates, a.n_q_heads, a.head_dim))
+        for b in range(self.w.n_candidates):
+            for h in range(a.n_q_heads):
+                g = h // G
+                out[b, h], _ = oracle.attend(self.q[b, h].astype(np.float64), self.K[b][:, g, :], self.V[b][:, g, :],
+                                             self.kself[b, g].astype(np.float64), self.vself[b, g].astype(np.float64))
+        return out
+
+    def score_spread(self) -> float:
+        """Largest gap between a row's top score and its median score (in units of q.k / sqrt(hd))."""
+        a = self.arch
+        G = a.n_q_heads // a.n_kv_heads
+        gap = 0.0
+        for b in range(self.w.n_candidates):
+            if len(self.K[b]) == 0:
+                continue
+            for h in range(a.n_q_heads):
+                Kf = ks.bf16_bits_to_f64(self.K[b][:, h // G, :])
+                s = Kf @ self.q[b, h].astype(np.float64) / np.sqrt(a.head_dim)
+                gap = max(gap, float(s.max() - np.median(s)))
+        return gap
+
+    def device(self):
+        torch = require_gpu()
+        pool = torch.from_numpy(self.pool.view(np.int16)).cuda()
+        q, k, v = (torch.from_numpy(np.ascontiguousarray(x)).cuda() for x in (self.q, self.kself, self.vself))
+        return pool, q, k, v
+
+
+def row_rel_err(got: np.ndarray, ref: np.ndarray) -> float:
+    """Largest per-(candidate, head) relative inf-norm error."""
+    num = np.abs(got - ref).max(axis=-1)
+    den = np.maximum(np.abs(ref).max(axis=-1), 1e-30)
+    return float((num / den).max())
