@@ -254,7 +254,12 @@ KVPRM_API int kvprm_debug_hidden(kvprm_ctx* ctx, float* d_out);
  * make it before any stream capture.  All calls share the array, which keeps
  * the last call's contents; calls that overlap on the GPU race with each other
  * and must be serialised by the caller.  An in-kernel bounded-wait timeout is
- * recorded in the array but not reported by this entry point. */
+ * recorded in the array but not reported by this entry point.
+ * The attention schedule is built on the host for each call and uploaded from
+ * pageable host memory, so the call blocks the host until the driver has
+ * staged those bytes.  A stream that is being captured into a CUDA graph is
+ * refused with KVPRM_EUNSUPPORTED (a graph would replay that one call's
+ * schedule from a host buffer that later calls overwrite). */
 #define KVPRM_NOALLOC_SCRATCH_BYTES (32u << 20)
 KVPRM_API int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, const int32_t* block_table,
                                       int32_t max_blocks_per_seq, const int32_t* seq_lens, int32_t n_candidates,
@@ -383,6 +388,29 @@ KVPRM_API int kvprm_plan_projection(int32_t M, int32_t K, int32_t n_pad, int32_t
  * bounded wait gave up since the last check (the flag is then cleared).
  * Synchronises the context's last stream. */
 KVPRM_API int kvprm_check_device(kvprm_ctx* ctx);
+
+/* Failure-detection test hooks (no counterpart in the paper: they let tests
+ * drive the error paths on the host, without faulting or hanging a GPU).
+ *  kvprm_debug_set_alloc_limit: from now on the library may allocate at most
+ *    `bytes` more device and pinned-host memory, process-wide (every allocation
+ *    lowers the remainder; -1 removes the limit).  An allocation beyond it fails
+ *    as if the device were full: kvprm_create, kvprm_score_host (growing its
+ *    device pool) and kvprm_set_lora return KVPRM_ENOMEM and leave an existing
+ *    context as it was.
+ *  kvprm_debug_inject_error: where = 1 makes the next scoring call on ctx
+ *    report a failed launch of its forward (KVPRM_ECUDA, nothing of the forward
+ *    enqueued) as a CUDA error would; where = 0 cancels it.  Later calls run
+ *    normally.
+ *  kvprm_debug_wait_probe: enqueues on `stream` one thread that waits, bounded
+ *    by limit_us (1 .. 2e6 microseconds), for a device flag that nothing sets,
+ *    with the same give-up protocol as every in-kernel wait: when the limit
+ *    passes it records its site (code 9) in the context's device error word and
+ *    returns, so the next kvprm_check_device (or blocking call) returns
+ *    KVPRM_ETIMEOUT and clears the word; the context stays usable.
+ * Errors: KVPRM_EINVAL (NULL context, bad argument), KVPRM_ECUDA. */
+KVPRM_API int kvprm_debug_set_alloc_limit(int64_t bytes);
+KVPRM_API int kvprm_debug_inject_error(kvprm_ctx* ctx, int32_t where);
+KVPRM_API int kvprm_debug_wait_probe(kvprm_ctx* ctx, int32_t limit_us, void* stream);
 
 /* Per-kernel-class timing of kvprm_score* calls, measured with CUDA events on
  * the scoring stream while enabled (one event pair per launch; programmatic

@@ -165,6 +165,16 @@ cudaError_t launch_head(const ModelDims& m, const float* h, const float* sumsq, 
                             rewards, ts);
 }
 
+__global__ void wait_probe_kernel(const int* flag, int* err, unsigned long long limit_ns) {
+  if (threadIdx.x == 0) flag_wait(flag, err, limit_ns, kDevProbeTimeout);
+}
+
+cudaError_t launch_wait_probe(const int* flag, int* err, unsigned long long limit_ns, cudaStream_t stream) {
+  if (limit_ns > kWaitTimeoutNs) limit_ns = kWaitTimeoutNs;
+  wait_probe_kernel<<<1, 32, 0, stream>>>(flag, err, limit_ns);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_split_hilo(const float* in, int64_t count, HiLo out, cudaStream_t stream) {
   int64_t blocks = (count + 255) / 256;
   if (blocks > 152 * 8) blocks = 152 * 8;

@@ -225,6 +225,9 @@ cudaError_t launch_head(const ModelDims& m, const float* h, const float* sumsq, 
                         const __nv_bfloat16* gain, const __nv_bfloat16* w_plus, const __nv_bfloat16* w_minus,
                         float* rewards, cudaStream_t stream, bool pdl, unsigned long long* ts = nullptr);
 cudaError_t launch_split_hilo(const float* in, int64_t count, HiLo out, cudaStream_t stream);
+// One thread waits (bounded by limit_ns, see flag_wait) for *flag to become nonzero; on timeout it
+// records kDevProbeTimeout in *err.  The failure-detection test hook behind kvprm_debug_wait_probe.
+cudaError_t launch_wait_probe(const int* flag, int* err, unsigned long long limit_ns, cudaStream_t stream);
 
 
 }  // namespace kvprm

@@ -7,6 +7,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -157,6 +158,10 @@ struct kvprm_ctx {
   double prof_ms[KVPRM_PROF_N] = {};
   std::string last_error;
   cudaStream_t last_stream = nullptr;
+  // failure-detection hooks: a scoring call reports an injected CUDA failure instead of launching
+  // (kvprm_debug_inject_error); a flag that nothing sets, for the bounded-wait probe
+  int inject_fail = 0;
+  int* probe_flag = nullptr;
 };
 
 namespace {
@@ -199,8 +204,26 @@ int make_map(kvprm_ctx* ctx, CUtensorMap* m, const void* base, uint64_t inner, u
   return KVPRM_OK;
 }
 
+// Device and pinned-host bytes the library may still allocate, process-wide (-1: no limit); lowered
+// by every allocation while set (kvprm_debug_set_alloc_limit, a failure-detection test hook).
+std::atomic<long long> g_alloc_budget{-1};
+
+bool take_budget(size_t bytes) {
+  long long cur = g_alloc_budget.load();
+  while (cur >= 0) {
+    if (static_cast<long long>(bytes) > cur) return false;
+    if (g_alloc_budget.compare_exchange_weak(cur, cur - static_cast<long long>(bytes))) return true;
+  }
+  return true;
+}
+
 template <typename T>
 int dalloc(kvprm_ctx* ctx, T** p, size_t count, const char* what) {
+  if (!take_budget(count * sizeof(T))) {
+    *p = nullptr;
+    return fail(ctx, KVPRM_ENOMEM, "allocation of %s (%zu bytes) exceeds the allocation budget", what,
+                count * sizeof(T));
+  }
   cudaError_t e = cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T) > 0 ? count * sizeof(T) : 16);
   if (e != cudaSuccess) {
     *p = nullptr;
@@ -244,6 +267,7 @@ void free_ctx(kvprm_ctx* c) {
   cudaFree(c->tc_prof);
   cudaFree(c->dummy_pool);
   cudaFree(c->dev_pool);
+  cudaFree(c->probe_flag);
   if (c->staging) cudaFreeHost(c->staging);
   if (c->h_rewards) cudaFreeHost(c->h_rewards);
   if (c->h_err) cudaFreeHost(c->h_err);
@@ -774,6 +798,10 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   if (ctx->layer_waits && (rc = enqueue_pool_copy(ctx, st))) return rc;
   ctx->last_n = n;
   ctx->last_stream = st;
+  if (ctx->inject_fail) {   // failure-detection hook: report a failed launch, enqueue nothing more
+    ctx->inject_fail = 0;
+    return cuda_fail(ctx, cudaErrorLaunchFailure, "injected failure of the forward's launch");
+  }
 
   if (!ctx->use_graph) {
     Enq E{ctx, st, ctx->use_pdl && !ctx->profile, ctx->profile, &ctx->live_marks};
@@ -988,7 +1016,12 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   CREATE_CK(dalloc(ctx, &ctx->rewards_d, static_cast<size_t>(Bmax), "rewards"));
   CREATE_CK(dalloc(ctx, &ctx->err_d, 1, "err"));
   CREATE_CK(dalloc(ctx, &ctx->dummy_pool, static_cast<size_t>(NL) * 2 * m.n_kv * 16 * m.hd, "dummy pool"));
+  CREATE_CK(dalloc(ctx, &ctx->probe_flag, 1, "wait probe flag"));
   {
+    if (!take_budget(sizeof(int32_t) * ctx->tables_ints + sizeof(float) * Bmax + sizeof(int))) {
+      free_ctx(ctx);
+      return KVPRM_ENOMEM;
+    }
     cudaError_t e =
         cudaMallocHost(reinterpret_cast<void**>(&ctx->staging), sizeof(int32_t) * ctx->tables_ints);
     if (e == cudaSuccess) e = cudaMallocHost(reinterpret_cast<void**>(&ctx->h_rewards), sizeof(float) * Bmax);
@@ -1152,6 +1185,7 @@ int kvprm_score_host(kvprm_ctx* ctx, const void* h_kv_pages, int64_t n_pages, co
       ctx->dev_pool_bytes = 0;
       drop_graph(ctx);
       ctx->pool_ptr = nullptr;
+      if (!take_budget(bytes)) return fail(ctx, KVPRM_ENOMEM, "device pool of %zu bytes exceeds the allocation budget", bytes);
       cudaError_t e = cudaMalloc(&ctx->dev_pool, bytes);
       if (e != cudaSuccess) {
         cudaGetLastError();
@@ -1344,6 +1378,7 @@ int kvprm_resolve(kvprm_ctx* ctx, int32_t b, int64_t* phys_row) {
 int kvprm_plan_projection(int32_t M, int32_t K, int32_t n_pad, int32_t num_sms, int32_t has_lo, int32_t gate_up,
                           kvprm_projection_plan* out) {
   if (!out || M < 1 || K < 1 || num_sms < 1 || n_pad < 16 || n_pad % 16) return KVPRM_EINVAL;
+  if (n_pad > 256) return KVPRM_EUNSUPPORTED;   // a context holds at most 256 candidates
   const GemmPlan g = kvprm::plan_gemm(M, K, n_pad, num_sms, has_lo != 0, gate_up != 0);
   out->m_tiles = g.m_tiles;
   out->k_tiles = g.k_tiles;
@@ -1400,6 +1435,28 @@ int kvprm_plan_attention(const int32_t* block_table, int32_t max_blocks_per_seq,
     std::memcpy(plan->slot_base, w.slot_base.data(), sizeof(int32_t) * w.slot_base.size());
     std::memcpy(plan->nslots, w.nslots.data(), sizeof(int32_t) * w.nslots.size());
   }
+  return KVPRM_OK;
+}
+
+int kvprm_debug_set_alloc_limit(int64_t bytes) {
+  g_alloc_budget.store(bytes < 0 ? -1 : static_cast<long long>(bytes));
+  return KVPRM_OK;
+}
+
+int kvprm_debug_inject_error(kvprm_ctx* ctx, int32_t where) {
+  if (!ctx) return KVPRM_EINVAL;
+  if (where != 0 && where != 1) return fail(ctx, KVPRM_EINVAL, "injection point %d: 0 (none) or 1", where);
+  ctx->inject_fail = where;
+  return KVPRM_OK;
+}
+
+int kvprm_debug_wait_probe(kvprm_ctx* ctx, int32_t limit_us, void* stream) {
+  if (!ctx) return KVPRM_EINVAL;
+  if (limit_us < 1 || limit_us > 2000000) return fail(ctx, KVPRM_EINVAL, "wait limit %d us outside [1, 2e6]", limit_us);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  CK(kvprm::launch_wait_probe(ctx->probe_flag, ctx->err_d, 1000ull * static_cast<unsigned long long>(limit_us), st),
+     "wait probe");
+  ctx->last_stream = st;
   return KVPRM_OK;
 }
 

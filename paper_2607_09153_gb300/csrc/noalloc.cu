@@ -14,6 +14,13 @@
 // and it keeps the last call's contents, so calls that overlap on the GPU (on
 // different streams, or from several host threads) race and corrupt each
 // other's results; serialise them.
+//
+// Each call builds its attention schedule on the host and uploads it into the
+// array with cudaMemcpyAsync from pageable host memory, so the call returns
+// only once the driver has staged those bytes (the host waits for the copy
+// engine).  For the same reason a call on a stream that is being captured is
+// refused: a graph would keep the host address of a buffer that later calls
+// overwrite, and the schedule of that one call.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
@@ -132,6 +139,12 @@ extern "C" int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, co
     }
   }
   if (max_pages > 0 && (!kv_layer || !al16(kv_layer))) return KVPRM_EINVAL;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  {
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(st, &cap) != cudaSuccess) return KVPRM_ECUDA;
+    if (cap != cudaStreamCaptureStatusNone) return KVPRM_EUNSUPPORTED;
+  }
 
   unsigned char* scratch = nullptr;
   int rc = setup_current_device(&scratch);
@@ -173,7 +186,6 @@ extern "C" int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, co
   CUtensorMap tm;
   if (kvprm::encode_pool_map(g_encode, &tm, pool, pages, n_kv_heads, head_dim) != CUDA_SUCCESS) return KVPRM_ECUDA;
 
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
   int* err = reinterpret_cast<int*>(scratch + cv.err);
   kvprm::HiLo Q{reinterpret_cast<__nv_bfloat16*>(scratch + cv.qhi), reinterpret_cast<__nv_bfloat16*>(scratch + cv.qlo)};
   __nv_bfloat16* ohi = reinterpret_cast<__nv_bfloat16*>(scratch + cv.ohi);

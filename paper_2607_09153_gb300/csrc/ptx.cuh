@@ -16,6 +16,7 @@
 namespace kvprm {
 
 constexpr int kDevTimeout = 1;                          // value written to the device error word
+constexpr int kDevProbeTimeout = 9;                     // the wait probe's flag wait (kvprm_debug_wait_probe)
 constexpr unsigned long long kWaitTimeoutNs = 2000000000ull;  // 2 s
 constexpr unsigned long long kErrPollNs = 20000ull;           // waits shorter than 20 us skip the error word
 
@@ -91,6 +92,25 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* e
       atomicCAS(err, 0, site);
       return false;
     }
+  }
+}
+
+// Wait until *flag is nonzero, bounded like mbar_wait: returns false (after
+// recording `site` in *err) once limit_ns of global time have passed, or, once
+// the wait has lasted kErrPollNs, as soon as another thread has flagged an
+// error.  No shared memory, asynchronous copy or tensor memory is involved, so
+// giving up leaves nothing in flight.
+__device__ __forceinline__ bool flag_wait(const int* flag, int* err, unsigned long long limit_ns, int site) {
+  const uint64_t t0 = global_timer_ns();
+  for (;;) {
+    if (*(volatile const int*)flag != 0) return true;
+    const uint64_t dt = global_timer_ns() - t0;
+    if (dt >= kErrPollNs && *(volatile int*)err != 0) return false;
+    if (dt > limit_ns) {
+      atomicCAS(err, 0, site);
+      return false;
+    }
+    __nanosleep(1000);
   }
 }
 

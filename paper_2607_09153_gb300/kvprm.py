@@ -101,6 +101,9 @@ def lib() -> ctypes.CDLL:
         L.kvprm_debug_layers.argtypes = [vp, ctypes.c_int, vp]
         L.kvprm_resolve.argtypes = [vp, i32, i64p]
         L.kvprm_check_device.argtypes = [vp]
+        L.kvprm_debug_set_alloc_limit.argtypes = [i64]
+        L.kvprm_debug_inject_error.argtypes = [vp, i32]
+        L.kvprm_debug_wait_probe.argtypes = [vp, i32, vp]
         L.kvprm_set_profile.argtypes = [vp, ctypes.c_int]
         L.kvprm_set_trace.argtypes = [vp, ctypes.c_int]
         L.kvprm_get_trace.argtypes = [vp, i32, i32p, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)]
@@ -273,6 +276,21 @@ def kvprm_resolve(ctx, b: int, length: int) -> np.ndarray:
 
 def kvprm_check_device(ctx) -> None:
     _check(ctx, lib().kvprm_check_device(ctx))
+
+
+def kvprm_debug_set_alloc_limit(n_bytes: int) -> None:
+    """Failure-detection hook: the library may allocate at most n_bytes more (-1: no limit)."""
+    rc = lib().kvprm_debug_set_alloc_limit(int(n_bytes))
+    if rc != KVPRM_OK:
+        raise KvprmError(rc, "kvprm_debug_set_alloc_limit failed")
+
+
+def kvprm_debug_inject_error(ctx, where: int = 1) -> None:
+    _check(ctx, lib().kvprm_debug_inject_error(ctx, int(where)))
+
+
+def kvprm_debug_wait_probe(ctx, limit_us: int, stream_ptr: int = 0) -> None:
+    _check(ctx, lib().kvprm_debug_wait_probe(ctx, int(limit_us), stream_ptr))
 
 
 def kvprm_set_profile(ctx, enable: bool) -> None:

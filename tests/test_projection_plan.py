@@ -55,3 +55,12 @@ def test_projection_plan_errors():
     for args in [(0, 64, 16, SMS), (64, 0, 16, SMS), (64, 64, 24, SMS), (64, 64, 16, 0)]:
         with pytest.raises(kp.KvprmError):
             kp.kvprm_plan_projection(*args)
+
+
+def test_projection_plan_beyond_context_batch():
+    # a context holds at most 256 candidates: larger padded batches are not plannable
+    for n_pad in (272, 512, 1024):
+        with pytest.raises(kp.KvprmError) as e:
+            kp.kvprm_plan_projection(4608, 3584, n_pad, SMS)
+        assert e.value.code == kp.KVPRM_EUNSUPPORTED
+    assert kp.kvprm_plan_projection(4608, 3584, 256, SMS)["tmem_cols"] <= 512
