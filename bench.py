@@ -4,16 +4,20 @@ One step = one kvprm_score call: the verify token of every candidate in the
 batch forwarded through all layers against its paged cache (embedding, per
 layer RMSNorm / QKV / RoPE / paged split-K attention / combine / O / RMSNorm /
 SiLU-gated MLP, final norm and the two-logit head).  Default workload: the
-1.5B-shaped scorer (28 layers, d=1536, 12/2 heads, hd=128, MLP 8960) scoring
-B=16 candidates with distinct caches of L=2048 (page size 16), seeded
-synthetic bf16 weights N(0, 0.02) and K/V N(0, 1).
+largest configuration that fits one GPU, the 8B-shaped scorer (32 layers,
+d=4096, 32/8 heads, hd=128, MLP 14336) scoring B=8 candidates with distinct
+caches of L=32768 (page size 16; 48.3 GB of weights and cache per call),
+seeded synthetic bf16 weights N(0, 0.02) and K/V N(0, 1).
 
 Printed (rank 0, one JSON line): scores/s over the timed steps with inputs
 resident in HBM (`value`), the same through the host-buffer C-ABI call with
 the cache copied host->device every step (`e2e`), the per-kernel-class CUDA
-event times of a second timed pass, the roofline of the dominant kernel and
-of the attention kernel, the SM clocks seen during the timed region, and the
-CPU oracle timed on a bounded sample of the same workload (`cpu_baseline`).
+event times of a profiled pass, the time each kernel class adds to the
+pipelined timeline of a traced call, the roofline of the dominant kernel and
+of the attention, the SM clocks seen during the timed region, the CPU oracle
+timed on a bounded sample of the same workload (`cpu_baseline`, with the
+single-thread oracle on the two small configurations), and `workloads`: the
+other four configurations measured the same way in the same run.
 
 `--impl reference` times the CPU oracle alone (the reference arm).
 Multi-GPU (torchrun): each rank scores its own replica batch (candidates
@@ -192,68 +196,89 @@ def ncu_traffic(kernel: str, workload: str):
 
 
 # ---------------------------------------------------------------- CPU oracle
-def cpu_oracle_time(w, tables, budget_s: float = 12.0, max_cands: int | None = None, depth: int = 1):
-    """Time the oracle (exact mode) on a bounded sample of the workload's candidates."""
-    import kvsynth as ks
-    import oracle
-    nthreads = os.cpu_count() or 1
-    a = w.arch
-    t0 = time.perf_counter()
-    W = ks.host_weights(a, w.seed, tables)
-    t_gen = time.perf_counter() - t0
-    cap = w.n_candidates if max_cands is None else min(max_cands, w.n_candidates)
+class OracleRunner:
+    """The oracle (exact mode) on a fixed sample of a workload's candidates: weights and the sample's
+    logical K/V are generated once, beforehand; one step scores the sample once."""
 
-    def run(ids):
-        kv = [[ks.host_kv_logical(w, l, b, tables) for b in ids] for l in range(a.n_layers)]
+    def __init__(self, w, tables, nthreads: int | None = None, depth: int = 1):
+        import kvsynth as ks
+        self.w, self.tables, self.depth = w, tables, depth
+        self.nthreads = nthreads or (os.cpu_count() or 1)
+        t0 = time.perf_counter()
+        self.W = ks.host_weights(w.arch, w.seed, tables)
+        self.t_gen = time.perf_counter() - t0
+        self.kv = {}
+
+    def step(self, ids) -> float:
+        import kvsynth as ks
+        import oracle
+        a = self.w.arch
+        for b in ids:
+            if b not in self.kv:
+                self.kv[b] = [ks.host_kv_logical(self.w, l, b, self.tables) for l in range(a.n_layers)]
+        kv = [[self.kv[b][l] for b in ids] for l in range(a.n_layers)]
         t = time.perf_counter()
-        oracle.score_dense(a, W, kv, mirror=False, want_attn=False, nthreads=nthreads, depth=depth)
+        oracle.score_dense(a, self.W, kv, mirror=False, want_attn=False, nthreads=self.nthreads, depth=self.depth)
         return time.perf_counter() - t
 
-    t1 = run([0])
-    n = int(max(1, min(cap, budget_s / max(t1, 1e-3))))
-    if n > 1:
-        ids = list(range(n))
-        tn = run(ids)
-    else:
-        ids, tn = [0], t1
-    return {"value": n / tn, "unit": "scores/s", "cores": nthreads, "kind": "oracle",
-            "sample": f"{n} of {w.n_candidates} candidates of {w.name}, fp64 exact mode, {tn:.2f} s "
-                      f"(weights generated beforehand in {t_gen:.1f} s, not timed)"}
+    def sample_size(self, budget_s: float) -> int:
+        """Candidates per step so that one step takes about budget_s (at least one)."""
+        t1 = self.step([0])
+        return int(max(1, min(self.w.n_candidates, budget_s / max(t1, 1e-3))))
+
+    def describe(self, n: int, t: float, steps: int = 1) -> str:
+        return (f"{n} of {self.w.n_candidates} candidates of {self.w.name} per step, fp64 exact mode, "
+                f"{t:.2f} s per step over {steps} step(s), {self.nthreads} thread(s) (weights generated "
+                f"beforehand in {self.t_gen:.1f} s and the sample's K/V before the first step, not timed)")
+
+
+def cpu_oracle_time(w, tables, budget_s: float = 12.0, depth: int = 1, nthreads: int | None = None):
+    """The oracle timed on a bounded sample of the workload's candidates (the first n)."""
+    r = OracleRunner(w, tables, nthreads, depth)
+    n = r.sample_size(budget_s)
+    t = r.step(list(range(n)))
+    return {"value": n / t, "unit": "scores/s", "cores": r.nthreads, "kind": "oracle", "sample": r.describe(n, t)}
 
 
 def run_reference(args, world, rank):
-    """The reference arm: the CPU oracle as it stands, on this host's cores."""
+    """The reference arm: the CPU oracle as it stands, on this host's cores.  One step scores a fixed
+    sample of the workload's candidates (sized so that a step takes ~--ref-step-s); ms_per_step is
+    that observed step time and value the sample's candidates per second."""
     if rank != 0:
         return
     import kvsynth as ks
     w = make_workload(args)
     t = ks.Tables.make()
-    samples = []
-    budget = max(5.0, 60.0 / max(1, args.steps + args.warmup))
+    runner = OracleRunner(w, t, depth=args.depth)
+    n = runner.sample_size(args.ref_step_s)
+    ids = list(range(n))
+    times = []
     for i in range(args.warmup + args.steps):
-        r = cpu_oracle_time(w, t, budget_s=budget, max_cands=4, depth=args.depth)
+        dt = runner.step(ids)
         if i >= args.warmup:
-            samples.append(r)
-    val = float(np.mean([s["value"] for s in samples]))
+            times.append(dt)
+    step_s = float(np.mean(times))
+    val = n / step_s
     line = {"impl": "reference", "metric": METRIC, "value": val, "unit": "scores/s", "n_gpus": args.gpus,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * w.n_candidates / val,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000.0 * step_s,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": workload_config(w, args),
-            "cpu_baseline": {"value": val, "unit": "scores/s", "cores": samples[0]["cores"], "kind": "oracle",
-                             "sample": samples[0]["sample"]},
+            "config": dict(workload_config(w, args), reference_step=f"{n} of {w.n_candidates} candidates"),
+            "cpu_baseline": {"value": val, "unit": "scores/s", "cores": runner.nthreads, "kind": "oracle",
+                             "sample": runner.describe(n, step_s, args.steps)},
             "e2e": {"value": val, "unit": "scores/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
 
-def make_workload(args):
-    """The named workload; with --lora R its scorer carries an adapter of rank R (alpha 32) apart from
-    the merged weights (every projection y = W x + (alpha / R) B (A x))."""
+def make_workload(args, name: str | None = None):
+    """The named workload (--workload unless `name` is given); with --lora R its scorer carries an
+    adapter of rank R (alpha 32) apart from the merged weights (every projection y = W x + (alpha / R)
+    B (A x)); with --layers N the same shapes with N layers (small profiler captures)."""
     import dataclasses
     import kvsynth as ks
-    w = ks.make_workload(args.workload)
+    w = ks.make_workload(name or args.workload)
     if args.lora:
         w.arch = dataclasses.replace(w.arch, lora_rank=args.lora)
-    if args.layers:   # the same shapes with fewer layers: small profiler captures of one layer's kernels
+    if args.layers:
         w.arch = dataclasses.replace(w.arch, n_layers=args.layers)
     return w
 
@@ -263,11 +288,15 @@ def workload_config(w, args) -> dict:
     return {"workload": w.name, "layers": a.n_layers, "d_model": a.d_model, "n_q_heads": a.n_q_heads,
             "n_kv_heads": a.n_kv_heads, "head_dim": a.head_dim, "d_ff": a.d_ff, "candidates": w.n_candidates,
             "seq_len_min": int(w.seq_lens.min()), "seq_len_max": int(w.seq_lens.max()), "page_size": a.page_size,
-            "unique_pages": int(len(set(np.concatenate([w.block_table[b, :(int(w.seq_lens[b]) + 15) // 16]
-                                                        for b in range(w.n_candidates)]).tolist()))),
+            "unique_pages": unique_pages(w),
             "l2": "inputs exceed L2 (weights + cache >> 129 MB); no flush", "parallelism": f"replicas{args.gpus}",
             **({"lora_rank": a.lora_rank, "lora_alpha": a.lora_alpha} if a.lora_rank else {}),
             **({"readout_depth": args.depth} if args.depth > 1 else {})}
+
+
+def unique_pages(w) -> int:
+    return int(len(set(np.concatenate([w.block_table[b, :(int(w.seq_lens[b]) + 15) // 16]
+                                       for b in range(w.n_candidates)]).tolist())))
 
 
 # ---------------------------------------------------------------- GPU arm
@@ -287,14 +316,16 @@ def make_scorer(dev, max_candidates: int, max_blocks: int):
     return sc
 
 
-def run_gpu(args, world, rank, local):
+def measure(w, args, world, local, steps: int, warmup: int, prof_steps: int, with_e2e: bool, clocks: bool):
+    """Time one workload: K scoring calls (kvprm_score_async, graph replay) with inputs resident in HBM,
+    then (with_e2e) the host-buffer call with the cache copied in every step, then a profiled pass
+    (per-kernel-class CUDA events, launch overlap off) and one traced call (device timeline, launch
+    overlap kept).  Returns a dict of measurements."""
     import torch
 
     import kvsynth as ks
     import paper_2607_09153_gb300 as kp
 
-    torch.cuda.set_device(local)
-    w = make_workload(args)
     tables = ks.Tables.make()
     dev = ks.DeviceInputs(w, tables)
     a = w.arch
@@ -311,72 +342,109 @@ def run_gpu(args, world, rank, local):
     def step():
         kp.kvprm_score_async(sc.ctx, pool_ptr, n_pages, bt, sl, B, d_rewards.data_ptr(), sp)
 
-    # ---- warm-up, then the device-resident timed region
-    for _ in range(args.warmup):
+    for _ in range(warmup):
         step()
     stream.synchronize()
-    clocks = ClockSampler(local)
+    clk = ClockSampler(local) if clocks else None
     barrier(world)
     torch.cuda.synchronize()
-    clocks.start()
+    if clk:
+        clk.start()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    host_s = []
     ev0.record(stream)
-    for _ in range(args.steps):
+    for _ in range(steps):
+        t0 = time.perf_counter()
         step()
+        host_s.append(time.perf_counter() - t0)
     ev1.record(stream)
     ev1.synchronize()
     torch.cuda.synchronize()
     barrier(world)
-    clk = clocks.stop()
-    ms = ev0.elapsed_time(ev1)
-    ms = max_over_ranks(ms, world)
-    value = world * B * args.steps / (ms / 1000.0)
+    clk_rec = clk.stop() if clk else None
+    ms = max_over_ranks(ev0.elapsed_time(ev1), world)
     kp.kvprm_check_device(sc.ctx)
+    out = {"ms": ms, "steps": steps, "clocks": clk_rec,
+           # host side of one call (validation, attention schedule, table upload, graph launch), measured
+           # while the GPU is busy with earlier calls
+           "host_us_per_call": round(1e6 * float(np.median(host_s)), 1)}
+    # the attention schedule alone, as the call builds it (kvprm_plan_attention, host only)
+    share = 3 if a.head_dim == 128 else 1
+    tp = time.perf_counter()
+    for _ in range(5):
+        kp.kvprm_plan_attention(w.block_table, w.seq_lens, a.n_kv_heads, a.n_q_heads // a.n_kv_heads,
+                                torch.cuda.get_device_properties(0).multi_processor_count, share | kp.KVPRM_PLAN_FUSE)
+    out["plan_us"] = round(1e6 * (time.perf_counter() - tp) / 5, 1)
 
-    # ---- end to end through the host-buffer call (cache copied H2D every step)
-    host_pool = dev.pool.cpu().pin_memory()
-    rewards = np.zeros(B, np.float32)
-    e2e_steps = max(3, args.steps // 10)
-    for _ in range(2):
-        kp.kvprm_score_host(sc.ctx, host_pool.data_ptr(), n_pages, bt, sl, B, sp, rewards)
-    barrier(world)
-    torch.cuda.synchronize()
-    t0 = time.perf_counter()
-    for _ in range(e2e_steps):
-        kp.kvprm_score_host(sc.ctx, host_pool.data_ptr(), n_pages, bt, sl, B, sp, rewards)
-    t_e2e = max_over_ranks(time.perf_counter() - t0, world)
-    e2e = {"value": world * B * e2e_steps / t_e2e, "unit": "scores/s",
-           "h2d_bytes_per_step": int(host_pool.numel() * 2 + bt.nbytes + sl.nbytes),
-           "d2h_bytes_per_step": int(B * 4 + 4), "steps": e2e_steps,
-           "path": "kvprm_score_host: pinned host cache + host tables -> rewards on host"}
-    del host_pool
+    if with_e2e:   # end to end through the host-buffer call (cache copied H2D every step)
+        host_pool = torch.empty(dev.pool.shape, dtype=dev.pool.dtype, pin_memory=True)
+        host_pool.copy_(dev.pool)
+        rewards = np.zeros(B, np.float32)
+        e2e_steps = max(3, steps // 10)
+        for _ in range(2):
+            kp.kvprm_score_host(sc.ctx, host_pool.data_ptr(), n_pages, bt, sl, B, sp, rewards)
+        barrier(world)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(e2e_steps):
+            kp.kvprm_score_host(sc.ctx, host_pool.data_ptr(), n_pages, bt, sl, B, sp, rewards)
+        t_e2e = max_over_ranks(time.perf_counter() - t0, world)
+        out["e2e"] = {"value": world * B * e2e_steps / t_e2e, "unit": "scores/s",
+                      "h2d_bytes_per_step": int(host_pool.numel() * 2 + bt.nbytes + sl.nbytes),
+                      "d2h_bytes_per_step": int(B * 4 + 4), "steps": e2e_steps,
+                      "path": "kvprm_score_host: pinned host cache + host tables -> rewards on host"}
+        del host_pool
 
-    # ---- second timed pass: per-kernel-class CUDA event times
-    prof_steps = max(3, min(args.steps, args.profile_steps))
+    # per-kernel-class CUDA event times (launch overlap off, each launch timed alone)
     kp.kvprm_set_profile(sc.ctx, True)
     for _ in range(prof_steps):
         step()
-    prof = kp.kvprm_get_profile(sc.ctx)
+    out["prof"] = kp.kvprm_get_profile(sc.ctx)
     kp.kvprm_set_profile(sc.ctx, False)
     stream.synchronize()
+    # one traced call: each launch's first-CTA start and last-CTA end with launch overlap kept
+    kp.kvprm_set_trace(sc.ctx, True)
+    step()
+    out["trace"] = kp.kvprm_get_trace(sc.ctx)
+    kp.kvprm_set_trace(sc.ctx, False)
+    stream.synchronize()
+    sc.close()
+    del dev
+    torch.cuda.empty_cache()
+    return out
 
-    launches_per_step = sum(n for n, _ in prof.values()) / prof_steps
+
+def pipelined_times(trace, n_layers: int) -> dict:
+    """Per kernel class, the time it adds to the call's timeline: from the later of its own start and
+    the previous launch's end to its own end (launch overlap kept), summed, per layer."""
+    tot = {}
+    prev_end = None
+    for cls, t0, t1 in trace:
+        begin = t0 if prev_end is None else max(t0, prev_end)
+        tot[cls] = tot.get(cls, 0.0) + max(0.0, t1 - begin)
+        prev_end = t1 if prev_end is None else max(prev_end, t1)
+    return {k: round(v / n_layers, 3) for k, v in tot.items()}
+
+
+def summarize(w, m: dict, world: int) -> dict:
+    """Rooflines and rates of one measured workload."""
+    a = w.arch
+    B = w.n_candidates
+    prof = m["prof"]
     alg = algorithmic_bytes(w)
     peaks = load_peaks()
+    prof_steps = max(1, max(n for n, _ in prof.values()) // max(1, a.n_layers)) if prof else 1
     kernels = {}
     for name, (n, tot) in prof.items():
-        if n == 0:
-            continue
-        kernels[name] = {"launches": n, "total_ms": round(tot, 4), "avg_us": round(1000 * tot / n, 3),
-                         "share": None}
-    total_ms = sum(k["total_ms"] for k in kernels.values())
+        if n:
+            kernels[name] = {"launches": n, "total_ms": round(tot, 4), "avg_us": round(1000 * tot / n, 3)}
+    total_ms = sum(k["total_ms"] for k in kernels.values()) or 1.0
     for k in kernels.values():
         k["share"] = round(k["total_ms"] / total_ms, 4)
-
-    # the attention step of a layer is one launch (private pages) or two (plus the tensor-core
-    # launch for pages that several candidates share): its time is their sum per layer
+    n_calls = prof.get("gemm_qkv", (0, 0))[0] // a.n_layers or 1
+    layers_timed = n_calls * a.n_layers
     classes = {"attention": ("attention", "attention_tc")}
-    layers_timed = prof_steps * a.n_layers
+    piped = pipelined_times(m["trace"], a.n_layers)
 
     def roof(name):
         parts = [c for c in classes.get(name, (name,)) if prof.get(c, (0, 0.0))[0] > 0]
@@ -385,44 +453,107 @@ def run_gpu(args, world, rank, local):
         per_layer = alg[name] / a.n_layers
         layer_s = tot / layers_timed / 1000.0
         ach = per_layer / layer_s / 1e9
+        pip_us = sum(piped.get(c, 0.0) for c in parts)
         return {"bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
                 "frac": round(ach / peaks["hbm_gbs"], 4), "peak_src": peaks["src"],
+                "frac_of_8tbs": round(ach / HBM_NOMINAL_GBS, 4),
                 "traffic": ncu_traffic(name, w.name) if len(parts) == 1 else None, "kernel": "+".join(parts),
                 "algorithmic_bytes_per_launch": int(per_layer), "launches_per_layer": round(n / layers_timed, 3),
-                "avg_launch_us": round(1000.0 * tot / n, 3), "time_per_layer_us": round(layer_s * 1e6, 3)}
+                "avg_launch_us": round(1000.0 * tot / n, 3), "time_per_layer_us": round(layer_s * 1e6, 3),
+                "pipelined_us_per_layer": round(pip_us, 3) if pip_us else None,
+                "pipelined_frac": round(per_layer / (pip_us * 1e-6) / 1e9 / peaks["hbm_gbs"], 4) if pip_us else None}
 
-    dominant = max((k for k in kernels if k in alg), key=lambda k: kernels[k]["total_ms"]
+    cand = [k for k in kernels if k in alg or k == "attention_tc"]
+    dominant = max((k for k in cand if k in alg), key=lambda k: kernels[k]["total_ms"]
                    + (kernels.get("attention_tc", {}).get("total_ms", 0.0) if k == "attention" else 0.0))
     attn = roof("attention")
-    # unique bytes (each referenced page once) are the roofline; logical bytes (each candidate's whole
-    # cache) are what a reader without page sharing would stream, for context on shared workloads
+    call_s = m["ms"] / m["steps"] / 1000.0
     logical = w.logical_kv_bytes()
-    attention_obj = {"achieved_gbs": attn["achieved"], "frac_of_8tbs": round(attn["achieved"] / HBM_NOMINAL_GBS, 4),
+    kv_tok = a.kv_bytes_per_token()
+    attention_obj = {"achieved_gbs": attn["achieved"], "frac_of_8tbs": attn["frac_of_8tbs"],
                      "frac_of_measured": attn["frac"], "unique_kv_bytes_per_step": alg["attention"],
                      "logical_kv_bytes_per_step": int(logical),
                      "logical_gbs": round(logical / a.n_layers / (attn["time_per_layer_us"] * 1e-6) / 1e9, 1),
-                     "time_per_layer_us": attn["time_per_layer_us"], "kernels": attn["kernel"]}
+                     "time_per_layer_us": attn["time_per_layer_us"], "kernels": attn["kernel"],
+                     "pipelined_us_per_layer": attn["pipelined_us_per_layer"],
+                     "pipelined_frac_of_8tbs": round(alg["attention"] / a.n_layers / (attn["pipelined_us_per_layer"]
+                                                      * 1e-6) / 1e9 / HBM_NOMINAL_GBS, 4)
+                     if attn["pipelined_us_per_layer"] else None}
     step_bytes = alg["call_total"]
+    return {
+        "scores_per_s": round(world * B / call_s, 2), "ms_per_call": round(call_s * 1e3, 5),
+        "us_per_call": round(call_s * 1e6, 2),
+        "kv_tokens_per_s": {"logical": round(logical / kv_tok / call_s, 1),
+                            "unique": round(alg["attention"] / kv_tok / call_s, 1)},
+        "whole_call": {"bytes_per_step": step_bytes, "achieved_gbs": round(step_bytes / call_s / 1e9, 1),
+                       "frac_of_8tbs": round(step_bytes / call_s / 1e9 / HBM_NOMINAL_GBS, 4),
+                       "frac_of_measured": round(step_bytes / call_s / 1e9 / peaks["hbm_gbs"], 4)},
+        "attention": attention_obj, "roofline": roof(dominant), "kernels": kernels,
+        "pipelined_us_per_layer": piped,
+        "host": {"us_per_call": m["host_us_per_call"], "plan_us": m["plan_us"]},
+        "launches_per_call": int(round(sum(n for n, _ in prof.values()) / max(1, n_calls))),
+        "profile_steps": prof_steps,
+    }
+
+
+OTHER_WORKLOADS = ("tiny", "qwen1p5b_b16_l2048", "beam7b_b64_p4096_s512", "mcts7b_b256_d4")
+
+
+def run_gpu(args, world, rank, local):
+    import torch
+    import kvsynth as ks
+    torch.cuda.set_device(local)
+    w = make_workload(args)
+    m = measure(w, args, world, local, args.steps, args.warmup, args.profile_steps, with_e2e=True, clocks=True)
+    sm = summarize(w, m, world)
     line = {
-        "metric": METRIC, "value": round(value, 2), "unit": "scores/s", "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 5), "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "accumulate": "f32",
+        "metric": METRIC, "value": round(world * w.n_candidates * args.steps / (m["ms"] / 1000.0), 2),
+        "unit": "scores/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(m["ms"] / args.steps, 5), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "accumulate": "f32",
         "data": "synthetic (seeded bf16 weights N(0,0.02), K/V N(0,1), random-init)",
         "config": workload_config(w, args),
-        "e2e": e2e,
-        "gpu_launches": int(round(launches_per_step)) * args.steps,
-        "roofline": roof(dominant),
-        "attention": attention_obj,
-        "whole_call": {"bytes_per_step": step_bytes,
-                       "achieved_gbs": round(step_bytes / (ms / args.steps / 1000.0) / 1e9, 1),
-                       "frac_of_8tbs": round(step_bytes / (ms / args.steps / 1000.0) / 1e9 / HBM_NOMINAL_GBS, 4)},
-        "kernels": kernels,
-        "profile_steps": prof_steps,
-        "clocks": clk,
+        "e2e": m["e2e"],
+        "gpu_launches": sm["launches_per_call"] * args.steps,
+        "roofline": sm["roofline"],
+        "attention": sm["attention"],
+        "whole_call": sm["whole_call"],
+        "kv_tokens_per_s": sm["kv_tokens_per_s"],
+        "host": sm["host"],
+        "kernels": sm["kernels"],
+        "pipelined_us_per_layer": sm["pipelined_us_per_layer"],
+        "profile_steps": sm["profile_steps"],
+        "clocks": m["clocks"],
     }
-    sc.close()
+    # the other configurations, measured the same way in the same run (shorter timed regions)
+    if world == 1 and not args.no_workloads and not args.layers and not args.lora and args.depth == 1:
+        line["workloads"] = {}
+        for name in OTHER_WORKLOADS:
+            if name == w.name:
+                continue
+            wo = make_workload(args, name)
+            mo = measure(wo, args, world, local, min(args.steps, 20), 3, 3, with_e2e=False, clocks=True)
+            so = summarize(wo, mo, world)
+            entry = {k: so[k] for k in ("scores_per_s", "ms_per_call", "kv_tokens_per_s", "whole_call", "host",
+                                        "launches_per_call")}
+            if name == "tiny":
+                entry["us_per_call"] = so["us_per_call"]
+            else:
+                entry["attention"] = {k: so["attention"][k] for k in ("achieved_gbs", "frac_of_8tbs", "frac_of_measured",
+                                                                     "time_per_layer_us", "pipelined_us_per_layer",
+                                                                     "pipelined_frac_of_8tbs", "kernels")}
+                entry["roofline"] = so["roofline"]
+            entry["config"] = workload_config(wo, args)
+            entry["clocks"] = mo["clocks"]
+            line["workloads"][name] = entry
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        tables = ks.Tables.make()
         line["cpu_baseline"] = cpu_oracle_time(w, tables, budget_s=args.cpu_budget, depth=args.depth)
+        if not args.layers and not args.lora and args.depth == 1:   # single-thread oracle on the two small configs
+            one = {}
+            for name, budget in (("tiny", 2.0), ("qwen1p5b_b16_l2048", 4.0)):
+                one[name] = cpu_oracle_time(make_workload(args, name), tables, budget_s=budget, nthreads=1)
+            line["cpu_baseline"]["single_thread"] = one
     if rank == 0:
         print(json.dumps(line), flush=True)
 
@@ -504,17 +635,21 @@ def main():
     import kvsynth as ks
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=1000)
-    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="qwen1p5b_b16_l2048", choices=list(ks.WORKLOAD_NAMES))
+    ap.add_argument("--workload", default="long8b_b8_l32768", choices=list(ks.WORKLOAD_NAMES))
+    ap.add_argument("--no-workloads", action="store_true",
+                    help="measure the --workload alone (by default the other configurations follow, shorter)")
+    ap.add_argument("--ref-step-s", type=float, default=3.0,
+                    help="reference arm: candidates per step chosen so that one step takes about this long")
     ap.add_argument("--depth", type=int, default=1,
                     help="verify tokens per candidate (depth-k readout; 1, the default: one)")
     ap.add_argument("--layers", type=int, default=0,
                     help="run the workload's shapes with this many layers (0: all; for small profiler captures)")
     ap.add_argument("--lora", type=int, default=0,
                     help="scorer adapter rank kept apart from the weights (0: merged weights, the default)")
-    ap.add_argument("--profile-steps", type=int, default=50)
+    ap.add_argument("--profile-steps", type=int, default=5)
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--attention-only", action="store_true",

@@ -49,7 +49,7 @@ class OracleCfg(ctypes.Structure):
                 ("n_kv_heads", ctypes.c_int), ("head_dim", ctypes.c_int), ("d_ff", ctypes.c_int),
                 ("rope_base", ctypes.c_double), ("rms_eps", ctypes.c_double), ("mirror", ctypes.c_int),
                 ("nthreads", ctypes.c_int), ("lora_rank", ctypes.c_int), ("lora_scale", ctypes.c_double),
-                ("depth", ctypes.c_int)]
+                ("depth", ctypes.c_int), ("qk_norm", ctypes.c_int)]
 
     @staticmethod
     def from_arch(arch, mirror: bool = True, nthreads: int | None = None, depth: int = 1) -> "OracleCfg":
@@ -57,11 +57,12 @@ class OracleCfg(ctypes.Structure):
         return OracleCfg(arch.n_layers, arch.d_model, arch.n_q_heads, arch.n_kv_heads, arch.head_dim, arch.d_ff,
                          float(arch.rope_base), float(arch.rms_eps), int(mirror),
                          int(nthreads or max(1, os.cpu_count() or 1)), rank,
-                         float(arch.lora_alpha) / rank if rank else 0.0, int(depth))
+                         float(arch.lora_alpha) / rank if rank else 0.0, int(depth),
+                         int(bool(getattr(arch, "qk_norm", False))))
 
 
 class DenseWeights(ctypes.Structure):
-    _fields_ = [("top", _u16p * 4), ("layer", ctypes.POINTER(_u16p) * 14)]
+    _fields_ = [("top", _u16p * 4), ("layer", ctypes.POINTER(_u16p) * 16)]
 
 
 class DenseKV(ctypes.Structure):
@@ -186,8 +187,8 @@ def score_synth(w, tables, cand_ids=None, mirror: bool = True, want_attn: bool =
 
 def score_dense(arch, weights: dict, kv: list, mirror: bool = True, want_attn: bool = True, want_hidden: bool = False,
                 nthreads: int | None = None, mutant: int = 0, depth: int = 1) -> Result:
-    """Score from explicit arrays.  weights = {'top': {kind: bits}, 'layers': [{kind: bits}]} (kinds 4..9, and
-    the adapter factors 10..17 when arch.lora_rank > 0);
+    """Score from explicit arrays.  weights = {'top': {kind: bits}, 'layers': [{kind: bits}]} (kinds 4..9, the
+    adapter factors 10..17 when arch.lora_rank > 0, the q/k norm gains 18, 19 when arch.qk_norm);
     kv[l][b] = (K_bits [L_b][nkv][hd], V_bits [L_b][nkv][hd])."""
     keep = []
     dw = DenseWeights()
@@ -195,7 +196,11 @@ def score_dense(arch, weights: dict, kv: list, mirror: bool = True, want_attn: b
         a, ap = _u16(weights["top"][k])
         keep.append(a)
         dw.top[k] = ap
-    kinds = range(4, 18) if getattr(arch, "lora_rank", 0) else range(4, 10)   # with an adapter: its factors too
+    kinds = list(range(4, 10))
+    if getattr(arch, "lora_rank", 0):   # with an adapter: its factors too
+        kinds += list(range(10, 18))
+    if getattr(arch, "qk_norm", False):   # with the per-head q/k norm: its gains
+        kinds += [18, 19]
     for kind in kinds:
         j = kind - 4
         ptrs = (_u16p * arch.n_layers)()

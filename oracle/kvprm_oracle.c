@@ -40,6 +40,11 @@
  *   cache and to tokens 0 .. t; the reward is read at the last one.  Internally
  *   candidate b is k rows b k + t.
  *
+ *   Per-head q/k norm (reading of the paper's Qwen3 scorers, Sec. 5 "Setup"):
+ *   with qk_norm set, each query head's and each key head's projection is
+ *   RMS-normalised over its head_dim entries, with that layer's gain vector
+ *   g_q or g_k [head_dim] (shared by all heads) and the same eps, before RoPE.
+ *
  *   Scorer adapter, Sec. 4.1 (f_{theta + Delta theta}, a LoRA adapter) and App.
  *   B.1 (rank r = 256, alpha = 32): when lora_rank > 0 each of the four
  *   projections y = W x above becomes y = W x + s B (A x) with its own factors
@@ -72,7 +77,7 @@
 /* weight kinds, as asked of the weight provider */
 enum { K_EMBED = 0, K_FINAL_NORM, K_W_PLUS, K_W_MINUS, K_ATTN_NORM, K_W_QKV, K_W_O, K_MLP_NORM, K_W_GATE_UP, K_W_DOWN,
        K_LORA_A_QKV, K_LORA_B_QKV, K_LORA_A_O, K_LORA_B_O, K_LORA_A_GATE_UP, K_LORA_B_GATE_UP, K_LORA_A_DOWN,
-       K_LORA_B_DOWN };
+       K_LORA_B_DOWN, K_Q_NORM, K_K_NORM };
 
 typedef int (*oracle_weight_fn)(void* user, int kind, int layer, uint16_t* out, int64_t n);
 typedef int (*oracle_kv_fn)(void* user, int layer, int cand, uint16_t* K, uint16_t* V, int64_t L);
@@ -85,6 +90,7 @@ typedef struct {
     int lora_rank;       /* 0: no adapter */
     double lora_scale;   /* s in y = W x + s B (A x) */
     int depth;           /* verify tokens per candidate (depth-k readout); 0 or 1: one */
+    int qk_norm;         /* 1: per-head RMSNorm of q and k before RoPE (gains K_Q_NORM, K_K_NORM) */
 } oracle_cfg;
 
 /* ------------------------------------------------------------------ numbers */
@@ -352,6 +358,7 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
     double *gu = calloc((size_t)nr * 2 * ff, 8), *a = calloc((size_t)nr * ff, 8);
     uint16_t** K = calloc((size_t)n, sizeof(uint16_t*));
     uint16_t** V = calloc((size_t)n, sizeof(uint16_t*));
+    uint16_t *gq = malloc(2 * (size_t)hd), *gk = malloc(2 * (size_t)hd);   /* q/k norm gains */
     /* adapter factors of the four projections (A [r][in], B [out][r]) and scratch */
     const int r = cfg->lora_rank;
     const int64_t in_of[4] = { d, (int64_t)nq * hd, d, ff }, out_of[4] = { qkv_rows, d, 2 * (int64_t)ff, d };
@@ -372,7 +379,7 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
         if (!lt || !ltmp) { rc = -2; goto done; }
     }
     if (!embed || !gfin || !wp || !wm || !gattn || !gmlp || !Wqkv || !Wo || !Wgu || !Wd || !h || !x || !qkv || !q ||
-        !ks || !vs || !o || !gu || !a || !K || !V) {
+        !ks || !vs || !o || !gu || !a || !K || !V || !gq || !gk) {
         rc = -2;
         goto done;
     }
@@ -393,6 +400,10 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
         if (wfn(wuser, K_ATTN_NORM, l, gattn, d) || wfn(wuser, K_W_QKV, l, Wqkv, (int64_t)qkv_rows * d) ||
             wfn(wuser, K_W_O, l, Wo, (int64_t)d * nq * hd) || wfn(wuser, K_MLP_NORM, l, gmlp, d) ||
             wfn(wuser, K_W_GATE_UP, l, Wgu, (int64_t)2 * ff * d) || wfn(wuser, K_W_DOWN, l, Wd, (int64_t)d * ff)) {
+            rc = -3;
+            goto done;
+        }
+        if (cfg->qk_norm && (wfn(wuser, K_Q_NORM, l, gq, hd) || wfn(wuser, K_K_NORM, l, gk, hd))) {
             rc = -3;
             goto done;
         }
@@ -428,10 +439,16 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
             for (int hh = 0; hh < nq; ++hh) {
                 double* qh = q + ((int64_t)i * nq + hh) * hd;
                 memcpy(qh, qr + (int64_t)hh * hd, 8 * (size_t)hd);
+#if ORACLE_MUTANT == 18 /* planted mistake: q/k norm applied after RoPE */
+                oracle_rope(qh, hd, pos, cfg->rope_base);
+                if (cfg->qk_norm) oracle_rmsnorm(qh, gq, hd, cfg->rms_eps, qh);
+#else
+                if (cfg->qk_norm) oracle_rmsnorm(qh, gq, hd, cfg->rms_eps, qh);
 #if ORACLE_MUTANT == 2 /* planted mistake: rotation in the wrong direction */
                 oracle_rope(qh, hd, -pos, cfg->rope_base);
 #else
                 oracle_rope(qh, hd, pos, cfg->rope_base);
+#endif
 #endif
                 for (int c = 0; c < hd; ++c) qh[c] = rnd(cfg, qh[c]);
             }
@@ -440,7 +457,17 @@ int oracle_score(const oracle_cfg* cfg, oracle_weight_fn wfn, void* wuser, oracl
                 double* vh = vs + ((int64_t)i * nkv + g) * hd;
                 memcpy(kh, qr + (int64_t)(nq + g) * hd, 8 * (size_t)hd);
                 memcpy(vh, qr + (int64_t)(nq + nkv + g) * hd, 8 * (size_t)hd);
+#if ORACLE_MUTANT == 19 /* planted mistake: the key norm takes the query norm's gain */
+                if (cfg->qk_norm) oracle_rmsnorm(kh, gq, hd, cfg->rms_eps, kh);
+#elif ORACLE_MUTANT == 18
+                (void)0;
+#else
+                if (cfg->qk_norm) oracle_rmsnorm(kh, gk, hd, cfg->rms_eps, kh);
+#endif
                 oracle_rope(kh, hd, pos, cfg->rope_base);
+#if ORACLE_MUTANT == 18
+                if (cfg->qk_norm) oracle_rmsnorm(kh, gk, hd, cfg->rms_eps, kh);
+#endif
                 for (int c = 0; c < hd; ++c) {
                     kh[c] = rnd(cfg, kh[c]);
                     vh[c] = rnd(cfg, vh[c]);
@@ -510,6 +537,7 @@ done:
     if (V)
         for (int i = 0; i < n; ++i) free(V[i]);
     free(K); free(V);
+    free(gq); free(gk);
     free(embed); free(gfin); free(wp); free(wm); free(gattn); free(gmlp);
     free(Wqkv); free(Wo); free(Wgu); free(Wd);
     for (int j = 0; j < 4; ++j) { free(LA[j]); free(LB[j]); }
@@ -522,11 +550,13 @@ done:
 /* Weights held in caller arrays: top[kind] for kinds 0..3, layer[kind-4][l] otherwise. */
 typedef struct {
     const uint16_t* top[4];
-    const uint16_t* const* layer[14];   /* kinds 4 .. 17 (the adapter factors may be NULL without an adapter) */
+    const uint16_t* const* layer[16];   /* kinds 4 .. 19 (adapter factors and q/k norm gains may be NULL when unused) */
 } oracle_dense_weights;
 
 int oracle_dense_weight_provider(void* user, int kind, int layer, uint16_t* out, int64_t n) {
     const oracle_dense_weights* w = (const oracle_dense_weights*)user;
+    if (kind < 0 || kind > K_K_NORM) return -1;
+    if (kind >= 4 && !w->layer[kind - 4]) return -1;
     const uint16_t* src = kind < 4 ? w->top[kind] : w->layer[kind - 4][layer];
     if (!src) return -1;
     memcpy(out, src, 2 * (size_t)n);

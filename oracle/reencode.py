@@ -8,7 +8,8 @@ decoder computes at the last position when the whole sequence
 computation of Eq. flops_forward, O(L^2)).  This module is that plain forward,
 written independently of the C oracle with PyTorch CPU library routines in
 float64 (``scaled_dot_product_attention`` with a causal mask and grouped
-heads, ``rms_norm``, ``silu``).  It returns the last position's P(+) and
+heads, ``rms_norm``, ``silu``); with ``arch.qk_norm`` each head's q and k are
+RMS-normalised (``rms_norm`` over head_dim, gains of kinds 18 and 19) before RoPE.  It returns the last position's P(+) and
 attention outputs and the per-layer key/value cache of positions < L, which is
 what a generator would have left behind.
 
@@ -81,6 +82,9 @@ def reencode(arch, weights: dict, xs: np.ndarray, mirror: bool = True, depth: in
         q = qkv[:, :nq * hd].reshape(T, nq, hd)
         k = qkv[:, nq * hd:(nq + nkv) * hd].reshape(T, nkv, hd)
         v = qkv[:, (nq + nkv) * hd:].reshape(T, nkv, hd)
+        if getattr(arch, "qk_norm", False):   # per-head RMSNorm of q and k (gains kinds 18, 19) before RoPE
+            q = F.rms_norm(q, (hd,), weight=_bits_to_f64(lw[18]), eps=arch.rms_eps)
+            k = F.rms_norm(k, (hd,), weight=_bits_to_f64(lw[19]), eps=arch.rms_eps)
         q = q * cos[:, None, :] + _rotate_half(q) * sin[:, None, :]
         k = k * cos[:, None, :] + _rotate_half(k) * sin[:, None, :]
         if mirror:

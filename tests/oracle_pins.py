@@ -190,5 +190,22 @@ def pin_depth_reencode(m=0, depth=3, lens=(0, 5, 17)):
             np.testing.assert_allclose(r.attn, attn, rtol=1e-9, atol=1e-12)
 
 
+def pin_qk_norm(m=0):
+    """With the per-head q/k RMSNorm (the paper's Qwen3 scorers) the verify-against-cache path still
+    equals the last position of the full causal re-encode, which normalises with torch's rms_norm; the
+    gains are drawn 1 + 0.2 N(0, 1), so a norm placed after RoPE or a swapped gain changes the result."""
+    import dataclasses
+    arch = dataclasses.replace(ks.ARCH_TINY, qk_norm=True)
+    for mirror in (False, True):
+        pin_reencode(m, lens=(0, 5, 17, 40), mirror=mirror, arch=arch)
+    # the norm must change the result: the same weights without it score differently
+    t = ks.Tables.make(0.2)
+    W = ks.host_weights(arch, 77, t)
+    xs = np.random.default_rng(5).normal(0, 1, (17, arch.d_model))
+    p_on, _, _ = reencode(arch, W, xs, False)
+    p_off, _, _ = reencode(ks.ARCH_TINY, W, xs, False)
+    assert abs(p_on - p_off) > 1e-6
+
+
 ALL_PINS = [pin_bf16_round, pin_rmsnorm, pin_rope, pin_attend, pin_reward, pin_reencode, pin_lora_merged,
-            pin_depth_reencode]
+            pin_depth_reencode, pin_qk_norm]

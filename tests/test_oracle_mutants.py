@@ -20,6 +20,8 @@ MUTANTS = {
     15: "adapter scale left out",
     16: "adapter term subtracted",
     17: "a verify token of a depth-k readout also sees the tokens after it",
+    18: "q/k norm applied after RoPE",
+    19: "the key norm takes the query norm's gain",
 }
 
 

@@ -33,6 +33,10 @@ def test_depth_readout_reencode(depth):
     P.pin_depth_reencode(depth=depth)
 
 
+def test_qk_norm_reencode():
+    P.pin_qk_norm()
+
+
 def test_lora_equals_merged():
     P.pin_lora_merged()
 
