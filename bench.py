@@ -307,9 +307,10 @@ def make_scorer(dev, max_candidates: int, max_blocks: int):
     wt = {"embed_verify": dev.top[ks.EMBED], "final_norm": dev.top[ks.FINAL_NORM], "w_plus": dev.top[ks.W_PLUS],
           "w_minus": dev.top[ks.W_MINUS],
           "layers": [{"attn_norm": L[ks.ATTN_NORM], "w_qkv": L[ks.W_QKV], "w_o": L[ks.W_O], "mlp_norm": L[ks.MLP_NORM],
-                      "w_gate_up": L[ks.W_GATE_UP], "w_down": L[ks.W_DOWN]} for L in dev.layers]}
+                      "w_gate_up": L[ks.W_GATE_UP], "w_down": L[ks.W_DOWN],
+                      **({"q_norm": L[ks.Q_NORM], "k_norm": L[ks.K_NORM]} if a.qk_norm else {})} for L in dev.layers]}
     sc = Scorer(a.n_layers, a.d_model, a.n_q_heads, a.n_kv_heads, a.head_dim, a.d_ff, wt, max_candidates, max_blocks,
-                a.rope_base, a.rms_eps)
+                a.rope_base, a.rms_eps, qk_norm=a.qk_norm)
     if a.lora_rank:   # the scorer adapter, kept apart from the base weights
         names = dict(zip(ks.LORA_KINDS, ("a_qkv", "b_qkv", "a_o", "b_o", "a_gate_up", "b_gate_up", "a_down", "b_down")))
         sc.set_lora(a.lora_rank, a.lora_alpha, [{names[k]: L[k] for k in ks.LORA_KINDS} for L in dev.layers])
@@ -351,12 +352,9 @@ def measure(w, args, world, local, steps: int, warmup: int, prof_steps: int, wit
     if clk:
         clk.start()
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    host_s = []
     ev0.record(stream)
     for _ in range(steps):
-        t0 = time.perf_counter()
         step()
-        host_s.append(time.perf_counter() - t0)
     ev1.record(stream)
     ev1.synchronize()
     torch.cuda.synchronize()
@@ -364,10 +362,16 @@ def measure(w, args, world, local, steps: int, warmup: int, prof_steps: int, wit
     clk_rec = clk.stop() if clk else None
     ms = max_over_ranks(ev0.elapsed_time(ev1), world)
     kp.kvprm_check_device(sc.ctx)
-    out = {"ms": ms, "steps": steps, "clocks": clk_rec,
-           # host side of one call (validation, attention schedule, table upload, graph launch), measured
-           # while the GPU is busy with earlier calls
-           "host_us_per_call": round(1e6 * float(np.median(host_s)), 1)}
+    # host side of one call (validation, attention schedule, table upload, graph launch), each call
+    # made with the GPU idle so that no wait for an earlier call's staging buffer is counted
+    host_s = []
+    for _ in range(5):
+        stream.synchronize()
+        t0 = time.perf_counter()
+        step()
+        host_s.append(time.perf_counter() - t0)
+    stream.synchronize()
+    out = {"ms": ms, "steps": steps, "clocks": clk_rec, "host_us_per_call": round(1e6 * float(np.median(host_s)), 1)}
     # the attention schedule alone, as the call builds it (kvprm_plan_attention, host only)
     share = 3 if a.head_dim == 128 else 1
     tp = time.perf_counter()

@@ -54,12 +54,17 @@ enum {
  *  {64, 128}, d_ff (SiLU-gated MLP width), page_size must be 16.
  *  rope_base: rotary base (rotate-half pairs (i, i + hd/2), angle
  *  p * base^(-2i/hd), the verify token at position p = L_b).  rms_eps: RMSNorm
- *  epsilon.  max_candidates in [1, 256]; max_blocks_per_seq = the row length of
- *  every block table passed to this context.
+ *  epsilon.  qk_norm: 0 (default) or 1 -- each query head's and key head's
+ *  projection is RMS-normalised over its head_dim entries (eps = rms_eps) with
+ *  the layer's gain vector before RoPE, as in the paper's Qwen3 scorers (Sec. 5
+ *  "Setup"); the gains are kvprm_weights.q_norm / k_norm.  max_candidates in
+ *  [1, 256]; max_blocks_per_seq = the row length of every block table passed
+ *  to this context.
  *  d_model, n_q_heads*head_dim and d_ff must be multiples of 64. */
 typedef struct {
   int32_t n_layers, d_model, n_q_heads, n_kv_heads, head_dim, d_ff, page_size;
   float rope_base, rms_eps;
+  int32_t qk_norm;
   int32_t max_candidates, max_blocks_per_seq;
 } kvprm_config;
 
@@ -74,7 +79,10 @@ typedef struct {
  *  w_o[l]       [d][n_q hd]
  *  mlp_norm[l]  [d]     pre-MLP RMSNorm gain
  *  w_gate_up[l] [2 d_ff][d]              rows: gate, then up
- *  w_down[l]    [d][d_ff]                                                   */
+ *  w_down[l]    [d][d_ff]
+ *  q_norm[l], k_norm[l] [head_dim]  per-head q / k RMSNorm gains (shared by the
+ *               heads of a layer); read only when cfg.qk_norm is set, else the
+ *               two members may be NULL                                     */
 typedef struct {
   const void* embed_verify;
   const void* final_norm;
@@ -86,6 +94,8 @@ typedef struct {
   const void* const* mlp_norm;
   const void* const* w_gate_up;
   const void* const* w_down;
+  const void* const* q_norm;
+  const void* const* k_norm;
 } kvprm_weights;
 
 typedef struct kvprm_ctx kvprm_ctx;

@@ -361,6 +361,27 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     }
     __syncthreads();   // every warp's reduced columns are in acc
     if (threadIdx.x == 0) trace_event(ts, 5);
+    // QKV with the per-head q/k RMSNorm: the factor of each (column, head of this tile) over the
+    // head's hd rows of the RMSNorm-scaled projection, 1/sqrt(mean(y^2) + eps) times the column's
+    // RMSNorm factor (v heads keep the latter alone); parked where RESID preloads its residual
+    float* qkf = hpre;   // [column][head of the tile]
+    if (ep.mode == GemmEpilogue::QKV && ep.qn_gain) {
+      const int hpt = kBM / ep.hd;   // heads per tile: 1 (hd 128) or 2 (hd 64)
+      for (int it = warp; it < nc * hpt; it += 4) {
+        const int cl = it / hpt, hh = it % hpt;
+        const float* col = acc + (cbeg + cl) * kBM + hh * ep.hd;
+        float sq = 0.f;
+        for (int r = lane; r < ep.hd; r += 32) sq += col[r] * col[r];
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) sq += __shfl_xor_sync(0xffffffffu, sq, off);
+        if (lane == 0) {
+          const float rs = ep.rs_sumsq ? rsc[cl] : 1.f;
+          const int head = m_tile * (kBM / ep.hd) + hh;
+          qkf[cl * 2 + hh] = head < ep.n_q + ep.n_kv ? rs / sqrtf(rs * rs * sq / ep.hd + ep.rs_eps) : rs;
+        }
+      }
+      __syncthreads();
+    }
     // Step 2: the epilogue over (row, column) pairs, all threads in parallel
     if (ep.mode == GemmEpilogue::PLAIN) {
       const int gm = m_tile * kBM + m;
@@ -563,6 +584,18 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       const int grow = m_tile * kBM + row_a;
       const int head = grow / hd, i = grow % hd;
       const bool rot = head < ep.n_q + ep.n_kv;
+      // per-head q/k RMSNorm: the gains of these rows (q heads: q_norm, k heads: k_norm)
+      const bool qkn = ep.qn_gain != nullptr && rot;
+      float gna[4] = {1.f, 1.f, 1.f, 1.f}, gnb[4] = {1.f, 1.f, 1.f, 1.f};
+      if (qkn) {
+        const __nv_bfloat16* gsrc = head < ep.n_q ? ep.qn_gain : ep.kn_gain;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          gna[e] = __bfloat162float(gsrc[i + e]);
+          gnb[e] = __bfloat162float(gsrc[i + half + e]);
+        }
+      }
+      const int hh_tile = row_a / hd;   // head of this tile
       auto store4 = [&](float* dst, __nv_bfloat16* dhi, __nv_bfloat16* dlo, int64_t o, const float (&x)[4]) {
         *reinterpret_cast<float4*>(dst + o) = make_float4(x[0], x[1], x[2], x[3]);
         if (dhi) {
@@ -582,7 +615,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       if (head < ep.n_q + 2 * ep.n_kv) {
 #pragma unroll 2
         for (int c = cbeg + cg; c < cend; c += 8) {
-          const float rs = ep.rs_sumsq ? rsc[c - cbeg] : 1.f;
+          const float rs = ep.qn_gain ? qkf[(c - cbeg) * 2 + hh_tile] : (ep.rs_sumsq ? rsc[c - cbeg] : 1.f);
           const float4 a4 = *reinterpret_cast<const float4*>(acc + c * kBM + row_a);
           const float4 b4 = *reinterpret_cast<const float4*>(acc + c * kBM + row_b);
           float4 r0 = make_float4(1.f, 0.f, 1.f, 0.f), r1 = r0;   // (cos, sin) of pairs i, i+1 / i+2, i+3
@@ -592,8 +625,8 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
             r1 = rp[1];
           }
           const float cs_[4] = {r0.x, r0.z, r1.x, r1.z}, sn_[4] = {r0.y, r0.w, r1.y, r1.w};
-          const float av[4] = {a4.x * rs, a4.y * rs, a4.z * rs, a4.w * rs};
-          const float bv[4] = {b4.x * rs, b4.y * rs, b4.z * rs, b4.w * rs};
+          const float av[4] = {a4.x * rs * gna[0], a4.y * rs * gna[1], a4.z * rs * gna[2], a4.w * rs * gna[3]};
+          const float bv[4] = {b4.x * rs * gnb[0], b4.y * rs * gnb[1], b4.z * rs * gnb[2], b4.w * rs * gnb[3]};
           float oa[4], ob[4];
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
@@ -627,6 +660,14 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       const int grow = m_tile * kBM + row_a;              // row of W_qkv
       const int head = grow / hd, i = grow % hd;          // i < half
       const bool rot = head < ep.n_q + ep.n_kv;   // q and k rows take RoPE, v rows do not
+      // per-head q/k RMSNorm (q heads: q_norm, k heads: k_norm gains of these two rows)
+      float gna = 1.f, gnb = 1.f;
+      if (ep.qn_gain && rot) {
+        const __nv_bfloat16* gsrc = head < ep.n_q ? ep.qn_gain : ep.kn_gain;
+        gna = __bfloat162float(gsrc[i]);
+        gnb = __bfloat162float(gsrc[i + half]);
+      }
+      const int hh_tile = row_a / hd;
       for (int c0 = cbeg + half_sel; c0 < cend; c0 += 2 * kEpiBatch) {
         // a batch's operands (accumulator pair and rotation), read before its first store
         float av[kEpiBatch], bv[kEpiBatch];
@@ -635,9 +676,9 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
         for (int k = 0; k < kEpiBatch; ++k) {
           const int c = c0 + 2 * k;
           const bool ok = c < cend;
-          const float rs = (ok && ep.rs_sumsq) ? rsc[c - cbeg] : 1.f;
-          av[k] = ok ? acc[c * kBM + row_a] * rs : 0.f;
-          bv[k] = ok ? acc[c * kBM + row_b] * rs : 0.f;
+          const float rs = !ok ? 1.f : (ep.qn_gain ? qkf[(c - cbeg) * 2 + hh_tile] : (ep.rs_sumsq ? rsc[c - cbeg] : 1.f));
+          av[k] = ok ? acc[c * kBM + row_a] * rs * gna : 0.f;
+          bv[k] = ok ? acc[c * kBM + row_b] * rs * gnb : 0.f;
           cs2[k] = (ok && rot) ? ep.rope[c * half + i] : make_float2(1.f, 0.f);
         }
 #pragma unroll

@@ -54,6 +54,11 @@ struct GemmEpilogue {
   __nv_bfloat16* q_lo = nullptr;
   float* kself = nullptr;
   float* vself = nullptr;
+  // QKV with the per-head q/k RMSNorm (when qn_gain is set): each q and k head's rows are scaled by
+  // 1/sqrt(mean over the head of y^2 + rs_eps) and the gain [hd] (q heads qn_gain, k heads kn_gain)
+  // before RoPE; y is the projection after the column's RMSNorm factor
+  const __nv_bfloat16* qn_gain = nullptr;
+  const __nv_bfloat16* kn_gain = nullptr;
   int ff = 0;            // SILU: output width; up rows start at row ff of W
   __nv_bfloat16* a_hi = nullptr;
   __nv_bfloat16* a_lo = nullptr;

@@ -67,6 +67,7 @@ struct kvprm_ctx {
   // borrowed weights
   const bf16 *embed = nullptr, *final_norm = nullptr, *w_plus = nullptr, *w_minus = nullptr;
   std::vector<const bf16*> attn_norm, mlp_norm;
+  std::vector<const bf16*> q_norm, k_norm;   // per-head q/k RMSNorm gains (cfg.qk_norm)
   std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_down;
   // depth-k readout (kvprm_set_readout_depth): verify tokens per candidate; candidate b of a call is
   // rows b depth .. b depth + depth - 1 of the batch (expanded tables below)
@@ -647,8 +648,13 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
     kvprm::GemmLowRank lr_qkv, lr_o, lr_gu, lr_down;
     int arc;
     if (lora && (arc = adapter(0, l, P.l_qkv, &ctx->tm_xhi, &ctx->tm_xlo, P.k_qkv, &lr_qkv))) return arc;
+    kvprm::GemmEpilogue eq_l = eq;   // this layer's per-head q/k RMSNorm gains, if the scorer has them
+    if (ctx->cfg.qk_norm) {
+      eq_l.qn_gain = ctx->q_norm[l];
+      eq_l.kn_gain = ctx->k_norm[l];
+    }
     LAUNCH(KVPRM_PROF_GEMM_QKV,
-           kvprm::launch_gemm(P.g_qkv, &ctx->tm_qkv[l], &ctx->tm_xhi, &ctx->tm_xlo, eq, np, ctx->err_d, st, pdl, TS,
+           kvprm::launch_gemm(P.g_qkv, &ctx->tm_qkv[l], &ctx->tm_xhi, &ctx->tm_xlo, eq_l, np, ctx->err_d, st, pdl, TS,
                               lora ? &lr_qkv : nullptr),
            "gemm_qkv");
     if (ctx->debug_flags & 2) {
@@ -896,6 +902,12 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   if (c.max_candidates < 1 || c.max_candidates > 256) return KVPRM_ECAPACITY;
   if (c.max_blocks_per_seq < 1) return KVPRM_EINVAL;
   if (!(c.rms_eps >= 0.f) || !(c.rope_base > 0.f)) return KVPRM_EINVAL;
+  if (c.qk_norm != 0 && c.qk_norm != 1) return KVPRM_EINVAL;
+  if (c.qk_norm) {
+    if (!w->q_norm || !w->k_norm) return KVPRM_EINVAL;
+    for (int l = 0; l < c.n_layers; ++l)
+      if (!w->q_norm[l] || !w->k_norm[l]) return KVPRM_EINVAL;
+  }
   if (!w->embed_verify || !w->final_norm || !w->w_plus || !w->w_minus || !w->attn_norm || !w->w_qkv || !w->w_o ||
       !w->mlp_norm || !w->w_gate_up || !w->w_down)
     return KVPRM_EINVAL;
@@ -961,6 +973,14 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   ctx->tm_o.resize(NL);
   ctx->tm_gu.resize(NL);
   ctx->tm_down.resize(NL);
+  if (c.qk_norm) {
+    ctx->q_norm.resize(NL);
+    ctx->k_norm.resize(NL);
+    for (int l = 0; l < NL; ++l) {
+      ctx->q_norm[l] = static_cast<const bf16*>(w->q_norm[l]);
+      ctx->k_norm[l] = static_cast<const bf16*>(w->k_norm[l]);
+    }
+  }
   for (int l = 0; l < NL; ++l) {
     ctx->attn_norm[l] = static_cast<const bf16*>(w->attn_norm[l]);
     ctx->mlp_norm[l] = static_cast<const bf16*>(w->mlp_norm[l]);

@@ -31,7 +31,7 @@ class KvprmConfig(ctypes.Structure):
     _fields_ = [("n_layers", ctypes.c_int32), ("d_model", ctypes.c_int32), ("n_q_heads", ctypes.c_int32),
                 ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32), ("d_ff", ctypes.c_int32),
                 ("page_size", ctypes.c_int32), ("rope_base", ctypes.c_float), ("rms_eps", ctypes.c_float),
-                ("max_candidates", ctypes.c_int32), ("max_blocks_per_seq", ctypes.c_int32)]
+                ("qk_norm", ctypes.c_int32), ("max_candidates", ctypes.c_int32), ("max_blocks_per_seq", ctypes.c_int32)]
 
 
 _VPP = ctypes.POINTER(ctypes.c_void_p)
@@ -40,7 +40,7 @@ _VPP = ctypes.POINTER(ctypes.c_void_p)
 class KvprmWeights(ctypes.Structure):
     _fields_ = [("embed_verify", ctypes.c_void_p), ("final_norm", ctypes.c_void_p), ("w_plus", ctypes.c_void_p),
                 ("w_minus", ctypes.c_void_p), ("attn_norm", _VPP), ("w_qkv", _VPP), ("w_o", _VPP),
-                ("mlp_norm", _VPP), ("w_gate_up", _VPP), ("w_down", _VPP)]
+                ("mlp_norm", _VPP), ("w_gate_up", _VPP), ("w_down", _VPP), ("q_norm", _VPP), ("k_norm", _VPP)]
 
 
 class KvprmProjectionPlan(ctypes.Structure):
@@ -342,23 +342,25 @@ class Scorer:
     """Owns a context for a scorer whose weights are torch bf16 CUDA tensors.
 
     weights = {'embed_verify', 'final_norm', 'w_plus', 'w_minus'} -> tensor, and
-    'layers' -> list of {'attn_norm', 'w_qkv', 'w_o', 'mlp_norm', 'w_gate_up', 'w_down'}."""
+    'layers' -> list of {'attn_norm', 'w_qkv', 'w_o', 'mlp_norm', 'w_gate_up', 'w_down'} (plus 'q_norm' and
+    'k_norm' with qk_norm=True)."""
 
     def __init__(self, n_layers, d_model, n_q_heads, n_kv_heads, head_dim, d_ff, weights: dict, max_candidates: int,
-                 max_blocks_per_seq: int, rope_base: float = 1e4, rms_eps: float = 1e-6):
+                 max_blocks_per_seq: int, rope_base: float = 1e4, rms_eps: float = 1e-6, qk_norm: bool = False):
         self.cfg = KvprmConfig(n_layers, d_model, n_q_heads, n_kv_heads, head_dim, d_ff, 16, rope_base, rms_eps,
-                               max_candidates, max_blocks_per_seq)
+                               int(qk_norm), max_candidates, max_blocks_per_seq)
         arr = ctypes.c_void_p * n_layers
         lay = weights["layers"]
-        self._arrays = {k: arr(*[lay[l][k].data_ptr() for l in range(n_layers)])
-                        for k in ("attn_norm", "w_qkv", "w_o", "mlp_norm", "w_gate_up", "w_down")}
+        kinds = ("attn_norm", "w_qkv", "w_o", "mlp_norm", "w_gate_up", "w_down") + (("q_norm", "k_norm") if qk_norm else ())
+        self._arrays = {k: arr(*[lay[l][k].data_ptr() for l in range(n_layers)]) for k in kinds}
         self._weights = weights   # keep the tensors alive
         cast = lambda a: ctypes.cast(a, _VPP)  # noqa: E731
         self.w = KvprmWeights(weights["embed_verify"].data_ptr(), weights["final_norm"].data_ptr(),
                               weights["w_plus"].data_ptr(), weights["w_minus"].data_ptr(),
                               cast(self._arrays["attn_norm"]), cast(self._arrays["w_qkv"]), cast(self._arrays["w_o"]),
                               cast(self._arrays["mlp_norm"]), cast(self._arrays["w_gate_up"]),
-                              cast(self._arrays["w_down"]))
+                              cast(self._arrays["w_down"]), cast(self._arrays["q_norm"]) if qk_norm else None,
+                              cast(self._arrays["k_norm"]) if qk_norm else None)
         self.ctx = kvprm_create(self.cfg, self.w)
 
     def set_depth(self, depth: int) -> None:

@@ -25,9 +25,10 @@ def make_scorer(dev: ks.DeviceInputs, max_candidates: int, max_blocks: int):
     wt = {"embed_verify": dev.top[ks.EMBED], "final_norm": dev.top[ks.FINAL_NORM], "w_plus": dev.top[ks.W_PLUS],
           "w_minus": dev.top[ks.W_MINUS],
           "layers": [{"attn_norm": L[ks.ATTN_NORM], "w_qkv": L[ks.W_QKV], "w_o": L[ks.W_O], "mlp_norm": L[ks.MLP_NORM],
-                      "w_gate_up": L[ks.W_GATE_UP], "w_down": L[ks.W_DOWN]} for L in dev.layers]}
+                      "w_gate_up": L[ks.W_GATE_UP], "w_down": L[ks.W_DOWN],
+                      **({"q_norm": L[ks.Q_NORM], "k_norm": L[ks.K_NORM]} if a.qk_norm else {})} for L in dev.layers]}
     sc = Scorer(a.n_layers, a.d_model, a.n_q_heads, a.n_kv_heads, a.head_dim, a.d_ff, wt, max_candidates, max_blocks,
-                a.rope_base, a.rms_eps)
+                a.rope_base, a.rms_eps, qk_norm=a.qk_norm)
     if a.lora_rank:   # the scorer adapter, kept apart from the weights
         names = dict(zip(ks.LORA_KINDS, ("a_qkv", "b_qkv", "a_o", "b_o", "a_gate_up", "b_gate_up", "a_down", "b_down")))
         sc.set_lora(a.lora_rank, a.lora_alpha, [{names[k]: L[k] for k in ks.LORA_KINDS} for L in dev.layers])

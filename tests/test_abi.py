@@ -36,3 +36,17 @@ def test_no_oracle_in_product():
                 text = open(os.path.join(dirpath, f)).read()
                 assert "import oracle" not in text and "from oracle" not in text, f
                 assert "kvprm_oracle" not in text, f
+
+
+def test_create_rejects_bad_qk_norm():
+    """Host-side validation of the q/k norm flag happens before any device call."""
+    L = kp.lib()
+    one = (ctypes.c_void_p * 1)(0x1000)
+    for flag, qn in ((1, None), (2, one), (-1, one)):
+        cfg = kp.KvprmConfig(1, 256, 4, 2, 64, 1024, 16, 1e4, 1e-6, flag, 4, 8)
+        cast = lambda a: ctypes.cast(a, kp.kvprm._VPP) if a is not None else None  # noqa: E731
+        w = kp.KvprmWeights(0x1000, 0x1000, 0x1000, 0x1000, cast(one), cast(one), cast(one), cast(one), cast(one),
+                            cast(one), cast(qn), cast(qn))
+        ctx = ctypes.c_void_p()
+        assert L.kvprm_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(ctx)) == kp.KVPRM_EINVAL
+        assert not ctx.value

@@ -327,3 +327,25 @@ def test_lora_with_depth_readout():
     r, attn, dev, sc = run_gpu(w, t, depth=3)
     compare(w, t, gpu_rewards=r, gpu_attn=attn, label="adapter r=64 with depth 3", depth=3)
     sc.close()
+
+
+# ---------------------------------------------------------------- per-head q/k RMSNorm (kvprm_config.qk_norm)
+def _qk(arch):
+    import dataclasses
+    return dataclasses.replace(arch, qk_norm=True)
+
+
+@pytest.mark.parametrize("make", [
+    lambda: ks.distinct("qkn_tiny", _qk(ks.ARCH_TINY), 401, [0, 5, 128, 333], gain_std=0.2),     # hd 64, two heads a tile
+    lambda: ks.distinct("qkn_15", _qk(ks.Arch(2, 1536, 12, 2, 128, 8960)), 402, [2048] * 16, gain_std=0.2),
+    lambda: ks.shared_prefix("qkn_7b", _qk(ks.Arch(2, 3584, 28, 4, 128, 18944)), 403, 64, 256, 20, gain_std=0.2),
+])
+def test_qk_norm(make):
+    """The paper's Qwen3 scorers normalise each q and k head before RoPE (Sec. 5 "Setup"): the QKV
+    epilogue's per-head RMSNorm (small- and large-batch kernel images) against the oracle's."""
+    t = ks.Tables.make(0.2)
+    w = make()
+    r, attn, dev, sc = run_gpu(w, t)
+    ids = None if w.n_candidates <= 16 else [0, 1, 31, 63]
+    compare(w, t, cand_ids=ids, gpu_rewards=r, gpu_attn=attn, label=f"qk_norm {w.name}")
+    sc.close()
