@@ -207,5 +207,106 @@ def pin_qk_norm(m=0):
     assert abs(p_on - p_off) > 1e-6
 
 
+# ---------------------------------------------------------------- KV Steering gradient (oracle/kvgrad.py)
+def _grad_case(seed=91, lens=(20, 7), arch=None):
+    """Tiny scorer with random gains and a random bf16 cache of the given lengths per candidate."""
+    arch = arch or ks.ARCH_TINY
+    t = ks.Tables.make(0.2)
+    W = ks.host_weights(arch, seed, t)
+    rng = np.random.default_rng(seed)
+    kv = [[(ks.f64_to_bf16_bits(rng.normal(0, 1, (L, arch.n_kv_heads, arch.head_dim))),
+            ks.f64_to_bf16_bits(rng.normal(0, 1, (L, arch.n_kv_heads, arch.head_dim)))) for L in lens]
+          for _ in range(arch.n_layers)]
+    return arch, W, kv
+
+
+def pin_grad_forward(m=0):
+    """The gradient oracle's own forward gives the C oracle's P(+) (two independent restatements of
+    Eq. score)."""
+    from oracle import kvgrad
+    arch, W, kv = _grad_case()
+    p, _, _ = kvgrad.score_grad(arch, W, kv, mutant=m if m >= 21 else 0)
+    r = oracle.score_dense(arch, W, kv, mirror=False, mutant=m if m < 21 else 0)
+    np.testing.assert_allclose(p, r.p_plus, rtol=0, atol=1e-12)
+
+
+def pin_grad_fd(m=0):
+    """Central finite differences of l = -log P(+) at sampled cached keys and values of every layer
+    (steps of 1e-4 in fp64: truncation error ~1e-9 relative) equal the analytic gradient."""
+    from oracle import kvgrad
+    arch, W, kv = _grad_case()
+    kvf = [[(kvgrad.bits_to_f64(K), kvgrad.bits_to_f64(V)) for K, V in row] for row in kv]
+    p, dK, dV = kvgrad.score_grad(arch, W, kvf, mutant=m if m >= 21 else 0)
+    rng = np.random.default_rng(3)
+    hstep = 1e-4
+    worst = 0.0
+    for _ in range(24):
+        l = int(rng.integers(arch.n_layers))
+        b = int(rng.integers(len(kvf[0])))
+        which = int(rng.integers(2))
+        A = kvf[l][b][which]
+        j, g, e = (int(rng.integers(n)) for n in A.shape)
+        vals = []
+        for sign in (1, -1):
+            A[j, g, e] += sign * hstep
+            vals.append(-np.log(kvgrad.score_grad(arch, W, kvf)[0][b]))
+            A[j, g, e] -= sign * hstep
+        fd = (vals[0] - vals[1]) / (2 * hstep)
+        an = (dK if which == 0 else dV)[l][b][j, g, e]
+        scale = max(np.abs(dK[l][b]).max(), np.abs(dV[l][b]).max())
+        worst = max(worst, abs(fd - an) / scale)
+    assert worst < 1e-6, worst
+
+
+def _torch_neg_log_p(arch, W, Ks, Vs):
+    """-log P(+) of one candidate written with torch library routines (rms_norm, softmax, silu) on
+    cache tensors Ks[l], Vs[l] [L][n_kv][hd] that may require grad."""
+    import torch.nn.functional as F
+    d, nq, nkv, hd, ff = arch.d_model, arch.n_q_heads, arch.n_kv_heads, arch.head_dim, arch.d_ff
+    f = lambda b: torch.from_numpy(ks.bf16_bits_to_f64(b))  # noqa: E731
+    L = Ks[0].shape[0]
+    inv = arch.rope_base ** (-torch.arange(0, hd, 2, dtype=torch.float64) / hd)
+    ang = torch.cat([L * inv, L * inv])
+    cos, sin = ang.cos(), ang.sin()
+    rot = lambda x: x * cos + torch.cat([-x[..., hd // 2:], x[..., :hd // 2]], -1) * sin  # noqa: E731
+    h = f(W["top"][0])
+    for l in range(arch.n_layers):
+        lw = W["layers"][l]
+        x = F.rms_norm(h, (d,), weight=f(lw[4]), eps=arch.rms_eps)
+        qkv = f(lw[5]).reshape(-1, d) @ x
+        q = rot(qkv[:nq * hd].reshape(nq, hd))
+        k = rot(qkv[nq * hd:(nq + nkv) * hd].reshape(nkv, hd))
+        v = qkv[(nq + nkv) * hd:].reshape(nkv, hd)
+        Kall = torch.cat([Ks[l], k[None]], 0)                  # [L+1][nkv][hd]
+        Vall = torch.cat([Vs[l], v[None]], 0)
+        Kg = Kall.repeat_interleave(nq // nkv, dim=1)          # [L+1][nq][hd]
+        Vg = Vall.repeat_interleave(nq // nkv, dim=1)
+        w = torch.softmax((Kg * q[None]).sum(-1) / hd ** 0.5, dim=0)   # [L+1][nq]
+        o = (w[..., None] * Vg).sum(0)
+        h = h + f(lw[6]).reshape(d, nq * hd) @ o.reshape(-1)
+        x = F.rms_norm(h, (d,), weight=f(lw[7]), eps=arch.rms_eps)
+        gu = f(lw[8]).reshape(2 * ff, d) @ x
+        h = h + f(lw[9]).reshape(d, ff) @ (F.silu(gu[:ff]) * gu[ff:])
+    x = F.rms_norm(h, (d,), weight=f(W["top"][1]), eps=arch.rms_eps)
+    z = torch.stack([x @ f(W["top"][3]), x @ f(W["top"][2])])
+    return -torch.log_softmax(z, 0)[1]
+
+
+def pin_grad_autograd(m=0):
+    """torch autograd through that separately written forward gives the oracle's gradient."""
+    from oracle import kvgrad
+    arch, W, kv = _grad_case(seed=92, lens=(13, 0, 33))
+    p, dK, dV = kvgrad.score_grad(arch, W, kv, mutant=m if m >= 21 else 0)
+    for b in range(len(kv[0])):
+        Ks = [torch.from_numpy(ks.bf16_bits_to_f64(kv[l][b][0])).requires_grad_() for l in range(arch.n_layers)]
+        Vs = [torch.from_numpy(ks.bf16_bits_to_f64(kv[l][b][1])).requires_grad_() for l in range(arch.n_layers)]
+        loss = _torch_neg_log_p(arch, W, Ks, Vs)
+        assert abs(loss.item() + np.log(p[b])) < 1e-12
+        loss.backward()
+        for l in range(arch.n_layers):
+            np.testing.assert_allclose(dK[l][b], Ks[l].grad.numpy(), rtol=1e-9, atol=1e-13)
+            np.testing.assert_allclose(dV[l][b], Vs[l].grad.numpy(), rtol=1e-9, atol=1e-13)
+
+
 ALL_PINS = [pin_bf16_round, pin_rmsnorm, pin_rope, pin_attend, pin_reward, pin_reencode, pin_lora_merged,
-            pin_depth_reencode, pin_qk_norm]
+            pin_depth_reencode, pin_qk_norm, pin_grad_forward, pin_grad_fd, pin_grad_autograd]

@@ -22,6 +22,9 @@ MUTANTS = {
     17: "a verify token of a depth-k readout also sees the tokens after it",
     18: "q/k norm applied after RoPE",
     19: "the key norm takes the query norm's gain",
+    21: "gradient: softmax backward without its -D term",
+    22: "gradient: RoPE backward rotated the wrong way",
+    23: "gradient: RMSNorm backward without its second term",
 }
 
 

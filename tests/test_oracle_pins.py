@@ -37,6 +37,44 @@ def test_qk_norm_reencode():
     P.pin_qk_norm()
 
 
+def test_grad_forward_matches_c_oracle():
+    P.pin_grad_forward()
+
+
+def test_grad_finite_differences():
+    P.pin_grad_fd()
+
+
+def test_grad_autograd():
+    P.pin_grad_autograd()
+
+
+def test_steer_step_lowers_each_loss():
+    """One step of KV Steering (App. C) with the cache kept in bf16 lowers -log P(+) of every candidate
+    with a distinct cache, and a shared page takes the summed gradient of the candidates reading it."""
+    from oracle import kvgrad
+    arch, W, kv = P._grad_case(seed=93, lens=(40, 25, 64))
+    _, dK, dV = kvgrad.score_grad(arch, W, kv)
+    gmax = max(max(np.abs(dK[l][b]).max(), np.abs(dV[l][b]).max()) for l in range(2) for b in range(3))
+    eta = 0.05 / gmax
+    kv2, hist = kvgrad.steer(arch, W, kv, eta, 1)
+    assert (hist[1] > hist[0]).all(), hist
+    # every updated value is a bf16 value
+    for l in range(arch.n_layers):
+        for b in range(3):
+            for A in kv2[l][b]:
+                assert np.array_equal(kvgrad.round_bf16(A), A)
+    # a shared prefix: the steered pages are identical for every candidate reading them
+    w = ks.shared_prefix("steer_pin", arch, 94, 3, 32, 9)
+    t = ks.Tables.make(0.2)
+    Wt = ks.host_weights(arch, w.seed, t)
+    kvw = [[ks.host_kv_logical(w, l, b, t) for b in range(3)] for l in range(arch.n_layers)]
+    kv3, hist3 = kvgrad.steer(arch, Wt, kvw, 0.5, 1, shared=w)
+    for l in range(arch.n_layers):
+        for b in (1, 2):
+            assert np.array_equal(kv3[l][b][0][:32], kv3[l][0][0][:32])
+
+
 def test_lora_equals_merged():
     P.pin_lora_merged()
 
