@@ -503,6 +503,45 @@ def summarize(w, m: dict, world: int) -> dict:
 OTHER_WORKLOADS = ("tiny", "qwen1p5b_b16_l2048", "beam7b_b64_p4096_s512", "mcts7b_b256_d4")
 
 
+def measure_steering(args, name: str, calls: int = 5) -> dict:
+    """KV Steering's gradient (kvprm_score_grad: the forward with its intermediates kept, then the
+    backward into every referenced page) on one workload: blocking calls timed on the host clock.
+    Algorithmic bytes per call: the weights twice (forward, then their transposes), the unique K/V
+    twice (forward and backward reads) and the gradient written in fp32 (twice the K/V bytes)."""
+    import torch
+
+    import kvsynth as ks
+    import paper_2607_09153_gb300 as kp
+    w = make_workload(args, name)
+    t = ks.Tables.make()
+    dev = ks.DeviceInputs(w, t)
+    sc = make_scorer(dev, w.n_candidates, w.max_blocks)
+    grad = torch.empty(dev.pool.shape, dtype=torch.float32, device="cuda")
+    st = torch.cuda.current_stream().cuda_stream
+    args_ = (sc.ctx, dev.pool.data_ptr(), dev.n_pages, w.block_table, w.seq_lens, w.n_candidates, grad.data_ptr(), st)
+    t0 = time.perf_counter()
+    kp.kvprm_score_grad(*args_)   # the first call also builds the transposed weights
+    first_s = time.perf_counter() - t0
+    kp.kvprm_score_grad(*args_)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(calls):
+        kp.kvprm_score_grad(*args_)
+    call_s = (time.perf_counter() - t0) / calls
+    alg = algorithmic_bytes(w)
+    step_bytes = 2 * alg["weights_total"] + 4 * alg["attention"]
+    peaks = load_peaks()
+    sc.close()
+    del grad, dev
+    torch.cuda.empty_cache()
+    return {"workload": name, "entry_point": "kvprm_score_grad", "grad_calls_per_s": round(1.0 / call_s, 2),
+            "ms_per_call": round(call_s * 1e3, 3), "first_call_ms": round(first_s * 1e3, 1),
+            "algorithmic_bytes_per_call": int(step_bytes),
+            "achieved_gbs": round(step_bytes / call_s / 1e9, 1),
+            "frac_of_measured": round(step_bytes / call_s / 1e9 / peaks["hbm_gbs"], 4), "calls": calls,
+            "timing": "blocking calls on the host clock (the call synchronises)"}
+
+
 def run_gpu(args, world, rank, local):
     import torch
     import kvsynth as ks
@@ -550,6 +589,8 @@ def run_gpu(args, world, rank, local):
             entry["config"] = workload_config(wo, args)
             entry["clocks"] = mo["clocks"]
             line["workloads"][name] = entry
+        if not args.no_steering:
+            line["steering"] = measure_steering(args, "qwen1p5b_b16_l2048")
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         tables = ks.Tables.make()
         line["cpu_baseline"] = cpu_oracle_time(w, tables, budget_s=args.cpu_budget, depth=args.depth)
@@ -656,6 +697,7 @@ def main():
     ap.add_argument("--profile-steps", type=int, default=5)
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-steering", action="store_true", help="skip the KV Steering gradient measurement")
     ap.add_argument("--attention-only", action="store_true",
                     help="time the paged attention alone on one layer of the workload's cache")
     args = ap.parse_args()

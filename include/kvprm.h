@@ -399,6 +399,47 @@ KVPRM_API int kvprm_plan_projection(int32_t M, int32_t K, int32_t n_pad, int32_t
  * Synchronises the context's last stream. */
 KVPRM_API int kvprm_check_device(kvprm_ctx* ctx);
 
+/* KV Steering (Sec. 6 "Discussion on Broader Applications"; App. C, Algorithm
+ * "KV Steering at agent handoff"): KV-PRM's score is differentiable in the
+ * cache, so the cache can be refined by gradient steps on l = -log P(+).
+ *
+ * kvprm_score_grad scores the candidates as kvprm_score does (rewards, host
+ * float [n_candidates], P(+)) and writes the gradient of the batch's loss
+ * sum_b -log P(+)_b with respect to every cached key and value:
+ *  d_grad  device float, the kv_pages layout [N_L][n_pages][2][n_kv_heads][16]
+ *          [head_dim] (16-byte aligned): for every page some candidate's block
+ *          table references, in every layer, dl/dK and dl/dV of its 16 slots
+ *          (slots past a candidate's length in its last page: 0; a page several
+ *          candidates read holds the sum of their gradients).  Pages no
+ *          candidate references are not written.
+ * The backward pass runs the verify-token forward with its intermediates
+ * kept, then the chain rule in reverse: each projection's transposed product
+ * on the forward's tensor-core GEMM, the attention read-out's backward over
+ * the pages (w_j = softmax weight, ds_j = w_j (do . V_j - do . o),
+ * dK_j += ds_j q / sqrt(hd), dV_j += w_j do), RoPE and RMSNorm backward.  The
+ * first call on a context builds library-owned transposed copies of the four
+ * projection matrices of every layer (as much device memory as the weights)
+ * and buffers for the intermediates (sized for max_candidates).
+ * Scope: merged weights (no kvprm_set_lora adapter), readout depth 1, qk_norm
+ * 0; otherwise KVPRM_EUNSUPPORTED.  Other errors as kvprm_score, KVPRM_ENOMEM.
+ * Blocking.  The caller's pages are only read.
+ *
+ * kvprm_steer runs `steps` steps of the algorithm on a caller-owned copy of the
+ * cache, kv_pages (device bf16, kvprm_score's layout, READ AND WRITTEN): each
+ * step takes the gradient at the current pages and sets every referenced
+ * page's keys and values to RNE_bf16(kv - eta * grad) (the cache stays bf16,
+ * the paper's precision); a page several candidates read takes their summed
+ * gradient once.  p_first / p_last (host float [n_candidates], may be NULL):
+ * P(+) before the first step and after the last.  Uses a library-owned fp32
+ * gradient buffer of the pool's size.  Same scope and errors as
+ * kvprm_score_grad; steps >= 0 (0 scores only).  Blocking. */
+KVPRM_API int kvprm_score_grad(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const int32_t* block_table,
+                               const int32_t* seq_lens, int32_t n_candidates, float* d_grad, float* rewards,
+                               void* stream);
+KVPRM_API int kvprm_steer(kvprm_ctx* ctx, void* kv_pages, int64_t n_pages, const int32_t* block_table,
+                          const int32_t* seq_lens, int32_t n_candidates, float eta, int32_t steps, float* p_first,
+                          float* p_last, void* stream);
+
 /* Failure-detection test hooks (no counterpart in the paper: they let tests
  * drive the error paths on the host, without faulting or hanging a GPU).
  *  kvprm_debug_set_alloc_limit: from now on the library may allocate at most

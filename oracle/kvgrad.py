@@ -62,16 +62,6 @@ def round_bf16(x: np.ndarray) -> np.ndarray:
     return np.ldexp(np.rint(m * 256.0) / 256.0, e)
 
 
-def _rmsnorm(h, g, eps):
-    r = 1.0 / np.sqrt(np.mean(h * h) + eps)
-    return h * r * g, r
-
-
-def _rmsnorm_back(h, g, r, dy):
-    """Gradient of y = h r g (r = (mean h^2 + eps)^-1/2) with respect to h."""
-    return r * (g * dy) - h * (r ** 3) * np.dot(g * dy, h) / h.size
-
-
 def _rope_angles(pos, hd, base):
     i = np.arange(hd // 2, dtype=np.float64)
     ang = pos * base ** (-2.0 * i / hd)
@@ -105,13 +95,25 @@ def _as_f64(a):
     return bits_to_f64(a) if a.dtype == np.uint16 else a.astype(np.float64)
 
 
+def _layer(arch, L):
+    """One layer's matrices as float64 (converted when needed, so that a full-size model need not be
+    held in float64 at once)."""
+    d, nq, nkv, hd, ff = arch.d_model, arch.n_q_heads, arch.n_kv_heads, arch.head_dim, arch.d_ff
+    return {ATTN_NORM: bits_to_f64(L[ATTN_NORM]), MLP_NORM: bits_to_f64(L[MLP_NORM]),
+            W_QKV: bits_to_f64(L[W_QKV]).reshape((nq + 2 * nkv) * hd, d),
+            W_O: bits_to_f64(L[W_O]).reshape(d, nq * hd),
+            W_GATE_UP: bits_to_f64(L[W_GATE_UP]).reshape(2 * ff, d),
+            W_DOWN: bits_to_f64(L[W_DOWN]).reshape(d, ff)}
+
+
 def score_grad(arch, weights: dict, kv: list, mutant: int = 0):
     """P(+), l = -log P(+) and dl/dK, dl/dV for every candidate.
 
     weights = {'top': {kind: bf16 bits}, 'layers': [{kind: bf16 bits}]}; kv[l][b] = (K, V), each
     [L_b][n_kv][hd] as bf16 bits or float64 values.  Returns (p_plus [n], dK, dV) with dK[l][b] and
     dV[l][b] float64 [L_b][n_kv][hd] (candidate b's logical positions; the caller adds the
-    contributions of candidates that share a page).
+    contributions of candidates that share a page).  The candidates' rows go through each projection
+    together (one matrix product per step); the attention read-out runs per candidate and head.
     mutant > 0 plants one mistake in the reverse pass (used only by the tests of the pins):
     21 drops the -D term of the softmax backward, 22 rotates the RoPE backward the wrong way,
     23 drops the second term of the RMSNorm backward."""
@@ -121,90 +123,95 @@ def score_grad(arch, weights: dict, kv: list, mutant: int = 0):
     eps = arch.rms_eps
     n = len(kv[0])
     top = {k: bits_to_f64(v) for k, v in weights["top"].items()}
-    lays = [{k: bits_to_f64(v) for k, v in L.items() if k in (ATTN_NORM, W_QKV, W_O, MLP_NORM, W_GATE_UP, W_DOWN)}
-            for L in weights["layers"]]
-    for l in range(NL):
-        lays[l][W_QKV] = lays[l][W_QKV].reshape((nq + 2 * nkv) * hd, d)
-        lays[l][W_O] = lays[l][W_O].reshape(d, nq * hd)
-        lays[l][W_GATE_UP] = lays[l][W_GATE_UP].reshape(2 * ff, d)
-        lays[l][W_DOWN] = lays[l][W_DOWN].reshape(d, ff)
     scale = 1.0 / np.sqrt(hd)
-    p_plus = np.empty(n)
-    dK = [[None] * n for _ in range(NL)]
-    dV = [[None] * n for _ in range(NL)]
-    for b in range(n):
-        Ks = [_as_f64(kv[l][b][0]).reshape(-1, nkv, hd) for l in range(NL)]
-        Vs = [_as_f64(kv[l][b][1]).reshape(-1, nkv, hd) for l in range(NL)]
-        L = Ks[0].shape[0]
-        c, s = _rope_angles(float(L), hd, arch.rope_base)
-        # ---------------- forward, every intermediate kept
-        h = top[EMBED].copy()
-        save = []
-        for l in range(NL):
-            P = lays[l]
-            x1, r1 = _rmsnorm(h, P[ATTN_NORM], eps)
-            qkv = P[W_QKV] @ x1
-            q = _rope(qkv[:nq * hd].reshape(nq, hd), c, s)
-            ks = _rope(qkv[nq * hd:(nq + nkv) * hd].reshape(nkv, hd), c, s)
-            vs = qkv[(nq + nkv) * hd:].reshape(nkv, hd)
-            o = np.empty((nq, hd))
-            w_all = np.empty((nq, L + 1))
+    Ks = [[_as_f64(kv[l][b][0]).reshape(-1, nkv, hd) for b in range(n)] for l in range(NL)]
+    Vs = [[_as_f64(kv[l][b][1]).reshape(-1, nkv, hd) for b in range(n)] for l in range(NL)]
+    lens = [Ks[0][b].shape[0] for b in range(n)]
+    cs = [_rope_angles(float(L), hd, arch.rope_base) for L in lens]
+    c = np.stack([x[0] for x in cs])[:, None, :]   # [n][1][hd/2]
+    s = np.stack([x[1] for x in cs])[:, None, :]
+
+    def rms(h, g):   # rows of h
+        r = 1.0 / np.sqrt(np.mean(h * h, axis=1) + eps)
+        return h * r[:, None] * g, r
+
+    def rms_back(h, g, r, dy):
+        return r[:, None] * (g * dy) - h * (r ** 3)[:, None] * np.sum(g * dy * h, axis=1)[:, None] / d
+
+    # ---------------- forward, every intermediate kept
+    h = np.tile(top[EMBED], (n, 1))
+    save = []
+    for l in range(NL):
+        P = _layer(arch, weights["layers"][l])
+        x1, r1 = rms(h, P[ATTN_NORM])
+        qkv = x1 @ P[W_QKV].T
+        q = _rope(qkv[:, :nq * hd].reshape(n, nq, hd), c, s)
+        ks = _rope(qkv[:, nq * hd:(nq + nkv) * hd].reshape(n, nkv, hd), c, s)
+        vs = qkv[:, (nq + nkv) * hd:].reshape(n, nkv, hd)
+        o = np.empty((n, nq, hd))
+        w_all = []
+        for b in range(n):
+            wb = np.empty((nq, lens[b] + 1))
             for hh in range(nq):
                 g = hh // G
-                sc = np.concatenate([Ks[l][:, g, :] @ q[hh], [ks[g] @ q[hh]]]) * scale
+                sc = np.concatenate([Ks[l][b][:, g, :] @ q[b, hh], [ks[b, g] @ q[b, hh]]]) * scale
                 w = np.exp(sc - sc.max())
                 w /= w.sum()
-                w_all[hh] = w
-                o[hh] = w[:L] @ Vs[l][:, g, :] + w[L] * vs[g]
-            h_mid = h + P[W_O] @ o.reshape(-1)
-            x2, r2 = _rmsnorm(h_mid, P[MLP_NORM], eps)
-            gu = P[W_GATE_UP] @ x2
-            u, t = gu[:ff], gu[ff:]
-            h_out = h_mid + P[W_DOWN] @ (_silu(u) * t)
-            save.append((h, r1, q, ks, vs, o, w_all, h_mid, r2, u, t))
-            h = h_out
-        xf, rf = _rmsnorm(h, top[FINAL_NORM], eps)
-        z_p, z_m = top[W_PLUS] @ xf, top[W_MINUS] @ xf
-        pp = 1.0 / (1.0 + np.exp(z_m - z_p))
-        p_plus[b] = pp
-        # ---------------- reverse pass of l = -log P(+)
-        dxf = (1.0 - pp) * (top[W_MINUS] - top[W_PLUS])
-        dh = _rmsnorm_back(h, top[FINAL_NORM], rf, dxf)
-        if mutant == 23:
-            dh = rf * (top[FINAL_NORM] * dxf)
-        for l in reversed(range(NL)):
-            P = lays[l]
-            h_in, r1, q, ks, vs, o, w_all, h_mid, r2, u, t = save[l]
-            # feed-forward block
-            da = P[W_DOWN].T @ dh
-            du = da * t * _silu_prime(u)
-            dt = da * _silu(u)
-            dx2 = P[W_GATE_UP].T @ np.concatenate([du, dt])
-            dh_mid = dh + _rmsnorm_back(h_mid, P[MLP_NORM], r2, dx2)
-            # attention block
-            do = (P[W_O].T @ dh_mid).reshape(nq, hd)
-            dq = np.zeros((nq, hd))
-            dks = np.zeros((nkv, hd))
-            dvs = np.zeros((nkv, hd))
+                wb[hh] = w
+                o[b, hh] = w[:lens[b]] @ Vs[l][b][:, g, :] + w[lens[b]] * vs[b, g]
+            w_all.append(wb)
+        h_mid = h + o.reshape(n, -1) @ P[W_O].T
+        x2, r2 = rms(h_mid, P[MLP_NORM])
+        gu = x2 @ P[W_GATE_UP].T
+        u, t = gu[:, :ff], gu[:, ff:]
+        h_out = h_mid + (_silu(u) * t) @ P[W_DOWN].T
+        save.append((h, r1, q, ks, vs, o, w_all, h_mid, r2, u, t))
+        h = h_out
+    xf, rf = rms(h, top[FINAL_NORM])
+    z_p, z_m = xf @ top[W_PLUS], xf @ top[W_MINUS]
+    p_plus = 1.0 / (1.0 + np.exp(z_m - z_p))
+    # ---------------- reverse pass of sum_b -log P(+)_b
+    dxf = (1.0 - p_plus)[:, None] * (top[W_MINUS] - top[W_PLUS])[None, :]
+    dh = rms_back(h, top[FINAL_NORM], rf, dxf)
+    if mutant == 23:
+        dh = rf[:, None] * (top[FINAL_NORM] * dxf)
+    dK = [[None] * n for _ in range(NL)]
+    dV = [[None] * n for _ in range(NL)]
+    for l in reversed(range(NL)):
+        P = _layer(arch, weights["layers"][l])
+        h_in, r1, q, ks, vs, o, w_all, h_mid, r2, u, t = save[l]
+        # feed-forward block
+        da = dh @ P[W_DOWN]
+        du = da * t * _silu_prime(u)
+        dt = da * _silu(u)
+        dx2 = np.concatenate([du, dt], axis=1) @ P[W_GATE_UP]
+        dh_mid = dh + rms_back(h_mid, P[MLP_NORM], r2, dx2)
+        # attention block
+        do = (dh_mid @ P[W_O]).reshape(n, nq, hd)
+        dq = np.zeros((n, nq, hd))
+        dks = np.zeros((n, nkv, hd))
+        dvs = np.zeros((n, nkv, hd))
+        for b in range(n):
+            L = lens[b]
             gK = np.zeros((L, nkv, hd))
             gV = np.zeros((L, nkv, hd))
             for hh in range(nq):
                 g = hh // G
-                w = w_all[hh]
-                D = 0.0 if mutant == 21 else do[hh] @ o[hh]
-                dp = np.concatenate([Vs[l][:, g, :] @ do[hh], [vs[g] @ do[hh]]])
+                w = w_all[b][hh]
+                D = 0.0 if mutant == 21 else do[b, hh] @ o[b, hh]
+                dp = np.concatenate([Vs[l][b][:, g, :] @ do[b, hh], [vs[b, g] @ do[b, hh]]])
                 ds = w * (dp - D)
-                gV[:, g, :] += np.outer(w[:L], do[hh])
-                gK[:, g, :] += np.outer(ds[:L], q[hh]) * scale
-                dvs[g] += w[L] * do[hh]
-                dks[g] += ds[L] * q[hh] * scale
-                dq[hh] = (ds[:L] @ Ks[l][:, g, :] + ds[L] * ks[g]) * scale
+                gV[:, g, :] += np.outer(w[:L], do[b, hh])
+                gK[:, g, :] += np.outer(ds[:L], q[b, hh]) * scale
+                dvs[b, g] += w[L] * do[b, hh]
+                dks[b, g] += ds[L] * q[b, hh] * scale
+                dq[b, hh] = (ds[:L] @ Ks[l][b][:, g, :] + ds[L] * ks[b, g]) * scale
             dK[l][b], dV[l][b] = gK, gV
-            sn = -s if mutant == 22 else s
-            dqkv = np.concatenate([_rope_back(dq, c, sn).reshape(-1), _rope_back(dks, c, sn).reshape(-1),
-                                   dvs.reshape(-1)])
-            dx1 = P[W_QKV].T @ dqkv
-            dh = dh_mid + _rmsnorm_back(h_in, P[ATTN_NORM], r1, dx1)
+        sn = -s if mutant == 22 else s
+        dqkv = np.concatenate([_rope_back(dq, c, sn).reshape(n, -1), _rope_back(dks, c, sn).reshape(n, -1),
+                               dvs.reshape(n, -1)], axis=1)
+        dx1 = dqkv @ P[W_QKV]
+        dh = dh_mid + rms_back(h_in, P[ATTN_NORM], r1, dx1)
     return p_plus, dK, dV
 
 

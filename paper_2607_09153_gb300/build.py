@@ -13,7 +13,7 @@ CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libkvprm.so")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
-SOURCES = ["kvprm_api.cu", "gemm_tc.cu", "attention.cu", "fused.cu", "noalloc.cu"]
+SOURCES = ["kvprm_api.cu", "gemm_tc.cu", "attention.cu", "fused.cu", "noalloc.cu", "grad.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
          "--expt-relaxed-constexpr"] + ARCH

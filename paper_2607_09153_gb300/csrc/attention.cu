@@ -349,6 +349,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
         mg.o_lo[o] = __float2bfloat16_rn(out - __bfloat162float(hi));
         if (mg.out_f32) mg.out_f32[o] = out;
         if (mg.dbg) mg.dbg[o] = out;
+        if (mg.lse && d == 0) mg.lse[hq0 + r] = Mt * kLn2 + logf(den);   // scores are in log2 units
       }
       if (threadIdx.x == 0) trace_event(ts, 3);   // this rank's outputs are written
     }

@@ -21,6 +21,7 @@ namespace kvprm {
 namespace ac {
 
 constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kStateWarps = 8;   // warps whose states a private run's merge folds
 
 // A fragments of one warp's query rows.
@@ -481,6 +482,7 @@ __device__ __forceinline__ void combine_group(int tid, int b, int g, int first, 
     mg.o_lo[o] = __float2bfloat16_rn(out - __bfloat162float(hi));
     if (mg.out_f32) mg.out_f32[o] = out;
     if (mg.dbg) mg.dbg[o] = out;
+    if (mg.lse && d == 0) mg.lse[hq0 + r] = Mt * kLn2 + logf(den);   // scores are in log2 units
   }
 }
 

@@ -433,6 +433,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
               hv = make_float4(h_in[k].x + a.x, h_in[k].y + a.y, h_in[k].z + a.z, h_in[k].w + a.w);
               const int64_t o = static_cast<int64_t>(c) * ep.M + gm0;
               *reinterpret_cast<float4*>(ep.h + o) = hv;
+              if (ep.h_copy) *reinterpret_cast<float4*>(ep.h_copy + o) = hv;
               if (ep.gain_next) {
                 const float x[4] = {hv.x * g4[0], hv.y * g4[1], hv.z * g4[2], hv.w * g4[3]};
                 uint32_t hi[2], lo[2];
@@ -503,6 +504,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
               float* hp = ep.h + static_cast<int64_t>(c) * ep.M + gm;
               hv = (hpreload ? hpre[(c - cbeg) * kBM + m] : *hp) + acc[c * kBM + m];
               *hp = hv;
+              if (ep.h_copy) ep.h_copy[static_cast<int64_t>(c) * ep.M + gm] = hv;
               if (ep.gain_next)
                 store_hilo(ep.x_hi, ep.x_lo, static_cast<int64_t>(c) * ep.M + gm, hv * __bfloat162float(ep.gain_next[gm]));
             }
@@ -550,6 +552,14 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
           const int64_t o = static_cast<int64_t>(c) * ep.ff + j0;
           *reinterpret_cast<uint4*>(ep.a_hi + o) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
           *reinterpret_cast<uint4*>(ep.a_lo + o) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+          if (ep.gu_save) {   // gate and up pre-activations (after the RMSNorm factor) for a backward pass
+            float4* gs = reinterpret_cast<float4*>(ep.gu_save + static_cast<int64_t>(c) * 2 * ep.ff + j0);
+            float4* us = reinterpret_cast<float4*>(ep.gu_save + static_cast<int64_t>(c) * 2 * ep.ff + ep.ff + j0);
+            gs[0] = make_float4(g[0] * rs, g[1] * rs, g[2] * rs, g[3] * rs);
+            gs[1] = make_float4(g[4] * rs, g[5] * rs, g[6] * rs, g[7] * rs);
+            us[0] = make_float4(u[0] * rs, u[1] * rs, u[2] * rs, u[3] * rs);
+            us[1] = make_float4(u[4] * rs, u[5] * rs, u[6] * rs, u[7] * rs);
+          }
         }
       }
     } else if (ep.mode == GemmEpilogue::SILU) {
@@ -569,8 +579,13 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
 #pragma unroll
           for (int k = 0; k < kEpiBatch; ++k) {
             const int c = c0 + 2 * k;
-            if (c < cend)
-            store_hilo(ep.a_hi, ep.a_lo, static_cast<int64_t>(c) * ep.ff + j, g[k] / (1.0f + expf(-g[k])) * u[k]);
+            if (c < cend) {
+              store_hilo(ep.a_hi, ep.a_lo, static_cast<int64_t>(c) * ep.ff + j, g[k] / (1.0f + expf(-g[k])) * u[k]);
+              if (ep.gu_save) {   // gate and up pre-activations for a backward pass
+                ep.gu_save[static_cast<int64_t>(c) * 2 * ep.ff + j] = g[k];
+                ep.gu_save[static_cast<int64_t>(c) * 2 * ep.ff + ep.ff + j] = u[k];
+              }
+            }
           }
         }
     } else if (LARGE && (ep.hd & 7) == 0) {

@@ -1,0 +1,459 @@
+// Backward pass of the verify-token forward, for KV Steering (Sec. 6; App. C, Algorithm "KV Steering
+// at agent handoff"): the gradient of l = sum_b -log P(+)_b with respect to every cached key and
+// value.  The projections' transposed products run on the forward's tensor-core GEMM against
+// transposed weight copies (kvprm_api.cu); this file holds the rest:
+//   transpose       W [rows][cols] -> W^T (bf16), once per context
+//   head_back       dh = d(-log P)/dh at the final RMSNorm: dx = (1 - P)(w_- - w_+)
+//   rms_back        dh = dres + r g dy - h r^3 (sum_i g_i dy_i h_i) / d,  r = (mean h^2 + eps)^-1/2
+//   silu_back       du = da t SiLU'(u),  dt = da SiLU(u)
+//   attn_back_pre   per (candidate, kv head): D_h = do_h . o_h and the self entry's terms
+//   attn_back_pages per run of cached pages: w_j = exp(q.K_j / sqrt(hd) - lse), ds_j = w_j (do.V_j - D),
+//                   dK_j = sum_h ds_j q_h / sqrt(hd), dV_j = sum_h w_j do_h, dq_h += ds_j K_j / sqrt(hd)
+//   rope_back       the rotation by the negative angle, and [dq; dk; dv] as the next GEMM's input
+//   zero_pages      clears the gradient of pages several candidates read (they are accumulated)
+//   steer_update    kv <- RNE_bf16(kv - eta grad) on the pages the block tables reference
+// Every product runs in fp32; a gradient that feeds a tensor-core contraction is stored as a bf16
+// (hi, lo) pair like the forward's activations.
+#include <cuda_bf16.h>
+
+#include "kernels.h"
+#include "ptx.cuh"
+
+namespace kvprm {
+
+namespace {
+
+typedef __nv_bfloat16 bf16;
+
+__device__ __forceinline__ void put_hilo(bf16* hi, bf16* lo, int64_t i, float x) {
+  const bf16 h = __float2bfloat16_rn(x);
+  hi[i] = h;
+  lo[i] = __float2bfloat16_rn(x - __bfloat162float(h));
+}
+
+// two block-wide sums at once (blockDim.x a multiple of 32, <= 1024); every thread gets both
+__device__ __forceinline__ float2 block_sum2(float a, float b, float2* red) {
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    a += __shfl_xor_sync(0xffffffffu, a, off);
+    b += __shfl_xor_sync(0xffffffffu, b, off);
+  }
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31, nw = blockDim.x >> 5;
+  __syncthreads();
+  if (l == 0) red[w] = make_float2(a, b);
+  __syncthreads();
+  float2 t = make_float2(0.f, 0.f);
+  for (int i = 0; i < nw; ++i) {
+    t.x += red[i].x;
+    t.y += red[i].y;
+  }
+  return t;
+}
+
+__global__ void transpose_kernel(const bf16* __restrict__ in, bf16* __restrict__ out, int rows, int cols) {
+  __shared__ bf16 tile[32][34];
+  const int c0 = blockIdx.x * 32, r0 = blockIdx.y * 32;
+  for (int j = threadIdx.y; j < 32; j += blockDim.y) {
+    const int r = r0 + j, c = c0 + threadIdx.x;
+    if (r < rows && c < cols) tile[j][threadIdx.x] = in[static_cast<int64_t>(r) * cols + c];
+  }
+  __syncthreads();
+  for (int j = threadIdx.y; j < 32; j += blockDim.y) {
+    const int c = c0 + j, r = r0 + threadIdx.x;
+    if (c < cols && r < rows) out[static_cast<int64_t>(c) * rows + r] = tile[threadIdx.x][j];
+  }
+}
+
+// One CTA per row: the loss gradient at the final residual stream h.
+__global__ void head_back_kernel(const float* __restrict__ h, const float* __restrict__ p_plus,
+                                 const bf16* __restrict__ gain, const bf16* __restrict__ w_plus,
+                                 const bf16* __restrict__ w_minus, int d, float eps, float* __restrict__ dh,
+                                 bf16* __restrict__ dh_hi, bf16* __restrict__ dh_lo) {
+  __shared__ float2 red[32];
+  const int b = blockIdx.x;
+  const float* hb = h + static_cast<int64_t>(b) * d;
+  const float q = 1.f - p_plus[b];   // d(-log P)/dz_- = 1 - P = -d(-log P)/dz_+
+  float ss = 0.f, sd = 0.f;
+  for (int i = threadIdx.x; i < d; i += blockDim.x) {
+    const float hv = hb[i];
+    const float gdy = __bfloat162float(gain[i]) * q * (__bfloat162float(w_minus[i]) - __bfloat162float(w_plus[i]));
+    ss += hv * hv;
+    sd += gdy * hv;
+  }
+  const float2 t = block_sum2(ss, sd, red);
+  const float r = rsqrtf(t.x / d + eps);
+  const float c = r * r * r * t.y / d;
+  for (int i = threadIdx.x; i < d; i += blockDim.x) {
+    const float gdy = __bfloat162float(gain[i]) * q * (__bfloat162float(w_minus[i]) - __bfloat162float(w_plus[i]));
+    const float v = r * gdy - hb[i] * c;
+    dh[static_cast<int64_t>(b) * d + i] = v;
+    if (dh_hi) put_hilo(dh_hi, dh_lo, static_cast<int64_t>(b) * d + i, v);
+  }
+}
+
+// One CTA per row: dh = dres + RMSNorm backward of (h, gain) applied to dy (may run in place:
+// dres == out).  h_bf16 (when set) is one bf16 row shared by every row (the embedding of layer 0).
+__global__ void rms_back_kernel(const float* __restrict__ h, const bf16* __restrict__ h_bf16,
+                                const bf16* __restrict__ gain, const float* __restrict__ dy, const float* dres, int d,
+                                float eps, float* out, bf16* __restrict__ o_hi, bf16* __restrict__ o_lo) {
+  __shared__ float2 red[32];
+  const int b = blockIdx.x;
+  const int64_t row = static_cast<int64_t>(b) * d;
+  float ss = 0.f, sd = 0.f;
+  for (int i = threadIdx.x; i < d; i += blockDim.x) {
+    const float hv = h_bf16 ? __bfloat162float(h_bf16[i]) : h[row + i];
+    ss += hv * hv;
+    sd += __bfloat162float(gain[i]) * dy[row + i] * hv;
+  }
+  const float2 t = block_sum2(ss, sd, red);
+  const float r = rsqrtf(t.x / d + eps);
+  const float c = r * r * r * t.y / d;
+  for (int i = threadIdx.x; i < d; i += blockDim.x) {
+    const float hv = h_bf16 ? __bfloat162float(h_bf16[i]) : h[row + i];
+    const float v = dres[row + i] + r * __bfloat162float(gain[i]) * dy[row + i] - hv * c;
+    out[row + i] = v;
+    if (o_hi) put_hilo(o_hi, o_lo, row + i, v);
+  }
+}
+
+// da [n][ff], gu [n][2 ff] (gate then up pre-activations) -> [du; dt] [n][2 ff] as hi/lo
+__global__ void silu_back_kernel(const float* __restrict__ da, const float* __restrict__ gu, int n, int ff,
+                                 bf16* __restrict__ o_hi, bf16* __restrict__ o_lo) {
+  const int64_t total = static_cast<int64_t>(n) * ff;
+  for (int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; e < total;
+       e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t b = e / ff, j = e - b * ff;
+    const float u = gu[b * 2 * ff + j], t = gu[b * 2 * ff + ff + j];
+    const float sg = 1.f / (1.f + expf(-u));
+    const float a = da[e];
+    put_hilo(o_hi, o_lo, b * 2 * ff + j, a * t * sg * (1.f + u * (1.f - sg)));
+    put_hilo(o_hi, o_lo, b * 2 * ff + ff + j, a * u * sg);
+  }
+}
+
+// One CTA of 128 threads per (row b, kv head g): D_h = do_h . o_h for the G query heads, and the
+// verify token's own entry: w_s = exp(q_h . k_s / sqrt(hd) - lse_h), ds_s = w_s (do_h . v_s - D_h),
+// dk_s = sum_h ds_s q_h / sqrt(hd), dv_s = sum_h w_s do_h, dq_h = ds_s k_s / sqrt(hd) (the pages add on).
+__global__ void attn_back_pre_kernel(const float* __restrict__ q, const float* __restrict__ ks,
+                                     const float* __restrict__ vs, const float* __restrict__ o,
+                                     const float* __restrict__ dout, const float* __restrict__ lse, int n_q, int n_kv,
+                                     int hd, float* __restrict__ D, float* __restrict__ dq, float* __restrict__ dks,
+                                     float* __restrict__ dvs) {
+  __shared__ float s_w[kMaxGroup], s_ds[kMaxGroup];
+  const int b = blockIdx.x / n_kv, g = blockIdx.x % n_kv, G = n_q / n_kv;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const float scale = rsqrtf(static_cast<float>(hd));
+  const int64_t hk = (static_cast<int64_t>(b) * n_kv + g) * hd;
+  for (int r = warp; r < G; r += blockDim.x >> 5) {
+    const int64_t hq = (static_cast<int64_t>(b) * n_q + g * G + r) * hd;
+    float dd = 0.f, sq = 0.f, dp = 0.f;
+    for (int e = lane; e < hd; e += 32) {
+      dd += dout[hq + e] * o[hq + e];
+      sq += q[hq + e] * ks[hk + e];
+      dp += dout[hq + e] * vs[hk + e];
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      dd += __shfl_xor_sync(0xffffffffu, dd, off);
+      sq += __shfl_xor_sync(0xffffffffu, sq, off);
+      dp += __shfl_xor_sync(0xffffffffu, dp, off);
+    }
+    if (lane == 0) {
+      const int64_t row = static_cast<int64_t>(b) * n_q + g * G + r;
+      const float w = expf(sq * scale - lse[row]);
+      D[row] = dd;
+      s_w[r] = w;
+      s_ds[r] = w * (dp - dd);
+    }
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; e < hd; e += blockDim.x) {
+    float ak = 0.f, av = 0.f;
+    for (int r = 0; r < G; ++r) {
+      const int64_t hq = (static_cast<int64_t>(b) * n_q + g * G + r) * hd;
+      ak += s_ds[r] * q[hq + e];
+      av += s_w[r] * dout[hq + e];
+      dq[hq + e] = s_ds[r] * ks[hk + e] * scale;
+    }
+    dks[hk + e] = ak * scale;
+    dvs[hk + e] = av;
+  }
+}
+
+// One CTA of 4 warps per unit {b, g, j0, j1}: candidate b's logical pages j0 .. j1 - 1 of kv head g.
+// Warp w takes tokens w, w + 4, .. of each page; each lane holds HD / 32 consecutive elements of
+// the token's key and value (read straight from HBM), of the G query rows and of their output
+// gradients, so every dot product is a lane-local sum and one warp reduction.  dK and dV of a page
+// only this candidate reads are stored; of a page several read (shared[page] != 0) they are added
+// with atomics (zero_pages cleared them).  dq is summed over the CTA's warps, then added atomically.
+template <int HD, int GMAX>
+__global__ void __launch_bounds__(128) attn_back_pages_kernel(
+    const int4* __restrict__ units, const int32_t* __restrict__ seq_lens, const int32_t* __restrict__ block_table,
+    int max_blocks, const bf16* __restrict__ pool_layer, const uint8_t* __restrict__ shared, const float* __restrict__ q,
+    const float* __restrict__ dout, const float* __restrict__ lse, const float* __restrict__ D, int n_q, int n_kv,
+    float* __restrict__ grad_layer, float* __restrict__ dq) {
+  constexpr int kPer = HD / 32;   // 4 (hd 128) or 2 (hd 64)
+  __shared__ float s_dq[4][GMAX][HD];
+  const int4 u = units[blockIdx.x];
+  const int b = u.x, g = u.y, j0 = u.z, j1 = u.w;
+  const int G = n_q / n_kv;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const float scale = rsqrtf(static_cast<float>(HD));
+  const int L = seq_lens[b];
+  float qr[GMAX][kPer], dr[GMAX][kPer], acc[GMAX][kPer];
+  float lse_r[GMAX], D_r[GMAX];
+#pragma unroll
+  for (int r = 0; r < GMAX; ++r) {
+    if (r < G) {
+      const int64_t row = static_cast<int64_t>(b) * n_q + g * G + r;
+#pragma unroll
+      for (int k = 0; k < kPer; ++k) {
+        qr[r][k] = q[row * HD + lane * kPer + k];
+        dr[r][k] = dout[row * HD + lane * kPer + k];
+        acc[r][k] = 0.f;
+      }
+      lse_r[r] = lse[row];
+      D_r[r] = D[row];
+    }
+  }
+  const int64_t page_elems = static_cast<int64_t>(2) * n_kv * 16 * HD;   // one page of one layer
+  for (int j = j0; j < j1; ++j) {
+    const int32_t p = block_table[static_cast<int64_t>(b) * max_blocks + j];
+    const int valid = min(16, L - 16 * j);
+    const bf16* kp = pool_layer + p * page_elems + static_cast<int64_t>(g) * 16 * HD;
+    const bf16* vp = kp + static_cast<int64_t>(n_kv) * 16 * HD;
+    float* gk = grad_layer + p * page_elems + static_cast<int64_t>(g) * 16 * HD;
+    float* gv = gk + static_cast<int64_t>(n_kv) * 16 * HD;
+    const bool sh = shared[p] != 0;
+    for (int t = warp; t < 16; t += 4) {
+      float kf[kPer], vf[kPer];
+      if constexpr (kPer == 4) {
+        const uint2 kb = *reinterpret_cast<const uint2*>(kp + t * HD + lane * 4);
+        const uint2 vb = *reinterpret_cast<const uint2*>(vp + t * HD + lane * 4);
+        const float2 k01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kb.x));
+        const float2 k23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kb.y));
+        const float2 v01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&vb.x));
+        const float2 v23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&vb.y));
+        kf[0] = k01.x; kf[1] = k01.y; kf[2] = k23.x; kf[3] = k23.y;
+        vf[0] = v01.x; vf[1] = v01.y; vf[2] = v23.x; vf[3] = v23.y;
+      } else {
+        const uint32_t kb = *reinterpret_cast<const uint32_t*>(kp + t * HD + lane * 2);
+        const uint32_t vb = *reinterpret_cast<const uint32_t*>(vp + t * HD + lane * 2);
+        const float2 k01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kb));
+        const float2 v01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&vb));
+        kf[0] = k01.x; kf[1] = k01.y;
+        vf[0] = v01.x; vf[1] = v01.y;
+      }
+      float dk[kPer], dv[kPer];
+#pragma unroll
+      for (int k = 0; k < kPer; ++k) dk[k] = dv[k] = 0.f;
+      if (t < valid) {
+#pragma unroll
+        for (int r = 0; r < GMAX; ++r) {
+          if (r >= G) break;
+          float s = 0.f, dp = 0.f;
+#pragma unroll
+          for (int k = 0; k < kPer; ++k) {
+            s += qr[r][k] * kf[k];
+            dp += dr[r][k] * vf[k];
+          }
+#pragma unroll
+          for (int off = 16; off > 0; off >>= 1) {
+            s += __shfl_xor_sync(0xffffffffu, s, off);
+            dp += __shfl_xor_sync(0xffffffffu, dp, off);
+          }
+          const float w = expf(s * scale - lse_r[r]);
+          const float ds = w * (dp - D_r[r]);
+#pragma unroll
+          for (int k = 0; k < kPer; ++k) {
+            dk[k] += ds * scale * qr[r][k];
+            dv[k] += w * dr[r][k];
+            acc[r][k] += ds * scale * kf[k];
+          }
+        }
+      }
+      float* gkt = gk + t * HD + lane * kPer;
+      float* gvt = gv + t * HD + lane * kPer;
+      if constexpr (kPer == 4) {
+        const float4 k4 = make_float4(dk[0], dk[1], dk[2], dk[3]);
+        const float4 v4 = make_float4(dv[0], dv[1], dv[2], dv[3]);
+        if (sh) {
+          atomicAdd(reinterpret_cast<float4*>(gkt), k4);
+          atomicAdd(reinterpret_cast<float4*>(gvt), v4);
+        } else {
+          *reinterpret_cast<float4*>(gkt) = k4;
+          *reinterpret_cast<float4*>(gvt) = v4;
+        }
+      } else {
+        if (sh) {
+#pragma unroll
+          for (int k = 0; k < kPer; ++k) {
+            atomicAdd(gkt + k, dk[k]);
+            atomicAdd(gvt + k, dv[k]);
+          }
+        } else {
+          *reinterpret_cast<float2*>(gkt) = make_float2(dk[0], dk[1]);
+          *reinterpret_cast<float2*>(gvt) = make_float2(dv[0], dv[1]);
+        }
+      }
+    }
+  }
+  // dq: the four warps' sums, then one atomic add per element
+#pragma unroll
+  for (int r = 0; r < GMAX; ++r)
+    if (r < G)
+#pragma unroll
+      for (int k = 0; k < kPer; ++k) s_dq[warp][r][lane * kPer + k] = acc[r][k];
+  __syncthreads();
+  for (int i = threadIdx.x; i < G * HD; i += blockDim.x) {
+    const int r = i / HD, e = i - r * HD;
+    const float v = s_dq[0][r][e] + s_dq[1][r][e] + s_dq[2][r][e] + s_dq[3][r][e];
+    atomicAdd(dq + (static_cast<int64_t>(b) * n_q + g * G + r) * HD + e, v);
+  }
+}
+
+// One CTA per row: [dq; dk; dv] before RoPE (the rotation by the negative angle of position L_b)
+// as the bf16 hi/lo input of the W_qkv^T product, [n][(n_q + 2 n_kv) hd].
+__global__ void rope_back_kernel(const float* __restrict__ dq, const float* __restrict__ dks,
+                                 const float* __restrict__ dvs, const float2* __restrict__ rope, int n_q, int n_kv,
+                                 int hd, bf16* __restrict__ o_hi, bf16* __restrict__ o_lo) {
+  const int b = blockIdx.x, half = hd / 2;
+  const int rows = (n_q + 2 * n_kv) * hd;
+  const int64_t ob = static_cast<int64_t>(b) * rows;
+  for (int e = threadIdx.x; e < (n_q + n_kv) * half; e += blockDim.x) {
+    const int head = e / half, i = e - head * half;
+    const float* src = head < n_q ? dq + (static_cast<int64_t>(b) * n_q + head) * hd
+                                  : dks + (static_cast<int64_t>(b) * n_kv + head - n_q) * hd;
+    const float2 cs = rope[static_cast<int64_t>(b) * half + i];
+    const float da = src[i], db = src[i + half];
+    put_hilo(o_hi, o_lo, ob + head * hd + i, da * cs.x + db * cs.y);
+    put_hilo(o_hi, o_lo, ob + head * hd + i + half, db * cs.x - da * cs.y);
+  }
+  for (int e = threadIdx.x; e < n_kv * hd; e += blockDim.x)
+    put_hilo(o_hi, o_lo, ob + (n_q + n_kv) * hd + e, dvs[static_cast<int64_t>(b) * n_kv * hd + e]);
+}
+
+// Zero every layer's gradient of the listed pages.
+__global__ void zero_pages_kernel(float* __restrict__ grad, const int32_t* __restrict__ pages, int n_list,
+                                  int n_layers, int64_t n_pages, int64_t page_elems) {
+  const int64_t per = page_elems / 4;
+  const int64_t total = static_cast<int64_t>(n_list) * n_layers * per;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t e = i % per, rest = i / per;
+    const int64_t l = rest % n_layers, k = rest / n_layers;
+    float4* dst = reinterpret_cast<float4*>(grad + (l * n_pages + pages[k]) * page_elems) + e;
+    *dst = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+}
+
+// kv <- RNE_bf16(kv - eta grad) for every layer of the listed pages.
+__global__ void steer_update_kernel(bf16* __restrict__ kv, const float* __restrict__ grad,
+                                    const int32_t* __restrict__ pages, int n_list, int n_layers, int64_t n_pages,
+                                    int64_t page_elems, float eta) {
+  const int64_t per = page_elems / 4;
+  const int64_t total = static_cast<int64_t>(n_list) * n_layers * per;
+  for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t e = i % per, rest = i / per;
+    const int64_t l = rest % n_layers, k = rest / n_layers;
+    const int64_t base = (l * n_pages + pages[k]) * page_elems + 4 * e;
+    const float4 gr = *reinterpret_cast<const float4*>(grad + base);
+    uint2 raw = *reinterpret_cast<const uint2*>(kv + base);
+    const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&raw.x));
+    const float2 c = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&raw.y));
+    const __nv_bfloat162 na = __floats2bfloat162_rn(a.x - eta * gr.x, a.y - eta * gr.y);
+    const __nv_bfloat162 nc = __floats2bfloat162_rn(c.x - eta * gr.z, c.y - eta * gr.w);
+    raw.x = *reinterpret_cast<const uint32_t*>(&na);
+    raw.y = *reinterpret_cast<const uint32_t*>(&nc);
+    *reinterpret_cast<uint2*>(kv + base) = raw;
+  }
+}
+
+unsigned grid_1d(int64_t total, int threads) {
+  int64_t b = (total + threads - 1) / threads;
+  if (b > 152 * 16) b = 152 * 16;
+  return static_cast<unsigned>(b < 1 ? 1 : b);
+}
+
+}  // namespace
+
+cudaError_t launch_transpose(const __nv_bfloat16* in, __nv_bfloat16* out, int rows, int cols, cudaStream_t st) {
+  const dim3 grid((cols + 31) / 32, (rows + 31) / 32);
+  if (grid.y > 65535u) return cudaErrorInvalidValue;
+  transpose_kernel<<<grid, dim3(32, 8), 0, st>>>(in, out, rows, cols);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_head_back(const float* h, const float* p_plus, const __nv_bfloat16* gain,
+                             const __nv_bfloat16* w_plus, const __nv_bfloat16* w_minus, int n, int d, float eps,
+                             float* dh, __nv_bfloat16* dh_hi, __nv_bfloat16* dh_lo, cudaStream_t st) {
+  head_back_kernel<<<n, 256, 0, st>>>(h, p_plus, gain, w_plus, w_minus, d, eps, dh, dh_hi, dh_lo);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rms_back(const float* h, const __nv_bfloat16* h_bf16, const __nv_bfloat16* gain, const float* dy,
+                            const float* dres, int n, int d, float eps, float* out, __nv_bfloat16* o_hi,
+                            __nv_bfloat16* o_lo, cudaStream_t st) {
+  rms_back_kernel<<<n, 256, 0, st>>>(h, h_bf16, gain, dy, dres, d, eps, out, o_hi, o_lo);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_silu_back(const float* da, const float* gu, int n, int ff, __nv_bfloat16* o_hi,
+                             __nv_bfloat16* o_lo, cudaStream_t st) {
+  silu_back_kernel<<<grid_1d(static_cast<int64_t>(n) * ff, 256), 256, 0, st>>>(da, gu, n, ff, o_hi, o_lo);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_attn_back(const AttnBackArgs& a, cudaStream_t st) {
+  if (a.n_q / a.n_kv > kMaxGroup || (a.hd != 64 && a.hd != 128)) return cudaErrorInvalidValue;
+  attn_back_pre_kernel<<<a.n * a.n_kv, 128, 0, st>>>(a.q, a.kself, a.vself, a.o, a.dout, a.lse, a.n_q, a.n_kv, a.hd,
+                                                     a.D, a.dq, a.dks, a.dvs);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess || a.n_units == 0) return e;
+  const int G = a.n_q / a.n_kv;
+  auto go = [&](auto kern) {
+    kern<<<a.n_units, 128, 0, st>>>(a.units, a.seq_lens, a.block_table, a.max_blocks, a.pool_layer, a.shared, a.q,
+                                    a.dout, a.lse, a.D, a.n_q, a.n_kv, a.grad_layer, a.dq);
+  };
+  if (a.hd == 128) {
+    if (G <= 4)
+      go(attn_back_pages_kernel<128, 4>);
+    else if (G <= 8)
+      go(attn_back_pages_kernel<128, 8>);
+    else
+      go(attn_back_pages_kernel<128, 16>);
+  } else {
+    if (G <= 4)
+      go(attn_back_pages_kernel<64, 4>);
+    else if (G <= 8)
+      go(attn_back_pages_kernel<64, 8>);
+    else
+      go(attn_back_pages_kernel<64, 16>);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_rope_back(const float* dq, const float* dks, const float* dvs, const float2* rope, int n, int n_q,
+                             int n_kv, int hd, __nv_bfloat16* o_hi, __nv_bfloat16* o_lo, cudaStream_t st) {
+  rope_back_kernel<<<n, 256, 0, st>>>(dq, dks, dvs, rope, n_q, n_kv, hd, o_hi, o_lo);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_zero_pages(float* grad, const int32_t* pages, int n_list, int n_layers, int64_t n_pages,
+                              int64_t page_elems, cudaStream_t st) {
+  if (n_list == 0) return cudaSuccess;
+  zero_pages_kernel<<<grid_1d(static_cast<int64_t>(n_list) * n_layers * (page_elems / 4), 256), 256, 0, st>>>(
+      grad, pages, n_list, n_layers, n_pages, page_elems);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_steer_update(__nv_bfloat16* kv, const float* grad, const int32_t* pages, int n_list, int n_layers,
+                                int64_t n_pages, int64_t page_elems, float eta, cudaStream_t st) {
+  if (n_list == 0) return cudaSuccess;
+  steer_update_kernel<<<grid_1d(static_cast<int64_t>(n_list) * n_layers * (page_elems / 4), 256), 256, 0, st>>>(
+      kv, grad, pages, n_list, n_layers, n_pages, page_elems, eta);
+  return cudaGetLastError();
+}
+
+}  // namespace kvprm

@@ -42,6 +42,11 @@ struct GemmEpilogue {
   const __nv_bfloat16* gain_next = nullptr;
   __nv_bfloat16* x_hi = nullptr;
   __nv_bfloat16* x_lo = nullptr;
+  // RESID: when set, the new h is also written here ([n][M]; kept for a backward pass)
+  float* h_copy = nullptr;
+  // SILU: when set, the gate and up pre-activations (after the RMSNorm factor) as [n][2 ff]: gate
+  // columns, then up (kept for a backward pass)
+  float* gu_save = nullptr;
   // QKV, SILU: when set, the input was h ⊙ gain and the accumulator is scaled
   // per candidate by the RMSNorm factor 1/sqrt(sum_t rs_sumsq[t][n] / rs_d + rs_eps)
   const float* rs_sumsq = nullptr;
@@ -177,6 +182,9 @@ struct AttnMerge {
   // depth-k readout: row b is verify token b % depth of its candidate and also attends to the
   // candidate's earlier tokens (rows b - b % depth .. b - 1); 1: each row its own entry only
   int depth = 1;
+  // optional [B][n_q]: the natural log of each row's softmax normaliser, log sum_j exp(q.k_j / sqrt(hd))
+  // over the cache and the self entries (kept for a backward pass)
+  float* lse = nullptr;
 };
 constexpr int kMaxReadoutDepth = 8;
 // q_hi / q_lo: bf16 pair of the rotated query [B][n_q][hd]; partial slot s of
@@ -230,6 +238,43 @@ cudaError_t launch_head(const ModelDims& m, const float* h, const float* sumsq, 
                         const __nv_bfloat16* gain, const __nv_bfloat16* w_plus, const __nv_bfloat16* w_minus,
                         float* rewards, cudaStream_t stream, bool pdl, unsigned long long* ts = nullptr);
 cudaError_t launch_split_hilo(const float* in, int64_t count, HiLo out, cudaStream_t stream);
+// ---------------------------------------------------------------- backward pass (KV Steering, grad.cu)
+constexpr int kMaxGroup = 16;   // query heads per kv head
+cudaError_t launch_transpose(const __nv_bfloat16* in, __nv_bfloat16* out, int rows, int cols, cudaStream_t st);
+// d(-log P(+))/dh at the final residual stream h [n][d]; dh fp32 and optionally as hi/lo
+cudaError_t launch_head_back(const float* h, const float* p_plus, const __nv_bfloat16* gain,
+                             const __nv_bfloat16* w_plus, const __nv_bfloat16* w_minus, int n, int d, float eps,
+                             float* dh, __nv_bfloat16* dh_hi, __nv_bfloat16* dh_lo, cudaStream_t st);
+// out = dres + RMSNorm backward at h (fp32 [n][d], or h_bf16: one bf16 row for every row) of dy
+cudaError_t launch_rms_back(const float* h, const __nv_bfloat16* h_bf16, const __nv_bfloat16* gain, const float* dy,
+                            const float* dres, int n, int d, float eps, float* out, __nv_bfloat16* o_hi,
+                            __nv_bfloat16* o_lo, cudaStream_t st);
+cudaError_t launch_silu_back(const float* da, const float* gu, int n, int ff, __nv_bfloat16* o_hi,
+                             __nv_bfloat16* o_lo, cudaStream_t st);
+// The attention read-out's backward of one layer.  units: int4 {b, g, j0, j1} (candidate b's logical
+// pages j0 .. j1 - 1 of kv head g); shared[page] != 0 for pages several candidates read (their
+// gradient accumulates atomically and must be zeroed first).
+struct AttnBackArgs {
+  int n, n_q, n_kv, hd;
+  const float *q, *kself, *vself, *o, *dout, *lse;   // forward saves [n][...] and d(out) [n][n_q hd]
+  float *D, *dq, *dks, *dvs;                         // [n][n_q], [n][n_q hd], [n][n_kv hd] x 2
+  const int4* units;
+  int n_units;
+  const int32_t* seq_lens;
+  const int32_t* block_table;
+  int max_blocks;
+  const __nv_bfloat16* pool_layer;                   // [n_pages][2][n_kv][16][hd]
+  const uint8_t* shared;
+  float* grad_layer;                                 // same layout, fp32
+};
+cudaError_t launch_attn_back(const AttnBackArgs& a, cudaStream_t st);
+cudaError_t launch_rope_back(const float* dq, const float* dks, const float* dvs, const float2* rope, int n, int n_q,
+                             int n_kv, int hd, __nv_bfloat16* o_hi, __nv_bfloat16* o_lo, cudaStream_t st);
+cudaError_t launch_zero_pages(float* grad, const int32_t* pages, int n_list, int n_layers, int64_t n_pages,
+                              int64_t page_elems, cudaStream_t st);
+cudaError_t launch_steer_update(__nv_bfloat16* kv, const float* grad, const int32_t* pages, int n_list, int n_layers,
+                                int64_t n_pages, int64_t page_elems, float eta, cudaStream_t st);
+
 // One thread waits (bounded by limit_ns, see flag_wait) for *flag to become nonzero; on timeout it
 // records kDevProbeTimeout in *err.  The failure-detection test hook behind kvprm_debug_wait_probe.
 cudaError_t launch_wait_probe(const int* flag, int* err, unsigned long long limit_ns, cudaStream_t stream);

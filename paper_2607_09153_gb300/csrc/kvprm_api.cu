@@ -7,6 +7,7 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <atomic>
 #include <cmath>
 #include <cstdarg>
@@ -56,6 +57,39 @@ struct ProfMark {
   cudaEvent_t a, b;
 };
 
+// Forward intermediates a backward pass needs (kvprm_score_grad), per layer l at l * (max_candidates
+// rows) of each array: the rotated q and the self k / v as the attention consumed them, the
+// attention output o and its softmax log-normaliser, the residual stream after the attention block
+// and after the layer, and the gate / up pre-activations.
+struct FwdSaves {
+  float *q = nullptr, *k = nullptr, *v = nullptr, *o = nullptr, *lse = nullptr;
+  float *hmid = nullptr, *hout = nullptr, *gu = nullptr;
+};
+
+// State of the KV Steering backward pass, built by the first kvprm_score_grad call on a context.
+struct GradState {
+  bool ready = false;
+  // library-owned transposed weights W^T [in][out] and their tensor maps (the backward's products
+  // dx = W^T dy run on the forward's GEMM with these as the streamed operand)
+  std::vector<__nv_bfloat16*> wt;   // per layer: qkv, o, gate_up, down
+  std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_down;
+  FwdSaves sv;
+  float *dh = nullptr, *tmp = nullptr, *D = nullptr, *dq = nullptr, *dks = nullptr, *dvs = nullptr;
+  __nv_bfloat16 *ghi = nullptr, *glo = nullptr;   // a gradient as the next product's bf16 hi/lo input
+  int tm_npad = -1;
+  CUtensorMap tm_d_hi{}, tm_d_lo{}, tm_gu_hi{}, tm_gu_lo{}, tm_qkv_hi{}, tm_qkv_lo{};
+  // per call: work units of the attention backward, shared-page flags and page lists
+  int4* units = nullptr;
+  size_t units_cap = 0;
+  uint8_t* shared = nullptr;
+  size_t shared_cap = 0;
+  int32_t* lists = nullptr;   // [shared pages][all referenced pages]
+  size_t lists_cap = 0;
+  int n_shared = 0, n_ref = 0;   // of the last call
+  float* grad_own = nullptr;   // kvprm_steer's gradient buffer
+  size_t grad_own_bytes = 0;
+};
+
 }  // namespace
 
 struct kvprm_ctx {
@@ -69,6 +103,7 @@ struct kvprm_ctx {
   std::vector<const bf16*> attn_norm, mlp_norm;
   std::vector<const bf16*> q_norm, k_norm;   // per-head q/k RMSNorm gains (cfg.qk_norm)
   std::vector<CUtensorMap> tm_qkv, tm_o, tm_gu, tm_down;
+  std::vector<const void*> w_qkv_src, w_o_src, w_gu_src, w_down_src;   // the borrowed matrices
   // depth-k readout (kvprm_set_readout_depth): verify tokens per candidate; candidate b of a call is
   // rows b depth .. b depth + depth - 1 of the batch (expanded tables below)
   int depth = 1;
@@ -163,6 +198,7 @@ struct kvprm_ctx {
   // (kvprm_debug_inject_error); a flag that nothing sets, for the bounded-wait probe
   int inject_fail = 0;
   int* probe_flag = nullptr;
+  GradState grad;
 };
 
 namespace {
@@ -269,6 +305,18 @@ void free_ctx(kvprm_ctx* c) {
   cudaFree(c->dummy_pool);
   cudaFree(c->dev_pool);
   cudaFree(c->probe_flag);
+  {
+    GradState& g = c->grad;
+    for (auto* p : g.wt) cudaFree(p);
+    cudaFree(g.sv.q);
+    cudaFree(g.dh);
+    cudaFree(g.ghi);
+    cudaFree(g.glo);
+    cudaFree(g.units);
+    cudaFree(g.shared);
+    cudaFree(g.lists);
+    cudaFree(g.grad_own);
+  }
   if (c->staging) cudaFreeHost(c->staging);
   if (c->h_rewards) cudaFreeHost(c->h_rewards);
   if (c->h_err) cudaFreeHost(c->h_err);
@@ -569,7 +617,7 @@ int enqueue_attention(kvprm_ctx* ctx, Enq& E, const kvprm::AttnShape& as, const 
   return KVPRM_OK;
 }
 
-int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
+int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E, const FwdSaves* sv = nullptr) {
   const ModelDims& m = ctx->md;
   const int n = P.n, np = P.n_pad;
   const int32_t* sl = ctx->tables_d;
@@ -653,18 +701,28 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
       eq_l.qn_gain = ctx->q_norm[l];
       eq_l.kn_gain = ctx->k_norm[l];
     }
+    const size_t Bm = static_cast<size_t>(ctx->cfg.max_candidates);
+    if (sv) {   // a backward pass follows: this layer's q, self k / v go to their saved slots
+      eq_l.q = sv->q + l * Bm * m.n_q * m.hd;
+      eq_l.kself = sv->k + l * Bm * m.n_kv * m.hd;
+      eq_l.vself = sv->v + l * Bm * m.n_kv * m.hd;
+    }
     LAUNCH(KVPRM_PROF_GEMM_QKV,
            kvprm::launch_gemm(P.g_qkv, &ctx->tm_qkv[l], &ctx->tm_xhi, &ctx->tm_xlo, eq_l, np, ctx->err_d, st, pdl, TS,
                               lora ? &lr_qkv : nullptr),
            "gemm_qkv");
     if (ctx->debug_flags & 2) {
       const size_t nq = static_cast<size_t>(n) * m.n_q * m.hd, nk = static_cast<size_t>(n) * m.n_kv * m.hd;
-      CK(cudaMemcpyAsync(ctx->dbg_q + l * nq, ctx->q, nq * 4, cudaMemcpyDeviceToDevice, st), "debug q");
-      CK(cudaMemcpyAsync(ctx->dbg_k + l * nk, ctx->kself, nk * 4, cudaMemcpyDeviceToDevice, st), "debug k");
-      CK(cudaMemcpyAsync(ctx->dbg_v + l * nk, ctx->vself, nk * 4, cudaMemcpyDeviceToDevice, st), "debug v");
+      CK(cudaMemcpyAsync(ctx->dbg_q + l * nq, eq_l.q, nq * 4, cudaMemcpyDeviceToDevice, st), "debug q");
+      CK(cudaMemcpyAsync(ctx->dbg_k + l * nk, eq_l.kself, nk * 4, cudaMemcpyDeviceToDevice, st), "debug k");
+      CK(cudaMemcpyAsync(ctx->dbg_v + l * nk, eq_l.vself, nk * 4, cudaMemcpyDeviceToDevice, st), "debug v");
     }
     float* dbg = (ctx->debug_flags & 1) ? ctx->dbg + static_cast<size_t>(l) * n * m.n_q * m.hd : nullptr;
-    const kvprm::AttnMerge mg{ctx->q, ctx->kself, ctx->vself, O.hi, O.lo, nullptr, dbg, ctx->depth};
+    kvprm::AttnMerge mg{eq_l.q, eq_l.kself, eq_l.vself, O.hi, O.lo, nullptr, dbg, ctx->depth};
+    if (sv) {
+      mg.out_f32 = sv->o + l * Bm * m.n_q * m.hd;
+      mg.lse = sv->lse + l * Bm * m.n_q;
+    }
     const kvprm::AttnWork wk = device_work(ctx);
     if (ctx->layer_waits)   // this layer's pages are still being copied in (kvprm_score_host)
       CK(cudaStreamWaitEvent(st, ctx->layer_ready[l], E.capturing ? cudaEventWaitExternal : cudaEventWaitDefault),
@@ -680,18 +738,22 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E) {
     kvprm::GemmEpilogue er_o = er;   // h += W_o o; x = h ⊙ g_mlp for the gate/up projection
     er_o.gain_next = ctx->mlp_norm[l];
     er_o.late_trigger = true;   // gate/up CTAs fit beside the O projection's
+    if (sv) er_o.h_copy = sv->hmid + l * Bm * m.d;
     if (lora && (arc = adapter(1, l, P.l_o, &ctx->tm_ohi, &ctx->tm_olo, P.k_o, &lr_o))) return arc;
     LAUNCH(KVPRM_PROF_GEMM_O,
            kvprm::launch_gemm(P.g_o, &ctx->tm_o[l], &ctx->tm_ohi, &ctx->tm_olo, er_o, np, ctx->err_d, st, pdl, TS,
                               lora ? &lr_o : nullptr),
            "gemm_o");
     if (lora && (arc = adapter(2, l, P.l_gu, &ctx->tm_xhi, &ctx->tm_xlo, P.k_gu, &lr_gu))) return arc;
+    kvprm::GemmEpilogue es_l = es;
+    if (sv) es_l.gu_save = sv->gu + l * Bm * 2 * m.ff;
     LAUNCH(KVPRM_PROF_GEMM_GATE_UP,
-           kvprm::launch_gemm(P.g_gu, &ctx->tm_gu[l], &ctx->tm_xhi, &ctx->tm_xlo, es, np, ctx->err_d, st, pdl, TS,
+           kvprm::launch_gemm(P.g_gu, &ctx->tm_gu[l], &ctx->tm_xhi, &ctx->tm_xlo, es_l, np, ctx->err_d, st, pdl, TS,
                               lora ? &lr_gu : nullptr),
            "gemm_gate_up");
     kvprm::GemmEpilogue er_d = er;   // h += W_down a; x = h ⊙ g_attn of the next layer
     er_d.gain_next = l + 1 < NL ? ctx->attn_norm[l + 1] : nullptr;
+    if (sv) er_d.h_copy = sv->hout + l * Bm * m.d;
     if (lora && (arc = adapter(3, l, P.l_down, &ctx->tm_ahi, &ctx->tm_alo, P.k_down, &lr_down))) return arc;
     LAUNCH(KVPRM_PROF_GEMM_DOWN,
            kvprm::launch_gemm(P.g_down, &ctx->tm_down[l], &ctx->tm_ahi, &ctx->tm_alo, er_d, np, ctx->err_d, st, pdl,
@@ -759,7 +821,7 @@ int enqueue_pool_copy(kvprm_ctx* ctx, cudaStream_t st) {
 }
 
 int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const int32_t* bt, const int32_t* sl, int32_t n,
-                 cudaStream_t st) {
+                 cudaStream_t st, const FwdSaves* sv = nullptr) {
   int max_pages = 0;
   int rc = validate_tables(ctx, n_pages, bt, sl, n, &max_pages);
   if (rc) return rc;
@@ -809,9 +871,9 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
     return cuda_fail(ctx, cudaErrorLaunchFailure, "injected failure of the forward's launch");
   }
 
-  if (!ctx->use_graph) {
+  if (!ctx->use_graph || sv) {   // a forward that keeps its intermediates runs eagerly
     Enq E{ctx, st, ctx->use_pdl && !ctx->profile, ctx->profile, &ctx->live_marks};
-    if ((rc = enqueue_forward(ctx, P, E))) return rc;
+    if ((rc = enqueue_forward(ctx, P, E, sv))) return rc;
     if (ctx->profile) {
       CK(cudaStreamSynchronize(st), "cudaStreamSynchronize(profile)");
       if ((rc = accumulate_marks(ctx, ctx->live_marks, true))) return rc;
@@ -875,6 +937,219 @@ int finish_blocking(kvprm_ctx* ctx, int32_t n, float* rewards, cudaStream_t st) 
     return fail(ctx, KVPRM_ETIMEOUT, "a bounded device wait timed out (code %d); results are invalid", site);
   }
   std::memcpy(rewards, ctx->h_rewards, sizeof(float) * n);
+  return KVPRM_OK;
+}
+
+// ---------------------------------------------------------------- KV Steering: backward pass
+// First kvprm_score_grad call: transposed weight copies, forward saves and backward buffers, sized
+// for max_candidates.
+int ensure_grad(kvprm_ctx* ctx, cudaStream_t st) {
+  GradState& g = ctx->grad;
+  if (g.ready) return KVPRM_OK;
+  const ModelDims& m = ctx->md;
+  const int NL = ctx->cfg.n_layers;
+  const size_t Bm = static_cast<size_t>(ctx->cfg.max_candidates);
+  const size_t nqh = static_cast<size_t>(m.n_q) * m.hd, nkh = static_cast<size_t>(m.n_kv) * m.hd;
+  int rc;
+  // saves: one allocation carved per array
+  const size_t per_layer = Bm * (nqh + 2 * nkh + nqh + m.n_q + 2 * static_cast<size_t>(m.d) + 2 * static_cast<size_t>(m.ff));
+  float* base = nullptr;
+  if ((rc = dalloc(ctx, &base, per_layer * NL, "backward saves"))) return rc;
+  FwdSaves& sv = g.sv;
+  float* p = base;
+  auto take = [&](size_t per) {
+    float* r = p;
+    p += per * NL;
+    return r;
+  };
+  sv.q = take(Bm * nqh);
+  sv.k = take(Bm * nkh);
+  sv.v = take(Bm * nkh);
+  sv.o = take(Bm * nqh);
+  sv.lse = take(Bm * m.n_q);
+  sv.hmid = take(Bm * m.d);
+  sv.hout = take(Bm * m.d);
+  sv.gu = take(Bm * 2 * static_cast<size_t>(m.ff));
+  // backward buffers
+  const size_t wmax = std::max<size_t>(std::max<size_t>(m.ff, m.d), nqh);
+  const size_t gmax = std::max<size_t>(std::max<size_t>(2 * static_cast<size_t>(m.ff), m.qkv_rows), m.d);
+  float* bb = nullptr;
+  if ((rc = dalloc(ctx, &bb, Bm * (m.d + wmax + m.n_q + nqh + 2 * nkh), "backward buffers"))) return rc;
+  g.dh = bb;
+  g.tmp = g.dh + Bm * m.d;
+  g.D = g.tmp + Bm * wmax;
+  g.dq = g.D + Bm * m.n_q;
+  g.dks = g.dq + Bm * nqh;
+  g.dvs = g.dks + Bm * nkh;
+  if ((rc = dalloc(ctx, &g.ghi, static_cast<size_t>(ctx->npad_max) * gmax, "backward hi"))) return rc;
+  if ((rc = dalloc(ctx, &g.glo, static_cast<size_t>(ctx->npad_max) * gmax, "backward lo"))) return rc;
+  // transposed weights: W [out][in] -> W^T [in][out], from the borrowed weights' tensor-map bases
+  g.tm_qkv.resize(NL);
+  g.tm_o.resize(NL);
+  g.tm_gu.resize(NL);
+  g.tm_down.resize(NL);
+  struct Mat {
+    int out, in;
+  } mats[4] = {{m.qkv_rows, m.d}, {m.d, m.n_q * m.hd}, {2 * m.ff, m.d}, {m.d, m.ff}};
+  for (int l = 0; l < NL; ++l) {
+    const void* src[4] = {ctx->w_qkv_src[l], ctx->w_o_src[l], ctx->w_gu_src[l], ctx->w_down_src[l]};
+    CUtensorMap* maps[4] = {&g.tm_qkv[l], &g.tm_o[l], &g.tm_gu[l], &g.tm_down[l]};
+    for (int j = 0; j < 4; ++j) {
+      bf16* wt = nullptr;
+      if ((rc = dalloc(ctx, &wt, static_cast<size_t>(mats[j].out) * mats[j].in, "transposed weights"))) return rc;
+      g.wt.push_back(wt);
+      CK(kvprm::launch_transpose(static_cast<const bf16*>(src[j]), wt, mats[j].out, mats[j].in, st), "transpose");
+      // W^T [in][out]: M = in rows, K = out columns
+      if ((rc = make_map(ctx, maps[j], wt, mats[j].out, mats[j].in, 64, 128, "transposed weights"))) return rc;
+    }
+  }
+  g.ready = true;
+  return KVPRM_OK;
+}
+
+int ensure_grad_maps(kvprm_ctx* ctx, int n_pad) {
+  GradState& g = ctx->grad;
+  if (g.tm_npad == n_pad) return KVPRM_OK;
+  const ModelDims& m = ctx->md;
+  int rc;
+  if ((rc = make_map(ctx, &g.tm_d_hi, g.ghi, m.d, n_pad, 64, n_pad, "grad hi (d)"))) return rc;
+  if ((rc = make_map(ctx, &g.tm_d_lo, g.glo, m.d, n_pad, 64, n_pad, "grad lo (d)"))) return rc;
+  if ((rc = make_map(ctx, &g.tm_gu_hi, g.ghi, 2 * static_cast<uint64_t>(m.ff), n_pad, 64, n_pad, "grad hi (gu)")))
+    return rc;
+  if ((rc = make_map(ctx, &g.tm_gu_lo, g.glo, 2 * static_cast<uint64_t>(m.ff), n_pad, 64, n_pad, "grad lo (gu)")))
+    return rc;
+  if ((rc = make_map(ctx, &g.tm_qkv_hi, g.ghi, m.qkv_rows, n_pad, 64, n_pad, "grad hi (qkv)"))) return rc;
+  if ((rc = make_map(ctx, &g.tm_qkv_lo, g.glo, m.qkv_rows, n_pad, 64, n_pad, "grad lo (qkv)"))) return rc;
+  g.tm_npad = n_pad;
+  return KVPRM_OK;
+}
+
+template <typename T>
+int grow(kvprm_ctx* ctx, T** p, size_t* cap, size_t need, const char* what) {
+  if (need <= *cap) return KVPRM_OK;
+  cudaFree(*p);
+  *p = nullptr;
+  *cap = 0;
+  int rc = dalloc(ctx, p, need, what);
+  if (rc) return rc;
+  *cap = need;
+  return KVPRM_OK;
+}
+
+// The gradient of sum_b -log P(+)_b with respect to the pages (all layers) into grad [N_L][n_pages]
+// [2][n_kv][16][hd] (fp32), and P(+) into ctx->rewards_d.  Blocking (the caller synchronises); on
+// return *n_ref / ref_pages hold the pages the tables reference (device list at lists + n_shared).
+int score_grad_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const int32_t* bt, const int32_t* sl,
+                      int32_t n, float* grad, cudaStream_t st, int* n_ref_out) {
+  if (ctx->lora_rank) return fail(ctx, KVPRM_EUNSUPPORTED, "the backward pass takes the merged weights (no adapter)");
+  if (ctx->depth != 1) return fail(ctx, KVPRM_EUNSUPPORTED, "the backward pass takes one verify token (depth 1)");
+  if (ctx->cfg.qk_norm) return fail(ctx, KVPRM_EUNSUPPORTED, "the backward pass does not implement the q/k norm");
+  if (n > 0 && !grad) return fail(ctx, KVPRM_EINVAL, "the gradient buffer is NULL");
+  if (grad && (reinterpret_cast<uintptr_t>(grad) & 15u)) return fail(ctx, KVPRM_EINVAL, "grad is not 16-byte aligned");
+  int max_pages = 0;
+  int rc = validate_tables(ctx, n_pages, bt, sl, n, &max_pages);
+  if (rc) return rc;
+  *n_ref_out = 0;
+  if (n == 0) return KVPRM_OK;
+  if ((rc = ensure_grad(ctx, st))) return rc;
+  GradState& g = ctx->grad;
+  // the forward, keeping its intermediates
+  if ((rc = score_device(ctx, kv_pages, n_pages, bt, sl, n, st, &g.sv))) return rc;
+  const ModelDims& m = ctx->md;
+  const int NL = ctx->cfg.n_layers, mb = ctx->cfg.max_blocks_per_seq;
+  const int np = (n + 15) / 16 * 16;
+  if ((rc = ensure_grad_maps(ctx, np))) return rc;
+  // host plan: work units (candidate, kv head, <= 8 pages) and the pages several candidates read
+  std::vector<int4> units;
+  std::vector<uint8_t> refs(static_cast<size_t>(n_pages > 0 ? n_pages : 1), 0);
+  constexpr int kUnitPages = 8;
+  for (int b = 0; b < n; ++b) {
+    const int pages = (sl[b] + 15) / 16;
+    for (int j = 0; j < pages; ++j) {
+      uint8_t& r = refs[bt[static_cast<int64_t>(b) * mb + j]];
+      if (r < 2) ++r;
+    }
+    for (int gg = 0; gg < m.n_kv; ++gg)
+      for (int j0 = 0; j0 < pages; j0 += kUnitPages) units.push_back(make_int4(b, gg, j0, std::min(pages, j0 + kUnitPages)));
+  }
+  std::vector<int32_t> lists;   // shared pages, then every referenced page
+  for (int64_t p = 0; p < n_pages; ++p)
+    if (refs[p] >= 2) lists.push_back(static_cast<int32_t>(p));
+  const int n_shared = static_cast<int>(lists.size());
+  for (int64_t p = 0; p < n_pages; ++p)
+    if (refs[p] >= 1) lists.push_back(static_cast<int32_t>(p));
+  for (auto& r : refs) r = r >= 2 ? 1 : 0;
+  if ((rc = grow(ctx, &g.units, &g.units_cap, std::max<size_t>(units.size(), 1), "backward units"))) return rc;
+  if ((rc = grow(ctx, &g.shared, &g.shared_cap, refs.size(), "shared-page flags"))) return rc;
+  if ((rc = grow(ctx, &g.lists, &g.lists_cap, std::max<size_t>(lists.size(), 1), "page lists"))) return rc;
+  if (!units.empty())
+    CK(cudaMemcpyAsync(g.units, units.data(), sizeof(int4) * units.size(), cudaMemcpyHostToDevice, st), "units");
+  CK(cudaMemcpyAsync(g.shared, refs.data(), refs.size(), cudaMemcpyHostToDevice, st), "shared flags");
+  if (!lists.empty())
+    CK(cudaMemcpyAsync(g.lists, lists.data(), sizeof(int32_t) * lists.size(), cudaMemcpyHostToDevice, st), "lists");
+  const int64_t page_elems = static_cast<int64_t>(2) * m.n_kv * 16 * m.hd;
+  CK(kvprm::launch_zero_pages(grad, g.lists, n_shared, NL, n_pages, page_elems, st), "zero shared pages");
+  // the backward products on the forward's GEMM (plain fp32 epilogue) against the transposed weights
+  auto gemm = [&](const CUtensorMap* w, int M, int K, const CUtensorMap* xh, const CUtensorMap* xl, float* out) {
+    const GemmPlan gp = kvprm::plan_gemm(M, K, np, ctx->num_sms, true, false);
+    kvprm::GemmEpilogue ep;
+    ep.mode = kvprm::GemmEpilogue::PLAIN;
+    ep.M = M;
+    ep.n_valid = n;
+    ep.out = out;
+    return kvprm::launch_gemm(gp, w, xh, xl, ep, np, ctx->err_d, st, false);
+  };
+  const size_t Bm = static_cast<size_t>(ctx->cfg.max_candidates);
+  const int nqh = m.n_q * m.hd, nkh = m.n_kv * m.hd;
+  const FwdSaves& sv = g.sv;
+  CK(kvprm::launch_head_back(ctx->h, ctx->rewards_d, ctx->final_norm, ctx->w_plus, ctx->w_minus, n, m.d, m.eps, g.dh,
+                             g.ghi, g.glo, st),
+     "head backward");
+  for (int l = NL - 1; l >= 0; --l) {
+    // feed-forward block: da = W_down^T dh; [du; dt]; dx2 = W_gate_up^T [du; dt]; dh_mid
+    CK(gemm(&g.tm_down[l], m.ff, m.d, &g.tm_d_hi, &g.tm_d_lo, g.tmp), "W_down^T product");
+    CK(kvprm::launch_silu_back(g.tmp, sv.gu + l * Bm * 2 * m.ff, n, m.ff, g.ghi, g.glo, st), "SiLU backward");
+    CK(gemm(&g.tm_gu[l], m.d, 2 * m.ff, &g.tm_gu_hi, &g.tm_gu_lo, g.tmp), "W_gate_up^T product");
+    CK(kvprm::launch_rms_back(sv.hmid + l * Bm * m.d, nullptr, ctx->mlp_norm[l], g.tmp, g.dh, n, m.d, m.eps, g.dh,
+                              g.ghi, g.glo, st),
+       "pre-MLP RMSNorm backward");
+    // attention block: do = W_o^T dh_mid, then the read-out's backward into this layer's pages
+    CK(gemm(&g.tm_o[l], nqh, m.d, &g.tm_d_hi, &g.tm_d_lo, g.tmp), "W_o^T product");
+    kvprm::AttnBackArgs a;
+    a.n = n;
+    a.n_q = m.n_q;
+    a.n_kv = m.n_kv;
+    a.hd = m.hd;
+    a.q = sv.q + l * Bm * nqh;
+    a.kself = sv.k + l * Bm * nkh;
+    a.vself = sv.v + l * Bm * nkh;
+    a.o = sv.o + l * Bm * nqh;
+    a.dout = g.tmp;
+    a.lse = sv.lse + l * Bm * m.n_q;
+    a.D = g.D;
+    a.dq = g.dq;
+    a.dks = g.dks;
+    a.dvs = g.dvs;
+    a.units = g.units;
+    a.n_units = static_cast<int>(units.size());
+    a.seq_lens = ctx->tables_d;
+    a.block_table = ctx->tables_d + ctx->cfg.max_candidates;
+    a.max_blocks = mb;
+    a.pool_layer = kv_pages ? static_cast<const bf16*>(kv_pages) + l * n_pages * page_elems : nullptr;
+    a.shared = g.shared;
+    a.grad_layer = grad + l * n_pages * page_elems;
+    CK(kvprm::launch_attn_back(a, st), "attention backward");
+    if (l == 0) break;   // below layer 0 lies only the verify token's embedding
+    // QKV projection: [dq; dk; dv] before RoPE, dx1 = W_qkv^T [...], dh of the layer below
+    CK(kvprm::launch_rope_back(g.dq, g.dks, g.dvs, ctx->rope, n, m.n_q, m.n_kv, m.hd, g.ghi, g.glo, st), "RoPE backward");
+    CK(gemm(&g.tm_qkv[l], m.d, m.qkv_rows, &g.tm_qkv_hi, &g.tm_qkv_lo, g.tmp), "W_qkv^T product");
+    CK(kvprm::launch_rms_back(sv.hout + (l - 1) * Bm * m.d, nullptr, ctx->attn_norm[l], g.tmp, g.dh, n, m.d, m.eps,
+                              g.dh, g.ghi, g.glo, st),
+       "pre-attention RMSNorm backward");
+  }
+  g.n_shared = n_shared;
+  g.n_ref = static_cast<int>(lists.size()) - n_shared;
+  *n_ref_out = g.n_ref;
   return KVPRM_OK;
 }
 
@@ -981,6 +1256,10 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
       ctx->k_norm[l] = static_cast<const bf16*>(w->k_norm[l]);
     }
   }
+  ctx->w_qkv_src.assign(w->w_qkv, w->w_qkv + NL);
+  ctx->w_o_src.assign(w->w_o, w->w_o + NL);
+  ctx->w_gu_src.assign(w->w_gate_up, w->w_gate_up + NL);
+  ctx->w_down_src.assign(w->w_down, w->w_down + NL);
   for (int l = 0; l < NL; ++l) {
     ctx->attn_norm[l] = static_cast<const bf16*>(w->attn_norm[l]);
     ctx->mlp_norm[l] = static_cast<const bf16*>(w->mlp_norm[l]);
@@ -1455,6 +1734,58 @@ int kvprm_plan_attention(const int32_t* block_table, int32_t max_blocks_per_seq,
     std::memcpy(plan->slot_base, w.slot_base.data(), sizeof(int32_t) * w.slot_base.size());
     std::memcpy(plan->nslots, w.nslots.data(), sizeof(int32_t) * w.nslots.size());
   }
+  return KVPRM_OK;
+}
+
+int kvprm_score_grad(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const int32_t* block_table,
+                     const int32_t* seq_lens, int32_t n_candidates, float* d_grad, float* rewards, void* stream) {
+  if (!ctx) return KVPRM_EINVAL;
+  if (n_candidates > 0 && !rewards) return fail(ctx, KVPRM_EINVAL, "rewards is NULL");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int n_ref = 0;
+  int rc = score_grad_device(ctx, kv_pages, n_pages, block_table, seq_lens, n_candidates, d_grad, st, &n_ref);
+  if (rc) return rc;
+  return finish_blocking(ctx, n_candidates, rewards, st);
+}
+
+int kvprm_steer(kvprm_ctx* ctx, void* kv_pages, int64_t n_pages, const int32_t* block_table, const int32_t* seq_lens,
+                int32_t n_candidates, float eta, int32_t steps, float* p_first, float* p_last, void* stream) {
+  if (!ctx) return KVPRM_EINVAL;
+  if (steps < 0) return fail(ctx, KVPRM_EINVAL, "steps = %d is negative", steps);
+  if (!std::isfinite(eta)) return fail(ctx, KVPRM_EINVAL, "eta is not finite");
+  if (n_candidates < 0) return fail(ctx, KVPRM_EINVAL, "n_candidates is negative");
+  if (n_pages < 0) return fail(ctx, KVPRM_EINVAL, "n_pages is negative");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (n_candidates == 0) return KVPRM_OK;
+  const ModelDims& m = ctx->md;
+  const int64_t page_elems = static_cast<int64_t>(2) * m.n_kv * 16 * m.hd;
+  const size_t bytes = static_cast<size_t>(ctx->cfg.n_layers) * static_cast<size_t>(n_pages) * page_elems * 4;
+  GradState& g = ctx->grad;
+  int rc;
+  if (bytes > g.grad_own_bytes) {
+    CK(cudaStreamSynchronize(st), "cudaStreamSynchronize(steering buffer)");
+    size_t cap = g.grad_own_bytes / 4;
+    if ((rc = grow(ctx, &g.grad_own, &cap, bytes / 4, "steering gradient"))) {
+      g.grad_own_bytes = 0;
+      return rc;
+    }
+    g.grad_own_bytes = bytes;
+  }
+  std::vector<float> host(static_cast<size_t>(n_candidates));
+  for (int t = 0; t < steps; ++t) {
+    int n_ref = 0;
+    if ((rc = score_grad_device(ctx, kv_pages, n_pages, block_table, seq_lens, n_candidates, g.grad_own, st, &n_ref)))
+      return rc;
+    if (t == 0 && p_first && (rc = finish_blocking(ctx, n_candidates, p_first, st))) return rc;
+    // every referenced page (the list after the shared ones), every layer
+    CK(kvprm::launch_steer_update(static_cast<bf16*>(kv_pages), g.grad_own, g.lists + g.n_shared, n_ref,
+                                  ctx->cfg.n_layers, n_pages, page_elems, eta, st),
+       "steering update");
+  }
+  if ((rc = score_device(ctx, kv_pages, n_pages, block_table, seq_lens, n_candidates, st))) return rc;
+  if ((rc = finish_blocking(ctx, n_candidates, host.data(), st))) return rc;
+  if (steps == 0 && p_first) std::memcpy(p_first, host.data(), sizeof(float) * n_candidates);
+  if (p_last) std::memcpy(p_last, host.data(), sizeof(float) * n_candidates);
   return KVPRM_OK;
 }
 

@@ -102,6 +102,8 @@ def lib() -> ctypes.CDLL:
         L.kvprm_resolve.argtypes = [vp, i32, i64p]
         L.kvprm_check_device.argtypes = [vp]
         L.kvprm_debug_set_alloc_limit.argtypes = [i64]
+        L.kvprm_score_grad.argtypes = [vp, vp, i64, i32p, i32p, i32, vp, f32p, vp]
+        L.kvprm_steer.argtypes = [vp, vp, i64, i32p, i32p, i32, ctypes.c_float, i32, f32p, f32p, vp]
         L.kvprm_debug_inject_error.argtypes = [vp, i32]
         L.kvprm_debug_wait_probe.argtypes = [vp, i32, vp]
         L.kvprm_set_profile.argtypes = [vp, ctypes.c_int]
@@ -169,6 +171,28 @@ def kvprm_score_host(ctx, h_kv_pages_ptr: int, n_pages: int, block_table, seq_le
     _check(ctx, lib().kvprm_score_host(ctx, h_kv_pages_ptr, n_pages, _p(bt, ctypes.c_int32), _p(sl, ctypes.c_int32),
                                        n, _p(out, ctypes.c_float), stream_ptr))
     return out
+
+
+def kvprm_score_grad(ctx, kv_pages_ptr: int, n_pages: int, block_table, seq_lens, n: int, d_grad_ptr: int,
+                     stream_ptr: int = 0) -> np.ndarray:
+    """KV Steering gradient: d(sum_b -log P(+)_b)/d(keys, values) into the device fp32 buffer d_grad
+    (the pool's layout); returns P(+) [n]."""
+    bt, sl = _i32(block_table), _i32(seq_lens)
+    out = np.zeros(n, np.float32)
+    _check(ctx, lib().kvprm_score_grad(ctx, kv_pages_ptr, n_pages, _p(bt, ctypes.c_int32), _p(sl, ctypes.c_int32), n,
+                                       d_grad_ptr, _p(out, ctypes.c_float), stream_ptr))
+    return out
+
+
+def kvprm_steer(ctx, kv_pages_ptr: int, n_pages: int, block_table, seq_lens, n: int, eta: float, steps: int,
+                stream_ptr: int = 0) -> tuple[np.ndarray, np.ndarray]:
+    """`steps` KV Steering steps on the (caller-owned, written) pages; returns P(+) before and after."""
+    bt, sl = _i32(block_table), _i32(seq_lens)
+    p0 = np.zeros(n, np.float32)
+    p1 = np.zeros(n, np.float32)
+    _check(ctx, lib().kvprm_steer(ctx, kv_pages_ptr, n_pages, _p(bt, ctypes.c_int32), _p(sl, ctypes.c_int32), n,
+                                  float(eta), int(steps), _p(p0, ctypes.c_float), _p(p1, ctypes.c_float), stream_ptr))
+    return p0, p1
 
 
 def kvprm_attention(ctx, kv_layer_ptr: int, n_pages: int, block_table, seq_lens, n: int, q_ptr: int, k_self_ptr: int,
