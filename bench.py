@@ -503,7 +503,17 @@ def summarize(w, m: dict, world: int) -> dict:
 OTHER_WORKLOADS = ("tiny", "qwen1p5b_b16_l2048", "beam7b_b64_p4096_s512", "mcts7b_b256_d4")
 
 
-def measure_steering(args, name: str, calls: int = 5) -> dict:
+def run_steering_only(args, world, rank, local):
+    """The KV Steering gradient alone on --workload (the case ncu captures of the backward use)."""
+    import torch
+    torch.cuda.set_device(local)
+    line = measure_steering(args, args.workload, calls=args.steps, warmup=args.warmup)
+    line["metric"] = "KV Steering gradient calls/s"
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+
+def measure_steering(args, name: str, calls: int = 5, warmup: int = 1) -> dict:
     """KV Steering's gradient (kvprm_score_grad: the forward with its intermediates kept, then the
     backward into every referenced page) on one workload: blocking calls timed on the host clock.
     Algorithmic bytes per call: the weights twice (forward, then their transposes), the unique K/V
@@ -522,7 +532,8 @@ def measure_steering(args, name: str, calls: int = 5) -> dict:
     t0 = time.perf_counter()
     kp.kvprm_score_grad(*args_)   # the first call also builds the transposed weights
     first_s = time.perf_counter() - t0
-    kp.kvprm_score_grad(*args_)
+    for _ in range(warmup):
+        kp.kvprm_score_grad(*args_)
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     for _ in range(calls):
@@ -578,7 +589,8 @@ def run_gpu(args, world, rank, local):
             mo = measure(wo, args, world, local, min(args.steps, 20), 3, 3, with_e2e=False, clocks=True)
             so = summarize(wo, mo, world)
             entry = {k: so[k] for k in ("scores_per_s", "ms_per_call", "kv_tokens_per_s", "whole_call", "host",
-                                        "launches_per_call")}
+                                        "launches_per_call", "pipelined_us_per_layer")}
+            entry["kernel_avg_us"] = {k: v["avg_us"] for k, v in so["kernels"].items()}
             if name == "tiny":
                 entry["us_per_call"] = so["us_per_call"]
             else:
@@ -698,6 +710,8 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-steering", action="store_true", help="skip the KV Steering gradient measurement")
+    ap.add_argument("--steering-only", action="store_true",
+                    help="time the KV Steering gradient (kvprm_score_grad) alone on --workload")
     ap.add_argument("--attention-only", action="store_true",
                     help="time the paged attention alone on one layer of the workload's cache")
     args = ap.parse_args()
@@ -708,6 +722,8 @@ def main():
         run_reference(args, world, rank)
     elif args.attention_only:
         run_attention_only(args, world, rank, local)
+    elif args.steering_only:
+        run_steering_only(args, world, rank, local)
     else:
         run_gpu(args, world, rank, local)
     if world > 1:

@@ -180,26 +180,52 @@ __global__ void attn_back_pre_kernel(const float* __restrict__ q, const float* _
   }
 }
 
-// One CTA of 4 warps per unit {b, g, j0, j1}: candidate b's logical pages j0 .. j1 - 1 of kv head g.
-// Warp w takes tokens w, w + 4, .. of each page; each lane holds HD / 32 consecutive elements of
-// the token's key and value (read straight from HBM), of the G query rows and of their output
+// One CTA of 4 warps per unit {b, g, j0, j1}: candidate b's logical pages j0 .. j1 - 1 (at most
+// kBackUnitPages) of kv head g.  Thread 0 bulk-copies the unit's K and V blocks (16 x HD bf16 each,
+// contiguous in the pool) into shared memory at once, so every byte of the unit is in flight before
+// any is used.  Warp w then takes tokens w, w + 4, .. of each page; each lane holds HD / 32
+// consecutive elements of the token's key and value, of the G query rows and of their output
 // gradients, so every dot product is a lane-local sum and one warp reduction.  dK and dV of a page
 // only this candidate reads are stored; of a page several read (shared[page] != 0) they are added
-// with atomics (zero_pages cleared them).  dq is summed over the CTA's warps, then added atomically.
+// with atomics (zero_pages cleared them).  dq is summed over the CTA's warps (in the shared memory
+// the pages occupied), then added atomically.
+constexpr int kBackUnitPages = kBackUnitPagesMax;
+
+template <int HD>
+constexpr size_t back_pages_smem() {
+  return static_cast<size_t>(kBackUnitPages) * 2 * 16 * HD * 2 + 16;   // the pages' K and V, the barrier
+}
+
 template <int HD, int GMAX>
 __global__ void __launch_bounds__(128) attn_back_pages_kernel(
     const int4* __restrict__ units, const int32_t* __restrict__ seq_lens, const int32_t* __restrict__ block_table,
     int max_blocks, const bf16* __restrict__ pool_layer, const uint8_t* __restrict__ shared, const float* __restrict__ q,
     const float* __restrict__ dout, const float* __restrict__ lse, const float* __restrict__ D, int n_q, int n_kv,
-    float* __restrict__ grad_layer, float* __restrict__ dq) {
+    float* __restrict__ grad_layer, float* __restrict__ dq, int* err) {
   constexpr int kPer = HD / 32;   // 4 (hd 128) or 2 (hd 64)
-  __shared__ float s_dq[4][GMAX][HD];
+  constexpr uint32_t kBlock = 16 * HD * 2;   // one page's K (or V) of one kv head, bytes
+  extern __shared__ __align__(16) uint8_t smem[];
+  bf16* s_kv = reinterpret_cast<bf16*>(smem);   // [page][K, V][16][HD]
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(kBackUnitPages) * 2 * kBlock);
   const int4 u = units[blockIdx.x];
   const int b = u.x, g = u.y, j0 = u.z, j1 = u.w;
+  const int npg = j1 - j0;   // 1 .. kBackUnitPages
   const int G = n_q / n_kv;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float scale = rsqrtf(static_cast<float>(HD));
   const int L = seq_lens[b];
+  const int64_t page_elems = static_cast<int64_t>(2) * n_kv * 16 * HD;   // one page of one layer
+  if (threadIdx.x == 0) {
+    mbar_init(bar, 1);
+    fence_mbar_init();
+    mbar_arrive_expect_tx(bar, static_cast<uint32_t>(npg) * 2 * kBlock);
+    for (int i = 0; i < npg; ++i) {
+      const int32_t p = block_table[static_cast<int64_t>(b) * max_blocks + j0 + i];
+      const bf16* kp = pool_layer + p * page_elems + static_cast<int64_t>(g) * 16 * HD;
+      bulk_load(s_kv + (2 * i) * 16 * HD, kp, kBlock, bar);
+      bulk_load(s_kv + (2 * i + 1) * 16 * HD, kp + static_cast<int64_t>(n_kv) * 16 * HD, kBlock, bar);
+    }
+  }
   float qr[GMAX][kPer], dr[GMAX][kPer], acc[GMAX][kPer];
   float lse_r[GMAX], D_r[GMAX];
 #pragma unroll
@@ -216,20 +242,27 @@ __global__ void __launch_bounds__(128) attn_back_pages_kernel(
       D_r[r] = D[row];
     }
   }
-  const int64_t page_elems = static_cast<int64_t>(2) * n_kv * 16 * HD;   // one page of one layer
-  for (int j = j0; j < j1; ++j) {
+  __syncthreads();   // the barrier is initialised
+  if (!mbar_wait(bar, 0, err)) {
+    // gave up (the error word is set): wait, bounded again, for the copies still landing in this
+    // CTA's shared memory before leaving
+    mbar_wait(bar, 0, err);
+    return;
+  }
+  for (int i = 0; i < npg; ++i) {
+    const int j = j0 + i;
     const int32_t p = block_table[static_cast<int64_t>(b) * max_blocks + j];
     const int valid = min(16, L - 16 * j);
-    const bf16* kp = pool_layer + p * page_elems + static_cast<int64_t>(g) * 16 * HD;
-    const bf16* vp = kp + static_cast<int64_t>(n_kv) * 16 * HD;
+    const bf16* ks = s_kv + (2 * i) * 16 * HD;
+    const bf16* vs = ks + 16 * HD;
     float* gk = grad_layer + p * page_elems + static_cast<int64_t>(g) * 16 * HD;
     float* gv = gk + static_cast<int64_t>(n_kv) * 16 * HD;
     const bool sh = shared[p] != 0;
     for (int t = warp; t < 16; t += 4) {
       float kf[kPer], vf[kPer];
       if constexpr (kPer == 4) {
-        const uint2 kb = *reinterpret_cast<const uint2*>(kp + t * HD + lane * 4);
-        const uint2 vb = *reinterpret_cast<const uint2*>(vp + t * HD + lane * 4);
+        const uint2 kb = *reinterpret_cast<const uint2*>(ks + t * HD + lane * 4);
+        const uint2 vb = *reinterpret_cast<const uint2*>(vs + t * HD + lane * 4);
         const float2 k01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kb.x));
         const float2 k23 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kb.y));
         const float2 v01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&vb.x));
@@ -237,8 +270,8 @@ __global__ void __launch_bounds__(128) attn_back_pages_kernel(
         kf[0] = k01.x; kf[1] = k01.y; kf[2] = k23.x; kf[3] = k23.y;
         vf[0] = v01.x; vf[1] = v01.y; vf[2] = v23.x; vf[3] = v23.y;
       } else {
-        const uint32_t kb = *reinterpret_cast<const uint32_t*>(kp + t * HD + lane * 2);
-        const uint32_t vb = *reinterpret_cast<const uint32_t*>(vp + t * HD + lane * 2);
+        const uint32_t kb = *reinterpret_cast<const uint32_t*>(ks + t * HD + lane * 2);
+        const uint32_t vb = *reinterpret_cast<const uint32_t*>(vs + t * HD + lane * 2);
         const float2 k01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&kb));
         const float2 v01 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&vb));
         kf[0] = k01.x; kf[1] = k01.y;
@@ -248,22 +281,33 @@ __global__ void __launch_bounds__(128) attn_back_pages_kernel(
 #pragma unroll
       for (int k = 0; k < kPer; ++k) dk[k] = dv[k] = 0.f;
       if (t < valid) {
+        // the G heads' two dot products, reduced over the warp together
+        float sv[GMAX], pv[GMAX];
+#pragma unroll
+        for (int r = 0; r < GMAX; ++r) {
+          sv[r] = 0.f;
+          pv[r] = 0.f;
+          if (r < G) {
+#pragma unroll
+            for (int k = 0; k < kPer; ++k) {
+              sv[r] += qr[r][k] * kf[k];
+              pv[r] += dr[r][k] * vf[k];
+            }
+          }
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1)
+#pragma unroll
+          for (int r = 0; r < GMAX; ++r)
+            if (r < G) {
+              sv[r] += __shfl_xor_sync(0xffffffffu, sv[r], off);
+              pv[r] += __shfl_xor_sync(0xffffffffu, pv[r], off);
+            }
 #pragma unroll
         for (int r = 0; r < GMAX; ++r) {
           if (r >= G) break;
-          float s = 0.f, dp = 0.f;
-#pragma unroll
-          for (int k = 0; k < kPer; ++k) {
-            s += qr[r][k] * kf[k];
-            dp += dr[r][k] * vf[k];
-          }
-#pragma unroll
-          for (int off = 16; off > 0; off >>= 1) {
-            s += __shfl_xor_sync(0xffffffffu, s, off);
-            dp += __shfl_xor_sync(0xffffffffu, dp, off);
-          }
-          const float w = expf(s * scale - lse_r[r]);
-          const float ds = w * (dp - D_r[r]);
+          const float w = expf(sv[r] * scale - lse_r[r]);
+          const float ds = w * (pv[r] - D_r[r]);
 #pragma unroll
           for (int k = 0; k < kPer; ++k) {
             dk[k] += ds * scale * qr[r][k];
@@ -298,16 +342,19 @@ __global__ void __launch_bounds__(128) attn_back_pages_kernel(
       }
     }
   }
-  // dq: the four warps' sums, then one atomic add per element
+  // dq: the four warps' sums (in the shared memory the pages occupied), then one atomic add each
+  __syncthreads();
+  float* s_dq = reinterpret_cast<float*>(smem);   // [4][GMAX][HD] <= the page buffer
 #pragma unroll
   for (int r = 0; r < GMAX; ++r)
     if (r < G)
 #pragma unroll
-      for (int k = 0; k < kPer; ++k) s_dq[warp][r][lane * kPer + k] = acc[r][k];
+      for (int k = 0; k < kPer; ++k) s_dq[(warp * GMAX + r) * HD + lane * kPer + k] = acc[r][k];
   __syncthreads();
   for (int i = threadIdx.x; i < G * HD; i += blockDim.x) {
     const int r = i / HD, e = i - r * HD;
-    const float v = s_dq[0][r][e] + s_dq[1][r][e] + s_dq[2][r][e] + s_dq[3][r][e];
+    const float v = s_dq[(0 * GMAX + r) * HD + e] + s_dq[(1 * GMAX + r) * HD + e] + s_dq[(2 * GMAX + r) * HD + e] +
+                    s_dq[(3 * GMAX + r) * HD + e];
     atomicAdd(dq + (static_cast<int64_t>(b) * n_q + g * G + r) * HD + e, v);
   }
 }
@@ -412,9 +459,10 @@ cudaError_t launch_attn_back(const AttnBackArgs& a, cudaStream_t st) {
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || a.n_units == 0) return e;
   const int G = a.n_q / a.n_kv;
+  const size_t smem = a.hd == 128 ? back_pages_smem<128>() : back_pages_smem<64>();
   auto go = [&](auto kern) {
-    kern<<<a.n_units, 128, 0, st>>>(a.units, a.seq_lens, a.block_table, a.max_blocks, a.pool_layer, a.shared, a.q,
-                                    a.dout, a.lse, a.D, a.n_q, a.n_kv, a.grad_layer, a.dq);
+    kern<<<a.n_units, 128, smem, st>>>(a.units, a.seq_lens, a.block_table, a.max_blocks, a.pool_layer, a.shared, a.q,
+                                       a.dout, a.lse, a.D, a.n_q, a.n_kv, a.grad_layer, a.dq, a.err);
   };
   if (a.hd == 128) {
     if (G <= 4)
@@ -432,6 +480,20 @@ cudaError_t launch_attn_back(const AttnBackArgs& a, cudaStream_t st) {
       go(attn_back_pages_kernel<64, 16>);
   }
   return cudaGetLastError();
+}
+
+cudaError_t grad_configure() {
+  cudaError_t e = cudaSuccess;
+  auto set = [&](auto kern, size_t bytes) {
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(bytes));
+  };
+  set(attn_back_pages_kernel<128, 4>, back_pages_smem<128>());
+  set(attn_back_pages_kernel<128, 8>, back_pages_smem<128>());
+  set(attn_back_pages_kernel<128, 16>, back_pages_smem<128>());
+  set(attn_back_pages_kernel<64, 4>, back_pages_smem<64>());
+  set(attn_back_pages_kernel<64, 8>, back_pages_smem<64>());
+  set(attn_back_pages_kernel<64, 16>, back_pages_smem<64>());
+  return e;
 }
 
 cudaError_t launch_rope_back(const float* dq, const float* dks, const float* dvs, const float2* rope, int n, int n_q,

@@ -266,7 +266,11 @@ struct AttnBackArgs {
   const __nv_bfloat16* pool_layer;                   // [n_pages][2][n_kv][16][hd]
   const uint8_t* shared;
   float* grad_layer;                                 // same layout, fp32
+  int* err;                                          // device error word (a bounded wait that gave up)
 };
+// units hold at most this many pages (the pages kernel stages them all in shared memory)
+constexpr int kBackUnitPagesMax = 8;
+cudaError_t grad_configure();
 cudaError_t launch_attn_back(const AttnBackArgs& a, cudaStream_t st);
 cudaError_t launch_rope_back(const float* dq, const float* dks, const float* dvs, const float2* rope, int n, int n_q,
                              int n_kv, int hd, __nv_bfloat16* o_hi, __nv_bfloat16* o_lo, cudaStream_t st);

@@ -1062,7 +1062,7 @@ int score_grad_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, con
   // host plan: work units (candidate, kv head, <= 8 pages) and the pages several candidates read
   std::vector<int4> units;
   std::vector<uint8_t> refs(static_cast<size_t>(n_pages > 0 ? n_pages : 1), 0);
-  constexpr int kUnitPages = 8;
+  constexpr int kUnitPages = kvprm::kBackUnitPagesMax;
   for (int b = 0; b < n; ++b) {
     const int pages = (sl[b] + 15) / 16;
     for (int j = 0; j < pages; ++j) {
@@ -1138,6 +1138,7 @@ int score_grad_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, con
     a.pool_layer = kv_pages ? static_cast<const bf16*>(kv_pages) + l * n_pages * page_elems : nullptr;
     a.shared = g.shared;
     a.grad_layer = grad + l * n_pages * page_elems;
+    a.err = ctx->err_d;
     CK(kvprm::launch_attn_back(a, st), "attention backward");
     if (l == 0) break;   // below layer 0 lies only the verify token's embedding
     // QKV projection: [dq; dk; dv] before RoPE, dx1 = W_qkv^T [...], dh of the layer below
@@ -1220,6 +1221,7 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   }
   CREATE_CK(cu(kvprm::gemm_configure(), "gemm_configure"));
   CREATE_CK(cu(kvprm::attention_configure(), "attention_configure"));
+  CREATE_CK(cu(kvprm::grad_configure(), "grad_configure"));
 
   ModelDims& m = ctx->md;
   m.d = c.d_model;
