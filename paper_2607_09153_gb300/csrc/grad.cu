@@ -359,6 +359,254 @@ __global__ void __launch_bounds__(128) attn_back_pages_kernel(
   }
 }
 
+// ---------------------------------------------------------------- attention backward on the tensor cores
+// The same unit of work (candidate b, kv head g, up to kBackUnitPages pages) for G <= 8 query heads
+// per kv head.  Thread 0 loads the unit's pages with the forward's tensor map (one 128-byte-swizzled
+// box per page: K then V), so each page's keys and values are addressed exactly as in the forward.
+// Each warp takes pages w, w + 4 and per page of 16 tokens computes, with mma.m16n8k16 (bf16 in,
+// fp32 accumulate) -- every fp32 operand entering as a bf16 (hi, lo) pair so that the products keep
+// ~16 bits:
+//   S  = Q K^T and dP = dO V^T   A = q (or dO) with the hi parts in rows 0..7 and the lo parts in
+//                                rows 8..15 of the same heads (their sum is the product), B = K or V
+//                                from shared memory (ldmatrix);
+//   w = exp(S / sqrt(hd) - lse), ds = w (dP - D) / sqrt(hd)     in registers, row = head;
+//   dq += ds K                   A = ds (hi rows 0..7, lo rows 8..15), B = K through ldmatrix.trans;
+//   dV = w^T dO, dK = ds^T Q     contractions over the heads: w and ds go through movmatrix (an 8x8
+//                                transpose in registers) into A fragments whose k columns 0..7 hold
+//                                the heads' hi parts and 8..15 their lo parts; B holds [dO_hi; dO_hi]
+//                                for one MMA and [dO_lo; 0] for a second, so the sum is
+//                                w_hi dO_hi + w_lo dO_hi + w_hi dO_lo (the lo x lo term, ~2^-16 of the
+//                                product, is left out);
+// then stores the page's dK and dV rows (or adds them atomically on a shared page).
+template <int HD>
+struct BackTcSmem {
+  static constexpr uint32_t kBlock = (HD / 64) * 16 * 128;   // one page's K (or V) of one kv head
+  static constexpr uint32_t kPage = 2 * kBlock;
+  static constexpr uint32_t kPages = 0;                      // [pages][K, V], as the forward's box lands
+  static constexpr int kLd = HD + 8;                          // padded row of the B matrices (elements)
+  static constexpr uint32_t kB = kPages + kBackUnitPages * kPage;   // [4][16][kLd] bf16: Q hh, Q l0, dO hh, dO l0
+  static constexpr uint32_t kBar = kB + 4 * 16 * kLd * 2;
+  static constexpr size_t kBytes = kBar + 16 + 1024;          // + alignment slack
+};
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~static_cast<uintptr_t>(1023));
+}
+
+__device__ __forceinline__ uint32_t movmatrix_trans(uint32_t a) {
+  uint32_t d;
+  asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(d) : "r"(a));
+  return d;
+}
+
+__device__ __forceinline__ float bf16_hi(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
+
+template <int HD>
+__global__ void __launch_bounds__(128) attn_back_tc_kernel(
+    const __grid_constant__ CUtensorMap tm_pool, int64_t layer_page0, const int4* __restrict__ units,
+    const int32_t* __restrict__ seq_lens, const int32_t* __restrict__ block_table, int max_blocks,
+    const uint8_t* __restrict__ shared, const float* __restrict__ q, const float* __restrict__ dout,
+    const float* __restrict__ lse, const float* __restrict__ D, int n_q, int n_kv, float* __restrict__ grad_layer,
+    float* __restrict__ dq, int* err) {
+  using SM = BackTcSmem<HD>;
+  constexpr int KS = HD / 16;   // 16-wide steps over the head dimension
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* base = align1024(smem_raw);
+  uint64_t* bar = reinterpret_cast<uint64_t*>(base + SM::kBar);
+  bf16* Bq_hh = reinterpret_cast<bf16*>(base + SM::kB);   // rows 0..7 q_hi of the heads, rows 8..15 q_hi again
+  bf16* Bq_l0 = Bq_hh + 16 * SM::kLd;                     // rows 0..7 q_lo, rows 8..15 zero
+  bf16* Bd_hh = Bq_l0 + 16 * SM::kLd;                     // the same for dO
+  bf16* Bd_l0 = Bd_hh + 16 * SM::kLd;
+  const int4 u = units[blockIdx.x];
+  const int b = u.x, g = u.y, j0 = u.z, npg = u.w - u.z;
+  const int G = n_q / n_kv;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, gid = lane >> 2, tig = lane & 3;
+  const float scale = rsqrtf(static_cast<float>(HD));
+  const int L = seq_lens[b];
+  const int64_t page_elems = static_cast<int64_t>(2) * n_kv * 16 * HD;
+  const int64_t row0 = static_cast<int64_t>(b) * n_q + static_cast<int64_t>(g) * G;   // the group's first row
+  if (threadIdx.x == 0) {
+    mbar_init(bar, 1);
+    fence_mbar_init();
+    tma_prefetch_desc(&tm_pool);
+    mbar_arrive_expect_tx(bar, static_cast<uint32_t>(npg) * SM::kPage);
+    const uint64_t pol = policy_evict_first();
+    for (int i = 0; i < npg; ++i) {
+      const int32_t p = block_table[static_cast<int64_t>(b) * max_blocks + j0 + i];
+      tma_load_5d(base + SM::kPages + i * SM::kPage, &tm_pool, bar, 0, 0, 0, g,
+                  static_cast<int32_t>(2 * (layer_page0 + p)), pol);
+    }
+  }
+  // the B matrices of dV and dK: [16 k rows][HD] bf16, k = head (hi parts twice, or lo parts then zeros)
+  for (int i = threadIdx.x; i < 16 * HD; i += blockDim.x) {
+    const int k = i / HD, e = i - k * HD, h = k & 7;
+    const bool ok = h < G;
+    const float qv = ok ? q[(row0 + h) * HD + e] : 0.f, dv = ok ? dout[(row0 + h) * HD + e] : 0.f;
+    const float qh = bf16_hi(qv), dh = bf16_hi(dv);
+    Bq_hh[k * SM::kLd + e] = __float2bfloat16_rn(qh);
+    Bd_hh[k * SM::kLd + e] = __float2bfloat16_rn(dh);
+    Bq_l0[k * SM::kLd + e] = __float2bfloat16_rn(k < 8 ? qv - qh : 0.f);
+    Bd_l0[k * SM::kLd + e] = __float2bfloat16_rn(k < 8 ? dv - dh : 0.f);
+  }
+  // A fragments of q and dO for S and dP: row gid the hi part, row gid + 8 the lo part of head gid
+  uint32_t qa[KS][4], da[KS][4];
+  {
+    const bool ok = gid < G;
+    const float* qr = q + (row0 + gid) * HD;
+    const float* dr = dout + (row0 + gid) * HD;
+#pragma unroll
+    for (int ks = 0; ks < KS; ++ks) {
+      const int c = ks * 16 + tig * 2;
+      float qv[4], dv[4];
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        const int cc = c + (t & 1) + 8 * (t >> 1);
+        qv[t] = ok ? qr[cc] : 0.f;
+        dv[t] = ok ? dr[cc] : 0.f;
+      }
+      qa[ks][0] = pack_bf16(qv[0], qv[1]);
+      qa[ks][1] = pack_bf16(qv[0] - bf16_hi(qv[0]), qv[1] - bf16_hi(qv[1]));
+      qa[ks][2] = pack_bf16(qv[2], qv[3]);
+      qa[ks][3] = pack_bf16(qv[2] - bf16_hi(qv[2]), qv[3] - bf16_hi(qv[3]));
+      da[ks][0] = pack_bf16(dv[0], dv[1]);
+      da[ks][1] = pack_bf16(dv[0] - bf16_hi(dv[0]), dv[1] - bf16_hi(dv[1]));
+      da[ks][2] = pack_bf16(dv[2], dv[3]);
+      da[ks][3] = pack_bf16(dv[2] - bf16_hi(dv[2]), dv[3] - bf16_hi(dv[3]));
+    }
+  }
+  const float lse_g = gid < G ? lse[row0 + gid] : 0.f;
+  const float D_g = gid < G ? D[row0 + gid] : 0.f;
+  float dqa[HD / 8][4];
+#pragma unroll
+  for (int n = 0; n < HD / 8; ++n) dqa[n][0] = dqa[n][1] = dqa[n][2] = dqa[n][3] = 0.f;
+  __syncthreads();   // the barrier is initialised and the B matrices are written
+  if (!__all_sync(0xffffffffu, mbar_wait(bar, 0, err))) {
+    // gave up (the error word is set): wait, bounded again, for the copies still landing in this
+    // CTA's shared memory before leaving
+    mbar_wait(bar, 0, err);
+    return;
+  }
+  const int mi = lane >> 3;
+  for (int i = warp; i < npg; i += 4) {
+    const int j = j0 + i;
+    const int32_t p = block_table[static_cast<int64_t>(b) * max_blocks + j];
+    const int valid = min(16, L - 16 * j);
+    const uint32_t kbase = smem_u32(base + SM::kPages + i * SM::kPage), vbase = kbase + SM::kBlock;
+    // S = Q K^T and dP = dO V^T over the page's 16 tokens (two n-tiles of 8)
+    float s0[4] = {0.f, 0.f, 0.f, 0.f}, s1[4] = {0.f, 0.f, 0.f, 0.f};
+    float p0[4] = {0.f, 0.f, 0.f, 0.f}, p1[4] = {0.f, 0.f, 0.f, 0.f};
+    {
+      const int tok = (mi >> 1) * 8 + (lane & 7);
+#pragma unroll
+      for (int ks = 0; ks < KS; ++ks) {
+        const int hdc = ks * 16 + (mi & 1) * 8;
+        const uint32_t off = (hdc >> 6) * 2048 + tok * 128 + ((((hdc & 63) >> 3) ^ (tok & 7)) << 4);
+        uint32_t kb[4], vb[4];
+        ldsm_x4(kbase + off, kb[0], kb[1], kb[2], kb[3]);
+        ldsm_x4(vbase + off, vb[0], vb[1], vb[2], vb[3]);
+        mma_bf16_16816(s0, qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], kb[0], kb[1]);
+        mma_bf16_16816(s1, qa[ks][0], qa[ks][1], qa[ks][2], qa[ks][3], kb[2], kb[3]);
+        mma_bf16_16816(p0, da[ks][0], da[ks][1], da[ks][2], da[ks][3], vb[0], vb[1]);
+        mma_bf16_16816(p1, da[ks][0], da[ks][1], da[ks][2], da[ks][3], vb[2], vb[3]);
+      }
+    }
+    // head gid, tokens tig*2, tig*2 + 1, 8 + tig*2, 9 + tig*2: the hi and lo rows summed
+    const float x[4] = {s0[0] + s0[2], s0[1] + s0[3], s1[0] + s1[2], s1[1] + s1[3]};
+    const float dp[4] = {p0[0] + p0[2], p0[1] + p0[3], p1[0] + p1[2], p1[1] + p1[3]};
+    float w[4], ds[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const int t = (e & 1) + tig * 2 + 8 * (e >> 1);
+      w[e] = (gid < G && t < valid) ? expf(x[e] * scale - lse_g) : 0.f;
+      ds[e] = w[e] * (dp[e] - D_g) * scale;
+    }
+    float wl[4], dl[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      wl[e] = w[e] - bf16_hi(w[e]);
+      dl[e] = ds[e] - bf16_hi(ds[e]);
+    }
+    // dq += ds K (K as the k x n operand through ldmatrix.trans, as V in the forward's P V)
+    {
+      const uint32_t a0 = pack_bf16(ds[0], ds[1]), a1 = pack_bf16(dl[0], dl[1]);
+      const uint32_t a2 = pack_bf16(ds[2], ds[3]), a3 = pack_bf16(dl[2], dl[3]);
+      const int tok = (mi & 1) * 8 + (lane & 7);
+#pragma unroll
+      for (int j2 = 0; j2 < HD / 16; ++j2) {
+        const int hdc = j2 * 16 + (mi >> 1) * 8;
+        uint32_t kb[4];
+        ldsm_x4_t(kbase + (hdc >> 6) * 2048 + tok * 128 + ((((hdc & 63) >> 3) ^ (tok & 7)) << 4), kb[0], kb[1],
+                  kb[2], kb[3]);
+        mma_bf16_16816(dqa[2 * j2], a0, a1, a2, a3, kb[0], kb[1]);
+        mma_bf16_16816(dqa[2 * j2 + 1], a0, a1, a2, a3, kb[2], kb[3]);
+      }
+    }
+    // w^T and ds^T as A fragments: rows = tokens, k 0..7 = the heads' hi parts, 8..15 their lo parts
+    const uint32_t wt0 = movmatrix_trans(pack_bf16(w[0], w[1])), wt1 = movmatrix_trans(pack_bf16(w[2], w[3]));
+    const uint32_t wt2 = movmatrix_trans(pack_bf16(wl[0], wl[1])), wt3 = movmatrix_trans(pack_bf16(wl[2], wl[3]));
+    const uint32_t st0 = movmatrix_trans(pack_bf16(ds[0], ds[1])), st1 = movmatrix_trans(pack_bf16(ds[2], ds[3]));
+    const uint32_t st2 = movmatrix_trans(pack_bf16(dl[0], dl[1])), st3 = movmatrix_trans(pack_bf16(dl[2], dl[3]));
+    float* gk = grad_layer + p * page_elems + static_cast<int64_t>(g) * 16 * HD;
+    float* gv = gk + static_cast<int64_t>(n_kv) * 16 * HD;
+    const bool sh = shared[p] != 0;
+    auto put = [&](float* dst, float a, float c) {
+      if (sh)
+        atomicAdd(reinterpret_cast<float2*>(dst), make_float2(a, c));
+      else
+        *reinterpret_cast<float2*>(dst) = make_float2(a, c);
+    };
+    {
+      const int krow = (mi & 1) * 8 + (lane & 7);
+#pragma unroll
+      for (int j2 = 0; j2 < HD / 16; ++j2) {
+        const int col = j2 * 16 + (mi >> 1) * 8;
+        uint32_t dh[4], dlo[4], qh[4], ql[4];
+        ldsm_x4_t(smem_u32(Bd_hh + krow * SM::kLd + col), dh[0], dh[1], dh[2], dh[3]);
+        ldsm_x4_t(smem_u32(Bd_l0 + krow * SM::kLd + col), dlo[0], dlo[1], dlo[2], dlo[3]);
+        ldsm_x4_t(smem_u32(Bq_hh + krow * SM::kLd + col), qh[0], qh[1], qh[2], qh[3]);
+        ldsm_x4_t(smem_u32(Bq_l0 + krow * SM::kLd + col), ql[0], ql[1], ql[2], ql[3]);
+        float v0[4] = {0.f, 0.f, 0.f, 0.f}, v1[4] = {0.f, 0.f, 0.f, 0.f};
+        float k0[4] = {0.f, 0.f, 0.f, 0.f}, k1[4] = {0.f, 0.f, 0.f, 0.f};
+        mma_bf16_16816(v0, wt0, wt1, wt2, wt3, dh[0], dh[1]);
+        mma_bf16_16816(v0, wt0, wt1, wt2, wt3, dlo[0], dlo[1]);
+        mma_bf16_16816(v1, wt0, wt1, wt2, wt3, dh[2], dh[3]);
+        mma_bf16_16816(v1, wt0, wt1, wt2, wt3, dlo[2], dlo[3]);
+        mma_bf16_16816(k0, st0, st1, st2, st3, qh[0], qh[1]);
+        mma_bf16_16816(k0, st0, st1, st2, st3, ql[0], ql[1]);
+        mma_bf16_16816(k1, st0, st1, st2, st3, qh[2], qh[3]);
+        mma_bf16_16816(k1, st0, st1, st2, st3, ql[2], ql[3]);
+        // C rows: token gid (elements 0, 1) and gid + 8 (2, 3); columns of the two n-tiles
+        const int c0 = j2 * 16 + tig * 2, c1 = c0 + 8;
+        put(gv + gid * HD + c0, v0[0], v0[1]);
+        put(gv + (gid + 8) * HD + c0, v0[2], v0[3]);
+        put(gv + gid * HD + c1, v1[0], v1[1]);
+        put(gv + (gid + 8) * HD + c1, v1[2], v1[3]);
+        put(gk + gid * HD + c0, k0[0], k0[1]);
+        put(gk + (gid + 8) * HD + c0, k0[2], k0[3]);
+        put(gk + gid * HD + c1, k1[0], k1[1]);
+        put(gk + (gid + 8) * HD + c1, k1[2], k1[3]);
+      }
+    }
+  }
+  // dq: rows gid (hi) and gid + 8 (lo) of head gid summed, the four warps' parts through shared
+  // memory (the page buffer, no longer read), then one atomic add per element
+  __syncthreads();
+  float* s_dq = reinterpret_cast<float*>(base);   // [4][8][HD] <= the page buffer
+#pragma unroll
+  for (int n = 0; n < HD / 8; ++n) {
+    const int c = n * 8 + tig * 2;
+    s_dq[(warp * 8 + gid) * HD + c] = dqa[n][0] + dqa[n][2];
+    s_dq[(warp * 8 + gid) * HD + c + 1] = dqa[n][1] + dqa[n][3];
+  }
+  __syncthreads();
+  for (int i2 = threadIdx.x; i2 < G * HD; i2 += blockDim.x) {
+    const int r = i2 / HD, e = i2 - r * HD;
+    const float v = s_dq[(0 * 8 + r) * HD + e] + s_dq[(1 * 8 + r) * HD + e] + s_dq[(2 * 8 + r) * HD + e] +
+                    s_dq[(3 * 8 + r) * HD + e];
+    atomicAdd(dq + (row0 + r) * HD + e, v);
+  }
+}
+
 // One CTA per row: [dq; dk; dv] before RoPE (the rotation by the negative angle of position L_b)
 // as the bf16 hi/lo input of the W_qkv^T product, [n][(n_q + 2 n_kv) hd].
 __global__ void rope_back_kernel(const float* __restrict__ dq, const float* __restrict__ dks,
@@ -459,6 +707,17 @@ cudaError_t launch_attn_back(const AttnBackArgs& a, cudaStream_t st) {
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || a.n_units == 0) return e;
   const int G = a.n_q / a.n_kv;
+  if (G <= 8 && a.tm_pool) {   // the tensor-core backward
+    if (a.hd == 128)
+      attn_back_tc_kernel<128><<<a.n_units, 128, BackTcSmem<128>::kBytes, st>>>(
+          *a.tm_pool, a.layer_page0, a.units, a.seq_lens, a.block_table, a.max_blocks, a.shared, a.q, a.dout, a.lse,
+          a.D, a.n_q, a.n_kv, a.grad_layer, a.dq, a.err);
+    else
+      attn_back_tc_kernel<64><<<a.n_units, 128, BackTcSmem<64>::kBytes, st>>>(
+          *a.tm_pool, a.layer_page0, a.units, a.seq_lens, a.block_table, a.max_blocks, a.shared, a.q, a.dout, a.lse,
+          a.D, a.n_q, a.n_kv, a.grad_layer, a.dq, a.err);
+    return cudaGetLastError();
+  }
   const size_t smem = a.hd == 128 ? back_pages_smem<128>() : back_pages_smem<64>();
   auto go = [&](auto kern) {
     kern<<<a.n_units, 128, smem, st>>>(a.units, a.seq_lens, a.block_table, a.max_blocks, a.pool_layer, a.shared, a.q,
@@ -493,6 +752,8 @@ cudaError_t grad_configure() {
   set(attn_back_pages_kernel<64, 4>, back_pages_smem<64>());
   set(attn_back_pages_kernel<64, 8>, back_pages_smem<64>());
   set(attn_back_pages_kernel<64, 16>, back_pages_smem<64>());
+  set(attn_back_tc_kernel<128>, BackTcSmem<128>::kBytes);
+  set(attn_back_tc_kernel<64>, BackTcSmem<64>::kBytes);
   return e;
 }
 

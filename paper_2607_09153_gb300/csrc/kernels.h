@@ -267,6 +267,10 @@ struct AttnBackArgs {
   const uint8_t* shared;
   float* grad_layer;                                 // same layout, fp32
   int* err;                                          // device error word (a bounded wait that gave up)
+  // the pool's tensor map (the forward's, one box per page) and this layer's first page unit; with
+  // group <= 8 the backward then runs on the tensor cores, else (or when NULL) on the CUDA cores
+  const CUtensorMap* tm_pool = nullptr;
+  int64_t layer_page0 = 0;
 };
 // units hold at most this many pages (the pages kernel stages them all in shared memory)
 constexpr int kBackUnitPagesMax = 8;

@@ -199,6 +199,7 @@ struct kvprm_ctx {
   int inject_fail = 0;
   int* probe_flag = nullptr;
   GradState grad;
+  bool grad_cuda_cores = false;   // KVPRM_GRAD_CUDA_CORES=1: the attention backward on the CUDA cores
 };
 
 namespace {
@@ -1139,6 +1140,8 @@ int score_grad_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, con
     a.shared = g.shared;
     a.grad_layer = grad + l * n_pages * page_elems;
     a.err = ctx->err_d;
+    a.tm_pool = kv_pages && !ctx->grad_cuda_cores ? &ctx->tm_pool : nullptr;   // the forward's map of this pool
+    a.layer_page0 = static_cast<int64_t>(l) * n_pages;
     CK(kvprm::launch_attn_back(a, st), "attention backward");
     if (l == 0) break;   // below layer 0 lies only the verify token's embedding
     // QKV projection: [dq; dk; dv] before RoPE, dx1 = W_qkv^T [...], dh of the layer below
@@ -1345,6 +1348,7 @@ int kvprm_create(const kvprm_config* cfg, const kvprm_weights* w, kvprm_ctx** ou
   CREATE_CK(cu(cudaEventCreateWithFlags(&ctx->pool_free, cudaEventDisableTiming), "cudaEventCreate"));
   ctx->use_graph = !env_off("KVPRM_NO_GRAPH");
   ctx->use_pdl = !env_off("KVPRM_NO_PDL");
+  ctx->grad_cuda_cores = env_off("KVPRM_GRAD_CUDA_CORES");
   // shared pages: on the tensor cores at head_dim 128, else one warp per candidate
   ctx->fuse_combine = !env_off("KVPRM_NO_FUSED_COMBINE");
   ctx->share_mode = env_off("KVPRM_NO_SHARING")
