@@ -474,7 +474,15 @@ def summarize(w, m: dict, world: int) -> dict:
     call_s = m["ms"] / m["steps"] / 1000.0
     logical = w.logical_kv_bytes()
     kv_tok = a.kv_bytes_per_token()
+    # with the combine (the split partials' merge) counted in the attention step's time
+    comb_n, comb_ms = prof.get("combine", (0, 0.0))
+    attn_comb_s = (attn["time_per_layer_us"] * 1e-6 + comb_ms / layers_timed / 1000.0) if comb_n else None
     attention_obj = {"achieved_gbs": attn["achieved"], "frac_of_8tbs": attn["frac_of_8tbs"],
+                     "with_combine": {"time_per_layer_us": round(attn_comb_s * 1e6, 3),
+                                      "frac_of_8tbs": round(alg["attention"] / a.n_layers / attn_comb_s / 1e9
+                                                            / HBM_NOMINAL_GBS, 4)} if attn_comb_s else
+                     {"time_per_layer_us": attn["time_per_layer_us"], "frac_of_8tbs": attn["frac_of_8tbs"],
+                      "note": "combine inside the attention launch (fused plan)"},
                      "frac_of_measured": attn["frac"], "unique_kv_bytes_per_step": alg["attention"],
                      "logical_kv_bytes_per_step": int(logical),
                      "logical_gbs": round(logical / a.n_layers / (attn["time_per_layer_us"] * 1e-6) / 1e9, 1),
@@ -596,7 +604,8 @@ def run_gpu(args, world, rank, local):
             else:
                 entry["attention"] = {k: so["attention"][k] for k in ("achieved_gbs", "frac_of_8tbs", "frac_of_measured",
                                                                      "time_per_layer_us", "pipelined_us_per_layer",
-                                                                     "pipelined_frac_of_8tbs", "kernels")}
+                                                                     "pipelined_frac_of_8tbs", "with_combine",
+                                                                     "kernels")}
                 entry["roofline"] = so["roofline"]
             entry["config"] = workload_config(wo, args)
             entry["clocks"] = mo["clocks"]

@@ -16,6 +16,8 @@
 // (hi, lo) pair like the forward's activations.
 #include <cuda_bf16.h>
 
+#include <utility>
+
 #include "kernels.h"
 #include "ptx.cuh"
 
@@ -70,6 +72,8 @@ __global__ void head_back_kernel(const float* __restrict__ h, const float* __res
                                  const bf16* __restrict__ w_minus, int d, float eps, float* __restrict__ dh,
                                  bf16* __restrict__ dh_hi, bf16* __restrict__ dh_lo) {
   __shared__ float2 red[32];
+  grid_dep_launch();
+  grid_dep_wait();   // every input is written by earlier kernels of the stream
   const int b = blockIdx.x;
   const float* hb = h + static_cast<int64_t>(b) * d;
   const float q = 1.f - p_plus[b];   // d(-log P)/dz_- = 1 - P = -d(-log P)/dz_+
@@ -97,6 +101,8 @@ __global__ void rms_back_kernel(const float* __restrict__ h, const bf16* __restr
                                 const bf16* __restrict__ gain, const float* __restrict__ dy, const float* dres, int d,
                                 float eps, float* out, bf16* __restrict__ o_hi, bf16* __restrict__ o_lo) {
   __shared__ float2 red[32];
+  grid_dep_launch();
+  grid_dep_wait();
   const int b = blockIdx.x;
   const int64_t row = static_cast<int64_t>(b) * d;
   float ss = 0.f, sd = 0.f;
@@ -119,6 +125,8 @@ __global__ void rms_back_kernel(const float* __restrict__ h, const bf16* __restr
 // da [n][ff], gu [n][2 ff] (gate then up pre-activations) -> [du; dt] [n][2 ff] as hi/lo
 __global__ void silu_back_kernel(const float* __restrict__ da, const float* __restrict__ gu, int n, int ff,
                                  bf16* __restrict__ o_hi, bf16* __restrict__ o_lo) {
+  grid_dep_launch();
+  grid_dep_wait();
   const int64_t total = static_cast<int64_t>(n) * ff;
   for (int64_t e = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; e < total;
        e += static_cast<int64_t>(gridDim.x) * blockDim.x) {
@@ -140,6 +148,8 @@ __global__ void attn_back_pre_kernel(const float* __restrict__ q, const float* _
                                      int hd, float* __restrict__ D, float* __restrict__ dq, float* __restrict__ dks,
                                      float* __restrict__ dvs) {
   __shared__ float s_w[kMaxGroup], s_ds[kMaxGroup];
+  grid_dep_launch();
+  grid_dep_wait();
   const int b = blockIdx.x / n_kv, g = blockIdx.x % n_kv, G = n_q / n_kv;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float scale = rsqrtf(static_cast<float>(hd));
@@ -207,6 +217,8 @@ __global__ void __launch_bounds__(128) attn_back_pages_kernel(
   extern __shared__ __align__(16) uint8_t smem[];
   bf16* s_kv = reinterpret_cast<bf16*>(smem);   // [page][K, V][16][HD]
   uint64_t* bar = reinterpret_cast<uint64_t*>(smem + static_cast<size_t>(kBackUnitPages) * 2 * kBlock);
+  grid_dep_launch();
+  grid_dep_wait();
   const int4 u = units[blockIdx.x];
   const int b = u.x, g = u.y, j0 = u.z, j1 = u.w;
   const int npg = j1 - j0;   // 1 .. kBackUnitPages
@@ -437,6 +449,10 @@ __global__ void __launch_bounds__(128) attn_back_tc_kernel(
                   static_cast<int32_t>(2 * (layer_page0 + p)), pol);
     }
   }
+  // the pages (an input of the whole pass) are in flight; q, dO, lse and D may be written by the
+  // kernels just before this one
+  grid_dep_launch();
+  grid_dep_wait();
   // the B matrices of dV and dK: [16 k rows][HD] bf16, k = head (hi parts twice, or lo parts then zeros)
   for (int i = threadIdx.x; i < 16 * HD; i += blockDim.x) {
     const int k = i / HD, e = i - k * HD, h = k & 7;
@@ -612,6 +628,8 @@ __global__ void __launch_bounds__(128) attn_back_tc_kernel(
 __global__ void rope_back_kernel(const float* __restrict__ dq, const float* __restrict__ dks,
                                  const float* __restrict__ dvs, const float2* __restrict__ rope, int n_q, int n_kv,
                                  int hd, bf16* __restrict__ o_hi, bf16* __restrict__ o_lo) {
+  grid_dep_launch();
+  grid_dep_wait();
   const int b = blockIdx.x, half = hd / 2;
   const int rows = (n_q + 2 * n_kv) * hd;
   const int64_t ob = static_cast<int64_t>(b) * rows;
@@ -631,6 +649,8 @@ __global__ void rope_back_kernel(const float* __restrict__ dq, const float* __re
 // Zero every layer's gradient of the listed pages.
 __global__ void zero_pages_kernel(float* __restrict__ grad, const int32_t* __restrict__ pages, int n_list,
                                   int n_layers, int64_t n_pages, int64_t page_elems) {
+  grid_dep_launch();
+  grid_dep_wait();
   const int64_t per = page_elems / 4;
   const int64_t total = static_cast<int64_t>(n_list) * n_layers * per;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
@@ -646,6 +666,8 @@ __global__ void zero_pages_kernel(float* __restrict__ grad, const int32_t* __res
 __global__ void steer_update_kernel(bf16* __restrict__ kv, const float* __restrict__ grad,
                                     const int32_t* __restrict__ pages, int n_list, int n_layers, int64_t n_pages,
                                     int64_t page_elems, float eta) {
+  grid_dep_launch();
+  grid_dep_wait();
   const int64_t per = page_elems / 4;
   const int64_t total = static_cast<int64_t>(n_list) * n_layers * per;
   for (int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; i < total;
@@ -663,6 +685,23 @@ __global__ void steer_update_kernel(bf16* __restrict__ kv, const float* __restri
     raw.y = *reinterpret_cast<const uint32_t*>(&nc);
     *reinterpret_cast<uint2*>(kv + base) = raw;
   }
+}
+
+// Launch with programmatic dependent launch: the kernel may start while the previous one in the
+// stream drains; every kernel here waits (griddepcontrol.wait) before touching what that one writes.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
 }
 
 unsigned grid_1d(int64_t total, int threads) {
@@ -683,45 +722,42 @@ cudaError_t launch_transpose(const __nv_bfloat16* in, __nv_bfloat16* out, int ro
 cudaError_t launch_head_back(const float* h, const float* p_plus, const __nv_bfloat16* gain,
                              const __nv_bfloat16* w_plus, const __nv_bfloat16* w_minus, int n, int d, float eps,
                              float* dh, __nv_bfloat16* dh_hi, __nv_bfloat16* dh_lo, cudaStream_t st) {
-  head_back_kernel<<<n, 256, 0, st>>>(h, p_plus, gain, w_plus, w_minus, d, eps, dh, dh_hi, dh_lo);
-  return cudaGetLastError();
+  return launch_pdl(head_back_kernel, dim3(n), dim3(256), 0, st, h, p_plus, gain, w_plus, w_minus, d, eps, dh, dh_hi,
+                    dh_lo);
 }
 
 cudaError_t launch_rms_back(const float* h, const __nv_bfloat16* h_bf16, const __nv_bfloat16* gain, const float* dy,
                             const float* dres, int n, int d, float eps, float* out, __nv_bfloat16* o_hi,
                             __nv_bfloat16* o_lo, cudaStream_t st) {
-  rms_back_kernel<<<n, 256, 0, st>>>(h, h_bf16, gain, dy, dres, d, eps, out, o_hi, o_lo);
-  return cudaGetLastError();
+  return launch_pdl(rms_back_kernel, dim3(n), dim3(256), 0, st, h, h_bf16, gain, dy, dres, d, eps, out, o_hi, o_lo);
 }
 
 cudaError_t launch_silu_back(const float* da, const float* gu, int n, int ff, __nv_bfloat16* o_hi,
                              __nv_bfloat16* o_lo, cudaStream_t st) {
-  silu_back_kernel<<<grid_1d(static_cast<int64_t>(n) * ff, 256), 256, 0, st>>>(da, gu, n, ff, o_hi, o_lo);
-  return cudaGetLastError();
+  return launch_pdl(silu_back_kernel, dim3(grid_1d(static_cast<int64_t>(n) * ff, 256)), dim3(256), 0, st, da, gu, n,
+                    ff, o_hi, o_lo);
 }
 
 cudaError_t launch_attn_back(const AttnBackArgs& a, cudaStream_t st) {
   if (a.n_q / a.n_kv > kMaxGroup || (a.hd != 64 && a.hd != 128)) return cudaErrorInvalidValue;
-  attn_back_pre_kernel<<<a.n * a.n_kv, 128, 0, st>>>(a.q, a.kself, a.vself, a.o, a.dout, a.lse, a.n_q, a.n_kv, a.hd,
-                                                     a.D, a.dq, a.dks, a.dvs);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch_pdl(attn_back_pre_kernel, dim3(a.n * a.n_kv), dim3(128), 0, st, a.q, a.kself, a.vself, a.o,
+                             a.dout, a.lse, a.n_q, a.n_kv, a.hd, a.D, a.dq, a.dks, a.dvs);
   if (e != cudaSuccess || a.n_units == 0) return e;
   const int G = a.n_q / a.n_kv;
   if (G <= 8 && a.tm_pool) {   // the tensor-core backward
     if (a.hd == 128)
-      attn_back_tc_kernel<128><<<a.n_units, 128, BackTcSmem<128>::kBytes, st>>>(
-          *a.tm_pool, a.layer_page0, a.units, a.seq_lens, a.block_table, a.max_blocks, a.shared, a.q, a.dout, a.lse,
-          a.D, a.n_q, a.n_kv, a.grad_layer, a.dq, a.err);
-    else
-      attn_back_tc_kernel<64><<<a.n_units, 128, BackTcSmem<64>::kBytes, st>>>(
-          *a.tm_pool, a.layer_page0, a.units, a.seq_lens, a.block_table, a.max_blocks, a.shared, a.q, a.dout, a.lse,
-          a.D, a.n_q, a.n_kv, a.grad_layer, a.dq, a.err);
-    return cudaGetLastError();
+      return launch_pdl(attn_back_tc_kernel<128>, dim3(a.n_units), dim3(128), BackTcSmem<128>::kBytes, st, *a.tm_pool,
+                        a.layer_page0, a.units, a.seq_lens, a.block_table, a.max_blocks, a.shared, a.q, a.dout, a.lse,
+                        a.D, a.n_q, a.n_kv, a.grad_layer, a.dq, a.err);
+    return launch_pdl(attn_back_tc_kernel<64>, dim3(a.n_units), dim3(128), BackTcSmem<64>::kBytes, st, *a.tm_pool,
+                      a.layer_page0, a.units, a.seq_lens, a.block_table, a.max_blocks, a.shared, a.q, a.dout, a.lse,
+                      a.D, a.n_q, a.n_kv, a.grad_layer, a.dq, a.err);
   }
   const size_t smem = a.hd == 128 ? back_pages_smem<128>() : back_pages_smem<64>();
+  cudaError_t le = cudaSuccess;
   auto go = [&](auto kern) {
-    kern<<<a.n_units, 128, smem, st>>>(a.units, a.seq_lens, a.block_table, a.max_blocks, a.pool_layer, a.shared, a.q,
-                                       a.dout, a.lse, a.D, a.n_q, a.n_kv, a.grad_layer, a.dq, a.err);
+    le = launch_pdl(kern, dim3(a.n_units), dim3(128), smem, st, a.units, a.seq_lens, a.block_table, a.max_blocks,
+                    a.pool_layer, a.shared, a.q, a.dout, a.lse, a.D, a.n_q, a.n_kv, a.grad_layer, a.dq, a.err);
   };
   if (a.hd == 128) {
     if (G <= 4)
@@ -738,7 +774,7 @@ cudaError_t launch_attn_back(const AttnBackArgs& a, cudaStream_t st) {
     else
       go(attn_back_pages_kernel<64, 16>);
   }
-  return cudaGetLastError();
+  return le;
 }
 
 cudaError_t grad_configure() {
@@ -759,24 +795,21 @@ cudaError_t grad_configure() {
 
 cudaError_t launch_rope_back(const float* dq, const float* dks, const float* dvs, const float2* rope, int n, int n_q,
                              int n_kv, int hd, __nv_bfloat16* o_hi, __nv_bfloat16* o_lo, cudaStream_t st) {
-  rope_back_kernel<<<n, 256, 0, st>>>(dq, dks, dvs, rope, n_q, n_kv, hd, o_hi, o_lo);
-  return cudaGetLastError();
+  return launch_pdl(rope_back_kernel, dim3(n), dim3(256), 0, st, dq, dks, dvs, rope, n_q, n_kv, hd, o_hi, o_lo);
 }
 
 cudaError_t launch_zero_pages(float* grad, const int32_t* pages, int n_list, int n_layers, int64_t n_pages,
                               int64_t page_elems, cudaStream_t st) {
   if (n_list == 0) return cudaSuccess;
-  zero_pages_kernel<<<grid_1d(static_cast<int64_t>(n_list) * n_layers * (page_elems / 4), 256), 256, 0, st>>>(
-      grad, pages, n_list, n_layers, n_pages, page_elems);
-  return cudaGetLastError();
+  return launch_pdl(zero_pages_kernel, dim3(grid_1d(static_cast<int64_t>(n_list) * n_layers * (page_elems / 4), 256)),
+                    dim3(256), 0, st, grad, pages, n_list, n_layers, n_pages, page_elems);
 }
 
 cudaError_t launch_steer_update(__nv_bfloat16* kv, const float* grad, const int32_t* pages, int n_list, int n_layers,
                                 int64_t n_pages, int64_t page_elems, float eta, cudaStream_t st) {
   if (n_list == 0) return cudaSuccess;
-  steer_update_kernel<<<grid_1d(static_cast<int64_t>(n_list) * n_layers * (page_elems / 4), 256), 256, 0, st>>>(
-      kv, grad, pages, n_list, n_layers, n_pages, page_elems, eta);
-  return cudaGetLastError();
+  return launch_pdl(steer_update_kernel, dim3(grid_1d(static_cast<int64_t>(n_list) * n_layers * (page_elems / 4), 256)),
+                    dim3(256), 0, st, kv, grad, pages, n_list, n_layers, n_pages, page_elems, eta);
 }
 
 }  // namespace kvprm

@@ -1098,7 +1098,7 @@ int score_grad_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, con
     ep.M = M;
     ep.n_valid = n;
     ep.out = out;
-    return kvprm::launch_gemm(gp, w, xh, xl, ep, np, ctx->err_d, st, false);
+    return kvprm::launch_gemm(gp, w, xh, xl, ep, np, ctx->err_d, st, ctx->use_pdl);
   };
   const size_t Bm = static_cast<size_t>(ctx->cfg.max_candidates);
   const int nqh = m.n_q * m.hd, nkh = m.n_kv * m.hd;
