@@ -72,14 +72,13 @@ constexpr int64_t kSharedCostPerCand = 2;
 // (8 / n)-th page of a stage and writing its own partial slot: warp w scores candidate w % n,
 // pages p with p % (8 / n) == w / n, into slot w of the segment.  (n <= 4 keeps every warp busy.)
 __host__ __device__ constexpr int shared_reps(int n_cands) { return kConsumerWarps / n_cands; }
-// a 64-token chunk of the tensor-core attention on one SM, in the same units, when it runs beside
-// the private pages' launch: kTcChunkCost, plus up to kTcContention as the private side's work
-// grows to 3x the tensor-core side's (its page stream takes HBM bandwidth and raises the chunks'
-// load latency).  Measured: ~1.8 us per chunk beside the beam suffixes (private work ~0.8x),
-// ~2.2 us beside the MCTS leaves (~6x), against ~0.043 us per unit on the private side; ~0.86 us
-// per chunk alone.
-constexpr int64_t kTcChunkCost = 40;
-constexpr int64_t kTcContention = 12;
+// The tensor-core launch, in the same units, when it runs beside the private pages' launch: a CTA
+// costs kTcChunkCost per 64-token chunk plus kTcCtaCost once (the first query load and pages'
+// latency, the last output read-out).  Fitted to the SM split that measured fastest on the beam
+// (86 of 152 SMs, 12 chunks per CTA) and MCTS (17 SMs, ~110 chunks per CTA) workloads: ~1.3 us per
+// chunk and ~8 us per CTA against ~0.045 us per unit on the private side.
+constexpr int64_t kTcChunkCost = 29;
+constexpr int64_t kTcCtaCost = 180;
 // pages shared by fewer candidates go to the persistent kernel as kind-1 runs: 2 units per page
 // and candidate there against kTcChunkCost / 4 per page on the tensor cores, whatever the tile's rows
 constexpr size_t kTcMinCands = 6;
@@ -611,47 +610,60 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(
     const float sl2 = kLog2e * rsqrtf(128.f);
     grid_dep_wait();   // q is written by the preceding kernel
     if (threadIdx.x == 64) trace_event(ts, 0);
+    // this thread's query row of segment `sg` (half 0 the hi part, half 1 the lo part), or null
+    // for a row past the tile's candidates
+    auto q_row = [&](const AttnSeg& sg) -> const __nv_bfloat16* {
+      const int ci = r / group, hr = r - ci * group;
+      if (ci >= sg.n_cands) return nullptr;
+      return (hsel ? q_lo : q_hi) +
+             (static_cast<int64_t>(wk.cands[sg.cand + ci]) * n_q + static_cast<int64_t>(sg.g) * group + hr) * 128;
+    };
+    // Q of segment `sg` into TMEM, then the arrival that lets the S MMAs of the segment start (the
+    // caller has seen every S MMA that read the previous segment's Q complete)
+    auto q_in = [&](const AttnSeg& sg, uint32_t k) {
+      const long long tq = tic();
+      const __nv_bfloat16* src = q_row(sg);
+      uint4 w[16];
+#pragma unroll
+      for (int e = 0; e < 16; ++e) w[e] = src ? *reinterpret_cast<const uint4*>(src + e * 8) : make_uint4(0u, 0u, 0u, 0u);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {   // 32 head-dim elements = 16 columns per store
+        float v[16];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          v[4 * e] = __uint_as_float(w[4 * j + e].x);
+          v[4 * e + 1] = __uint_as_float(w[4 * j + e].y);
+          v[4 * e + 2] = __uint_as_float(w[4 * j + e].z);
+          v[4 * e + 3] = __uint_as_float(w[4 * j + e].w);
+        }
+        tmem_st16(trow + (hsel ? kColQlo : kColQhi) + j * 16, v);
+      }
+      tmem_wait_st();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(q_ready);
+      if (lane == 0 && warp == 2) {
+        toc(11, tq);
+        event(6, k);
+      }
+    };
     uint32_t u = 0, k = 0;
     bool ok = true;
+    if (seg0 < seg1) q_in(wk.segs[seg0], 0);
     for (int si = seg0; si < seg1; ++si, ++k) {
       const AttnSeg sg = wk.segs[si];
       const int nch = chunks(sg);
       const int ci = r / group, hr = r - ci * group;
       const bool live = ci < sg.n_cands;
-      // Q of this row into TMEM: half 0 the hi part, half 1 the lo part (every MMA of the
-      // previous segment has completed)
-      const long long tq = tic();
-      {
-        const int64_t row0 =
-            live ? (static_cast<int64_t>(wk.cands[sg.cand + ci]) * n_q + static_cast<int64_t>(sg.g) * group + hr) * 128
-                 : 0;
-        const __nv_bfloat16* src = hsel ? q_lo : q_hi;
-        uint4 w[16];
-#pragma unroll
-        for (int e = 0; e < 16; ++e) w[e] = live ? *reinterpret_cast<const uint4*>(src + row0 + e * 8) : make_uint4(0u, 0u, 0u, 0u);
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {   // 32 head-dim elements = 16 columns per store
-          float v[16];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            v[4 * e] = __uint_as_float(w[4 * j + e].x);
-            v[4 * e + 1] = __uint_as_float(w[4 * j + e].y);
-            v[4 * e + 2] = __uint_as_float(w[4 * j + e].z);
-            v[4 * e + 3] = __uint_as_float(w[4 * j + e].w);
-          }
-          tmem_st16(trow + (hsel ? kColQlo : kColQhi) + j * 16, v);
-        }
-        tmem_wait_st();
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(q_ready);
-      }
-      if (lane == 0 && warp == 2) {
-        toc(11, tq);
-        event(6, k);
-      }
       float m = -INFINITY, l = 0.f;
       for (int c = 0; c < nch; ++c, ++u) {
+        if (c == nch - 1 && si + 1 < seg1) {   // the next segment's query row on its way to L1
+          const __nv_bfloat16* nq = q_row(wk.segs[si + 1]);
+          if (nq) {
+            prefetch_l1(nq);
+            prefetch_l1(nq + 64);
+          }
+        }
         const uint32_t b = u % kTcSBufs;
         long long t0 = tic();
         if (ok) ok = __all_sync(0xffffffffu, mbar_wait(&s_full[b], (u / kTcSBufs) & 1u, err));
@@ -746,6 +758,9 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(
         }
       }
       if (threadIdx.x == 64 && si == seg1 - 1) trace_event(ts, 1);
+      // every S MMA of this segment has completed (its last S was read above): the next segment's Q
+      // goes into TMEM now, so that its S MMAs run while this segment's O is read out
+      if (si + 1 < seg1) q_in(wk.segs[si + 1], k + 1);
       // the segment's partial slots: (m, l) and the unnormalised O of every live row, my half of O
       const uint32_t lb = (u - 1) % kTcSBufs;
       const long long to = tic();
@@ -858,7 +873,9 @@ size_t attn_slot_capacity(int max_candidates, int n_kv, int num_sms) {
 //     of <= 8 candidates (share = 1: scored by the persistent kernel, one
 //     warp per candidate) or of <= 128 / G candidates (share = 2: one
 //     tensor-core tile of up to 128 query rows, see attn_tc_kernel), one run
-//     per chunk.  Every other page of a candidate goes to its private run.
+//     per chunk, except that chunks of the same kind with the same candidates
+//     (from different sets) share one run over all their pages.  Every other
+//     page of a candidate goes to its private run.
 //  2. The (run, kv head) pairs are laid end to end on a cost axis (a page
 //     costs kPrivateCost, or kSharedCostPerCand per candidate) and each page goes to the CTA whose
 //     equal share of the axis holds the page's midpoint; the pages of a pair
@@ -952,29 +969,64 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
       for (size_t i = 0; i < order.size(); ++i) order[i] = static_cast<int>(i);
       std::sort(order.begin(), order.end(),
                 [&](int a, int b2) { return group_pages[a].front() < group_pages[b2].front(); });
+      // Runs: each group's candidates cut into tiles; tiles of the same kind with the same candidate
+      // list (an MCTS tile of 16 leaves under a depth-1 edge and the depth-2 edge above those same
+      // leaves) become one run over both groups' pages, so that its query rows are loaded and its
+      // partials written once.  Attention is invariant to the order of the keys.
+      struct Tile {
+        int kind;
+        std::vector<int32_t> cands;
+        std::vector<int> groups;
+      };
+      std::vector<Tile> tiles;
+      std::unordered_map<uint64_t, std::vector<int>> tile_idx;   // hash of (kind, candidates) -> tiles
       for (int gi : order) {
         const auto& c = group_cands[gi];
-        const auto& pg = group_pages[gi];
-        const int page_off = static_cast<int>(w.pages.size());
-        w.pages.insert(w.pages.end(), pg.begin(), pg.end());
         // tensor-core tiles: as few as possible, with the candidates spread evenly over them
         const bool tc = share >= 2 && c.size() >= kTcMinCands;
         const size_t per = tc ? static_cast<size_t>(kTcRows / group) : static_cast<size_t>(kConsumerWarps);
         const size_t n_chunks = (c.size() + per - 1) / per;
         for (size_t k = 0, c0 = 0; k < n_chunks; ++k) {
           const size_t c1 = tc ? c.size() * (k + 1) / n_chunks : std::min(c.size(), c0 + per);
-          Run r;
-          r.kind = tc ? 2 : 1;
-          r.cand = static_cast<int>(w.cands.size());
-          r.n_cands = static_cast<int>(c1 - c0);
-          r.page_off = page_off;
-          r.n_pages = static_cast<int>(pg.size());
-          r.last_valid = 16;
-          r.cost = kSharedCostPerCand * r.n_cands;
-          w.cands.insert(w.cands.end(), c.begin() + c0, c.begin() + c1);
-          runs.push_back(r);
+          const int kind = tc ? 2 : 1;
+          const uint64_t h = hash_list(c.data() + c0, static_cast<int>(c1 - c0)) * 3 + static_cast<uint64_t>(kind);
+          int ti = -1;
+          for (int t : tile_idx[h])
+            if (tiles[t].kind == kind && tiles[t].cands.size() == c1 - c0 &&
+                std::equal(tiles[t].cands.begin(), tiles[t].cands.end(), c.begin() + c0))
+              ti = t;
+          if (ti < 0) {
+            ti = static_cast<int>(tiles.size());
+            tiles.push_back(Tile{kind, std::vector<int32_t>(c.begin() + c0, c.begin() + c1), {}});
+            tile_idx[h].push_back(ti);
+          }
+          tiles[ti].groups.push_back(gi);
           c0 = c1;
         }
+      }
+      std::vector<int> group_off(group_cands.size(), -1);   // a single group's pages, stored once
+      for (const Tile& t : tiles) {
+        Run r;
+        r.kind = t.kind;
+        r.cand = static_cast<int>(w.cands.size());
+        r.n_cands = static_cast<int>(t.cands.size());
+        if (t.groups.size() == 1) {
+          const int gi = t.groups[0];
+          if (group_off[gi] < 0) {
+            group_off[gi] = static_cast<int>(w.pages.size());
+            w.pages.insert(w.pages.end(), group_pages[gi].begin(), group_pages[gi].end());
+          }
+          r.page_off = group_off[gi];
+          r.n_pages = static_cast<int>(group_pages[gi].size());
+        } else {
+          r.page_off = static_cast<int>(w.pages.size());
+          for (int gi : t.groups) w.pages.insert(w.pages.end(), group_pages[gi].begin(), group_pages[gi].end());
+          r.n_pages = static_cast<int>(w.pages.size()) - r.page_off;
+        }
+        r.last_valid = 16;
+        r.cost = kSharedCostPerCand * r.n_cands;
+        w.cands.insert(w.cands.end(), t.cands.begin(), t.cands.end());
+        runs.push_back(r);
       }
     }
   }
@@ -1003,14 +1055,20 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
     else
       total += static_cast<int64_t>(r.n_pages) * r.cost * n_kv;
   }
-  // SMs for the private launch: all of them, or (share 3, both kinds of work) the share that makes
-  // both launches end together when they run side by side
+  // SMs for the private launch: all of them, or (share 3, both kinds of work) the split that makes
+  // the later of the two launches end soonest when they run side by side
   int priv_ctas = n_ctas, tc_ctas = n_ctas;
   if (share == 3 && total > 0 && tc_chunks > 0 && n_ctas >= 2) {
-    const int64_t base = tc_chunks * kTcChunkCost;
-    const int64_t wt = base + tc_chunks * kTcContention * std::min<int64_t>(total, 3 * base) / (3 * base);
-    tc_ctas = static_cast<int>(std::min<int64_t>(n_ctas - 1, std::max<int64_t>(1, (n_ctas * wt + (wt + total) / 2) /
-                                                                                        (wt + total))));
+    int64_t best = INT64_MAX;
+    for (int x = 1; x < n_ctas; ++x) {
+      const int64_t t_tc = (tc_chunks + x - 1) / x * kTcChunkCost + kTcCtaCost;
+      const int64_t t_pr = (total + (n_ctas - x) - 1) / (n_ctas - x);
+      const int64_t t = std::max(t_tc, t_pr);
+      if (t < best) {
+        best = t;
+        tc_ctas = x;
+      }
+    }
     priv_ctas = n_ctas - tc_ctas;
     w.tc_concurrent = true;
   }

@@ -15,6 +15,7 @@ import kvsynth as ks
 import paper_2607_09153_gb300.kvprm as kp
 
 PRIVATE_COST, SHARED_COST_PER_CAND = 4, 2   # the planner's per-page cost model
+TC_CHUNK_COST, TC_CTA_COST = 29, 180        # its tensor-core launch: per 64-token chunk, per CTA
 
 
 def check_plan(bt, sl, n_kv, group, n_ctas, share):
@@ -148,6 +149,32 @@ def test_shared_prefix_tensor_core_tiles():
     assert len(per_tile_head) == 3 * 2 and set(per_tile_head.values()) == {pre}, "each tile reads the prefix once"
 
 
+@pytest.mark.parametrize("share", [1, 2, 3])
+def test_tiles_with_the_same_candidates_share_one_run(share):
+    # an MCTS-like tree: pages 0..9 shared by all 32 candidates (G = 7: two tensor-core tiles of
+    # 16), pages 10..21 by candidates 0..15 and pages 22..29 by candidates 16..31, then 2 own pages
+    # each.  Each tile of the 32-candidate group has the same candidates as one of the smaller
+    # groups: one run over both groups' pages (10 + 12 or 10 + 8).  On the persistent kernel (runs
+    # of <= 8 candidates) the same holds run by run.
+    n = 32
+    bt = np.zeros((n, 24), np.int32)
+    sl = np.zeros(n, np.int32)
+    for b in range(n):
+        mid = (10 + np.arange(12)) if b < 16 else (22 + np.arange(8))
+        row = np.concatenate([np.arange(10), mid, 100 + 2 * b + np.arange(2)])
+        bt[b, :len(row)] = row
+        sl[b] = 16 * len(row) - 5
+    p = check_plan(bt, sl, 2, 7, 40, share)
+    kind = 2 if share >= 2 else 1
+    runs = collections.defaultdict(int)   # (candidate offset, kv head) -> pages
+    for seg in p["segs"][p["segs"][:, 0] == kind]:
+        runs[(int(seg[2]), int(seg[1]))] += int(seg[5])
+    if kind == 2:
+        assert sorted(runs.values()) == [18, 18, 22, 22], runs
+    else:
+        assert sorted(runs.values()) == [18] * 4 + [22] * 4, runs
+
+
 @pytest.mark.parametrize("n_share, kind", [(4, 1), (5, 1), (6, 2), (9, 2)])
 def test_small_shared_groups_stay_on_the_persistent_kernel(n_share, kind):
     # pages shared by fewer than 6 candidates are scored as kind-1 runs even in the tensor-core modes
@@ -173,6 +200,16 @@ def test_concurrent_split_shares_the_sms():
     sl = np.full(n, 16 * (pre + own), np.int32)
     p3 = check_plan(bt, sl, 2, 7, 64, 3)
     assert p3["n_tc_ctas"] >= 1 and p3["n_ctas"] >= 1 and p3["n_tc_ctas"] + p3["n_ctas"] <= 64
+    # the split minimises the later launch's end under the cost model: a tensor-core CTA costs 29 per
+    # 64-token chunk plus 180, a private page 4 (both per kv head)
+    chunks = 2 * ((pre + 3) // 4) * len(set(p3["segs"][p3["segs"][:, 0] == 2][:, 2].tolist()))
+    units = 2 * n * own * PRIVATE_COST
+
+    def later_end(x):
+        return max(-(-chunks // x) * TC_CHUNK_COST + TC_CTA_COST, -(-units // (64 - x)))
+
+    x = p3["n_tc_ctas"]
+    assert all(later_end(x) <= later_end(y) for y in range(1, 64))
     p2 = check_plan(bt, sl, 2, 7, 64, 2)   # serial: each launch planned over all SMs
     assert p2["n_ctas"] == 64 and p2["n_tc_ctas"] == 64
 
