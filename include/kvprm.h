@@ -297,7 +297,11 @@ KVPRM_API int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, con
  * P, 3 for values; 4 the softmax waiting for S, 5 for the previous O before a
  * rescale; 6 the loader waiting for a free key stage, 7 for a free value
  * stage; 8 reading S, 9 computing and storing P, 10 a segment's O read-out,
- * 11 loading Q; 12 chunks scored; 13 the CTA's lifetime. */
+ * 11 loading Q; 12 chunks scored; 13 the CTA's lifetime.  Bit 6: the combine
+ * of one verify token per candidate takes its flat form (one warp per query
+ * head, every slot's partial loaded in one round) at every batch size, not
+ * only when the (candidate, kv head) pairs exceed one wave of the general
+ * form (same result up to rounding; exercises the flat form). */
 KVPRM_API int kvprm_set_debug(kvprm_ctx* ctx, int flags);
 KVPRM_API int kvprm_debug_attn_out(kvprm_ctx* ctx, float* d_out);
 KVPRM_API int kvprm_debug_layers(kvprm_ctx* ctx, int which, void* d_out);

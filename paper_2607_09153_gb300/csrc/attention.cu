@@ -377,6 +377,85 @@ __global__ void __launch_bounds__(W * 32) attn_combine_kernel(
   trace_end(ts);
 }
 
+// The combine of a single verify token per candidate, flat: one CTA per (candidate, kv head) and
+// one warp per query head of the group, lane i holding head-dim elements i + 32 j.  A round issues
+// every load it uses (up to kFlatSlots partial slots' (m, l) and O values; in the first round also
+// q, k_self and v_self) before using any, so it costs one memory round trip; the slots then merge
+// into the running (M, L, acc) started from the verify token's own entry.  No shared memory and no
+// CTA barrier, so CTAs are short and many fit on an SM.
+constexpr int kFlatSlots = 8;
+
+template <int HD>
+__global__ void __launch_bounds__(512) attn_combine_flat_kernel(
+    const int32_t* __restrict__ slot_base, const int32_t* __restrict__ nslots, int n_q, int n_kv, int group,
+    const float* __restrict__ part_o, const float* __restrict__ part_ml, AttnMerge mg, unsigned long long* ts) {
+  constexpr int kPer = HD / 32;
+  trace_begin(ts);
+  grid_dep_launch();
+  const int cg = blockIdx.x, b = cg / n_kv, g = cg - b * n_kv;
+  const int r = static_cast<int>(threadIdx.x >> 5), lane = static_cast<int>(threadIdx.x & 31);
+  const int first = slot_base[cg], ns = nslots[cg];   // host-uploaded before the call: no wait needed
+  const int64_t hq = static_cast<int64_t>(b) * n_q + static_cast<int64_t>(g) * group + r;
+  const int64_t hk = static_cast<int64_t>(b) * n_kv + g;
+  grid_dep_wait();   // the partials (and q, k_self, v_self) are written by earlier kernels
+  if (threadIdx.x == 0) trace_event(ts, 0);
+  float2 ml[kFlatSlots];
+  float o[kFlatSlots][kPer];
+  auto load_round = [&](int s0) {
+#pragma unroll
+    for (int k = 0; k < kFlatSlots; ++k) {
+      const bool in = s0 + k < ns;
+      const int64_t pr = (static_cast<int64_t>(first) + (in ? s0 + k : 0)) * group + r;
+      ml[k] = in ? __ldcg(reinterpret_cast<const float2*>(part_ml) + pr) : make_float2(-INFINITY, 0.f);
+#pragma unroll
+      for (int j = 0; j < kPer; ++j) o[k][j] = in ? __ldcg(part_o + pr * HD + lane + 32 * j) : 0.f;
+    }
+  };
+  float qd[kPer], kd[kPer], acc[kPer];
+#pragma unroll
+  for (int j = 0; j < kPer; ++j) {
+    qd[j] = __ldcg(mg.q + hq * HD + lane + 32 * j);
+    kd[j] = __ldcg(mg.kself + hk * HD + lane + 32 * j);
+    acc[j] = __ldcg(mg.vself + hk * HD + lane + 32 * j);
+  }
+  load_round(0);
+  // the verify token's own entry: score q . k_self (log2 units), weight 1 at M = that score
+  float dot = 0.f;
+#pragma unroll
+  for (int j = 0; j < kPer; ++j) dot += qd[j] * kd[j];
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
+  float M = dot * (kLog2e * rsqrtf(static_cast<float>(HD))), L = 1.f;
+  for (int s0 = 0;; s0 += kFlatSlots) {
+#pragma unroll
+    for (int k = 0; k < kFlatSlots; ++k) {
+      if (ml[k].x == -INFINITY) continue;   // past the last slot, or a slot with no token (warp-uniform)
+      const float Mn = fmaxf(M, ml[k].x);
+      const float sc = exp2f(M - Mn), w = exp2f(ml[k].x - Mn);
+      L = L * sc + w * ml[k].y;
+#pragma unroll
+      for (int j = 0; j < kPer; ++j) acc[j] = acc[j] * sc + w * o[k][j];
+      M = Mn;
+    }
+    if (s0 + kFlatSlots >= ns) break;
+    load_round(s0 + kFlatSlots);
+  }
+  const float inv = 1.f / L;
+#pragma unroll
+  for (int j = 0; j < kPer; ++j) {
+    const float out = acc[j] * inv;
+    const int64_t oi = hq * HD + lane + 32 * j;
+    const __nv_bfloat16 hi = __float2bfloat16_rn(out);
+    mg.o_hi[oi] = hi;
+    mg.o_lo[oi] = __float2bfloat16_rn(out - __bfloat162float(hi));
+    if (mg.out_f32) mg.out_f32[oi] = out;
+    if (mg.dbg) mg.dbg[oi] = out;
+  }
+  if (mg.lse && lane == 0) mg.lse[hq] = M * kLn2 + logf(L);   // scores are in log2 units
+  if (threadIdx.x == 0) trace_event(ts, 1);
+  trace_end(ts);
+}
+
 // ---------------------------------------------------------------- shared pages on the tensor cores
 // attn_tc_kernel: persistent CTAs, each scoring its range of kind-2 segments
 // (wk.tc_cta).  A segment is a tile of <= 128 / G candidates that all
@@ -1345,7 +1424,7 @@ cudaError_t launch_attention_tc(const AttnShape& s, const AttnWork& wk, const CU
 
 cudaError_t launch_attn_combine(const AttnShape& s, const AttnWork& wk, int n, const float* part_o,
                                 const float* part_ml, const AttnMerge& mg, cudaStream_t stream, bool pdl,
-                                unsigned long long* ts) {
+                                unsigned long long* ts, bool force_flat) {
   if (n == 0) return cudaSuccess;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(static_cast<unsigned>(n) * s.n_kv, 1, 1);
@@ -1367,6 +1446,18 @@ cudaError_t launch_attn_combine(const AttnShape& s, const AttnWork& wk, int n, c
       sms = 1;
   }
   const bool narrow = static_cast<int64_t>(n) * s.n_kv > 6 * static_cast<int64_t>(sms);
+  // A single verify token per candidate with more pairs than one wave of the general form (whose
+  // 4-warp CTAs then take two waves of several memory round trips each): the flat combine, about
+  // 1 % more MCTS scores per second; fewer pairs keep the general form (measured no faster flat).
+  if (mg.depth == 1 && (narrow || force_flat)) {
+    cfg.dynamicSmemBytes = 0;
+    cfg.blockDim = dim3(32 * static_cast<unsigned>(s.group), 1, 1);
+    if (s.hd == 128)
+      return cudaLaunchKernelEx(&cfg, attn_combine_flat_kernel<128>, wk.slot_base, wk.nslots, s.n_q, s.n_kv, s.group,
+                                part_o, part_ml, mg, ts);
+    return cudaLaunchKernelEx(&cfg, attn_combine_flat_kernel<64>, wk.slot_base, wk.nslots, s.n_q, s.n_kv, s.group,
+                              part_o, part_ml, mg, ts);
+  }
 #define KVPRM_COMBINE_W(HD_, R_, W_)                                                                               \
   do {                                                                                                           \
     cfg.dynamicSmemBytes = CombineShape<HD_, R_, W_>::kBytes;                                                    \

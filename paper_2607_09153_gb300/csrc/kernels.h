@@ -209,10 +209,12 @@ cudaError_t launch_attention_tc(const AttnShape& s, const AttnWork& wk, const CU
                                 float margin, int* err, cudaStream_t stream, bool pdl,
                                 unsigned long long* ts = nullptr, unsigned long long* prof = nullptr);
 // Merge every (candidate, kv head)'s slots (wk.slot_base / wk.nslots) of the
-// n candidates with the self entry into the attention output.
+// n candidates with the self entry into the attention output.  A single verify
+// token per candidate takes the flat form when its (candidate, kv head) pairs
+// outnumber one wave of the general form (or always, with force_flat).
 cudaError_t launch_attn_combine(const AttnShape& s, const AttnWork& wk, int n, const float* part_o,
                                 const float* part_ml, const AttnMerge& mg, cudaStream_t stream, bool pdl,
-                                unsigned long long* ts = nullptr);
+                                unsigned long long* ts = nullptr, bool force_flat = false);
 cudaError_t launch_resolve(const int32_t* bt, const int32_t* seq_lens, int max_blocks, int b, int64_t* out,
                            cudaStream_t stream);
 

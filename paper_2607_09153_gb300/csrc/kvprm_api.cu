@@ -734,7 +734,8 @@ int enqueue_forward(kvprm_ctx* ctx, const CallPlan& P, Enq& E, const FwdSaves* s
     }
     if (wk.fuse_cs == 0)   // else the attention launch merged the slots itself
       LAUNCH(KVPRM_PROF_COMBINE,
-             kvprm::launch_attn_combine(ctx->as, wk, n, ctx->apart_o, ctx->apart_ml, mg, st, pdl, TS),
+             kvprm::launch_attn_combine(ctx->as, wk, n, ctx->apart_o, ctx->apart_ml, mg, st, pdl, TS,
+                                        (ctx->debug_flags & 64) != 0),
              "attn_combine");
     kvprm::GemmEpilogue er_o = er;   // h += W_o o; x = h ⊙ g_mlp for the gate/up projection
     er_o.gain_next = ctx->mlp_norm[l];
@@ -1548,7 +1549,9 @@ int kvprm_attention(kvprm_ctx* ctx, const void* kv_layer, int64_t n_pages, const
   const kvprm::AttnWork wk = device_work(ctx);
   if ((rc = enqueue_attention(ctx, E, as, wk, 0, Q, mg, false))) return rc;
   if (wk.fuse_cs == 0)
-    LAUNCH(KVPRM_PROF_COMBINE, kvprm::launch_attn_combine(as, wk, n, ctx->apart_o, ctx->apart_ml, mg, st, false),
+    LAUNCH(KVPRM_PROF_COMBINE,
+           kvprm::launch_attn_combine(as, wk, n, ctx->apart_o, ctx->apart_ml, mg, st, false, TS,
+                                      (ctx->debug_flags & 64) != 0),
            "attn_combine");
   ctx->last_n = n;
   ctx->last_stream = st;

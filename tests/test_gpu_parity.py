@@ -125,13 +125,40 @@ def test_fused_combine(lens, fused, monkeypatch):
 
 
 def test_narrow_combine():
-    # more (candidate, kv head) pairs than six per SM: the combine runs with four warps per pair
-    # (240 candidates x 4 kv heads = 960 > 6 x 152; a context holds at most 256 candidates)
+    # more (candidate, kv head) pairs than one wave of the general combine (240 candidates x 4 kv
+    # heads = 960 > 6 x 152; a context holds at most 256 candidates): the flat combine
     t = ks.Tables.make(0.2)
     lens = [int(x) for x in np.random.default_rng(47).integers(0, 60, size=240)]
     w = ks.distinct("narrow", ks.Arch(2, 256, 8, 4, 64, 512), 47, lens, gain_std=0.2)
     r, attn, _, _ = run_gpu(w, t)
     compare(w, t, gpu_rewards=r, gpu_attn=attn, label="narrow combine, 240 candidates x 4 kv heads")
+
+
+def test_narrow_combine_depth_readout():
+    # the same number of pairs from a depth-2 readout (120 candidates x 2 rows x 4 kv heads): the
+    # general combine with four warps per pair and the causal verify-token entries
+    t = ks.Tables.make(0.2)
+    lens = [int(x) for x in np.random.default_rng(48).integers(0, 60, size=120)]
+    w = ks.distinct("narrow_d2", ks.Arch(2, 256, 8, 4, 64, 512), 48, lens, gain_std=0.2)
+    r, attn, _, _ = run_gpu(w, t, depth=2)
+    compare(w, t, gpu_rewards=r, gpu_attn=attn, label="narrow combine, depth 2", depth=2)
+
+
+# debug flag 64: the flat combine at every batch size
+@pytest.mark.parametrize("make", [
+    # empty and ragged caches, one to many partial slots per (candidate, kv head), head_dim 64
+    lambda: ks.distinct("flat", ks.ARCH_TINY, 61, [0, 1, 15, 17, 300, 2500], gain_std=0.2),
+    # head_dim 128, G = 7, shared pages (tensor-core and persistent partials) and private suffixes
+    lambda: ks.shared_prefix("flat_tc", ARCH_G7, 62, 20, 530, 40, gain_std=0.2),
+    lambda: ks.mcts_tree("flat_tree", ARCH_G7, 63, branching=3, depth=3, lo=5, hi=90, gain_std=0.2),
+    # G = 16 (16 warps per CTA)
+    lambda: ks.distinct("flat_g16", ks.Arch(2, 512, 16, 1, 64, 512), 64, [0, 50, 129, 3000], gain_std=0.2),
+])
+def test_flat_combine(make):
+    t = ks.Tables.make(0.2)
+    w = make()
+    r, attn, _, _ = run_gpu(w, t, extra_flags=64)
+    compare(w, t, gpu_rewards=r, gpu_attn=attn, label=f"flat combine {w.name}")
 
 
 def test_attention_teacher_forced():

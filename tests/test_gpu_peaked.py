@@ -4,8 +4,9 @@ key dominating late in the sequence, runs of identical keys sharing the top scor
 queries whose scores spread over tens of units.  Every attention plan is covered: the fused-combine
 plan, the persistent kernel with the combine launch, shared runs of <= 4 candidates on the
 persistent kernel, the tensor-core tiles of shared pages with the production rescale margin, an
-MCTS tree mixing the last two, and (end to end) the depth-k combine.  Tolerances are the ones every
-parity test uses: 2e-3 relative per (candidate, head) or (layer, candidate), 1e-3 on P(+)."""
+MCTS tree mixing the last two, both forms of the combine launch, and (end to end) the depth-k
+combine.  Tolerances are the ones every parity test uses: 2e-3 relative per (candidate, head) or
+(layer, candidate), 1e-3 on P(+)."""
 import numpy as np
 import pytest
 
@@ -24,7 +25,7 @@ def _last(w, b):
     return int(w.cand_seg[b][-1]), int(w.cand_off[b][-1])
 
 
-def _run(case: PlantedCase, label: str, min_spread: float = 30.0):
+def _run(case: PlantedCase, label: str, min_spread: float = 30.0, flags: int = 0):
     torch = require_gpu()
     import paper_2607_09153_gb300 as kp
     w, a = case.w, case.arch
@@ -32,6 +33,8 @@ def _run(case: PlantedCase, label: str, min_spread: float = 30.0):
     assert spread >= min_spread, f"{label}: top-to-median score gap {spread:.1f} is not peaked"
     dev = ks.DeviceInputs(ks.distinct("host", a, 1, [16]), ks.Tables.make())   # weights for a context only
     sc = make_scorer(dev, w.n_candidates, w.max_blocks)
+    if flags:
+        kp.kvprm_set_debug(sc.ctx, flags)
     pool, q, k, v = case.device()
     B = w.n_candidates
     out = torch.full((B, a.n_q_heads, a.head_dim), float("nan"), dtype=torch.float32, device="cuda")
@@ -56,13 +59,16 @@ def test_peaked_fused_combine():
     _run(PlantedCase(w, ks.Tables.make(), 1, needles, runs=[(2, 1000, 24)]), "fused combine")
 
 
-def test_peaked_persistent_and_combine():
-    # ragged lengths: the persistent kernel (private runs, merger warp) and the combine launch;
-    # candidate 4's top score is a run of 64 identical keys near its end, candidate 6 has no cache
+@pytest.mark.parametrize("flat", [False, True])
+def test_peaked_persistent_and_combine(flat):
+    # ragged lengths: the persistent kernel (private runs, merger warp) and the combine launch (its
+    # general form, or the flat form with debug flag 64); candidate 4's top score is a run of 64
+    # identical keys near its end, candidate 6 has no cache
     lens = [1, 17, 250, 2049, 4096, 33, 0]
     w = ks.distinct("pk_persist", ARCH_G6, 202, lens)
     needles = [_last(w, b) for b in (0, 1, 2, 3, 5)] + [(3, 5)]
-    _run(PlantedCase(w, ks.Tables.make(), 2, needles, runs=[(4, 4000, 64)]), "persistent + combine")
+    _run(PlantedCase(w, ks.Tables.make(), 2, needles, runs=[(4, 4000, 64)]), f"persistent + combine flat={flat}",
+         flags=64 if flat else 0)
 
 
 def test_peaked_shared_runs():
@@ -89,11 +95,13 @@ def test_peaked_tensor_cores(B, prefix, suffix):
          f"tensor cores B={B} prefix={prefix}")
 
 
-def test_peaked_tree_mixed():
+@pytest.mark.parametrize("flat", [False, True])
+def test_peaked_tree_mixed(flat):
     # MCTS tree: depth-1 groups of 9 on the tensor cores, depth-2 groups of 3 on the persistent kernel
     w = ks.mcts_tree("pk_tree", ARCH_G7, 206, branching=3, depth=3, lo=100, hi=400)
     needles = [_last(w, b) for b in range(w.n_candidates)] + [(0, 50)]
-    _run(PlantedCase(w, ks.Tables.make(), 6, needles, runs=[(0, 10, 32)]), "tree, tensor cores + shared runs")
+    _run(PlantedCase(w, ks.Tables.make(), 6, needles, runs=[(0, 10, 32)]),
+         f"tree, tensor cores + shared runs, flat={flat}", flags=64 if flat else 0)
 
 
 # ---------------------------------------------------------------- end to end, peaked query/key projections
