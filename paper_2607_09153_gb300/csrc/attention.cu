@@ -760,6 +760,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(
           tmem_ld16_nowait(trow + b * 64 + hsel * 32, v0);
           tmem_ld16_nowait(trow + b * 64 + hsel * 32 + 16, v1);
           tmem_wait_ld();
+          tmem_hold(v0);
+          tmem_hold(v1);
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
             x[j] = v0[j];
@@ -854,6 +856,8 @@ __global__ void __launch_bounds__(kTcThreads, 1) attn_tc_kernel(
 #pragma unroll
         for (int q = 0; q < 4; ++q) tmem_ld16_nowait(trow + kColO + hsel * 64 + q * 16, v[q]);
         tmem_wait_ld();
+#pragma unroll
+        for (int q = 0; q < 4; ++q) tmem_hold(v[q]);
         if (live) {
 #pragma unroll
           for (int q = 0; q < 4; ++q)

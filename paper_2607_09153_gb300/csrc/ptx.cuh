@@ -275,6 +275,12 @@ __device__ __forceinline__ void tmem_ld16_nowait(uint32_t taddr, float (&v)[16])
       : "r"(taddr));
 }
 __device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+// After tmem_wait_ld: ties the registers a tmem_ld16_nowait filled to a point after the wait (the
+// empty volatile statements keep their order behind it), so that no use of them is scheduled earlier.
+__device__ __forceinline__ void tmem_hold(float (&v)[16]) {
+#pragma unroll
+  for (int i = 0; i < 16; ++i) asm volatile("" : "+f"(v[i]));
+}
 // Each thread of a warp writes 16 consecutive fp32 columns of its own TMEM lane
 // (complete with tmem_wait_st before an MMA may read them).
 __device__ __forceinline__ void tmem_st16(uint32_t taddr, const float (&v)[16]) {
