@@ -88,6 +88,11 @@ struct GradState {
   int n_shared = 0, n_ref = 0;   // of the last call
   float* grad_own = nullptr;   // kvprm_steer's gradient buffer
   size_t grad_own_bytes = 0;
+  // the forward with saves and the backward of a call, captured once and replayed while every launch
+  // parameter and buffer they bake in is unchanged (the key)
+  cudaGraphExec_t gexec = nullptr;
+  std::vector<int64_t> gkey;
+  std::vector<ProfMark> marks;   // unused: profiled calls run eagerly
 };
 
 }  // namespace
@@ -317,6 +322,7 @@ void free_ctx(kvprm_ctx* c) {
     cudaFree(g.shared);
     cudaFree(g.lists);
     cudaFree(g.grad_own);
+    if (g.gexec) cudaGraphExecDestroy(g.gexec);
   }
   if (c->staging) cudaFreeHost(c->staging);
   if (c->h_rewards) cudaFreeHost(c->h_rewards);
@@ -822,8 +828,11 @@ int enqueue_pool_copy(kvprm_ctx* ctx, cudaStream_t st) {
   return KVPRM_OK;
 }
 
+// With `prepared` set, the call is planned and its tables uploaded (stream-ordered on `st`), and
+// its plan returned there instead of enqueueing the forward (the gradient call enqueues the forward
+// together with the backward).
 int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const int32_t* bt, const int32_t* sl, int32_t n,
-                 cudaStream_t st, const FwdSaves* sv = nullptr) {
+                 cudaStream_t st, const FwdSaves* sv = nullptr, CallPlan* prepared = nullptr) {
   int max_pages = 0;
   int rc = validate_tables(ctx, n_pages, bt, sl, n, &max_pages);
   if (rc) return rc;
@@ -871,6 +880,10 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   if (ctx->inject_fail) {   // failure-detection hook: report a failed launch, enqueue nothing more
     ctx->inject_fail = 0;
     return cuda_fail(ctx, cudaErrorLaunchFailure, "injected failure of the forward's launch");
+  }
+  if (prepared) {
+    *prepared = P;
+    return KVPRM_OK;
   }
 
   if (!ctx->use_graph || sv) {   // a forward that keeps its intermediates runs eagerly
@@ -1055,8 +1068,9 @@ int score_grad_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, con
   if (n == 0) return KVPRM_OK;
   if ((rc = ensure_grad(ctx, st))) return rc;
   GradState& g = ctx->grad;
-  // the forward, keeping its intermediates
-  if ((rc = score_device(ctx, kv_pages, n_pages, bt, sl, n, st, &g.sv))) return rc;
+  // the call's plan and tables (the forward itself is enqueued below, with the backward)
+  CallPlan P;
+  if ((rc = score_device(ctx, kv_pages, n_pages, bt, sl, n, st, &g.sv, &P))) return rc;
   const ModelDims& m = ctx->md;
   const int NL = ctx->cfg.n_layers, mb = ctx->cfg.max_blocks_per_seq;
   const int np = (n + 15) / 16 * 16;
@@ -1089,72 +1103,120 @@ int score_grad_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, con
   CK(cudaMemcpyAsync(g.shared, refs.data(), refs.size(), cudaMemcpyHostToDevice, st), "shared flags");
   if (!lists.empty())
     CK(cudaMemcpyAsync(g.lists, lists.data(), sizeof(int32_t) * lists.size(), cudaMemcpyHostToDevice, st), "lists");
-  const int64_t page_elems = static_cast<int64_t>(2) * m.n_kv * 16 * m.hd;
-  CK(kvprm::launch_zero_pages(grad, g.lists, n_shared, NL, n_pages, page_elems, st), "zero shared pages");
-  // the backward products on the forward's GEMM (plain fp32 epilogue) against the transposed weights
-  auto gemm = [&](const CUtensorMap* w, int M, int K, const CUtensorMap* xh, const CUtensorMap* xl, float* out) {
-    const GemmPlan gp = kvprm::plan_gemm(M, K, np, ctx->num_sms, true, false);
-    kvprm::GemmEpilogue ep;
-    ep.mode = kvprm::GemmEpilogue::PLAIN;
-    ep.M = M;
-    ep.n_valid = n;
-    ep.out = out;
-    return kvprm::launch_gemm(gp, w, xh, xl, ep, np, ctx->err_d, st, ctx->use_pdl);
-  };
-  const size_t Bm = static_cast<size_t>(ctx->cfg.max_candidates);
-  const int nqh = m.n_q * m.hd, nkh = m.n_kv * m.hd;
-  const FwdSaves& sv = g.sv;
-  CK(kvprm::launch_head_back(ctx->h, ctx->rewards_d, ctx->final_norm, ctx->w_plus, ctx->w_minus, n, m.d, m.eps, g.dh,
-                             g.ghi, g.glo, st),
-     "head backward");
-  for (int l = NL - 1; l >= 0; --l) {
-    // feed-forward block: da = W_down^T dh; [du; dt]; dx2 = W_gate_up^T [du; dt]; dh_mid
-    CK(gemm(&g.tm_down[l], m.ff, m.d, &g.tm_d_hi, &g.tm_d_lo, g.tmp), "W_down^T product");
-    CK(kvprm::launch_silu_back(g.tmp, sv.gu + l * Bm * 2 * m.ff, n, m.ff, g.ghi, g.glo, st), "SiLU backward");
-    CK(gemm(&g.tm_gu[l], m.d, 2 * m.ff, &g.tm_gu_hi, &g.tm_gu_lo, g.tmp), "W_gate_up^T product");
-    CK(kvprm::launch_rms_back(sv.hmid + l * Bm * m.d, nullptr, ctx->mlp_norm[l], g.tmp, g.dh, n, m.d, m.eps, g.dh,
-                              g.ghi, g.glo, st),
-       "pre-MLP RMSNorm backward");
-    // attention block: do = W_o^T dh_mid, then the read-out's backward into this layer's pages
-    CK(gemm(&g.tm_o[l], nqh, m.d, &g.tm_d_hi, &g.tm_d_lo, g.tmp), "W_o^T product");
-    kvprm::AttnBackArgs a;
-    a.n = n;
-    a.n_q = m.n_q;
-    a.n_kv = m.n_kv;
-    a.hd = m.hd;
-    a.q = sv.q + l * Bm * nqh;
-    a.kself = sv.k + l * Bm * nkh;
-    a.vself = sv.v + l * Bm * nkh;
-    a.o = sv.o + l * Bm * nqh;
-    a.dout = g.tmp;
-    a.lse = sv.lse + l * Bm * m.n_q;
-    a.D = g.D;
-    a.dq = g.dq;
-    a.dks = g.dks;
-    a.dvs = g.dvs;
-    a.units = g.units;
-    a.n_units = static_cast<int>(units.size());
-    a.seq_lens = ctx->tables_d;
-    a.block_table = ctx->tables_d + ctx->cfg.max_candidates;
-    a.max_blocks = mb;
-    a.pool_layer = kv_pages ? static_cast<const bf16*>(kv_pages) + l * n_pages * page_elems : nullptr;
-    a.shared = g.shared;
-    a.grad_layer = grad + l * n_pages * page_elems;
-    a.err = ctx->err_d;
-    a.tm_pool = kv_pages && !ctx->grad_cuda_cores ? &ctx->tm_pool : nullptr;   // the forward's map of this pool
-    a.layer_page0 = static_cast<int64_t>(l) * n_pages;
-    CK(kvprm::launch_attn_back(a, st), "attention backward");
-    if (l == 0) break;   // below layer 0 lies only the verify token's embedding
-    // QKV projection: [dq; dk; dv] before RoPE, dx1 = W_qkv^T [...], dh of the layer below
-    CK(kvprm::launch_rope_back(g.dq, g.dks, g.dvs, ctx->rope, n, m.n_q, m.n_kv, m.hd, g.ghi, g.glo, st), "RoPE backward");
-    CK(gemm(&g.tm_qkv[l], m.d, m.qkv_rows, &g.tm_qkv_hi, &g.tm_qkv_lo, g.tmp), "W_qkv^T product");
-    CK(kvprm::launch_rms_back(sv.hout + (l - 1) * Bm * m.d, nullptr, ctx->attn_norm[l], g.tmp, g.dh, n, m.d, m.eps,
-                              g.dh, g.ghi, g.glo, st),
-       "pre-attention RMSNorm backward");
-  }
   g.n_shared = n_shared;
   g.n_ref = static_cast<int>(lists.size()) - n_shared;
   *n_ref_out = g.n_ref;
+  const int64_t page_elems = static_cast<int64_t>(2) * m.n_kv * 16 * m.hd;
+  const size_t Bm = static_cast<size_t>(ctx->cfg.max_candidates);
+  const int nqh = m.n_q * m.hd, nkh = m.n_kv * m.hd;
+  const FwdSaves& sv = g.sv;
+  // the forward with its saves, then the backward, on stream `s`
+  auto enqueue = [&](cudaStream_t s, Enq& E) -> int {
+    int r = enqueue_forward(ctx, P, E, &sv);
+    if (r) return r;
+    CK(kvprm::launch_zero_pages(grad, g.lists, n_shared, NL, n_pages, page_elems, s), "zero shared pages");
+    // the backward products on the forward's GEMM (plain fp32 epilogue) against the transposed weights
+    auto gemm = [&](const CUtensorMap* w, int M, int K, const CUtensorMap* xh, const CUtensorMap* xl, float* out) {
+      const GemmPlan gp = kvprm::plan_gemm(M, K, np, ctx->num_sms, true, false);
+      kvprm::GemmEpilogue ep;
+      ep.mode = kvprm::GemmEpilogue::PLAIN;
+      ep.M = M;
+      ep.n_valid = n;
+      ep.out = out;
+      return kvprm::launch_gemm(gp, w, xh, xl, ep, np, ctx->err_d, s, ctx->use_pdl);
+    };
+    CK(kvprm::launch_head_back(ctx->h, ctx->rewards_d, ctx->final_norm, ctx->w_plus, ctx->w_minus, n, m.d, m.eps, g.dh,
+                               g.ghi, g.glo, s),
+       "head backward");
+    for (int l = NL - 1; l >= 0; --l) {
+      // feed-forward block: da = W_down^T dh; [du; dt]; dx2 = W_gate_up^T [du; dt]; dh_mid
+      CK(gemm(&g.tm_down[l], m.ff, m.d, &g.tm_d_hi, &g.tm_d_lo, g.tmp), "W_down^T product");
+      CK(kvprm::launch_silu_back(g.tmp, sv.gu + l * Bm * 2 * m.ff, n, m.ff, g.ghi, g.glo, s), "SiLU backward");
+      CK(gemm(&g.tm_gu[l], m.d, 2 * m.ff, &g.tm_gu_hi, &g.tm_gu_lo, g.tmp), "W_gate_up^T product");
+      CK(kvprm::launch_rms_back(sv.hmid + l * Bm * m.d, nullptr, ctx->mlp_norm[l], g.tmp, g.dh, n, m.d, m.eps, g.dh,
+                                g.ghi, g.glo, s),
+         "pre-MLP RMSNorm backward");
+      // attention block: do = W_o^T dh_mid, then the read-out's backward into this layer's pages
+      CK(gemm(&g.tm_o[l], nqh, m.d, &g.tm_d_hi, &g.tm_d_lo, g.tmp), "W_o^T product");
+      kvprm::AttnBackArgs a;
+      a.n = n;
+      a.n_q = m.n_q;
+      a.n_kv = m.n_kv;
+      a.hd = m.hd;
+      a.q = sv.q + l * Bm * nqh;
+      a.kself = sv.k + l * Bm * nkh;
+      a.vself = sv.v + l * Bm * nkh;
+      a.o = sv.o + l * Bm * nqh;
+      a.dout = g.tmp;
+      a.lse = sv.lse + l * Bm * m.n_q;
+      a.D = g.D;
+      a.dq = g.dq;
+      a.dks = g.dks;
+      a.dvs = g.dvs;
+      a.units = g.units;
+      a.n_units = static_cast<int>(units.size());
+      a.seq_lens = ctx->tables_d;
+      a.block_table = ctx->tables_d + ctx->cfg.max_candidates;
+      a.max_blocks = mb;
+      a.pool_layer = kv_pages ? static_cast<const bf16*>(kv_pages) + l * n_pages * page_elems : nullptr;
+      a.shared = g.shared;
+      a.grad_layer = grad + l * n_pages * page_elems;
+      a.err = ctx->err_d;
+      a.tm_pool = kv_pages && !ctx->grad_cuda_cores ? &ctx->tm_pool : nullptr;   // the forward's map of this pool
+      a.layer_page0 = static_cast<int64_t>(l) * n_pages;
+      CK(kvprm::launch_attn_back(a, s), "attention backward");
+      if (l == 0) break;   // below layer 0 lies only the verify token's embedding
+      // QKV projection: [dq; dk; dv] before RoPE, dx1 = W_qkv^T [...], dh of the layer below
+      CK(kvprm::launch_rope_back(g.dq, g.dks, g.dvs, ctx->rope, n, m.n_q, m.n_kv, m.hd, g.ghi, g.glo, s), "RoPE backward");
+      CK(gemm(&g.tm_qkv[l], m.d, m.qkv_rows, &g.tm_qkv_hi, &g.tm_qkv_lo, g.tmp), "W_qkv^T product");
+      CK(kvprm::launch_rms_back(sv.hout + (l - 1) * Bm * m.d, nullptr, ctx->attn_norm[l], g.tmp, g.dh, n, m.d, m.eps,
+                                g.dh, g.ghi, g.glo, s),
+         "pre-attention RMSNorm backward");
+    }
+    return KVPRM_OK;
+  };
+  if (!ctx->use_graph || ctx->profile) {   // eager (profiled calls time each launch)
+    Enq E{ctx, st, ctx->use_pdl && !ctx->profile, ctx->profile, &ctx->live_marks};
+    if ((rc = enqueue(st, E))) return rc;
+    if (ctx->profile) {
+      CK(cudaStreamSynchronize(st), "cudaStreamSynchronize(profile)");
+      if ((rc = accumulate_marks(ctx, ctx->live_marks, true))) return rc;
+    }
+    return KVPRM_OK;
+  }
+  // the graph of this call: everything its launches take by value or by address
+  const std::vector<int64_t> key = {
+      n, P.n_pad, P.attn_ctas, ctx->work_host.n_tc_ctas, ctx->work_host.tc_concurrent ? 1 : 0,
+      ctx->work_host.fuse_cs, ctx->work_host.n_tc > 0 ? 1 : 0, ctx->work_host.n_ctas, ctx->debug_flags,
+      ctx->use_pdl ? 1 : 0, ctx->trace ? 1 : 0, ctx->layer_waits ? 1 : 0, ctx->as.layer_pages,
+      reinterpret_cast<int64_t>(kv_pages), n_pages, reinterpret_cast<int64_t>(grad),
+      static_cast<int64_t>(units.size()), n_shared, static_cast<int64_t>(lists.size()),
+      reinterpret_cast<int64_t>(g.units), reinterpret_cast<int64_t>(g.lists), reinterpret_cast<int64_t>(g.shared),
+      ctx->grad_cuda_cores ? 1 : 0, reinterpret_cast<int64_t>(ctx->pool_ptr)};
+  if (!(g.gexec && key == g.gkey)) {
+    if (g.gexec) cudaGraphExecDestroy(g.gexec);
+    g.gexec = nullptr;
+    g.gkey.clear();
+    CK(cudaStreamBeginCapture(ctx->cap_stream, cudaStreamCaptureModeThreadLocal), "cudaStreamBeginCapture(gradient)");
+    Enq E{ctx, ctx->cap_stream, ctx->use_pdl, false, &g.marks};
+    E.capturing = true;
+    rc = enqueue(ctx->cap_stream, E);
+    cudaGraph_t graph = nullptr;
+    cudaError_t e = cudaStreamEndCapture(ctx->cap_stream, &graph);
+    if (rc) {
+      if (graph) cudaGraphDestroy(graph);
+      return rc;
+    }
+    if (e != cudaSuccess) return cuda_fail(ctx, e, "cudaStreamEndCapture(gradient)");
+    e = cudaGraphInstantiate(&g.gexec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (e != cudaSuccess) {
+      g.gexec = nullptr;
+      return cuda_fail(ctx, e, "cudaGraphInstantiate(gradient)");
+    }
+    g.gkey = key;
+  }
+  CK(cudaGraphLaunch(g.gexec, st), "cudaGraphLaunch(gradient)");
   return KVPRM_OK;
 }
 
