@@ -327,8 +327,11 @@ KVPRM_API int kvprm_resolve(kvprm_ctx* ctx, int32_t b, int64_t* phys_row);
  * 128 / group candidates whose 4-page chunks are cut into equal ranges, one
  * per CTA of a separate launch (at most n_ctas of them); 3 (what scoring
  * contexts with head_dim 128 use) as 2, with the n_ctas SMs split between the
- * two launches in proportion to their estimated time (n_ctas + n_tc_ctas <=
- * the given n_ctas), so that they run side by side.  Kind-2 segments follow
+ * two launches so that the later one, estimated under a cost model (a
+ * tensor-core CTA: 29 units per chunk plus 180; a private page 4, a shared
+ * page 2 per candidate), ends soonest (n_ctas + n_tc_ctas <= the given
+ * n_ctas), so that they run side by side.  Shared tiles of different groups
+ * with the same candidates form one run over all their pages.  Kind-2 segments follow
  * the persistent CTAs' segments (segs[cta_seg[n_ctas]] on), and tensor-core
  * CTA k scores segments segs[tc_cta[k]] .. segs[tc_cta[k + 1] - 1].
  * Outputs go to caller-owned arrays with the capacities given (elements); the
@@ -390,10 +393,12 @@ KVPRM_API int kvprm_plan_attention(const int32_t* block_table, int32_t max_block
  *  cluster       CTAs per thread-block cluster (split-K ranks)
  *  tiles_per_cta m-tiles each CTA takes (1, or 2 for large batches)
  *  stages        shared-memory ring stages; tmem_cols tensor-memory columns; smem_bytes per CTA
+ *  threads       threads per CTA: 256 where one CTA fits per SM and n_pad >= 64, else 128
  * Errors: KVPRM_EINVAL (M, K or num_sms < 1, n_pad not a positive multiple of 16, out NULL). */
 typedef struct {
   int32_t m_tiles, k_tiles, kt_per_split, cluster, tiles_per_cta, stages, tmem_cols;
   int64_t smem_bytes;
+  int32_t threads;
 } kvprm_projection_plan;
 KVPRM_API int kvprm_plan_projection(int32_t M, int32_t K, int32_t n_pad, int32_t num_sms, int32_t has_lo,
                                     int32_t gate_up, kvprm_projection_plan* out);

@@ -68,7 +68,7 @@ __device__ __forceinline__ void store_hilo(__nv_bfloat16* hi, __nv_bfloat16* lo,
 // with 16-byte accesses (the 4-warp CTA is otherwise bound by 2- and 4-byte stores and by one load
 // latency per column).
 template <bool LARGE>
-__global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant__ CUtensorMap tmW,
+__global__ void __launch_bounds__(256) gemm_cluster_kernel(const __grid_constant__ CUtensorMap tmW,
                                                            const __grid_constant__ CUtensorMap tmX,
                                                            const __grid_constant__ CUtensorMap tmXlo, int has_lo,
                                                            const __grid_constant__ CUtensorMap tmB,
@@ -251,7 +251,10 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
   if (threadIdx.x == 0) trace_event(ts, 2);   // all MMAs of this CTA completed
   tc_fence_after();
   float* acc = reinterpret_cast<float*>(smem);   // the ring is idle once `done` has fired
-  const int m = warp * 32 + lane;
+  // 4 warps, or 8 (large batches with one CTA per SM): warps w and w + 4 share TMEM lane quadrant w,
+  // i.e. the tile's rows 32 w .. 32 w + 31, and take alternate 16-column groups (or columns)
+  const int nw = static_cast<int>(blockDim.x >> 5), nwh = nw >> 2, wh = warp >> 2;
+  const int m = (warp & 3) * 32 + lane;
   const bool merged = has_lo && 2 * n_pad <= 256;
   const uint32_t tile_cols = tmem_cols / static_cast<uint32_t>(mt);
   // one m-tile at a time: park it, reduce it over the cluster (split K), write its epilogue; with two
@@ -260,10 +263,10 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     const int m_tile = m_tile0 + tt;
     const uint32_t tcol = static_cast<uint32_t>(tt) * tile_cols;
     if (tt > 0 && cs > 1) cluster_wait();   // matches the arrive after the previous tile's reduction
-    for (int c0 = 0; c0 < n_pad; c0 += 16) {
+    for (int c0 = 16 * wh; c0 < n_pad; c0 += 16 * nwh) {
       float v[16];
       if (nk > 0 && have) {
-        const uint32_t t = tmem + (static_cast<uint32_t>(warp * 32) << 16) + tcol + static_cast<uint32_t>(c0);
+        const uint32_t t = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16) + tcol + static_cast<uint32_t>(c0);
         tmem_ld16(t, v);
         if (merged) {
           float w[16];
@@ -294,21 +297,22 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       // Without split K (cs = 1) the parked accumulator is already the sum.
       if (LARGE && (cs == 4 || cs == 8)) {
         // four consecutive rows of one column per thread (a warp covers a column's 128 rows), 16 / CS
-        // columns per round: 16 loads of 16 bytes in flight, the CS ranks' copies of each
+        // columns per round: 16 loads of 16 bytes in flight, the CS ranks' copies of each; warp w takes
+        // columns cbeg + w, cbeg + w + nw, ...
         auto vreduce = [&](auto cs_c) {
           constexpr int CS = decltype(cs_c)::value, PER = 16 / CS;
           const int rq = static_cast<int>(threadIdx.x) & 31, cg = static_cast<int>(threadIdx.x) >> 5;
-          for (int c0 = cbeg + cg; c0 < cend; c0 += 4 * PER) {
+          for (int c0 = cbeg + cg; c0 < cend; c0 += nw * PER) {
             float4 v[16];
 #pragma unroll
-            for (int k = 0; k < 16; ++k) {   // rank k % CS of column c0 + 4 (k / CS)
-              const int cc = c0 + 4 * (k / CS);
+            for (int k = 0; k < 16; ++k) {   // rank k % CS of column c0 + nw (k / CS)
+              const int cc = c0 + nw * (k / CS);
               v[k] = cc < cend ? ld_cluster4(acc + cc * kBM + 4 * rq, static_cast<uint32_t>(k % CS))
                                : make_float4(0.f, 0.f, 0.f, 0.f);
             }
 #pragma unroll
             for (int j = 0; j < PER; ++j) {
-              const int cc = c0 + 4 * j;
+              const int cc = c0 + nw * j;
               if (cc >= cend) continue;
               const float4* u = v + CS * j;
               auto add = [](float4 x, float4 y) { return make_float4(x.x + y.x, x.y + y.y, x.z + y.z, x.w + y.w); };
@@ -324,7 +328,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
           vreduce(std::integral_constant<int, 8>{});
       } else if (cs > 1) {
         const int step = cs <= 8 ? 2 : 1;
-        for (int c = cbeg; c < cend; c += step) {
+        for (int c = cbeg + wh * step; c < cend; c += step * nwh) {
           const bool two = step == 2 && c + 1 < cend;
           float v[16];
 #pragma unroll
@@ -367,7 +371,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     float* qkf = hpre;   // [column][head of the tile]
     if (ep.mode == GemmEpilogue::QKV && ep.qn_gain) {
       const int hpt = kBM / ep.hd;   // heads per tile: 1 (hd 128) or 2 (hd 64)
-      for (int it = warp; it < nc * hpt; it += 4) {
+      for (int it = warp; it < nc * hpt; it += nw) {
         const int cl = it / hpt, hh = it % hpt;
         const float* col = acc + (cbeg + cl) * kBM + hh * ep.hd;
         float sq = 0.f;
@@ -386,11 +390,11 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
     if (ep.mode == GemmEpilogue::PLAIN) {
       const int gm = m_tile * kBM + m;
       if (gm < ep.M)
-        for (int c = cbeg; c < cend; ++c) ep.out[static_cast<int64_t>(c) * ep.M + gm] = acc[c * kBM + m];
+        for (int c = cbeg + wh; c < cend; c += nwh) ep.out[static_cast<int64_t>(c) * ep.M + gm] = acc[c * kBM + m];
     } else if (LARGE && ep.mode == GemmEpilogue::LOWRANK) {   // t = s (A x), hi/lo [n][r]; large image only
       const int gm = m_tile * kBM + m;
       if (gm < ep.M)
-        for (int c = cbeg; c < cend; ++c)
+        for (int c = cbeg + wh; c < cend; c += nwh)
           store_hilo(ep.t_hi, ep.t_lo, static_cast<int64_t>(c) * ep.M + gm, ep.lr_scale * acc[c * kBM + m]);
     } else if (ep.mode == GemmEpilogue::RESID && LARGE) {
       // pass 1, 16 columns at a time with the group's residual loads in flight before the first use:
@@ -414,17 +418,17 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
           g4[2] = gc.x;
           g4[3] = gc.y;
         }
-        for (int c0 = cbeg + cg; c0 < cend; c0 += 4 * 8) {
+        for (int c0 = cbeg + cg; c0 < cend; c0 += nw * 8) {
           float4 h_in[8];
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
-            const int c = c0 + 4 * k;
+            const int c = c0 + nw * k;
             h_in[k] = (c < cend && rows_ok) ? *reinterpret_cast<const float4*>(ep.h + static_cast<int64_t>(c) * ep.M + gm0)
                                             : make_float4(0.f, 0.f, 0.f, 0.f);
           }
 #pragma unroll
           for (int k = 0; k < 8; ++k) {
-            const int c = c0 + 4 * k;
+            const int c = c0 + nw * k;
             if (c >= cend) break;
             float4* ap = reinterpret_cast<float4*>(acc + c * kBM + 4 * rq);
             const float4 a = *ap;
@@ -452,8 +456,8 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
             *ap = make_float4(hv.x * hv.x, hv.y * hv.y, hv.z * hv.z, hv.w * hv.w);
           }
         }
-      } else {
-        for (int c0 = cbeg; c0 < cend; c0 += 16) {
+      } else {   // warps w and w + 4 share rows: alternate 16-column groups
+        for (int c0 = cbeg + 16 * wh; c0 < cend; c0 += 16 * nwh) {
           float h_in[16];
 #pragma unroll
           for (int j = 0; j < 16; ++j) {
@@ -530,7 +534,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       const int j0 = m_tile * 64 + 8 * rg;   // ff % 8 == 0: a row group is all valid or all past ff
       if (j0 < ep.ff) {
 #pragma unroll 2
-        for (int c = cbeg + cg; c < cend; c += 16) {
+        for (int c = cbeg + cg; c < cend; c += 4 * nw) {   // 4 nw column groups of 8 threads
           const float rs = ep.rs_sumsq ? rsc[c - cbeg] : 1.f;
           const float4* gp = reinterpret_cast<const float4*>(acc + c * kBM + 8 * rg);
           const float4* up = reinterpret_cast<const float4*>(acc + c * kBM + 64 + 8 * rg);
@@ -563,14 +567,15 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
         }
       }
     } else if (ep.mode == GemmEpilogue::SILU) {
-      const int r = m & 63, half_sel = m >> 6;   // two column groups of 64 threads
+      // 2 nhalf column groups of 64 threads (rows m and m + 64 of a column share a group)
+      const int r = m & 63, ng = 2 * nwh, grp = (m >> 6) + 2 * wh;
       const int j = m_tile * 64 + r;
       if (j < ep.ff)
-        for (int c0 = cbeg + half_sel; c0 < cend; c0 += 2 * kEpiBatch) {
+        for (int c0 = cbeg + grp; c0 < cend; c0 += ng * kEpiBatch) {
           float g[kEpiBatch], u[kEpiBatch];   // a batch's operands, read before its first store
 #pragma unroll
           for (int k = 0; k < kEpiBatch; ++k) {
-            const int c = c0 + 2 * k;
+            const int c = c0 + ng * k;
             const bool ok = c < cend;
             const float rs = (ok && ep.rs_sumsq) ? rsc[c - cbeg] : 1.f;
             g[k] = ok ? acc[c * kBM + r] * rs : 0.f;
@@ -578,7 +583,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
           }
 #pragma unroll
           for (int k = 0; k < kEpiBatch; ++k) {
-            const int c = c0 + 2 * k;
+            const int c = c0 + ng * k;
             if (c < cend) {
               store_hilo(ep.a_hi, ep.a_lo, static_cast<int64_t>(c) * ep.ff + j, g[k] / (1.0f + expf(-g[k])) * u[k]);
               if (ep.gu_save) {   // gate and up pre-activations for a backward pass
@@ -629,7 +634,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
       };
       if (head < ep.n_q + 2 * ep.n_kv) {
 #pragma unroll 2
-        for (int c = cbeg + cg; c < cend; c += 8) {
+        for (int c = cbeg + cg; c < cend; c += 2 * nw) {   // 2 nw column groups of 16 threads
           const float rs = ep.qn_gain ? qkf[(c - cbeg) * 2 + hh_tile] : (ep.rs_sumsq ? rsc[c - cbeg] : 1.f);
           const float4 a4 = *reinterpret_cast<const float4*>(acc + c * kBM + row_a);
           const float4 b4 = *reinterpret_cast<const float4*>(acc + c * kBM + row_b);
@@ -667,8 +672,8 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
           }
         }
       }
-    } else {   // QKV: pair p = m & 63 of this tile, two column groups of 64 threads
-      const int p = m & 63, half_sel = m >> 6;
+    } else {   // QKV: pair p = m & 63 of this tile, 2 nhalf column groups of 64 threads
+      const int p = m & 63, ng = 2 * nwh, grp = (m >> 6) + 2 * wh;
       const int hd = ep.hd, half = hd / 2;
       const int row_a = (p / half) * hd + (p % half);   // first element of the pair, within the tile
       const int row_b = row_a + half;
@@ -683,13 +688,13 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
         gnb = __bfloat162float(gsrc[i + half]);
       }
       const int hh_tile = row_a / hd;
-      for (int c0 = cbeg + half_sel; c0 < cend; c0 += 2 * kEpiBatch) {
+      for (int c0 = cbeg + grp; c0 < cend; c0 += ng * kEpiBatch) {
         // a batch's operands (accumulator pair and rotation), read before its first store
         float av[kEpiBatch], bv[kEpiBatch];
         float2 cs2[kEpiBatch];
 #pragma unroll
         for (int k = 0; k < kEpiBatch; ++k) {
-          const int c = c0 + 2 * k;
+          const int c = c0 + ng * k;
           const bool ok = c < cend;
           const float rs = !ok ? 1.f : (ep.qn_gain ? qkf[(c - cbeg) * 2 + hh_tile] : (ep.rs_sumsq ? rsc[c - cbeg] : 1.f));
           av[k] = ok ? acc[c * kBM + row_a] * rs * gna : 0.f;
@@ -698,7 +703,7 @@ __global__ void __launch_bounds__(128) gemm_cluster_kernel(const __grid_constant
         }
 #pragma unroll
         for (int k = 0; k < kEpiBatch; ++k) {
-          const int c = c0 + 2 * k;
+          const int c = c0 + ng * k;
           if (c >= cend) break;
           float a = av[k], b = bv[k];
           if (rot) {
@@ -814,6 +819,10 @@ GemmPlan plan_gemm(int M, int K, int n_pad, int num_sms, bool has_lo, bool gate_
       p.tmem_cols = 2 * p.tmem_cols;
     }
   }
+  // one CTA per SM (large batches, shared memory above half the SM's): eight warps instead of four at no
+  // cost in occupancy, so that the parking, the cluster reduction and the epilogue after the MMAs (tens
+  // of microseconds per layer at B = 256) run on twice the warps; the large-batch image only
+  p.threads = (n_pad >= 64 && p.smem_bytes + 1024 > 228u * 1024u / 2) ? 256 : 128;
   return p;
 }
 
@@ -834,7 +843,9 @@ cudaError_t launch_gemm(const GemmPlan& p, const CUtensorMap* tmW, const CUtenso
                         unsigned long long* ts, const GemmLowRank* lr) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((p.m_tiles + p.mt - 1) / p.mt * p.cluster, 1, 1);
-  cfg.blockDim = dim3(128, 1, 1);
+  const bool large = n_pad >= 64 || ep.mode == GemmEpilogue::LOWRANK;
+  if (p.threads != 128 && (p.threads != 256 || !large)) return cudaErrorInvalidValue;
+  cfg.blockDim = dim3(static_cast<unsigned>(p.threads), 1, 1);
   cfg.dynamicSmemBytes = p.smem_bytes;
   cfg.stream = stream;
   cudaLaunchAttribute attr[2];
@@ -856,7 +867,7 @@ cudaError_t launch_gemm(const GemmPlan& p, const CUtensorMap* tmW, const CUtenso
   const int k_main = with_lr ? lr->k_main : p.k_tiles;
   // the adapter's A x (LOWRANK) runs on the large-batch image at every batch size, so that the
   // small-batch image keeps its register allocation
-  if (n_pad >= 64 || ep.mode == GemmEpilogue::LOWRANK)
+  if (large)
     return cudaLaunchKernelEx(&cfg, gemm_cluster_kernel<true>, *tmW, *tmX, xlo, p.has_lo ? 1 : 0, mb, mt, mtl, k_main,
                               p.k_tiles, p.cluster, p.stages, p.tmem_cols, n_pad, p.mt, ep, err, ts);
   if (p.mt != 1) return cudaErrorInvalidValue;   // two m-tiles per CTA exist in the large-batch image only

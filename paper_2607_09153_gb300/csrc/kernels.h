@@ -25,6 +25,8 @@ struct GemmPlan {
   // m-tiles per CTA: 2 for a gate/up projection without split K whose one-tile CTAs would need two
   // waves (large batches); the CTA's stage then holds both weight tiles and one activation tile
   int mt = 1;
+  // threads per CTA: 128, or 256 where one CTA fits per SM (the large-batch image only)
+  int threads = 128;
   uint32_t tmem_cols = 32;
   size_t smem_bytes = 0;
 };
@@ -147,8 +149,8 @@ struct AttnWorkHost {
 // of <= 8 candidates by the persistent kernel; 2 shared pages scored on the
 // tensor cores (head_dim 128 only), tiles of <= 128 / group candidates, each
 // launch planned over all n_ctas SMs; 3 as 2, with the SMs split between the
-// tensor-core and the private launch in proportion to their estimated time,
-// so the two can run concurrently.
+// tensor-core and the private launch so that the later of the two (estimated
+// under a cost model) ends soonest, and the two run concurrently.
 bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks, int n_kv, int group, int n_ctas,
                      size_t slot_limit, int share, AttnWorkHost& w);
 // The plan with the combine fused into the attention launch, for calls where

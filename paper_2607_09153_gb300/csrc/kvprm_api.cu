@@ -1758,6 +1758,7 @@ int kvprm_plan_projection(int32_t M, int32_t K, int32_t n_pad, int32_t num_sms, 
   out->stages = g.stages;
   out->tmem_cols = static_cast<int32_t>(g.tmem_cols);
   out->smem_bytes = static_cast<int64_t>(g.smem_bytes);
+  out->threads = g.threads;
   return KVPRM_OK;
 }
 

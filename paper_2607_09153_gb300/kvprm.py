@@ -45,7 +45,8 @@ class KvprmWeights(ctypes.Structure):
 
 class KvprmProjectionPlan(ctypes.Structure):
     _fields_ = [(k, ctypes.c_int32) for k in ("m_tiles", "k_tiles", "kt_per_split", "cluster", "tiles_per_cta",
-                                               "stages", "tmem_cols")] + [("smem_bytes", ctypes.c_int64)]
+                                               "stages", "tmem_cols")] + [("smem_bytes", ctypes.c_int64),
+                                                                          ("threads", ctypes.c_int32)]
 
 
 class KvprmLora(ctypes.Structure):

@@ -244,3 +244,37 @@ def test_grad_mcts_tree_hd128():
     p_ref, pages, _, _ = _oracle(w, t)
     _compare(w.name, w, p, grad, p_ref, pages)
     sc.close()
+
+
+def test_grad_graph_matches_eager(monkeypatch):
+    """The gradient call's captured graph (the default) against the same call with eager launches
+    (KVPRM_NO_GRAPH=1): the same kernels, so the same values up to the order of float atomics on
+    pages several candidates read; and a second replay of the graph agrees with the first."""
+    torch = require_gpu()
+    import paper_2607_09153_gb300 as kp
+    t = ks.Tables.make(0.2)
+    w = ks.mcts_tree("g_graph", ks.ARCH_TINY, 510, branching=2, depth=3, lo=5, hi=60, gain_std=0.2)
+    dev = ks.DeviceInputs(w, t)
+    st = torch.cuda.current_stream().cuda_stream
+    out = []
+    for eager in (False, True):
+        if eager:
+            monkeypatch.setenv("KVPRM_NO_GRAPH", "1")
+        sc = make_scorer(dev, w.n_candidates, w.max_blocks)
+        grads = []
+        for _ in range(2):
+            grad = torch.full(dev.pool.shape, float("nan"), dtype=torch.float32, device="cuda")
+            p = kp.kvprm_score_grad(sc.ctx, dev.pool.data_ptr(), dev.n_pages, w.block_table, w.seq_lens,
+                                    w.n_candidates, grad.data_ptr(), st)
+            grads.append((p, grad))
+        kp.kvprm_check_device(sc.ctx)
+        out.append(grads)
+        sc.close()
+    refs = set(int(x) for b in range(w.n_candidates) for x in w.block_table[b, :(int(w.seq_lens[b]) + 15) // 16])
+    idx = sorted(refs)
+    (pg0, g0), (pg1, g1) = out[0]
+    (pe, ge), _ = out[1]
+    scale = float(ge[:, idx].abs().max())
+    for p, g in ((pg0, g0), (pg1, g1)):
+        assert np.abs(p - pe).max() <= 1e-6
+        assert float((g[:, idx] - ge[:, idx]).abs().max()) <= 1e-5 * scale
