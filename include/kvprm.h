@@ -393,7 +393,7 @@ KVPRM_API int kvprm_plan_attention(const int32_t* block_table, int32_t max_block
  *  cluster       CTAs per thread-block cluster (split-K ranks)
  *  tiles_per_cta m-tiles each CTA takes (1, or 2 for large batches)
  *  stages        shared-memory ring stages; tmem_cols tensor-memory columns; smem_bytes per CTA
- *  threads       threads per CTA: 256 where one CTA fits per SM and n_pad >= 64, else 128
+ *  threads       threads per CTA: 256 for n_pad >= 64 (the large-batch kernel image), else 128
  * Errors: KVPRM_EINVAL (M, K or num_sms < 1, n_pad not a positive multiple of 16, out NULL). */
 typedef struct {
   int32_t m_tiles, k_tiles, kt_per_split, cluster, tiles_per_cta, stages, tmem_cols;

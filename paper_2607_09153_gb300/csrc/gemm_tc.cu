@@ -68,7 +68,7 @@ __device__ __forceinline__ void store_hilo(__nv_bfloat16* hi, __nv_bfloat16* lo,
 // with 16-byte accesses (the 4-warp CTA is otherwise bound by 2- and 4-byte stores and by one load
 // latency per column).
 template <bool LARGE>
-__global__ void __launch_bounds__(256) gemm_cluster_kernel(const __grid_constant__ CUtensorMap tmW,
+__global__ void __launch_bounds__(256, 2) gemm_cluster_kernel(const __grid_constant__ CUtensorMap tmW,
                                                            const __grid_constant__ CUtensorMap tmX,
                                                            const __grid_constant__ CUtensorMap tmXlo, int has_lo,
                                                            const __grid_constant__ CUtensorMap tmB,
@@ -251,7 +251,7 @@ __global__ void __launch_bounds__(256) gemm_cluster_kernel(const __grid_constant
   if (threadIdx.x == 0) trace_event(ts, 2);   // all MMAs of this CTA completed
   tc_fence_after();
   float* acc = reinterpret_cast<float*>(smem);   // the ring is idle once `done` has fired
-  // 4 warps, or 8 (large batches with one CTA per SM): warps w and w + 4 share TMEM lane quadrant w,
+  // 4 warps, or 8 (the large-batch image): warps w and w + 4 share TMEM lane quadrant w,
   // i.e. the tile's rows 32 w .. 32 w + 31, and take alternate 16-column groups (or columns)
   const int nw = static_cast<int>(blockDim.x >> 5), nwh = nw >> 2, wh = warp >> 2;
   const int m = (warp & 3) * 32 + lane;
@@ -819,10 +819,9 @@ GemmPlan plan_gemm(int M, int K, int n_pad, int num_sms, bool has_lo, bool gate_
       p.tmem_cols = 2 * p.tmem_cols;
     }
   }
-  // one CTA per SM (large batches, shared memory above half the SM's): eight warps instead of four at no
-  // cost in occupancy, so that the parking, the cluster reduction and the epilogue after the MMAs (tens
-  // of microseconds per layer at B = 256) run on twice the warps; the large-batch image only
-  p.threads = (n_pad >= 64 && p.smem_bytes + 1024 > 228u * 1024u / 2) ? 256 : 128;
+  // the large-batch image runs eight warps instead of four (registers for two such CTAs per SM), so
+  // that the parking, the cluster reduction and the epilogue after the MMAs run on twice the warps
+  p.threads = n_pad >= 64 ? 256 : 128;
   return p;
 }
 

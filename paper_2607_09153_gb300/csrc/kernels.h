@@ -25,7 +25,7 @@ struct GemmPlan {
   // m-tiles per CTA: 2 for a gate/up projection without split K whose one-tile CTAs would need two
   // waves (large batches); the CTA's stage then holds both weight tiles and one activation tile
   int mt = 1;
-  // threads per CTA: 128, or 256 where one CTA fits per SM (the large-batch image only)
+  // threads per CTA: 256 on the large-batch image (n_pad >= 64), else 128
   int threads = 128;
   uint32_t tmem_cols = 32;
   size_t smem_bytes = 0;
