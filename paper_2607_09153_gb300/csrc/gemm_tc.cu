@@ -759,8 +759,15 @@ GemmPlan plan_gemm(int M, int K, int n_pad, int num_sms, bool has_lo, bool gate_
   // SMs at once (two per SM when two CTAs' shared memory fits, else one: at B = 256 a stage holds
   // 64 KB of activations) and gives every rank at least two K tiles
   const int per_sm = p.smem_bytes + 1024 <= 228u * 1024u / 2 ? 2 : 1;
+  // A cluster is placed whole on one GPC.  With two CTAs per SM, a grid that needs (nearly) every
+  // slot cannot be placed in one wave while the preceding kernel still holds part of the SMs
+  // (programmatic dependent launch places this grid's first clusters early, half-filling SMs in a
+  // pattern that strands slots): the 7B QKV projection at B = 64, 36 clusters of 8 = 288 of 304
+  // slots, had its last clusters start ~10 us after the preceding kernel ended.  Such grids keep
+  // within 7/8 of the slots.
+  const int slots = per_sm == 2 ? per_sm * num_sms * 7 / 8 : per_sm * num_sms;
   int cs = 1;
-  while (cs < 16 && p.m_tiles * cs * 2 <= per_sm * num_sms && cs * 4 <= p.k_tiles && cs * 2 <= n_pad) cs *= 2;
+  while (cs < 16 && p.m_tiles * cs * 2 <= slots && cs * 4 <= p.k_tiles && cs * 2 <= n_pad) cs *= 2;
   p.cluster = cs;
   p.splits = cs;
   p.kt_per_split = (p.k_tiles + cs - 1) / cs;

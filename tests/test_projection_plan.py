@@ -66,3 +66,20 @@ def test_projection_plan_beyond_context_batch():
             kp.kvprm_plan_projection(4608, 3584, n_pad, SMS)
         assert e.value.code == kp.KVPRM_EUNSUPPORTED
     assert kp.kvprm_plan_projection(4608, 3584, 256, SMS)["tmem_cols"] <= 512
+
+
+@pytest.mark.parametrize("arch", [ks.ARCH_TINY, ks.ARCH_1P5B, ks.ARCH_7B, ks.ARCH_8B])
+@pytest.mark.parametrize("n_pad", [16, 32, 64, 96, 128, 256])
+def test_projection_plan_cluster_placement(arch, n_pad):
+    """Whole clusters are placed on one GPC: where two CTAs share an SM, a split-K grid keeps within
+    7/8 of the CTA slots, so that it is placed in one wave beside the preceding kernel's CTAs (the
+    7B QKV projection at B = 64 takes clusters of 4, 144 CTAs, not 36 clusters of 8 = 288 of 304)."""
+    for name, M, K, gu in _shapes(arch):
+        p = kp.kvprm_plan_projection(M, K, n_pad, SMS, True, gu)
+        if p["cluster"] == 1:
+            continue
+        two_per_sm = p["smem_bytes"] + 1024 <= 228 * 1024 // 2
+        ctas = (p["m_tiles"] + p["tiles_per_cta"] - 1) // p["tiles_per_cta"] * p["cluster"]
+        assert ctas <= (2 * SMS * 7 // 8 if two_per_sm else SMS), f"{name} n_pad={n_pad}: {ctas} CTAs"
+    qkv = kp.kvprm_plan_projection(ks.ARCH_7B.qkv_rows, ks.ARCH_7B.d_model, 64, SMS)
+    assert (qkv["cluster"], qkv["m_tiles"]) == (4, 36)
