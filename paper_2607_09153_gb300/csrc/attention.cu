@@ -75,9 +75,10 @@ __host__ __device__ constexpr int shared_reps(int n_cands) { return kConsumerWar
 // The tensor-core launch, in the same units, when it runs beside the private pages' launch: a CTA
 // costs kTcChunkCost per 64-token chunk plus kTcCtaCost once (the first query load and pages'
 // latency, the last output read-out).  Fitted to the SM split that measured fastest on the beam
-// (86 of 152 SMs, 12 chunks per CTA) and MCTS (17 SMs, ~110 chunks per CTA) workloads: ~1.3 us per
-// chunk and ~8 us per CTA against ~0.045 us per unit on the private side.
-constexpr int64_t kTcChunkCost = 29;
+// (86 of 152 SMs, 12 chunks per CTA) and MCTS (16 SMs, ~115 chunks per CTA) workloads: ~1.2 us per
+// chunk and ~8 us per CTA against ~0.045 us per unit on the private side (a sweep of 24-29 units
+// per chunk and 150-210 per CTA moved the MCTS attention by a few percent, 26 fastest; beam alike).
+constexpr int64_t kTcChunkCost = 26;
 constexpr int64_t kTcCtaCost = 180;
 // pages shared by fewer candidates go to the persistent kernel as kind-1 runs: 2 units per page
 // and candidate there against kTcChunkCost / 4 per page on the tensor cores, whatever the tile's rows
@@ -238,7 +239,15 @@ __global__ void __launch_bounds__(kThreads, 1) attn_kernel(
               process_page<HD, TWO_ROWS>(q, kb, kb + SM::kBlockBytes, valid, lane, st);
             }
           } else {         // this replica's pages of this stage, for this warp's candidate
-            for (int pi = part; pi < npg; pi += reps) {
+            int pi = part;
+            if (!TWO_ROWS)   // two pages at a time: their dependent steps overlap
+              for (; pi + reps < npg; pi += 2 * reps) {
+                const int va = p0 + pi == sg.n_pages - 1 ? sg.last_valid : 16;
+                const int vb = p0 + pi + reps == sg.n_pages - 1 ? sg.last_valid : 16;
+                const uint32_t ka = sbase + pi * SM::kPageBytes, kb = sbase + (pi + reps) * SM::kPageBytes;
+                process_page_pair<HD>(q, ka, ka + SM::kBlockBytes, va, kb, kb + SM::kBlockBytes, vb, lane, st);
+              }
+            for (; pi < npg; pi += reps) {
               const int valid = p0 + pi == sg.n_pages - 1 ? sg.last_valid : 16;
               const uint32_t kb = sbase + pi * SM::kPageBytes;
               process_page<HD, TWO_ROWS>(q, kb, kb + SM::kBlockBytes, valid, lane, st);

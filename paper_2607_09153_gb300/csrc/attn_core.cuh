@@ -207,6 +207,120 @@ __device__ __forceinline__ void process_page(const WarpQ<HD>& q, uint32_t kbase,
   }
 }
 
+// Two pages (A, then B) of a shared run for one warp's packed query rows (group <= 8).  The
+// arithmetic of two process_page calls, except that the two pages' 32 scores per row meet one
+// running-maximum update (the online softmax over a 32-token block), so the second page's score
+// MMAs, maximum and exponentials proceed beside the first's: a warp scoring several pages of a
+// stage for one candidate is otherwise held by each page's chain of dependent steps.
+template <int HD>
+__device__ __forceinline__ void process_page_pair(const WarpQ<HD>& q, uint32_t kbA, uint32_t vbA, int validA,
+                                                  uint32_t kbB, uint32_t vbB, int validB, int lane,
+                                                  WarpState<HD>& st) {
+  const int tig = lane & 3;
+  const float sl2 = kLog2e * rsqrtf(static_cast<float>(HD));
+  // S = Q K^T for both pages: [page][n-tile of 8 tokens][4] (four independent accumulation chains)
+  float s[2][2][4];
+#pragma unroll
+  for (int pg = 0; pg < 2; ++pg)
+#pragma unroll
+    for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) s[pg][nt][i] = 0.f;
+  {
+    const int mi = lane >> 3, r = lane & 7;
+    const int tok = (mi >> 1) * 8 + r;
+#pragma unroll
+    for (int pg = 0; pg < 2; ++pg) {
+      const uint32_t kbase = pg ? kbB : kbA;
+#pragma unroll
+      for (int h = 0; h < HD / 64; ++h) {   // K fragments of four K steps at a time (register budget)
+        uint32_t kb[4][4];
+#pragma unroll
+        for (int k4 = 0; k4 < 4; ++k4) {
+          const int hdc = (4 * h + k4) * 16 + (mi & 1) * 8;
+          const uint32_t addr = kbase + (hdc >> 6) * 2048 + tok * 128 + ((((hdc & 63) >> 3) ^ (tok & 7)) << 4);
+          ldsm_x4(addr, kb[k4][0], kb[k4][1], kb[k4][2], kb[k4][3]);
+        }
+#pragma unroll
+        for (int k4 = 0; k4 < 4; ++k4) {
+          const int ks = 4 * h + k4;
+          mma_bf16_16816(s[pg][0], q.a0[ks], q.a1[ks], q.a2[ks], q.a3[ks], kb[k4][0], kb[k4][1]);
+          mma_bf16_16816(s[pg][1], q.a0[ks], q.a1[ks], q.a2[ks], q.a3[ks], kb[k4][2], kb[k4][3]);
+        }
+      }
+    }
+  }
+  const int c0 = tig * 2, c1 = tig * 2 + 1, c2 = 8 + tig * 2, c3 = 9 + tig * 2;
+  float x[2][4];
+  float mx = -INFINITY;
+#pragma unroll
+  for (int pg = 0; pg < 2; ++pg) {
+    const int valid = pg ? validB : validA;
+    // hi (row gid) + lo (row gid + 8) parts of the same head
+    x[pg][0] = c0 < valid ? (s[pg][0][0] + s[pg][0][2]) * sl2 : -INFINITY;
+    x[pg][1] = c1 < valid ? (s[pg][0][1] + s[pg][0][3]) * sl2 : -INFINITY;
+    x[pg][2] = c2 < valid ? (s[pg][1][0] + s[pg][1][2]) * sl2 : -INFINITY;
+    x[pg][3] = c3 < valid ? (s[pg][1][1] + s[pg][1][3]) * sl2 : -INFINITY;
+    mx = fmaxf(mx, fmaxf(fmaxf(x[pg][0], x[pg][1]), fmaxf(x[pg][2], x[pg][3])));
+  }
+  mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+  mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+  const float m_new = fmaxf(st.m[0], mx);
+  if (__any_sync(0xffffffffu, m_new > st.m[0])) {   // warp-uniform: rescale O by 2^(m_old - m_new)
+    const float alpha = exp2f(st.m[0] - m_new);
+    st.l[0] *= alpha;
+#pragma unroll
+    for (int n = 0; n < HD / 8; ++n) {
+      st.o[n][0] *= alpha;
+      st.o[n][1] *= alpha;
+      st.o[n][2] *= alpha;
+      st.o[n][3] *= alpha;
+    }
+    st.m[0] = m_new;
+  }
+  uint32_t ph[2][4];   // A fragments of P per page: rows gid = P_hi, gid + 8 = P_lo
+#pragma unroll
+  for (int pg = 0; pg < 2; ++pg) {
+    float p[4];
+#pragma unroll
+    for (int i2 = 0; i2 < 4; ++i2) p[i2] = exp2f(x[pg][i2] - m_new);
+    st.l[0] += (p[0] + p[1]) + (p[2] + p[3]);
+    float hi[4], lo[4];
+#pragma unroll
+    for (int i2 = 0; i2 < 4; ++i2) {
+      hi[i2] = __bfloat162float(__float2bfloat16_rn(p[i2]));
+      lo[i2] = p[i2] - hi[i2];
+    }
+    ph[pg][0] = pack_bf16(hi[0], hi[1]);
+    ph[pg][1] = pack_bf16(lo[0], lo[1]);
+    ph[pg][2] = pack_bf16(hi[2], hi[3]);
+    ph[pg][3] = pack_bf16(lo[2], lo[3]);
+  }
+  // O += P V for page A, then page B (V^T fragments through ldmatrix.trans)
+  const int mi = lane >> 3;
+  const int tok = (mi & 1) * 8 + (lane & 7);
+#pragma unroll
+  for (int pg = 0; pg < 2; ++pg) {
+    const uint32_t vbase = pg ? vbB : vbA;
+#pragma unroll
+    for (int h = 0; h < HD / 64; ++h) {   // V fragments of four 16-column groups at a time (register budget)
+      uint32_t vb[4][4];
+#pragma unroll
+      for (int k4 = 0; k4 < 4; ++k4) {
+        const int hdc = (4 * h + k4) * 16 + (mi >> 1) * 8;
+        const uint32_t addr = vbase + (hdc >> 6) * 2048 + tok * 128 + ((((hdc & 63) >> 3) ^ (tok & 7)) << 4);
+        ldsm_x4_t(addr, vb[k4][0], vb[k4][1], vb[k4][2], vb[k4][3]);
+      }
+#pragma unroll
+      for (int k4 = 0; k4 < 4; ++k4) {
+        const int j2 = 4 * h + k4;
+        mma_bf16_16816(st.o[2 * j2], ph[pg][0], ph[pg][1], ph[pg][2], ph[pg][3], vb[k4][0], vb[k4][1]);
+        mma_bf16_16816(st.o[2 * j2 + 1], ph[pg][0], ph[pg][1], ph[pg][2], ph[pg][3], vb[k4][2], vb[k4][3]);
+      }
+    }
+  }
+}
+
 // End of a run of pages for one warp: fold the lo-part rows onto their heads
 // (packed layout) and quad-reduce the row sums.
 template <int HD, bool TWO_ROWS>
