@@ -76,7 +76,7 @@ __host__ __device__ constexpr int shared_reps(int n_cands) { return kConsumerWar
 // costs kTcChunkCost per 64-token chunk plus kTcCtaCost once (the first query load and pages'
 // latency, the last output read-out).  Fitted to the SM split that measured fastest on the beam
 // (86 of 152 SMs, 12 chunks per CTA) and MCTS (16 SMs, ~115 chunks per CTA) workloads: ~1.2 us per
-// chunk and ~8 us per CTA against ~0.045 us per unit on the private side (a sweep of 24-29 units
+// chunk and ~8 us per CTA against ~0.045 us per unit on the private side (a sweep of 24-32 units
 // per chunk and 150-210 per CTA moved the MCTS attention by a few percent, 26 fastest; beam alike).
 constexpr int64_t kTcChunkCost = 26;
 constexpr int64_t kTcCtaCost = 180;
