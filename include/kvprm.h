@@ -300,8 +300,8 @@ KVPRM_API int kvprm_attention_noalloc(const void* kv_layer, int64_t n_pages, con
  * 11 loading Q; 12 chunks scored; 13 the CTA's lifetime.  Bit 6: the combine
  * of one verify token per candidate takes its flat form (one warp per query
  * head, every slot's partial loaded in one round) at every batch size, not
- * only when the (candidate, kv head) pairs exceed one wave of the general
- * form (same result up to rounding; exercises the flat form). */
+ * only when the (candidate, kv head) pairs outnumber the SMs (same result up
+ * to rounding; exercises the flat form). */
 KVPRM_API int kvprm_set_debug(kvprm_ctx* ctx, int flags);
 KVPRM_API int kvprm_debug_attn_out(kvprm_ctx* ctx, float* d_out);
 KVPRM_API int kvprm_debug_layers(kvprm_ctx* ctx, int which, void* d_out);

@@ -1458,11 +1458,13 @@ cudaError_t launch_attn_combine(const AttnShape& s, const AttnWork& wk, int n, c
                                                  cudaSuccess)
       sms = 1;
   }
-  const bool narrow = static_cast<int64_t>(n) * s.n_kv > 6 * static_cast<int64_t>(sms);
-  // A single verify token per candidate with more pairs than one wave of the general form (whose
-  // 4-warp CTAs then take two waves of several memory round trips each): the flat combine, about
-  // 1 % more MCTS scores per second; fewer pairs keep the general form (measured no faster flat).
-  if (mg.depth == 1 && (narrow || force_flat)) {
+  const int64_t pairs = static_cast<int64_t>(n) * s.n_kv;
+  const bool narrow = pairs > 6 * static_cast<int64_t>(sms);
+  // A single verify token per candidate with more (candidate, kv head) pairs than SMs: the flat
+  // combine, one memory round trip per warp (beam's 256 pairs: 17.09k -> 17.30k scores/s; MCTS's
+  // 1,024, where the general form's 4-warp CTAs took two waves of several round trips: ~1 %); fewer
+  // pairs keep the general form (long 8B's 64: the flat form 0.6 % slower).
+  if (mg.depth == 1 && (pairs > sms || force_flat)) {
     cfg.dynamicSmemBytes = 0;
     cfg.blockDim = dim3(32 * static_cast<unsigned>(s.group), 1, 1);
     if (s.hd == 128)

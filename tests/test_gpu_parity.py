@@ -126,7 +126,7 @@ def test_fused_combine(lens, fused, monkeypatch):
 
 def test_narrow_combine():
     # more (candidate, kv head) pairs than one wave of the general combine (240 candidates x 4 kv
-    # heads = 960 > 6 x 152; a context holds at most 256 candidates): the flat combine
+    # heads = 960 > 6 x 152; a context holds at most 256 candidates), and than the SMs: the flat combine
     t = ks.Tables.make(0.2)
     lens = [int(x) for x in np.random.default_rng(47).integers(0, 60, size=240)]
     w = ks.distinct("narrow", ks.Arch(2, 256, 8, 4, 64, 512), 47, lens, gain_std=0.2)
