@@ -242,15 +242,16 @@ def cpu_oracle_time(w, tables, budget_s: float = 12.0, depth: int = 1, nthreads:
 
 def run_reference(args, world, rank):
     """The reference arm: the CPU oracle as it stands, on this host's cores.  One step scores a fixed
-    sample of the workload's candidates (sized so that a step takes ~--ref-step-s); ms_per_step is
-    that observed step time and value the sample's candidates per second."""
+    sample of the workload's candidates, sized by the rule the main arm's cpu_baseline uses (about
+    --cpu-budget of work, or ~--ref-step-s per step when given); ms_per_step is that observed step
+    time and value the sample's candidates per second."""
     if rank != 0:
         return
     import kvsynth as ks
     w = make_workload(args)
     t = ks.Tables.make()
     runner = OracleRunner(w, t, depth=args.depth)
-    n = runner.sample_size(args.ref_step_s)
+    n = runner.sample_size(args.ref_step_s if args.ref_step_s > 0 else args.cpu_budget)
     ids = list(range(n))
     times = []
     for i in range(args.warmup + args.steps):
@@ -707,8 +708,9 @@ def main():
     ap.add_argument("--workload", default="long8b_b8_l32768", choices=list(ks.WORKLOAD_NAMES))
     ap.add_argument("--no-workloads", action="store_true",
                     help="measure the --workload alone (by default the other configurations follow, shorter)")
-    ap.add_argument("--ref-step-s", type=float, default=3.0,
-                    help="reference arm: candidates per step chosen so that one step takes about this long")
+    ap.add_argument("--ref-step-s", type=float, default=0.0,
+                    help="reference arm: candidates per step chosen so that one step takes about this long "
+                         "(0, the default: the --cpu-budget rule, so the arm times the cpu_baseline's sample)")
     ap.add_argument("--depth", type=int, default=1,
                     help="verify tokens per candidate (depth-k readout; 1, the default: one)")
     ap.add_argument("--layers", type=int, default=0,
