@@ -1167,11 +1167,43 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
   const int C = total == 0 ? 0
                            : static_cast<int>(std::max<int64_t>(
                                  1, std::min<int64_t>(priv_ctas, total / (kPagesPerStage * kPrivateCost))));
+  // The (run, kv head) pairs in axis order: the pairs of shared runs (bound by their MMAs: a warp
+  // per candidate scores every page) interleaved with the private pairs (bound by HBM) in proportion
+  // to their cost, so that every CTA's range mixes both kinds and its ring fetches the private pages
+  // of a later segment while its warps score the shared pages of the current one.
+  std::vector<std::pair<int, int>> pairs;
+  {
+    std::vector<std::pair<int, int>> sh, pv;
+    int64_t c_sh = 0, c_pv = 0;
+    for (size_t ri = 0; ri < runs.size(); ++ri) {
+      const Run& r = runs[ri];
+      if (r.kind == 2) continue;
+      for (int g = 0; g < n_kv; ++g) (r.kind == 1 ? sh : pv).emplace_back(static_cast<int>(ri), g);
+      (r.kind == 1 ? c_sh : c_pv) += static_cast<int64_t>(r.n_pages) * r.cost * n_kv;
+    }
+    auto cost_of = [&](const std::pair<int, int>& pr) {
+      return static_cast<int64_t>(runs[pr.first].n_pages) * runs[pr.first].cost;
+    };
+    size_t a = 0, b = 0;
+    int64_t d_sh = 0, d_pv = 0;   // cost laid so far of each kind
+    while (a < sh.size() || b < pv.size()) {
+      // the kind whose laid fraction of its own total is smaller goes next
+      const bool take_sh = b >= pv.size() || (a < sh.size() && d_sh * c_pv <= d_pv * c_sh);
+      if (take_sh) {
+        d_sh += cost_of(sh[a]);
+        pairs.push_back(sh[a++]);
+      } else {
+        d_pv += cost_of(pv[b]);
+        pairs.push_back(pv[b++]);
+      }
+    }
+  }
   std::vector<int> seg_cta;
   int64_t pos = 0;   // cost position of the current pair's first unit
-  for (const Run& r : runs) {
-    if (r.kind == 2) continue;
-    for (int g = 0; g < n_kv; ++g) {
+  for (const auto& pr : pairs) {
+    const Run& r = runs[pr.first];
+    {
+      const int g = pr.second;
       const int units = r.n_pages;
       const int64_t c = r.cost;
       int i = 0;
