@@ -208,9 +208,17 @@ KVPRM_API int kvprm_score_async(kvprm_ctx* ctx, const void* kv_pages, int64_t n_
                       const int32_t* seq_lens, int32_t n_candidates, float* d_rewards, void* stream);
 
 /* As kvprm_score, but with the cache in HOST memory: h_kv_pages has the
- * kv_pages layout above (pinned memory gives full copy bandwidth).  The pages
- * are copied into a library-owned device pool (grown on demand) on `stream`
- * before scoring; rewards is a host array.  Blocking. */
+ * kv_pages layout above.  The pages are copied, layer by layer, into a
+ * library-owned device pool (grown on demand) after the work already on
+ * `stream`, and each layer's attention waits only for its own layer, so the
+ * copy of later layers overlaps the scoring of earlier ones; rewards is a host
+ * array.  Blocking.  Pinned host memory (page-locked by cudaHostAlloc or
+ * cudaHostRegister; first and last byte checked) at a 16-byte aligned address
+ * is read by a copy kernel (64 CTAs of 128 threads, 64 MB per launch) that
+ * shares SMs with the scoring kernels and holds the host link at its full
+ * rate; any other host memory goes through the copy engine (cudaMemcpyAsync).
+ * While the copy runs, the forward's kernels are launched without
+ * programmatic dependent launch. */
 KVPRM_API int kvprm_score_host(kvprm_ctx* ctx, const void* h_kv_pages, int64_t n_pages, const int32_t* block_table,
                      const int32_t* seq_lens, int32_t n_candidates, float* rewards, void* stream);
 

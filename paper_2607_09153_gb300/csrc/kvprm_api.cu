@@ -807,30 +807,61 @@ void drop_graph(kvprm_ctx* ctx) {
   ctx->gkey = GraphKey();
 }
 
-// Score into ctx->rewards_d on stream `st` (stream-ordered).
+// The device address of host memory [p, p + bytes) when the GPU can read all of it as pinned memory:
+// its first and last byte page-locked (cudaMemoryTypeHost) and mapped at one contiguous device range,
+// p and bytes 16-byte aligned; else null (pageable memory, or anything the query cannot vouch for).
+const void* pinned_device_view(const void* p, size_t bytes) {
+  if (!p || bytes == 0 || !aligned16(p) || (bytes & 15u)) return nullptr;
+  const uint8_t* last = static_cast<const uint8_t*>(p) + bytes - 1;
+  cudaPointerAttributes a0{}, a1{};
+  if (cudaPointerGetAttributes(&a0, p) != cudaSuccess || cudaPointerGetAttributes(&a1, last) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  if (a0.type != cudaMemoryTypeHost || a1.type != cudaMemoryTypeHost || !a0.devicePointer || !a1.devicePointer)
+    return nullptr;
+  if (static_cast<const uint8_t*>(a1.devicePointer) - static_cast<const uint8_t*>(a0.devicePointer) !=
+      static_cast<std::ptrdiff_t>(bytes - 1))
+    return nullptr;
+  return aligned16(a0.devicePointer) ? a0.devicePointer : nullptr;
+}
+
 // kvprm_score_host's cache copy: layer by layer, in layer order on ONE copy stream (the copy engine
 // drains one stream's queue before the next, so layers spread over several streams arrive out of
 // order), after the work already on `st` (an earlier call may still read the pool, and this call's
 // tables go first, so that the small table copies do not queue behind the cache); layer l's event
-// gates layer l's attention.
+// gates layer l's attention.  Pinned host memory is pulled by SM loads (launch_pool_pull) in 64 MB
+// launches, so that a scoring kernel whose CTAs cannot be placed beside the copy's waits for at most
+// one launch (~0.3 ms): with one launch per layer (1 GB, ~5 ms) the long 8B call took 248-264 ms,
+// in 64 MB launches 177 ms, against 163 ms for its 34 GB at the link's ~211 GB/s.  Other host
+// memory goes through the copy engine.
 int enqueue_pool_copy(kvprm_ctx* ctx, cudaStream_t st) {
   CK(cudaEventRecord(ctx->pool_free, st), "cudaEventRecord(pool free)");
   const size_t layer_bytes = ctx->host_pool_bytes / static_cast<size_t>(ctx->cfg.n_layers);
   cudaStream_t cs = ctx->copy_stream;
   CK(cudaStreamWaitEvent(cs, ctx->pool_free, 0), "cudaStreamWaitEvent(pool)");
+  const void* src = pinned_device_view(ctx->host_pool, ctx->host_pool_bytes);
+  const size_t piece = size_t(64) << 20;
   for (int l = 0; l < ctx->cfg.n_layers; ++l) {
-    CK(cudaMemcpyAsync(static_cast<uint8_t*>(ctx->dev_pool) + l * layer_bytes,
-                       static_cast<const uint8_t*>(ctx->host_pool) + l * layer_bytes, layer_bytes,
-                       cudaMemcpyHostToDevice, cs),
-       "cudaMemcpyAsync(pool layer)");
+    uint8_t* dst = static_cast<uint8_t*>(ctx->dev_pool) + l * layer_bytes;
+    if (src) {
+      for (size_t off = 0; off < layer_bytes; off += piece)
+        CK(kvprm::launch_pool_pull(static_cast<const uint8_t*>(src) + l * layer_bytes + off, dst + off,
+                                   std::min(piece, layer_bytes - off), cs),
+           "pool_pull_kernel");
+    } else {
+      CK(cudaMemcpyAsync(dst, static_cast<const uint8_t*>(ctx->host_pool) + l * layer_bytes, layer_bytes,
+                         cudaMemcpyHostToDevice, cs),
+         "cudaMemcpyAsync(pool layer)");
+    }
     CK(cudaEventRecord(ctx->layer_ready[l], cs), "cudaEventRecord(layer ready)");
   }
   return KVPRM_OK;
 }
 
-// With `prepared` set, the call is planned and its tables uploaded (stream-ordered on `st`), and
-// its plan returned there instead of enqueueing the forward (the gradient call enqueues the forward
-// together with the backward).
+// Score into ctx->rewards_d on stream `st` (stream-ordered).  With `prepared` set, the call is
+// planned and its tables uploaded (stream-ordered on `st`), and its plan returned there instead of
+// enqueueing the forward (the gradient call enqueues the forward together with the backward).
 int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const int32_t* bt, const int32_t* sl, int32_t n,
                  cudaStream_t st, const FwdSaves* sv = nullptr, CallPlan* prepared = nullptr) {
   int max_pages = 0;
@@ -886,8 +917,12 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
     return KVPRM_OK;
   }
 
+  // While the cache of a host-buffer call is being copied in by SM loads, no launch is made early:
+  // a kernel that programmatic dependent launch places ahead of its predecessor's end holds SM slots
+  // the copy's CTAs would use (long 8B from pinned memory: 177.5 ms per call with, 171.5 ms without).
+  const bool pdl = ctx->use_pdl && !ctx->profile && !ctx->layer_waits;
   if (!ctx->use_graph || sv) {   // a forward that keeps its intermediates runs eagerly
-    Enq E{ctx, st, ctx->use_pdl && !ctx->profile, ctx->profile, &ctx->live_marks};
+    Enq E{ctx, st, pdl, ctx->profile, &ctx->live_marks};
     if ((rc = enqueue_forward(ctx, P, E, sv))) return rc;
     if (ctx->profile) {
       CK(cudaStreamSynchronize(st), "cudaStreamSynchronize(profile)");
@@ -907,14 +942,14 @@ int score_device(kvprm_ctx* ctx, const void* kv_pages, int64_t n_pages, const in
   key.n_tc = ctx->work_host.n_tc > 0 ? 1 : 0;
   key.debug = ctx->debug_flags;
   key.profile = ctx->profile ? 1 : 0;
-  key.pdl = ctx->use_pdl ? 1 : 0;
+  key.pdl = pdl ? 1 : 0;
   key.trace = ctx->trace ? 1 : 0;
   key.pool = pool;
   key.n_pages = pages;
   if (!(ctx->gexec && key == ctx->gkey)) {
     drop_graph(ctx);
     CK(cudaStreamBeginCapture(ctx->cap_stream, cudaStreamCaptureModeThreadLocal), "cudaStreamBeginCapture");
-    Enq E{ctx, ctx->cap_stream, ctx->use_pdl && !ctx->profile, ctx->profile, &ctx->graph_marks};
+    Enq E{ctx, ctx->cap_stream, pdl, ctx->profile, &ctx->graph_marks};
     E.capturing = true;
     rc = enqueue_forward(ctx, P, E);
     cudaGraph_t graph = nullptr;

@@ -220,10 +220,23 @@ def test_deterministic_and_host_path():
     r1, _, dev, sc = run_gpu(w, t, debug=False)
     r2 = sc.score(dev.pool, w.block_table, w.seq_lens)
     assert np.array_equal(r1.astype(np.float32), r2)
+    sp = torch.cuda.current_stream().cuda_stream
+    # the host cache pinned, pageable, and pinned at an address 8 bytes off a 16-byte boundary: the
+    # same rewards, bit for bit, and the pinned buffer again after the others
     host_pool = dev.pool.cpu().pin_memory()
-    r3 = kp.kvprm_score_host(sc.ctx, host_pool.data_ptr(), dev.n_pages, w.block_table, w.seq_lens, w.n_candidates,
-                             torch.cuda.current_stream().cuda_stream)
+    r3 = kp.kvprm_score_host(sc.ctx, host_pool.data_ptr(), dev.n_pages, w.block_table, w.seq_lens, w.n_candidates, sp)
     assert np.array_equal(r3, r2)
+    pageable = dev.pool.cpu()
+    assert not pageable.is_pinned()
+    r4 = kp.kvprm_score_host(sc.ctx, pageable.data_ptr(), dev.n_pages, w.block_table, w.seq_lens, w.n_candidates, sp)
+    assert np.array_equal(r4, r2)
+    raw = torch.empty(host_pool.numel() * 2 + 16, dtype=torch.uint8).pin_memory()
+    off = (8 - raw.data_ptr()) % 16
+    raw[off:off + host_pool.numel() * 2].copy_(host_pool.view(-1).view(torch.uint8))
+    r5 = kp.kvprm_score_host(sc.ctx, raw.data_ptr() + off, dev.n_pages, w.block_table, w.seq_lens, w.n_candidates, sp)
+    assert np.array_equal(r5, r2)
+    r6 = kp.kvprm_score_host(sc.ctx, host_pool.data_ptr(), dev.n_pages, w.block_table, w.seq_lens, w.n_candidates, sp)
+    assert np.array_equal(r6, r2)
     d = torch.empty(w.n_candidates, dtype=torch.float32, device="cuda")
     sc.score_async(dev.pool, w.block_table, w.seq_lens, d)
     torch.cuda.synchronize()
