@@ -394,9 +394,12 @@ def measure(w, args, world, local, steps: int, warmup: int, prof_steps: int, wit
         for _ in range(e2e_steps):
             kp.kvprm_score_host(sc.ctx, host_pool.data_ptr(), n_pages, bt, sl, B, sp, rewards)
         t_e2e = max_over_ranks(time.perf_counter() - t0, world)
+        h2d = int(host_pool.numel() * 2 + bt.nbytes + sl.nbytes)
         out["e2e"] = {"value": world * B * e2e_steps / t_e2e, "unit": "scores/s",
-                      "h2d_bytes_per_step": int(host_pool.numel() * 2 + bt.nbytes + sl.nbytes),
-                      "d2h_bytes_per_step": int(B * 4 + 4), "steps": e2e_steps,
+                      "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": int(B * 4 + 4), "steps": e2e_steps,
+                      # host->device bytes moved per second inside the timed region (the host link's
+                      # ~211 GB/s bounds it: the call is copy-bound)
+                      "h2d_gbs": round(h2d * e2e_steps / t_e2e / 1e9, 1),
                       "path": "kvprm_score_host: pinned host cache + host tables -> rewards on host"}
         del host_pool
 
