@@ -291,11 +291,5 @@ cudaError_t launch_steer_update(__nv_bfloat16* kv, const float* grad, const int3
 // records kDevProbeTimeout in *err.  The failure-detection test hook behind kvprm_debug_wait_probe.
 cudaError_t launch_wait_probe(const int* flag, int* err, unsigned long long limit_ns, cudaStream_t stream);
 
-// Copy `bytes` (a multiple of 16; both addresses 16-byte aligned, else cudaErrorInvalidValue) from
-// device-accessible pinned host memory `src` into device memory `dst` with kPoolPullCtas CTAs of
-// 128 threads doing SM loads.
-constexpr int kPoolPullCtas = 64;
-cudaError_t launch_pool_pull(const void* src, void* dst, size_t bytes, cudaStream_t stream);
-
 
 }  // namespace kvprm

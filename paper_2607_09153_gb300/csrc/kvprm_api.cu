@@ -807,6 +807,44 @@ void drop_graph(kvprm_ctx* ctx) {
   ctx->gkey = GraphKey();
 }
 
+// Host-resident cache pages into the device pool by SM loads of pinned host memory: every thread
+// moves 16 bytes per step, four steps in flight (grid-stride).  Measured on GB300 (8 GB of pinned
+// memory): 64 CTAs of 4 warps hold the host link at ~211 GB/s on every copy, where copy-engine
+// copies of the same buffer ran at ~211 GB/s on most copies and ~120 GB/s on others.  Small CTAs
+// (128 threads, no shared memory, the maximum shared-memory carve-out) share SMs with the scoring
+// kernels that run meanwhile.
+__global__ void __launch_bounds__(128) pool_pull_kernel(const uint4* __restrict__ src, uint4* __restrict__ dst,
+                                                        int64_t n) {
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  int64_t i = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
+  for (; i + 3 * stride < n; i += 4 * stride) {
+    const uint4 a = src[i], b = src[i + stride], c = src[i + 2 * stride], d = src[i + 3 * stride];
+    dst[i] = a;
+    dst[i + stride] = b;
+    dst[i + 2 * stride] = c;
+    dst[i + 3 * stride] = d;
+  }
+  for (; i < n; i += stride) dst[i] = src[i];
+}
+
+constexpr int kPoolPullCtas = 64;
+
+// Copy `bytes` (a multiple of 16; both addresses 16-byte aligned, else cudaErrorInvalidValue) from
+// device-accessible pinned host memory `src` into device memory `dst`.
+cudaError_t launch_pool_pull(const void* src, void* dst, size_t bytes, cudaStream_t stream) {
+  if (bytes == 0) return cudaSuccess;
+  if ((reinterpret_cast<uintptr_t>(src) | reinterpret_cast<uintptr_t>(dst) | bytes) & 15u) return cudaErrorInvalidValue;
+  // the SMs keep the shared-memory configuration of the scoring kernels while these CTAs sit beside
+  // them (a CTA preferring a larger L1 would wait for an SM to drain first)
+  static const cudaError_t carve =
+      cudaFuncSetAttribute(pool_pull_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           static_cast<int>(cudaSharedmemCarveoutMaxShared));
+  if (carve != cudaSuccess) return carve;
+  pool_pull_kernel<<<kPoolPullCtas, 128, 0, stream>>>(static_cast<const uint4*>(src), static_cast<uint4*>(dst),
+                                                      static_cast<int64_t>(bytes / 16));
+  return cudaGetLastError();
+}
+
 // The device address of host memory [p, p + bytes) when the GPU can read all of it as pinned memory:
 // its first and last byte page-locked (cudaMemoryTypeHost) and mapped at one contiguous device range,
 // p and bytes 16-byte aligned; else null (pageable memory, or anything the query cannot vouch for).
@@ -846,7 +884,7 @@ int enqueue_pool_copy(kvprm_ctx* ctx, cudaStream_t st) {
     uint8_t* dst = static_cast<uint8_t*>(ctx->dev_pool) + l * layer_bytes;
     if (src) {
       for (size_t off = 0; off < layer_bytes; off += piece)
-        CK(kvprm::launch_pool_pull(static_cast<const uint8_t*>(src) + l * layer_bytes + off, dst + off,
+        CK(launch_pool_pull(static_cast<const uint8_t*>(src) + l * layer_bytes + off, dst + off,
                                    std::min(piece, layer_bytes - off), cs),
            "pool_pull_kernel");
     } else {
