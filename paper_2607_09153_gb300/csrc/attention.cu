@@ -1013,48 +1013,88 @@ bool build_attn_work(const int32_t* bt, const int32_t* sl, int n, int max_blocks
   std::vector<uint8_t> is_shared(static_cast<size_t>(n) * max_blocks, 0);
   std::vector<Run> runs;
   if (share && total_refs > 0) {
-    std::unordered_map<int32_t, std::vector<int32_t>> refs;   // page -> candidates (full refs)
-    refs.reserve(static_cast<size_t>(total_refs));
-    bool any_dup = false;
+    // Every full page's referencing candidates, in increasing candidate order.  Page ids up to a few
+    // times the number of references index dense arrays (counts, offsets, one list of all
+    // references: no allocation per page); sparser ids go through a hash map.
+    int32_t max_page = -1, min_page = 0;
+    int64_t full_refs = 0;
     for (int b = 0; b < n; ++b) {
       const int nfull = sl[b] / 16;
+      full_refs += nfull;
       for (int j = 0; j < nfull; ++j) {
-        auto& v = refs[bt[static_cast<int64_t>(b) * max_blocks + j]];
-        v.push_back(b);
-        if (v.size() > 1) any_dup = true;
+        const int32_t pg = bt[static_cast<int64_t>(b) * max_blocks + j];
+        max_page = std::max(max_page, pg);
+        min_page = std::min(min_page, pg);
+      }
+    }
+    const bool dense = min_page >= 0 && static_cast<int64_t>(max_page) + 1 <= 8 * full_refs + 65536;
+    std::vector<int32_t> ref_off, ref_list;                            // dense: CSR over page ids
+    std::unordered_map<int32_t, std::vector<int32_t>> refs;           // sparse
+    bool any_dup = false;
+    if (dense) {
+      ref_off.assign(static_cast<size_t>(max_page) + 2, 0);
+      for (int b = 0; b < n; ++b)
+        for (int j = 0, nfull = sl[b] / 16; j < nfull; ++j) ++ref_off[bt[static_cast<int64_t>(b) * max_blocks + j] + 1];
+      for (size_t pg = 1; pg < ref_off.size(); ++pg) {
+        any_dup = any_dup || ref_off[pg] > 1;
+        ref_off[pg] += ref_off[pg - 1];
+      }
+      ref_list.resize(static_cast<size_t>(full_refs));
+      std::vector<int32_t> fill(ref_off.begin(), ref_off.end() - 1);
+      for (int b = 0; b < n; ++b)
+        for (int j = 0, nfull = sl[b] / 16; j < nfull; ++j) ref_list[fill[bt[static_cast<int64_t>(b) * max_blocks + j]]++] = b;
+    } else {
+      refs.reserve(static_cast<size_t>(total_refs));
+      for (int b = 0; b < n; ++b) {
+        const int nfull = sl[b] / 16;
+        for (int j = 0; j < nfull; ++j) {
+          auto& v = refs[bt[static_cast<int64_t>(b) * max_blocks + j]];
+          v.push_back(b);
+          if (v.size() > 1) any_dup = true;
+        }
       }
     }
     if (any_dup) {
       std::vector<std::vector<int32_t>> group_cands, group_pages;
       std::unordered_map<uint64_t, int> gidx;
+      std::vector<uint8_t> in_group_dense(dense ? static_cast<size_t>(max_page) + 1 : 0, 0);
       std::unordered_map<int32_t, char> in_group;
-      for (auto& kv : refs) {
-        const std::vector<int32_t>& c = kv.second;
-        if (c.size() < 2) continue;
-        bool once = true;   // a candidate listing the page twice keeps it private
-        for (size_t i = 1; i < c.size(); ++i)
-          if (c[i] == c[i - 1]) once = false;   // candidates were appended in increasing order
-        if (!once) continue;
-        const uint64_t h = hash_list(c.data(), static_cast<int>(c.size()));
+      // a page referenced (in full) by the candidates c[0 .. len), in increasing order
+      auto consider = [&](int32_t page, const int32_t* c, size_t len) {
+        if (len < 2) return;
+        for (size_t i = 1; i < len; ++i)
+          if (c[i] == c[i - 1]) return;   // a candidate listing the page twice keeps it private
+        const uint64_t h = hash_list(c, static_cast<int>(len));
         auto itg = gidx.find(h);
         int gi;
         if (itg != gidx.end()) {
-          if (group_cands[itg->second] != c) continue;   // hash collision: keep it private
+          const std::vector<int32_t>& g = group_cands[itg->second];
+          if (g.size() != len || !std::equal(g.begin(), g.end(), c)) return;   // hash collision: private
           gi = itg->second;
         } else {
           gi = static_cast<int>(group_cands.size());
           gidx.emplace(h, gi);
-          group_cands.push_back(c);
+          group_cands.emplace_back(c, c + len);
           group_pages.emplace_back();
         }
-        group_pages[gi].push_back(kv.first);
-        in_group[kv.first] = 1;
+        group_pages[gi].push_back(page);
+        if (dense)
+          in_group_dense[page] = 1;
+        else
+          in_group[page] = 1;
+      };
+      if (dense) {
+        for (int32_t pg = 0; pg <= max_page; ++pg)
+          consider(pg, ref_list.data() + ref_off[pg], static_cast<size_t>(ref_off[pg + 1] - ref_off[pg]));
+      } else {
+        for (auto& kv : refs) consider(kv.first, kv.second.data(), kv.second.size());
       }
       for (int b = 0; b < n; ++b) {
         const int nfull = sl[b] / 16;
-        for (int j = 0; j < nfull; ++j)
-          if (in_group.count(bt[static_cast<int64_t>(b) * max_blocks + j]))
-            is_shared[static_cast<size_t>(b) * max_blocks + j] = 1;
+        for (int j = 0; j < nfull; ++j) {
+          const int32_t pg = bt[static_cast<int64_t>(b) * max_blocks + j];
+          if (dense ? in_group_dense[pg] != 0 : in_group.count(pg) != 0) is_shared[static_cast<size_t>(b) * max_blocks + j] = 1;
+        }
       }
       for (auto& pgs : group_pages) std::sort(pgs.begin(), pgs.end());   // deterministic contents
       std::vector<int> order(group_cands.size());   // deterministic group order
@@ -1327,11 +1367,28 @@ bool build_attn_work_fused(const int32_t* bt, const int32_t* sl, int n, int max_
   if (cs == 0 || (hi + cs - 1) / cs > kFuseMaxPages) return false;
   if (static_cast<size_t>(pairs) * cs > slot_limit) return false;
   {   // a page referenced twice (sharing, or a repeat) is left to the persistent plan
-    std::unordered_map<int32_t, char> seen;
-    seen.reserve(static_cast<size_t>(n) * hi);
+    int32_t pmin = 0, pmax = -1;
+    int64_t refs = 0;
     for (int b = 0; b < n; ++b)
-      for (int j = 0, np = (sl[b] + 15) / 16; j < np; ++j)
-        if (!seen.emplace(bt[static_cast<int64_t>(b) * max_blocks + j], 1).second) return false;
+      for (int j = 0, np = (sl[b] + 15) / 16; j < np; ++j, ++refs) {
+        pmin = std::min(pmin, bt[static_cast<int64_t>(b) * max_blocks + j]);
+        pmax = std::max(pmax, bt[static_cast<int64_t>(b) * max_blocks + j]);
+      }
+    if (pmin >= 0 && static_cast<int64_t>(pmax) + 1 <= 8 * refs + 65536) {   // dense page ids: a flag each
+      std::vector<uint8_t> seen(static_cast<size_t>(pmax) + 1, 0);
+      for (int b = 0; b < n; ++b)
+        for (int j = 0, np = (sl[b] + 15) / 16; j < np; ++j) {
+          uint8_t& f = seen[bt[static_cast<int64_t>(b) * max_blocks + j]];
+          if (f) return false;
+          f = 1;
+        }
+    } else {
+      std::unordered_map<int32_t, char> seen;
+      seen.reserve(static_cast<size_t>(refs));
+      for (int b = 0; b < n; ++b)
+        for (int j = 0, np = (sl[b] + 15) / 16; j < np; ++j)
+          if (!seen.emplace(bt[static_cast<int64_t>(b) * max_blocks + j], 1).second) return false;
+    }
   }
   w = AttnWorkHost();
   w.fuse_cs = cs;
