@@ -15,7 +15,7 @@ import kvsynth as ks
 import paper_2607_09153_gb300.kvprm as kp
 
 PRIVATE_COST, SHARED_COST_PER_CAND = 4, 2   # the planner's per-page cost model
-TC_CHUNK_COST, TC_CTA_COST = 29, 180        # its tensor-core launch: per 64-token chunk, per CTA
+TC_CHUNK_COST, TC_CTA_COST = 26, 180        # its tensor-core launch: per 64-token chunk, per CTA
 
 
 def check_plan(bt, sl, n_kv, group, n_ctas, share):
@@ -200,7 +200,7 @@ def test_concurrent_split_shares_the_sms():
     sl = np.full(n, 16 * (pre + own), np.int32)
     p3 = check_plan(bt, sl, 2, 7, 64, 3)
     assert p3["n_tc_ctas"] >= 1 and p3["n_ctas"] >= 1 and p3["n_tc_ctas"] + p3["n_ctas"] <= 64
-    # the split minimises the later launch's end under the cost model: a tensor-core CTA costs 29 per
+    # the split minimises the later launch's end under the cost model: a tensor-core CTA costs 26 per
     # 64-token chunk plus 180, a private page 4 (both per kv head)
     chunks = 2 * ((pre + 3) // 4) * len(set(p3["segs"][p3["segs"][:, 0] == 2][:, 2].tolist()))
     units = 2 * n * own * PRIVATE_COST
@@ -324,3 +324,19 @@ def test_depth_rows_stream_each_page_once(k):
         for pg in p["pages"][off:off + npg]:
             streams[(int(pg), g)] += 1
     assert set(streams.values()) == {1}
+
+
+@pytest.mark.parametrize("share", [1, 3])
+def test_sparse_page_ids_plan_alike(share):
+    """Page ids far larger than the number of references (and a negative one, which only the host-only
+    planner entry accepts unchecked) take the planner's hash-map path instead of its dense arrays:
+    the schedule is the same up to the renaming of the pages."""
+    w = ks.mcts_tree("sparse", ks.Arch(1, 256, 14, 2, 128, 256), 29, branching=3, depth=3, lo=5, hi=90)
+    bt, sl = np.asarray(w.block_table, np.int32), np.asarray(w.seq_lens, np.int32)
+    dense = check_plan(bt, sl, 2, 7, 64, share)
+    for rename in (lambda x: x * 4099 + 11, lambda x: x - 1):
+        bt2 = rename(bt.astype(np.int64)).astype(np.int32)
+        p = kp.kvprm_plan_attention(bt2, sl, 2, 7, 64, share)
+        for k in ("segs", "cta_seg", "cands", "slots", "slot_base", "nslots"):
+            np.testing.assert_array_equal(p[k], dense[k], err_msg=k)
+        np.testing.assert_array_equal(p["pages"], rename(np.asarray(dense["pages"], np.int64)).astype(np.int32))
