@@ -871,8 +871,9 @@ const void* pinned_device_view(const void* p, size_t bytes) {
 // gates layer l's attention.  Pinned host memory is pulled by SM loads (launch_pool_pull) in 64 MB
 // launches, so that a scoring kernel whose CTAs cannot be placed beside the copy's waits for at most
 // one launch (~0.3 ms): with one launch per layer (1 GB, ~5 ms) the long 8B call took 248-264 ms,
-// in 64 MB launches 177 ms, against 163 ms for its 34 GB at the link's ~211 GB/s.  Other host
-// memory goes through the copy engine.
+// in 64 MB launches 177 ms, and 172 ms with the forward launched without programmatic dependent
+// launch (score_device), against 163 ms for its 34 GB at the link's ~211 GB/s.  Other host memory
+// goes through the copy engine.
 int enqueue_pool_copy(kvprm_ctx* ctx, cudaStream_t st) {
   CK(cudaEventRecord(ctx->pool_free, st), "cudaEventRecord(pool free)");
   const size_t layer_bytes = ctx->host_pool_bytes / static_cast<size_t>(ctx->cfg.n_layers);
@@ -885,7 +886,7 @@ int enqueue_pool_copy(kvprm_ctx* ctx, cudaStream_t st) {
     if (src) {
       for (size_t off = 0; off < layer_bytes; off += piece)
         CK(launch_pool_pull(static_cast<const uint8_t*>(src) + l * layer_bytes + off, dst + off,
-                                   std::min(piece, layer_bytes - off), cs),
+                            std::min(piece, layer_bytes - off), cs),
            "pool_pull_kernel");
     } else {
       CK(cudaMemcpyAsync(dst, static_cast<const uint8_t*>(ctx->host_pool) + l * layer_bytes, layer_bytes,
