@@ -422,6 +422,16 @@ class Scorer:
         n_pages = kv_pages.shape[1]
         return kvprm_score(self.ctx, kv_pages.data_ptr(), n_pages, block_table, seq_lens, len(seq_lens), st)
 
+    def score_host(self, kv_pages, block_table, seq_lens, stream=None) -> np.ndarray:
+        """As score, with kv_pages a contiguous CPU bf16 tensor (pinned memory is copied in by the
+        library's copy kernel at the host link's full rate; pageable memory by the copy engine)."""
+        import torch
+        if kv_pages.device.type != "cpu" or not kv_pages.is_contiguous():
+            raise ValueError("score_host takes a contiguous CPU tensor; use score for a device cache")
+        st = (stream or torch.cuda.current_stream()).cuda_stream
+        return kvprm_score_host(self.ctx, kv_pages.data_ptr(), kv_pages.shape[1], block_table, seq_lens, len(seq_lens),
+                                st)
+
     def score_async(self, kv_pages, block_table, seq_lens, d_rewards, stream=None) -> None:
         import torch
         st = (stream or torch.cuda.current_stream()).cuda_stream

@@ -41,4 +41,9 @@ def test_readme_example():
     lens2 = np.full(4, 128, np.int32)
     p2 = scorer.score(kv, bt2, lens2)
     assert abs(p2[0] - p[0]) < 1e-6 and abs(p2[1] - p2[0]) < 1e-6 and abs(p2[2] - p2[0]) < 1e-5, (p, p2)
+    # the same cache held in host memory (pinned, then pageable): the same rewards, bit for bit
+    assert np.array_equal(scorer.score_host(kv.cpu().pin_memory(), bt, lens), p)
+    assert np.array_equal(scorer.score_host(kv.cpu(), bt, lens), p)
+    with pytest.raises(ValueError):
+        scorer.score_host(kv, bt, lens)
     scorer.close()
