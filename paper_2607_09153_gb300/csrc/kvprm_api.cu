@@ -1644,7 +1644,12 @@ int kvprm_score_host(kvprm_ctx* ctx, const void* h_kv_pages, int64_t n_pages, co
   ctx->layer_waits = false;
   ctx->host_pool = nullptr;
   ctx->host_pool_bytes = 0;
-  if (rc) return rc;
+  if (rc) {
+    // a call that failed after its cache copy was enqueued still returns only once nothing reads the
+    // caller's host buffer any more
+    if (bytes > 0 && cudaStreamSynchronize(ctx->copy_stream) != cudaSuccess) cudaGetLastError();
+    return rc;
+  }
   return finish_blocking(ctx, n, rewards, st);
 }
 
